@@ -27,7 +27,7 @@ Paper passages followed (section / equation labels of the paper):
   * Sec. 4.1 Eq. (6) and Appendix Eq. (cond-batched-bound),
     (cond-final-cert), (cond-bank-mixture) for the diagnostics.
 
-Readings where the paper is silent or ambiguous (each is listed in the design doc):
+Readings taken where the paper is silent or ambiguous:
   * The probe enters as ``W_h = O_h P`` (d x 4); only ||Z_h[i]|| and
     ||Z_h||_F are used.
   * Softmax keys: all N visual keys plus text keys 0..t (causal), scale

@@ -1,0 +1,484 @@
+// C-ABI entry points of libgmc.so (declared and documented in include/gmc.h):
+// argument validation, workspace carving and the launch sequence of one call.
+#include <math.h>
+#include <string.h>
+
+#include <atomic>
+#include <mutex>
+#include <unordered_map>
+
+#include "common.cuh"
+#include "kernels.cuh"
+
+using namespace gmc;
+
+namespace gmc {
+
+cudaError_t set_smem_limit(const void* func, size_t bytes) {
+  static std::mutex mu;
+  static std::unordered_map<const void*, size_t> done;
+  if (bytes <= 48 * 1024) return cudaSuccess;
+  std::lock_guard<std::mutex> lk(mu);
+  auto it = done.find(func);
+  if (it != done.end() && it->second >= bytes) return cudaSuccess;
+  cudaError_t e =
+      cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+  if (e == cudaSuccess) done[func] = bytes;
+  return e;
+}
+
+}  // namespace gmc
+
+namespace {
+
+constexpr size_t ALIGN = 256;
+constexpr int MAX_N_BUILD = 8192;
+
+struct Carver {
+  char* base;
+  size_t off = 0;
+  template <typename T> T* take(size_t count) {
+    const size_t at = off;
+    off += (count * sizeof(T) + ALIGN - 1) & ~(ALIGN - 1);
+    return base ? reinterpret_cast<T*>(base + at) : nullptr;
+  }
+};
+
+bool params_ok(const gmc_params& p) {
+  return p.batch_b >= 1 && p.pool_mult >= 1 && p.pool_mult * p.batch_b <= GMC_MAX_POOL &&
+         p.resp_temp > 0.f && p.resp_eps >= 0.f && p.tau_v > 0.f && p.tau_s > 0.f &&
+         p.beta_G >= 0.f && p.beta_V >= 0.f && p.beta_S >= 0.f && p.landmarks >= 1 &&
+         p.landmarks <= 64 && p.max_head_clusters >= 1 &&
+         p.max_head_clusters <= GMC_MAX_HEADS && p.head_eps > 0.f && p.terminal_q_weight > 0.f &&
+         p.lambda_mass >= 0.f && p.eps_mass > 0.f && p.gate_scale > 0.f && p.gate_pow > 0.f &&
+         p.ambig_margin > 0.f && p.pop_strength >= 0.f && p.pop_strength <= 1.f &&
+         p.rms_eps >= 0.f && p.norm_eps > 0.f && (p.check_mode == 0 || p.check_mode == 1);
+}
+
+int effective_K(int K, int N) { return K < 1 ? 1 : (K > N ? N : K); }
+
+// Shape checks shared by gmc_compress / gmc_transport.
+int check_problem(const gmc_problem* prob, int N, int T, int d, int D) {
+  if (!prob) return GMC_ERR_ARG;
+  if (prob->B < 1 || prob->grid_h < 1 || prob->grid_w < 1 || N < 1 ||
+      (long long)prob->grid_h * prob->grid_w != N || T < 1 || d < 1 || D < 1 || prob->Hkv < 1)
+    return GMC_ERR_ARG;
+  if (prob->dtype != GMC_F32 && prob->dtype != GMC_BF16) return GMC_ERR_ARG;
+  if (N > MAX_N_BUILD || D > 8192 || d > 1024) return GMC_ERR_UNSUPPORTED;
+  if (prob->dtype == GMC_BF16 && (d % 8 != 0 || D % 8 != 0)) return GMC_ERR_UNSUPPORTED;
+  if (prob->dtype == GMC_F32 && (d % 4 != 0 || D % 8 != 0)) return GMC_ERR_UNSUPPORTED;
+  return GMC_OK;
+}
+
+bool aligned(const void* p, size_t a) { return ((uintptr_t)p % a) == 0; }
+
+Dims make_dims(const gmc_problem* prob, const gmc_params& p, int N, int T, int H, int d, int D,
+               int K) {
+  Dims dm;
+  dm.B = prob->B; dm.N = N; dm.T = T; dm.H = H; dm.Hkv = prob->Hkv; dm.d = d; dm.D = D;
+  dm.K = K; dm.gh = prob->grid_h; dm.gw = prob->grid_w; dm.L = p.landmarks;
+  dm.M = H * T + N + p.landmarks * p.landmarks;
+  dm.dtype = prob->dtype;
+  dm.toff = prob->text_offsets;
+  return dm;
+}
+
+// Workspace of gmc_compress.  base == nullptr only measures.
+size_t carve_compress(const Dims& dm, Scratch* s, char* base) {
+  Carver c{base};
+  Scratch t{};
+  const size_t B = dm.B, N = dm.N, H = dm.H, T = dm.T, M = dm.M, K = dm.K;
+  t.nP = ceil_div(dm.N, ROWS_PER_BLOCK);
+  t.nHG = ceil_div(dm.N, HG_TOK);
+  t.nA = ceil_div(dm.N, ASSIGN_WARPS);
+  t.nSel = 0;
+  t.status = c.take<uint32_t>(4);
+  t.A = c.take<float>(B * H * T * N);
+  t.rs = c.take<float>(B * H * T);
+  t.Z = c.take<float>(B * H * N * 4);
+  t.zn2 = c.take<float>(B * H * N);
+  t.sigpart = c.take<float>(B * t.nP * H);
+  t.sigma = c.take<float>(B * H);
+  t.hgpart = c.take<double>(B * t.nHG * H * H);
+  t.W2 = c.take<float>(B * H * N);
+  t.omega = c.take<float>(B * H);
+  t.ebar = c.take<float>(B * N);
+  t.rn = c.take<float>(B * N);
+  t.rmsh = c.take<float>(B * N);
+  t.cos = c.take<float>(B * N * N);
+  t.C = c.take<float>(B * M * N);
+  t.scol = c.take<uint16_t>(B * M * N);
+  t.u0 = c.take<long long>(B * N);
+  t.support = c.take<int32_t>(B * K);
+  t.slot = c.take<int32_t>(B * N);
+  t.order = c.take<int32_t>(B * K);
+  t.delta = c.take<float>(B * N);
+  t.dpart = c.take<double>(B * t.nA * 2);
+  t.pi = c.take<int32_t>(B * N);
+  t.mass = c.take<float>(B * N);
+  t.selpart = nullptr;
+  t.fexp = nullptr;
+  if (s) *s = t;
+  return c.off;
+}
+
+int fixed_point_exponent(double total) {
+  if (!(total > 0.0) || !isfinite(total)) return 61;
+  int e = 61 - (int)ceil(log2(total));
+  return e < -60 ? -60 : (e > 120 ? 120 : e);
+}
+
+int fill_trace_layout(int B, const gmc_params& p, int N, int H, int K, gmc_trace_layout* o) {
+  if (B < 1 || N < 1 || H < 0 || K < 1) return GMC_ERR_ARG;
+  gmc_trace_layout L{};
+  L.rounds_max = (K + p.batch_b - 1) / p.batch_b + 1;
+  L.pool_size = p.pool_mult * p.batch_b;
+  size_t off = sizeof(gmc_trace_header);
+  auto take = [&](size_t bytes) {
+    size_t at = off;
+    off += (bytes + 15) & ~(size_t)15;
+    return at;
+  };
+  L.off_order = take(4 * (size_t)K);
+  L.off_round_end = take(4 * (size_t)L.rounds_max);
+  L.off_pool = take(4 * (size_t)L.rounds_max * L.pool_size);
+  L.off_centres = take(4 * (size_t)p.max_head_clusters);
+  L.off_head_assign = take(4 * (size_t)H);
+  L.off_omega = take(4 * (size_t)H);
+  L.off_pi = take(4 * (size_t)N);
+  L.off_ebar = take(4 * (size_t)N);
+  L.off_mass = take(4 * (size_t)N);
+  L.bytes_per_image = (off + 15) & ~(size_t)15;
+  *o = L;
+  return GMC_OK;
+}
+
+TraceView make_trace_view(void* trace, const gmc_trace_layout& L) {
+  TraceView tv{};
+  tv.base = (char*)trace;
+  tv.stride = L.bytes_per_image;
+  tv.off_order = L.off_order;
+  tv.off_round_end = L.off_round_end;
+  tv.off_pool = L.off_pool;
+  tv.off_centres = L.off_centres;
+  tv.off_head_assign = L.off_head_assign;
+  tv.off_omega = L.off_omega;
+  tv.off_pi = L.off_pi;
+  tv.off_ebar = L.off_ebar;
+  tv.off_mass = L.off_mass;
+  tv.rounds_max = L.rounds_max;
+  tv.pool_size = L.pool_size;
+  return tv;
+}
+
+int cuda_fail(cudaError_t e) {
+  if (e == cudaSuccess) return GMC_OK;
+  cudaGetLastError();
+  return GMC_ERR_CUDA;
+}
+
+#define GMC_TRY(expr)                         \
+  do {                                        \
+    cudaError_t _e = (expr);                  \
+    if (_e != cudaSuccess) return cuda_fail(_e); \
+  } while (0)
+
+std::atomic<uint64_t> g_launches{0};
+
+// Stage timing for benchmarks: events on the call's own stream.
+struct Profiler {
+  static constexpr int MAXEV = 16;
+  std::mutex mu;
+  bool on = false, valid = false;
+  cudaEvent_t ev[MAXEV] = {};
+  const char* names[MAXEV] = {};
+  int n = 0;
+  cudaError_t begin(cudaStream_t st) {
+    n = 0;
+    valid = false;
+    if (!on) return cudaSuccess;
+    if (!ev[0])
+      for (int k = 0; k < MAXEV; ++k) {
+        cudaError_t e = cudaEventCreate(&ev[k]);
+        if (e != cudaSuccess) return e;
+      }
+    return cudaEventRecord(ev[n++], st);
+  }
+  cudaError_t mark(const char* name, cudaStream_t st) {
+    if (!on || n >= MAXEV) return cudaSuccess;
+    names[n - 1] = name;
+    return cudaEventRecord(ev[n++], st);
+  }
+};
+Profiler g_prof;
+
+#define GMC_STAGE(name, nkernels, expr)              \
+  do {                                               \
+    GMC_TRY(expr);                                   \
+    g_launches += (nkernels);                        \
+    GMC_TRY(g_prof.mark(name, st));                  \
+  } while (0)
+
+}  // namespace
+
+extern "C" {
+
+void gmc_default_params(gmc_params* p) {
+  if (!p) return;
+  p->batch_b = 16;
+  p->pool_mult = 4;
+  p->resp_temp = 0.1f;
+  p->resp_eps = 1e-12f;
+  p->tau_v = 0.2f;
+  p->tau_s = 0.02f;
+  p->beta_G = 0.5f;
+  p->beta_V = 0.5f;
+  p->beta_S = 0.25f;
+  p->landmarks = 16;
+  p->max_head_clusters = 4;
+  p->head_eps = 0.05f;
+  p->terminal_q_weight = 2.f;
+  p->lambda_mass = 1.f;
+  p->eps_mass = 1e-8f;
+  p->assign_spatial_w = 0.5f;
+  p->gate_scale = 0.08f;
+  p->gate_pow = 8.f;
+  p->ambig_margin = 0.05f;
+  p->pop_strength = 0.5f;
+  p->rms_eps = 1e-6f;
+  p->norm_eps = 1e-12f;
+  p->check_mode = 0;
+}
+
+const char* gmc_error_string(int code) {
+  switch (code) {
+    case GMC_OK: return "GMC_OK";
+    case GMC_ERR_ARG: return "GMC_ERR_ARG: invalid argument";
+    case GMC_ERR_UNSUPPORTED: return "GMC_ERR_UNSUPPORTED: shape outside this build's limits";
+    case GMC_ERR_WORKSPACE: return "GMC_ERR_WORKSPACE: workspace too small";
+    case GMC_ERR_CUDA: return "GMC_ERR_CUDA: CUDA launch or query failed";
+    default: return "GMC: unknown code";
+  }
+}
+
+const char* gmc_version(void) { return "gmc 0.1.0 sm_103a"; }
+
+size_t gmc_workspace_size(const gmc_problem* prob, int N, int T, int H, int d, int D, int K) {
+  if (check_problem(prob, N, T, d, D) != GMC_OK || H < 1 || H > GMC_MAX_HEADS ||
+      H % prob->Hkv != 0)
+    return 0;
+  gmc_params p;
+  gmc_default_params(&p);
+  const Dims dm = make_dims(prob, p, N, T, H, d, D, effective_K(K, N));
+  return carve_compress(dm, nullptr, nullptr);
+}
+
+int gmc_get_trace_layout(const gmc_problem* prob, const gmc_params* params, int N, int T, int H,
+                         int K, gmc_trace_layout* out) {
+  if (!prob || !out || T < 1) return GMC_ERR_ARG;
+  gmc_params p;
+  if (params) p = *params; else gmc_default_params(&p);
+  if (!params_ok(p)) return GMC_ERR_ARG;
+  return fill_trace_layout(prob->B, p, N, H, effective_K(K, N), out);
+}
+
+size_t gmc_trace_size(const gmc_problem* prob, const gmc_params* params, int N, int T, int H,
+                      int K) {
+  gmc_trace_layout L;
+  if (gmc_get_trace_layout(prob, params, N, T, H, K, &L) != GMC_OK) return 0;
+  return (size_t)prob->B * L.bytes_per_image;
+}
+
+int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* hidden,
+                 const void* keys, const void* queries, const int32_t* pos_ids,
+                 const float* vo_probe, int N, int T, int H, int d, int D, int K,
+                 int32_t* out_idx, void* out_hidden, void* out_kv, int32_t* out_pos,
+                 void* workspace, size_t ws_bytes, void* trace, gmc_stream_t stream_) {
+  int rc = check_problem(prob, N, T, d, D);
+  if (rc != GMC_OK) return rc;
+  if (H < 1 || H % prob->Hkv != 0) return GMC_ERR_ARG;
+  if (H > GMC_MAX_HEADS) return GMC_ERR_UNSUPPORTED;
+  gmc_params p;
+  if (params) p = *params; else gmc_default_params(&p);
+  if (!params_ok(p)) return GMC_ERR_ARG;
+  if (!hidden || !keys || !queries || !pos_ids || !vo_probe || !out_idx || !out_hidden ||
+      !out_kv || !out_pos || !workspace)
+    return GMC_ERR_ARG;
+  if (!aligned(hidden, 16) || !aligned(keys, 16) || !aligned(queries, 16) ||
+      !aligned(vo_probe, 16) || !aligned(out_hidden, 16) || !aligned(out_kv, 16) ||
+      !aligned(workspace, ALIGN) || (trace && !aligned(trace, 16)))
+    return GMC_ERR_ARG;
+  const int Ke = effective_K(K, N);
+  const Dims dm = make_dims(prob, p, N, T, H, d, D, Ke);
+  Scratch s;
+  const size_t need = carve_compress(dm, &s, (char*)workspace);
+  if (ws_bytes < need) return GMC_ERR_WORKSPACE;
+  cudaStream_t st = (cudaStream_t)stream_;
+  gmc_trace_layout L;
+  TraceView tv{};
+  if (trace) {
+    fill_trace_layout(dm.B, p, N, H, Ke, &L);
+    tv = make_trace_view(trace, L);
+    GMC_TRY(cudaMemsetAsync(trace, 0, (size_t)dm.B * L.bytes_per_image, st));
+  }
+  std::lock_guard<std::mutex> lk(g_prof.mu);
+  GMC_TRY(cudaMemsetAsync(s.status, 0, sizeof(uint32_t), st));
+  if (Ke == N) {  // K = N returns the unmodified execution
+    GMC_TRY(launch_identity(dm, hidden, keys, pos_ids, out_idx, out_hidden, out_kv, out_pos,
+                            s.status, st));
+    g_launches += 1;
+    return GMC_OK;
+  }
+  const int fx = fixed_point_exponent((double)p.beta_G + p.beta_V + p.beta_S);
+  GMC_TRY(cudaMemsetAsync(s.u0, 0, sizeof(long long) * dm.B * N, st));
+  GMC_TRY(g_prof.begin(st));
+  GMC_STAGE("rownorm", 1, launch_rownorm(dm, hidden, p.norm_eps, s, st));
+  GMC_STAGE("probe", 2, launch_probe(dm, keys, vo_probe, p, s, st));
+  GMC_STAGE("message", 1, launch_message(dm, keys, queries, s, st));
+  GMC_STAGE("heads", 3, launch_heads(dm, p, s, tv, st));
+  GMC_STAGE("gram", 1, launch_gram(dm, hidden, s, st));
+  GMC_STAGE("clients", 1, launch_build_clients(dm, p, fx, s, st));
+  GMC_STAGE("select", 1,
+            launch_select(dm.B, N, Ke, dm.M, dm.toff, H, T, p.landmarks * p.landmarks, p, fx,
+                          nullptr, s.C, s.scol, s.u0, s.order, s.support, s.slot, nullptr,
+                          s.status, tv, st));
+  GMC_STAGE("assign", 2, launch_assign(dm, p, s, tv, st));
+  GMC_STAGE("transport", 2,
+            launch_transport(dm, p, hidden, keys, pos_ids, s.support, s.pi, s.mass, s.rmsh,
+                             out_idx, out_hidden, out_kv, out_pos, s.status, st));
+  g_prof.valid = g_prof.on;
+  return GMC_OK;
+}
+
+// ---------------------------------------------------------------------------
+// gmc_select
+// ---------------------------------------------------------------------------
+static size_t carve_select(int B, int M, int N, int K, Scratch* s, char* base) {
+  Carver c{base};
+  Scratch t{};
+  t.nSel = 64;
+  t.status = c.take<uint32_t>(4);
+  t.C = c.take<float>((size_t)B * M * N);
+  t.scol = c.take<uint16_t>((size_t)B * M * N);
+  t.u0 = c.take<long long>((size_t)B * N);
+  t.order = c.take<int32_t>((size_t)B * K);
+  t.support = c.take<int32_t>((size_t)B * K);
+  t.slot = c.take<int32_t>((size_t)B * N);
+  t.selpart = c.take<double>((size_t)B * t.nSel);
+  t.fexp = c.take<int32_t>((size_t)B);
+  if (s) *s = t;
+  return c.off;
+}
+
+size_t gmc_select_workspace_size(int B, int M, int N, int K, const gmc_params* params) {
+  (void)params;
+  if (B < 1 || M < 1 || N < 1 || N > MAX_N_BUILD || K < 1 || K > N) return 0;
+  return carve_select(B, M, N, K, nullptr, nullptr);
+}
+
+int gmc_select(const float* clients, int B, int M, int N, int K, const gmc_params* params,
+               int32_t* out_idx, void* workspace, size_t ws_bytes, void* trace,
+               gmc_stream_t stream_) {
+  if (!clients || !out_idx || !workspace || B < 1 || M < 1 || N < 1 || K < 1 || K > N)
+    return GMC_ERR_ARG;
+  if (N > MAX_N_BUILD) return GMC_ERR_UNSUPPORTED;
+  if (!aligned(workspace, ALIGN) || (trace && !aligned(trace, 16))) return GMC_ERR_ARG;
+  gmc_params p;
+  if (params) p = *params; else gmc_default_params(&p);
+  if (!params_ok(p)) return GMC_ERR_ARG;
+  Scratch s;
+  const size_t need = carve_select(B, M, N, K, &s, (char*)workspace);
+  if (ws_bytes < need) return GMC_ERR_WORKSPACE;
+  cudaStream_t st = (cudaStream_t)stream_;
+  TraceView tv{};
+  if (trace) {
+    gmc_trace_layout L;
+    fill_trace_layout(B, p, N, 0, K, &L);
+    tv = make_trace_view(trace, L);
+    GMC_TRY(cudaMemsetAsync(trace, 0, (size_t)B * L.bytes_per_image, st));
+  }
+  GMC_TRY(cudaMemsetAsync(s.status, 0, sizeof(uint32_t), st));
+  GMC_TRY(cudaMemcpyAsync(s.C, clients, sizeof(float) * B * (size_t)M * N,
+                          cudaMemcpyDeviceToDevice, st));
+  GMC_TRY(cudaMemsetAsync(s.u0, 0, sizeof(long long) * B * (size_t)N, st));
+  GMC_TRY(launch_select_prep(s.C, B, M, N, s, st));
+  GMC_TRY(launch_select(B, N, K, M, nullptr, 0, 1, 0, p, 0, s.fexp, s.C, s.scol, s.u0, s.order,
+                        s.support, s.slot, out_idx, s.status, tv, st));
+  g_launches += 4;
+  return GMC_OK;
+}
+
+// ---------------------------------------------------------------------------
+// gmc_transport
+// ---------------------------------------------------------------------------
+size_t gmc_transport_workspace_size(const gmc_problem* prob, int N, int T, int K) {
+  if (!prob || prob->B < 1 || N < 1 || T < 1 || K < 1 || K > N) return 0;
+  Carver c{nullptr};
+  c.take<uint32_t>(4);
+  c.take<float>((size_t)prob->B * N);
+  return c.off;
+}
+
+int gmc_transport(const gmc_problem* prob, const gmc_params* params, const void* hidden,
+                  const void* keys, const int32_t* pos_ids, const int32_t* support,
+                  const int32_t* assign, const float* weights, int N, int T, int d, int D, int K,
+                  int32_t* out_idx, void* out_hidden, void* out_kv, int32_t* out_pos,
+                  void* workspace, size_t ws_bytes, gmc_stream_t stream_) {
+  int rc = check_problem(prob, N, T, d, D);
+  if (rc != GMC_OK) return rc;
+  if (K < 1 || K > N) return GMC_ERR_ARG;
+  gmc_params p;
+  if (params) p = *params; else gmc_default_params(&p);
+  if (!params_ok(p)) return GMC_ERR_ARG;
+  if (!hidden || !keys || !pos_ids || !support || !assign || !weights || !out_idx ||
+      !out_hidden || !out_kv || !out_pos || !workspace)
+    return GMC_ERR_ARG;
+  if (!aligned(hidden, 16) || !aligned(keys, 16) || !aligned(out_hidden, 16) ||
+      !aligned(out_kv, 16) || !aligned(workspace, ALIGN))
+    return GMC_ERR_ARG;
+  if (ws_bytes < gmc_transport_workspace_size(prob, N, T, K)) return GMC_ERR_WORKSPACE;
+  Carver c{(char*)workspace};
+  uint32_t* status = c.take<uint32_t>(4);
+  float* rmsh = c.take<float>((size_t)prob->B * N);
+  cudaStream_t st = (cudaStream_t)stream_;
+  const Dims dm = make_dims(prob, p, N, T, 0, d, D, K);
+  GMC_TRY(cudaMemsetAsync(status, 0, sizeof(uint32_t), st));
+  GMC_TRY(launch_rms_rows(dm, hidden, rmsh, status, st));
+  GMC_TRY(launch_transport(dm, p, hidden, keys, pos_ids, support, assign, weights, rmsh, out_idx,
+                           out_hidden, out_kv, out_pos, status, st));
+  g_launches += 3;
+  return GMC_OK;
+}
+
+int gmc_profile_enable(int on) {
+  std::lock_guard<std::mutex> lk(g_prof.mu);
+  g_prof.on = on != 0;
+  g_prof.valid = false;
+  return GMC_OK;
+}
+
+int gmc_profile_read(float* ms, const char** names, int max) {
+  std::lock_guard<std::mutex> lk(g_prof.mu);
+  if (!g_prof.valid || g_prof.n < 2) return -1;
+  if (cudaEventSynchronize(g_prof.ev[g_prof.n - 1]) != cudaSuccess) return cuda_fail(cudaErrorUnknown), -1;
+  const int ns = g_prof.n - 1;
+  for (int k = 0; k < ns && k < max; ++k) {
+    float t = 0.f;
+    cudaEventElapsedTime(&t, g_prof.ev[k], g_prof.ev[k + 1]);
+    if (ms) ms[k] = t;
+    if (names) names[k] = g_prof.names[k];
+  }
+  return ns;
+}
+
+uint64_t gmc_launch_count(void) { return g_launches.load(); }
+
+int gmc_read_status(const void* workspace, uint32_t* status, gmc_stream_t stream_) {
+  if (!workspace || !status) return GMC_ERR_ARG;
+  cudaStream_t st = (cudaStream_t)stream_;
+  GMC_TRY(cudaStreamSynchronize(st));
+  GMC_TRY(cudaMemcpy(status, workspace, sizeof(uint32_t), cudaMemcpyDeviceToHost));
+  return GMC_OK;
+}
+
+}  // extern "C"

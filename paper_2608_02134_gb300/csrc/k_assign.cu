@@ -1,0 +1,150 @@
+// Population assignment (appendix Eq. (cond-assignment), (cond-population-gate)).
+//
+// For a discarded token i, delta_i is the gap between its largest and
+// second-largest cosine to the support (0 when |S| = 1); Delta_bar is the mean
+// gap over the discarded tokens (0 when none is discarded);
+//   s_x = 1 - exp(-(Delta_bar / gate_scale)^gate_pow)
+//   g_i = exp(-(delta_i / ambig_margin)^gate_pow)
+//   pi(i) = argmax_{j in S} cos_ij + lambda_p s_x g_i exp(-||p_i - p_j||^2 / tau_s)
+// (ties to the lowest j); selected tokens represent themselves.  The
+// population weights are m_i = (1 - alpha s_x) + alpha s_x ebar_i.
+#include "common.cuh"
+#include "kernels.cuh"
+
+namespace gmc {
+
+// Pass 1: delta_i per discarded token; per-block partial sums of delta and counts.
+__global__ void k_assign_gap(const float* __restrict__ cos, const int32_t* __restrict__ support,
+                             const int32_t* __restrict__ slot, const int32_t* toff, int B, int N,
+                             int K, int Tmax, float* delta, double* dpart, int nA,
+                             uint32_t* status) {
+  __shared__ double sd[ASSIGN_WARPS];
+  __shared__ int sc[ASSIGN_WARPS];
+  const int b = blockIdx.y;
+  const TextGeom tg = text_geom(toff, b, B, Tmax, status);
+  if (tg.T == 0) return;
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int i = blockIdx.x * ASSIGN_WARPS + w;
+  double dv = 0.0;
+  int dc = 0;
+  if (i < N && slot[(size_t)b * N + i] < 0) {
+    const float* row = cos + ((size_t)b * N + i) * N;
+    const int32_t* S = support + (size_t)b * K;
+    float m1 = -INFINITY, m2 = -INFINITY;
+    for (int k = lane; k < K; k += 32) {
+      const float v = row[S[k]];
+      if (v > m1) { m2 = m1; m1 = v; } else if (v > m2) { m2 = v; }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float b1 = __shfl_xor_sync(FULL, m1, o), b2 = __shfl_xor_sync(FULL, m2, o);
+      const float hi = fmaxf(m1, b1);
+      m2 = fmaxf(fminf(m1, b1), fmaxf(m2, b2));
+      m1 = hi;
+    }
+    const float d = K > 1 ? m1 - m2 : 0.f;
+    if (lane == 0) delta[(size_t)b * N + i] = d;
+    dv = d;
+    dc = 1;
+  } else if (i < N && lane == 0) {
+    delta[(size_t)b * N + i] = 0.f;
+  }
+  if (lane == 0) {
+    sd[w] = dv;
+    sc[w] = dc;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double s = 0.0;
+    int c = 0;
+    for (int q = 0; q < ASSIGN_WARPS; ++q) {
+      s += sd[q];
+      c += sc[q];
+    }
+    dpart[((size_t)b * nA + blockIdx.x) * 2 + 0] = s;
+    dpart[((size_t)b * nA + blockIdx.x) * 2 + 1] = (double)c;
+  }
+}
+
+// Pass 2: s_x, the gated spatial assignment, and the population weights.
+__global__ void k_assign_pick(const float* __restrict__ cos, const int32_t* __restrict__ support,
+                              const int32_t* __restrict__ slot, const float* __restrict__ delta,
+                              const double* __restrict__ dpart, int nA,
+                              const float* __restrict__ ebar, const int32_t* toff, int B, int N,
+                              int K, int Tmax, int gh, int gw, float gate_scale, float gate_pow,
+                              float ambig_margin, float lambda_p, float tau_s, float alpha,
+                              int32_t* pi, float* mass, TraceView tv, uint32_t* status) {
+  const int b = blockIdx.y;
+  const TextGeom tg = text_geom(toff, b, B, Tmax, status);
+  if (tg.T == 0) return;
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  // every warp reduces the partials in the same fixed order
+  double s = 0.0, c = 0.0;
+  for (int q = lane; q < nA; q += 32) {
+    s += dpart[((size_t)b * nA + q) * 2 + 0];
+    c += dpart[((size_t)b * nA + q) * 2 + 1];
+  }
+  s = warp_sum(s);
+  c = warp_sum(c);
+  const double dbar = c > 0.0 ? s / c : 0.0;
+  const double sxd = 1.0 - exp(-pow(dbar / gate_scale, (double)gate_pow));
+  const float sx = (float)sxd;
+  if (blockIdx.x == 0 && threadIdx.x == 0 && tv.base) {
+    tv.header(b)->s_x = sx;
+    tv.header(b)->delta_bar = (float)dbar;
+  }
+  const int i = blockIdx.x * ASSIGN_WARPS + w;
+  if (i >= N) return;
+  const float eb = ebar[(size_t)b * N + i];
+  const float m = (1.f - alpha * sx) + alpha * sx * eb;
+  int choice = i;
+  if (slot[(size_t)b * N + i] < 0) {
+    const float gi = expf(-powf(delta[(size_t)b * N + i] / ambig_margin, gate_pow));
+    const float coef = lambda_p * sx * gi;
+    const float piy = ((i / gw) + 0.5f) / gh, pix = ((i % gw) + 0.5f) / gw;
+    const float* row = cos + ((size_t)b * N + i) * N;
+    const int32_t* S = support + (size_t)b * K;
+    float best = -INFINITY;
+    int bk = 0x7fffffff;
+    for (int k = lane; k < K; k += 32) {
+      const int j = S[k];
+      float v = row[j];
+      if (coef > 0.f) {
+        const float dy = ((j / gw) + 0.5f) / gh - piy, dx = ((j % gw) + 0.5f) / gw - pix;
+        v += coef * expf(-(dy * dy + dx * dx) / tau_s);
+      }
+      if (v > best) { best = v; bk = k; }  // k ascending within a lane: first max kept
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float ob = __shfl_xor_sync(FULL, best, o);
+      const int ok = __shfl_xor_sync(FULL, bk, o);
+      if (ob > best || (ob == best && ok < bk)) { best = ob; bk = ok; }
+    }
+    choice = S[bk];
+  }
+  if (lane == 0) {
+    pi[(size_t)b * N + i] = choice;
+    mass[(size_t)b * N + i] = m;
+    if (tv.base) {
+      tv.at<int32_t>(b, tv.off_pi)[i] = choice;
+      tv.at<float>(b, tv.off_mass)[i] = m;
+    }
+  }
+}
+
+cudaError_t launch_assign(const Dims& dm, const gmc_params& p, Scratch& s, const TraceView& tv,
+                          cudaStream_t st) {
+  dim3 grid(s.nA, dm.B);
+  k_assign_gap<<<grid, 32 * ASSIGN_WARPS, 0, st>>>(s.cos, s.support, s.slot, dm.toff, dm.B, dm.N,
+                                                   dm.K, dm.T, s.delta, s.dpart, s.nA, s.status);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  k_assign_pick<<<grid, 32 * ASSIGN_WARPS, 0, st>>>(
+      s.cos, s.support, s.slot, s.delta, s.dpart, s.nA, s.ebar, dm.toff, dm.B, dm.N, dm.K, dm.T,
+      dm.gh, dm.gw, p.gate_scale, p.gate_pow, p.ambig_margin, p.assign_spatial_w, p.tau_s,
+      p.pop_strength, s.pi, s.mass, tv, s.status);
+  return cudaGetLastError();
+}
+
+}  // namespace gmc

@@ -1,0 +1,130 @@
+// Internal interface between the C-ABI layer (gmc_api.cu) and the kernel
+// translation units.  Nothing here is exported from libgmc.so.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "../../include/gmc.h"
+
+namespace gmc {
+
+// Shapes of one call; every per-image buffer is strided by T (= T_max).
+struct Dims {
+  int B, N, T, H, Hkv, d, D, K, gh, gw, L;  // L = landmarks per side
+  int M;                                    // H*T + N + L*L: client rows per image (max)
+  int dtype;                                // GMC_F32 / GMC_BF16
+  const int32_t* toff;                      // device text offsets or nullptr
+};
+
+// Trace record layout passed by value to kernels (byte offsets, 0 = absent).
+struct TraceView {
+  char* base;  // nullptr: no trace
+  size_t stride, off_order, off_round_end, off_pool, off_centres, off_head_assign, off_omega,
+      off_pi, off_ebar, off_mass;
+  int rounds_max, pool_size;
+  __device__ __forceinline__ char* rec(int b) const { return base + (size_t)b * stride; }
+  __device__ __forceinline__ gmc_trace_header* header(int b) const {
+    return reinterpret_cast<gmc_trace_header*>(rec(b));
+  }
+  template <typename T> __device__ __forceinline__ T* at(int b, size_t off) const {
+    return reinterpret_cast<T*>(rec(b) + off);
+  }
+};
+
+// Device scratch carved out of the caller's workspace.
+struct Scratch {
+  uint32_t* status;
+  float* A;          // [B][H][T][N]   native attention slice (visual columns)
+  float* rs;         // [B][H][T]      sum_i ||u_i^{h,t}|| (0: inactive row)
+  float* Z;          // [B][H][N][4]   probe values Z_h[i]
+  float* zn2;        // [B][H][N]      ||Z_h[i]||^2
+  float* sigpart;    // [B][nP][H]     block partials of ||Z_h||_F^2
+  float* sigma;      // [B][H]         mass coordinate sigma_h
+  double* hgpart;    // [B][nHG][H*H]  block partials of the head-pattern Gram
+  float* W2;         // [B][H][N]      sum_t nu_t A[h,t,i]^2
+  float* omega;      // [B][H]
+  float* ebar;       // [B][N]
+  float* rn;         // [B][N]         1 / max(||h_i||, eps)
+  float* rmsh;       // [B][N]         rms(h_i)
+  float* cos;        // [B][N][N]      cosine of boundary states
+  float* C;          // [B][M][N]      client matrix, then in-place residual survivor values
+  uint16_t* scol;    // [B][M][N]      survivor token index
+  long long* u0;     // [B][N]         fixed-point column sums of C
+  int32_t* support;  // [B][K]         ascending
+  int32_t* slot;     // [B][N]         position in support or -1
+  int32_t* order;    // [B][K]         selection order
+  float* delta;      // [B][N]
+  double* dpart;     // [B][nA][2]     partial sums of delta and counts over discarded tokens
+  int32_t* pi;       // [B][N]
+  float* mass;       // [B][N]
+  double* selpart;   // [B][64]        select-path total mass partials
+  int32_t* fexp;     // [B]            select-path fixed-point exponents
+  int nP, nHG, nA, nSel;
+};
+
+constexpr int ROWS_PER_BLOCK = 8;  // rownorm / probe / client builder blocks
+constexpr int HG_TOK = 8;          // tokens per head-statistics block
+constexpr int ASSIGN_WARPS = 8;    // tokens per assignment block
+
+// Launch wrappers.  Each returns the first CUDA error it saw.
+cudaError_t launch_rownorm(const Dims&, const void* hidden, float norm_eps, Scratch&, cudaStream_t);
+cudaError_t launch_probe(const Dims&, const void* keys, const float* W, const gmc_params&, Scratch&,
+                         cudaStream_t);
+cudaError_t launch_message(const Dims&, const void* keys, const void* queries, Scratch&,
+                           cudaStream_t);
+cudaError_t launch_heads(const Dims&, const gmc_params&, Scratch&, const TraceView&, cudaStream_t);
+cudaError_t launch_gram(const Dims&, const void* hidden, Scratch&, cudaStream_t);
+cudaError_t launch_build_clients(const Dims&, const gmc_params&, int fx_exp, Scratch&,
+                                 cudaStream_t);
+cudaError_t launch_select(int B, int N, int K, int M, const int32_t* toff, int H, int T, int L2,
+                          const gmc_params&, int fx_exp, const int32_t* fexp_per_image, float* C,
+                          uint16_t* scol, const long long* u0, int32_t* order, int32_t* support,
+                          int32_t* slot, int32_t* out_idx, uint32_t* status, const TraceView&,
+                          cudaStream_t);
+cudaError_t launch_select_prep(const float* C, int B, int M, int N, Scratch&, cudaStream_t);
+cudaError_t launch_assign(const Dims&, const gmc_params&, Scratch&, const TraceView&,
+                          cudaStream_t);
+cudaError_t launch_transport(const Dims&, const gmc_params&, const void* hidden, const void* keys,
+                             const int32_t* pos, const int32_t* support, const int32_t* pi,
+                             const float* mass, const float* rmsh, int32_t* out_idx,
+                             void* out_hidden, void* out_kv, int32_t* out_pos, uint32_t* status,
+                             cudaStream_t);
+cudaError_t launch_identity(const Dims&, const void* hidden, const void* keys, const int32_t* pos,
+                            int32_t* out_idx, void* out_hidden, void* out_kv, int32_t* out_pos,
+                            uint32_t* status, cudaStream_t);
+cudaError_t launch_rms_rows(const Dims&, const void* hidden, float* rmsh, uint32_t* status,
+                            cudaStream_t);
+
+}  // namespace gmc
+
+namespace gmc {
+// Element offsets of one image's rows in the ABI layouts (see include/gmc.h).
+struct SeqIdx {
+  size_t s;   // b*N + off_b: first input sequence row of the image
+  size_t o;   // b*K + off_b: first output row of the image
+  int R, Ro;  // N + T_b, K + T_b
+  __host__ __device__ SeqIdx(int b, int N, int K, int off, int Tb)
+      : s((size_t)b * N + off), o((size_t)b * K + off), R(N + Tb), Ro(K + Tb) {}
+  __host__ __device__ size_t hidden_row(int r, int D) const { return (s + r) * (size_t)D; }
+  __host__ __device__ size_t key_row(int r, int HD) const { return (2 * s + r) * (size_t)HD; }
+  __host__ __device__ size_t value_row(int r, int HD) const { return (2 * s + R + r) * (size_t)HD; }
+  __host__ __device__ size_t pos(int axis, int r) const { return 3 * s + (size_t)axis * R + r; }
+  __host__ __device__ size_t out_hidden_row(int r, int D) const { return (o + r) * (size_t)D; }
+  __host__ __device__ size_t out_kv_row(int which, int r, int HD) const {
+    return (2 * o + (size_t)which * Ro + r) * (size_t)HD;
+  }
+  __host__ __device__ size_t out_pos(int axis, int r) const { return 3 * o + (size_t)axis * Ro + r; }
+};
+}  // namespace gmc
+
+namespace gmc {
+// Raise a kernel's dynamic shared-memory limit when a launch needs more than
+// the 48 KB default (idempotent; remembers the largest value set per kernel).
+cudaError_t set_smem_limit(const void* func, size_t bytes);
+}  // namespace gmc
+
+namespace gmc {
+cudaError_t launch_gram_simt(const Dims&, const void* hidden, Scratch&, cudaStream_t);
+}  // namespace gmc

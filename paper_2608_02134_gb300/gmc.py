@@ -1,0 +1,287 @@
+"""Python binding of libgmc.so: the same entry points as include/gmc.h.
+
+Argument marshalling only: every step of the compression runs in the CUDA
+library.  Tensors are torch tensors (device memory, or pinned host memory for
+the staged host path); the library is loaded on first use and a missing or
+unloadable build raises -- there is no fallback.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass, fields
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libgmc.so")
+
+GMC_OK, GMC_ERR_ARG, GMC_ERR_UNSUPPORTED, GMC_ERR_WORKSPACE, GMC_ERR_CUDA = range(5)
+GMC_F32, GMC_BF16 = 0, 1
+STATUS_NONFINITE, STATUS_TIMEOUT, STATUS_TEXT_LEN, STATUS_INTERNAL = 0x1, 0x2, 0x4, 0x8
+
+EXPORTS = (
+    "gmc_default_params", "gmc_workspace_size", "gmc_compress", "gmc_get_trace_layout",
+    "gmc_trace_size", "gmc_select_workspace_size", "gmc_select",
+    "gmc_transport_workspace_size", "gmc_transport", "gmc_read_status", "gmc_error_string",
+    "gmc_version", "gmc_profile_enable", "gmc_profile_read", "gmc_launch_count",
+)
+
+
+class Params(ctypes.Structure):
+    _fields_ = [
+        ("batch_b", ctypes.c_int), ("pool_mult", ctypes.c_int),
+        ("resp_temp", ctypes.c_float), ("resp_eps", ctypes.c_float),
+        ("tau_v", ctypes.c_float), ("tau_s", ctypes.c_float),
+        ("beta_G", ctypes.c_float), ("beta_V", ctypes.c_float), ("beta_S", ctypes.c_float),
+        ("landmarks", ctypes.c_int), ("max_head_clusters", ctypes.c_int),
+        ("head_eps", ctypes.c_float), ("terminal_q_weight", ctypes.c_float),
+        ("lambda_mass", ctypes.c_float), ("eps_mass", ctypes.c_float),
+        ("assign_spatial_w", ctypes.c_float), ("gate_scale", ctypes.c_float),
+        ("gate_pow", ctypes.c_float), ("ambig_margin", ctypes.c_float),
+        ("pop_strength", ctypes.c_float), ("rms_eps", ctypes.c_float),
+        ("norm_eps", ctypes.c_float), ("check_mode", ctypes.c_int),
+    ]
+
+
+class Problem(ctypes.Structure):
+    _fields_ = [("B", ctypes.c_int), ("grid_h", ctypes.c_int), ("grid_w", ctypes.c_int),
+                ("Hkv", ctypes.c_int), ("dtype", ctypes.c_int), ("text_offsets", ctypes.c_void_p)]
+
+
+class TraceHeader(ctypes.Structure):
+    _fields_ = [("K", ctypes.c_int32), ("rounds", ctypes.c_int32), ("n_clusters", ctypes.c_int32),
+                ("filled", ctypes.c_int32), ("s_x", ctypes.c_float), ("delta_bar", ctypes.c_float),
+                ("F_S", ctypes.c_float * 3), ("F_V", ctypes.c_float * 3), ("c_B", ctypes.c_float),
+                ("reserved", ctypes.c_int32 * 3)]
+
+
+class TraceLayout(ctypes.Structure):
+    _fields_ = [("bytes_per_image", ctypes.c_size_t), ("rounds_max", ctypes.c_int),
+                ("pool_size", ctypes.c_int), ("off_order", ctypes.c_size_t),
+                ("off_round_end", ctypes.c_size_t), ("off_pool", ctypes.c_size_t),
+                ("off_centres", ctypes.c_size_t), ("off_head_assign", ctypes.c_size_t),
+                ("off_omega", ctypes.c_size_t), ("off_pi", ctypes.c_size_t),
+                ("off_ebar", ctypes.c_size_t), ("off_mass", ctypes.c_size_t)]
+
+
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    """Load libgmc.so (raises if it is missing: build it with __graft_entry__.build())."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError(f"{LIB_PATH} is missing; build it with `python -c 'import __graft_entry__ as g; g.build()'`")
+    L = ctypes.CDLL(LIB_PATH)
+    vp, sz, i = ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int
+    P, PP = ctypes.POINTER(Params), ctypes.POINTER(Problem)
+    L.gmc_default_params.argtypes = [P]
+    L.gmc_default_params.restype = None
+    L.gmc_workspace_size.argtypes = [PP, i, i, i, i, i, i]
+    L.gmc_workspace_size.restype = sz
+    L.gmc_compress.argtypes = [PP, P, vp, vp, vp, vp, vp, i, i, i, i, i, i, vp, vp, vp, vp, vp,
+                               sz, vp, vp]
+    L.gmc_compress.restype = i
+    L.gmc_get_trace_layout.argtypes = [PP, P, i, i, i, i, ctypes.POINTER(TraceLayout)]
+    L.gmc_get_trace_layout.restype = i
+    L.gmc_trace_size.argtypes = [PP, P, i, i, i, i]
+    L.gmc_trace_size.restype = sz
+    L.gmc_select_workspace_size.argtypes = [i, i, i, i, P]
+    L.gmc_select_workspace_size.restype = sz
+    L.gmc_select.argtypes = [vp, i, i, i, i, P, vp, vp, sz, vp, vp]
+    L.gmc_select.restype = i
+    L.gmc_transport_workspace_size.argtypes = [PP, i, i, i]
+    L.gmc_transport_workspace_size.restype = sz
+    L.gmc_transport.argtypes = [PP, P, vp, vp, vp, vp, vp, vp, i, i, i, i, i, vp, vp, vp, vp, vp,
+                                sz, vp]
+    L.gmc_transport.restype = i
+    L.gmc_read_status.argtypes = [vp, ctypes.POINTER(ctypes.c_uint32), vp]
+    L.gmc_read_status.restype = i
+    L.gmc_error_string.argtypes = [i]
+    L.gmc_error_string.restype = ctypes.c_char_p
+    L.gmc_version.argtypes = []
+    L.gmc_version.restype = ctypes.c_char_p
+    L.gmc_profile_enable.argtypes = [i]
+    L.gmc_profile_enable.restype = i
+    L.gmc_profile_read.argtypes = [ctypes.POINTER(ctypes.c_float), ctypes.POINTER(ctypes.c_char_p), i]
+    L.gmc_profile_read.restype = i
+    L.gmc_launch_count.argtypes = []
+    L.gmc_launch_count.restype = ctypes.c_uint64
+    _lib = L
+    return L
+
+
+class GMCError(RuntimeError):
+    pass
+
+
+def _check(rc: int):
+    if rc != GMC_OK:
+        raise GMCError(lib().gmc_error_string(rc).decode())
+
+
+def default_params(**overrides) -> Params:
+    p = Params()
+    lib().gmc_default_params(ctypes.byref(p))
+    for k, v in overrides.items():
+        if k not in {f[0] for f in Params._fields_}:
+            raise KeyError(k)
+        setattr(p, k, v)
+    return p
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def problem(B, grid_h, grid_w, Hkv, dtype, text_offsets=None) -> Problem:
+    return Problem(B, grid_h, grid_w, Hkv, dtype, None if text_offsets is None else text_offsets.data_ptr())
+
+
+def workspace_size(prob: Problem, N, T, H, d, D, K) -> int:
+    return int(lib().gmc_workspace_size(ctypes.byref(prob), N, T, H, d, D, K))
+
+
+def trace_layout(prob: Problem, params: Params, N, T, H, K) -> TraceLayout:
+    L = TraceLayout()
+    _check(lib().gmc_get_trace_layout(ctypes.byref(prob), ctypes.byref(params), N, T, H, K, ctypes.byref(L)))
+    return L
+
+
+def alloc_workspace(nbytes: int, device="cuda") -> torch.Tensor:
+    # torch's caching allocator returns 512-byte aligned blocks
+    return torch.empty(max(nbytes, 256), dtype=torch.uint8, device=device)
+
+
+def compress(prob: Problem, params: Params, hidden, keys, queries, pos_ids, vo_probe,
+             N, T, H, d, D, K, out_idx, out_hidden, out_kv, out_pos, workspace, trace=None,
+             stream=None):
+    """gmc_compress on device tensors (see include/gmc.h for layouts)."""
+    _check(lib().gmc_compress(
+        ctypes.byref(prob), ctypes.byref(params), _ptr(hidden), _ptr(keys), _ptr(queries),
+        _ptr(pos_ids), _ptr(vo_probe), N, T, H, d, D, K, _ptr(out_idx), _ptr(out_hidden),
+        _ptr(out_kv), _ptr(out_pos), _ptr(workspace), workspace.numel(), _ptr(trace),
+        _stream(stream)))
+
+
+def select(clients, B, M, N, K, params: Params, out_idx, workspace, trace=None, stream=None):
+    _check(lib().gmc_select(_ptr(clients), B, M, N, K, ctypes.byref(params), _ptr(out_idx),
+                            _ptr(workspace), workspace.numel(), _ptr(trace), _stream(stream)))
+
+
+def select_workspace_size(B, M, N, K, params: Params) -> int:
+    return int(lib().gmc_select_workspace_size(B, M, N, K, ctypes.byref(params)))
+
+
+def transport(prob: Problem, params: Params, hidden, keys, pos_ids, support, assign, weights,
+              N, T, d, D, K, out_idx, out_hidden, out_kv, out_pos, workspace, stream=None):
+    _check(lib().gmc_transport(
+        ctypes.byref(prob), ctypes.byref(params), _ptr(hidden), _ptr(keys), _ptr(pos_ids),
+        _ptr(support), _ptr(assign), _ptr(weights), N, T, d, D, K, _ptr(out_idx),
+        _ptr(out_hidden), _ptr(out_kv), _ptr(out_pos), _ptr(workspace), workspace.numel(),
+        _stream(stream)))
+
+
+def transport_workspace_size(prob: Problem, N, T, K) -> int:
+    return int(lib().gmc_transport_workspace_size(ctypes.byref(prob), N, T, K))
+
+
+def read_status(workspace, stream=None) -> int:
+    st = ctypes.c_uint32(0)
+    _check(lib().gmc_read_status(_ptr(workspace), ctypes.byref(st), _stream(stream)))
+    return int(st.value)
+
+
+def version() -> str:
+    return lib().gmc_version().decode()
+
+
+def profile_enable(on: bool):
+    lib().gmc_profile_enable(1 if on else 0)
+
+
+def profile_read() -> dict:
+    """Per-stage milliseconds of the last profiled gmc_compress call."""
+    ms = (ctypes.c_float * 16)()
+    names = (ctypes.c_char_p * 16)()
+    n = lib().gmc_profile_read(ms, names, 16)
+    return {names[k].decode(): float(ms[k]) for k in range(max(n, 0))}
+
+
+def launch_count() -> int:
+    return int(lib().gmc_launch_count())
+
+
+# ---------------------------------------------------------------------------
+# Convenience: one call on a workload, outputs as torch tensors
+# ---------------------------------------------------------------------------
+@dataclass
+class Outputs:
+    idx: torch.Tensor
+    hidden: torch.Tensor
+    kv: torch.Tensor
+    pos: torch.Tensor
+    K: int
+    trace: torch.Tensor | None = None
+    layout: TraceLayout | None = None
+
+
+class Compressor:
+    """Holds device buffers for repeated gmc_compress calls on one problem shape.
+
+    Inputs are device tensors in the C-ABI layout; ``run`` launches one call
+    on the current stream.  ``run_host`` stages pinned host inputs in, runs,
+    and copies the outputs back (the end-to-end path through host memory).
+    """
+
+    def __init__(self, B, grid_h, grid_w, T, H, Hkv, d, D, K, dtype, text_lengths=None,
+                 params: Params | None = None, trace=False, device="cuda"):
+        self.B, self.gh, self.gw, self.T, self.H, self.Hkv, self.d, self.D = B, grid_h, grid_w, T, H, Hkv, d, D
+        self.N = grid_h * grid_w
+        self.Kr = K
+        self.K = min(self.N, max(1, K))
+        self.dtype = dtype
+        self.tdt = torch.bfloat16 if dtype == GMC_BF16 else torch.float32
+        self.params = params or default_params()
+        self.device = device
+        lens = list(text_lengths) if text_lengths is not None else [T] * B
+        self.text_lengths = lens
+        off = [0]
+        for t in lens:
+            off.append(off[-1] + t)
+        self.offsets = torch.tensor(off, dtype=torch.int32, device=device) if text_lengths is not None else None
+        self.prob = problem(B, grid_h, grid_w, Hkv, dtype, self.offsets)
+        ws = workspace_size(self.prob, self.N, T, H, d, D, K)
+        if ws == 0:
+            raise GMCError("invalid problem for gmc_workspace_size")
+        self.workspace = alloc_workspace(ws, device)
+        tot_text = off[-1]
+        Kx = self.K
+        self.out_idx = torch.empty(B * Kx, dtype=torch.int32, device=device)
+        self.out_hidden = torch.empty((B * Kx + tot_text, D), dtype=self.tdt, device=device)
+        self.out_kv = torch.empty((2 * (B * Kx + tot_text), Hkv, d), dtype=self.tdt, device=device)
+        self.out_pos = torch.empty(3 * (B * Kx + tot_text), dtype=torch.int32, device=device)
+        self.trace = None
+        self.layout = None
+        if trace:
+            self.layout = trace_layout(self.prob, self.params, self.N, T, H, K)
+            self.trace = torch.zeros(B * self.layout.bytes_per_image, dtype=torch.uint8, device=device)
+
+    def run(self, hidden, keys, queries, pos_ids, vo_probe, stream=None):
+        compress(self.prob, self.params, hidden, keys, queries, pos_ids, vo_probe, self.N, self.T,
+                 self.H, self.d, self.D, self.Kr, self.out_idx, self.out_hidden, self.out_kv,
+                 self.out_pos, self.workspace, self.trace, stream)
+        return Outputs(self.out_idx, self.out_hidden, self.out_kv, self.out_pos, self.K, self.trace,
+                       self.layout)
+
+    def status(self, stream=None) -> int:
+        return read_status(self.workspace, stream)

@@ -1,0 +1,134 @@
+"""Run workloads through the C-ABI on the GPU and compare them with the oracle."""
+
+from __future__ import annotations
+
+from dataclasses import dataclass
+
+import numpy as np
+import torch
+
+from oracle import gmc_oracle as O
+from paper_2608_02134_gb300 import gmc, workloads
+from tests import parity
+
+
+@dataclass
+class GpuRun:
+    wl: workloads.Workload
+    comp: gmc.Compressor
+    idx: np.ndarray
+    hidden: np.ndarray      # float64 values
+    hidden_raw: np.ndarray  # raw bits (uint16 for bf16, float32 for fp32)
+    kv: np.ndarray
+    pos: np.ndarray
+    status: int
+    traces: list
+
+
+def to_device(wl: workloads.Workload, device="cuda"):
+    arr = wl.abi_arrays()
+    out = {}
+    for k, v in arr.items():
+        if k == "text_offsets":
+            continue
+        t = torch.from_numpy(np.ascontiguousarray(v))
+        if v.dtype == np.uint16:
+            t = t.view(torch.int16).view(torch.bfloat16)
+        out[k] = t.to(device)
+    return out
+
+
+def run(wl: workloads.Workload, params=None, trace=True, inputs=None) -> GpuRun:
+    dt = gmc.GMC_BF16 if wl.dtype == "bf16" else gmc.GMC_F32
+    inp = inputs or to_device(wl)
+    comp = gmc.Compressor(wl.B, wl.gh, wl.gw, wl.T_max, wl.H, wl.Hkv, wl.d, wl.D, wl.K, dt,
+                          text_lengths=wl.T if wl.ragged else None, params=params, trace=trace)
+    out = comp.run(inp["hidden"], inp["keys"], inp["queries"], inp["pos_ids"], inp["vo_probe"])
+    torch.cuda.synchronize()
+    status = comp.status()
+    hid = out.hidden.float().cpu().numpy().astype(np.float64)
+    raw = (out.hidden.view(torch.int16).cpu().numpy().view(np.uint16) if dt == gmc.GMC_BF16
+           else out.hidden.cpu().numpy())
+    traces = []
+    if trace:
+        traces = parity.parse_trace(out.trace.cpu().numpy(), out.layout, wl.B, comp.K, wl.H, wl.N,
+                                    comp.params.max_head_clusters)
+    return GpuRun(wl, comp, out.idx.cpu().numpy(), hid, raw, out.kv.float().cpu().numpy(),
+                  out.pos.cpu().numpy(), status, traces)
+
+
+def oracle_params(p: gmc.Params) -> dict:
+    return O.params(batch_b=p.batch_b, pool_mult=p.pool_mult, resp_temp=p.resp_temp,
+                    resp_eps=p.resp_eps, tau_v=p.tau_v, tau_s=p.tau_s, beta_G=p.beta_G,
+                    beta_V=p.beta_V, beta_S=p.beta_S, landmarks=p.landmarks,
+                    max_head_clusters=p.max_head_clusters, head_eps=p.head_eps,
+                    terminal_q_weight=p.terminal_q_weight, lambda_mass=p.lambda_mass,
+                    eps_mass=p.eps_mass, assign_spatial_w=p.assign_spatial_w,
+                    gate_scale=p.gate_scale, gate_pow=p.gate_pow, ambig_margin=p.ambig_margin,
+                    pop_strength=p.pop_strength, rms_eps=p.rms_eps, norm_eps=p.norm_eps)
+
+
+@dataclass
+class ImageReport:
+    b: int
+    dec: parity.Decisions
+    hidden_err: float
+    sx_err: float
+    n_rounds: int
+
+
+def compare_image(g: GpuRun, b: int, hidden_tol: float) -> ImageReport:
+    """Forced oracle run along the GPU's decisions; validate them; compare outputs."""
+    wl = g.wl
+    K = g.comp.K
+    N, H = wl.N, wl.H
+    T = wl.T[b]
+    off = int(np.sum(wl.T[:b]))
+    im = wl.image(b)
+    tr = g.traces[b]
+    p = oracle_params(g.comp.params)
+    f = lambda a: np.asarray(a, dtype=np.float64)
+    nc = min(p["max_head_clusters"], H)
+    forced = dict(centres=tr.centres[:nc].tolist(), head_assign=tr.head_assign.tolist(),
+                  rounds=tr.forced_rounds(), pi=tr.pi)
+    res = O.compress(f(im.hidden), f(im.keys), f(im.values), f(im.queries), im.pos, f(wl.probe()),
+                     wl.gh, wl.gw, wl.K, p, forced=forced)
+    dec = parity.Decisions()
+    tag = f"{wl.name}[b={b}]"
+    parity.check_heads(res.heads, dec, tag)
+    parity.check_selection(res.selection, p["pool_mult"] * p["batch_b"], dec, tag)
+    parity.check_assignment(res.assignment, res.support, dec, tag)
+    # outputs of this image
+    o = b * K + off
+    idx = g.idx[b * K:(b + 1) * K]
+    if not np.array_equal(idx, res.support):
+        dec.failures.append(f"{tag} out_idx differs from the forced support")
+    rows = g.hidden[o:o + K + T]
+    err = parity.rel_row_err(rows[:K], res.out_hidden[:K])
+    if err > hidden_tol:
+        dec.failures.append(f"{tag} transported rows max rel err {err:.3e} > {hidden_tol}")
+    if not np.array_equal(rows[K:], f(im.hidden[N:])):
+        dec.failures.append(f"{tag} text rows are not bit-exact copies")
+    kvo = g.kv[2 * o:2 * (o + K + T)].reshape(2, K + T, wl.Hkv, wl.d)
+    if not np.array_equal(kvo, res.out_kv):
+        dec.failures.append(f"{tag} compact K/V rows differ")
+    pos = g.pos[3 * o:3 * (o + K + T)].reshape(3, K + T)
+    if not np.array_equal(pos, res.out_pos):
+        dec.failures.append(f"{tag} position ids differ")
+    sx_err = abs(tr.s_x - res.assignment.s_x)
+    if sx_err > 1e-4:
+        dec.failures.append(f"{tag} s_x {tr.s_x} vs {res.assignment.s_x}")
+    if not np.allclose(tr.omega, res.heads.omega, rtol=1e-4, atol=1e-7):
+        dec.failures.append(f"{tag} head weights differ")
+    if not np.allclose(tr.ebar, res.ebar, rtol=1e-4, atol=1e-6):
+        dec.failures.append(f"{tag} ebar differs (max {np.max(np.abs(tr.ebar - res.ebar)):.2e})")
+    if not np.allclose(tr.mass, res.m, rtol=1e-5, atol=1e-6):
+        dec.failures.append(f"{tag} population weights differ")
+    if tr.n_clusters != res.heads.n_clusters:
+        dec.failures.append(f"{tag} cluster count {tr.n_clusters} vs {res.heads.n_clusters}")
+    sat = O.bank_saturation(res.clients, res.support)
+    for q, bank in enumerate(("grounded", "appearance", "spatial")):
+        fs, fv, _ = sat[bank]
+        if abs(tr.F_S[q] - fs) > 1e-4 * max(fv, 1e-12) or abs(tr.F_V[q] - fv) > 1e-4 * max(fv, 1e-12):
+            dec.failures.append(f"{tag} bank {bank} F(S)/F(V) {tr.F_S[q]}/{tr.F_V[q]} vs {fs}/{fv}")
+    return ImageReport(b, dec, err, sx_err, len(res.selection.rounds))

@@ -1,0 +1,116 @@
+"""CPU tests of the C-ABI library: it builds, loads without a GPU, exports every
+entry point include/gmc.h declares, and its host-side logic (defaults, sizing,
+argument validation) behaves as documented.  No compute call is made."""
+
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def gmc():
+    from paper_2608_02134_gb300 import build
+    build.build()
+    from paper_2608_02134_gb300 import gmc as g
+    g.lib()
+    return g
+
+
+def declared_functions():
+    src = open(os.path.join(ROOT, "include", "gmc.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(gmc_\w+)\s*\(", src)))
+
+
+def test_every_declared_symbol_is_exported(gmc):
+    names = declared_functions()
+    assert len(names) >= 12
+    L = ctypes.CDLL(gmc.LIB_PATH)
+    for n in names:
+        assert hasattr(L, n), f"{n} declared in include/gmc.h but not exported"
+    assert set(names) == set(gmc.EXPORTS)
+
+
+def test_defaults_are_the_papers_configuration(gmc):
+    """Table "Shared GMC configuration" (fixed-token settings)."""
+    p = gmc.default_params()
+    assert (p.batch_b, p.pool_mult, p.landmarks, p.max_head_clusters) == (16, 4, 16, 4)
+    vals = dict(resp_temp=0.1, tau_v=0.2, tau_s=0.02, beta_V=0.5, beta_S=0.25, lambda_mass=1.0,
+                eps_mass=1e-8, assign_spatial_w=0.5, gate_scale=0.08, gate_pow=8.0,
+                ambig_margin=0.05, pop_strength=0.5, terminal_q_weight=2.0, head_eps=0.05)
+    for k, v in vals.items():
+        assert getattr(p, k) == pytest.approx(v, rel=1e-6), k
+    assert p.check_mode == 0
+    assert gmc.version().startswith("gmc ")
+
+
+def test_struct_sizes_match_header(gmc):
+    # 23 four-byte fields / 6 fields with one pointer
+    assert ctypes.sizeof(gmc.Params) == 23 * 4
+    assert ctypes.sizeof(gmc.TraceHeader) == 64
+
+
+def test_workspace_and_trace_sizing(gmc):
+    pr = gmc.problem(1, 36, 36, 4, gmc.GMC_BF16)
+    ws = gmc.workspace_size(pr, 1296, 64, 28, 128, 3584, 257)
+    # it holds at least the client matrix and the attention slice
+    M = 28 * 64 + 1296 + 256
+    assert ws >= M * 1296 * 4 + 28 * 64 * 1296 * 4
+    pr32 = gmc.problem(32, 36, 36, 4, gmc.GMC_BF16)
+    assert gmc.workspace_size(pr32, 1296, 64, 28, 128, 3584, 257) > 31 * ws
+    assert gmc.workspace_size(gmc.problem(1, 36, 35, 4, 1), 1296, 64, 28, 128, 3584, 257) == 0
+    assert gmc.workspace_size(pr, 1296, 64, 30, 128, 3584, 257) == 0      # H % Hkv != 0
+    L = gmc.trace_layout(pr, gmc.default_params(), 1296, 64, 28, 257)
+    assert L.rounds_max == 17 + 1 and L.pool_size == 64
+    assert L.off_order >= 64 and L.bytes_per_image % 16 == 0
+    assert L.off_mass + 4 * 1296 <= L.bytes_per_image
+    assert gmc.lib().gmc_trace_size(ctypes.byref(pr32), None, 1296, 64, 28, 257) == 32 * L.bytes_per_image
+
+
+def _compress_rc(gmc, prob=None, ws_bytes=1 << 40, null=None, params=None, **shape):
+    lib = gmc.lib()
+    sh = dict(N=64, T=8, H=4, d=64, D=256, K=16)
+    sh.update(shape)
+    prob = prob or gmc.problem(1, 8, 8, 4, gmc.GMC_F32)
+    fake = ctypes.c_void_p(1 << 20)    # aligned, never dereferenced: validation fails first
+    ptrs = [fake] * 9
+    if null is not None:
+        ptrs[null] = None
+    h, k, q, pos, w, oi, oh, okv, op = ptrs
+    return lib.gmc_compress(ctypes.byref(prob), params, h, k, q, pos, w, sh["N"], sh["T"], sh["H"],
+                            sh["d"], sh["D"], sh["K"], oi, oh, okv, op, fake, ws_bytes, None, None)
+
+
+def test_argument_validation(gmc):
+    assert _compress_rc(gmc, null=0) == gmc.GMC_ERR_ARG
+    assert _compress_rc(gmc, null=6) == gmc.GMC_ERR_ARG
+    assert _compress_rc(gmc, N=63) == gmc.GMC_ERR_ARG                     # N != grid_h*grid_w
+    assert _compress_rc(gmc, H=6) == gmc.GMC_ERR_ARG                      # H % Hkv
+    assert _compress_rc(gmc, T=0) == gmc.GMC_ERR_ARG
+    assert _compress_rc(gmc, H=128, prob=gmc.problem(1, 8, 8, 4, 0)) == gmc.GMC_ERR_UNSUPPORTED
+    assert _compress_rc(gmc, D=250) == gmc.GMC_ERR_UNSUPPORTED           # D % 8
+    assert _compress_rc(gmc, ws_bytes=1024) == gmc.GMC_ERR_WORKSPACE
+    bad = gmc.default_params(batch_b=64, pool_mult=4)                    # pool 256 > GMC_MAX_POOL
+    assert _compress_rc(gmc, params=ctypes.byref(bad)) == gmc.GMC_ERR_ARG
+    assert _compress_rc(gmc, prob=gmc.problem(1, 8, 8, 4, 7)) == gmc.GMC_ERR_ARG   # dtype
+    assert "WORKSPACE" in gmc.lib().gmc_error_string(gmc.GMC_ERR_WORKSPACE).decode()
+
+
+def test_select_and_transport_validation(gmc):
+    lib = gmc.lib()
+    fake = ctypes.c_void_p(1 << 20)
+    p = gmc.default_params()
+    assert lib.gmc_select(fake, 1, 10, 20, 25, ctypes.byref(p), fake, fake, 1 << 30, None, None) \
+        == gmc.GMC_ERR_ARG                                                 # K > N
+    assert lib.gmc_select(fake, 1, 10, 20, 5, ctypes.byref(p), fake, fake, 16, None, None) \
+        == gmc.GMC_ERR_WORKSPACE
+    assert gmc.select_workspace_size(1, 10, 20, 5, p) >= 10 * 20 * 6
+    pr = gmc.problem(1, 4, 5, 1, gmc.GMC_F32)
+    assert gmc.transport_workspace_size(pr, 20, 3, 5) > 0
+    assert lib.gmc_transport(ctypes.byref(pr), None, fake, fake, fake, fake, fake, fake, 20, 3, 8,
+                             16, 0, fake, fake, fake, fake, fake, 1 << 30, None) == gmc.GMC_ERR_ARG
+    assert lib.gmc_read_status(None, None, None) == gmc.GMC_ERR_ARG

@@ -1,0 +1,129 @@
+"""GPU parity: gmc_compress through the C-ABI against the fp64 oracle.
+
+Bar (per image): every discrete choice is a valid choice of the oracle's
+fp64 values within the relative margin 1e-4 (so the kept indices are
+bit-exact wherever the margin exceeds it); transported rows within max
+row-relative error 1e-3 (fp32 inputs) or 2e-2 (bf16 inputs, fp32
+accumulation); text rows, compact K/V and position ids bit-exact.
+"""
+
+import numpy as np
+import pytest
+import torch
+
+pytestmark = pytest.mark.gpu
+
+TOL_F32, TOL_BF16 = 1e-3, 2e-2
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2608_02134_gb300 import gmc
+    gmc.lib()
+
+
+def _check(g, images, tol):
+    from tests import gpu_harness as GH
+    assert g.status == 0, f"device status {g.status:#x}"
+    reports = [GH.compare_image(g, b, tol) for b in images]
+    fails = [f for r in reports for f in r.dec.failures]
+    ties = sum(len(r.dec.near_ties) for r in reports)
+    checked = sum(r.dec.checked for r in reports)
+    print(f"{g.wl.name}: {checked} decisions checked, {ties} near-ties followed, "
+          f"max hidden err {max(r.hidden_err for r in reports):.2e}")
+    assert not fails, "\n".join(fails[:20])
+    return reports
+
+
+def test_tiny_fp32():
+    from paper_2608_02134_gb300 import workloads
+    from tests import gpu_harness as GH
+    wl = workloads.make("tiny")
+    _check(GH.run(wl), [0], TOL_F32)
+
+
+@pytest.mark.parametrize("K", [64, 128, 192])
+def test_llava_shape(K):
+    from paper_2608_02134_gb300 import workloads
+    from tests import gpu_harness as GH
+    wl = workloads.make("llava", K=K)
+    _check(GH.run(wl), [0], TOL_BF16)
+
+
+def test_qwen_shape():
+    from paper_2608_02134_gb300 import workloads
+    from tests import gpu_harness as GH
+    wl = workloads.make("qwen")
+    _check(GH.run(wl), [0], TOL_BF16)
+
+
+def test_document_shape():
+    from paper_2608_02134_gb300 import workloads
+    from tests import gpu_harness as GH
+    wl = workloads.make("doc")
+    _check(GH.run(wl), [0], TOL_BF16)
+
+
+def test_serving_batch_sampled():
+    """32 ragged images in one call; the oracle checks a sample of them."""
+    from paper_2608_02134_gb300 import workloads
+    from tests import gpu_harness as GH
+    wl = workloads.make("serving")
+    g = GH.run(wl)
+    _check(g, [0, 13, 31], TOL_BF16)
+    # every image: support sorted, unique, in range, and the right size
+    K = g.comp.K
+    for b in range(wl.B):
+        s = g.idx[b * K:(b + 1) * K]
+        assert np.all(np.diff(s) > 0) and s[0] >= 0 and s[-1] < wl.N
+
+
+@pytest.mark.parametrize("shape", [
+    dict(gh=5, gw=7, H=3, Hkv=1, d=16, D=40, T=3, K=9),      # ragged tiles, GQA 3:1
+    dict(gh=6, gw=6, H=2, Hkv=2, d=8, D=16, T=1, K=1),       # one text query, K = 1
+    dict(gh=9, gw=11, H=8, Hkv=2, d=32, D=64, T=17, K=40),   # more heads than clusters
+])
+def test_small_shapes_fp32(shape):
+    from paper_2608_02134_gb300 import workloads
+    from tests import gpu_harness as GH
+    K = shape.pop("K")
+    T = shape.pop("T")
+    wl = workloads.make("tiny", K=K, T=T, **shape)
+    _check(GH.run(wl), [0], TOL_F32)
+
+
+def test_small_shape_bf16_strong_gate():
+    """Low hidden dimension spreads the cosines, so s_x > 0 and the spatial term acts."""
+    from paper_2608_02134_gb300 import workloads
+    from tests import gpu_harness as GH
+    wl = workloads.make("qwen", gh=12, gw=12, T=20, D=64, H=8, Hkv=2, K=30)
+    g = GH.run(wl)
+    reps = _check(g, [0], TOL_BF16)
+    assert g.traces[0].s_x > 0.0
+
+
+def test_identity_when_K_equals_N():
+    from paper_2608_02134_gb300 import workloads
+    from tests import gpu_harness as GH
+    wl = workloads.make("tiny", K=64)
+    g = GH.run(wl, trace=False)
+    im = wl.image(0)
+    assert np.array_equal(g.idx, np.arange(64))
+    assert np.array_equal(g.hidden, im.hidden.astype(np.float64))
+    assert np.array_equal(g.pos, im.pos.reshape(-1))
+    wl2 = workloads.make("tiny", K=500)        # K_r > N clamps to N: identity
+    g2 = GH.run(wl2, trace=False)
+    assert np.array_equal(g2.hidden, im.hidden.astype(np.float64))
+
+
+def test_deterministic_repeat():
+    from paper_2608_02134_gb300 import workloads
+    from tests import gpu_harness as GH
+    wl = workloads.make("llava", K=128)
+    inp = GH.to_device(wl)
+    a = GH.run(wl, inputs=inp)
+    b = GH.run(wl, inputs=inp)
+    assert np.array_equal(a.idx, b.idx)
+    assert np.array_equal(a.hidden_raw, b.hidden_raw)
