@@ -241,6 +241,42 @@ int gmc_transport(const gmc_problem* prob, const gmc_params* params, const void*
                   void* workspace, size_t ws_bytes, gmc_stream_t stream);
 
 /*
+ * gmc_transport_noalloc -- gmc_transport for callers that cannot allocate
+ * device memory.  The paper has no counterpart: this is a deployment variant.
+ *
+ * Who needs it: code that may only launch work into memory someone else
+ * already owns -- an inference-engine plugin inside its enqueue(), a caller
+ * that is inside a CUDA graph capture (an allocation there breaks or
+ * invalidates the capture), a server whose device pool is fixed at start-up.
+ * Such callers pass inputs and outputs exactly as for gmc_transport, but no
+ * workspace: the scratch (a status word and one float per visual row) lives
+ * in a fixed array inside libgmc.so, sized for GMC_NOALLOC_MAX_ROWS visual
+ * rows (B * N) plus 256 bytes.  Every GPU that loads the library keeps that
+ * array (about 256 KiB) until the process exits.
+ *
+ *   - Larger problems (B * N > GMC_NOALLOC_MAX_ROWS) are rejected with
+ *     GMC_ERR_UNSUPPORTED before anything is launched.
+ *   - It calls no cudaMalloc, cudaFree or other allocating routine.
+ *   - The first call made with a given device current looks up the array's
+ *     device address (cudaGetSymbolAddress) and caches it; make that first
+ *     call before any stream capture that includes this entry point.
+ *   - All calls share the one array.  Calls that overlap on the GPU (other
+ *     streams, other host threads) race on it; serialise them.  The status
+ *     word is cleared at the start of every call; the rest is overwritten.
+ *   - device_status: NULL, or a caller-owned device uint32 that receives the
+ *     GMC_STATUS_* bits of this call (cleared first); with NULL the bits stay
+ *     in the library's array and cannot be read back.
+ *   - Its kernels are not counted by gmc_launch_count().
+ * Arguments, layouts and results are those of gmc_transport.
+ */
+#define GMC_NOALLOC_MAX_ROWS 65536
+int gmc_transport_noalloc(const gmc_problem* prob, const gmc_params* params, const void* hidden,
+                          const void* keys, const int32_t* pos_ids, const int32_t* support,
+                          const int32_t* assign, const float* weights, int N, int T, int d, int D,
+                          int K, int32_t* out_idx, void* out_hidden, void* out_kv,
+                          int32_t* out_pos, uint32_t* device_status, gmc_stream_t stream);
+
+/*
  * Synchronise `stream`, then copy the device status word of `workspace`
  * (as passed to the last call that used it) into *status.  The word is
  * cleared at the start of every gmc_compress / gmc_select / gmc_transport

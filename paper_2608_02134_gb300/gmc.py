@@ -26,6 +26,7 @@ EXPORTS = (
     "gmc_trace_size", "gmc_select_workspace_size", "gmc_select",
     "gmc_transport_workspace_size", "gmc_transport", "gmc_read_status", "gmc_error_string",
     "gmc_version", "gmc_profile_enable", "gmc_profile_read", "gmc_launch_count",
+    "gmc_transport_noalloc",
 )
 
 
@@ -111,6 +112,9 @@ def lib() -> ctypes.CDLL:
     L.gmc_profile_read.restype = i
     L.gmc_launch_count.argtypes = []
     L.gmc_launch_count.restype = ctypes.c_uint64
+    L.gmc_transport_noalloc.argtypes = [PP, P, vp, vp, vp, vp, vp, vp, i, i, i, i, i, vp, vp, vp,
+                                        vp, vp, vp]
+    L.gmc_transport_noalloc.restype = i
     _lib = L
     return L
 
@@ -189,6 +193,16 @@ def transport(prob: Problem, params: Params, hidden, keys, pos_ids, support, ass
         _ptr(support), _ptr(assign), _ptr(weights), N, T, d, D, K, _ptr(out_idx),
         _ptr(out_hidden), _ptr(out_kv), _ptr(out_pos), _ptr(workspace), workspace.numel(),
         _stream(stream)))
+
+
+def transport_noalloc(prob: Problem, params: Params, hidden, keys, pos_ids, support, assign,
+                      weights, N, T, d, D, K, out_idx, out_hidden, out_kv, out_pos,
+                      device_status=None, stream=None):
+    """gmc_transport_noalloc: gmc_transport without a workspace (scratch inside the library)."""
+    _check(lib().gmc_transport_noalloc(
+        ctypes.byref(prob), ctypes.byref(params), _ptr(hidden), _ptr(keys), _ptr(pos_ids),
+        _ptr(support), _ptr(assign), _ptr(weights), N, T, d, D, K, _ptr(out_idx),
+        _ptr(out_hidden), _ptr(out_kv), _ptr(out_pos), _ptr(device_status), _stream(stream)))
 
 
 def transport_workspace_size(prob: Problem, N, T, K) -> int:
