@@ -224,6 +224,19 @@ int gmc_select(const float* clients, int B, int M, int N, int K, const gmc_param
                gmc_stream_t stream);
 
 /*
+ * gmc_cosine -- the cosine matrix of the visual boundary states alone,
+ * cos_ij = h_i . h_j / (max(||h_i||, eps) max(||h_j||, eps)) (appendix Eq.
+ * (cond-aux-clients), (cond-assignment)), as gmc_compress computes it: bf16
+ * states on the tcgen05 tensor cores with fp32 accumulation, fp32 states on
+ * CUDA cores.  hidden as gmc_compress (only the visual rows are read);
+ * out_cos fp32 [B][N][N].  d is not used.
+ */
+size_t gmc_cosine_workspace_size(const gmc_problem* prob, int N);
+int gmc_cosine(const gmc_problem* prob, const gmc_params* params, const void* hidden, int N,
+               int T, int D, float* out_cos, void* workspace, size_t ws_bytes,
+               gmc_stream_t stream);
+
+/*
  * gmc_transport -- population transport and physical compaction for a given
  * support and assignment (Sec. 3.4, Eq. (5); appendix Eq. (cond-transport);
  * Algorithm 1 step 6).  Inputs as gmc_compress, plus

@@ -409,6 +409,44 @@ int gmc_select(const float* clients, int B, int M, int N, int K, const gmc_param
 }
 
 // ---------------------------------------------------------------------------
+// gmc_cosine
+// ---------------------------------------------------------------------------
+size_t gmc_cosine_workspace_size(const gmc_problem* prob, int N) {
+  if (!prob || prob->B < 1 || N < 1) return 0;
+  Carver c{nullptr};
+  c.take<uint32_t>(4);
+  c.take<float>((size_t)prob->B * N * 2);
+  return c.off;
+}
+
+int gmc_cosine(const gmc_problem* prob, const gmc_params* params, const void* hidden, int N,
+               int T, int D, float* out_cos, void* workspace, size_t ws_bytes,
+               gmc_stream_t stream_) {
+  int rc = check_problem(prob, N, T, 8, D);
+  if (rc != GMC_OK) return rc;
+  gmc_params p;
+  if (params) p = *params; else gmc_default_params(&p);
+  if (!params_ok(p)) return GMC_ERR_ARG;
+  if (!hidden || !out_cos || !workspace) return GMC_ERR_ARG;
+  if (!aligned(hidden, 16) || !aligned(out_cos, 16) || !aligned(workspace, ALIGN))
+    return GMC_ERR_ARG;
+  if (ws_bytes < gmc_cosine_workspace_size(prob, N)) return GMC_ERR_WORKSPACE;
+  Carver c{(char*)workspace};
+  Scratch s{};
+  s.status = c.take<uint32_t>(4);
+  s.rn = c.take<float>((size_t)prob->B * N);
+  s.rmsh = c.take<float>((size_t)prob->B * N);
+  s.cos = out_cos;
+  cudaStream_t st = (cudaStream_t)stream_;
+  const Dims dm = make_dims(prob, p, N, T, 0, 8, D, 1);
+  GMC_TRY(cudaMemsetAsync(s.status, 0, sizeof(uint32_t), st));
+  GMC_TRY(launch_rownorm(dm, hidden, p.norm_eps, s, st));
+  GMC_TRY(launch_gram(dm, hidden, s, st));
+  g_launches += 2;
+  return GMC_OK;
+}
+
+// ---------------------------------------------------------------------------
 // gmc_transport
 // ---------------------------------------------------------------------------
 size_t gmc_transport_workspace_size(const gmc_problem* prob, int N, int T, int K) {

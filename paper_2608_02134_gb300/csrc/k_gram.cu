@@ -77,6 +77,9 @@ cudaError_t launch_gram_simt(const Dims& dm, const void* hidden, Scratch& s, cud
 }
 
 cudaError_t launch_gram(const Dims& dm, const void* hidden, Scratch& s, cudaStream_t st) {
+  // bf16 states with at least one full 128-row tile: tcgen05 (k_gram_tc.cu);
+  // fp32 states (exact fp32 products) and tiny grids: the CUDA-core kernel above.
+  if (gram_tc_supported(dm)) return launch_gram_tc(dm, hidden, s, st);
   return launch_gram_simt(dm, hidden, s, st);
 }
 

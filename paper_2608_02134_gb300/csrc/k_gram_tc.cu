@@ -1,0 +1,231 @@
+// Cosine matrix of the boundary states on the tcgen05 tensor cores (bf16 path).
+//
+// cos_ij = (h_i . h_j) / (n_i n_j): the appearance clients of appendix Eq.
+// (cond-aux-clients) and the assignment cosines of Eq. (cond-assignment).  The
+// Gram runs on the raw bf16 states with fp32 accumulation in tensor memory and
+// is normalised afterwards in fp32 (the states are never rounded after
+// normalisation).
+//
+// One CTA computes one 128 x 128 tile of the upper triangle (I <= J) and writes
+// it and its mirror.  Warp 0 / lane 0 streams 64-wide K slices of both row
+// blocks with TMA (128-byte swizzle) through a 6-stage mbarrier ring; warp 1 /
+// lane 0 issues tcgen05.mma (M = N = 128, K = 16) into a 128-column TMEM
+// accumulator; all four warps then read their 32 TMEM lanes and store.  The
+// last, ragged tile of an image is shifted inward (start N - 128) so every TMA
+// box lies inside the image's own rows; it stores only the rows and columns
+// the previous tile does not own.
+#include "common.cuh"
+#include "kernels.cuh"
+#include "tc.cuh"
+
+namespace gmc {
+
+namespace {
+constexpr int BM = 128, BK = 64, STAGES = 6;
+constexpr int TILE_BYTES = BM * BK * 2;  // 16 KiB per operand per stage
+constexpr long long WAIT_CYCLES = 4000000000LL;  // about two seconds
+
+struct GramCtl {
+  uint64_t full[STAGES];
+  uint64_t empty[STAGES];
+  uint64_t done;
+  uint32_t tmem;
+  volatile int abort;
+};
+
+constexpr size_t GRAM_SMEM = 1024 + 2 * STAGES * TILE_BYTES + sizeof(GramCtl);
+}  // namespace
+
+__global__ void __launch_bounds__(128, 1)
+    k_gram_tc(const __grid_constant__ CUtensorMap tmap, const int32_t* toff, int B, int N,
+              int Tmax, int D, const float* __restrict__ rn, float* cos, uint32_t* status) {
+  extern __shared__ uint8_t sm_raw[];
+  uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* tilesA = base;
+  uint8_t* tilesB = base + STAGES * TILE_BYTES;
+  GramCtl* ctl = reinterpret_cast<GramCtl*>(base + 2 * STAGES * TILE_BYTES);
+
+  const int b = blockIdx.y;
+  const TextGeom tg = text_geom(toff, b, B, Tmax, status);
+  if (tg.T == 0) return;
+  const int nt = ceil_div(N, BM);
+  int t = blockIdx.x, I = 0;
+  while (t >= nt - I) {
+    t -= nt - I;
+    ++I;
+  }
+  const int J = I + t;
+  const int r0 = min(I * BM, N - BM), c0 = min(J * BM, N - BM);
+  const int row_base = (int)((size_t)b * N + tg.off);  // first visual row of the image
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nk = ceil_div(D, BK);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      tc::mbar_init(&ctl->full[s], 1);
+      tc::mbar_init(&ctl->empty[s], 1);
+    }
+    tc::mbar_init(&ctl->done, 1);
+    ctl->abort = 0;
+    tc::fence_mbar_init();
+    tc::prefetch_tmap(&tmap);
+  }
+  if (warp == 0) {
+    tc::tmem_alloc(&ctl->tmem, 128);
+    tc::tmem_relinquish();
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = ctl->tmem;
+  const long long deadline = clock64() + WAIT_CYCLES;
+  int issued = 0;  // producer: stages loaded
+
+  if (warp == 0) {
+    if (lane == 0) {
+      for (int kb = 0; kb < nk; ++kb) {
+        const int s = kb % STAGES;
+        const uint32_t ph = (uint32_t)(kb / STAGES) & 1u;
+        if (kb >= STAGES && !tc::mbar_wait(&ctl->empty[s], ph ^ 1u, deadline)) {
+          ctl->abort = 1;
+          break;
+        }
+        if (ctl->abort) break;
+        tc::mbar_arrive_expect_tx(&ctl->full[s], 2 * TILE_BYTES);
+        tc::tma_load_2d(tilesA + s * TILE_BYTES, &tmap, kb * BK, row_base + r0, &ctl->full[s]);
+        tc::tma_load_2d(tilesB + s * TILE_BYTES, &tmap, kb * BK, row_base + c0, &ctl->full[s]);
+        ++issued;
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc = tc::idesc_bf16_f32(BM, BM);
+      for (int kb = 0; kb < nk; ++kb) {
+        const int s = kb % STAGES;
+        const uint32_t ph = (uint32_t)(kb / STAGES) & 1u;
+        if (!tc::mbar_wait(&ctl->full[s], ph, deadline)) {
+          ctl->abort = 1;
+          break;
+        }
+        tc::fence_after_sync();
+        const uint64_t ad = tc::desc_sw128_kmajor(tilesA + s * TILE_BYTES);
+        const uint64_t bd = tc::desc_sw128_kmajor(tilesB + s * TILE_BYTES);
+#pragma unroll
+        for (int kk = 0; kk < BK / 16; ++kk)
+          tc::mma_bf16(tmem, ad + 2 * kk, bd + 2 * kk, idesc, (kb | kk) != 0);
+        tc::mma_commit(&ctl->empty[s]);
+      }
+      tc::mma_commit(&ctl->done);  // also on abort, so the epilogue wakes up
+    }
+    __syncwarp();
+  }
+
+  bool ok = tc::mbar_wait(&ctl->done, 0, deadline);
+  ok = __all_sync(FULL, ok && !ctl->abort);
+  tc::fence_after_sync();
+  if (ok) {
+    const int i = r0 + warp * 32 + lane;  // this thread's TMEM lane = output row
+    const bool own_row = i >= I * BM;
+    const float ri = rn[(size_t)b * N + i];
+    float* crow = cos + ((size_t)b * N + i) * N;
+#pragma unroll 1
+    for (int cc = 0; cc < BM / 32; ++cc) {
+      float v[32];
+      tc::tmem_ld32(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(cc * 32), v);
+      const int j0 = c0 + cc * 32;
+#pragma unroll
+      for (int q = 0; q < 32; ++q) {
+        const int j = j0 + q;
+        v[q] = v[q] * ri * rn[(size_t)b * N + j];
+      }
+      if (own_row) {
+        if (j0 >= J * BM) {
+#pragma unroll
+          for (int q = 0; q < 32; q += 4)
+            *reinterpret_cast<float4*>(crow + j0 + q) = make_float4(v[q], v[q + 1], v[q + 2], v[q + 3]);
+        } else {
+          for (int q = 0; q < 32; ++q)
+            if (j0 + q >= J * BM) crow[j0 + q] = v[q];
+        }
+      }
+      if (I != J) {  // mirror: row j of the transposed block, coalesced over the warp's lanes
+#pragma unroll
+        for (int q = 0; q < 32; ++q) {
+          const int j = j0 + q;
+          if (own_row && j >= J * BM) cos[((size_t)b * N + j) * N + i] = v[q];
+        }
+      }
+    }
+  }
+  if (!ok && threadIdx.x == 0) set_status(status, GMC_STATUS_TIMEOUT);
+  if (warp == 0 && lane == 0 && !ok) {
+    // drain TMA copies still in flight into this CTA's shared memory
+    const long long d2 = clock64() + WAIT_CYCLES;
+    for (int kb = (issued > STAGES ? issued - STAGES : 0); kb < issued; ++kb)
+      if (!tc::mbar_wait(&ctl->full[kb % STAGES], (uint32_t)(kb / STAGES) & 1u, d2)) break;
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  if (warp == 0) tc::tmem_dealloc(tmem, 128);
+}
+
+// ---------------------------------------------------------------------------
+// host side
+// ---------------------------------------------------------------------------
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+static EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+// 2-D bf16 tensor map: rows of `row_elems` elements, `rows` rows, row pitch
+// `pitch_elems`; box = 64 elements x `box_rows` rows, 128-byte swizzle.
+cudaError_t make_tmap_bf16(CUtensorMap* map, const void* base, uint64_t row_elems, uint64_t rows,
+                           uint64_t pitch_elems, uint32_t box_rows) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return cudaErrorNotSupported;
+  const cuuint64_t dims[2] = {row_elems, rows};
+  const cuuint64_t strides[1] = {pitch_elems * 2};
+  const cuuint32_t box[2] = {64, box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
+                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+bool gram_tc_supported(const Dims& dm) {
+  return dm.dtype == GMC_BF16 && dm.N >= BM && dm.D >= BK;
+}
+
+cudaError_t launch_gram_tc(const Dims& dm, const void* hidden, Scratch& s, cudaStream_t st) {
+  CUtensorMap map;
+  // Rows of every image are addressed from the buffer start; the declared row
+  // count is an upper bound (B * (N + T)), every box read lies inside the
+  // image's visual rows.
+  cudaError_t e = make_tmap_bf16(&map, hidden, (uint64_t)dm.D,
+                                 (uint64_t)dm.B * (uint64_t)(dm.N + dm.T), (uint64_t)dm.D, BM);
+  if (e != cudaSuccess) return e;
+  if ((e = set_smem_limit((const void*)k_gram_tc, GRAM_SMEM)) != cudaSuccess) return e;
+  const int nt = ceil_div(dm.N, BM);
+  dim3 grid(nt * (nt + 1) / 2, dm.B);
+  k_gram_tc<<<grid, 128, GRAM_SMEM, st>>>(map, dm.toff, dm.B, dm.N, dm.T, dm.D, s.rn, s.cos,
+                                          s.status);
+  return cudaGetLastError();
+}
+
+}  // namespace gmc

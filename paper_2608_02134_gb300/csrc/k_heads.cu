@@ -100,10 +100,22 @@ __global__ void k_head_stats(const float* __restrict__ A, const float* __restric
   }
 }
 
-// One block per image: reduce the Gram, farthest-first clustering, omega_h.
+// One block per image: reduce the Gram, then one warp runs farthest-first
+// clustering and the head weights (two heads per lane, H <= 64).
 // Ties: the first centre is the lowest-index largest pattern, each next centre
 // the lowest-index head of smallest max-cosine, and a head joins the earliest
 // centre among equally similar ones.
+__device__ __forceinline__ void warp_argbest(double& v, int& idx, bool want_max) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const double ov = __shfl_xor_sync(FULL, v, o);
+    const int oi = __shfl_xor_sync(FULL, idx, o);
+    const bool better = want_max ? (ov > v || (ov == v && oi < idx))
+                                 : (ov < v || (ov == v && oi < idx));
+    if (oi >= 0 && (idx < 0 || better)) { v = ov; idx = oi; }
+  }
+}
+
 __global__ void k_head_cluster(const double* __restrict__ hgpart, int nHG,
                                const float* __restrict__ rs, const int32_t* toff, int B, int N,
                                int Tmax, int H, int max_clusters, float head_eps, float* omega,
@@ -133,72 +145,96 @@ __global__ void k_head_cluster(const double* __restrict__ hgpart, int nHG,
     cs[p] = (a > 0.0 && c > 0.0) ? HG[p] / sqrt(a * c) : 0.0;
   }
   __syncthreads();
-  if (threadIdx.x != 0) return;
-  int centres[GMC_MAX_HEADS];
-  int assign[GMC_MAX_HEADS];
-  bool is_c[GMC_MAX_HEADS];
+  if (threadIdx.x >= 32) return;
+  const int lane = threadIdx.x;
+  const int h0 = lane, h1 = lane + 32;  // this lane's heads (if < H)
   const int nc = min(max_clusters, H);
-  int first = 0;
-  for (int h = 1; h < H; ++h)
-    if (pre[h] > pre[first]) first = h;
-  for (int h = 0; h < H; ++h) is_c[h] = false;
-  centres[0] = first;
-  is_c[first] = true;
+  int centres[GMC_MAX_HEADS];
+  bool c0 = false, c1 = false;  // is h0 / h1 a centre
+  {
+    double v = -1.0;
+    int idx = -1;
+    if (h0 < H) { v = pre[h0]; idx = h0; }
+    if (h1 < H && (idx < 0 || pre[h1] > v)) { v = pre[h1]; idx = h1; }
+    warp_argbest(v, idx, true);
+    centres[0] = idx;
+  }
+  c0 = (h0 == centres[0]);
+  c1 = (h1 == centres[0]);
   for (int c = 1; c < nc; ++c) {
-    int best = -1;
-    double bv = 0.0;
-    for (int h = 0; h < H; ++h) {
-      if (is_c[h]) continue;
+    double v = 0.0;
+    int idx = -1;
+    for (int q = 0; q < 2; ++q) {
+      const int h = q ? h1 : h0;
+      if (h >= H || (q ? c1 : c0)) continue;
       double mc = -INFINITY;
       for (int k = 0; k < c; ++k) mc = fmax(mc, cs[h * H + centres[k]]);
-      if (best < 0 || mc < bv) { best = h; bv = mc; }
+      if (idx < 0 || mc < v) { v = mc; idx = h; }
     }
-    centres[c] = best;
-    is_c[best] = true;
+    warp_argbest(v, idx, false);
+    centres[c] = idx;
+    c0 |= (h0 == idx);
+    c1 |= (h1 == idx);
   }
-  int count[GMC_MAX_HEADS];
-  for (int k = 0; k < nc; ++k) count[k] = 0;
-  for (int h = 0; h < H; ++h) {
+  int as0 = 0, as1 = 0;
+  for (int q = 0; q < 2; ++q) {
+    const int h = q ? h1 : h0;
+    if (h >= H) continue;
     int bk = 0;
     for (int k = 1; k < nc; ++k)
       if (cs[h * H + centres[k]] > cs[h * H + centres[bk]]) bk = k;
-    assign[h] = bk;
-    count[bk]++;
+    if (q) as1 = bk; else as0 = bk;
   }
+  // every lane needs every head's cluster: gather through shuffles
+  auto cluster_of = [&](int g) {
+    const int src = g & 31;
+    const int a0 = __shfl_sync(FULL, as0, src), a1 = __shfl_sync(FULL, as1, src);
+    return g < 32 ? a0 : a1;
+  };
+  int asg[GMC_MAX_HEADS];
+  for (int g = 0; g < H; ++g) asg[g] = cluster_of(g);
   int C = 0;
-  for (int k = 0; k < nc; ++k) C += count[k] > 0;
+  double inv0 = 0.0, inv1 = 0.0;
+  double invsum[GMC_MAX_HEADS];
   for (int k = 0; k < nc; ++k) {
-    if (count[k] == 0) continue;
-    double nrm2 = 0.0;  // ||sum_{g in c} u_g||^2
-    for (int g = 0; g < H; ++g)
-      if (assign[g] == k)
-        for (int g2 = 0; g2 < H; ++g2)
-          if (assign[g2] == k) nrm2 += cs[g * H + g2];
+    int cnt = 0;
+    for (int g = 0; g < H; ++g) cnt += asg[g] == k;
+    if (cnt == 0) { invsum[k] = 0.0; continue; }
+    ++C;
+    // ||sum_{g in k} u_g||^2 = sum over pairs in the cluster, rows split over lanes
+    double part = 0.0;
+    for (int q = 0; q < 2; ++q) {
+      const int g = q ? h1 : h0;
+      if (g >= H || asg[g] != k) continue;
+      for (int g2 = 0; g2 < H; ++g2)
+        if (asg[g2] == k) part += cs[g * H + g2];
+    }
+    const double nrm2 = warp_sum(part);
     const double nrm = nrm2 > 0.0 ? sqrt(nrm2) : 0.0;
-    double invsum = 0.0;
-    for (int h = 0; h < H; ++h) {
-      if (assign[h] != k) continue;
+    double mine = 0.0;
+    for (int q = 0; q < 2; ++q) {
+      const int h = q ? h1 : h0;
+      if (h >= H || asg[h] != k) continue;
       double dot = 0.0;
       for (int g = 0; g < H; ++g)
-        if (assign[g] == k) dot += cs[h * H + g];
+        if (asg[g] == k) dot += cs[h * H + g];
       const double dh = 1.0 - (nrm > 0.0 ? dot / nrm : 0.0);
-      pre[h] = 1.0 / (dh + head_eps);  // reuse: inverse-dispersion weight
-      invsum += pre[h];
+      const double inv = 1.0 / (dh + head_eps);
+      if (q) inv1 = inv; else inv0 = inv;
+      mine += inv;
     }
-    for (int h = 0; h < H; ++h)
-      if (assign[h] == k) omega[(size_t)b * H + h] = (float)(pre[h] / invsum / C);
+    invsum[k] = warp_sum(mine);
   }
+  if (h0 < H) omega[(size_t)b * H + h0] = (float)(inv0 / invsum[as0] / C);
+  if (h1 < H) omega[(size_t)b * H + h1] = (float)(inv1 / invsum[as1] / C);
   if (tv.base) {
-    gmc_trace_header* hd = tv.header(b);
-    hd->n_clusters = C;
+    if (lane == 0) tv.header(b)->n_clusters = C;
     int32_t* tc = tv.at<int32_t>(b, tv.off_centres);
-    for (int k = 0; k < max_clusters; ++k) tc[k] = k < nc ? centres[k] : -1;
+    for (int k = lane; k < max_clusters; k += 32) tc[k] = k < nc ? centres[k] : -1;
     int32_t* ta = tv.at<int32_t>(b, tv.off_head_assign);
     float* to = tv.at<float>(b, tv.off_omega);
-    for (int h = 0; h < H; ++h) {
-      ta[h] = assign[h];
-      to[h] = omega[(size_t)b * H + h];
-    }
+    if (h0 < H) { ta[h0] = as0; to[h0] = (float)(inv0 / invsum[as0] / C); }
+    if (h1 < H) { ta[h1] = as1; to[h1] = (float)(inv1 / invsum[as1] / C); }
   }
 }
 

@@ -127,4 +127,6 @@ cudaError_t set_smem_limit(const void* func, size_t bytes);
 
 namespace gmc {
 cudaError_t launch_gram_simt(const Dims&, const void* hidden, Scratch&, cudaStream_t);
+cudaError_t launch_gram_tc(const Dims&, const void* hidden, Scratch&, cudaStream_t);
+bool gram_tc_supported(const Dims&);
 }  // namespace gmc

@@ -26,7 +26,7 @@ EXPORTS = (
     "gmc_trace_size", "gmc_select_workspace_size", "gmc_select",
     "gmc_transport_workspace_size", "gmc_transport", "gmc_read_status", "gmc_error_string",
     "gmc_version", "gmc_profile_enable", "gmc_profile_read", "gmc_launch_count",
-    "gmc_transport_noalloc",
+    "gmc_transport_noalloc", "gmc_cosine_workspace_size", "gmc_cosine",
 )
 
 
@@ -115,6 +115,10 @@ def lib() -> ctypes.CDLL:
     L.gmc_transport_noalloc.argtypes = [PP, P, vp, vp, vp, vp, vp, vp, i, i, i, i, i, vp, vp, vp,
                                         vp, vp, vp]
     L.gmc_transport_noalloc.restype = i
+    L.gmc_cosine_workspace_size.argtypes = [PP, i]
+    L.gmc_cosine_workspace_size.restype = sz
+    L.gmc_cosine.argtypes = [PP, P, vp, i, i, i, vp, vp, sz, vp]
+    L.gmc_cosine.restype = i
     _lib = L
     return L
 
@@ -203,6 +207,16 @@ def transport_noalloc(prob: Problem, params: Params, hidden, keys, pos_ids, supp
         ctypes.byref(prob), ctypes.byref(params), _ptr(hidden), _ptr(keys), _ptr(pos_ids),
         _ptr(support), _ptr(assign), _ptr(weights), N, T, d, D, K, _ptr(out_idx),
         _ptr(out_hidden), _ptr(out_kv), _ptr(out_pos), _ptr(device_status), _stream(stream)))
+
+
+def cosine(prob: Problem, params: Params, hidden, N, T, D, out_cos, workspace=None, stream=None):
+    """gmc_cosine: cos [B][N][N] of the visual states (the Gram stage alone)."""
+    if workspace is None:
+        workspace = alloc_workspace(int(lib().gmc_cosine_workspace_size(ctypes.byref(prob), N)),
+                                    out_cos.device)
+    _check(lib().gmc_cosine(ctypes.byref(prob), ctypes.byref(params), _ptr(hidden), N, T, D,
+                            _ptr(out_cos), _ptr(workspace), workspace.numel(), _stream(stream)))
+    return workspace
 
 
 def transport_workspace_size(prob: Problem, N, T, K) -> int:
