@@ -118,6 +118,7 @@ size_t carve_compress(const Dims& dm, Scratch* s, char* base) {
   t.mass = c.take<float>(B * N);
   t.selpart = nullptr;
   t.fexp = nullptr;
+  t.Qp = c.take<__nv_bfloat16>(B * dm.Hkv * (size_t)message_rq(dm) * dm.d);
   if (s) *s = t;
   return c.off;
 }
@@ -334,7 +335,7 @@ int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* 
   GMC_TRY(g_prof.begin(st));
   GMC_STAGE("rownorm", 1, launch_rownorm(dm, hidden, p.norm_eps, s, st));
   GMC_STAGE("probe", 2, launch_probe(dm, keys, vo_probe, p, s, st));
-  GMC_STAGE("message", 1, launch_message(dm, keys, queries, s, st));
+  GMC_STAGE("message", message_tc_supported(dm) ? 2 : 1, launch_message(dm, keys, queries, s, st));
   GMC_STAGE("heads", 3, launch_heads(dm, p, s, tv, st));
   GMC_STAGE("gram", 1, launch_gram(dm, hidden, s, st));
   GMC_STAGE("clients", 1, launch_build_clients(dm, p, fx, s, st));

@@ -1,0 +1,315 @@
+// Native boundary attention slice on the tcgen05 tensor cores (bf16 path).
+//
+// For image b and key/value head g, the rows of the A operand are the text
+// queries of the query heads of group g, packed as (j, t) -> j*T_b + t, and the
+// B operand runs over the image's keys (N visual rows, then T_b text rows).
+// The CTA owns 128 query rows and walks every 128-key tile twice:
+//   pass 0: online softmax statistics (max, sum of exp) per query row over the
+//           keys it may see (all visual keys and text keys 0..t, scale 1/sqrt(d));
+//   pass 1: A[h,t,i] = exp(s_i - max) / sum for the visual keys i < N, and
+//           rs[h,t] = sum_i A[h,t,i] g_h(i) with g_h(i) = sqrt(||Z_h[i]||^2 + sigma_h^2).
+// Recomputing the logits costs one more small MMA pass and avoids writing and
+// re-reading raw scores.  This is appendix Eq. (cond-native-message): the
+// visual slice of the native causal softmax, not renormalised over the image.
+//
+// Roles: warp 8 / lane 0 loads the query tile once and streams key tiles with
+// TMA through a 4-stage ring; warp 9 / lane 0 issues tcgen05.mma into two
+// 128-column TMEM accumulators (double buffered); warps 0..7 read the
+// accumulators (warp w: TMEM lanes 32*(w%4).., columns 64*(w/4)..) and do the
+// softmax arithmetic.  Every wait is clock-bounded.
+#include "common.cuh"
+#include "kernels.cuh"
+#include "tc.cuh"
+
+namespace gmc {
+
+cudaError_t make_tmap_bf16(CUtensorMap* map, const void* base, uint64_t row_elems, uint64_t rows,
+                           uint64_t pitch_elems, uint32_t box_rows);
+
+namespace {
+constexpr int BM = 128, BK = 64, STAGES = 4;
+constexpr int TILE_BYTES = BM * BK * 2;
+constexpr int EPI_WARPS = 8, THREADS = 32 * (EPI_WARPS + 2);
+constexpr long long WAIT_CYCLES = 4000000000LL;
+
+struct MsgCtl {
+  uint64_t qfull;
+  uint64_t full[STAGES];
+  uint64_t empty[STAGES];
+  uint64_t accf[2];
+  uint64_t acce[2];
+  uint32_t tmem;
+  volatile int abort;
+  float stat_m[2][BM];
+  float stat_l[2][BM];
+  float rsum[2][BM];
+};
+
+size_t msg_smem_bytes(int nkb) {
+  return 1024 + (size_t)nkb * TILE_BYTES * (1 + STAGES) + sizeof(MsgCtl);
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(tc::smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ void epi_barrier() {
+  asm volatile("bar.sync 1, %0;" ::"n"(EPI_WARPS * 32) : "memory");
+}
+}  // namespace
+
+// Q [T_b rows][H][d] of every image -> Qp [B][Hkv][RQ][d], row j*T_b + t of
+// group g holding query head g*grp + j; rows >= grp*T_b are zero.
+__global__ void k_pack_q(const __nv_bfloat16* __restrict__ queries, const int32_t* toff, int B,
+                         int Tmax, int H, int Hkv, int d, int RQ, __nv_bfloat16* Qp,
+                         uint32_t* status) {
+  const int b = blockIdx.z, g = blockIdx.y;
+  const TextGeom tg = text_geom(toff, b, B, Tmax, status);
+  const int grp = H / Hkv;
+  const int lane = threadIdx.x & 31;
+  const int row = blockIdx.x * 8 + (threadIdx.x >> 5);
+  if (row >= RQ) return;
+  uint4* dst = reinterpret_cast<uint4*>(Qp + (((size_t)b * Hkv + g) * RQ + row) * d);
+  const int nv = d / 8;
+  if (tg.T > 0 && row < grp * tg.T) {
+    const int j = row / tg.T, t = row % tg.T;
+    const uint4* src = reinterpret_cast<const uint4*>(
+        queries + ((size_t)tg.off + t) * H * d + (size_t)(g * grp + j) * d);
+    for (int q = lane; q < nv; q += 32) dst[q] = src[q];
+  } else {
+    for (int q = lane; q < nv; q += 32) dst[q] = make_uint4(0, 0, 0, 0);
+  }
+}
+
+__global__ void __launch_bounds__(THREADS, 1)
+    k_message_tc(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
+                 const int32_t* toff, int B, int N, int Tmax, int H, int Hkv, int d, int RQ,
+                 const float* __restrict__ zn2, const float* __restrict__ sigma, float* A,
+                 float* rs, uint32_t* status) {
+  extern __shared__ uint8_t sm_raw[];
+  uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  const int nkb = d / BK;
+  uint8_t* Qs = base;
+  uint8_t* Ks = base + (size_t)nkb * TILE_BYTES;
+  MsgCtl* ctl = reinterpret_cast<MsgCtl*>(base + (size_t)nkb * TILE_BYTES * (1 + STAGES));
+
+  const int b = blockIdx.z, g = blockIdx.y, tile = blockIdx.x;
+  const TextGeom tg = text_geom(toff, b, B, Tmax, status);
+  const int grp = H / Hkv;
+  if (tg.T == 0 || tile * BM >= grp * tg.T) return;  // uniform per CTA
+  const int Tb = tg.T;
+  const int nkeys = N + Tb;
+  const int nkt = ceil_div(nkeys, BM);
+  const int iters = 2 * nkt;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int qrow0 = (int)(((size_t)b * Hkv + g) * RQ + (size_t)tile * BM);
+  const int krow0 = (int)(2 * ((size_t)b * N + tg.off));
+
+  if (threadIdx.x == 0) {
+    tc::mbar_init(&ctl->qfull, 1);
+    for (int s = 0; s < STAGES; ++s) {
+      tc::mbar_init(&ctl->full[s], 1);
+      tc::mbar_init(&ctl->empty[s], 1);
+    }
+    for (int q = 0; q < 2; ++q) {
+      tc::mbar_init(&ctl->accf[q], 1);
+      tc::mbar_init(&ctl->acce[q], EPI_WARPS);
+    }
+    ctl->abort = 0;
+    tc::fence_mbar_init();
+    tc::prefetch_tmap(&qmap);
+    tc::prefetch_tmap(&kmap);
+  }
+  if (warp == 0) {
+    tc::tmem_alloc(&ctl->tmem, 256);
+    tc::tmem_relinquish();
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = ctl->tmem;
+  const long long deadline = clock64() + WAIT_CYCLES;
+
+  if (warp == EPI_WARPS) {  // ---------------- TMA producer
+    int issued = 0;
+    if (lane == 0) {
+      tc::mbar_arrive_expect_tx(&ctl->qfull, nkb * TILE_BYTES);
+      for (int kb = 0; kb < nkb; ++kb)
+        tc::tma_load_2d(Qs + kb * TILE_BYTES, &qmap, kb * BK, qrow0, &ctl->qfull);
+      for (int it = 0; it < iters; ++it) {
+        const int s = it % STAGES, c = it % nkt;
+        const uint32_t ph = (uint32_t)(it / STAGES) & 1u;
+        if (it >= STAGES && !tc::mbar_wait(&ctl->empty[s], ph ^ 1u, deadline)) {
+          ctl->abort = 1;
+          break;
+        }
+        if (ctl->abort) break;
+        tc::mbar_arrive_expect_tx(&ctl->full[s], nkb * TILE_BYTES);
+        for (int kb = 0; kb < nkb; ++kb)
+          tc::tma_load_2d(Ks + ((size_t)s * nkb + kb) * TILE_BYTES, &kmap, g * d + kb * BK,
+                          krow0 + c * BM, &ctl->full[s]);
+        ++issued;
+      }
+      if (ctl->abort) {  // drain copies still landing in this CTA's shared memory
+        const long long d2 = clock64() + WAIT_CYCLES;
+        tc::mbar_wait(&ctl->qfull, 0, d2);
+        for (int it = (issued > STAGES ? issued - STAGES : 0); it < issued; ++it)
+          if (!tc::mbar_wait(&ctl->full[it % STAGES], (uint32_t)(it / STAGES) & 1u, d2)) break;
+      }
+    }
+    __syncwarp();
+  } else if (warp == EPI_WARPS + 1) {  // ---------------- MMA issuer
+    if (lane == 0) {
+      const uint32_t idesc = tc::idesc_bf16_f32(BM, BM);
+      bool ok = tc::mbar_wait(&ctl->qfull, 0, deadline);
+      for (int it = 0; ok && it < iters; ++it) {
+        const int s = it % STAGES, buf = it & 1;
+        if (!tc::mbar_wait(&ctl->full[s], (uint32_t)(it / STAGES) & 1u, deadline) ||
+            (it >= 2 && !tc::mbar_wait(&ctl->acce[buf], (uint32_t)((it >> 1) - 1) & 1u, deadline))) {
+          ok = false;
+          break;
+        }
+        tc::fence_after_sync();
+        const uint32_t dst = tmem + (uint32_t)(buf * BM);
+        for (int kb = 0; kb < nkb; ++kb) {
+          const uint64_t ad = tc::desc_sw128_kmajor(Qs + kb * TILE_BYTES);
+          const uint64_t bd = tc::desc_sw128_kmajor(Ks + ((size_t)s * nkb + kb) * TILE_BYTES);
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk)
+            tc::mma_bf16(dst, ad + 2 * kk, bd + 2 * kk, idesc, (kb | kk) != 0);
+        }
+        tc::mma_commit(&ctl->empty[s]);
+        tc::mma_commit(&ctl->accf[buf]);
+      }
+      if (!ok) ctl->abort = 1;
+    }
+    __syncwarp();
+  } else {  // ---------------- epilogue warps 0..7
+    const int quarter = warp & 3, half = warp >> 2;
+    const int r = quarter * 32 + lane;           // tile row == TMEM lane
+    const int R = tile * BM + r;                 // packed row
+    const bool valid = R < grp * Tb;
+    const int j = valid ? R / Tb : 0, t = valid ? R % Tb : 0;
+    const int h = g * grp + j;
+    const float scale = rsqrtf((float)d);
+    const float sg = sigma[(size_t)b * H + h];
+    const float sg2 = sg * sg;
+    const float* zr = zn2 + ((size_t)b * H + h) * N;
+    float* arow = A + (((size_t)b * H + h) * Tmax + t) * N;
+    const int kvis = N + t + 1;                  // keys this query may see
+    float m = -INFINITY, l = 0.f, rsum = 0.f, M = 0.f, invL = 0.f;
+    for (int it = 0; it < iters; ++it) {
+      const int buf = it & 1, c = it % nkt;
+      bool ok = tc::mbar_wait(&ctl->accf[buf], (uint32_t)(it >> 1) & 1u, deadline);
+      ok = __all_sync(FULL, ok && !ctl->abort);
+      float v[64];
+      if (ok) {
+        tc::fence_after_sync();
+        const uint32_t ta = tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(buf * BM + half * 64);
+        tc::tmem_ld32(ta, v);
+        tc::tmem_ld32(ta + 32, v + 32);
+      }
+      tc::fence_before_sync();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ctl->acce[buf]);
+      if (!ok) {
+        if (it == nkt - 1) epi_barrier();
+        continue;
+      }
+      const int k0 = c * BM + half * 64;
+      if (it < nkt) {  // pass 0: running max / sum over the visible keys
+        float mt = -INFINITY;
+#pragma unroll
+        for (int q = 0; q < 64; ++q) {
+          v[q] *= scale;
+          if (k0 + q < kvis) mt = fmaxf(mt, v[q]);
+        }
+        if (mt > -INFINITY) {
+          const float mn = fmaxf(m, mt);
+          float acc = l * expf(m - mn);
+#pragma unroll
+          for (int q = 0; q < 64; ++q)
+            if (k0 + q < kvis) acc += expf(v[q] - mn);
+          l = acc;
+          m = mn;
+        }
+        if (it == nkt - 1) {  // combine the two column halves of every row
+          ctl->stat_m[half][r] = m;
+          ctl->stat_l[half][r] = l;
+          epi_barrier();
+          const float mo = ctl->stat_m[half ^ 1][r], lo = ctl->stat_l[half ^ 1][r];
+          M = fmaxf(m, mo);
+          const float L = (m > -INFINITY ? l * expf(m - M) : 0.f) +
+                          (mo > -INFINITY ? lo * expf(mo - M) : 0.f);
+          invL = 1.f / L;
+        }
+      } else if (valid && k0 < N) {  // pass 1: normalised visual columns
+        const int nv = min(64, N - k0);
+        if (nv == 64 && (N & 3) == 0) {
+#pragma unroll
+          for (int q = 0; q < 64; q += 4) {
+            const float4 z = *reinterpret_cast<const float4*>(zr + k0 + q);
+            float4 o;
+            o.x = expf(v[q] * scale - M) * invL;
+            o.y = expf(v[q + 1] * scale - M) * invL;
+            o.z = expf(v[q + 2] * scale - M) * invL;
+            o.w = expf(v[q + 3] * scale - M) * invL;
+            *reinterpret_cast<float4*>(arow + k0 + q) = o;
+            rsum = fmaf(o.x, sqrtf(z.x + sg2), rsum);
+            rsum = fmaf(o.y, sqrtf(z.y + sg2), rsum);
+            rsum = fmaf(o.z, sqrtf(z.z + sg2), rsum);
+            rsum = fmaf(o.w, sqrtf(z.w + sg2), rsum);
+          }
+        } else {
+          for (int q = 0; q < nv; ++q) {
+            const float p = expf(v[q] * scale - M) * invL;
+            arow[k0 + q] = p;
+            rsum = fmaf(p, sqrtf(zr[k0 + q] + sg2), rsum);
+          }
+        }
+      }
+    }
+    ctl->rsum[half][r] = rsum;
+    epi_barrier();
+    if (half == 0 && valid && !ctl->abort)
+      rs[((size_t)b * H + h) * Tmax + t] = rsum + ctl->rsum[1][r];
+  }
+  if (threadIdx.x == 0 && ctl->abort) set_status(status, GMC_STATUS_TIMEOUT);
+  tc::fence_before_sync();
+  __syncthreads();
+  if (warp == 0) tc::tmem_dealloc(tmem, 256);
+}
+
+bool message_tc_supported(const Dims& dm) {
+  return dm.dtype == GMC_BF16 && dm.N >= BM && (dm.d == 64 || dm.d == 128);
+}
+
+int message_rq(const Dims& dm) { return ceil_div((dm.H / dm.Hkv) * dm.T, BM) * BM; }
+
+cudaError_t launch_message_tc(const Dims& dm, const void* keys, const void* queries, Scratch& s,
+                              cudaStream_t st) {
+  const int RQ = message_rq(dm);
+  k_pack_q<<<dim3(ceil_div(RQ, 8), dm.Hkv, dm.B), 256, 0, st>>>(
+      (const __nv_bfloat16*)queries, dm.toff, dm.B, dm.T, dm.H, dm.Hkv, dm.d, RQ, s.Qp, s.status);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  CUtensorMap qmap, kmap;
+  if ((e = make_tmap_bf16(&qmap, s.Qp, dm.d, (uint64_t)dm.B * dm.Hkv * RQ, dm.d, BM)) != cudaSuccess)
+    return e;
+  // keys of every image, addressed from the buffer start; the declared row
+  // count is an upper bound, every box read lies inside the image's K block or
+  // the V block that follows it.
+  if ((e = make_tmap_bf16(&kmap, keys, (uint64_t)dm.Hkv * dm.d,
+                          2ull * dm.B * (uint64_t)(dm.N + dm.T), (uint64_t)dm.Hkv * dm.d, BM)) !=
+      cudaSuccess)
+    return e;
+  const int nkb = dm.d / BK;
+  const size_t smem = msg_smem_bytes(nkb);
+  if ((e = set_smem_limit((const void*)k_message_tc, smem)) != cudaSuccess) return e;
+  dim3 grid(RQ / BM, dm.Hkv, dm.B);
+  k_message_tc<<<grid, THREADS, smem, st>>>(qmap, kmap, dm.toff, dm.B, dm.N, dm.T, dm.H, dm.Hkv,
+                                            dm.d, RQ, s.zn2, s.sigma, s.A, s.rs, s.status);
+  return cudaGetLastError();
+}
+
+}  // namespace gmc

@@ -2,6 +2,7 @@
 // translation units.  Nothing here is exported from libgmc.so.
 #pragma once
 
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stddef.h>
 #include <stdint.h>
@@ -61,6 +62,7 @@ struct Scratch {
   float* mass;       // [B][N]
   double* selpart;   // [B][64]        select-path total mass partials
   int32_t* fexp;     // [B]            select-path fixed-point exponents
+  __nv_bfloat16* Qp; // [B][Hkv][RQ][d] packed text queries of each KV group (tcgen05 path)
   int nP, nHG, nA, nSel;
 };
 
@@ -129,4 +131,8 @@ namespace gmc {
 cudaError_t launch_gram_simt(const Dims&, const void* hidden, Scratch&, cudaStream_t);
 cudaError_t launch_gram_tc(const Dims&, const void* hidden, Scratch&, cudaStream_t);
 bool gram_tc_supported(const Dims&);
+cudaError_t launch_message_tc(const Dims&, const void* keys, const void* queries, Scratch&,
+                              cudaStream_t);
+bool message_tc_supported(const Dims&);
+int message_rq(const Dims&);  // packed query rows per (image, KV group)
 }  // namespace gmc
