@@ -83,8 +83,10 @@ Dims make_dims(const gmc_problem* prob, const gmc_params& p, int N, int T, int H
   return dm;
 }
 
+R0State carve_round0(Carver& c, size_t B, size_t N, size_t M);
+
 // Workspace of gmc_compress.  base == nullptr only measures.
-size_t carve_compress(const Dims& dm, Scratch* s, char* base) {
+size_t carve_compress(const Dims& dm, Scratch* s, char* base, R0State* r0s = nullptr) {
   Carver c{base};
   Scratch t{};
   const size_t B = dm.B, N = dm.N, H = dm.H, T = dm.T, M = dm.M, K = dm.K;
@@ -100,6 +102,7 @@ size_t carve_compress(const Dims& dm, Scratch* s, char* base) {
   t.sigpart = c.take<float>(B * t.nP * H);
   t.sigma = c.take<float>(B * H);
   t.hgpart = c.take<double>(B * t.nHG * H * H);
+  t.HG = c.take<double>(B * H * H);
   t.W2 = c.take<float>(B * H * N);
   t.omega = c.take<float>(B * H);
   t.ebar = c.take<float>(B * N);
@@ -120,7 +123,21 @@ size_t carve_compress(const Dims& dm, Scratch* s, char* base) {
   t.fexp = nullptr;
   t.Qp = c.take<__nv_bfloat16>(B * dm.Hkv * (size_t)message_rq(dm) * dm.d);
   if (s) *s = t;
+  R0State r0 = carve_round0(c, B, N, M);
+  if (r0s && base) *r0s = r0;
   return c.off;
+}
+
+R0State carve_round0(Carver& c, size_t B, size_t N, size_t M) {
+  R0State r;
+  r.pool = c.take<int32_t>(B * GMC_MAX_POOL);
+  r.info = c.take<int32_t>(B * 4);
+  r.s0 = c.take<long long>(B * GMC_MAX_POOL);
+  r.u1 = c.take<long long>(B * N);
+  r.bcov = c.take<float>(B * M);
+  r.cnt = c.take<int32_t>(B * M);
+  r.fv = c.take<long long>(B * 4);
+  return r;
 }
 
 int fixed_point_exponent(double total) {
@@ -312,7 +329,8 @@ int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* 
   const int Ke = effective_K(K, N);
   const Dims dm = make_dims(prob, p, N, T, H, d, D, Ke);
   Scratch s;
-  const size_t need = carve_compress(dm, &s, (char*)workspace);
+  R0State r0;
+  const size_t need = carve_compress(dm, &s, (char*)workspace, &r0);
   if (ws_bytes < need) return GMC_ERR_WORKSPACE;
   cudaStream_t st = (cudaStream_t)stream_;
   gmc_trace_layout L;
@@ -336,13 +354,16 @@ int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* 
   GMC_STAGE("rownorm", 1, launch_rownorm(dm, hidden, p.norm_eps, s, st));
   GMC_STAGE("probe", 2, launch_probe(dm, keys, vo_probe, p, s, st));
   GMC_STAGE("message", message_tc_supported(dm) ? 2 : 1, launch_message(dm, keys, queries, s, st));
-  GMC_STAGE("heads", 3, launch_heads(dm, p, s, tv, st));
+  GMC_STAGE("heads", 4, launch_heads(dm, p, s, tv, st));
   GMC_STAGE("gram", 1, launch_gram(dm, hidden, s, st));
   GMC_STAGE("clients", 1, launch_build_clients(dm, p, fx, s, st));
-  GMC_STAGE("select", 1,
-            launch_select(dm.B, N, Ke, dm.M, dm.toff, H, T, p.landmarks * p.landmarks, p, fx,
-                          nullptr, s.C, s.scol, s.u0, s.order, s.support, s.slot, nullptr,
-                          s.status, tv, st));
+  GMC_STAGE("select", 4,
+            launch_round0(r0, dm.B, N, Ke, dm.M, dm.toff, H, T, p.landmarks * p.landmarks, p, fx,
+                          nullptr, s.C, s.scol, s.u0, s.order, s.status, tv, st) != cudaSuccess
+                ? cudaErrorLaunchFailure
+                : launch_select(r0, dm.B, N, Ke, dm.M, dm.toff, H, T, p.landmarks * p.landmarks,
+                                p, fx, nullptr, s.C, s.scol, s.u0, s.order, s.support, s.slot,
+                                nullptr, s.status, tv, st));
   GMC_STAGE("assign", 2, launch_assign(dm, p, s, tv, st));
   GMC_STAGE("transport", 2,
             launch_transport(dm, p, hidden, keys, pos_ids, s.support, s.pi, s.mass, s.rmsh,
@@ -354,7 +375,8 @@ int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* 
 // ---------------------------------------------------------------------------
 // gmc_select
 // ---------------------------------------------------------------------------
-static size_t carve_select(int B, int M, int N, int K, Scratch* s, char* base) {
+static size_t carve_select(int B, int M, int N, int K, Scratch* s, char* base,
+                           R0State* r0s = nullptr) {
   Carver c{base};
   Scratch t{};
   t.nSel = 64;
@@ -368,6 +390,8 @@ static size_t carve_select(int B, int M, int N, int K, Scratch* s, char* base) {
   t.selpart = c.take<double>((size_t)B * t.nSel);
   t.fexp = c.take<int32_t>((size_t)B);
   if (s) *s = t;
+  R0State r0 = carve_round0(c, (size_t)B, (size_t)N, (size_t)M);
+  if (r0s && base) *r0s = r0;
   return c.off;
 }
 
@@ -388,7 +412,8 @@ int gmc_select(const float* clients, int B, int M, int N, int K, const gmc_param
   if (params) p = *params; else gmc_default_params(&p);
   if (!params_ok(p)) return GMC_ERR_ARG;
   Scratch s;
-  const size_t need = carve_select(B, M, N, K, &s, (char*)workspace);
+  R0State r0;
+  const size_t need = carve_select(B, M, N, K, &s, (char*)workspace, &r0);
   if (ws_bytes < need) return GMC_ERR_WORKSPACE;
   cudaStream_t st = (cudaStream_t)stream_;
   TraceView tv{};
@@ -403,9 +428,11 @@ int gmc_select(const float* clients, int B, int M, int N, int K, const gmc_param
                           cudaMemcpyDeviceToDevice, st));
   GMC_TRY(cudaMemsetAsync(s.u0, 0, sizeof(long long) * B * (size_t)N, st));
   GMC_TRY(launch_select_prep(s.C, B, M, N, s, st));
-  GMC_TRY(launch_select(B, N, K, M, nullptr, 0, 1, 0, p, 0, s.fexp, s.C, s.scol, s.u0, s.order,
-                        s.support, s.slot, out_idx, s.status, tv, st));
-  g_launches += 4;
+  GMC_TRY(launch_round0(r0, B, N, K, M, nullptr, 0, 1, 0, p, 0, s.fexp, s.C, s.scol, s.u0,
+                        s.order, s.status, tv, st));
+  GMC_TRY(launch_select(r0, B, N, K, M, nullptr, 0, 1, 0, p, 0, s.fexp, s.C, s.scol, s.u0,
+                        s.order, s.support, s.slot, out_idx, s.status, tv, st));
+  g_launches += 7;
   return GMC_OK;
 }
 

@@ -116,7 +116,19 @@ __device__ __forceinline__ void warp_argbest(double& v, int& idx, bool want_max)
   }
 }
 
-__global__ void k_head_cluster(const double* __restrict__ hgpart, int nHG,
+// The pattern Gram: sum of the token-block partials, one warp per (image, entry),
+// lanes over the blocks (fixed order, so the sum is reproducible).
+__global__ void k_hg_reduce(const double* __restrict__ hgpart, int nHG, int B, int HH, double* HG) {
+  const int w = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (w >= B * HH) return;
+  const int b = w / HH, p = w % HH;
+  double s = 0.0;
+  for (int k = lane; k < nHG; k += 32) s += hgpart[((size_t)b * nHG + k) * HH + p];
+  s = warp_sum(s);
+  if (lane == 0) HG[(size_t)b * HH + p] = s;
+}
+
+__global__ void k_head_cluster(const double* __restrict__ HGred,
                                const float* __restrict__ rs, const int32_t* toff, int B, int N,
                                int Tmax, int H, int max_clusters, float head_eps, float* omega,
                                TraceView tv, uint32_t* status) {
@@ -127,11 +139,7 @@ __global__ void k_head_cluster(const double* __restrict__ hgpart, int nHG,
   double* HG = sm_hc;            // [H*H]
   double* cs = HG + H * H;       // [H*H] pattern cosines
   double* pre = cs + H * H;      // [H]
-  for (int p = threadIdx.x; p < H * H; p += blockDim.x) {
-    double s = 0.0;
-    for (int k = 0; k < nHG; ++k) s += hgpart[((size_t)b * nHG + k) * H * H + p];
-    HG[p] = s;
-  }
+  for (int p = threadIdx.x; p < H * H; p += blockDim.x) HG[p] = HGred[(size_t)b * H * H + p];
   __syncthreads();
   for (int h = threadIdx.x; h < H; h += blockDim.x) {
     double s1 = 0.0;
@@ -281,9 +289,12 @@ cudaError_t launch_heads(const Dims& dm, const gmc_params& p, Scratch& s, const 
                                                      H, p.terminal_q_weight, s.hgpart, s.nHG,
                                                      s.W2, s.status);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  const int warps = dm.B * H * H;
+  k_hg_reduce<<<ceil_div(warps * 32, 256), 256, 0, st>>>(s.hgpart, s.nHG, dm.B, H * H, s.HG);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
   size_t smem2 = sizeof(double) * (2 * (size_t)H * H + H);
   if ((e = set_smem_limit((const void*)k_head_cluster, smem2)) != cudaSuccess) return e;
-  k_head_cluster<<<dm.B, 128, smem2, st>>>(s.hgpart, s.nHG, s.rs, dm.toff, dm.B, dm.N, dm.T, H,
+  k_head_cluster<<<dm.B, 128, smem2, st>>>(s.HG, s.rs, dm.toff, dm.B, dm.N, dm.T, H,
                                           p.max_head_clusters, p.head_eps, s.omega, tv, s.status);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   k_energy<<<dm.B, 1024, 0, st>>>(s.omega, s.zn2, s.sigma, s.W2, dm.toff, dm.B, dm.N, dm.T, H,

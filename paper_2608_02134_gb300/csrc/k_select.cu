@@ -12,29 +12,51 @@
 // and in every later round (b only grows), so it never contributes to a gain,
 // a responsibility or a coverage update again.  After the first (dense) round
 // each client row keeps only its "survivors" {i : Cbar_mi > b_m}, compacted in
-// place, and every later round touches only those.  This is exact, not an
-// approximation: the skipped entries are exactly the zero residuals.  (A
-// pool member with R_mi = 0 still counts exp(0) = 1 in row m's softmax
-// denominator; the kernel adds those terms explicitly.)
+// place, and later rounds touch only those.  This is exact, not an
+// approximation: the skipped entries are exactly the zero residuals.  (A pool
+// member with R_mi = 0 still counts exp(0) = 1 in row m's softmax
+// denominator; the kernel adds those terms explicitly.)  Survivor lists start
+// in global memory (in place over Cbar, row-major, processed by 8-lane groups)
+// and move into the CTA's shared memory as soon as they all fit there, sorted
+// by token ("flat mode"): then the responsibilities and the coverage update
+// read only the pool's and the batch's token segments, and the gain update
+// sums every token's residuals in registers.
+//
+// The first round (dense, S empty) runs over the whole GPU (k_round0.cu); this
+// kernel continues from round 1 with the survivor lists it left.
 //
 // Parallel layout.  The CS CTAs of a cluster split the client rows; each CTA
-// keeps its rows' coverage b_m and survivor counts in shared memory and the
-// survivor lists in global memory (in place over Cbar).  Gains and scores are
-// summed in 64-bit fixed point, so the reductions across warps and CTAs
-// (shared / distributed-shared-memory atomics) are exact and deterministic.
-// Every CTA holds the same selected-set bitmap and derives the same control
-// decisions, so all CTAs run the same number of cluster barriers.
+// keeps its rows' coverage b_m, survivor counts and lists.  Gains and scores
+// are summed in 64-bit fixed point, so every reduction (shared-memory atomics
+// inside a CTA, distributed-shared-memory loads / atomics across the cluster)
+// is exact and order-independent: the solver is deterministic.  Per round:
+//   gains: each CTA reduces one slice of tokens over the cluster and
+//          broadcasts it, so every CTA holds the full gain vector;
+//   pool:  every CTA selects the same pool locally (histogram + exact tie
+//          ranking), slots numbered in ascending token order;
+//   scores: pushed into every CTA by atomics; every CTA picks the same batch.
+// Three cluster barriers per round; all control decisions are derived from
+// data every CTA holds identically, so all CTAs run the same barriers.
 #include <cooperative_groups.h>
 
 #include "common.cuh"
 #include "kernels.cuh"
+#include "select_common.cuh"
 
 namespace cg = cooperative_groups;
 
 namespace gmc {
 
+namespace {
 constexpr int SEL_THREADS = 512;
+constexpr int SEL_WARPS = SEL_THREADS / 32;
 constexpr int SEL_MAX_CS = 16;
+constexpr int HBINS = sel::HBINS;
+constexpr int UNR = 4;     // entries in flight per lane in a sweep
+constexpr int PCL = 8;     // pool entries a lane keeps in registers (8 lanes x 8 >= pool of 64)
+constexpr int DEADROW = 0xFFFF;  // flat mode: row id of an entry whose residual is zero
+constexpr int FU = 4;      // flat mode: entries a thread loads ahead in a walk
+constexpr size_t SMEM_LIMIT = 227 * 1024;
 
 struct SelArgs {
   int B, N, K, Mstride, H, Tmax, L2;
@@ -53,65 +75,118 @@ struct SelArgs {
   int32_t* out_idx;
   uint32_t* status;
   TraceView tv;
+  int cap;              // survivor entries that fit in shared memory
+  int rpc;              // rows one CTA can own
+  R0State r0;           // state after the first round
 };
 
 struct SelSmem {
-  long long* u_part;   // [N]   this CTA's partial gains (fixed point)
-  long long* u_slice;  // [SL]  reduced gains of this CTA's token slice
-  long long* cand_u;   // [CS][P] candidates pushed by every CTA
-  int* cand_j;         // [CS][P]
-  int* ncand;          // [CS]
-  int* pool;           // [P]
-  long long* s_acc;    // [P]   cluster-wide scores
-  long long* s_loc;    // [P]   this CTA's partial scores
-  int* batch;          // [P]
-  int* inb;            // [P]   pool slot is in the batch
-  short* poolslot;     // [N]   pool slot of a token or -1
-  unsigned char* sel;  // [N]   selected flags
-  float* bcov;         // [RPC] coverage b_m of this CTA's rows
-  int* cnt;            // [RPC] survivor count (-1: row still dense)
-  long long* fb;       // [8]   bank sums F_S[3], F_V[3] (fixed point)
-  int* scal;           // [8]   S count, Pt, nb, rounds, filled, nloc
+  unsigned* u_lo;       // [N]  this CTA's partial gains of the next round, low 32 bits
+  unsigned* u_hi;       // [N]  high 32 bits (carries included)
+  long long* u_full;    // [N]  gains of the current round (every CTA)
+  int* hist;            // [HBINS]
+  int* bnd;             // [N]  tokens in the boundary histogram bin
+  unsigned char* inpool;  // [N]
+  unsigned char* sel;   // [N]
+  short* poolslot;      // [N]  pool slot of a token or -1
+  int* pool;            // [P]
+  long long* s_acc;     // [P]  cluster-wide scores
+  unsigned long long* sw;  // [SEL_WARPS][P] per-warp partial scores
+  long long* s_part;    // [P]  this CTA's scores, read by the whole cluster
+  int* batch;           // [P]
+  int* inb;             // [P]
+  int* wsum;            // [32] scan scratch
+  float* bcov;          // [RPC] coverage b_m of this CTA's rows
+  int* cnt;             // [RPC] survivors (-1: row still dense)
+  int* rmaxb;           // [RPC] flat mode: bits of the row's largest pool residual
+  int* npl;             // [RPC] flat mode: pool entries of the row
+  unsigned long long* z64;  // [RPC] flat mode: softmax denominator (fixed point 2^40)
+  int* bnb;             // [RPC] flat mode: bits of the row's largest batch value
+  long long* bfix;      // [RPC] flat mode: coverage in fixed point
+  int* cstart;          // [N+1] flat mode: first entry of every token
+  int* rowb;            // [SEL_MAX_CS + 1] first client row of every CTA of the cluster
+  long long* fb;        // [8]  F_S[3], F_V[3] (fixed point)
+  int* scal;            // [16] Bstar, c_hi, Pt, nbnd, cursor, global rows left
+  float* svals;         // [cap]
+  uint16_t* scols;      // [cap]
+  uint16_t* srows;      // [cap] flat mode: row of every entry (DEADROW: residual zero)
 };
 
-__host__ __device__ inline size_t sel_smem_bytes(int N, int CS, int P, int RPC, SelSmem* o,
-                                                 char* base) {
+enum { SC_BSTAR = 0, SC_CHI, SC_PT, SC_NBND, SC_CURSOR, SC_GLOBAL, SC_NEED };
+
+__host__ __device__ inline size_t sel_fixed_bytes(int N, int P, int RPC, SelSmem* o, char* base) {
   size_t off = 0;
   auto take = [&](size_t bytes) {
     size_t at = off;
     off += (bytes + 15) & ~(size_t)15;
     return base ? base + at : nullptr;
   };
-  const int SL = (N + CS - 1) / CS;
   char* p;
-  p = take(sizeof(long long) * N);      if (o) o->u_part = (long long*)p;
-  p = take(sizeof(long long) * SL);     if (o) o->u_slice = (long long*)p;
-  p = take(sizeof(long long) * CS * P); if (o) o->cand_u = (long long*)p;
-  p = take(sizeof(int) * CS * P);       if (o) o->cand_j = (int*)p;
-  p = take(sizeof(int) * CS);           if (o) o->ncand = (int*)p;
-  p = take(sizeof(int) * P);            if (o) o->pool = (int*)p;
-  p = take(sizeof(long long) * P);      if (o) o->s_acc = (long long*)p;
-  p = take(sizeof(long long) * P);      if (o) o->s_loc = (long long*)p;
-  p = take(sizeof(int) * P);            if (o) o->batch = (int*)p;
-  p = take(sizeof(int) * P);            if (o) o->inb = (int*)p;
-  p = take(sizeof(short) * N);          if (o) o->poolslot = (short*)p;
-  p = take(N);                          if (o) o->sel = (unsigned char*)p;
-  p = take(sizeof(float) * RPC);        if (o) o->bcov = (float*)p;
-  p = take(sizeof(int) * RPC);          if (o) o->cnt = (int*)p;
-  p = take(sizeof(long long) * 8);      if (o) o->fb = (long long*)p;
-  p = take(sizeof(int) * 8);            if (o) o->scal = (int*)p;
+  p = take(sizeof(unsigned) * N);   if (o) o->u_lo = (unsigned*)p;
+  p = take(sizeof(unsigned) * N);   if (o) o->u_hi = (unsigned*)p;
+  p = take(sizeof(long long) * N);  if (o) o->u_full = (long long*)p;
+  p = take(sizeof(int) * HBINS);    if (o) o->hist = (int*)p;
+  p = take(sizeof(int) * N);        if (o) o->bnd = (int*)p;
+  p = take(N);                      if (o) o->inpool = (unsigned char*)p;
+  p = take(N);                      if (o) o->sel = (unsigned char*)p;
+  p = take(sizeof(short) * N);      if (o) o->poolslot = (short*)p;
+  p = take(sizeof(int) * P);        if (o) o->pool = (int*)p;
+  p = take(sizeof(long long) * P);  if (o) o->s_acc = (long long*)p;
+  p = take(sizeof(unsigned long long) * SEL_WARPS * P);  if (o) o->sw = (unsigned long long*)p;
+  p = take(sizeof(long long) * P);  if (o) o->s_part = (long long*)p;
+  p = take(sizeof(int) * P);        if (o) o->batch = (int*)p;
+  p = take(sizeof(int) * P);        if (o) o->inb = (int*)p;
+  p = take(sizeof(int) * 32);       if (o) o->wsum = (int*)p;
+  p = take(sizeof(float) * RPC);    if (o) o->bcov = (float*)p;
+  p = take(sizeof(int) * RPC);      if (o) o->cnt = (int*)p;
+  p = take(sizeof(int) * RPC);      if (o) o->rmaxb = (int*)p;
+  p = take(sizeof(int) * RPC);      if (o) o->npl = (int*)p;
+  p = take(sizeof(unsigned long long) * RPC); if (o) o->z64 = (unsigned long long*)p;
+  p = take(sizeof(int) * RPC);      if (o) o->bnb = (int*)p;
+  p = take(sizeof(long long) * RPC);  if (o) o->bfix = (long long*)p;
+  p = take(sizeof(int) * (N + 1));  if (o) o->cstart = (int*)p;
+  p = take(sizeof(int) * (SEL_MAX_CS + 1));  if (o) o->rowb = (int*)p;
+  p = take(sizeof(long long) * 8);  if (o) o->fb = (long long*)p;
+  p = take(sizeof(int) * 16);       if (o) o->scal = (int*)p;
   return off;
 }
 
-__device__ __forceinline__ bool key_before(long long ua, int ja, long long ub, int jb) {
-  return ua > ub || (ua == ub && ja < jb);
+using sel::key_before;
+using sel::lanemask_lt;
+using sel::block_exclusive_scan;
+
+// Exact 64-bit fixed-point add into shared memory as two 32-bit atomics: the
+// low word wraps and its carry goes to the high word, so the pair always holds
+// the exact sum, whatever the order of the additions.
+__device__ __forceinline__ void add_fix(unsigned* lo, unsigned* hi, unsigned long long v) {
+  const unsigned vl = (unsigned)v, vh = (unsigned)(v >> 32);
+  const unsigned old = atomicAdd(lo, vl);
+  const unsigned up = vh + ((old + vl) < old ? 1u : 0u);
+  if (up) atomicAdd(hi, up);
+}
+__device__ __forceinline__ long long get_fix(const unsigned* lo, const unsigned* hi) {
+  return (long long)(((unsigned long long)*hi << 32) | *lo);
 }
 
-__device__ __forceinline__ unsigned lanemask_lt() {
-  unsigned m;
-  asm("mov.u32 %0, %%lanemask_lt;" : "=r"(m));
-  return m;
+// Reductions inside an aligned group of G = 8 lanes (mask `gm`).
+constexpr int G = 8;
+__device__ __forceinline__ float group_max(float v, unsigned gm) {
+#pragma unroll
+  for (int o = G / 2; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(gm, v, o));
+  return v;
 }
+__device__ __forceinline__ float group_sum(float v, unsigned gm) {
+#pragma unroll
+  for (int o = G / 2; o > 0; o >>= 1) v += __shfl_xor_sync(gm, v, o);
+  return v;
+}
+__device__ __forceinline__ int group_sum(int v, unsigned gm) {
+#pragma unroll
+  for (int o = G / 2; o > 0; o >>= 1) v += __shfl_xor_sync(gm, v, o);
+  return v;
+}
+
+}  // namespace
 
 __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
   extern __shared__ __align__(16) char sm_sel[];
@@ -119,7 +194,7 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
   const int CS = (int)cluster.num_blocks();
   const int r = (int)cluster.block_rank();
   const int b = blockIdx.x / CS;
-  const int N = a.N, P = a.P;
+  const int N = a.N, P = a.P, K = a.K;
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
 
   // Image geometry: rows [0, MG) grounded, [MG, MG+N) appearance, rest spatial.
@@ -134,93 +209,164 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
     MG = a.H * tg.T;
     Mb = MG + N + a.L2;
   }
-  const int RPC = (a.Mstride + CS - 1) / CS;
-  const int mlo = r * RPC, mhi = min(Mb, mlo + RPC);
+  const int RPC = a.rpc;  // capacity of the per-row arrays of one CTA
   const int SL = (N + CS - 1) / CS;
   const int jlo = r * SL, jhi = min(N, jlo + SL);
-  const int K = a.K;
 
   SelSmem s;
-  sel_smem_bytes(N, CS, P, RPC, &s, sm_sel);
+  const size_t fixed = sel_fixed_bytes(N, P, RPC, &s, sm_sel);
+  s.svals = reinterpret_cast<float*>(sm_sel + fixed);
+  s.scols = reinterpret_cast<uint16_t*>(sm_sel + fixed + sizeof(float) * (size_t)a.cap);
+  s.srows = s.scols + a.cap;
   const int e = a.fexp ? a.fexp[b] : a.fx_exp;
   const float fxs = ldexpf(1.f, e);
   float* Cimg = a.C + (size_t)b * a.Mstride * N;
   uint16_t* Simg = a.scol + (size_t)b * a.Mstride * N;
 
+  // state after the first round (k_round0.cu); a first round with an empty
+  // pool leaves the gains of the empty support and nothing selected
+  const int Pt0 = valid ? a.r0.info[b * 4] : 0;
+  const int nb0 = Pt0 > 0 ? a.r0.info[b * 4 + 1] : 0;
   for (int j = threadIdx.x; j < N; j += blockDim.x) {
-    s.u_part[j] = 0;
+    s.u_lo[j] = 0;
+    s.u_hi[j] = 0;
+    s.u_full[j] = Pt0 > 0 ? a.r0.u1[(size_t)b * N + j] : a.u0[(size_t)b * N + j];
     s.poolslot[j] = -1;
     s.sel[j] = 0;
+    s.inpool[j] = 0;
   }
-  for (int j = jlo + threadIdx.x; j < jhi; j += blockDim.x) s.u_slice[j - jlo] = a.u0[(size_t)b * N + j];
   for (int k = threadIdx.x; k < P; k += blockDim.x) s.s_acc[k] = 0;
+  if (threadIdx.x < 8) s.fb[threadIdx.x] = 0;
+  if (threadIdx.x < 16) s.scal[threadIdx.x] = 0;
+  if (threadIdx.x == 0) s.scal[SC_GLOBAL] = 1;
+  // Rows are split over the cluster so every CTA holds about the same number
+  // of survivors (weight: survivors + 16 per row); every CTA computes the same
+  // split.  Without a first round, or if a part would exceed RPC rows, the
+  // rows are split evenly.
+  if (threadIdx.x <= SEL_MAX_CS) s.rowb[threadIdx.x] = Mb;
+  __syncthreads();
+  bool balanced = false;
+  if (Pt0 > 0 && CS > 1) {
+    const int chunk = (Mb + blockDim.x - 1) / blockDim.x;
+    const int m0 = min(Mb, (int)threadIdx.x * chunk), m1 = min(Mb, m0 + chunk);
+    const int32_t* cgl = a.r0.cnt + (size_t)b * a.Mstride;
+    int wsum = 0;
+    for (int m = m0; m < m1; ++m) wsum += cgl[m] + 16;
+    int W = 0;
+    int run = block_exclusive_scan(wsum, s.wsum, &W);
+    for (int m = m0; m < m1; ++m) {
+      const int wm = cgl[m] + 16;
+      // CTA c starts after the row where the preceding weight reaches c*W/CS
+      for (int c = 1; c < CS; ++c) {
+        const long long tgt = (long long)c * W / CS;
+        if (run < tgt && run + wm >= tgt) atomicMin(&s.rowb[c], m + 1);
+      }
+      run += wm;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      s.rowb[0] = 0;
+      int prev = 0, ok = 1;
+      for (int c = 1; c <= CS; ++c) {
+        int bc = c < CS ? s.rowb[c] : Mb;
+        if (bc < prev) bc = prev;
+        if (c < CS) s.rowb[c] = bc;
+        if (bc - prev > RPC) ok = 0;
+        prev = bc;
+      }
+      s.scal[SC_NEED] = ok;
+    }
+    __syncthreads();
+    balanced = s.scal[SC_NEED] != 0;
+  }
+  const int even = (Mb + CS - 1) / CS;
+  const int mlo = balanced ? s.rowb[r] : min(Mb, r * even);
+  const int mhi = balanced ? (r + 1 < CS ? s.rowb[r + 1] : Mb) : min(Mb, mlo + even);
+  const int nrows = max(0, mhi - mlo);
   for (int q = threadIdx.x; q < RPC; q += blockDim.x) {
-    s.bcov[q] = 0.f;
-    s.cnt[q] = -1;
+    const bool have = Pt0 > 0 && q < nrows;
+    s.bcov[q] = have ? a.r0.bcov[(size_t)b * a.Mstride + mlo + q] : 0.f;
+    s.cnt[q] = have ? a.r0.cnt[(size_t)b * a.Mstride + mlo + q] : 0;
+    s.bfix[q] = 0;
+    s.rmaxb[q] = 0;
+    s.npl[q] = 0;
+    s.z64[q] = 0;
+    s.bnb[q] = 0;
   }
-  if (threadIdx.x < 8) {
-    s.fb[threadIdx.x] = 0;
-    s.scal[threadIdx.x] = 0;
-  }
+  __syncthreads();
+  for (int q = threadIdx.x; q < nb0; q += blockDim.x) s.sel[a.order[(size_t)b * K + q]] = 1;
   cluster.sync();
-  if (!valid) return;  // uniform across the cluster: nobody touches this CTA again
+  if (!valid) return;  // uniform across the cluster
+
+  // Move this CTA's survivor lists from global into shared memory once they
+  // all fit, sorted by token (a counting sort): the entries of token j are
+  // [cstart[j], cstart[j+1]).  The order inside a token's segment depends on
+  // the schedule; nothing computed from it does (integer and max reductions).
+  auto migrate = [&]() {
+    if (!s.scal[SC_GLOBAL] || nrows >= DEADROW) return;  // row ids are stored in 16 bits
+    int mine = 0;
+    for (int q = threadIdx.x; q < nrows; q += blockDim.x) mine += s.cnt[q];
+    int tot = 0;
+    block_exclusive_scan(mine, s.wsum, &tot);
+    if (tot > a.cap) return;  // uniform over the block
+    for (int j = threadIdx.x; j < N; j += blockDim.x) s.bnd[j] = 0;
+    __syncthreads();
+    for (int q = wid; q < nrows; q += nw) {
+      const uint16_t* gc = Simg + (size_t)(mlo + q) * N;
+      const int n = s.cnt[q];
+      for (int k = lane; k < n; k += 32) atomicAdd(&s.bnd[gc[k]], 1);
+    }
+    __syncthreads();
+    {
+      const int per = (N + blockDim.x - 1) / blockDim.x;
+      const int j0 = min(N, (int)threadIdx.x * per), j1 = min(N, j0 + per);
+      int c = 0;
+      for (int j = j0; j < j1; ++j) c += s.bnd[j];
+      int at = block_exclusive_scan(c, s.wsum, nullptr);
+      for (int j = j0; j < j1; ++j) {
+        const int n = s.bnd[j];
+        s.cstart[j] = at;
+        s.bnd[j] = at;  // fill cursor of token j
+        at += n;
+      }
+      if (threadIdx.x == 0) s.cstart[N] = tot;
+    }
+    __syncthreads();
+    for (int q = wid; q < nrows; q += nw) {
+      const float* gv = Cimg + (size_t)(mlo + q) * N;
+      const uint16_t* gc = Simg + (size_t)(mlo + q) * N;
+      const int n = s.cnt[q];
+      for (int k = lane; k < n; k += 32) {
+        const int j = gc[k];
+        const int pos = atomicAdd(&s.bnd[j], 1);
+        s.svals[pos] = gv[k];
+        s.scols[pos] = (uint16_t)j;
+        s.srows[pos] = (uint16_t)q;
+      }
+    }
+    for (int q = threadIdx.x; q < nrows; q += blockDim.x) s.bfix[q] = to_fix(s.bcov[q], fxs);
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      s.scal[SC_CURSOR] = tot;
+      s.scal[SC_GLOBAL] = 0;
+    }
+    __syncthreads();
+  };
+  if (Pt0 > 0) migrate();
 
   const int rounds_max = (K + a.bsz - 1) / a.bsz + 1;
-  int S_count = 0, rnd = 0, filled = 0;
-  bool done = false;
-  while (!done) {
-    // ---- A: local candidates of this CTA's token slice -------------------
-    int npos_local = 0;
-    for (int j = jlo + threadIdx.x; j < jhi; j += blockDim.x) {
-      const long long uj = s.u_slice[j - jlo];
-      if (s.sel[j] || uj <= 0) continue;
-      int rank = 0;
-      for (int k = jlo; k < jhi; ++k) {
-        const long long uk = s.u_slice[k - jlo];
-        rank += (!s.sel[k] && uk > 0 && key_before(uk, k, uj, j));
-      }
-      ++npos_local;
-      if (rank < P) {
-        for (int c = 0; c < CS; ++c) {
-          cluster.map_shared_rank(s.cand_u, c)[r * P + rank] = uj;
-          cluster.map_shared_rank(s.cand_j, c)[r * P + rank] = j;
-        }
-      }
+  int S_count = nb0, rnd = Pt0 > 0 ? 1 : 0, filled = 0;
+  const int sub = lane / G, gl = lane % G;
+  const unsigned gm = 0xFFu << (sub * G);
+  const unsigned lt = lanemask_lt() & gm;
+  while (S_count < K) {
+    if (rnd >= rounds_max) {  // cannot happen (each round adds >= 1 token); guard the loop
+      if (threadIdx.x == 0) set_status(a.status, GMC_STATUS_INTERNAL);
+      break;
     }
-    {
-      __shared__ int cnt_sh;
-      if (threadIdx.x == 0) cnt_sh = 0;
-      __syncthreads();
-      if (npos_local) atomicAdd(&cnt_sh, npos_local);
-      __syncthreads();
-      if (threadIdx.x == 0) {
-        const int nloc = min(P, cnt_sh);
-        s.scal[5] = nloc;
-        for (int c = 0; c < CS; ++c) cluster.map_shared_rank(s.ncand, c)[r] = nloc;
-      }
-    }
-    cluster.sync();  // B1: every CTA's candidates are visible everywhere
-
-    // ---- B: global pool ranks; reset this CTA's gain partials ------------
-    int total = 0;
-    for (int c = 0; c < CS; ++c) total += s.ncand[c];
-    const int Pt = min(P, total);
-    const int nloc = s.scal[5];
-    for (int k = threadIdx.x; k < nloc; k += blockDim.x) {
-      const long long uk = s.cand_u[r * P + k];
-      const int jk = s.cand_j[r * P + k];
-      int grank = 0;
-      for (int c = 0; c < CS; ++c) {
-        const int nc = s.ncand[c];
-        for (int q = 0; q < nc; ++q)
-          grank += key_before(s.cand_u[c * P + q], s.cand_j[c * P + q], uk, jk);
-      }
-      if (grank < Pt)
-        for (int c = 0; c < CS; ++c) cluster.map_shared_rank(s.pool, c)[grank] = jk;
-    }
-    for (int j = threadIdx.x; j < N; j += blockDim.x) s.u_part[j] = 0;
-    cluster.sync();  // B2: the pool is visible everywhere
-
+    // ---- pool of this round ------------------------------------------------------
+    sel::PoolScratch pw{s.hist, s.bnd, s.inpool, s.wsum, s.scal + 8};
+    const int Pt = sel::select_pool(s.u_full, s.sel, N, P, pw, s.pool, s.poolslot);
     if (Pt == 0) {
       // Zero-gain remainder: fill in ascending source order (F unchanged).
       const int need = K - S_count;
@@ -249,178 +395,307 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
       __syncthreads();
       break;
     }
-
-    // ---- C: responsibilities over the pool -------------------------------
-    for (int k = threadIdx.x; k < Pt; k += blockDim.x) {
-      s.poolslot[s.pool[k]] = (short)k;
-      s.s_loc[k] = 0;
+    for (int k = threadIdx.x; k < SEL_WARPS * Pt; k += blockDim.x) s.sw[k] = 0;
+    if (r == 0 && a.tv.base && threadIdx.x < a.tv.pool_size) {
+      int32_t* tp = a.tv.at<int32_t>(b, a.tv.off_pool) + (size_t)rnd * a.tv.pool_size;
+      tp[threadIdx.x] = threadIdx.x < Pt ? s.pool[threadIdx.x] : -1;
     }
     __syncthreads();
-    for (int m = mlo + wid; m < mhi; m += nw) {
-      const int q = m - mlo;
-      const float bm = s.bcov[q];
-      const int n = s.cnt[q];
-      const float* crow = Cimg + (size_t)m * N;
-      const uint16_t* jrow = Simg + (size_t)m * N;
-      // pass 1: max residual and number of positive pool entries
+
+    // ---- flat mode (every list of this CTA in shared memory, sorted by token):
+    // the responsibilities touch only the pool tokens' segments, one warp per
+    // pool token; per-row values are order-independent (max of positive floats
+    // as integers, fixed-point sums), so nothing depends on the schedule.
+    const bool flat = !s.scal[SC_GLOBAL];
+    const float z_one = 1099511627776.f;  // 2^40: fixed-point scale of the softmax denominators
+    const float z_inv = 1.f / z_one;
+    if (flat) {
+      // largest pool residual and number of pool entries of every row
+      for (int k = wid; k < Pt; k += nw) {
+        const int j = s.pool[k];
+        for (int p = s.cstart[j] + lane; p < s.cstart[j + 1]; p += 32) {
+          const int q = s.srows[p];
+          if (q == DEADROW) continue;
+          atomicMax(&s.rmaxb[q], __float_as_int(s.svals[p] - s.bcov[q]));
+          atomicAdd(&s.npl[q], 1);
+        }
+      }
+      __syncthreads();
+      // softmax denominators, exact in 2^-40
+      for (int k = wid; k < Pt; k += nw) {
+        const int j = s.pool[k];
+        for (int p = s.cstart[j] + lane; p < s.cstart[j + 1]; p += 32) {
+          const int q = s.srows[p];
+          if (q == DEADROW) continue;
+          const float tau = a.resp_temp * __int_as_float(s.rmaxb[q]) + a.resp_eps;
+          atomicAdd(&s.z64[q], (unsigned long long)__float2ll_rn(
+                                   expf((s.svals[p] - s.bcov[q]) / tau) * z_one));
+        }
+      }
+      __syncthreads();
+      // s_k = sum_m rho_mk R_mk: one warp owns pool slot k, so its sum is this CTA's score
+      for (int k = wid; k < Pt; k += nw) {
+        const int j = s.pool[k];
+        unsigned long long acc = 0;
+        for (int p = s.cstart[j] + lane; p < s.cstart[j + 1]; p += 32) {
+          const int q = s.srows[p];
+          if (q == DEADROW) continue;
+          const float tau = a.resp_temp * __int_as_float(s.rmaxb[q]) + a.resp_eps;
+          const float z = (float)s.z64[q] * z_inv + (float)(Pt - s.npl[q]);
+          const float R = s.svals[p] - s.bcov[q];
+          acc += (unsigned long long)to_fix(expf(R / tau) / z * R, fxs);
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(FULL, acc, o);
+        if (lane == 0) s.s_part[k] = (long long)acc;
+      }
+    }
+    if (!flat) {
+    // ---- responsibilities of this CTA's rows over the pool (8-lane group per row)
+    // One sweep of the row finds its pool entries; each lane keeps up to PCL of
+    // them in registers for the softmax (more: a second sweep).
+    for (int q0 = wid * (32 / G); q0 < nrows; q0 += nw * (32 / G)) {
+      const int q = q0 + sub;
+      const int n = q < nrows ? s.cnt[q] : 0;
+      const float bm = q < nrows ? s.bcov[q] : 0.f;
+      const float* vals = Cimg + (size_t)(mlo + q) * N;
+      const uint16_t* cols = Simg + (size_t)(mlo + q) * N;
       float rmax = 0.f;
-      int npool = 0;
-      if (n < 0) {
-        for (int k = lane; k < Pt; k += 32) {
-          const float R = crow[s.pool[k]] - bm;
-          if (R > 0.f) { rmax = fmaxf(rmax, R); ++npool; }
+      int npool = 0, ncache = 0, mine = 0;  // mine: pool entries this lane saw
+      float cv[PCL] = {};
+      int cs[PCL] = {};
+      bool spill = false;
+      for (int k0 = gl; k0 < n; k0 += UNR * G) {
+        int cc[UNR];
+        float vv[UNR];
+#pragma unroll
+        for (int u = 0; u < UNR; ++u) {
+          const int k = k0 + u * G;
+          cc[u] = k < n ? (int)cols[k] : -1;
+          vv[u] = k < n ? vals[k] : 0.f;
         }
-      } else {
-        for (int k = lane; k < n; k += 32) {
-          if (s.poolslot[jrow[k]] >= 0) {
-            const float R = crow[k] - bm;
-            rmax = fmaxf(rmax, R);
-            ++npool;
-          }
-        }
-      }
-      rmax = warp_max(rmax);
-      npool = warp_sum_int(npool);
-      if (npool == 0) continue;
-      const float tau = a.resp_temp * rmax + a.resp_eps;
-      // pass 2: softmax denominator (zero-residual pool entries add exp(0) = 1)
-      float z = 0.f;
-      if (n < 0) {
-        for (int k = lane; k < Pt; k += 32) {
-          const float R = crow[s.pool[k]] - bm;
-          if (R > 0.f) z += expf(R / tau);
-        }
-      } else {
-        for (int k = lane; k < n; k += 32)
-          if (s.poolslot[jrow[k]] >= 0) z += expf((crow[k] - bm) / tau);
-      }
-      z = warp_sum(z) + (float)(Pt - npool);
-      const float invz = 1.f / z;
-      // pass 3: s_i += rho_mi R_mi
-      if (n < 0) {
-        for (int k = lane; k < Pt; k += 32) {
-          const float R = crow[s.pool[k]] - bm;
-          if (R > 0.f)
-            atomicAdd((unsigned long long*)&s.s_loc[k],
-                      (unsigned long long)to_fix(expf(R / tau) * invz * R, fxs));
-        }
-      } else {
-        for (int k = lane; k < n; k += 32) {
-          const int ps = s.poolslot[jrow[k]];
+#pragma unroll
+        for (int u = 0; u < UNR; ++u) {
+          const int ps = cc[u] >= 0 ? s.poolslot[cc[u]] : -1;
           if (ps >= 0) {
-            const float R = crow[k] - bm;
-            atomicAdd((unsigned long long*)&s.s_loc[ps],
-                      (unsigned long long)to_fix(expf(R / tau) * invz * R, fxs));
+            rmax = fmaxf(rmax, vv[u] - bm);
+#pragma unroll
+            for (int t = 0; t < PCL; ++t)
+              if (t == mine) {
+                cv[t] = vv[u];
+                cs[t] = ps;
+              }
+            spill |= mine >= PCL;
+            ++mine;
           }
         }
       }
+      rmax = group_max(rmax, gm);
+      npool = group_sum(mine, gm);
+      const bool any_spill = __any_sync(gm, spill);
+      ncache = mine < PCL ? mine : PCL;
+      if (npool > 0) {
+        const float tau = a.resp_temp * rmax + a.resp_eps;
+        float z = 0.f;
+        if (!any_spill) {
+#pragma unroll
+          for (int t = 0; t < PCL; ++t)
+            if (t < ncache) z += expf((cv[t] - bm) / tau);
+        } else {
+          for (int k = gl; k < n; k += G)
+            if (s.poolslot[cols[k]] >= 0) z += expf((vals[k] - bm) / tau);
+        }
+        z = group_sum(z, gm) + (float)(Pt - npool);
+        const float invz = 1.f / z;
+        if (!any_spill) {
+#pragma unroll
+          for (int t = 0; t < PCL; ++t)
+            if (t < ncache) {
+              const float R = cv[t] - bm;
+              atomicAdd(&s.sw[wid * Pt + cs[t]],
+                        (unsigned long long)to_fix(expf(R / tau) * invz * R, fxs));
+            }
+        } else {
+          for (int k = gl; k < n; k += G) {
+            const int ps = s.poolslot[cols[k]];
+            if (ps >= 0) {
+              const float R = vals[k] - bm;
+              atomicAdd(&s.sw[wid * Pt + ps],
+                        (unsigned long long)to_fix(expf(R / tau) * invz * R, fxs));
+            }
+          }
+        }
+      }
+    }
     }
     __syncthreads();
+    if (!flat)
+      for (int k = threadIdx.x; k < Pt; k += blockDim.x) {
+        unsigned long long v = 0;
+        for (int w2 = 0; w2 < SEL_WARPS; ++w2) v += s.sw[w2 * Pt + k];
+        s.s_part[k] = (long long)v;
+      }
+    cluster.sync();  // every CTA's scores are complete
     for (int k = threadIdx.x; k < Pt; k += blockDim.x) {
-      const unsigned long long v = (unsigned long long)s.s_loc[k];
-      if (v)
-        for (int c = 0; c < CS; ++c)
-          atomicAdd((unsigned long long*)cluster.map_shared_rank(s.s_acc, c) + k, v);
+      long long v[SEL_MAX_CS];
+#pragma unroll
+      for (int c = 0; c < SEL_MAX_CS; ++c) v[c] = c < CS ? cluster.map_shared_rank(s.s_part, c)[k] : 0;
+      long long t = 0;
+#pragma unroll
+      for (int c = 0; c < SEL_MAX_CS; ++c) t += v[c];
+      s.s_acc[k] = t;
     }
-    cluster.sync();  // B3: the scores are complete everywhere
+    __syncthreads();
 
-    // ---- D: batch, coverage update, survivor filter, next gains ----------
+    // ---- batch, coverage update, survivor filter, next gains ------------------
     const int nb = min(a.bsz, min(Pt, K - S_count));
     for (int k = threadIdx.x; k < Pt; k += blockDim.x) {
-      const long long sk = s.s_acc[k];
-      const int jk = s.pool[k];
-      int rank = 0;
-      for (int q = 0; q < Pt; ++q) rank += key_before(s.s_acc[q], s.pool[q], sk, jk);
+      const int rank = sel::score_rank(s.s_acc, s.pool, Pt, k);
       s.inb[k] = rank < nb;
-      if (rank < nb) s.batch[rank] = jk;
+      if (rank < nb) s.batch[rank] = s.pool[k];
     }
     __syncthreads();
     for (int q = threadIdx.x; q < nb; q += blockDim.x) {
       s.sel[s.batch[q]] = 1;
       if (r == 0) a.order[(size_t)b * K + S_count + q] = s.batch[q];
     }
-    if (r == 0 && a.tv.base && threadIdx.x == 0) {
-      int32_t* tp = a.tv.at<int32_t>(b, a.tv.off_pool) + (size_t)rnd * a.tv.pool_size;
-      for (int k = 0; k < a.tv.pool_size; ++k) tp[k] = k < Pt ? s.pool[k] : -1;
+    if (r == 0 && a.tv.base && threadIdx.x == 0)
       a.tv.at<int32_t>(b, a.tv.off_round_end)[rnd] = S_count + nb;
+    if (flat) {
+      // coverage update: largest batch value per row, one warp per batch token
+      for (int k = wid; k < nb; k += nw) {
+        const int j = s.batch[k];
+        for (int p = s.cstart[j] + lane; p < s.cstart[j + 1]; p += 32) {
+          const int q = s.srows[p];
+          if (q != DEADROW) atomicMax(&s.bnb[q], __float_as_int(s.svals[p]));
+        }
+      }
+      __syncthreads();
+      for (int q = threadIdx.x; q < nrows; q += blockDim.x) {
+        const float bn = fmaxf(s.bcov[q], __int_as_float(s.bnb[q]));
+        s.bcov[q] = bn;
+        s.bfix[q] = to_fix(bn, fxs);
+        s.bnb[q] = 0;
+        s.rmaxb[q] = 0;
+        s.npl[q] = 0;
+        s.z64[q] = 0;
+      }
+      __syncthreads();
+      // survivor filter (dead entries marked in place) and next-round gains: each
+      // thread walks a contiguous slice (an odd length keeps a warp's threads on
+      // distinct banks) and sums every token's residuals in a register
+      const int tot = s.scal[SC_CURSOR];
+      const int per = ((tot + SEL_THREADS - 1) / SEL_THREADS) | 1;
+      const int p0s = min(tot, (int)threadIdx.x * per), p1s = min(tot, p0s + per);
+      int jc = -1;
+      unsigned long long acc = 0;
+      for (int p0 = p0s; p0 < p1s; p0 += FU) {
+        int qq[FU], jj[FU];
+        float cc[FU];
+#pragma unroll
+        for (int u = 0; u < FU; ++u) {
+          const bool in = p0 + u < p1s;
+          qq[u] = in ? (int)s.srows[p0 + u] : DEADROW;
+          jj[u] = in ? (int)s.scols[p0 + u] : 0;
+          cc[u] = in ? s.svals[p0 + u] : 0.f;
+        }
+#pragma unroll
+        for (int u = 0; u < FU; ++u) {
+          if (qq[u] == DEADROW) continue;
+          if (cc[u] > s.bcov[qq[u]]) {
+            if (jj[u] != jc) {
+              if (acc) add_fix(&s.u_lo[jc], &s.u_hi[jc], acc);
+              jc = jj[u];
+              acc = 0;
+            }
+            acc += (unsigned long long)(to_fix(cc[u], fxs) - s.bfix[qq[u]]);
+          } else {
+            s.srows[p0 + u] = (uint16_t)DEADROW;
+          }
+        }
+      }
+      if (acc) add_fix(&s.u_lo[jc], &s.u_hi[jc], acc);
     }
-    const bool dense_round = (rnd == 0);
-    for (int m = mlo + wid; m < mhi; m += nw) {
-      const int q = m - mlo;
-      const float bm = s.bcov[q];
-      const int n = s.cnt[q];
-      float* crow = Cimg + (size_t)m * N;
-      uint16_t* jrow = Simg + (size_t)m * N;
+    if (!flat) {
+    for (int q0 = wid * (32 / G); q0 < nrows; q0 += nw * (32 / G)) {
+      const int q = q0 + sub;
+      const int n = q < nrows ? s.cnt[q] : 0;
+      const float bm = q < nrows ? s.bcov[q] : 0.f;
+      float* vals = Cimg + (size_t)(mlo + q) * N;
+      uint16_t* cols = Simg + (size_t)(mlo + q) * N;
       float bnew = bm;
-      if (n < 0) {
-        for (int t = lane; t < nb; t += 32) bnew = fmaxf(bnew, crow[s.batch[t]]);
-      } else {
-        for (int k = lane; k < n; k += 32) {
-          const int ps = s.poolslot[jrow[k]];
-          if (ps >= 0 && s.inb[ps]) bnew = fmaxf(bnew, crow[k]);
+      for (int k0 = gl; k0 < n; k0 += UNR * G) {
+        int cc[UNR];
+        float vv[UNR];
+#pragma unroll
+        for (int u = 0; u < UNR; ++u) {
+          const int k = k0 + u * G;
+          cc[u] = k < n ? (int)cols[k] : -1;
+          vv[u] = k < n ? vals[k] : 0.f;
+        }
+#pragma unroll
+        for (int u = 0; u < UNR; ++u) {
+          const int ps = cc[u] >= 0 ? s.poolslot[cc[u]] : -1;
+          if (ps >= 0 && s.inb[ps]) bnew = fmaxf(bnew, vv[u]);
         }
       }
-      bnew = warp_max(bnew);
+      bnew = group_max(bnew, gm);
       const long long fb_new = to_fix(bnew, fxs);
-      const int len = n < 0 ? N : n;
       int w = 0;
-      float rowmax = 0.f;
-      for (int base = 0; base < len; base += 32) {
-        const int k = base + lane;
-        float c = 0.f;
-        int j = 0;
-        if (k < len) {
-          c = crow[k];
-          j = n < 0 ? k : jrow[k];
+      for (int base = 0; base < n; base += UNR * G) {
+        float c[UNR];
+        int jj[UNR];
+#pragma unroll
+        for (int u = 0; u < UNR; ++u) {
+          const int k = base + u * G + gl;
+          c[u] = k < n ? vals[k] : 0.f;
+          jj[u] = k < n ? (int)cols[k] : 0;
         }
-        rowmax = fmaxf(rowmax, c);
-        const bool keep = k < len && c > bnew;
-        const unsigned msk = __ballot_sync(FULL, keep);
-        __syncwarp();  // every lane has read its entry before any lane overwrites one
-        if (keep) {
-          const int pos = w + __popc(msk & lanemask_lt());
-          crow[pos] = c;
-          jrow[pos] = (uint16_t)j;
-          atomicAdd((unsigned long long*)&s.u_part[j],
-                    (unsigned long long)(to_fix(c, fxs) - fb_new));
+        __syncwarp(gm);  // the group has read all UNR*G entries before any overwrite
+#pragma unroll
+        for (int u = 0; u < UNR; ++u) {
+          const int k = base + u * G + gl;
+          const bool keep = k < n && c[u] > bnew;
+          const unsigned msk = __ballot_sync(gm, keep);
+          if (keep) {
+            const int pos = w + __popc(msk & lt);
+            vals[pos] = c[u];
+            cols[pos] = (uint16_t)jj[u];
+            add_fix(&s.u_lo[jj[u]], &s.u_hi[jj[u]],
+                    (unsigned long long)(to_fix(c[u], fxs) - fb_new));
+          }
+          w += __popc(msk);
         }
-        w += __popc(msk);
       }
-      if (lane == 0) {
+      if (gl == 0 && q < nrows) {
         s.bcov[q] = bnew;
         s.cnt[q] = w;
       }
-      if (dense_round) {
-        rowmax = warp_max(rowmax);
-        if (lane == 0) {
-          const int bank = m < MG ? 0 : (m < MG + N ? 1 : 2);
-          atomicAdd((unsigned long long*)&s.fb[3 + bank], (unsigned long long)to_fix(rowmax, fxs));
-        }
-      }
+    }
     }
     __syncthreads();
     for (int k = threadIdx.x; k < Pt; k += blockDim.x) {
       s.poolslot[s.pool[k]] = -1;
       s.s_acc[k] = 0;
     }
+    if (!flat) migrate();
     S_count += nb;
     ++rnd;
     if (S_count >= K) break;
-    if (rnd >= rounds_max) {  // cannot happen (each round adds >= 1 token); guard the loop
-      if (threadIdx.x == 0) set_status(a.status, GMC_STATUS_INTERNAL);
-      break;
-    }
-    cluster.sync();  // B4: every CTA's gain partials are complete
+    cluster.sync();  // every CTA's gain partials are complete
 
-    // ---- E: reduce this CTA's token slice of the gains --------------------
+    // ---- gains of the next round: reduce this CTA's token slice, broadcast it ----
     for (int j = jlo + threadIdx.x; j < jhi; j += blockDim.x) {
       long long t = 0;
-      for (int c = 0; c < CS; ++c) t += cluster.map_shared_rank(s.u_part, c)[j];
-      s.u_slice[j - jlo] = t;
+      for (int c = 0; c < CS; ++c)
+        t += get_fix(cluster.map_shared_rank(s.u_lo, c) + j, cluster.map_shared_rank(s.u_hi, c) + j);
+      for (int c = 0; c < CS; ++c) cluster.map_shared_rank(s.u_full, c)[j] = t;
     }
-    // Only a block barrier: the next remote writes (candidates) target arrays
-    // nobody reads now, and u_part is reset only after B1.
-    __syncthreads();
+    cluster.sync();  // full gains everywhere; partials no longer read
+    for (int j = threadIdx.x; j < N; j += blockDim.x) {
+      s.u_lo[j] = 0;
+      s.u_hi[j] = 0;
+    }
   }
 
   // ---- final: coverage per bank, sorted support, trace ---------------------
@@ -434,13 +709,9 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
     if (f0) atomicAdd((unsigned long long*)&fb0[0], (unsigned long long)f0);
     if (f1) atomicAdd((unsigned long long*)&fb0[1], (unsigned long long)f1);
     if (f2) atomicAdd((unsigned long long*)&fb0[2], (unsigned long long)f2);
-    __syncthreads();
-    if (r != 0 && threadIdx.x < 3 && s.fb[3 + threadIdx.x])
-      atomicAdd((unsigned long long*)&fb0[3 + threadIdx.x], (unsigned long long)s.fb[3 + threadIdx.x]);
   }
   cluster.sync();
   if (r != 0) return;
-  // ascending support and slot map (one warp, ballot prefix over the flags)
   if (wid == 0) {
     int cnt = 0;
     for (int base = 0; base < N; base += 32) {
@@ -466,7 +737,7 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
       const double inv = ldexp(1.0, -e);
       for (int q = 0; q < 3; ++q) {
         hd->F_S[q] = (float)((double)s.fb[q] * inv);
-        hd->F_V[q] = (float)((double)s.fb[3 + q] * inv);
+        hd->F_V[q] = (float)((double)a.r0.fv[(size_t)b * 4 + q] * inv);
       }
       hd->c_B = -1.f;  // not computed by this build
     }
@@ -483,7 +754,7 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
 
 static int g_num_sms = 0;
 
-cudaError_t launch_select(int B, int N, int K, int M, const int32_t* toff, int H, int T, int L2,
+cudaError_t launch_select(const R0State& r0, int B, int N, int K, int M, const int32_t* toff, int H, int T, int L2,
                           const gmc_params& p, int fx_exp, const int32_t* fexp, float* C,
                           uint16_t* scol, const long long* u0, int32_t* order, int32_t* support,
                           int32_t* slot, int32_t* out_idx, uint32_t* status, const TraceView& tv,
@@ -513,12 +784,28 @@ cudaError_t launch_select(int B, int N, int K, int M, const int32_t* toff, int H
   a.order = order; a.support = support; a.slot = slot; a.out_idx = out_idx;
   a.status = status;
   a.tv = tv;
+  a.r0 = r0;
   int CS = 1;
   while (CS * 2 <= SEL_MAX_CS && (long long)B * CS * 2 <= g_num_sms) CS *= 2;
   for (; CS >= 1; CS /= 2) {
-    const int RPC = (M + CS - 1) / CS;
-    const size_t smem = sel_smem_bytes(N, CS, a.P, RPC, nullptr, nullptr);
-    if (smem > 227 * 1024) continue;
+    // Row capacity of one CTA: room for a balanced split that gives a CTA up to
+    // 2x its even share of rows while leaving space for 16K survivor entries;
+    // else the even share alone.
+    const int even = (M + CS - 1) / CS;
+    int RPC = 0;
+    size_t fixed = 0;
+    for (int f = 2; f >= 1; f /= 2) {
+      RPC = min(M, f * even);
+      fixed = sel_fixed_bytes(N, a.P, RPC, nullptr, nullptr);
+      if (fixed + 8 * 16384 + 16 <= SMEM_LIMIT || (f == 1 && fixed + 1024 <= SMEM_LIMIT)) break;
+      RPC = 0;
+    }
+    if (RPC == 0) continue;
+    a.rpc = RPC;
+    // the rest of the shared memory holds survivor entries (value, token, row: 8 bytes)
+    a.cap = (int)((SMEM_LIMIT - fixed - 16) / 8);
+    a.cap &= ~7;
+    const size_t smem = fixed + (size_t)a.cap * 8 + 16;
     if ((e = set_smem_limit((const void*)k_select, smem)) != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(B * CS);

@@ -44,6 +44,7 @@ struct Scratch {
   float* sigpart;    // [B][nP][H]     block partials of ||Z_h||_F^2
   float* sigma;      // [B][H]         mass coordinate sigma_h
   double* hgpart;    // [B][nHG][H*H]  block partials of the head-pattern Gram
+  double* HG;        // [B][H*H]       head-pattern Gram
   float* W2;         // [B][H][N]      sum_t nu_t A[h,t,i]^2
   float* omega;      // [B][H]
   float* ebar;       // [B][N]
@@ -80,7 +81,21 @@ cudaError_t launch_heads(const Dims&, const gmc_params&, Scratch&, const TraceVi
 cudaError_t launch_gram(const Dims&, const void* hidden, Scratch&, cudaStream_t);
 cudaError_t launch_build_clients(const Dims&, const gmc_params&, int fx_exp, Scratch&,
                                  cudaStream_t);
-cudaError_t launch_select(int B, int N, int K, int M, const int32_t* toff, int H, int T, int L2,
+// State left by the first (dense) selection round, run over the whole GPU.
+struct R0State {
+  int32_t* pool;   // [B][P]  first-round pool (-1 padded)
+  int32_t* info;   // [B][4]  pool size, batch size
+  long long* s0;   // [B][P]  first-round scores (fixed point)
+  long long* u1;   // [B][N]  second-round gains (fixed point)
+  float* bcov;     // [B][M]  coverage b_m after the first batch
+  int32_t* cnt;    // [B][M]  survivors per row (lists in place over Cbar / scol)
+  long long* fv;   // [B][4]  F_b(V) per bank (fixed point)
+};
+cudaError_t launch_round0(const R0State&, int B, int N, int K, int M, const int32_t* toff, int H,
+                          int T, int L2, const gmc_params&, int fx_exp, const int32_t* fexp,
+                          float* C, uint16_t* scol, const long long* u0, int32_t* order,
+                          uint32_t* status, const TraceView&, cudaStream_t);
+cudaError_t launch_select(const R0State&, int B, int N, int K, int M, const int32_t* toff, int H, int T, int L2,
                           const gmc_params&, int fx_exp, const int32_t* fexp_per_image, float* C,
                           uint16_t* scol, const long long* u0, int32_t* order, int32_t* support,
                           int32_t* slot, int32_t* out_idx, uint32_t* status, const TraceView&,
