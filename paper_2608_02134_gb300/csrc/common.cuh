@@ -67,6 +67,22 @@ __device__ __forceinline__ double from_fix(long long q, double inv_scale) {
   return (double)q * inv_scale;
 }
 
+// 4-byte asynchronous global -> shared copy; a false predicate writes zero
+// (source size 0, nothing is read from src).
+__device__ __forceinline__ void cp_async4(void* smem, const void* src, bool pred) {
+  const unsigned sa = (unsigned)__cvta_generic_to_shared(smem);
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(sa), "l"(src),
+               "r"(pred ? 4 : 0)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+template <int Pending>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(Pending) : "memory");
+}
+
 __device__ __forceinline__ void set_status(uint32_t* status, uint32_t bit) {
   if (status) atomicOr(status, bit);
 }

@@ -93,16 +93,19 @@ size_t carve_compress(const Dims& dm, Scratch* s, char* base, R0State* r0s = nul
   t.nP = ceil_div(dm.N, ROWS_PER_BLOCK);
   t.nHG = ceil_div(dm.N, HG_TOK);
   t.nA = ceil_div(dm.N, ASSIGN_WARPS);
+  t.nE = ceil_div(dm.N, ENERGY_THREADS);
   t.nSel = 0;
   t.status = c.take<uint32_t>(4);
   t.A = c.take<float>(B * H * T * N);
-  t.rs = c.take<float>(B * H * T);
+  t.nRS = message_splits(dm);
+  t.rs = c.take<float>(B * H * (size_t)t.nRS * T);
+  t.mpart = c.take<float2>(B * dm.Hkv * (size_t)message_rq(dm) * t.nRS);
   t.Z = c.take<float>(B * H * N * 4);
   t.zn2 = c.take<float>(B * H * N);
   t.sigpart = c.take<float>(B * t.nP * H);
   t.sigma = c.take<float>(B * H);
   t.hgpart = c.take<double>(B * t.nHG * H * H);
-  t.HG = c.take<double>(B * H * H);
+  t.HG = c.take<double>(B * (H * H + H));
   t.W2 = c.take<float>(B * H * N);
   t.omega = c.take<float>(B * H);
   t.ebar = c.take<float>(B * N);
@@ -117,6 +120,7 @@ size_t carve_compress(const Dims& dm, Scratch* s, char* base, R0State* r0s = nul
   t.order = c.take<int32_t>(B * K);
   t.delta = c.take<float>(B * N);
   t.dpart = c.take<double>(B * t.nA * 2);
+  t.epart = c.take<float>(B * t.nE);
   t.pi = c.take<int32_t>(B * N);
   t.mass = c.take<float>(B * N);
   t.selpart = nullptr;

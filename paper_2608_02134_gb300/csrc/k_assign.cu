@@ -70,7 +70,8 @@ __global__ void k_assign_gap(const float* __restrict__ cos, const int32_t* __res
 __global__ void k_assign_pick(const float* __restrict__ cos, const int32_t* __restrict__ support,
                               const int32_t* __restrict__ slot, const float* __restrict__ delta,
                               const double* __restrict__ dpart, int nA,
-                              const float* __restrict__ ebar, const int32_t* toff, int B, int N,
+                              const float* __restrict__ energy, const float* __restrict__ epart,
+                              int nE, const int32_t* toff, int B, int N,
                               int K, int Tmax, int gh, int gw, float gate_scale, float gate_pow,
                               float ambig_margin, float lambda_p, float tau_s, float alpha,
                               int32_t* pi, float* mass, TraceView tv, uint32_t* status) {
@@ -86,16 +87,19 @@ __global__ void k_assign_pick(const float* __restrict__ cos, const int32_t* __re
   }
   s = warp_sum(s);
   c = warp_sum(c);
-  const double dbar = c > 0.0 ? s / c : 0.0;
-  const double sxd = 1.0 - exp(-pow(dbar / gate_scale, (double)gate_pow));
-  const float sx = (float)sxd;
+  const float dbar = c > 0.0 ? (float)(s / c) : 0.f;
+  double et = 0.0;  // sum of the message energies, block sums in a fixed order
+  for (int q = lane; q < nE; q += 32) et += epart[(size_t)b * nE + q];
+  et = warp_sum(et);
+  const double emean = et / N;
+  const float sx = 1.f - expf(-powf(dbar / gate_scale, gate_pow));
   if (blockIdx.x == 0 && threadIdx.x == 0 && tv.base) {
     tv.header(b)->s_x = sx;
-    tv.header(b)->delta_bar = (float)dbar;
+    tv.header(b)->delta_bar = dbar;
   }
   const int i = blockIdx.x * ASSIGN_WARPS + w;
   if (i >= N) return;
-  const float eb = ebar[(size_t)b * N + i];
+  const float eb = emean > 0.0 ? (float)(energy[(size_t)b * N + i] / emean) : 1.f;
   const float m = (1.f - alpha * sx) + alpha * sx * eb;
   int choice = i;
   if (slot[(size_t)b * N + i] < 0) {
@@ -129,6 +133,7 @@ __global__ void k_assign_pick(const float* __restrict__ cos, const int32_t* __re
     if (tv.base) {
       tv.at<int32_t>(b, tv.off_pi)[i] = choice;
       tv.at<float>(b, tv.off_mass)[i] = m;
+      tv.at<float>(b, tv.off_ebar)[i] = eb;
     }
   }
 }
@@ -141,7 +146,8 @@ cudaError_t launch_assign(const Dims& dm, const gmc_params& p, Scratch& s, const
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   k_assign_pick<<<grid, 32 * ASSIGN_WARPS, 0, st>>>(
-      s.cos, s.support, s.slot, s.delta, s.dpart, s.nA, s.ebar, dm.toff, dm.B, dm.N, dm.K, dm.T,
+      s.cos, s.support, s.slot, s.delta, s.dpart, s.nA, s.ebar, s.epart, s.nE, dm.toff, dm.B,
+      dm.N, dm.K, dm.T,
       dm.gh, dm.gw, p.gate_scale, p.gate_pow, p.ambig_margin, p.assign_spatial_w, p.tau_s,
       p.pop_strength, s.pi, s.mass, tv, s.status);
   return cudaGetLastError();

@@ -22,7 +22,7 @@ struct RowInfo {
 };
 
 __global__ void __launch_bounds__(256) k_build_clients(
-    const float* __restrict__ A, const float* __restrict__ rs, const float* __restrict__ zn2,
+    const float* __restrict__ A, const float* __restrict__ rs, int nRS, const float* __restrict__ zn2,
     const float* __restrict__ sigma, const float* __restrict__ omega,
     const float* __restrict__ cos, const int32_t* toff, int B, int N, int Tmax, int H, int M,
     int gh, int gw, int L, float beta_G, float beta_V, float beta_S, float tau_v, float tau_s,
@@ -40,7 +40,8 @@ __global__ void __launch_bounds__(256) k_build_clients(
     RowInfo inf{-1, 0, 0, 0.f, 0.f};
     if (m < MG) {
       const int h = m / Tb, t = m % Tb;
-      const float rsv = rs[((size_t)b * H + h) * Tmax + t];
+      float rsv = 0.f;  // parts over key splits, fixed order
+      for (int q = 0; q < nRS; ++q) rsv += rs[(((size_t)b * H + h) * nRS + q) * Tmax + t];
       const float nu = (t == Tb - 1 ? wq : 1.f) / ((float)(Tb - 1) + wq);
       inf = RowInfo{0, h, t, rsv > 0.f ? beta_G * omega[(size_t)b * H + h] * nu / rsv : 0.f, 0.f};
     } else if (m < MG + N) {
@@ -105,7 +106,7 @@ cudaError_t launch_build_clients(const Dims& dm, const gmc_params& p, int fx_exp
                                  cudaStream_t st) {
   dim3 grid(ceil_div(dm.M, ROWS_PER_BLOCK), dm.B);
   k_build_clients<<<grid, 32 * ROWS_PER_BLOCK, 0, st>>>(
-      s.A, s.rs, s.zn2, s.sigma, s.omega, s.cos, dm.toff, dm.B, dm.N, dm.T, dm.H, dm.M, dm.gh,
+      s.A, s.rs, s.nRS, s.zn2, s.sigma, s.omega, s.cos, dm.toff, dm.B, dm.N, dm.T, dm.H, dm.M, dm.gh,
       dm.gw, dm.L, p.beta_G, p.beta_V, p.beta_S, p.tau_v, p.tau_s, p.terminal_q_weight,
       ldexpf(1.f, fx_exp), p.check_mode, s.C, s.u0, s.status);
   return cudaGetLastError();

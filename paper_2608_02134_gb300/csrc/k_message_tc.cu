@@ -3,14 +3,19 @@
 // For image b and key/value head g, the rows of the A operand are the text
 // queries of the query heads of group g, packed as (j, t) -> j*T_b + t, and the
 // B operand runs over the image's keys (N visual rows, then T_b text rows).
-// The CTA owns 128 query rows and walks every 128-key tile twice:
-//   pass 0: online softmax statistics (max, sum of exp) per query row over the
-//           keys it may see (all visual keys and text keys 0..t, scale 1/sqrt(d));
-//   pass 1: A[h,t,i] = exp(s_i - max) / sum for the visual keys i < N, and
-//           rs[h,t] = sum_i A[h,t,i] g_h(i) with g_h(i) = sqrt(||Z_h[i]||^2 + sigma_h^2).
+// A CTA owns 128 query rows and one split: a contiguous range of 128-key
+// tiles.  Two launches:
+//   statistics: online softmax statistics (max, sum of exp) per query row over
+//           the split's keys it may see (all visual keys and text keys 0..t,
+//           scale 1/sqrt(d)), written per split;
+//   write:  the splits' statistics merged in a fixed order, then for the
+//           split's visual keys i < N A[h,t,i] = exp(s_i - max) / sum, and the
+//           split's part of rs[h,t] = sum_i A[h,t,i] g_h(i) with
+//           g_h(i) = sqrt(||Z_h[i]||^2 + sigma_h^2).
 // Recomputing the logits costs one more small MMA pass and avoids writing and
-// re-reading raw scores.  This is appendix Eq. (cond-native-message): the
-// visual slice of the native causal softmax, not renormalised over the image.
+// re-reading raw scores; the splits put every SM to work on one image.  This
+// is appendix Eq. (cond-native-message): the visual slice of the native causal
+// softmax, not renormalised over the image.
 //
 // Roles: warp 8 / lane 0 loads the query tile once and streams key tiles with
 // TMA through a 4-stage ring; warp 9 / lane 0 issues tcgen05.mma into two
@@ -27,7 +32,8 @@ cudaError_t make_tmap_bf16(CUtensorMap* map, const void* base, uint64_t row_elem
                            uint64_t pitch_elems, uint32_t box_rows);
 
 namespace {
-constexpr int BM = 128, BK = 64, STAGES = 4;
+constexpr int BM = 128, BK = 64, STAGES = 2;
+constexpr int SPLIT_TARGET_CTAS = 152;  // one wave of one CTA per SM on a 152-SM GB300
 constexpr int TILE_BYTES = BM * BK * 2;
 constexpr int EPI_WARPS = 8, THREADS = 32 * (EPI_WARPS + 2);
 constexpr long long WAIT_CYCLES = 4000000000LL;
@@ -44,6 +50,21 @@ struct MsgCtl {
   float stat_l[2][BM];
   float rsum[2][BM];
 };
+
+struct MsgSplit {
+  int kt_per;  // key tiles per split
+  int n;       // splits
+};
+
+MsgSplit msg_split(int B, int Hkv, int RQ, int N, int T) {
+  const int nkt = (N + T + BM - 1) / BM;
+  const int base = (RQ / BM) * Hkv * B;
+  const int target = SPLIT_TARGET_CTAS / base > 1 ? SPLIT_TARGET_CTAS / base : 1;
+  MsgSplit sp;
+  sp.kt_per = (nkt + target - 1) / target;
+  sp.n = (nkt + sp.kt_per - 1) / sp.kt_per;
+  return sp;
+}
 
 size_t msg_smem_bytes(int nkb) {
   return 1024 + (size_t)nkb * TILE_BYTES * (1 + STAGES) + sizeof(MsgCtl);
@@ -83,6 +104,7 @@ __global__ void k_pack_q(const __nv_bfloat16* __restrict__ queries, const int32_
 __global__ void __launch_bounds__(THREADS, 1)
     k_message_tc(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
                  const int32_t* toff, int B, int N, int Tmax, int H, int Hkv, int d, int RQ,
+                 int mode, int kt_per, int nsplit, float2* part,
                  const float* __restrict__ zn2, const float* __restrict__ sigma, float* A,
                  float* rs, uint32_t* status) {
   extern __shared__ uint8_t sm_raw[];
@@ -93,14 +115,15 @@ __global__ void __launch_bounds__(THREADS, 1)
   uint8_t* Ks = base + (size_t)nkb * TILE_BYTES;
   MsgCtl* ctl = reinterpret_cast<MsgCtl*>(base + (size_t)nkb * TILE_BYTES * (1 + STAGES));
 
-  const int b = blockIdx.z, g = blockIdx.y, tile = blockIdx.x;
+  const int b = blockIdx.z / nsplit, split = blockIdx.z % nsplit, g = blockIdx.y, tile = blockIdx.x;
   const TextGeom tg = text_geom(toff, b, B, Tmax, status);
   const int grp = H / Hkv;
   if (tg.T == 0 || tile * BM >= grp * tg.T) return;  // uniform per CTA
   const int Tb = tg.T;
   const int nkeys = N + Tb;
   const int nkt = ceil_div(nkeys, BM);
-  const int iters = 2 * nkt;
+  const int c0 = split * kt_per, c1 = min(nkt, c0 + kt_per);
+  const int iters = max(0, c1 - c0);  // an image with fewer keys than the widest one
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int qrow0 = (int)(((size_t)b * Hkv + g) * RQ + (size_t)tile * BM);
   const int krow0 = (int)(2 * ((size_t)b * N + tg.off));
@@ -137,7 +160,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       for (int kb = 0; kb < nkb; ++kb)
         tc::tma_load_2d(Qs + kb * TILE_BYTES, &qmap, kb * BK, qrow0, &ctl->qfull);
       for (int it = 0; it < iters; ++it) {
-        const int s = it % STAGES, c = it % nkt;
+        const int s = it % STAGES, c = c0 + it;
         const uint32_t ph = (uint32_t)(it / STAGES) & 1u;
         if (it >= STAGES && !tc::mbar_wait(&ctl->empty[s], ph ^ 1u, deadline)) {
           ctl->abort = 1;
@@ -197,9 +220,20 @@ __global__ void __launch_bounds__(THREADS, 1)
     const float* zr = zn2 + ((size_t)b * H + h) * N;
     float* arow = A + (((size_t)b * H + h) * Tmax + t) * N;
     const int kvis = N + t + 1;                  // keys this query may see
+    float2* prow = part + ((((size_t)b * Hkv + g) * RQ) + (size_t)tile * BM + r) * nsplit;
     float m = -INFINITY, l = 0.f, rsum = 0.f, M = 0.f, invL = 0.f;
+    if (mode == 1 && valid) {  // merge the splits' statistics in a fixed order
+      M = -INFINITY;
+      for (int q = 0; q < nsplit; ++q) M = fmaxf(M, prow[q].x);
+      float L = 0.f;
+      for (int q = 0; q < nsplit; ++q) {
+        const float2 st = prow[q];
+        if (st.x > -INFINITY) L += st.y * expf(st.x - M);
+      }
+      invL = 1.f / L;
+    }
     for (int it = 0; it < iters; ++it) {
-      const int buf = it & 1, c = it % nkt;
+      const int buf = it & 1, c = c0 + it;
       bool ok = tc::mbar_wait(&ctl->accf[buf], (uint32_t)(it >> 1) & 1u, deadline);
       ok = __all_sync(FULL, ok && !ctl->abort);
       float v[64];
@@ -212,12 +246,9 @@ __global__ void __launch_bounds__(THREADS, 1)
       tc::fence_before_sync();
       __syncwarp();
       if (lane == 0) mbar_arrive(&ctl->acce[buf]);
-      if (!ok) {
-        if (it == nkt - 1) epi_barrier();
-        continue;
-      }
+      if (!ok) continue;
       const int k0 = c * BM + half * 64;
-      if (it < nkt) {  // pass 0: running max / sum over the visible keys
+      if (mode == 0) {  // running max / sum over the visible keys
         float mt = -INFINITY;
 #pragma unroll
         for (int q = 0; q < 64; ++q) {
@@ -233,17 +264,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           l = acc;
           m = mn;
         }
-        if (it == nkt - 1) {  // combine the two column halves of every row
-          ctl->stat_m[half][r] = m;
-          ctl->stat_l[half][r] = l;
-          epi_barrier();
-          const float mo = ctl->stat_m[half ^ 1][r], lo = ctl->stat_l[half ^ 1][r];
-          M = fmaxf(m, mo);
-          const float L = (m > -INFINITY ? l * expf(m - M) : 0.f) +
-                          (mo > -INFINITY ? lo * expf(mo - M) : 0.f);
-          invL = 1.f / L;
-        }
-      } else if (valid && k0 < N) {  // pass 1: normalised visual columns
+      } else if (valid && k0 < N) {  // normalised visual columns
         const int nv = min(64, N - k0);
         if (nv == 64 && (N & 3) == 0) {
 #pragma unroll
@@ -269,10 +290,24 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
       }
     }
-    ctl->rsum[half][r] = rsum;
-    epi_barrier();
-    if (half == 0 && valid && !ctl->abort)
-      rs[((size_t)b * H + h) * Tmax + t] = rsum + ctl->rsum[1][r];
+    if (mode == 0) {  // combine the two column halves of every row
+      ctl->stat_m[half][r] = m;
+      ctl->stat_l[half][r] = l;
+      epi_barrier();
+      if (half == 0 && !ctl->abort) {
+        const float mo = ctl->stat_m[1][r], lo = ctl->stat_l[1][r];
+        const float Mc = fmaxf(m, mo);
+        const float Lc = Mc > -INFINITY ? (m > -INFINITY ? l * expf(m - Mc) : 0.f) +
+                                              (mo > -INFINITY ? lo * expf(mo - Mc) : 0.f)
+                                        : 0.f;
+        prow[split] = make_float2(Mc, Lc);
+      }
+    } else {
+      ctl->rsum[half][r] = rsum;
+      epi_barrier();
+      if (half == 0 && valid && !ctl->abort)
+        rs[(((size_t)b * H + h) * nsplit + split) * Tmax + t] = rsum + ctl->rsum[1][r];
+    }
   }
   if (threadIdx.x == 0 && ctl->abort) set_status(status, GMC_STATUS_TIMEOUT);
   tc::fence_before_sync();
@@ -285,6 +320,10 @@ bool message_tc_supported(const Dims& dm) {
 }
 
 int message_rq(const Dims& dm) { return ceil_div((dm.H / dm.Hkv) * dm.T, BM) * BM; }
+
+int message_splits(const Dims& dm) {
+  return message_tc_supported(dm) ? msg_split(dm.B, dm.Hkv, message_rq(dm), dm.N, dm.T).n : 1;
+}
 
 cudaError_t launch_message_tc(const Dims& dm, const void* keys, const void* queries, Scratch& s,
                               cudaStream_t st) {
@@ -306,10 +345,15 @@ cudaError_t launch_message_tc(const Dims& dm, const void* keys, const void* quer
   const int nkb = dm.d / BK;
   const size_t smem = msg_smem_bytes(nkb);
   if ((e = set_smem_limit((const void*)k_message_tc, smem)) != cudaSuccess) return e;
-  dim3 grid(RQ / BM, dm.Hkv, dm.B);
-  k_message_tc<<<grid, THREADS, smem, st>>>(qmap, kmap, dm.toff, dm.B, dm.N, dm.T, dm.H, dm.Hkv,
-                                            dm.d, RQ, s.zn2, s.sigma, s.A, s.rs, s.status);
-  return cudaGetLastError();
+  const MsgSplit sp = msg_split(dm.B, dm.Hkv, RQ, dm.N, dm.T);
+  dim3 grid(RQ / BM, dm.Hkv, dm.B * sp.n);
+  for (int mode = 0; mode < 2; ++mode) {
+    k_message_tc<<<grid, THREADS, smem, st>>>(qmap, kmap, dm.toff, dm.B, dm.N, dm.T, dm.H, dm.Hkv,
+                                              dm.d, RQ, mode, sp.kt_per, sp.n, s.mpart, s.zn2,
+                                              s.sigma, s.A, s.rs, s.status);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  }
+  return cudaSuccess;
 }
 
 }  // namespace gmc

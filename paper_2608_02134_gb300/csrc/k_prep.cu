@@ -5,9 +5,11 @@
 
 namespace gmc {
 
-// ||h_i|| in fp64 for every visual row: x_i = h_i / max(||h_i||, eps) (appendix
+// ||h_i|| for every visual row: x_i = h_i / max(||h_i||, eps) (appendix
 // "Population assignment and transport") and rms(h_i) = ||h_i|| / sqrt(D) for the
-// RMS restoration R_j of Eq. (5).  One warp per row, 16-byte loads.
+// RMS restoration R_j of Eq. (5).  One warp per row, 16-byte loads; each lane
+// sums D / 32 squares in fp32 (relative error ~1e-6 at D = 4096), the warp tree
+// adds the lane sums.
 template <typename Tin>
 __global__ void k_rownorm(const Tin* __restrict__ hidden, const int32_t* toff, int B, int N,
                           int K, int Tmax, int D, float norm_eps, float* rn, float* rmsh,
@@ -21,21 +23,21 @@ __global__ void k_rownorm(const Tin* __restrict__ hidden, const int32_t* toff, i
   const SeqIdx sq(b, N, K, tg.off, tg.T);
   const Tin* row = hidden + sq.hidden_row(i, D);
   constexpr int V = 16 / sizeof(Tin);
-  double acc = 0.0;
+  float acc = 0.f;
   for (int k = lane * V; k < D; k += 32 * V) {
     uint4 raw = *reinterpret_cast<const uint4*>(row + k);
     const Tin* e = reinterpret_cast<const Tin*>(&raw);
 #pragma unroll
     for (int v = 0; v < V; ++v) {
-      float x = to_f32(e[v]);
-      acc += (double)x * x;
+      const float x = to_f32(e[v]);
+      acc = fmaf(x, x, acc);
     }
   }
   acc = warp_sum(acc);
   if (lane == 0) {
-    double n = sqrt(acc);
-    if (rn) rn[(size_t)b * N + i] = (float)(1.0 / fmax(n, (double)norm_eps));
-    rmsh[(size_t)b * N + i] = (float)sqrt(acc / D);
+    const float n = sqrtf(acc);
+    if (rn) rn[(size_t)b * N + i] = 1.f / fmaxf(n, norm_eps);
+    rmsh[(size_t)b * N + i] = sqrtf(acc / (float)D);
   }
 }
 

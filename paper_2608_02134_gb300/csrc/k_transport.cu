@@ -16,6 +16,7 @@
 namespace gmc {
 
 constexpr int TR_VEC = 8;  // elements per thread per row
+constexpr int TR_ILP = 4;  // member rows in flight per thread
 
 template <typename Tin> struct Vec8;
 template <> struct Vec8<__nv_bfloat16> {
@@ -70,7 +71,7 @@ __global__ void __launch_bounds__(1024) k_transport(
   float acc[TR_VEC];
 #pragma unroll
   for (int q = 0; q < TR_VEC; ++q) acc[q] = 0.f;
-  double Msum = 0.0;
+  float Msum = 0.f;
   for (int base = 0; base < N; base += blockDim.x) {
     const int i = base + threadIdx.x;
     const bool mine = i < N && pi[(size_t)b * N + i] == j;
@@ -88,27 +89,38 @@ __global__ void __launch_bounds__(1024) k_transport(
       members[before + __popc(bal & lt)] = i;
     }
     __syncthreads();
-    for (int q = 0; q < total; ++q) {  // ascending source order
-      const int src = members[q];
-      const float wgt = mass[(size_t)b * N + src];
-      Msum += wgt;
-      if (active) {
-        float v[TR_VEC];
-        Vec8<Tin>::load(hidden + sq.hidden_row(src, D) + e0, v);
+    // ascending source order; TR_ILP member rows are loaded before any is added
+    for (int q0 = 0; q0 < total; q0 += TR_ILP) {
+      float v[TR_ILP][TR_VEC], wg[TR_ILP];
 #pragma unroll
-        for (int t = 0; t < TR_VEC; ++t) acc[t] = fmaf(wgt, v[t], acc[t]);
+      for (int u = 0; u < TR_ILP; ++u) {
+        wg[u] = 0.f;
+        if (q0 + u < total) {
+          const int src = members[q0 + u];
+          wg[u] = mass[(size_t)b * N + src];
+          if (active) Vec8<Tin>::load(hidden + sq.hidden_row(src, D) + e0, v[u]);
+        }
       }
+#pragma unroll
+      for (int u = 0; u < TR_ILP; ++u)
+        if (q0 + u < total) {
+          Msum += wg[u];
+          if (active) {
+#pragma unroll
+            for (int t = 0; t < TR_VEC; ++t) acc[t] = fmaf(wg[u], v[u][t], acc[t]);
+          }
+        }
     }
     __syncthreads();
   }
-  const float invM = (float)(1.0 / Msum);
-  double ss = 0.0;
+  const float invM = 1.f / Msum;
+  float ssf = 0.f;
 #pragma unroll
   for (int t = 0; t < TR_VEC; ++t) {
     acc[t] *= invM;
-    if (active) ss += (double)acc[t] * acc[t];
+    if (active) ssf = fmaf(acc[t], acc[t], ssf);
   }
-  ss = block_reduce(ss, red, OpAdd(), 0.0);
+  const double ss = block_reduce((double)ssf, red, OpAdd(), 0.0);
   const float rc = (float)sqrt(ss / D);
   const float scale = rmsh[(size_t)b * N + j] / (rc + rms_eps);
   if (active) {

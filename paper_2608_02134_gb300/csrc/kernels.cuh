@@ -38,16 +38,17 @@ struct TraceView {
 struct Scratch {
   uint32_t* status;
   float* A;          // [B][H][T][N]   native attention slice (visual columns)
-  float* rs;         // [B][H][T]      sum_i ||u_i^{h,t}|| (0: inactive row)
+  float* rs;         // [B][H][nRS][T] parts of sum_i ||u_i^{h,t}|| over key splits (sum: 0 = inactive row)
+  float2* mpart;     // [B][Hkv][RQ][nRS] per-split softmax (max, sum) of the packed query rows
   float* Z;          // [B][H][N][4]   probe values Z_h[i]
   float* zn2;        // [B][H][N]      ||Z_h[i]||^2
   float* sigpart;    // [B][nP][H]     block partials of ||Z_h||_F^2
   float* sigma;      // [B][H]         mass coordinate sigma_h
   double* hgpart;    // [B][nHG][H*H]  block partials of the head-pattern Gram
-  double* HG;        // [B][H*H]       head-pattern Gram
+  double* HG;        // [B][H*H + H]   head-pattern Gram, then sum_t rs[h,t] per head
   float* W2;         // [B][H][N]      sum_t nu_t A[h,t,i]^2
   float* omega;      // [B][H]
-  float* ebar;       // [B][N]
+  float* ebar;       // [B][N]  message energy e_i (the assignment divides by its mean)
   float* rn;         // [B][N]         1 / max(||h_i||, eps)
   float* rmsh;       // [B][N]         rms(h_i)
   float* cos;        // [B][N][N]      cosine of boundary states
@@ -59,17 +60,19 @@ struct Scratch {
   int32_t* order;    // [B][K]         selection order
   float* delta;      // [B][N]
   double* dpart;     // [B][nA][2]     partial sums of delta and counts over discarded tokens
+  float* epart;      // [B][nE]        block sums of the message energies e_i
   int32_t* pi;       // [B][N]
   float* mass;       // [B][N]
   double* selpart;   // [B][64]        select-path total mass partials
   int32_t* fexp;     // [B]            select-path fixed-point exponents
   __nv_bfloat16* Qp; // [B][Hkv][RQ][d] packed text queries of each KV group (tcgen05 path)
-  int nP, nHG, nA, nSel;
+  int nP, nHG, nA, nSel, nE, nRS;
 };
 
 constexpr int ROWS_PER_BLOCK = 8;  // rownorm / probe / client builder blocks
 constexpr int HG_TOK = 8;          // tokens per head-statistics block
 constexpr int ASSIGN_WARPS = 8;    // tokens per assignment block
+constexpr int ENERGY_THREADS = 256;  // tokens per block of the message-energy kernel
 
 // Launch wrappers.  Each returns the first CUDA error it saw.
 cudaError_t launch_rownorm(const Dims&, const void* hidden, float norm_eps, Scratch&, cudaStream_t);
@@ -150,4 +153,5 @@ cudaError_t launch_message_tc(const Dims&, const void* keys, const void* queries
                               cudaStream_t);
 bool message_tc_supported(const Dims&);
 int message_rq(const Dims&);  // packed query rows per (image, KV group)
+int message_splits(const Dims&);  // key splits of the message slice (parts of rs)
 }  // namespace gmc
