@@ -60,8 +60,23 @@ struct OpMax { __device__ float operator()(float a, float b) const { return fmax
 // 64-bit integer.  Integer sums do not depend on the order of the additions,
 // so every gain / score reduction below is deterministic however the threads
 // are scheduled, and exact for terms >= 2^-(e-24).
+// x * 2^e rounded to the nearest integer (ties to even), for 0 <= x * 2^e < 2^63
+// (every caller converts a non-negative value).  A 64-bit float-to-integer
+// conversion runs on the narrow fp64 pipe of this GPU, so the value is split
+// into two 32-bit conversions: v = x * 2^e is exact (power-of-two scale),
+// hi = floor(v / 2^32) and lo = v - hi 2^32 are exact floats (v >= 2^32 makes v
+// a multiple of 2^9), and only lo can carry a fraction.
 __device__ __forceinline__ long long to_fix(float x, float scale) {
-  return __float2ll_rn(x * scale);  // x * 2^e is exact in fp32 (power-of-two scale)
+  const float v = x * scale;
+  const float hi = floorf(v * 2.3283064365386963e-10f);  // 2^-32
+  const float lo = fmaf(hi, -4294967296.f, v);             // exact
+  return (long long)(((unsigned long long)__float2uint_rz(hi) << 32) + __float2uint_rn(lo));
+}
+
+// A non-negative 64-bit fixed-point integer as fp32 (within one ulp; the same
+// on every call) without the fp64-pipe conversion.
+__device__ __forceinline__ float fix_to_float(unsigned long long q) {
+  return fmaf(__uint2float_rn((unsigned)(q >> 32)), 4294967296.f, __uint2float_rn((unsigned)q));
 }
 __device__ __forceinline__ double from_fix(long long q, double inv_scale) {
   return (double)q * inv_scale;

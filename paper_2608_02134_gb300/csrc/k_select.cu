@@ -56,6 +56,7 @@ constexpr int UNR = 4;     // entries in flight per lane in a sweep
 constexpr int PCL = 8;     // pool entries a lane keeps in registers (8 lanes x 8 >= pool of 64)
 constexpr int DEADROW = 0xFFFF;  // flat mode: row id of an entry whose residual is zero
 constexpr int FU = 4;      // flat mode: entries a thread loads ahead in a walk
+constexpr int CU = 8;      // flat mode: entries a thread moves per compaction chunk
 constexpr size_t SMEM_LIMIT = 227 * 1024;
 
 struct SelArgs {
@@ -428,8 +429,8 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
           const int q = s.srows[p];
           if (q == DEADROW) continue;
           const float tau = a.resp_temp * __int_as_float(s.rmaxb[q]) + a.resp_eps;
-          atomicAdd(&s.z64[q], (unsigned long long)__float2ll_rn(
-                                   expf((s.svals[p] - s.bcov[q]) / tau) * z_one));
+          atomicAdd(&s.z64[q],
+                    (unsigned long long)to_fix(expf((s.svals[p] - s.bcov[q]) / tau), z_one));
         }
       }
       __syncthreads();
@@ -441,7 +442,7 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
           const int q = s.srows[p];
           if (q == DEADROW) continue;
           const float tau = a.resp_temp * __int_as_float(s.rmaxb[q]) + a.resp_eps;
-          const float z = (float)s.z64[q] * z_inv + (float)(Pt - s.npl[q]);
+          const float z = fix_to_float(s.z64[q]) * z_inv + (float)(Pt - s.npl[q]);
           const float R = s.svals[p] - s.bcov[q];
           acc += (unsigned long long)to_fix(expf(R / tau) / z * R, fxs);
         }
@@ -580,6 +581,7 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
         s.npl[q] = 0;
         s.z64[q] = 0;
       }
+      for (int j = threadIdx.x; j < N; j += blockDim.x) s.bnd[j] = 0;  // live entries per token
       __syncthreads();
       // survivor filter (dead entries marked in place) and next-round gains: each
       // thread walks a contiguous slice (an odd length keeps a warp's threads on
@@ -587,7 +589,7 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
       const int tot = s.scal[SC_CURSOR];
       const int per = ((tot + SEL_THREADS - 1) / SEL_THREADS) | 1;
       const int p0s = min(tot, (int)threadIdx.x * per), p1s = min(tot, p0s + per);
-      int jc = -1;
+      int jc = -1, nj = 0, mylive = 0;
       unsigned long long acc = 0;
       for (int p0 = p0s; p0 < p1s; p0 += FU) {
         int qq[FU], jj[FU];
@@ -605,16 +607,70 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
           if (cc[u] > s.bcov[qq[u]]) {
             if (jj[u] != jc) {
               if (acc) add_fix(&s.u_lo[jc], &s.u_hi[jc], acc);
+              if (nj) atomicAdd(&s.bnd[jc], nj);
               jc = jj[u];
               acc = 0;
+              nj = 0;
             }
             acc += (unsigned long long)(to_fix(cc[u], fxs) - s.bfix[qq[u]]);
+            ++nj;
+            ++mylive;
           } else {
             s.srows[p0 + u] = (uint16_t)DEADROW;
           }
         }
       }
       if (acc) add_fix(&s.u_lo[jc], &s.u_hi[jc], acc);
+      if (nj) atomicAdd(&s.bnd[jc], nj);
+      // Once fewer than 60% of the entries are live, drop the dead ones: the
+      // live entries move down in order (token-major order is kept) and the
+      // token segments restart at the prefix sums of the live counts.
+      int live = 0;
+      block_exclusive_scan(mylive, s.wsum, &live);
+      if (live * 5 < tot * 3) {
+        {
+          const int perj = (N + SEL_THREADS - 1) / SEL_THREADS;
+          const int j0 = min(N, (int)threadIdx.x * perj), j1 = min(N, j0 + perj);
+          int c = 0;
+          for (int j = j0; j < j1; ++j) c += s.bnd[j];
+          int at = block_exclusive_scan(c, s.wsum, nullptr);
+          for (int j = j0; j < j1; ++j) {
+            s.cstart[j] = at;
+            at += s.bnd[j];
+          }
+          if (threadIdx.x == 0) s.cstart[N] = live;
+        }
+        // chunks of CU entries per thread: every thread reads its chunk before the
+        // scan's barriers and writes after them, always at or below the source
+        int dst = 0;
+        for (int base = 0; base < tot; base += SEL_THREADS * CU) {
+          const int p0 = base + threadIdx.x * CU;
+          uint16_t mq[CU], mj[CU];
+          float mc[CU];
+          unsigned m = 0;
+#pragma unroll
+          for (int u = 0; u < CU; ++u) {
+            const bool in = p0 + u < tot;
+            mq[u] = in ? s.srows[p0 + u] : (uint16_t)DEADROW;
+            mj[u] = in ? s.scols[p0 + u] : (uint16_t)0;
+            mc[u] = in ? s.svals[p0 + u] : 0.f;
+            m |= (unsigned)(mq[u] != DEADROW) << u;
+          }
+          int chunk_live = 0;
+          const int ex = dst + block_exclusive_scan(__popc(m), s.wsum, &chunk_live);
+#pragma unroll
+          for (int u = 0; u < CU; ++u)
+            if ((m >> u) & 1u) {
+              const int d = ex + __popc(m & ((1u << u) - 1u));
+              s.srows[d] = mq[u];
+              s.scols[d] = mj[u];
+              s.svals[d] = mc[u];
+            }
+          dst += chunk_live;
+        }
+        __syncthreads();
+        if (threadIdx.x == 0) s.scal[SC_CURSOR] = dst;
+      }
     }
     if (!flat) {
     for (int q0 = wid * (32 / G); q0 < nrows; q0 += nw * (32 / G)) {
