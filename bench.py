@@ -55,20 +55,23 @@ def workload_config(wl) -> dict:
 # ---------------------------------------------------------------------------
 # oracle timing (runs in a child process with a fixed BLAS thread count)
 # ---------------------------------------------------------------------------
-def oracle_sample(name: str, n: int) -> dict:
+def oracle_sample(name: str, n: int, min_seconds: float = 10.0) -> dict:
+    """Oracle boundaries of the workload until min_seconds of CPU work (at most n)."""
     import numpy as np
     from oracle import gmc_oracle as O
     from paper_2608_02134_gb300 import workloads
     wl = workloads.make(name)
     f = lambda a: np.asarray(a, dtype=np.float64)
     t = 0.0
-    for k in range(n):
+    k = 0
+    while k < n and (k == 0 or t < min_seconds):
         im = wl.image(k % wl.B)
         t0 = time.perf_counter()
         O.compress(f(im.hidden), f(im.keys), f(im.values), f(im.queries), im.pos, f(wl.probe()),
                    wl.gh, wl.gw, wl.K)
         t += time.perf_counter() - t0
-    return {"seconds": t, "boundaries": n}
+        k += 1
+    return {"seconds": t, "boundaries": k}
 
 
 def run_oracle_child(name: str, n: int, cores: int) -> dict:
@@ -153,7 +156,11 @@ def stage_work(wl) -> dict:
     w["gram"] = ("tensor", B * 2.0 * N * N * D)                        # the N x N cosine block
     w["message"] = ("hbm", B * (H * Tm * N * 4 + 2 * (N + Tm) * Hkv * d * es + Tm * H * d * es))
     w["clients"] = ("hbm", B * (M * N * 4 + H * Tm * N * 4 + N * N * 4))
-    w["select"] = ("hbm", B * (M * N * 4.0))                            # one read of the clients
+    # selection: one read of the M x N clients per round; the dense first round
+    # is its own stage, the rounds after it are k_select's
+    rounds = -(-K // 16)
+    w["round0"] = ("hbm", B * (M * N * 4.0))
+    w["select"] = ("hbm", B * (rounds - 1) * (M * N * 4.0))
     w["transport"] = ("hbm", B * ((N + Tm) * D * es + (K + Tm) * D * es
                                   + 2 * (K + Tm) * 2 * Hkv * d * es + 2 * 3 * (K + Tm) * 4 + 3 * N * 4))
     w["heads"] = ("hbm", B * (H * Tm * N * 4))
@@ -161,6 +168,31 @@ def stage_work(wl) -> dict:
     w["probe"] = ("hbm", B * N * Hkv * d * es)
     w["rownorm"] = ("hbm", B * N * D * es)
     return w
+
+
+# DRAM bytes per launch from an ncu capture (profiles/dram_traffic_qwen.txt); a
+# line counts only while the sha256 of its kernel's source files is unchanged.
+def recorded_traffic(stage: str):
+    import hashlib
+    path = os.path.join(ROOT, "profiles", "dram_traffic_qwen.txt")
+    try:
+        lines = open(path).read().splitlines()
+    except OSError:
+        return None
+    for ln in lines:
+        f = dict(kv.split("=", 1) for kv in ln.split() if "=" in kv)
+        if f.get("stage") != stage:
+            continue
+        h = hashlib.sha256()
+        for src in f.get("files", "").split(","):
+            try:
+                h.update(open(os.path.join(ROOT, "paper_2608_02134_gb300", "csrc", src), "rb").read())
+            except OSError:
+                return None
+        if h.hexdigest()[:16] != f.get("sha"):
+            return None
+        return int(f["dram_bytes"])
+    return None
 
 
 def peaks() -> dict:
@@ -181,9 +213,9 @@ def run_gmc(args):
 
     from paper_2608_02134_gb300 import gmc, workloads
 
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
+    from paper_2608_02134_gb300 import replicas
+
+    rank, world, local = replicas.rank_info()
     if world > 1:
         torch.cuda.set_device(local)
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
@@ -236,12 +268,8 @@ def run_gmc(args):
         torch.cuda.synchronize(dev)
     barrier()
     launches = gmc.launch_count() - launches0
-    ms = sum(a.elapsed_time(b) for a, b in evs) / args.steps
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
-    value = world * wl.B * 1000.0 / ms
+    ms = replicas.max_over_ranks(sum(a.elapsed_time(b) for a, b in evs) / args.steps, dev)
+    value = replicas.job_rate(world, wl.B, ms)
 
     # ---- per-stage profile (separate pass, events on the same stream) --------
     gmc.profile_enable(True)
@@ -279,11 +307,7 @@ def run_gmc(args):
         b.record(stream)
     torch.cuda.synchronize(dev)
     barrier()
-    e2e_ms = sum(a.elapsed_time(b) for a, b in eev) / e2e_steps
-    if world > 1:
-        t = torch.tensor([e2e_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t.item())
+    e2e_ms = replicas.max_over_ranks(sum(a.elapsed_time(b) for a, b in eev) / e2e_steps, dev)
 
     if rank != 0:
         if world > 1:
@@ -294,27 +318,32 @@ def run_gmc(args):
     pk = peaks()
     work = stage_work(wl)
     dom = max(prof, key=prof.get) if prof else None
-    roof = None
-    if dom:
-        bound, amount = work[dom]
-        sec = prof[dom] / 1e3
+
+    def roofline(stage):
+        bound, amount = work[stage]
+        sec = prof[stage] / 1e3
         if bound == "tensor":
             ach, peak, unit = amount / sec / 1e12, pk["bf16_tflops"], "TFLOP/s"
         else:
             ach, peak, unit = amount / sec / 1e9, pk["hbm_gbs"], "GB/s"
-        roof = {"kernel": dom, "bound": bound, "achieved": round(ach, 3), "peak": peak, "unit": unit,
-                "frac": round(ach / peak, 5), "peak_source": pk["source"], "traffic": None,
-                "algorithmic": amount, "ms": round(prof[dom], 5)}
+        return {"kernel": stage, "bound": bound, "achieved": round(ach, 3), "peak": peak,
+                "unit": unit, "frac": round(ach / peak, 5), "peak_source": pk["source"],
+                "traffic": recorded_traffic(stage) if wl.name == "qwen" else None,
+                "algorithmic": amount, "ms": round(prof[stage], 5)}
+
+    roof = roofline(dom) if dom else None
+    stage_roofs = {k: {f: v for f, v in roofline(k).items() if f in ("bound", "achieved", "unit", "frac", "traffic")}
+                   for k in prof if k in work}
 
     cpu = None
     if not args.no_cpu_baseline:
         cores = os.cpu_count() or 1
         try:
-            o = run_oracle_child(args.workload, 1, cores)
+            o = run_oracle_child(args.workload, 64, cores)
             cpu = {"value": round(o["boundaries"] / o["seconds"], 6), "unit": UNIT, "cores": cores,
                    "kind": "oracle",
-                   "sample": f"{o['boundaries']} boundary of the {args.workload} workload, fp64 numpy, "
-                             f"{o['seconds']:.2f} s"}
+                   "sample": f"{o['boundaries']} boundaries of the {args.workload} workload (about 10 s "
+                             f"of CPU work: {o['seconds']:.2f} s), fp64 numpy oracle"}
         except Exception as e:  # keep the GPU line even if the host run fails
             cpu = {"value": None, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": f"failed: {e}"}
 
@@ -325,10 +354,11 @@ def run_gmc(args):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "bf16" if wl.dtype == "bf16" else "f32", "data": "synthetic",
         "config": workload_config(wl) | {"parallelism": f"replicas x{world}"},
-        "e2e": {"value": round(world * wl.B * 1000.0 / e2e_ms, 3), "unit": UNIT,
+        "e2e": {"value": round(replicas.job_rate(world, wl.B, e2e_ms), 3), "unit": UNIT,
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": round(e2e_ms, 5)},
         "gpu_launches": int(launches),
         "roofline": roof,
+        "stage_roofline": stage_roofs,
         "stages_ms": {k: round(v, 5) for k, v in prof.items()},
         "clocks": clk.summary(),
         "cpu_baseline": cpu,

@@ -357,17 +357,17 @@ int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* 
   GMC_TRY(g_prof.begin(st));
   GMC_STAGE("rownorm", 1, launch_rownorm(dm, hidden, p.norm_eps, s, st));
   GMC_STAGE("probe", 2, launch_probe(dm, keys, vo_probe, p, s, st));
-  GMC_STAGE("message", message_tc_supported(dm) ? 2 : 1, launch_message(dm, keys, queries, s, st));
+  GMC_STAGE("message", message_tc_supported(dm) ? 3 : 1, launch_message(dm, keys, queries, s, st));
   GMC_STAGE("heads", 4, launch_heads(dm, p, s, tv, st));
   GMC_STAGE("gram", 1, launch_gram(dm, hidden, s, st));
   GMC_STAGE("clients", 1, launch_build_clients(dm, p, fx, s, st));
-  GMC_STAGE("select", 4,
+  GMC_STAGE("round0", 3,
             launch_round0(r0, dm.B, N, Ke, dm.M, dm.toff, H, T, p.landmarks * p.landmarks, p, fx,
-                          nullptr, s.C, s.scol, s.u0, s.order, s.status, tv, st) != cudaSuccess
-                ? cudaErrorLaunchFailure
-                : launch_select(r0, dm.B, N, Ke, dm.M, dm.toff, H, T, p.landmarks * p.landmarks,
-                                p, fx, nullptr, s.C, s.scol, s.u0, s.order, s.support, s.slot,
-                                nullptr, s.status, tv, st));
+                          nullptr, s.C, s.scol, s.u0, s.order, s.status, tv, st));
+  GMC_STAGE("select", 1,
+            launch_select(r0, dm.B, N, Ke, dm.M, dm.toff, H, T, p.landmarks * p.landmarks, p, fx,
+                          nullptr, s.C, s.scol, s.u0, s.order, s.support, s.slot, nullptr, s.status,
+                          tv, st));
   GMC_STAGE("assign", 2, launch_assign(dm, p, s, tv, st));
   GMC_STAGE("transport", 2,
             launch_transport(dm, p, hidden, keys, pos_ids, s.support, s.pi, s.mass, s.rmsh,
