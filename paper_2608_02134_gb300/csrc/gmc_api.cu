@@ -369,7 +369,7 @@ int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* 
                           nullptr, s.C, s.scol, s.u0, s.order, s.support, s.slot, nullptr, s.status,
                           tv, st));
   GMC_STAGE("assign", 2, launch_assign(dm, p, s, tv, st));
-  GMC_STAGE("transport", 2,
+  GMC_STAGE("transport", 1,
             launch_transport(dm, p, hidden, keys, pos_ids, s.support, s.pi, s.mass, s.rmsh,
                              out_idx, out_hidden, out_kv, out_pos, s.status, st));
   g_prof.valid = g_prof.on;

@@ -6,17 +6,25 @@
 // is normalised afterwards in fp32 (the states are never rounded after
 // normalisation).
 //
-// One CTA computes one 128 x 128 tile of the upper triangle (I <= J) and writes
-// it and its mirror.  Warp 0 / lane 0 streams 64-wide K slices of both row
+// A cluster of two CTAs computes one 128 x 128 tile of the upper triangle
+// (I <= J) and writes it and its mirror; the CTAs split the contraction over
+// D in two halves (one SM streams half the operand bytes, twice as many SMs
+// work).  In each CTA warp 0 / lane 0 streams 64-wide K slices of both row
 // blocks with TMA (128-byte swizzle) through a 6-stage mbarrier ring; warp 1 /
 // lane 0 issues tcgen05.mma (M = N = 128, K = 16) into a 128-column TMEM
-// accumulator; all four warps then read their 32 TMEM lanes and store.  The
-// last, ragged tile of an image is shifted inward (start N - 128) so every TMA
-// box lies inside the image's own rows; it stores only the rows and columns
-// the previous tile does not own.
+// accumulator.  Then each CTA parks the column half its peer finishes in its
+// own shared memory, and finishes its half with the peer's partial read over
+// distributed shared memory: one fp32 addition of two partials, the same value
+// in both orders.  The last, ragged tile of an image is shifted inward (start
+// N - 128) so every TMA box lies inside the image's own rows; it stores only
+// the rows and columns the previous tile does not own.
+#include <cooperative_groups.h>
+
 #include "common.cuh"
 #include "kernels.cuh"
 #include "tc.cuh"
+
+namespace cg = cooperative_groups;
 
 namespace gmc {
 
@@ -46,11 +54,13 @@ __global__ void __launch_bounds__(128, 1)
   uint8_t* tilesB = base + STAGES * TILE_BYTES;
   GramCtl* ctl = reinterpret_cast<GramCtl*>(base + 2 * STAGES * TILE_BYTES);
 
+  cg::cluster_group cluster = cg::this_cluster();
+  const int kpart = (int)cluster.block_rank();  // 0 or 1: which half of the contraction
   const int b = blockIdx.y;
   const TextGeom tg = text_geom(toff, b, B, Tmax, status);
-  if (tg.T == 0) return;
+  if (tg.T == 0) return;  // uniform over the cluster
   const int nt = ceil_div(N, BM);
-  int t = blockIdx.x, I = 0;
+  int t = blockIdx.x >> 1, I = 0;
   while (t >= nt - I) {
     t -= nt - I;
     ++I;
@@ -59,7 +69,8 @@ __global__ void __launch_bounds__(128, 1)
   const int r0 = min(I * BM, N - BM), c0 = min(J * BM, N - BM);
   const int row_base = (int)((size_t)b * N + tg.off);  // first visual row of the image
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int nk = ceil_div(D, BK);
+  const int nk_all = ceil_div(D, BK), kh = (nk_all + 1) / 2;
+  const int kb0 = kpart * kh, nk = max(0, min(nk_all, kb0 + kh) - kb0);  // this CTA's K slices
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -93,8 +104,8 @@ __global__ void __launch_bounds__(128, 1)
         }
         if (ctl->abort) break;
         tc::mbar_arrive_expect_tx(&ctl->full[s], 2 * TILE_BYTES);
-        tc::tma_load_2d(tilesA + s * TILE_BYTES, &tmap, kb * BK, row_base + r0, &ctl->full[s]);
-        tc::tma_load_2d(tilesB + s * TILE_BYTES, &tmap, kb * BK, row_base + c0, &ctl->full[s]);
+        tc::tma_load_2d(tilesA + s * TILE_BYTES, &tmap, (kb0 + kb) * BK, row_base + r0, &ctl->full[s]);
+        tc::tma_load_2d(tilesB + s * TILE_BYTES, &tmap, (kb0 + kb) * BK, row_base + c0, &ctl->full[s]);
         ++issued;
       }
     }
@@ -125,20 +136,48 @@ __global__ void __launch_bounds__(128, 1)
   bool ok = tc::mbar_wait(&ctl->done, 0, deadline);
   ok = __all_sync(FULL, ok && !ctl->abort);
   tc::fence_after_sync();
+  const int row = warp * 32 + lane;  // this thread's TMEM lane = tile row
+  // the column half the peer finishes, column-major [64][128] in the (now idle)
+  // operand ring; a CTA without K slices contributes zeros
+  float* park = reinterpret_cast<float*>(tilesA);
+  const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
   if (ok) {
-    const int i = r0 + warp * 32 + lane;  // this thread's TMEM lane = output row
+#pragma unroll 1
+    for (int cc = 0; cc < 2; ++cc) {
+      float v[32];
+      if (nk > 0) {
+        tc::tmem_ld32(trow + (uint32_t)((1 - kpart) * 64 + cc * 32), v);
+      } else {
+#pragma unroll
+        for (int q = 0; q < 32; ++q) v[q] = 0.f;
+      }
+#pragma unroll
+      for (int q = 0; q < 32; ++q) park[(cc * 32 + q) * BM + row] = v[q];
+    }
+  }
+  tc::fence_before_sync();
+  cluster.sync();  // both parked halves are complete
+  tc::fence_after_sync();
+  if (ok) {
+    const float* peer = cluster.map_shared_rank(park, 1 - kpart);
+    const int i = r0 + row;  // output row
     const bool own_row = i >= I * BM;
     const float ri = rn[(size_t)b * N + i];
     float* crow = cos + ((size_t)b * N + i) * N;
 #pragma unroll 1
-    for (int cc = 0; cc < BM / 32; ++cc) {
+    for (int cc = 0; cc < 2; ++cc) {
       float v[32];
-      tc::tmem_ld32(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(cc * 32), v);
-      const int j0 = c0 + cc * 32;
+      if (nk > 0) {
+        tc::tmem_ld32(trow + (uint32_t)(kpart * 64 + cc * 32), v);
+      } else {
+#pragma unroll
+        for (int q = 0; q < 32; ++q) v[q] = 0.f;
+      }
+      const int j0 = c0 + kpart * 64 + cc * 32;
 #pragma unroll
       for (int q = 0; q < 32; ++q) {
         const int j = j0 + q;
-        v[q] = v[q] * ri * rn[(size_t)b * N + j];
+        v[q] = (v[q] + peer[(cc * 32 + q) * BM + row]) * ri * rn[(size_t)b * N + j];
       }
       if (own_row) {
         if (j0 >= J * BM) {
@@ -159,6 +198,7 @@ __global__ void __launch_bounds__(128, 1)
       }
     }
   }
+  cluster.sync();  // the peer has read this CTA's parked half
   if (!ok && threadIdx.x == 0) set_status(status, GMC_STATUS_TIMEOUT);
   if (warp == 0 && lane == 0 && !ok) {
     // drain TMA copies still in flight into this CTA's shared memory
@@ -222,10 +262,20 @@ cudaError_t launch_gram_tc(const Dims& dm, const void* hidden, Scratch& s, cudaS
   if (e != cudaSuccess) return e;
   if ((e = set_smem_limit((const void*)k_gram_tc, GRAM_SMEM)) != cudaSuccess) return e;
   const int nt = ceil_div(dm.N, BM);
-  dim3 grid(nt * (nt + 1) / 2, dm.B);
-  k_gram_tc<<<grid, 128, GRAM_SMEM, st>>>(map, dm.toff, dm.B, dm.N, dm.T, dm.D, s.rn, s.cos,
-                                          s.status);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2 * (nt * (nt + 1) / 2), dm.B);
+  cfg.blockDim = dim3(128);
+  cfg.dynamicSmemBytes = GRAM_SMEM;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, k_gram_tc, map, dm.toff, dm.B, dm.N, dm.T, dm.D,
+                            (const float*)s.rn, s.cos, s.status);
 }
 
 }  // namespace gmc

@@ -34,14 +34,12 @@ __global__ void __launch_bounds__(512) k_r0_pool(const long long* __restrict__ u
   w.hist = reinterpret_cast<int*>(p);       p += sizeof(int) * sel::HBINS;
   w.bnd = reinterpret_cast<int*>(p);        p += sizeof(int) * N;
   w.wsum = reinterpret_cast<int*>(p);       p += sizeof(int) * 32;
-  w.scal = reinterpret_cast<int*>(p);       p += sizeof(int) * 4;
+  w.scal = reinterpret_cast<int*>(p);       p += sizeof(int) * 8;
   int* pool = reinterpret_cast<int*>(p);    p += sizeof(int) * P;
-  w.inpool = reinterpret_cast<unsigned char*>(p);  p += N;
+  w.tmp = reinterpret_cast<int*>(p);        p += sizeof(int) * P;
   unsigned char* selz = reinterpret_cast<unsigned char*>(p);
-  for (int j = threadIdx.x; j < N; j += blockDim.x) {
-    w.inpool[j] = 0;
-    selz[j] = 0;
-  }
+  for (int j = threadIdx.x; j < N; j += blockDim.x) selz[j] = 0;
+  for (int h = threadIdx.x; h < sel::HBINS; h += blockDim.x) w.hist[h] = 0;
   __syncthreads();
   const int Pt = sel::select_pool(u0 + (size_t)b * N, selz, N, P, w, pool, nullptr);
   for (int k = threadIdx.x; k < P; k += blockDim.x) pool0[(size_t)b * P + k] = k < Pt ? pool[k] : -1;
@@ -129,9 +127,13 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_filter(
   }
   if (threadIdx.x < 3) fb[threadIdx.x] = 0;
   __syncthreads();
-  for (int k = threadIdx.x; k < Pt; k += blockDim.x) {
-    const int rank = sel::score_rank(sc, pool, Pt, k);
-    if (rank < nb) batch[rank] = pool[k];
+  {
+    const int lane = threadIdx.x & 31, gl = lane & 7;
+    const unsigned gm = 0xFFu << (lane & 24);
+    for (int k = threadIdx.x >> 3; k < Pt; k += blockDim.x >> 3) {  // 8 lanes per pool token
+      const int rank = sel::group_score_rank(sc, pool, Pt, k, gl, gm);
+      if (gl == 0 && rank < nb) batch[rank] = pool[k];
+    }
   }
   __syncthreads();
   if (blockIdx.x == 0) {  // record the first batch once per image
@@ -242,7 +244,7 @@ cudaError_t launch_round0(const R0State& r0, int B, int N, int K, int M, const i
   if ((e = cudaMemsetAsync(r0.u1, 0, sizeof(long long) * (size_t)B * N, st)) != cudaSuccess) return e;
   if ((e = cudaMemsetAsync(r0.fv, 0, sizeof(long long) * B * 4, st)) != cudaSuccess) return e;
   if ((e = cudaMemsetAsync(r0.info, 0, sizeof(int32_t) * B * 4, st)) != cudaSuccess) return e;
-  const size_t smem = sizeof(int) * (sel::HBINS + N + 32 + 4 + P) + 2 * (size_t)N + 64;
+  const size_t smem = sizeof(int) * (sel::HBINS + N + 32 + 8 + 2 * P) + (size_t)N + 64;
   if ((e = set_smem_limit((const void*)k_r0_pool, smem)) != cudaSuccess) return e;
   const int uniform = (H == 0);
   k_r0_pool<<<B, 512, smem, st>>>(u0, B, N, P, uniform ? nullptr : toff, T, r0.pool, r0.info,

@@ -87,7 +87,7 @@ struct SelSmem {
   long long* u_full;    // [N]  gains of the current round (every CTA)
   int* hist;            // [HBINS]
   int* bnd;             // [N]  tokens in the boundary histogram bin
-  unsigned char* inpool;  // [N]
+  int* tmp;             // [P]  pool tokens in arrival order (select_pool)
   unsigned char* sel;   // [N]
   short* poolslot;      // [N]  pool slot of a token or -1
   int* pool;            // [P]
@@ -128,7 +128,7 @@ __host__ __device__ inline size_t sel_fixed_bytes(int N, int P, int RPC, SelSmem
   p = take(sizeof(long long) * N);  if (o) o->u_full = (long long*)p;
   p = take(sizeof(int) * HBINS);    if (o) o->hist = (int*)p;
   p = take(sizeof(int) * N);        if (o) o->bnd = (int*)p;
-  p = take(N);                      if (o) o->inpool = (unsigned char*)p;
+  p = take(sizeof(int) * P);        if (o) o->tmp = (int*)p;
   p = take(N);                      if (o) o->sel = (unsigned char*)p;
   p = take(sizeof(short) * N);      if (o) o->poolslot = (short*)p;
   p = take(sizeof(int) * P);        if (o) o->pool = (int*)p;
@@ -234,9 +234,9 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
     s.u_full[j] = Pt0 > 0 ? a.r0.u1[(size_t)b * N + j] : a.u0[(size_t)b * N + j];
     s.poolslot[j] = -1;
     s.sel[j] = 0;
-    s.inpool[j] = 0;
   }
   for (int k = threadIdx.x; k < P; k += blockDim.x) s.s_acc[k] = 0;
+  for (int h = threadIdx.x; h < HBINS; h += blockDim.x) s.hist[h] = 0;  // select_pool keeps it zero
   if (threadIdx.x < 8) s.fb[threadIdx.x] = 0;
   if (threadIdx.x < 16) s.scal[threadIdx.x] = 0;
   if (threadIdx.x == 0) s.scal[SC_GLOBAL] = 1;
@@ -358,6 +358,7 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
   const int rounds_max = (K + a.bsz - 1) / a.bsz + 1;
   int S_count = nb0, rnd = Pt0 > 0 ? 1 : 0, filled = 0;
   const int sub = lane / G, gl = lane % G;
+  const int gid = wid * (32 / G) + sub, ngrp = nw * (32 / G);  // 8-lane groups of the block
   const unsigned gm = 0xFFu << (sub * G);
   const unsigned lt = lanemask_lt() & gm;
   while (S_count < K) {
@@ -366,7 +367,7 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
       break;
     }
     // ---- pool of this round ------------------------------------------------------
-    sel::PoolScratch pw{s.hist, s.bnd, s.inpool, s.wsum, s.scal + 8};
+    sel::PoolScratch pw{s.hist, s.bnd, s.tmp, s.wsum, s.scal + 8};
     const int Pt = sel::select_pool(s.u_full, s.sel, N, P, pw, s.pool, s.poolslot);
     if (Pt == 0) {
       // Zero-gain remainder: fill in ascending source order (F unchanged).
@@ -404,17 +405,17 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
     __syncthreads();
 
     // ---- flat mode (every list of this CTA in shared memory, sorted by token):
-    // the responsibilities touch only the pool tokens' segments, one warp per
-    // pool token; per-row values are order-independent (max of positive floats
+    // the responsibilities touch only the pool tokens' segments, one 8-lane
+    // group per pool token; per-row values are order-independent (max of positive floats
     // as integers, fixed-point sums), so nothing depends on the schedule.
     const bool flat = !s.scal[SC_GLOBAL];
     const float z_one = 1099511627776.f;  // 2^40: fixed-point scale of the softmax denominators
     const float z_inv = 1.f / z_one;
     if (flat) {
       // largest pool residual and number of pool entries of every row
-      for (int k = wid; k < Pt; k += nw) {
+      for (int k = gid; k < Pt; k += ngrp) {
         const int j = s.pool[k];
-        for (int p = s.cstart[j] + lane; p < s.cstart[j + 1]; p += 32) {
+        for (int p = s.cstart[j] + gl; p < s.cstart[j + 1]; p += G) {
           const int q = s.srows[p];
           if (q == DEADROW) continue;
           atomicMax(&s.rmaxb[q], __float_as_int(s.svals[p] - s.bcov[q]));
@@ -423,9 +424,9 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
       }
       __syncthreads();
       // softmax denominators, exact in 2^-40
-      for (int k = wid; k < Pt; k += nw) {
+      for (int k = gid; k < Pt; k += ngrp) {
         const int j = s.pool[k];
-        for (int p = s.cstart[j] + lane; p < s.cstart[j + 1]; p += 32) {
+        for (int p = s.cstart[j] + gl; p < s.cstart[j + 1]; p += G) {
           const int q = s.srows[p];
           if (q == DEADROW) continue;
           const float tau = a.resp_temp * __int_as_float(s.rmaxb[q]) + a.resp_eps;
@@ -434,11 +435,11 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
         }
       }
       __syncthreads();
-      // s_k = sum_m rho_mk R_mk: one warp owns pool slot k, so its sum is this CTA's score
-      for (int k = wid; k < Pt; k += nw) {
+      // s_k = sum_m rho_mk R_mk: one group owns pool slot k, so its sum is this CTA's score
+      for (int k = gid; k < Pt; k += ngrp) {
         const int j = s.pool[k];
         unsigned long long acc = 0;
-        for (int p = s.cstart[j] + lane; p < s.cstart[j + 1]; p += 32) {
+        for (int p = s.cstart[j] + gl; p < s.cstart[j + 1]; p += G) {
           const int q = s.srows[p];
           if (q == DEADROW) continue;
           const float tau = a.resp_temp * __int_as_float(s.rmaxb[q]) + a.resp_eps;
@@ -447,8 +448,8 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
           acc += (unsigned long long)to_fix(expf(R / tau) / z * R, fxs);
         }
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(FULL, acc, o);
-        if (lane == 0) s.s_part[k] = (long long)acc;
+        for (int o = G / 2; o > 0; o >>= 1) acc += __shfl_xor_sync(gm, acc, o);
+        if (gl == 0) s.s_part[k] = (long long)acc;
       }
     }
     if (!flat) {
@@ -550,10 +551,12 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
 
     // ---- batch, coverage update, survivor filter, next gains ------------------
     const int nb = min(a.bsz, min(Pt, K - S_count));
-    for (int k = threadIdx.x; k < Pt; k += blockDim.x) {
-      const int rank = sel::score_rank(s.s_acc, s.pool, Pt, k);
-      s.inb[k] = rank < nb;
-      if (rank < nb) s.batch[rank] = s.pool[k];
+    for (int k = gid; k < Pt; k += ngrp) {  // 8 lanes rank each pool token
+      const int rank = sel::group_score_rank(s.s_acc, s.pool, Pt, k, gl, gm);
+      if (gl == 0) {
+        s.inb[k] = rank < nb;
+        if (rank < nb) s.batch[rank] = s.pool[k];
+      }
     }
     __syncthreads();
     for (int q = threadIdx.x; q < nb; q += blockDim.x) {
@@ -563,10 +566,10 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
     if (r == 0 && a.tv.base && threadIdx.x == 0)
       a.tv.at<int32_t>(b, a.tv.off_round_end)[rnd] = S_count + nb;
     if (flat) {
-      // coverage update: largest batch value per row, one warp per batch token
-      for (int k = wid; k < nb; k += nw) {
+      // coverage update: largest batch value per row, one 8-lane group per batch token
+      for (int k = gid; k < nb; k += ngrp) {
         const int j = s.batch[k];
-        for (int p = s.cstart[j] + lane; p < s.cstart[j + 1]; p += 32) {
+        for (int p = s.cstart[j] + gl; p < s.cstart[j + 1]; p += G) {
           const int q = s.srows[p];
           if (q != DEADROW) atomicMax(&s.bnb[q], __float_as_int(s.svals[p]));
         }

@@ -57,40 +57,78 @@ __device__ inline int block_exclusive_scan(int v, int* wsum, int* total) {
 
 // Shared-memory scratch of select_pool.
 struct PoolScratch {
-  int* hist;              // [HBINS]
-  int* bnd;               // [N]
-  unsigned char* inpool;  // [N], all zero on entry and on return
-  int* wsum;              // [32]
-  int* scal;              // [4]
+  int* hist;  // [HBINS], all zero on entry and on return
+  int* bnd;   // [N]
+  int* tmp;   // [P]  pool tokens in arrival order
+  int* wsum;  // [32]
+  int* scal;  // [5]
 };
+
+// Warp-aggregated append: every lane with `want` gets a distinct index from
+// *counter (order within the warp by lane).  All lanes of the warp call it.
+__device__ __forceinline__ int warp_append(bool want, int* counter) {
+  const unsigned m = __ballot_sync(FULL, want);
+  const int leader = m ? __ffs(m) - 1 : 0;  // lowest appending lane
+  int base = 0;
+  if (m && (int)(threadIdx.x & 31) == leader) base = atomicAdd(counter, __popc(m));
+  base = __shfl_sync(FULL, base, leader);
+  return base + __popc(m & lanemask_lt());
+}
+
+// Position of x among n distinct ints a[0..n) (the number smaller than x),
+// counted by the 8 lanes of an aligned group (mask gm); every group lane gets it.
+__device__ __forceinline__ int group_rank_of(const int* a, int n, int x, int gl, unsigned gm) {
+  int c = 0;
+  for (int k = gl; k < n; k += 8) c += a[k] < x;
+  c += __shfl_xor_sync(gm, c, 1);
+  c += __shfl_xor_sync(gm, c, 2);
+  c += __shfl_xor_sync(gm, c, 4);
+  return c;
+}
 
 // Pool of one round: the min(P, #{u_i > 0}) tokens with sel[i] == 0 of largest
 // gain u (fixed point), ties to the lower index.  A histogram over an
 // exponent/mantissa bucket finds the boundary bucket; tokens inside it are
-// ranked exactly.  Slots are numbered in ascending token order: pool[0..Pt).
+// ranked exactly.  Pool tokens arrive in any order and take the slot of their
+// rank by token index, so slots ascend with the token: pool[0..Pt).
 // poolslot (optional) receives the slot of every pool token.  Returns Pt.
-// Every thread of the block must call it; the result does not depend on
-// thread scheduling.
+// Every thread of the block must call it (blockDim a multiple of 32, N
+// rounded up to the block is walked by whole warps); the result does not
+// depend on thread scheduling.
 __device__ inline int select_pool(const long long* u, const unsigned char* sel, int N, int P,
                                   PoolScratch w, int* pool, short* poolslot) {
-  for (int k = threadIdx.x; k < HBINS; k += blockDim.x) w.hist[k] = 0;
-  if (threadIdx.x == 0) w.scal[3] = 0;
-  __syncthreads();
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  if (threadIdx.x < 5) w.scal[threadIdx.x] = 0;
   for (int j = threadIdx.x; j < N; j += blockDim.x) {
     const long long v = u[j];
     if (!sel[j] && v > 0) atomicAdd(&w.hist[gain_bucket(v)], 1);
   }
   __syncthreads();
   {
-    // Every thread sums a contiguous range of bins; the thread whose range
-    // holds the P-th largest candidate finds the boundary bin inside it.
+    // Every thread owns a contiguous range of buckets (zeroed again here); the
+    // thread whose range holds the P-th largest candidate finds the boundary
+    // bucket inside it.
     const int per = (HBINS + blockDim.x - 1) / blockDim.x;
     const int h0 = min(HBINS, (int)threadIdx.x * per), h1 = min(HBINS, h0 + per);
     int part = 0;
     for (int h = h0; h < h1; ++h) part += w.hist[h];
-    int npos = 0;
-    const int below = block_exclusive_scan(part, w.wsum, &npos);
-    const int above = npos - below - part;  // candidates in higher bins
+    int x = part;  // inclusive prefix within the warp
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(FULL, x, o);
+      if (lane >= o) x += y;
+    }
+    if (lane == 31) w.wsum[wid] = x;
+    __syncthreads();
+    int t = lane < nw ? w.wsum[lane] : 0;  // warp totals, prefix over warps by shuffles
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(FULL, t, o);
+      if (lane >= o) t += y;
+    }
+    const int npos = __shfl_sync(FULL, t, 31);
+    const int wbefore = wid > 0 ? __shfl_sync(FULL, t, wid - 1) : 0;
+    const int above = npos - (wbefore + x);  // candidates in higher buckets
     if (npos <= P) {
       if (threadIdx.x == 0) {
         w.scal[0] = -1;    // every candidate is in the pool
@@ -109,17 +147,24 @@ __device__ inline int select_pool(const long long* u, const unsigned char* sel, 
       w.scal[1] = cum;
       w.scal[2] = P;
     }
+    for (int h = h0; h < h1; ++h) w.hist[h] = 0;
   }
   __syncthreads();
   const int Pt = w.scal[2];
   const int bstar = w.scal[0];
   if (Pt > 0) {
-    for (int j = threadIdx.x; j < N; j += blockDim.x) {
-      const long long v = u[j];
-      if (sel[j] || v <= 0) continue;
-      const int k = gain_bucket(v);
-      if (k > bstar) w.inpool[j] = 1;
-      else if (k == bstar) w.bnd[atomicAdd(&w.scal[3], 1)] = j;
+    for (int j0 = wid * 32; j0 < N; j0 += nw * 32) {  // whole warps: aggregated appends
+      const int j = j0 + lane;
+      int k = -1;
+      if (j < N) {
+        const long long v = u[j];
+        if (!sel[j] && v > 0) k = gain_bucket(v);
+      }
+      const bool up = k > bstar, at = k >= 0 && k == bstar;
+      const int pu = warp_append(up, &w.scal[4]);
+      const int pb = warp_append(at, &w.scal[3]);
+      if (up) w.tmp[pu] = j;
+      if (at) w.bnd[pb] = j;
     }
     __syncthreads();
     if (bstar >= 0) {
@@ -132,25 +177,38 @@ __device__ inline int select_pool(const long long* u, const unsigned char* sel, 
           const int j2 = w.bnd[q2];
           rank += key_before(u[j2], j2, v, j);
         }
-        if (rank < need) w.inpool[j] = 1;
+        if (rank < need) w.tmp[w.scal[1] + rank] = j;  // after the tokens above the bucket
       }
     }
     __syncthreads();
-    const int per = (N + blockDim.x - 1) / blockDim.x;
-    const int j0 = threadIdx.x * per, j1 = min(N, j0 + per);
-    int mine = 0;
-    for (int j = j0; j < j1; ++j) mine += w.inpool[j];
-    int slot = block_exclusive_scan(mine, w.wsum, nullptr);
-    for (int j = j0; j < j1; ++j)
-      if (w.inpool[j]) {
+    // slot = rank by token index: one 8-lane group per pool token
+    const int gl = lane & 7;
+    const unsigned gm = 0xFFu << (lane & 24);
+    for (int k0 = threadIdx.x >> 3; k0 < Pt; k0 += blockDim.x >> 3) {
+      const int j = w.tmp[k0];
+      const int slot = group_rank_of(w.tmp, Pt, j, gl, gm);
+      if (gl == 0) {
         pool[slot] = j;
         if (poolslot) poolslot[j] = (short)slot;
-        w.inpool[j] = 0;
-        ++slot;
       }
+    }
   }
   __syncthreads();
   return Pt;
+}
+
+// Rank of pool slot k among the Pt slots by (score desc, token asc), counted by
+// the 8 lanes of an aligned group (mask gm).
+__device__ __forceinline__ int group_score_rank(const long long* s, const int* pool, int Pt, int k,
+                                                int gl, unsigned gm) {
+  const long long sk = s[k];
+  const int jk = pool[k];
+  int rank = 0;
+  for (int q = gl; q < Pt; q += 8) rank += key_before(s[q], pool[q], sk, jk);
+  rank += __shfl_xor_sync(gm, rank, 1);
+  rank += __shfl_xor_sync(gm, rank, 2);
+  rank += __shfl_xor_sync(gm, rank, 4);
+  return rank;
 }
 
 // Rank of pool slot k among the Pt slots by (score desc, token asc).
