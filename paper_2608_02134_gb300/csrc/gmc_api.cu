@@ -90,12 +90,13 @@ size_t carve_compress(const Dims& dm, Scratch* s, char* base, R0State* r0s = nul
   Carver c{base};
   Scratch t{};
   const size_t B = dm.B, N = dm.N, H = dm.H, T = dm.T, M = dm.M, K = dm.K;
-  t.nP = ceil_div(dm.N, ROWS_PER_BLOCK);
+  t.nP = ceil_div(dm.N, PROBE_TOK);
   t.nHG = ceil_div(dm.N, HG_TOK);
   t.nA = ceil_div(dm.N, ASSIGN_WARPS);
   t.nE = ceil_div(dm.N, ENERGY_THREADS);
   t.nSel = 0;
-  t.status = c.take<uint32_t>(4);
+  t.status = c.take<uint32_t>(4 + B);  // status word, then one probe ticket per image
+  t.tick = t.status + 4;
   t.A = c.take<float>(B * H * T * N);
   t.nRS = message_splits(dm);
   t.rs = c.take<float>(B * H * (size_t)t.nRS * T);
@@ -234,6 +235,31 @@ struct Profiler {
 };
 Profiler g_prof;
 
+// A second stream per device for the branch of the path that does not depend
+// on the message slice (row norms -> cosine Gram), forked from and joined back
+// into the caller's stream with events.  Created on first use on each device;
+// calls are serialised by the host lock of gmc_compress.
+struct SideStream {
+  cudaStream_t st = nullptr;
+  cudaEvent_t fork = nullptr, join = nullptr;
+};
+SideStream g_side[64];
+
+cudaError_t side_stream(SideStream** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  SideStream& sd = g_side[dev];
+  if (!sd.st) {
+    if ((e = cudaStreamCreateWithFlags(&sd.st, cudaStreamNonBlocking)) != cudaSuccess) return e;
+    if ((e = cudaEventCreateWithFlags(&sd.fork, cudaEventDisableTiming)) != cudaSuccess) return e;
+    if ((e = cudaEventCreateWithFlags(&sd.join, cudaEventDisableTiming)) != cudaSuccess) return e;
+  }
+  *out = &sd;
+  return cudaSuccess;
+}
+
 #define GMC_STAGE(name, nkernels, expr)              \
   do {                                               \
     GMC_TRY(expr);                                   \
@@ -345,7 +371,7 @@ int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* 
     GMC_TRY(cudaMemsetAsync(trace, 0, (size_t)dm.B * L.bytes_per_image, st));
   }
   std::lock_guard<std::mutex> lk(g_prof.mu);
-  GMC_TRY(cudaMemsetAsync(s.status, 0, sizeof(uint32_t), st));
+  GMC_TRY(cudaMemsetAsync(s.status, 0, sizeof(uint32_t) * (4 + dm.B), st));  // status, probe tickets
   if (Ke == N) {  // K = N returns the unmodified execution
     GMC_TRY(launch_identity(dm, hidden, keys, pos_ids, out_idx, out_hidden, out_kv, out_pos,
                             s.status, st));
@@ -355,11 +381,26 @@ int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* 
   const int fx = fixed_point_exponent((double)p.beta_G + p.beta_V + p.beta_S);
   GMC_TRY(cudaMemsetAsync(s.u0, 0, sizeof(long long) * dm.B * N, st));
   GMC_TRY(g_prof.begin(st));
-  GMC_STAGE("rownorm", 1, launch_rownorm(dm, hidden, p.norm_eps, s, st));
-  GMC_STAGE("probe", 2, launch_probe(dm, keys, vo_probe, p, s, st));
-  GMC_STAGE("message", message_tc_supported(dm) ? 3 : 1, launch_message(dm, keys, queries, s, st));
-  GMC_STAGE("heads", 4, launch_heads(dm, p, s, tv, st));
-  GMC_STAGE("gram", 1, launch_gram(dm, hidden, s, st));
+  if (g_prof.on) {  // stage timing: every stage in turn on the caller's stream
+    GMC_STAGE("rownorm", 1, launch_rownorm(dm, hidden, p.norm_eps, s, st));
+    GMC_STAGE("probe", 1, launch_probe(dm, keys, vo_probe, p, s, st));
+    GMC_STAGE("message", message_tc_supported(dm) ? 3 : 1, launch_message(dm, keys, queries, s, st));
+    GMC_STAGE("heads", 4, launch_heads(dm, p, s, tv, st));
+    GMC_STAGE("gram", 1, launch_gram(dm, hidden, s, st));
+  } else {
+    // row norms and the cosine Gram run beside probe -> message -> heads
+    SideStream* sd = nullptr;
+    GMC_TRY(side_stream(&sd));
+    GMC_TRY(cudaEventRecord(sd->fork, st));
+    GMC_TRY(cudaStreamWaitEvent(sd->st, sd->fork, 0));
+    GMC_STAGE("rownorm", 1, launch_rownorm(dm, hidden, p.norm_eps, s, sd->st));
+    GMC_STAGE("gram", 1, launch_gram(dm, hidden, s, sd->st));
+    GMC_TRY(cudaEventRecord(sd->join, sd->st));
+    GMC_STAGE("probe", 1, launch_probe(dm, keys, vo_probe, p, s, st));
+    GMC_STAGE("message", message_tc_supported(dm) ? 3 : 1, launch_message(dm, keys, queries, s, st));
+    GMC_STAGE("heads", 4, launch_heads(dm, p, s, tv, st));
+    GMC_TRY(cudaStreamWaitEvent(st, sd->join, 0));
+  }
   GMC_STAGE("clients", 1, launch_build_clients(dm, p, fx, s, st));
   GMC_STAGE("round0", 3,
             launch_round0(r0, dm.B, N, Ke, dm.M, dm.toff, H, T, p.landmarks * p.landmarks, p, fx,

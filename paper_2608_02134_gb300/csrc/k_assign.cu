@@ -20,16 +20,19 @@ __global__ void k_assign_gap(const float* __restrict__ cos, const int32_t* __res
                              uint32_t* status) {
   __shared__ double sd[ASSIGN_WARPS];
   __shared__ int sc[ASSIGN_WARPS];
+  extern __shared__ int sS[];  // the support of the image, staged once per block
   const int b = blockIdx.y;
   const TextGeom tg = text_geom(toff, b, B, Tmax, status);
   if (tg.T == 0) return;
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const int i = blockIdx.x * ASSIGN_WARPS + w;
+  for (int k = threadIdx.x; k < K; k += blockDim.x) sS[k] = support[(size_t)b * K + k];
+  __syncthreads();
   double dv = 0.0;
   int dc = 0;
   if (i < N && slot[(size_t)b * N + i] < 0) {
     const float* row = cos + ((size_t)b * N + i) * N;
-    const int32_t* S = support + (size_t)b * K;
+    const int32_t* S = sS;
     float m1 = -INFINITY, m2 = -INFINITY;
     for (int k = lane; k < K; k += 32) {
       const float v = row[S[k]];
@@ -75,31 +78,40 @@ __global__ void k_assign_pick(const float* __restrict__ cos, const int32_t* __re
                               int K, int Tmax, int gh, int gw, float gate_scale, float gate_pow,
                               float ambig_margin, float lambda_p, float tau_s, float alpha,
                               int32_t* pi, float* mass, TraceView tv, uint32_t* status) {
+  __shared__ float gate[3];      // dbar, s_x, mean energy
+  extern __shared__ int sS[];  // the support of the image, staged once per block
   const int b = blockIdx.y;
   const TextGeom tg = text_geom(toff, b, B, Tmax, status);
   if (tg.T == 0) return;
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-  // every warp reduces the partials in the same fixed order
-  double s = 0.0, c = 0.0;
-  for (int q = lane; q < nA; q += 32) {
-    s += dpart[((size_t)b * nA + q) * 2 + 0];
-    c += dpart[((size_t)b * nA + q) * 2 + 1];
+  for (int k = threadIdx.x; k < K; k += blockDim.x) sS[k] = support[(size_t)b * K + k];
+  if (w == 0) {  // the partials in a fixed order (every block the same)
+    double s = 0.0, c = 0.0, et = 0.0;
+    for (int q = lane; q < nA; q += 32) {
+      s += dpart[((size_t)b * nA + q) * 2 + 0];
+      c += dpart[((size_t)b * nA + q) * 2 + 1];
+    }
+    for (int q = lane; q < nE; q += 32) et += epart[(size_t)b * nE + q];  // message energies
+    s = warp_sum(s);
+    c = warp_sum(c);
+    et = warp_sum(et);
+    if (lane == 0) {
+      const float db = c > 0.0 ? (float)(s / c) : 0.f;
+      gate[0] = db;
+      gate[1] = 1.f - expf(-powf(db / gate_scale, gate_pow));
+      gate[2] = (float)(et / N);
+    }
   }
-  s = warp_sum(s);
-  c = warp_sum(c);
-  const float dbar = c > 0.0 ? (float)(s / c) : 0.f;
-  double et = 0.0;  // sum of the message energies, block sums in a fixed order
-  for (int q = lane; q < nE; q += 32) et += epart[(size_t)b * nE + q];
-  et = warp_sum(et);
-  const double emean = et / N;
-  const float sx = 1.f - expf(-powf(dbar / gate_scale, gate_pow));
+  __syncthreads();
+  const float dbar = gate[0], sx = gate[1];
+  const float emean = gate[2];
   if (blockIdx.x == 0 && threadIdx.x == 0 && tv.base) {
     tv.header(b)->s_x = sx;
     tv.header(b)->delta_bar = dbar;
   }
   const int i = blockIdx.x * ASSIGN_WARPS + w;
   if (i >= N) return;
-  const float eb = emean > 0.0 ? (float)(energy[(size_t)b * N + i] / emean) : 1.f;
+  const float eb = emean > 0.f ? energy[(size_t)b * N + i] / emean : 1.f;
   const float m = (1.f - alpha * sx) + alpha * sx * eb;
   int choice = i;
   if (slot[(size_t)b * N + i] < 0) {
@@ -107,7 +119,7 @@ __global__ void k_assign_pick(const float* __restrict__ cos, const int32_t* __re
     const float coef = lambda_p * sx * gi;
     const float piy = ((i / gw) + 0.5f) / gh, pix = ((i % gw) + 0.5f) / gw;
     const float* row = cos + ((size_t)b * N + i) * N;
-    const int32_t* S = support + (size_t)b * K;
+    const int32_t* S = sS;
     float best = -INFINITY;
     int bk = 0x7fffffff;
     for (int k = lane; k < K; k += 32) {
@@ -141,11 +153,15 @@ __global__ void k_assign_pick(const float* __restrict__ cos, const int32_t* __re
 cudaError_t launch_assign(const Dims& dm, const gmc_params& p, Scratch& s, const TraceView& tv,
                           cudaStream_t st) {
   dim3 grid(s.nA, dm.B);
-  k_assign_gap<<<grid, 32 * ASSIGN_WARPS, 0, st>>>(s.cos, s.support, s.slot, dm.toff, dm.B, dm.N,
+  const size_t smem = sizeof(int) * (size_t)dm.K;
+  cudaError_t e0;
+  if ((e0 = set_smem_limit((const void*)k_assign_gap, smem)) != cudaSuccess) return e0;
+  if ((e0 = set_smem_limit((const void*)k_assign_pick, smem)) != cudaSuccess) return e0;
+  k_assign_gap<<<grid, 32 * ASSIGN_WARPS, smem, st>>>(s.cos, s.support, s.slot, dm.toff, dm.B, dm.N,
                                                    dm.K, dm.T, s.delta, s.dpart, s.nA, s.status);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  k_assign_pick<<<grid, 32 * ASSIGN_WARPS, 0, st>>>(
+  k_assign_pick<<<grid, 32 * ASSIGN_WARPS, smem, st>>>(
       s.cos, s.support, s.slot, s.delta, s.dpart, s.nA, s.ebar, s.epart, s.nE, dm.toff, dm.B,
       dm.N, dm.K, dm.T,
       dm.gh, dm.gw, p.gate_scale, p.gate_pow, p.ambig_margin, p.assign_spatial_w, p.tau_s,

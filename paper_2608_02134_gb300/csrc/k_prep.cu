@@ -1,5 +1,7 @@
 // Per-token preparation: boundary-state norms, probe values and the mass
 // coordinate, and the K = N identity copy.
+#include <algorithm>
+
 #include "common.cuh"
 #include "kernels.cuh"
 
@@ -42,65 +44,86 @@ __global__ void k_rownorm(const Tin* __restrict__ hidden, const int32_t* toff, i
 }
 
 // Z_h[i] = V_{kv(h)}[i] W_h (Eq. (1): (V_h O_h) P with W_h = O_h P), ||Z_h[i]||^2,
-// and per-block partial sums of ||Z_h||_F^2.  A block covers ROWS_PER_BLOCK
-// tokens and every head; warp per (token, head) with lanes over the head dim.
+// per-block partial sums of ||Z_h||_F^2, and
+// sigma_h = sqrt(lambda_mass) * max(||Z_h||_F / sqrt(N r), eps_mass) (Eq. (1)).
+// A block covers PR_TOK tokens of one KV group: the values and the group's
+// W_h are staged in shared memory, one thread per (token, head) computes the
+// four probe coordinates.  The last block of an image to finish (a ticket per
+// image, zeroed with the status word) sums the partials in a fixed order.
+constexpr int PR_TOK = PROBE_TOK;
+
 template <typename Tin>
-__global__ void k_probe(const Tin* __restrict__ keys, const float* __restrict__ W,
-                        const int32_t* toff, int B, int N, int K, int Tmax, int H, int Hkv, int d,
-                        float* Z, float* zn2, float* sigpart, int nP, uint32_t* status) {
-  extern __shared__ float sm_probe[];  // [ROWS_PER_BLOCK][H]
-  const int b = blockIdx.y;
+__global__ void __launch_bounds__(256) k_probe(
+    const Tin* __restrict__ keys, const float* __restrict__ W, const int32_t* toff, int B, int N,
+    int K, int Tmax, int H, int Hkv, int d, float lambda_mass, float eps_mass, float* Z,
+    float* zn2, float* sigpart, int nP, float* sigma, uint32_t* tick, uint32_t* status) {
+  extern __shared__ float4 sm_probe4[];
+  __shared__ int last;
+  const int b = blockIdx.z, g = blockIdx.y, pb = blockIdx.x;
   const TextGeom tg = text_geom(toff, b, B, Tmax, status);
-  if (tg.T == 0) return;
+  if (tg.T == 0) return;  // uniform over the image
   const SeqIdx sq(b, N, K, tg.off, tg.T);
-  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
-  const int i0 = blockIdx.x * ROWS_PER_BLOCK;
-  const int grp = H / Hkv, HD = Hkv * d;
-  for (int p = wid; p < ROWS_PER_BLOCK * H; p += nw) {
-    const int ii = p / H, h = p % H, i = i0 + ii;
-    float z0 = 0.f, z1 = 0.f, z2 = 0.f, z3 = 0.f;
-    if (i < N) {
-      const Tin* v = keys + sq.value_row(i, HD) + (size_t)(h / grp) * d;
-      const float4* w4 = reinterpret_cast<const float4*>(W + (size_t)h * d * 4);
-      for (int k = lane; k < d; k += 32) {
-        float x = to_f32(v[k]);
-        float4 w = w4[k];
-        z0 = fmaf(x, w.x, z0);
-        z1 = fmaf(x, w.y, z1);
-        z2 = fmaf(x, w.z, z2);
-        z3 = fmaf(x, w.w, z3);
-      }
-      z0 = warp_sum(z0); z1 = warp_sum(z1); z2 = warp_sum(z2); z3 = warp_sum(z3);
-      if (lane == 0) {
-        const size_t o = ((size_t)b * H + h) * N + i;
-        reinterpret_cast<float4*>(Z)[o] = make_float4(z0, z1, z2, z3);
-        zn2[o] = z0 * z0 + z1 * z1 + z2 * z2 + z3 * z3;
-      }
-    }
-    if (lane == 0) sm_probe[ii * H + h] = z0 * z0 + z1 * z1 + z2 * z2 + z3 * z3;
+  const int grp = H / Hkv, HD = Hkv * d, i0 = pb * PR_TOK;
+  float4* Ws = sm_probe4;                                    // [grp][d + 1]
+  float* Vs = reinterpret_cast<float*>(Ws + grp * (d + 1));  // [PR_TOK][d + 1] (padded rows)
+  float* zs = Vs + PR_TOK * (d + 1);                         // [PR_TOK][grp]
+  const float4* W4 = reinterpret_cast<const float4*>(W) + (size_t)g * grp * d;
+  for (int idx = threadIdx.x; idx < grp * d; idx += blockDim.x)
+    Ws[(idx / d) * (d + 1) + idx % d] = W4[idx];
+  constexpr int VE = 16 / sizeof(Tin);  // elements per 16-byte load
+  for (int idx = threadIdx.x; idx < PR_TOK * d / VE; idx += blockDim.x) {
+    const int ii = idx / (d / VE), k = (idx % (d / VE)) * VE, i = i0 + ii;
+    uint4 raw = make_uint4(0, 0, 0, 0);
+    if (i < N) raw = *reinterpret_cast<const uint4*>(keys + sq.value_row(i, HD) + (size_t)g * d + k);
+    const Tin* e = reinterpret_cast<const Tin*>(&raw);
+#pragma unroll
+    for (int q = 0; q < VE; ++q) Vs[ii * (d + 1) + k + q] = to_f32(e[q]);
   }
   __syncthreads();
-  for (int h = threadIdx.x; h < H; h += blockDim.x) {
-    float s = 0.f;
-    for (int ii = 0; ii < ROWS_PER_BLOCK; ++ii) s += sm_probe[ii * H + h];  // fixed order
-    sigpart[((size_t)b * nP + blockIdx.x) * H + h] = s;
+  for (int task = threadIdx.x; task < PR_TOK * grp; task += blockDim.x) {
+    const int ii = task / grp, jh = task % grp, i = i0 + ii;
+    const float* v = Vs + ii * (d + 1);
+    const float4* w = Ws + jh * (d + 1);
+    float z0 = 0.f, z1 = 0.f, z2 = 0.f, z3 = 0.f;
+#pragma unroll 4
+    for (int k = 0; k < d; ++k) {
+      const float x = v[k];
+      const float4 c = w[k];
+      z0 = fmaf(x, c.x, z0);
+      z1 = fmaf(x, c.y, z1);
+      z2 = fmaf(x, c.z, z2);
+      z3 = fmaf(x, c.w, z3);
+    }
+    const float n2 = z0 * z0 + z1 * z1 + z2 * z2 + z3 * z3;
+    if (i < N) {
+      const size_t o = ((size_t)b * H + g * grp + jh) * N + i;
+      reinterpret_cast<float4*>(Z)[o] = make_float4(z0, z1, z2, z3);
+      zn2[o] = n2;
+    }
+    zs[ii * grp + jh] = i < N ? n2 : 0.f;
   }
-}
-
-// sigma_h = sqrt(lambda_mass) * max(||Z_h||_F / sqrt(N r), eps_mass), Eq. (1).
-// One warp per (image, head); partials summed in a fixed order.
-__global__ void k_sigma(const float* sigpart, int nP, int B, int N, int H, float lambda_mass,
-                        float eps_mass, float* sigma) {
-  const int w = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
-  if (w >= B * H) return;
-  const int b = w / H, h = w % H;
-  double s = 0.0;
-  for (int p = lane; p < nP; p += 32) s += sigpart[((size_t)b * nP + p) * H + h];
-  s = warp_sum(s);
-  if (lane == 0) {
-    double fro = sqrt(s);
-    double v = sqrt((double)lambda_mass) * fmax(fro / sqrt((double)N * 4.0), (double)eps_mass);
-    sigma[(size_t)b * H + h] = (float)v;
+  __syncthreads();
+  for (int jh = threadIdx.x; jh < grp; jh += blockDim.x) {
+    float sacc = 0.f;
+    for (int ii = 0; ii < PR_TOK; ++ii) sacc += zs[ii * grp + jh];  // fixed order
+    sigpart[((size_t)b * nP + pb) * H + g * grp + jh] = sacc;
+  }
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) last = atomicAdd(&tick[b], 1u) == (unsigned)(nP * Hkv - 1);
+  __syncthreads();
+  if (!last) return;
+  __threadfence();
+  // the image's partials: loaded by the whole block, summed per head in a fixed order
+  float* ps = Vs;  // reuse: nP * H floats (the host sizes this region for both uses)
+  for (int q = threadIdx.x; q < nP * H; q += blockDim.x)
+    ps[q] = __ldcg(&sigpart[(size_t)b * nP * H + q]);
+  __syncthreads();
+  for (int h = threadIdx.x; h < H; h += blockDim.x) {
+    double sacc = 0.0;
+    for (int q = 0; q < nP; ++q) sacc += (double)ps[q * H + h];
+    const float fro = (float)sqrt(sacc);
+    sigma[(size_t)b * H + h] = sqrtf(lambda_mass) * fmaxf(fro / sqrtf((float)N * 4.f), eps_mass);
   }
 }
 
@@ -160,21 +183,24 @@ cudaError_t launch_rms_rows(const Dims& dm, const void* hidden, float* rmsh, uin
 
 cudaError_t launch_probe(const Dims& dm, const void* keys, const float* W, const gmc_params& p,
                          Scratch& s, cudaStream_t st) {
-  dim3 grid(s.nP, dm.B);
-  size_t smem = sizeof(float) * ROWS_PER_BLOCK * dm.H;
-  if (dm.dtype == GMC_BF16)
-    k_probe<__nv_bfloat16><<<grid, 256, smem, st>>>((const __nv_bfloat16*)keys, W, dm.toff, dm.B,
-                                                    dm.N, dm.K, dm.T, dm.H, dm.Hkv, dm.d, s.Z,
-                                                    s.zn2, s.sigpart, s.nP, s.status);
-  else
+  const int grp = dm.H / dm.Hkv;
+  dim3 grid(s.nP, dm.Hkv, dm.B);
+  const size_t smem = sizeof(float4) * grp * (dm.d + 1) +
+                      sizeof(float) * (std::max((size_t)PR_TOK * (dm.d + 1), (size_t)s.nP * dm.H) +
+                                       (size_t)PR_TOK * grp);
+  cudaError_t e;
+  if (dm.dtype == GMC_BF16) {
+    if ((e = set_smem_limit((const void*)k_probe<__nv_bfloat16>, smem)) != cudaSuccess) return e;
+    k_probe<__nv_bfloat16><<<grid, 256, smem, st>>>(
+        (const __nv_bfloat16*)keys, W, dm.toff, dm.B, dm.N, dm.K, dm.T, dm.H, dm.Hkv, dm.d,
+        p.lambda_mass, p.eps_mass, s.Z, s.zn2, s.sigpart, s.nP, s.sigma, s.tick, s.status);
+  } else {
+    if ((e = set_smem_limit((const void*)k_probe<float>, smem)) != cudaSuccess) return e;
     k_probe<float><<<grid, 256, smem, st>>>((const float*)keys, W, dm.toff, dm.B, dm.N, dm.K,
-                                            dm.T, dm.H, dm.Hkv, dm.d, s.Z, s.zn2, s.sigpart,
-                                            s.nP, s.status);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  const int warps = dm.B * dm.H;
-  k_sigma<<<ceil_div(warps * 32, 256), 256, 0, st>>>(s.sigpart, s.nP, dm.B, dm.N, dm.H,
-                                                     p.lambda_mass, p.eps_mass, s.sigma);
+                                            dm.T, dm.H, dm.Hkv, dm.d, p.lambda_mass, p.eps_mass,
+                                            s.Z, s.zn2, s.sigpart, s.nP, s.sigma, s.tick,
+                                            s.status);
+  }
   return cudaGetLastError();
 }
 

@@ -43,6 +43,7 @@ struct Scratch {
   float* Z;          // [B][H][N][4]   probe values Z_h[i]
   float* zn2;        // [B][H][N]      ||Z_h[i]||^2
   float* sigpart;    // [B][nP][H]     block partials of ||Z_h||_F^2
+  uint32_t* tick;    // [B]            last-block tickets of the probe (zeroed with status)
   float* sigma;      // [B][H]         mass coordinate sigma_h
   double* hgpart;    // [B][nHG][H*H]  block partials of the head-pattern Gram
   double* HG;        // [B][H*H + H]   head-pattern Gram, then sum_t rs[h,t] per head
@@ -72,6 +73,7 @@ struct Scratch {
 constexpr int ROWS_PER_BLOCK = 8;  // rownorm / probe / client builder blocks
 constexpr int HG_TOK = 8;          // tokens per head-statistics block
 constexpr int ASSIGN_WARPS = 8;    // tokens per assignment block
+constexpr int PROBE_TOK = 32;       // tokens per probe block
 constexpr int ENERGY_THREADS = 256;  // tokens per block of the message-energy kernel
 
 // Launch wrappers.  Each returns the first CUDA error it saw.
