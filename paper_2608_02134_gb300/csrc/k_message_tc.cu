@@ -22,9 +22,13 @@
 // 128-column TMEM accumulators (double buffered); warps 0..7 read the
 // accumulators (warp w: TMEM lanes 32*(w%4).., columns 64*(w/4)..) and do the
 // softmax arithmetic.  Every wait is clock-bounded.
+#include <cooperative_groups.h>
+
 #include "common.cuh"
 #include "kernels.cuh"
 #include "tc.cuh"
+
+namespace cg = cooperative_groups;
 
 namespace gmc {
 
@@ -50,6 +54,24 @@ struct MsgCtl {
   float stat_l[2][BM];
   float rsum[2][BM];
 };
+
+// Control block of the fused kernel: barriers and this CTA's per-row
+// statistics, read by the other CTAs of the cluster.
+struct FusedCtl {
+  uint64_t qfull;
+  uint64_t full[STAGES];
+  uint64_t empty[STAGES];
+  uint64_t accdone;
+  uint32_t tmem;
+  volatile int abort;
+  float stat_m[2][BM];
+  float stat_l[2][BM];
+  float rsum[2][BM];
+  float cl_m[BM];  // the split's statistics per query row, for the whole cluster
+  float cl_l[BM];
+};
+constexpr int FUSED_MAX_TILES = 4;     // key tiles a CTA keeps in TMEM (4 x 128 columns)
+constexpr int FUSED_MAX_CLUSTER = 8;   // portable cluster size
 
 struct MsgSplit {
   int kt_per;  // key tiles per split
@@ -315,6 +337,224 @@ __global__ void __launch_bounds__(THREADS, 1)
   if (warp == 0) tc::tmem_dealloc(tmem, 256);
 }
 
+// Single-launch variant: the key splits of one query tile form a thread-block
+// cluster.  Every CTA keeps its split's logits in TMEM (at most FUSED_MAX_TILES
+// 128-column tiles), publishes its per-row (max, sum) in shared memory, and
+// after one cluster barrier merges all splits' statistics in a fixed order
+// (distributed shared memory) before writing A and its part of rs from the
+// resident logits.  Same results as the two launches of k_message_tc.
+__global__ void __launch_bounds__(THREADS, 1)
+    k_message_fused(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
+                    const int32_t* toff, int B, int N, int Tmax, int H, int Hkv, int d, int RQ,
+                    int kt_per, int nsplit, uint32_t tmem_cols, const float* __restrict__ zn2,
+                    const float* __restrict__ sigma, float* A, float* rs, uint32_t* status) {
+  extern __shared__ uint8_t sm_raw[];
+  cg::cluster_group cluster = cg::this_cluster();
+  uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  const int nkb = d / BK;
+  uint8_t* Qs = base;
+  uint8_t* Ks = base + (size_t)nkb * TILE_BYTES;
+  FusedCtl* ctl = reinterpret_cast<FusedCtl*>(base + (size_t)nkb * TILE_BYTES * (1 + STAGES));
+
+  const int b = blockIdx.z / nsplit, split = (int)cluster.block_rank(), g = blockIdx.y,
+            tile = blockIdx.x;
+  const TextGeom tg = text_geom(toff, b, B, Tmax, status);
+  const int grp = H / Hkv;
+  if (tg.T == 0 || tile * BM >= grp * tg.T) return;  // uniform over the cluster (same b, tile)
+  const int Tb = tg.T;
+  const int nkt = ceil_div(N + Tb, BM);
+  const int c0 = split * kt_per, c1 = min(nkt, c0 + kt_per);
+  const int iters = max(0, c1 - c0);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int qrow0 = (int)(((size_t)b * Hkv + g) * RQ + (size_t)tile * BM);
+  const int krow0 = (int)(2 * ((size_t)b * N + tg.off));
+
+  if (threadIdx.x == 0) {
+    tc::mbar_init(&ctl->qfull, 1);
+    for (int s = 0; s < STAGES; ++s) {
+      tc::mbar_init(&ctl->full[s], 1);
+      tc::mbar_init(&ctl->empty[s], 1);
+    }
+    tc::mbar_init(&ctl->accdone, 1);
+    ctl->abort = 0;
+    tc::fence_mbar_init();
+    tc::prefetch_tmap(&qmap);
+    tc::prefetch_tmap(&kmap);
+  }
+  if (warp == 0) {
+    tc::tmem_alloc(&ctl->tmem, tmem_cols);
+    tc::tmem_relinquish();
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = ctl->tmem;
+  const long long deadline = clock64() + WAIT_CYCLES;
+  const float scale = rsqrtf((float)d);
+  const int quarter = warp & 3, half = (warp >> 2) & 1;
+  const int r = quarter * 32 + lane;  // tile row == TMEM lane (epilogue warps)
+  const int R = tile * BM + r;
+  const bool valid = R < grp * Tb;
+  const int j = valid ? R / Tb : 0, t = valid ? R % Tb : 0;
+  const int h = g * grp + j;
+  const int kvis = N + t + 1;
+
+  if (warp == EPI_WARPS) {  // ---------------- TMA producer
+    int issued = 0;
+    if (lane == 0) {
+      tc::mbar_arrive_expect_tx(&ctl->qfull, nkb * TILE_BYTES);
+      for (int kb = 0; kb < nkb; ++kb)
+        tc::tma_load_2d(Qs + kb * TILE_BYTES, &qmap, kb * BK, qrow0, &ctl->qfull);
+      for (int it = 0; it < iters; ++it) {
+        const int s = it % STAGES;
+        const uint32_t ph = (uint32_t)(it / STAGES) & 1u;
+        if (it >= STAGES && !tc::mbar_wait(&ctl->empty[s], ph ^ 1u, deadline)) {
+          ctl->abort = 1;
+          break;
+        }
+        if (ctl->abort) break;
+        tc::mbar_arrive_expect_tx(&ctl->full[s], nkb * TILE_BYTES);
+        for (int kb = 0; kb < nkb; ++kb)
+          tc::tma_load_2d(Ks + ((size_t)s * nkb + kb) * TILE_BYTES, &kmap, g * d + kb * BK,
+                          krow0 + (c0 + it) * BM, &ctl->full[s]);
+        ++issued;
+      }
+      if (ctl->abort) {  // drain copies still landing in this CTA's shared memory
+        const long long d2 = clock64() + WAIT_CYCLES;
+        tc::mbar_wait(&ctl->qfull, 0, d2);
+        for (int it = (issued > STAGES ? issued - STAGES : 0); it < issued; ++it)
+          if (!tc::mbar_wait(&ctl->full[it % STAGES], (uint32_t)(it / STAGES) & 1u, d2)) break;
+      }
+    }
+    __syncwarp();
+  } else if (warp == EPI_WARPS + 1) {  // ---------------- MMA issuer: tile it -> columns it*128
+    if (lane == 0) {
+      const uint32_t idesc = tc::idesc_bf16_f32(BM, BM);
+      bool ok = tc::mbar_wait(&ctl->qfull, 0, deadline);
+      for (int it = 0; ok && it < iters; ++it) {
+        const int s = it % STAGES;
+        if (!tc::mbar_wait(&ctl->full[s], (uint32_t)(it / STAGES) & 1u, deadline)) {
+          ok = false;
+          break;
+        }
+        tc::fence_after_sync();
+        const uint32_t dst = tmem + (uint32_t)(it * BM);
+        for (int kb = 0; kb < nkb; ++kb) {
+          const uint64_t ad = tc::desc_sw128_kmajor(Qs + kb * TILE_BYTES);
+          const uint64_t bd = tc::desc_sw128_kmajor(Ks + ((size_t)s * nkb + kb) * TILE_BYTES);
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk)
+            tc::mma_bf16(dst, ad + 2 * kk, bd + 2 * kk, idesc, (kb | kk) != 0);
+        }
+        tc::mma_commit(&ctl->empty[s]);
+      }
+      if (!ok) ctl->abort = 1;
+      tc::mma_commit(&ctl->accdone);  // also with no tile or on abort
+    }
+    __syncwarp();
+  }
+
+  // ---- epilogue warps: this split's statistics -------------------------------
+  bool ok = true;
+  if (warp < EPI_WARPS) {
+    ok = tc::mbar_wait(&ctl->accdone, 0, deadline);
+    ok = __all_sync(FULL, ok && !ctl->abort);
+    tc::fence_after_sync();
+    float m = -INFINITY, l = 0.f;
+    for (int it = 0; ok && it < iters; ++it) {
+      float v[64];
+      const uint32_t ta = tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(it * BM + half * 64);
+      tc::tmem_ld32(ta, v);
+      tc::tmem_ld32(ta + 32, v + 32);
+      const int k0 = (c0 + it) * BM + half * 64;
+      float mt = -INFINITY;
+#pragma unroll
+      for (int q = 0; q < 64; ++q) {
+        v[q] *= scale;
+        if (k0 + q < kvis) mt = fmaxf(mt, v[q]);
+      }
+      if (mt > -INFINITY) {
+        const float mn = fmaxf(m, mt);
+        float acc = l * expf(m - mn);
+#pragma unroll
+        for (int q = 0; q < 64; ++q)
+          if (k0 + q < kvis) acc += expf(v[q] - mn);
+        l = acc;
+        m = mn;
+      }
+    }
+    ctl->stat_m[half][r] = m;
+    ctl->stat_l[half][r] = l;
+    epi_barrier();
+    if (half == 0) {
+      const float mo = ctl->stat_m[1][r], lo = ctl->stat_l[1][r];
+      const float Mc = fmaxf(m, mo);
+      ctl->cl_m[r] = Mc;
+      ctl->cl_l[r] = Mc > -INFINITY ? (m > -INFINITY ? l * expf(m - Mc) : 0.f) +
+                                          (mo > -INFINITY ? lo * expf(mo - Mc) : 0.f)
+                                    : 0.f;
+    }
+  }
+  cluster.sync();  // every split's statistics are published
+
+  if (warp < EPI_WARPS) {
+    // merge the splits in a fixed order, then the normalised visual columns
+    float M = -INFINITY, L = 0.f;
+    for (int q = 0; q < nsplit; ++q) M = fmaxf(M, cluster.map_shared_rank(ctl->cl_m, q)[r]);
+    for (int q = 0; q < nsplit; ++q) {
+      const float mq = cluster.map_shared_rank(ctl->cl_m, q)[r];
+      if (mq > -INFINITY) L += cluster.map_shared_rank(ctl->cl_l, q)[r] * expf(mq - M);
+    }
+    const float invL = 1.f / L;
+    const float sg = sigma[(size_t)b * H + h];
+    const float sg2 = sg * sg;
+    const float* zr = zn2 + ((size_t)b * H + h) * N;
+    float* arow = A + (((size_t)b * H + h) * Tmax + t) * N;
+    float rsum = 0.f;
+    for (int it = 0; ok && it < iters; ++it) {
+      const int k0 = (c0 + it) * BM + half * 64;
+      if (k0 >= N) continue;  // uniform over the warp
+      float v[64];
+      const uint32_t ta = tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(it * BM + half * 64);
+      tc::tmem_ld32(ta, v);  // warp-collective: every lane loads, valid rows use it
+      tc::tmem_ld32(ta + 32, v + 32);
+      if (!valid) continue;
+      const int nv = min(64, N - k0);
+      if (nv == 64 && (N & 3) == 0) {
+#pragma unroll
+        for (int q = 0; q < 64; q += 4) {
+          const float4 z = *reinterpret_cast<const float4*>(zr + k0 + q);
+          float4 o;
+          o.x = expf(v[q] * scale - M) * invL;
+          o.y = expf(v[q + 1] * scale - M) * invL;
+          o.z = expf(v[q + 2] * scale - M) * invL;
+          o.w = expf(v[q + 3] * scale - M) * invL;
+          *reinterpret_cast<float4*>(arow + k0 + q) = o;
+          rsum = fmaf(o.x, sqrtf(z.x + sg2), rsum);
+          rsum = fmaf(o.y, sqrtf(z.y + sg2), rsum);
+          rsum = fmaf(o.z, sqrtf(z.z + sg2), rsum);
+          rsum = fmaf(o.w, sqrtf(z.w + sg2), rsum);
+        }
+      } else {
+        for (int q = 0; q < nv; ++q) {
+          const float p = expf(v[q] * scale - M) * invL;
+          arow[k0 + q] = p;
+          rsum = fmaf(p, sqrtf(zr[k0 + q] + sg2), rsum);
+        }
+      }
+    }
+    ctl->rsum[half][r] = rsum;
+    epi_barrier();
+    if (half == 0 && valid && ok)
+      rs[(((size_t)b * H + h) * nsplit + split) * Tmax + t] = rsum + ctl->rsum[1][r];
+  }
+  if (threadIdx.x == 0 && ctl->abort) set_status(status, GMC_STATUS_TIMEOUT);
+  tc::fence_before_sync();
+  cluster.sync();  // the other CTAs have read this CTA's statistics
+  if (warp == 0) tc::tmem_dealloc(tmem, tmem_cols);
+}
+
 bool message_tc_supported(const Dims& dm) {
   return dm.dtype == GMC_BF16 && dm.N >= BM && (dm.d == 64 || dm.d == 128);
 }
@@ -347,6 +587,30 @@ cudaError_t launch_message_tc(const Dims& dm, const void* keys, const void* quer
   if ((e = set_smem_limit((const void*)k_message_tc, smem)) != cudaSuccess) return e;
   const MsgSplit sp = msg_split(dm.B, dm.Hkv, RQ, dm.N, dm.T);
   dim3 grid(RQ / BM, dm.Hkv, dm.B * sp.n);
+  if (sp.kt_per <= FUSED_MAX_TILES && sp.n <= FUSED_MAX_CLUSTER) {
+    uint32_t cols = 32;
+    while (cols < (uint32_t)(sp.kt_per * BM)) cols *= 2;
+    const size_t fsmem = 1024 + (size_t)nkb * TILE_BYTES * (1 + STAGES) + sizeof(FusedCtl);
+    if ((e = set_smem_limit((const void*)k_message_fused, fsmem)) != cudaSuccess) return e;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = dim3(THREADS);
+    cfg.dynamicSmemBytes = fsmem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 1;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = sp.n;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int ncl = 0;
+    if (cudaOccupancyMaxActiveClusters(&ncl, (void*)k_message_fused, &cfg) == cudaSuccess && ncl > 0)
+      return cudaLaunchKernelEx(&cfg, k_message_fused, qmap, kmap, dm.toff, dm.B, dm.N, dm.T, dm.H,
+                                dm.Hkv, dm.d, RQ, sp.kt_per, sp.n, cols, (const float*)s.zn2,
+                                (const float*)s.sigma, s.A, s.rs, s.status);
+    cudaGetLastError();  // no co-resident cluster: the two launches below
+  }
   for (int mode = 0; mode < 2; ++mode) {
     k_message_tc<<<grid, THREADS, smem, st>>>(qmap, kmap, dm.toff, dm.B, dm.N, dm.T, dm.H, dm.Hkv,
                                               dm.d, RQ, mode, sp.kt_per, sp.n, s.mpart, s.zn2,
