@@ -55,6 +55,10 @@ struct MsgCtl {
   float rsum[2][BM];
 };
 
+// Fused kernel: 16 epilogue warps (warp w reads TMEM lanes 32*(w%4).. and the
+// 32-column quarter w/4 of every tile), then the TMA producer and MMA warps.
+constexpr int FE_WARPS = 16, FT_THREADS = 32 * (FE_WARPS + 2);
+
 // Control block of the fused kernel: barriers and this CTA's per-row
 // statistics, read by the other CTAs of the cluster.
 struct FusedCtl {
@@ -64,12 +68,16 @@ struct FusedCtl {
   uint64_t accdone;
   uint32_t tmem;
   volatile int abort;
-  float stat_m[2][BM];
-  float stat_l[2][BM];
-  float rsum[2][BM];
+  float stat_m[4][BM];
+  float stat_l[4][BM];
+  float rsum[4][BM];
   float cl_m[BM];  // the split's statistics per query row, for the whole cluster
   float cl_l[BM];
 };
+
+__device__ __forceinline__ void fused_epi_barrier() {
+  asm volatile("bar.sync 1, %0;" ::"n"(FE_WARPS * 32) : "memory");
+}
 constexpr int FUSED_MAX_TILES = 4;     // key tiles a CTA keeps in TMEM (4 x 128 columns)
 constexpr int FUSED_MAX_CLUSTER = 8;   // portable cluster size
 
@@ -343,7 +351,7 @@ __global__ void __launch_bounds__(THREADS, 1)
 // after one cluster barrier merges all splits' statistics in a fixed order
 // (distributed shared memory) before writing A and its part of rs from the
 // resident logits.  Same results as the two launches of k_message_tc.
-__global__ void __launch_bounds__(THREADS, 1)
+__global__ void __launch_bounds__(FT_THREADS, 1)
     k_message_fused(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
                     const int32_t* toff, int B, int N, int Tmax, int H, int Hkv, int d, int RQ,
                     int kt_per, int nsplit, uint32_t tmem_cols, const float* __restrict__ zn2,
@@ -392,7 +400,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   const uint32_t tmem = ctl->tmem;
   const long long deadline = clock64() + WAIT_CYCLES;
   const float scale = rsqrtf((float)d);
-  const int quarter = warp & 3, half = (warp >> 2) & 1;
+  const int quarter = warp & 3, cq = (warp >> 2) & 3;  // lane quarter, column quarter
   const int r = quarter * 32 + lane;  // tile row == TMEM lane (epilogue warps)
   const int R = tile * BM + r;
   const bool valid = R < grp * Tb;
@@ -400,7 +408,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   const int h = g * grp + j;
   const int kvis = N + t + 1;
 
-  if (warp == EPI_WARPS) {  // ---------------- TMA producer
+  if (warp == FE_WARPS) {  // ---------------- TMA producer
     int issued = 0;
     if (lane == 0) {
       tc::mbar_arrive_expect_tx(&ctl->qfull, nkb * TILE_BYTES);
@@ -428,7 +436,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       }
     }
     __syncwarp();
-  } else if (warp == EPI_WARPS + 1) {  // ---------------- MMA issuer: tile it -> columns it*128
+  } else if (warp == FE_WARPS + 1) {  // ---------------- MMA issuer: tile it -> columns it*128
     if (lane == 0) {
       const uint32_t idesc = tc::idesc_bf16_f32(BM, BM);
       bool ok = tc::mbar_wait(&ctl->qfull, 0, deadline);
@@ -457,20 +465,18 @@ __global__ void __launch_bounds__(THREADS, 1)
 
   // ---- epilogue warps: this split's statistics -------------------------------
   bool ok = true;
-  if (warp < EPI_WARPS) {
+  if (warp < FE_WARPS) {
     ok = tc::mbar_wait(&ctl->accdone, 0, deadline);
     ok = __all_sync(FULL, ok && !ctl->abort);
     tc::fence_after_sync();
     float m = -INFINITY, l = 0.f;
     for (int it = 0; ok && it < iters; ++it) {
-      float v[64];
-      const uint32_t ta = tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(it * BM + half * 64);
-      tc::tmem_ld32(ta, v);
-      tc::tmem_ld32(ta + 32, v + 32);
-      const int k0 = (c0 + it) * BM + half * 64;
+      float v[32];
+      tc::tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(it * BM + cq * 32), v);
+      const int k0 = (c0 + it) * BM + cq * 32;
       float mt = -INFINITY;
 #pragma unroll
-      for (int q = 0; q < 64; ++q) {
+      for (int q = 0; q < 32; ++q) {
         v[q] *= scale;
         if (k0 + q < kvis) mt = fmaxf(mt, v[q]);
       }
@@ -478,27 +484,32 @@ __global__ void __launch_bounds__(THREADS, 1)
         const float mn = fmaxf(m, mt);
         float acc = l * expf(m - mn);
 #pragma unroll
-        for (int q = 0; q < 64; ++q)
+        for (int q = 0; q < 32; ++q)
           if (k0 + q < kvis) acc += expf(v[q] - mn);
         l = acc;
         m = mn;
       }
     }
-    ctl->stat_m[half][r] = m;
-    ctl->stat_l[half][r] = l;
-    epi_barrier();
-    if (half == 0) {
-      const float mo = ctl->stat_m[1][r], lo = ctl->stat_l[1][r];
-      const float Mc = fmaxf(m, mo);
+    ctl->stat_m[cq][r] = m;
+    ctl->stat_l[cq][r] = l;
+    fused_epi_barrier();
+    if (cq == 0) {  // the four column quarters of the row, in order
+      float Mc = -INFINITY;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) Mc = fmaxf(Mc, ctl->stat_m[q][r]);
+      float Lc = 0.f;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float mq = ctl->stat_m[q][r];
+        if (mq > -INFINITY) Lc += ctl->stat_l[q][r] * expf(mq - Mc);
+      }
       ctl->cl_m[r] = Mc;
-      ctl->cl_l[r] = Mc > -INFINITY ? (m > -INFINITY ? l * expf(m - Mc) : 0.f) +
-                                          (mo > -INFINITY ? lo * expf(mo - Mc) : 0.f)
-                                    : 0.f;
+      ctl->cl_l[r] = Lc;
     }
   }
   cluster.sync();  // every split's statistics are published
 
-  if (warp < EPI_WARPS) {
+  if (warp < FE_WARPS) {
     // merge the splits in a fixed order, then the normalised visual columns
     float M = -INFINITY, L = 0.f;
     for (int q = 0; q < nsplit; ++q) M = fmaxf(M, cluster.map_shared_rank(ctl->cl_m, q)[r]);
@@ -513,17 +524,16 @@ __global__ void __launch_bounds__(THREADS, 1)
     float* arow = A + (((size_t)b * H + h) * Tmax + t) * N;
     float rsum = 0.f;
     for (int it = 0; ok && it < iters; ++it) {
-      const int k0 = (c0 + it) * BM + half * 64;
+      const int k0 = (c0 + it) * BM + cq * 32;
       if (k0 >= N) continue;  // uniform over the warp
-      float v[64];
-      const uint32_t ta = tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(it * BM + half * 64);
-      tc::tmem_ld32(ta, v);  // warp-collective: every lane loads, valid rows use it
-      tc::tmem_ld32(ta + 32, v + 32);
+      float v[32];
+      // warp-collective: every lane loads, valid rows use it
+      tc::tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(it * BM + cq * 32), v);
       if (!valid) continue;
-      const int nv = min(64, N - k0);
-      if (nv == 64 && (N & 3) == 0) {
+      const int nv = min(32, N - k0);
+      if (nv == 32 && (N & 3) == 0) {
 #pragma unroll
-        for (int q = 0; q < 64; q += 4) {
+        for (int q = 0; q < 32; q += 4) {
           const float4 z = *reinterpret_cast<const float4*>(zr + k0 + q);
           float4 o;
           o.x = expf(v[q] * scale - M) * invL;
@@ -544,10 +554,11 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
       }
     }
-    ctl->rsum[half][r] = rsum;
-    epi_barrier();
-    if (half == 0 && valid && ok)
-      rs[(((size_t)b * H + h) * nsplit + split) * Tmax + t] = rsum + ctl->rsum[1][r];
+    ctl->rsum[cq][r] = rsum;
+    fused_epi_barrier();
+    if (cq == 0 && valid && ok)
+      rs[(((size_t)b * H + h) * nsplit + split) * Tmax + t] =
+          ((ctl->rsum[0][r] + ctl->rsum[1][r]) + ctl->rsum[2][r]) + ctl->rsum[3][r];
   }
   if (threadIdx.x == 0 && ctl->abort) set_status(status, GMC_STATUS_TIMEOUT);
   tc::fence_before_sync();
@@ -594,7 +605,7 @@ cudaError_t launch_message_tc(const Dims& dm, const void* keys, const void* quer
     if ((e = set_smem_limit((const void*)k_message_fused, fsmem)) != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = grid;
-    cfg.blockDim = dim3(THREADS);
+    cfg.blockDim = dim3(FT_THREADS);
     cfg.dynamicSmemBytes = fsmem;
     cfg.stream = st;
     cudaLaunchAttribute attr[1];
