@@ -93,7 +93,7 @@ size_t carve_compress(const Dims& dm, Scratch* s, char* base, R0State* r0s = nul
   t.nP = ceil_div(dm.N, PROBE_TOK);
   t.nHG = ceil_div(dm.N, HG_TOK);
   t.nA = ceil_div(dm.N, ASSIGN_WARPS);
-  t.nE = ceil_div(dm.N, ENERGY_THREADS);
+  t.nE = t.nA;  // energy block sums come from the assignment gap kernel
   t.nSel = 0;
   t.status = c.take<uint32_t>(4 + B);  // status word, then one probe ticket per image
   t.tick = t.status + 4;
@@ -385,7 +385,7 @@ int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* 
     GMC_STAGE("rownorm", 1, launch_rownorm(dm, hidden, p.norm_eps, s, st));
     GMC_STAGE("probe", 1, launch_probe(dm, keys, vo_probe, p, s, st));
     GMC_STAGE("message", message_tc_supported(dm) ? 3 : 1, launch_message(dm, keys, queries, s, st));
-    GMC_STAGE("heads", 4, launch_heads(dm, p, s, tv, st));
+    GMC_STAGE("heads", 3, launch_heads(dm, p, s, tv, st));
     GMC_STAGE("gram", 1, launch_gram(dm, hidden, s, st));
   } else {
     // row norms and the cosine Gram run beside probe -> message -> heads
@@ -398,7 +398,7 @@ int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* 
     GMC_TRY(cudaEventRecord(sd->join, sd->st));
     GMC_STAGE("probe", 1, launch_probe(dm, keys, vo_probe, p, s, st));
     GMC_STAGE("message", message_tc_supported(dm) ? 3 : 1, launch_message(dm, keys, queries, s, st));
-    GMC_STAGE("heads", 4, launch_heads(dm, p, s, tv, st));
+    GMC_STAGE("heads", 3, launch_heads(dm, p, s, tv, st));
     GMC_TRY(cudaStreamWaitEvent(st, sd->join, 0));
   }
   GMC_STAGE("clients", 1, launch_build_clients(dm, p, fx, s, st));

@@ -14,12 +14,18 @@
 namespace gmc {
 
 // Pass 1: delta_i per discarded token; per-block partial sums of delta and counts.
+// Also the message energy of every token (appendix Eq. (cond-grounded-energy)):
+//   e_i = (sum_h omega_h g_h(i)^2 sum_t nu_t A[h,t,i]^2)^{1/2},  g_h(i)^2 = ||Z_h[i]||^2 + sigma_h^2,
+// lanes over the heads, and per-block sums of e (the mean normalises ebar in pass 2).
 __global__ void k_assign_gap(const float* __restrict__ cos, const int32_t* __restrict__ support,
                              const int32_t* __restrict__ slot, const int32_t* toff, int B, int N,
-                             int K, int Tmax, float* delta, double* dpart, int nA,
-                             uint32_t* status) {
+                             int K, int Tmax, int H, const float* __restrict__ omega,
+                             const float* __restrict__ zn2, const float* __restrict__ sigma,
+                             const float* __restrict__ W2, float* energy, float* epart,
+                             float* delta, double* dpart, int nA, uint32_t* status) {
   __shared__ double sd[ASSIGN_WARPS];
   __shared__ int sc[ASSIGN_WARPS];
+  __shared__ float se[ASSIGN_WARPS];
   extern __shared__ int sS[];  // the support of the image, staged once per block
   const int b = blockIdx.y;
   const TextGeom tg = text_geom(toff, b, B, Tmax, status);
@@ -28,6 +34,17 @@ __global__ void k_assign_gap(const float* __restrict__ cos, const int32_t* __res
   const int i = blockIdx.x * ASSIGN_WARPS + w;
   for (int k = threadIdx.x; k < K; k += blockDim.x) sS[k] = support[(size_t)b * K + k];
   __syncthreads();
+  float e = 0.f;
+  if (i < N) {
+    float e2 = 0.f;
+    for (int h = lane; h < H; h += 32) {
+      const size_t o = ((size_t)b * H + h) * N + i;
+      const float sg = sigma[(size_t)b * H + h];
+      e2 = fmaf(omega[(size_t)b * H + h] * (zn2[o] + sg * sg), W2[o], e2);
+    }
+    e = sqrtf(warp_sum(e2));
+    if (lane == 0) energy[(size_t)b * N + i] = e;
+  }
   double dv = 0.0;
   int dc = 0;
   if (i < N && slot[(size_t)b * N + i] < 0) {
@@ -55,17 +72,21 @@ __global__ void k_assign_gap(const float* __restrict__ cos, const int32_t* __res
   if (lane == 0) {
     sd[w] = dv;
     sc[w] = dc;
+    se[w] = e;
   }
   __syncthreads();
   if (threadIdx.x == 0) {
     double s = 0.0;
     int c = 0;
+    float es = 0.f;
     for (int q = 0; q < ASSIGN_WARPS; ++q) {
       s += sd[q];
       c += sc[q];
+      es += se[q];
     }
     dpart[((size_t)b * nA + blockIdx.x) * 2 + 0] = s;
     dpart[((size_t)b * nA + blockIdx.x) * 2 + 1] = (double)c;
+    epart[(size_t)b * nA + blockIdx.x] = es;
   }
 }
 
@@ -157,8 +178,9 @@ cudaError_t launch_assign(const Dims& dm, const gmc_params& p, Scratch& s, const
   cudaError_t e0;
   if ((e0 = set_smem_limit((const void*)k_assign_gap, smem)) != cudaSuccess) return e0;
   if ((e0 = set_smem_limit((const void*)k_assign_pick, smem)) != cudaSuccess) return e0;
-  k_assign_gap<<<grid, 32 * ASSIGN_WARPS, smem, st>>>(s.cos, s.support, s.slot, dm.toff, dm.B, dm.N,
-                                                   dm.K, dm.T, s.delta, s.dpart, s.nA, s.status);
+  k_assign_gap<<<grid, 32 * ASSIGN_WARPS, smem, st>>>(
+      s.cos, s.support, s.slot, dm.toff, dm.B, dm.N, dm.K, dm.T, dm.H, s.omega, s.zn2, s.sigma,
+      s.W2, s.ebar, s.epart, s.delta, s.dpart, s.nA, s.status);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   k_assign_pick<<<grid, 32 * ASSIGN_WARPS, smem, st>>>(

@@ -44,12 +44,12 @@ __global__ void k_head_stats(const float* __restrict__ A, const float* __restric
   const int nhb = (H + HG_HB - 1) / HG_HB, Hp = nhb * HG_HB;
   const int ntiles = nhb * (nhb + 1) / 2;
   float* Abuf = sm_hs;                          // [2][Hp][HG_RS], rows >= H stay zero
-  float* acc = Abuf + 2 * (size_t)Hp * HG_RS;   // [npairs][HG_TOK]
-  float* w2 = acc + (size_t)npairs * HG_TOK;    // [H][HG_TOK]
-  unsigned short* tiles = reinterpret_cast<unsigned short*>(w2 + H * HG_TOK);  // [ntiles]
+  float* acc = Abuf + 2 * (size_t)Hp * HG_RS;   // [2][npairs][HG_TOK], one per block half
+  float* w2 = acc + 2 * (size_t)npairs * HG_TOK;  // [2][H][HG_TOK]
+  unsigned short* tiles = reinterpret_cast<unsigned short*>(w2 + 2 * H * HG_TOK);  // [ntiles]
   const int i0 = blockIdx.x * HG_TOK;
-  for (int p = threadIdx.x; p < npairs * HG_TOK; p += blockDim.x) acc[p] = 0.f;
-  for (int p = threadIdx.x; p < H * HG_TOK; p += blockDim.x) w2[p] = 0.f;
+  for (int p = threadIdx.x; p < 2 * npairs * HG_TOK; p += blockDim.x) acc[p] = 0.f;
+  for (int p = threadIdx.x; p < 2 * H * HG_TOK; p += blockDim.x) w2[p] = 0.f;
   for (int p = H * HG_RS + threadIdx.x; p < Hp * HG_RS; p += blockDim.x) {
     Abuf[p] = 0.f;
     Abuf[(size_t)Hp * HG_RS + p] = 0.f;
@@ -59,7 +59,8 @@ __global__ void k_head_stats(const float* __restrict__ A, const float* __restric
     for (int hb = 0; hb < nhb; ++hb)
       for (int gb = hb; gb < nhb; ++gb) tiles[p++] = (unsigned short)(hb * 256 + gb);
   }
-  // chunks of HG_TC queries, staged with cp.async one chunk ahead (double buffer)
+  // Queries in pairs of HG_TC-chunks: both are staged with cp.async, then the
+  // two halves of the block work on one chunk each into their own sums.
   auto stage = [&](int t0, float* buf) {
     const int tc = min(HG_TC, Tb - t0);
     for (int idx = threadIdx.x; idx < H * HG_TC * HG_TOK; idx += blockDim.x) {
@@ -70,18 +71,19 @@ __global__ void k_head_stats(const float* __restrict__ A, const float* __restric
     }
     cp_async_commit();
   };
-  stage(0, Abuf);
-  for (int t0 = 0, cidx = 0; t0 < Tb; t0 += HG_TC, ++cidx) {
-    const int tc = min(HG_TC, Tb - t0);
-    float* Ablk = Abuf + (size_t)(cidx & 1) * Hp * HG_RS;
-    if (t0 + HG_TC < Tb) {
-      stage(t0 + HG_TC, Abuf + (size_t)((cidx + 1) & 1) * Hp * HG_RS);
-      cp_async_wait<1>();
-    } else {
-      cp_async_wait<0>();
-    }
+  const int hsz = blockDim.x / 2, half = threadIdx.x / hsz, ht = threadIdx.x % hsz;
+  float* accH = acc + (size_t)half * npairs * HG_TOK;
+  float* w2H = w2 + (size_t)half * H * HG_TOK;
+  for (int tp = 0; tp < Tb; tp += 2 * HG_TC) {
+    __syncthreads();  // both buffers are free
+    stage(tp, Abuf);
+    stage(tp + HG_TC, Abuf + (size_t)Hp * HG_RS);
+    cp_async_wait<0>();
     __syncthreads();
-    for (int task = threadIdx.x; task < ntiles * HG_TOK; task += blockDim.x) {
+    const int t0 = tp + half * HG_TC;
+    const int tc = max(0, min(HG_TC, Tb - t0));
+    const float* Ablk = Abuf + (size_t)half * Hp * HG_RS;
+    for (int task = ht; task < ntiles * HG_TOK; task += hsz) {
       const int tile = task / HG_TOK, ii = task % HG_TOK;
       const int hb = tiles[tile] >> 8, gb = tiles[tile] & 255;
       const float* ah = Ablk + (size_t)hb * HG_HB * HG_RS + ii;
@@ -108,10 +110,10 @@ __global__ void k_head_stats(const float* __restrict__ A, const float* __restric
 #pragma unroll
         for (int v = 0; v < HG_HB; ++v) {
           const int h = hb * HG_HB + u, g = gb * HG_HB + v;
-          if (h <= g && g < H) acc[pair_index(h, g, H) * HG_TOK + ii] += sacc[u][v];
+          if (h <= g && g < H) accH[pair_index(h, g, H) * HG_TOK + ii] += sacc[u][v];
         }
     }
-    for (int q = threadIdx.x; q < H * HG_TOK; q += blockDim.x) {
+    for (int q = ht; q < H * HG_TOK; q += hsz) {
       const int h = q / HG_TOK, ii = q % HG_TOK;
       const float* ah = Ablk + h * HG_RS;
       float sw = 0.f;
@@ -119,10 +121,10 @@ __global__ void k_head_stats(const float* __restrict__ A, const float* __restric
         const float a = ah[tt * HG_TOK + ii];
         sw = fmaf(query_weight(t0 + tt, Tb, wq) * a, a, sw);
       }
-      w2[q] += sw;
+      w2H[q] += sw;
     }
-    __syncthreads();  // the buffer is restaged two chunks later
   }
+  __syncthreads();
   double* out = hgpart + ((size_t)b * nHG + blockIdx.x) * H * H;
   for (int p = threadIdx.x; p < H * H; p += blockDim.x) {
     const int h = p / H, g = p % H;
@@ -136,14 +138,14 @@ __global__ void k_head_stats(const float* __restrict__ A, const float* __restric
       const float4 zh = reinterpret_cast<const float4*>(Z)[((size_t)b * H + h) * N + i];
       const float4 zg = reinterpret_cast<const float4*>(Z)[((size_t)b * H + g) * N + i];
       const float w = fmaf(zh.x, zg.x, fmaf(zh.y, zg.y, fmaf(zh.z, zg.z, fmaf(zh.w, zg.w, sh * sgv))));
-      v = fmaf(w, acc[pi * HG_TOK + ii], v);
+      v = fmaf(w, acc[pi * HG_TOK + ii] + acc[((size_t)npairs + pi) * HG_TOK + ii], v);
     }
     out[h * H + g] = v;
     out[g * H + h] = v;
   }
   for (int q = threadIdx.x; q < H * HG_TOK; q += blockDim.x) {
     const int h = q / HG_TOK, i = i0 + q % HG_TOK;
-    if (i < N) W2[((size_t)b * H + h) * N + i] = w2[q];
+    if (i < N) W2[((size_t)b * H + h) * N + i] = w2[q] + w2[H * HG_TOK + q];
   }
 }
 
@@ -266,21 +268,28 @@ __global__ void k_head_cluster(const double* __restrict__ HGred,
     asg[h] = bk;
   }
   __syncthreads();
-  for (int h = threadIdx.x; h < H; h += blockDim.x) {
+  // sums over heads as warp trees (two heads per lane, fixed order)
+  const int nw = blockDim.x >> 5;
+  for (int h = wid; h < H; h += nw) {
     double d = 0.0;
-    for (int g = 0; g < H; ++g)
-      if (asg[g] == asg[h]) d += cs[h * H + g];
-    dot[h] = d;
+    if (lane < H && asg[lane] == asg[h]) d += cs[h * H + lane];
+    if (lane + 32 < H && asg[lane + 32] == asg[h]) d += cs[h * H + lane + 32];
+    d = warp_sum(d);
+    if (lane == 0) dot[h] = d;
   }
   __syncthreads();
   // ||sum_{g in k} u_g||^2 (in cosine units) = sum over the cluster's dot values
-  for (int k = threadIdx.x; k < nc; k += blockDim.x) {
+  for (int k = wid; k < nc; k += nw) {
     double sk = 0.0;
     int n = 0;
-    for (int h = 0; h < H; ++h)
-      if (asg[h] == k) { sk += dot[h]; ++n; }
-    csum[k] = sk > 0.0 ? 1.0 / sqrt(sk) : 0.0;  // 1 / ||sum_{g in k} u_g||
-    ccnt[k] = n;
+    if (lane < H && asg[lane] == k) { sk += dot[lane]; ++n; }
+    if (lane + 32 < H && asg[lane + 32] == k) { sk += dot[lane + 32]; ++n; }
+    sk = warp_sum(sk);
+    n = warp_sum_int(n);
+    if (lane == 0) {
+      csum[k] = sk > 0.0 ? 1.0 / sqrt(sk) : 0.0;  // 1 / ||sum_{g in k} u_g||
+      ccnt[k] = n;
+    }
   }
   __syncthreads();
   for (int h = threadIdx.x; h < H; h += blockDim.x) {
@@ -288,11 +297,12 @@ __global__ void k_head_cluster(const double* __restrict__ HGred,
     inv[h] = 1.0 / (dh + head_eps);
   }
   __syncthreads();
-  for (int k = threadIdx.x; k < nc; k += blockDim.x) {
+  for (int k = wid; k < nc; k += nw) {
     double sk = 0.0;
-    for (int h = 0; h < H; ++h)
-      if (asg[h] == k) sk += inv[h];
-    isum[k] = sk;
+    if (lane < H && asg[lane] == k) sk += inv[lane];
+    if (lane + 32 < H && asg[lane + 32] == k) sk += inv[lane + 32];
+    sk = warp_sum(sk);
+    if (lane == 0) isum[k] = sk;
   }
   __syncthreads();
   int C = 0;
@@ -312,44 +322,16 @@ __global__ void k_head_cluster(const double* __restrict__ HGred,
   }
 }
 
-// e_i = (sum_h omega_h g_h(i)^2 sum_t nu_t A[h,t,i]^2)^{1/2} per token, and the
-// block sums of e (fixed-order tree).  The normalisation ebar_i = e_i / mean(e)
-// (uniform 1 if the mean vanishes) is applied by its consumer, the assignment.
-__global__ void __launch_bounds__(ENERGY_THREADS) k_energy(
-    const float* __restrict__ omega, const float* __restrict__ zn2,
-    const float* __restrict__ sigma, const float* __restrict__ W2, const int32_t* toff, int B,
-    int N, int Tmax, int H, float* ebar, float* epart, int nE, uint32_t* status) {
-  __shared__ float red[32];
-  const int b = blockIdx.y;
-  const TextGeom tg = text_geom(toff, b, B, Tmax, status);
-  if (tg.T == 0) return;
-  const int i = blockIdx.x * ENERGY_THREADS + threadIdx.x;
-  float e = 0.f;
-  if (i < N) {
-    float e2 = 0.f;
-#pragma unroll 4
-    for (int h = 0; h < H; ++h) {
-      const size_t o = ((size_t)b * H + h) * N + i;
-      const float sg = sigma[(size_t)b * H + h];
-      e2 = fmaf(omega[(size_t)b * H + h] * (zn2[o] + sg * sg), W2[o], e2);
-    }
-    e = sqrtf(e2);
-    ebar[(size_t)b * N + i] = e;
-  }
-  const float tot = block_reduce(e, red, OpAdd(), 0.f);
-  if (threadIdx.x == 0) epart[(size_t)b * nE + blockIdx.x] = tot;
-}
-
 cudaError_t launch_heads(const Dims& dm, const gmc_params& p, Scratch& s, const TraceView& tv,
                          cudaStream_t st) {
   const int H = dm.H, npairs = H * (H + 1) / 2;
   const int nhb = (H + HG_HB - 1) / HG_HB;
-  size_t smem = sizeof(float) * (2 * (size_t)nhb * HG_HB * HG_RS + (size_t)npairs * HG_TOK +
-                                 H * HG_TOK) +
+  size_t smem = sizeof(float) * (2 * (size_t)nhb * HG_HB * HG_RS + 2 * (size_t)npairs * HG_TOK +
+                                 2 * H * HG_TOK) +
                 sizeof(unsigned short) * (nhb * (nhb + 1) / 2) + 16;
   cudaError_t e = set_smem_limit((const void*)k_head_stats, smem);
   if (e != cudaSuccess) return e;
-  k_head_stats<<<dim3(s.nHG, dm.B), 256, smem, st>>>(s.A, s.Z, s.sigma, dm.toff, dm.B, dm.N, dm.T,
+  k_head_stats<<<dim3(s.nHG, dm.B), 512, smem, st>>>(s.A, s.Z, s.sigma, dm.toff, dm.B, dm.N, dm.T,
                                                      H, p.terminal_q_weight, s.hgpart, s.nHG,
                                                      s.W2, s.status);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
@@ -363,9 +345,6 @@ cudaError_t launch_heads(const Dims& dm, const gmc_params& p, Scratch& s, const 
   k_head_cluster<<<dm.B, 256, smem2, st>>>(s.HG, dm.toff, dm.B, dm.N, dm.T, H,
                                           p.max_head_clusters, p.head_eps, s.omega, tv, s.status);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  k_energy<<<dim3(s.nE, dm.B), ENERGY_THREADS, 0, st>>>(s.omega, s.zn2, s.sigma, s.W2, dm.toff,
-                                                        dm.B, dm.N, dm.T, H, s.ebar, s.epart,
-                                                        s.nE, s.status);
   return cudaGetLastError();
 }
 

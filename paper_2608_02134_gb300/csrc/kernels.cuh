@@ -74,7 +74,6 @@ constexpr int ROWS_PER_BLOCK = 8;  // rownorm / probe / client builder blocks
 constexpr int HG_TOK = 8;          // tokens per head-statistics block
 constexpr int ASSIGN_WARPS = 8;    // tokens per assignment block
 constexpr int PROBE_TOK = 32;       // tokens per probe block
-constexpr int ENERGY_THREADS = 256;  // tokens per block of the message-energy kernel
 
 // Launch wrappers.  Each returns the first CUDA error it saw.
 cudaError_t launch_rownorm(const Dims&, const void* hidden, float norm_eps, Scratch&, cudaStream_t);
