@@ -15,10 +15,13 @@
 namespace gmc {
 
 struct RowInfo {
-  int kind;     // 0 grounded, 1 appearance, 2 spatial, -1 none
-  int a, c;     // grounded: (h, t); appearance: (m, -); spatial: (la, lb)
-  float scale;  // multiplies the unnormalised value
-  float shift;  // subtracted inside exp (row max of the logit)
+  int kind;       // 0 grounded, 1 appearance, 2 spatial, -1 none
+  size_t src;     // grounded: A row offset; appearance: cos row offset
+  size_t zrow;    // grounded: ||Z_h||^2 row offset
+  float scale;    // multiplies the unnormalised value
+  float shift;    // appearance: row max of the cosine; spatial: smallest distance^2
+  float sg2;      // grounded: sigma_h^2
+  float ly, lx;   // spatial: landmark coordinates
 };
 
 __global__ void __launch_bounds__(256) k_build_clients(
@@ -37,13 +40,18 @@ __global__ void __launch_bounds__(256) k_build_clients(
   if (r0 >= Mb) return;
   {
     const int m = r0 + w;
-    RowInfo inf{-1, 0, 0, 0.f, 0.f};
+    RowInfo inf{-1, 0, 0, 0.f, 0.f, 0.f, 0.f, 0.f};
     if (m < MG) {
       const int h = m / Tb, t = m % Tb;
       float rsv = 0.f;  // parts over key splits, fixed order
       for (int q = 0; q < nRS; ++q) rsv += rs[(((size_t)b * H + h) * nRS + q) * Tmax + t];
       const float nu = (t == Tb - 1 ? wq : 1.f) / ((float)(Tb - 1) + wq);
-      inf = RowInfo{0, h, t, rsv > 0.f ? beta_G * omega[(size_t)b * H + h] * nu / rsv : 0.f, 0.f};
+      const float sg = sigma[(size_t)b * H + h];
+      inf.kind = 0;
+      inf.src = (((size_t)b * H + h) * Tmax + t) * N;
+      inf.zrow = ((size_t)b * H + h) * N;
+      inf.scale = rsv > 0.f ? beta_G * omega[(size_t)b * H + h] * nu / rsv : 0.f;
+      inf.sg2 = sg * sg;
     } else if (m < MG + N) {
       const int a = m - MG;
       const float* row = cos + ((size_t)b * N + a) * N;
@@ -53,7 +61,10 @@ __global__ void __launch_bounds__(256) k_build_clients(
       float z = 0.f;
       for (int j = lane; j < N; j += 32) z += expf((row[j] - mx) / tau_v);
       z = warp_sum(z);
-      inf = RowInfo{1, a, 0, beta_V / ((float)N * z), mx};
+      inf.kind = 1;
+      inf.src = ((size_t)b * N + a) * N;
+      inf.scale = beta_V / ((float)N * z);
+      inf.shift = mx;
     } else if (m < Mb) {
       const int l = m - MG - N;
       const int la = l / L, lb = l % L;
@@ -70,28 +81,31 @@ __global__ void __launch_bounds__(256) k_build_clients(
         z += expf(-(dy * dy + dx * dx - mn) / tau_s);
       }
       z = warp_sum(z);
-      inf = RowInfo{2, la, lb, beta_S / ((float)(L * L) * z), mn};
+      inf.kind = 2;
+      inf.scale = beta_S / ((float)(L * L) * z);
+      inf.shift = mn;
+      inf.ly = ly;
+      inf.lx = lx;
     }
     if (lane == 0) ri[w] = inf;
   }
   __syncthreads();
   const int nrows = min(ROWS_PER_BLOCK, Mb - r0);
+  const float itv = 1.f / tau_v, its = 1.f / tau_s;
   for (int j = threadIdx.x; j < N; j += blockDim.x) {
     long long colsum = 0;
-    const float py = ((j / gw) + 0.5f) / gh, px = ((j % gw) + 0.5f) / gw;
+    const int jr = j / gw;
+    const float py = (jr + 0.5f) / gh, px = ((j - jr * gw) + 0.5f) / gw;
     for (int q = 0; q < nrows; ++q) {
-      const RowInfo inf = ri[q];
+      const RowInfo& inf = ri[q];
       float v = 0.f;
       if (inf.kind == 0) {
-        const size_t o = ((size_t)b * H + inf.a) * N + j;
-        const float sg = sigma[(size_t)b * H + inf.a];
-        const float a = A[(((size_t)b * H + inf.a) * Tmax + inf.c) * N + j];
-        v = a * sqrtf(zn2[o] + sg * sg) * inf.scale;
+        v = A[inf.src + j] * sqrtf(zn2[inf.zrow + j] + inf.sg2) * inf.scale;
       } else if (inf.kind == 1) {
-        v = expf((cos[((size_t)b * N + inf.a) * N + j] - inf.shift) / tau_v) * inf.scale;
+        v = expf((cos[inf.src + j] - inf.shift) * itv) * inf.scale;
       } else if (inf.kind == 2) {
-        const float dy = py - (inf.a + 0.5f) / L, dx = px - (inf.c + 0.5f) / L;
-        v = expf(-(dy * dy + dx * dx - inf.shift) / tau_s) * inf.scale;
+        const float dy = py - inf.ly, dx = px - inf.lx;
+        v = expf((inf.shift - (dy * dy + dx * dx)) * its) * inf.scale;
       }
       if (check && !isfinite(v)) set_status(status, GMC_STATUS_NONFINITE);
       C[((size_t)b * M + r0 + q) * N + j] = v;
