@@ -32,7 +32,8 @@ sys.path.insert(0, ROOT)
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--steps", type=int, default=None,
+                    help="timed steps (default 400 for gmc: about 0.3 s, several clock samples; 5 for the oracle)")
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--workload", default="qwen")
     ap.add_argument("--impl", default="gmc", choices=["gmc", "reference"])
@@ -101,7 +102,7 @@ class ClockSampler:
     def __enter__(self):
         try:
             self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.idx}", f"--query-gpu={self.Q}",
-                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                          "--format=csv,noheader,nounits", "-lms", "50"],
                                          stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.th = threading.Thread(target=self._read, daemon=True)
             self.th.start()
@@ -405,6 +406,8 @@ def run_reference(args):
 
 def main():
     args = parse()
+    if args.steps is None:
+        args.steps = 5 if args.impl == "reference" else 400
     if args.oracle_sample:
         print(json.dumps(oracle_sample(args.oracle_sample, args.oracle_n)))
         return
