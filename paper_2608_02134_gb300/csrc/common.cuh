@@ -90,6 +90,10 @@ __device__ __forceinline__ void cp_async4(void* smem, const void* src, bool pred
                "r"(pred ? 4 : 0)
                : "memory");
 }
+__device__ __forceinline__ void cp_async16(void* smem, const void* src) {
+  const unsigned sa = (unsigned)__cvta_generic_to_shared(smem);
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(sa), "l"(src) : "memory");
+}
 __device__ __forceinline__ void cp_async_commit() {
   asm volatile("cp.async.commit_group;" ::: "memory");
 }

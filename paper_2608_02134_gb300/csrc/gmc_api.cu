@@ -95,8 +95,11 @@ size_t carve_compress(const Dims& dm, Scratch* s, char* base, R0State* r0s = nul
   t.nA = ceil_div(dm.N, ASSIGN_WARPS);
   t.nE = t.nA;  // energy block sums come from the assignment gap kernel
   t.nSel = 0;
-  t.status = c.take<uint32_t>(4 + B);  // status word, then one probe ticket per image
+  // status word, one probe ticket per image, then the carrier membership
+  // bitmaps: one block, zeroed by one memset per call
+  t.status = c.take<uint32_t>(4 + B + B * K * (size_t)ceil_div(dm.N, 32));
   t.tick = t.status + 4;
+  t.mbits = t.tick + B;
   t.A = c.take<float>(B * H * T * N);
   t.nRS = message_splits(dm);
   t.rs = c.take<float>(B * H * (size_t)t.nRS * T);
@@ -371,7 +374,9 @@ int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* 
     GMC_TRY(cudaMemsetAsync(trace, 0, (size_t)dm.B * L.bytes_per_image, st));
   }
   std::lock_guard<std::mutex> lk(g_prof.mu);
-  GMC_TRY(cudaMemsetAsync(s.status, 0, sizeof(uint32_t) * (4 + dm.B), st));  // status, probe tickets
+  // status, probe tickets, membership bitmaps
+  GMC_TRY(cudaMemsetAsync(
+      s.status, 0, sizeof(uint32_t) * (4 + dm.B + (size_t)dm.B * dm.K * ceil_div(dm.N, 32)), st));
   if (Ke == N) {  // K = N returns the unmodified execution
     GMC_TRY(launch_identity(dm, hidden, keys, pos_ids, out_idx, out_hidden, out_kv, out_pos,
                             s.status, st));
@@ -412,7 +417,7 @@ int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* 
   GMC_STAGE("assign", 2, launch_assign(dm, p, s, tv, st));
   GMC_STAGE("transport", 1,
             launch_transport(dm, p, hidden, keys, pos_ids, s.support, s.pi, s.mass, s.rmsh,
-                             out_idx, out_hidden, out_kv, out_pos, s.status, st));
+                             s.mbits, out_idx, out_hidden, out_kv, out_pos, s.status, st));
   g_prof.valid = g_prof.on;
   return GMC_OK;
 }
@@ -555,8 +560,8 @@ int gmc_transport(const gmc_problem* prob, const gmc_params* params, const void*
   const Dims dm = make_dims(prob, p, N, T, 0, d, D, K);
   GMC_TRY(cudaMemsetAsync(status, 0, sizeof(uint32_t), st));
   GMC_TRY(launch_rms_rows(dm, hidden, rmsh, status, st));
-  GMC_TRY(launch_transport(dm, p, hidden, keys, pos_ids, support, assign, weights, rmsh, out_idx,
-                           out_hidden, out_kv, out_pos, status, st));
+  GMC_TRY(launch_transport(dm, p, hidden, keys, pos_ids, support, assign, weights, rmsh, nullptr,
+                           out_idx, out_hidden, out_kv, out_pos, status, st));
   g_launches += 3;
   return GMC_OK;
 }

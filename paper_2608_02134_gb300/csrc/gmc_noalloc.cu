@@ -94,7 +94,7 @@ extern "C" int gmc_transport_noalloc(const gmc_problem* prob, const gmc_params* 
   if ((e = cudaMemsetAsync(status, 0, sizeof(uint32_t), st)) != cudaSuccess ||
       (e = launch_rms_rows(dm, hidden, rmsh, status, st)) != cudaSuccess ||
       (e = launch_transport(dm, p, hidden, keys, pos_ids, support, assign, weights, rmsh,
-                            out_idx, out_hidden, out_kv, out_pos, status, st)) != cudaSuccess) {
+                            nullptr, out_idx, out_hidden, out_kv, out_pos, status, st)) != cudaSuccess) {
     cudaGetLastError();
     return GMC_ERR_CUDA;
   }

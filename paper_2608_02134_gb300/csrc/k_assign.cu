@@ -7,7 +7,10 @@
 //   g_i = exp(-(delta_i / ambig_margin)^gate_pow)
 //   pi(i) = argmax_{j in S} cos_ij + lambda_p s_x g_i exp(-||p_i - p_j||^2 / tau_s)
 // (ties to the lowest j); selected tokens represent themselves.  The
-// population weights are m_i = (1 - alpha s_x) + alpha s_x ebar_i.
+// population weights are m_i = (1 - alpha s_x) + alpha s_x ebar_i.  Token i
+// also sets bit i of its carrier's membership bitmap (atomicOr: the bitmap
+// does not depend on the order of the writes), which the transport reads
+// instead of scanning the whole assignment.
 #include "common.cuh"
 #include "kernels.cuh"
 
@@ -98,7 +101,8 @@ __global__ void k_assign_pick(const float* __restrict__ cos, const int32_t* __re
                               int nE, const int32_t* toff, int B, int N,
                               int K, int Tmax, int gh, int gw, float gate_scale, float gate_pow,
                               float ambig_margin, float lambda_p, float tau_s, float alpha,
-                              int32_t* pi, float* mass, TraceView tv, uint32_t* status) {
+                              int32_t* pi, float* mass, uint32_t* mbits, TraceView tv,
+                              uint32_t* status) {
   __shared__ float gate[3];      // dbar, s_x, mean energy
   extern __shared__ int sS[];  // the support of the image, staged once per block
   const int b = blockIdx.y;
@@ -163,6 +167,9 @@ __global__ void k_assign_pick(const float* __restrict__ cos, const int32_t* __re
   if (lane == 0) {
     pi[(size_t)b * N + i] = choice;
     mass[(size_t)b * N + i] = m;
+    const int nw = (N + 31) >> 5;
+    const int ks = slot[(size_t)b * N + choice];  // choice is in the support
+    atomicOr(&mbits[((size_t)b * K + ks) * nw + (i >> 5)], 1u << (i & 31));
     if (tv.base) {
       tv.at<int32_t>(b, tv.off_pi)[i] = choice;
       tv.at<float>(b, tv.off_mass)[i] = m;
@@ -187,7 +194,7 @@ cudaError_t launch_assign(const Dims& dm, const gmc_params& p, Scratch& s, const
       s.cos, s.support, s.slot, s.delta, s.dpart, s.nA, s.ebar, s.epart, s.nE, dm.toff, dm.B,
       dm.N, dm.K, dm.T,
       dm.gh, dm.gw, p.gate_scale, p.gate_pow, p.ambig_margin, p.assign_spatial_w, p.tau_s,
-      p.pop_strength, s.pi, s.mass, tv, s.status);
+      p.pop_strength, s.pi, s.mass, s.mbits, tv, s.status);
   return cudaGetLastError();
 }
 

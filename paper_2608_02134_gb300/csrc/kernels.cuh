@@ -63,6 +63,7 @@ struct Scratch {
   double* dpart;     // [B][nA][2]     partial sums of delta and counts over discarded tokens
   float* epart;      // [B][nE]        block sums of the message energies e_i
   int32_t* pi;       // [B][N]
+  uint32_t* mbits;   // [B][K][ceil(N/32)] members of each carrier slot, bit i = token i
   float* mass;       // [B][N]
   double* selpart;   // [B][64]        select-path total mass partials
   int32_t* fexp;     // [B]            select-path fixed-point exponents
@@ -109,9 +110,9 @@ cudaError_t launch_assign(const Dims&, const gmc_params&, Scratch&, const TraceV
                           cudaStream_t);
 cudaError_t launch_transport(const Dims&, const gmc_params&, const void* hidden, const void* keys,
                              const int32_t* pos, const int32_t* support, const int32_t* pi,
-                             const float* mass, const float* rmsh, int32_t* out_idx,
-                             void* out_hidden, void* out_kv, int32_t* out_pos, uint32_t* status,
-                             cudaStream_t);
+                             const float* mass, const float* rmsh, const uint32_t* mbits,
+                             int32_t* out_idx, void* out_hidden, void* out_kv, int32_t* out_pos,
+                             uint32_t* status, cudaStream_t);
 cudaError_t launch_identity(const Dims&, const void* hidden, const void* keys, const int32_t* pos,
                             int32_t* out_idx, void* out_hidden, void* out_kv, int32_t* out_pos,
                             uint32_t* status, cudaStream_t);
