@@ -12,10 +12,12 @@
 // work).  In each CTA warp 0 / lane 0 streams 64-wide K slices of both row
 // blocks with TMA (128-byte swizzle) through a 6-stage mbarrier ring; warp 1 /
 // lane 0 issues tcgen05.mma (M = N = 128, K = 16) into a 128-column TMEM
-// accumulator.  Then each CTA parks the column half its peer finishes in its
-// own shared memory, and finishes its half with the peer's partial read over
-// distributed shared memory: one fp32 addition of two partials, the same value
-// in both orders.  The last, ragged tile of an image is shifted inward (start
+// accumulator; warps 2 and 3 stage the tile's reciprocal row and column norms.
+// Then each CTA parks the column half its peer finishes in its own shared
+// memory, and finishes its half with the peer's partial read over distributed
+// shared memory: one fp32 addition of two partials, the same value in both
+// orders.  The epilogue runs on all 16 warps: warp w reads TMEM lane quarter
+// w % 4 and 16 of the half's 64 columns.  The last, ragged tile of an image is shifted inward (start
 // N - 128) so every TMA box lies inside the image's own rows; it stores only
 // the rows and columns the previous tile does not own.
 #include <cooperative_groups.h>
@@ -30,6 +32,7 @@ namespace gmc {
 
 namespace {
 constexpr int BM = 128, BK = 64, STAGES = 6;
+constexpr int GRAM_THREADS = 512;  // 16 warps: 4 TMEM lane quarters x 4 column groups
 constexpr int TILE_BYTES = BM * BK * 2;  // 16 KiB per operand per stage
 constexpr long long WAIT_CYCLES = 4000000000LL;  // about two seconds
 
@@ -39,12 +42,14 @@ struct GramCtl {
   uint64_t done;
   uint32_t tmem;
   volatile int abort;
+  float rnr[BM];  // reciprocal norms of the tile's rows
+  float rnc[BM];  // and of its columns
 };
 
 constexpr size_t GRAM_SMEM = 1024 + 2 * STAGES * TILE_BYTES + sizeof(GramCtl);
 }  // namespace
 
-__global__ void __launch_bounds__(128, 1)
+__global__ void __launch_bounds__(GRAM_THREADS, 1)
     k_gram_tc(const __grid_constant__ CUtensorMap tmap, const int32_t* toff, int B, int N,
               int Tmax, int D, const float* __restrict__ rn, float* cos, uint32_t* status) {
   extern __shared__ uint8_t sm_raw[];
@@ -131,29 +136,32 @@ __global__ void __launch_bounds__(128, 1)
       tc::mma_commit(&ctl->done);  // also on abort, so the epilogue wakes up
     }
     __syncwarp();
+  } else if (warp < 4) {
+    // reciprocal norms of the tile's rows (warp 2) and columns (warp 3)
+    const int o = warp == 2 ? r0 : c0;
+    float* dst = warp == 2 ? ctl->rnr : ctl->rnc;
+    for (int q = lane; q < BM; q += 32) dst[q] = rn[(size_t)b * N + o + q];
   }
 
-  bool ok = tc::mbar_wait(&ctl->done, 0, deadline);
-  ok = __all_sync(FULL, ok && !ctl->abort);
+  bool ok = tc::mbar_wait(&ctl->done, 0, deadline) && !ctl->abort;
+  ok = __syncthreads_and(ok);  // also publishes the norms
   tc::fence_after_sync();
-  const int row = warp * 32 + lane;  // this thread's TMEM lane = tile row
+  const int quarter = warp & 3, grp = warp >> 2;
+  const int row = quarter * 32 + lane;  // this thread's TMEM lane = tile row
   // the column half the peer finishes, column-major [64][128] in the (now idle)
   // operand ring; a CTA without K slices contributes zeros
   float* park = reinterpret_cast<float*>(tilesA);
-  const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+  const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
   if (ok) {
-#pragma unroll 1
-    for (int cc = 0; cc < 2; ++cc) {
-      float v[32];
-      if (nk > 0) {
-        tc::tmem_ld32(trow + (uint32_t)((1 - kpart) * 64 + cc * 32), v);
-      } else {
+    float v[16];
+    if (nk > 0) {
+      tc::tmem_ld16(trow + (uint32_t)((1 - kpart) * 64 + grp * 16), v);
+    } else {
 #pragma unroll
-        for (int q = 0; q < 32; ++q) v[q] = 0.f;
-      }
-#pragma unroll
-      for (int q = 0; q < 32; ++q) park[(cc * 32 + q) * BM + row] = v[q];
+      for (int q = 0; q < 16; ++q) v[q] = 0.f;
     }
+#pragma unroll
+    for (int q = 0; q < 16; ++q) park[(grp * 16 + q) * BM + row] = v[q];
   }
   tc::fence_before_sync();
   cluster.sync();  // both parked halves are complete
@@ -162,39 +170,36 @@ __global__ void __launch_bounds__(128, 1)
     const float* peer = cluster.map_shared_rank(park, 1 - kpart);
     const int i = r0 + row;  // output row
     const bool own_row = i >= I * BM;
-    const float ri = rn[(size_t)b * N + i];
-    float* crow = cos + ((size_t)b * N + i) * N;
-#pragma unroll 1
-    for (int cc = 0; cc < 2; ++cc) {
-      float v[32];
-      if (nk > 0) {
-        tc::tmem_ld32(trow + (uint32_t)(kpart * 64 + cc * 32), v);
-      } else {
+    const float ri = ctl->rnr[row];
+    float v[16];
+    if (nk > 0) {
+      tc::tmem_ld16(trow + (uint32_t)(kpart * 64 + grp * 16), v);
+    } else {
 #pragma unroll
-        for (int q = 0; q < 32; ++q) v[q] = 0.f;
-      }
-      const int j0 = c0 + kpart * 64 + cc * 32;
+      for (int q = 0; q < 16; ++q) v[q] = 0.f;
+    }
+    const int jl = kpart * 64 + grp * 16;  // first column of this warp, within the tile
+    const int j0 = c0 + jl;
 #pragma unroll
-      for (int q = 0; q < 32; ++q) {
+    for (int q = 0; q < 16; ++q)
+      v[q] = (v[q] + peer[(grp * 16 + q) * BM + row]) * ri * ctl->rnc[jl + q];
+    // own rows: the warp's 32 x 16 block goes through shared memory (padded
+    // rows), then every store instruction writes two 64-byte row segments
+    float* st = reinterpret_cast<float*>(tilesB) + warp * (32 * 17);
+#pragma unroll
+    for (int q = 0; q < 16; ++q) st[lane * 17 + q] = v[q];
+    __syncwarp();
+#pragma unroll 4
+    for (int k = 0; k < 16; ++k) {
+      const int rr = 2 * k + (lane >> 4), cq = lane & 15;  // block row, column
+      const int ii = r0 + quarter * 32 + rr, jj = j0 + cq;
+      if (ii >= I * BM && jj >= J * BM) cos[((size_t)b * N + ii) * N + jj] = st[rr * 17 + cq];
+    }
+    if (I != J) {  // mirror: row j of the transposed block, coalesced over the warp's lanes
+#pragma unroll
+      for (int q = 0; q < 16; ++q) {
         const int j = j0 + q;
-        v[q] = (v[q] + peer[(cc * 32 + q) * BM + row]) * ri * rn[(size_t)b * N + j];
-      }
-      if (own_row) {
-        if (j0 >= J * BM) {
-#pragma unroll
-          for (int q = 0; q < 32; q += 4)
-            *reinterpret_cast<float4*>(crow + j0 + q) = make_float4(v[q], v[q + 1], v[q + 2], v[q + 3]);
-        } else {
-          for (int q = 0; q < 32; ++q)
-            if (j0 + q >= J * BM) crow[j0 + q] = v[q];
-        }
-      }
-      if (I != J) {  // mirror: row j of the transposed block, coalesced over the warp's lanes
-#pragma unroll
-        for (int q = 0; q < 32; ++q) {
-          const int j = j0 + q;
-          if (own_row && j >= J * BM) cos[((size_t)b * N + j) * N + i] = v[q];
-        }
+        if (own_row && j >= J * BM) cos[((size_t)b * N + j) * N + i] = v[q];
       }
     }
   }
@@ -264,7 +269,7 @@ cudaError_t launch_gram_tc(const Dims& dm, const void* hidden, Scratch& s, cudaS
   const int nt = ceil_div(dm.N, BM);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(2 * (nt * (nt + 1) / 2), dm.B);
-  cfg.blockDim = dim3(128);
+  cfg.blockDim = dim3(GRAM_THREADS);
   cfg.dynamicSmemBytes = GRAM_SMEM;
   cfg.stream = st;
   cudaLaunchAttribute attr[1];

@@ -24,6 +24,8 @@ def _cos_ref(h64: torch.Tensor) -> torch.Tensor:
     (1, 16, 8, 256, [5], torch.bfloat16),          # exactly one 128-row tile
     (3, 10, 20, 512, [7, 1, 30], torch.bfloat16),  # shifted last tile, ragged text offsets
     (2, 24, 24, 4096, [32, 32], torch.bfloat16),
+    (2, 12, 12, 128, [9, 1], torch.bfloat16),      # 2 x 2 tiles, 16-row ragged edge, T_b = 1
+    (1, 13, 11, 256, [4], torch.bfloat16),         # N % 4 != 0: CUDA-core path
     (1, 10, 10, 40, [3], torch.float32),           # CUDA-core path
 ])
 def test_cosine_matches_fp64_reference(B, gh, gw, D, tlens, dtype):
