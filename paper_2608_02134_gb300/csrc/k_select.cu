@@ -643,32 +643,41 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
           }
           if (threadIdx.x == 0) s.cstart[N] = live;
         }
-        // chunks of CU entries per thread: every thread reads its chunk before the
-        // scan's barriers and writes after them, always at or below the source
+        // chunks of 32 CU entries per warp, entry seg + 32 u + lane read by
+        // lane (bank-conflict free); ballots keep the order.  Every thread reads
+        // before the scan's barriers and writes after them, always at or below
+        // the source.
         int dst = 0;
+        const unsigned lt = (1u << lane) - 1u;
         for (int base = 0; base < tot; base += SEL_THREADS * CU) {
-          const int p0 = base + threadIdx.x * CU;
+          const int seg = base + wid * (32 * CU);
           uint16_t mq[CU], mj[CU];
           float mc[CU];
-          unsigned m = 0;
+          unsigned bal[CU];
+          int wcount = 0;
 #pragma unroll
           for (int u = 0; u < CU; ++u) {
-            const bool in = p0 + u < tot;
-            mq[u] = in ? s.srows[p0 + u] : (uint16_t)DEADROW;
-            mj[u] = in ? s.scols[p0 + u] : (uint16_t)0;
-            mc[u] = in ? s.svals[p0 + u] : 0.f;
-            m |= (unsigned)(mq[u] != DEADROW) << u;
+            const int p = seg + u * 32 + lane;
+            const bool in = p < tot;
+            mq[u] = in ? s.srows[p] : (uint16_t)DEADROW;
+            mj[u] = in ? s.scols[p] : (uint16_t)0;
+            mc[u] = in ? s.svals[p] : 0.f;
+            bal[u] = __ballot_sync(FULL, mq[u] != DEADROW);
+            wcount += __popc(bal[u]);
           }
           int chunk_live = 0;
-          const int ex = dst + block_exclusive_scan(__popc(m), s.wsum, &chunk_live);
+          int off = dst + block_exclusive_scan(lane == 0 ? wcount : 0, s.wsum, &chunk_live);
+          off = __shfl_sync(FULL, off, 0);
 #pragma unroll
-          for (int u = 0; u < CU; ++u)
-            if ((m >> u) & 1u) {
-              const int d = ex + __popc(m & ((1u << u) - 1u));
+          for (int u = 0; u < CU; ++u) {
+            if ((bal[u] >> lane) & 1u) {
+              const int d = off + __popc(bal[u] & lt);
               s.srows[d] = mq[u];
               s.scols[d] = mj[u];
               s.svals[d] = mc[u];
             }
+            off += __popc(bal[u]);
+          }
           dst += chunk_live;
         }
         __syncthreads();
