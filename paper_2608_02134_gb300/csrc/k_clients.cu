@@ -6,6 +6,11 @@
 //   appearance m = 0..N-1:       beta_V / N * softmax_i(cos_mi / tau_v)
 //   spatial    l = 0..L*L-1:     beta_S / L^2 * softmax_i(-||p_i - l_l||^2 / tau_s)
 // with p_i = ((r+.5)/gh, (c+.5)/gw) and landmarks ((a+.5)/L, (b+.5)/L).
+// The spatial softmax separates over the grid: ||p_i - l||^2 = dy_r^2 + dx_c^2,
+// so its smallest distance is min dy^2 + min dx^2 and its normaliser is
+// (sum_r exp(-dy_r^2 / tau_s)) (sum_c exp(-dx_c^2 / tau_s)) (each factor
+// shifted by its own minimum): gh + gw terms instead of N.  The appearance
+// row's max and normaliser come from one online pass over the cosine row.
 // The column sums u0_i = sum_m Cbar_mi (the singleton gains of the empty
 // support) are accumulated in 64-bit fixed point, so they are exact sums of
 // the fp32 entries and independent of the order the blocks finish in.
@@ -15,16 +20,46 @@
 namespace gmc {
 
 struct RowInfo {
-  int kind;       // 0 grounded, 1 appearance, 2 spatial, -1 none
-  size_t src;     // grounded: A row offset; appearance: cos row offset
-  size_t zrow;    // grounded: ||Z_h||^2 row offset
-  float scale;    // multiplies the unnormalised value
-  float shift;    // appearance: row max of the cosine; spatial: smallest distance^2
-  float sg2;      // grounded: sigma_h^2
-  float ly, lx;   // spatial: landmark coordinates
+  int kind;        // 0 grounded, 1 appearance, 2 spatial, -1 none
+  const float* x;  // grounded: A row; appearance: cosine row; else nullptr
+  const float* z;  // grounded: ||Z_h||^2 row; else nullptr
+  float scale;     // multiplies the unnormalised value
+  float shift;     // appearance: row max of the cosine; spatial: smallest distance^2
+  float sg2;       // grounded: sigma_h^2
+  float ly, lx;    // spatial: landmark coordinates
 };
 
-__global__ void __launch_bounds__(256) k_build_clients(
+// Online (max, sum of exp((x - max) / tau)) of a row, one lane's share: 8
+// loads in flight at a time; the running sum is rescaled when a group of 8
+// raises the max.
+__device__ __forceinline__ void row_softmax_stats(const float* row, int N, float itau, int lane,
+                                                  float& m, float& z) {
+  m = -INFINITY;
+  z = 0.f;
+  for (int j0 = lane; j0 < N; j0 += 32 * 8) {
+    float x[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) x[u] = j0 + 32 * u < N ? row[j0 + 32 * u] : -INFINITY;
+    float m8 = x[0];
+#pragma unroll
+    for (int u = 1; u < 8; ++u) m8 = fmaxf(m8, x[u]);
+    if (m8 > m) {
+      z = m == -INFINITY ? 0.f : z * expf((m - m8) * itau);
+      m = m8;
+    }
+#pragma unroll
+    for (int u = 0; u < 8; ++u) z += x[u] == -INFINITY ? 0.f : expf((x[u] - m) * itau);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {  // merge the lanes' (max, sum) pairs
+    const float om = __shfl_xor_sync(FULL, m, o), oz = __shfl_xor_sync(FULL, z, o);
+    const float nm = fmaxf(m, om);
+    z = (z == 0.f ? 0.f : z * expf((m - nm) * itau)) + (oz == 0.f ? 0.f : oz * expf((om - nm) * itau));
+    m = nm;
+  }
+}
+
+__global__ void __launch_bounds__(256, 4) k_build_clients(
     const float* __restrict__ A, const float* __restrict__ rs, int nRS, const float* __restrict__ zn2,
     const float* __restrict__ sigma, const float* __restrict__ omega,
     const float* __restrict__ cos, const int32_t* toff, int B, int N, int Tmax, int H, int M,
@@ -40,7 +75,7 @@ __global__ void __launch_bounds__(256) k_build_clients(
   if (r0 >= Mb) return;
   {
     const int m = r0 + w;
-    RowInfo inf{-1, 0, 0, 0.f, 0.f, 0.f, 0.f, 0.f};
+    RowInfo inf{-1, nullptr, nullptr, 0.f, 0.f, 0.f, 0.f, 0.f};
     if (m < MG) {
       const int h = m / Tb, t = m % Tb;
       float rsv = 0.f;  // parts over key splits, fixed order
@@ -48,42 +83,48 @@ __global__ void __launch_bounds__(256) k_build_clients(
       const float nu = (t == Tb - 1 ? wq : 1.f) / ((float)(Tb - 1) + wq);
       const float sg = sigma[(size_t)b * H + h];
       inf.kind = 0;
-      inf.src = (((size_t)b * H + h) * Tmax + t) * N;
-      inf.zrow = ((size_t)b * H + h) * N;
+      inf.x = A + (((size_t)b * H + h) * Tmax + t) * N;
+      inf.z = zn2 + ((size_t)b * H + h) * N;
       inf.scale = rsv > 0.f ? beta_G * omega[(size_t)b * H + h] * nu / rsv : 0.f;
       inf.sg2 = sg * sg;
     } else if (m < MG + N) {
       const int a = m - MG;
       const float* row = cos + ((size_t)b * N + a) * N;
-      float mx = -INFINITY;
-      for (int j = lane; j < N; j += 32) mx = fmaxf(mx, row[j]);
-      mx = warp_max(mx);
-      float z = 0.f;
-      for (int j = lane; j < N; j += 32) z += expf((row[j] - mx) / tau_v);
-      z = warp_sum(z);
+      float mx, z;
+      row_softmax_stats(row, N, 1.f / tau_v, lane, mx, z);
       inf.kind = 1;
-      inf.src = ((size_t)b * N + a) * N;
+      inf.x = row;
       inf.scale = beta_V / ((float)N * z);
       inf.shift = mx;
     } else if (m < Mb) {
       const int l = m - MG - N;
       const int la = l / L, lb = l % L;
       const float ly = (la + 0.5f) / L, lx = (lb + 0.5f) / L;
-      float mn = INFINITY;
-      for (int j = lane; j < N; j += 32) {
-        const float dy = ((j / gw) + 0.5f) / gh - ly, dx = ((j % gw) + 0.5f) / gw - lx;
-        mn = fminf(mn, dy * dy + dx * dx);
+      float mny = INFINITY, mnx = INFINITY;
+      for (int r = lane; r < gh; r += 32) {
+        const float dy = (r + 0.5f) / gh - ly;
+        mny = fminf(mny, dy * dy);
       }
-      mn = -warp_max(-mn);
-      float z = 0.f;
-      for (int j = lane; j < N; j += 32) {
-        const float dy = ((j / gw) + 0.5f) / gh - ly, dx = ((j % gw) + 0.5f) / gw - lx;
-        z += expf(-(dy * dy + dx * dx - mn) / tau_s);
+      for (int c = lane; c < gw; c += 32) {
+        const float dx = (c + 0.5f) / gw - lx;
+        mnx = fminf(mnx, dx * dx);
       }
-      z = warp_sum(z);
+      mny = -warp_max(-mny);
+      mnx = -warp_max(-mnx);
+      float zy = 0.f, zx = 0.f;
+      for (int r = lane; r < gh; r += 32) {
+        const float dy = (r + 0.5f) / gh - ly;
+        zy += expf(-(dy * dy - mny) / tau_s);
+      }
+      for (int c = lane; c < gw; c += 32) {
+        const float dx = (c + 0.5f) / gw - lx;
+        zx += expf(-(dx * dx - mnx) / tau_s);
+      }
+      zy = warp_sum(zy);
+      zx = warp_sum(zx);
       inf.kind = 2;
-      inf.scale = beta_S / ((float)(L * L) * z);
-      inf.shift = mn;
+      inf.scale = beta_S / ((float)(L * L) * (zy * zx));
+      inf.shift = mny + mnx;
       inf.ly = ly;
       inf.lx = lx;
     }
@@ -96,13 +137,23 @@ __global__ void __launch_bounds__(256) k_build_clients(
     long long colsum = 0;
     const int jr = j / gw;
     const float py = (jr + 0.5f) / gh, px = ((j - jr * gw) + 0.5f) / gw;
-    for (int q = 0; q < nrows; ++q) {
+    // every row's operands are loaded before any is used
+    float xv[ROWS_PER_BLOCK], zv[ROWS_PER_BLOCK];
+#pragma unroll
+    for (int q = 0; q < ROWS_PER_BLOCK; ++q) {
+      const RowInfo& inf = ri[q];
+      xv[q] = q < nrows && inf.x ? inf.x[j] : 0.f;
+      zv[q] = q < nrows && inf.z ? inf.z[j] : 0.f;
+    }
+#pragma unroll
+    for (int q = 0; q < ROWS_PER_BLOCK; ++q) {
+      if (q >= nrows) break;
       const RowInfo& inf = ri[q];
       float v = 0.f;
       if (inf.kind == 0) {
-        v = A[inf.src + j] * sqrtf(zn2[inf.zrow + j] + inf.sg2) * inf.scale;
+        v = xv[q] * sqrtf(zv[q] + inf.sg2) * inf.scale;
       } else if (inf.kind == 1) {
-        v = expf((cos[inf.src + j] - inf.shift) * itv) * inf.scale;
+        v = expf((xv[q] - inf.shift) * itv) * inf.scale;
       } else if (inf.kind == 2) {
         const float dy = py - inf.ly, dx = px - inf.lx;
         v = expf((inf.shift - (dy * dy + dx * dx)) * its) * inf.scale;
