@@ -384,8 +384,7 @@ int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* 
     return GMC_OK;
   }
   const int fx = fixed_point_exponent((double)p.beta_G + p.beta_V + p.beta_S);
-  GMC_TRY(cudaMemsetAsync(s.u0, 0, sizeof(long long) * dm.B * N, st));
-  GMC_TRY(g_prof.begin(st));
+  GMC_TRY(g_prof.begin(st));  // k_probe zeroes the column sums u0 of the client build
   if (g_prof.on) {  // stage timing: every stage in turn on the caller's stream
     GMC_STAGE("rownorm", 1, launch_rownorm(dm, hidden, p.norm_eps, s, st));
     GMC_STAGE("probe", 1, launch_probe(dm, keys, vo_probe, p, s, st));

@@ -56,10 +56,14 @@ template <typename Tin>
 __global__ void __launch_bounds__(256) k_probe(
     const Tin* __restrict__ keys, const float* __restrict__ W, const int32_t* toff, int B, int N,
     int K, int Tmax, int H, int Hkv, int d, float lambda_mass, float eps_mass, float* Z,
-    float* zn2, float* sigpart, int nP, float* sigma, uint32_t* tick, uint32_t* status) {
+    float* zn2, float* sigpart, int nP, float* sigma, uint32_t* tick, long long* u0,
+    uint32_t* status) {
   extern __shared__ float4 sm_probe4[];
   __shared__ int last;
   const int b = blockIdx.z, g = blockIdx.y, pb = blockIdx.x;
+  // the client build's column sums start at zero (it runs after this kernel)
+  if (u0 && g == 0 && threadIdx.x < PR_TOK && pb * PR_TOK + (int)threadIdx.x < N)
+    u0[(size_t)b * N + pb * PR_TOK + threadIdx.x] = 0;
   const TextGeom tg = text_geom(toff, b, B, Tmax, status);
   if (tg.T == 0) return;  // uniform over the image
   const SeqIdx sq(b, N, K, tg.off, tg.T);
@@ -193,13 +197,13 @@ cudaError_t launch_probe(const Dims& dm, const void* keys, const float* W, const
     if ((e = set_smem_limit((const void*)k_probe<__nv_bfloat16>, smem)) != cudaSuccess) return e;
     k_probe<__nv_bfloat16><<<grid, 256, smem, st>>>(
         (const __nv_bfloat16*)keys, W, dm.toff, dm.B, dm.N, dm.K, dm.T, dm.H, dm.Hkv, dm.d,
-        p.lambda_mass, p.eps_mass, s.Z, s.zn2, s.sigpart, s.nP, s.sigma, s.tick, s.status);
+        p.lambda_mass, p.eps_mass, s.Z, s.zn2, s.sigpart, s.nP, s.sigma, s.tick, s.u0, s.status);
   } else {
     if ((e = set_smem_limit((const void*)k_probe<float>, smem)) != cudaSuccess) return e;
     k_probe<float><<<grid, 256, smem, st>>>((const float*)keys, W, dm.toff, dm.B, dm.N, dm.K,
                                             dm.T, dm.H, dm.Hkv, dm.d, p.lambda_mass, p.eps_mass,
                                             s.Z, s.zn2, s.sigpart, s.nP, s.sigma, s.tick,
-                                            s.status);
+                                            s.u0, s.status);
   }
   return cudaGetLastError();
 }

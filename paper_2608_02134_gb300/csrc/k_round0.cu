@@ -22,9 +22,14 @@ constexpr int R0_ROWS = 8;  // rows per block (one warp each)
 
 __global__ void __launch_bounds__(512) k_r0_pool(const long long* __restrict__ u0, int B, int N,
                                                    int P, const int32_t* toff, int Tmax,
-                                                   int32_t* pool0, int32_t* info, uint32_t* status) {
+                                                   int32_t* pool0, int32_t* info, long long* s0,
+                                                   long long* u1, long long* fv, uint32_t* status) {
   extern __shared__ __align__(16) char sm_r0p[];
   const int b = blockIdx.x;
+  // the accumulators of the next two kernels start at zero
+  for (int k = threadIdx.x; k < P; k += blockDim.x) s0[(size_t)b * P + k] = 0;
+  for (int j = threadIdx.x; j < N; j += blockDim.x) u1[(size_t)b * N + j] = 0;
+  if (threadIdx.x < 4) fv[(size_t)b * 4 + threadIdx.x] = 0;
   if (toff && text_geom(toff, b, B, Tmax, nullptr).T == 0) {
     if (threadIdx.x == 0) info[b * 4] = 0;
     return;
@@ -109,6 +114,8 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_filter(
   __shared__ long long sc[GMC_MAX_POOL];
   __shared__ int batch[GMC_MAX_POOL];
   __shared__ long long fb[3];
+  // the block's contributions to the next gains, one global atomic per column at the end
+  extern __shared__ unsigned long long uacc[];  // [N]
   const int b = blockIdx.y;
   const int Pt = info[b * 4];
   if (Pt == 0) return;
@@ -126,6 +133,7 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_filter(
     sc[k] = s0[(size_t)b * P + k];
   }
   if (threadIdx.x < 3) fb[threadIdx.x] = 0;
+  for (int j = threadIdx.x; j < N; j += blockDim.x) uacc[j] = 0;
   __syncthreads();
   {
     const int lane = threadIdx.x & 31, gl = lane & 7;
@@ -153,7 +161,6 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_filter(
     for (int t = lane; t < nb; t += 32) bnew = fmaxf(bnew, vals[batch[t]]);
     bnew = warp_max(bnew);
     const long long fb_new = to_fix(bnew, fxs);
-    long long* ub = u1 + (size_t)b * N;
     int w = 0;
     float rowmax = 0.f;
     if ((N & 3) == 0) {
@@ -194,8 +201,7 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_filter(
                 const int j = 4 * k4 + e2;
                 vals[pos] = c4[e2];
                 cols[pos] = (uint16_t)j;
-                atomicAdd((unsigned long long*)&ub[j],
-                          (unsigned long long)(to_fix(c4[e2], fxs) - fb_new));
+                atomicAdd(&uacc[j], (unsigned long long)(to_fix(c4[e2], fxs) - fb_new));
                 ++pos;
               }
           }
@@ -215,7 +221,7 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_filter(
           const int pos = w + __popc(msk & sel::lanemask_lt());
           vals[pos] = c;
           cols[pos] = (uint16_t)k;
-          atomicAdd((unsigned long long*)&ub[k], (unsigned long long)(to_fix(c, fxs) - fb_new));
+          atomicAdd(&uacc[k], (unsigned long long)(to_fix(c, fxs) - fb_new));
         }
         w += __popc(msk);
       }
@@ -231,6 +237,9 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_filter(
   __syncthreads();
   if (threadIdx.x < 3 && fb[threadIdx.x])
     atomicAdd((unsigned long long*)&fv[(size_t)b * 4 + threadIdx.x], (unsigned long long)fb[threadIdx.x]);
+  unsigned long long* ub = reinterpret_cast<unsigned long long*>(u1 + (size_t)b * N);
+  for (int j = threadIdx.x; j < N; j += blockDim.x)
+    if (uacc[j]) atomicAdd(&ub[j], uacc[j]);
 }
 
 cudaError_t launch_round0(const R0State& r0, int B, int N, int K, int M, const int32_t* toff,
@@ -240,21 +249,19 @@ cudaError_t launch_round0(const R0State& r0, int B, int N, int K, int M, const i
                           cudaStream_t st) {
   const int P = p.pool_mult * p.batch_b;
   cudaError_t e;
-  if ((e = cudaMemsetAsync(r0.s0, 0, sizeof(long long) * B * P, st)) != cudaSuccess) return e;
-  if ((e = cudaMemsetAsync(r0.u1, 0, sizeof(long long) * (size_t)B * N, st)) != cudaSuccess) return e;
-  if ((e = cudaMemsetAsync(r0.fv, 0, sizeof(long long) * B * 4, st)) != cudaSuccess) return e;
-  if ((e = cudaMemsetAsync(r0.info, 0, sizeof(int32_t) * B * 4, st)) != cudaSuccess) return e;
   const size_t smem = sizeof(int) * (sel::HBINS + N + 32 + 8 + 2 * P) + (size_t)N + 64;
   if ((e = set_smem_limit((const void*)k_r0_pool, smem)) != cudaSuccess) return e;
   const int uniform = (H == 0);
   k_r0_pool<<<B, 512, smem, st>>>(u0, B, N, P, uniform ? nullptr : toff, T, r0.pool, r0.info,
-                                  status);
+                                  r0.s0, r0.u1, r0.fv, status);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   dim3 grid(ceil_div(M, R0_ROWS), B);
   k_r0_rho<<<grid, 32 * R0_ROWS, 0, st>>>(C, B, N, M, H, L2, toff, T, uniform, r0.pool, r0.info,
                                           P, p.resp_temp, p.resp_eps, fx_exp, fexp, r0.s0);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  k_r0_filter<<<grid, 32 * R0_ROWS, 0, st>>>(C, scol, B, N, K, M, H, L2, toff, T, uniform, r0.pool,
+  const size_t fsm = sizeof(unsigned long long) * (size_t)N;
+  if ((e = set_smem_limit((const void*)k_r0_filter, fsm)) != cudaSuccess) return e;
+  k_r0_filter<<<grid, 32 * R0_ROWS, fsm, st>>>(C, scol, B, N, K, M, H, L2, toff, T, uniform, r0.pool,
                                              r0.info, r0.s0, P, p.batch_b, fx_exp, fexp, r0.u1,
                                              r0.bcov, r0.cnt, r0.fv, order, tv);
   return cudaGetLastError();
