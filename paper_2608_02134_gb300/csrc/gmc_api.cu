@@ -95,11 +95,13 @@ size_t carve_compress(const Dims& dm, Scratch* s, char* base, R0State* r0s = nul
   t.nA = ceil_div(dm.N, ASSIGN_WARPS);
   t.nE = t.nA;  // energy block sums come from the assignment gap kernel
   t.nSel = 0;
-  // status word, one probe ticket per image, then the carrier membership
-  // bitmaps: one block, zeroed by one memset per call
-  t.status = c.take<uint32_t>(4 + B + B * K * (size_t)ceil_div(dm.N, 32));
+  // status word, one probe and one assignment ticket per image, then the
+  // carrier membership bitmaps: one block, zeroed by one memset per call
+  t.status = c.take<uint32_t>(4 + 2 * B + B * K * (size_t)ceil_div(dm.N, 32));
   t.tick = t.status + 4;
-  t.mbits = t.tick + B;
+  t.tick2 = t.tick + B;
+  t.mbits = t.tick2 + B;
+  t.gatev = c.take<float>(B * 4);
   t.A = c.take<float>(B * H * T * N);
   t.nRS = message_splits(dm);
   t.rs = c.take<float>(B * H * (size_t)t.nRS * T);
@@ -374,9 +376,10 @@ int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* 
     GMC_TRY(cudaMemsetAsync(trace, 0, (size_t)dm.B * L.bytes_per_image, st));
   }
   std::lock_guard<std::mutex> lk(g_prof.mu);
-  // status, probe tickets, membership bitmaps
+  // status, tickets, membership bitmaps
   GMC_TRY(cudaMemsetAsync(
-      s.status, 0, sizeof(uint32_t) * (4 + dm.B + (size_t)dm.B * dm.K * ceil_div(dm.N, 32)), st));
+      s.status, 0, sizeof(uint32_t) * (4 + 2 * dm.B + (size_t)dm.B * dm.K * ceil_div(dm.N, 32)),
+      st));
   if (Ke == N) {  // K = N returns the unmodified execution
     GMC_TRY(launch_identity(dm, hidden, keys, pos_ids, out_idx, out_hidden, out_kv, out_pos,
                             s.status, st));

@@ -20,15 +20,19 @@ namespace gmc {
 // Also the message energy of every token (appendix Eq. (cond-grounded-energy)):
 //   e_i = (sum_h omega_h g_h(i)^2 sum_t nu_t A[h,t,i]^2)^{1/2},  g_h(i)^2 = ||Z_h[i]||^2 + sigma_h^2,
 // lanes over the heads, and per-block sums of e (the mean normalises ebar in pass 2).
+// The last block of an image to finish (ticket) adds the block partials in a
+// fixed order and stores Delta_bar, s_x and the mean energy for pass 2.
 __global__ void k_assign_gap(const float* __restrict__ cos, const int32_t* __restrict__ support,
                              const int32_t* __restrict__ slot, const int32_t* toff, int B, int N,
                              int K, int Tmax, int H, const float* __restrict__ omega,
                              const float* __restrict__ zn2, const float* __restrict__ sigma,
                              const float* __restrict__ W2, float* energy, float* epart,
-                             float* delta, double* dpart, int nA, uint32_t* status) {
+                             float* delta, double* dpart, int nA, float gate_scale,
+                             float gate_pow, uint32_t* tick, float* gatev, uint32_t* status) {
   __shared__ double sd[ASSIGN_WARPS];
   __shared__ int sc[ASSIGN_WARPS];
   __shared__ float se[ASSIGN_WARPS];
+  __shared__ int last;
   extern __shared__ int sS[];  // the support of the image, staged once per block
   const int b = blockIdx.y;
   const TextGeom tg = text_geom(toff, b, B, Tmax, status);
@@ -90,46 +94,48 @@ __global__ void k_assign_gap(const float* __restrict__ cos, const int32_t* __res
     dpart[((size_t)b * nA + blockIdx.x) * 2 + 0] = s;
     dpart[((size_t)b * nA + blockIdx.x) * 2 + 1] = (double)c;
     epart[(size_t)b * nA + blockIdx.x] = es;
+    __threadfence();
+    last = atomicAdd(&tick[b], 1u) == (unsigned)(nA - 1);
+  }
+  __syncthreads();
+  if (last && w == 0) {  // the partials in a fixed order (fp32: at most 2 N per image)
+    __threadfence();
+    float s = 0.f, c = 0.f, et = 0.f;
+    for (int q = lane; q < nA; q += 32) {
+      s += (float)__ldcg(&dpart[((size_t)b * nA + q) * 2 + 0]);
+      c += (float)__ldcg(&dpart[((size_t)b * nA + q) * 2 + 1]);
+      et += __ldcg(&epart[(size_t)b * nA + q]);
+    }
+    s = warp_sum(s);
+    c = warp_sum(c);
+    et = warp_sum(et);
+    if (lane == 0) {
+      const float db = c > 0.f ? s / c : 0.f;
+      gatev[(size_t)b * 4 + 0] = db;
+      gatev[(size_t)b * 4 + 1] = 1.f - expf(-powf(db / gate_scale, gate_pow));
+      gatev[(size_t)b * 4 + 2] = et / (float)N;
+    }
   }
 }
 
 // Pass 2: s_x, the gated spatial assignment, and the population weights.
 __global__ void k_assign_pick(const float* __restrict__ cos, const int32_t* __restrict__ support,
                               const int32_t* __restrict__ slot, const float* __restrict__ delta,
-                              const double* __restrict__ dpart, int nA,
-                              const float* __restrict__ energy, const float* __restrict__ epart,
-                              int nE, const int32_t* toff, int B, int N,
-                              int K, int Tmax, int gh, int gw, float gate_scale, float gate_pow,
-                              float ambig_margin, float lambda_p, float tau_s, float alpha,
+                              const float* __restrict__ gatev, const float* __restrict__ energy,
+                              const int32_t* toff, int B, int N, int K, int Tmax, int gh, int gw,
+                              float gate_pow, float ambig_margin, float lambda_p, float tau_s,
+                              float alpha,
                               int32_t* pi, float* mass, uint32_t* mbits, TraceView tv,
                               uint32_t* status) {
-  __shared__ float gate[3];      // dbar, s_x, mean energy
   extern __shared__ int sS[];  // the support of the image, staged once per block
   const int b = blockIdx.y;
   const TextGeom tg = text_geom(toff, b, B, Tmax, status);
   if (tg.T == 0) return;
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   for (int k = threadIdx.x; k < K; k += blockDim.x) sS[k] = support[(size_t)b * K + k];
-  if (w == 0) {  // the partials in a fixed order (every block the same)
-    double s = 0.0, c = 0.0, et = 0.0;
-    for (int q = lane; q < nA; q += 32) {
-      s += dpart[((size_t)b * nA + q) * 2 + 0];
-      c += dpart[((size_t)b * nA + q) * 2 + 1];
-    }
-    for (int q = lane; q < nE; q += 32) et += epart[(size_t)b * nE + q];  // message energies
-    s = warp_sum(s);
-    c = warp_sum(c);
-    et = warp_sum(et);
-    if (lane == 0) {
-      const float db = c > 0.0 ? (float)(s / c) : 0.f;
-      gate[0] = db;
-      gate[1] = 1.f - expf(-powf(db / gate_scale, gate_pow));
-      gate[2] = (float)(et / N);
-    }
-  }
+  const float dbar = gatev[(size_t)b * 4 + 0], sx = gatev[(size_t)b * 4 + 1];
+  const float emean = gatev[(size_t)b * 4 + 2];
   __syncthreads();
-  const float dbar = gate[0], sx = gate[1];
-  const float emean = gate[2];
   if (blockIdx.x == 0 && threadIdx.x == 0 && tv.base) {
     tv.header(b)->s_x = sx;
     tv.header(b)->delta_bar = dbar;
@@ -187,13 +193,13 @@ cudaError_t launch_assign(const Dims& dm, const gmc_params& p, Scratch& s, const
   if ((e0 = set_smem_limit((const void*)k_assign_pick, smem)) != cudaSuccess) return e0;
   k_assign_gap<<<grid, 32 * ASSIGN_WARPS, smem, st>>>(
       s.cos, s.support, s.slot, dm.toff, dm.B, dm.N, dm.K, dm.T, dm.H, s.omega, s.zn2, s.sigma,
-      s.W2, s.ebar, s.epart, s.delta, s.dpart, s.nA, s.status);
+      s.W2, s.ebar, s.epart, s.delta, s.dpart, s.nA, p.gate_scale, p.gate_pow, s.tick2, s.gatev,
+      s.status);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   k_assign_pick<<<grid, 32 * ASSIGN_WARPS, smem, st>>>(
-      s.cos, s.support, s.slot, s.delta, s.dpart, s.nA, s.ebar, s.epart, s.nE, dm.toff, dm.B,
-      dm.N, dm.K, dm.T,
-      dm.gh, dm.gw, p.gate_scale, p.gate_pow, p.ambig_margin, p.assign_spatial_w, p.tau_s,
+      s.cos, s.support, s.slot, s.delta, s.gatev, s.ebar, dm.toff, dm.B, dm.N, dm.K, dm.T,
+      dm.gh, dm.gw, p.gate_pow, p.ambig_margin, p.assign_spatial_w, p.tau_s,
       p.pop_strength, s.pi, s.mass, s.mbits, tv, s.status);
   return cudaGetLastError();
 }

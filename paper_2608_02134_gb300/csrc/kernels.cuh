@@ -44,6 +44,8 @@ struct Scratch {
   float* zn2;        // [B][H][N]      ||Z_h[i]||^2
   float* sigpart;    // [B][nP][H]     block partials of ||Z_h||_F^2
   uint32_t* tick;    // [B]            last-block tickets of the probe (zeroed with status)
+  uint32_t* tick2;   // [B]            last-block tickets of the assignment gap pass (same)
+  float* gatev;      // [B][4]         Delta_bar, s_x, mean message energy
   float* sigma;      // [B][H]         mass coordinate sigma_h
   double* hgpart;    // [B][nHG][H*H]  block partials of the head-pattern Gram
   double* HG;        // [B][H*H + H]   head-pattern Gram, then sum_t rs[h,t] per head
