@@ -102,6 +102,14 @@ __device__ __forceinline__ void cp_async_wait() {
   asm volatile("cp.async.wait_group %0;" ::"n"(Pending) : "memory");
 }
 
+// Programmatic dependent launch: every kernel of the path is launched so it may
+// begin while the previous kernel on its stream is still running, and its
+// first statement waits here until that kernel has completed and its writes
+// are visible.  Only the launch and the block set-up overlap; no memory is
+// touched before the wait.  Without the launch attribute the wait returns at
+// once.
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 __device__ __forceinline__ void set_status(uint32_t* status, uint32_t bit) {
   if (status) atomicOr(status, bit);
 }

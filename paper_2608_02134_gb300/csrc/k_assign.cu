@@ -29,6 +29,7 @@ __global__ void k_assign_gap(const float* __restrict__ cos, const int32_t* __res
                              const float* __restrict__ W2, float* energy, float* epart,
                              float* delta, double* dpart, int nA, float gate_scale,
                              float gate_pow, uint32_t* tick, float* gatev, uint32_t* status) {
+  grid_dep_wait();
   __shared__ double sd[ASSIGN_WARPS];
   __shared__ int sc[ASSIGN_WARPS];
   __shared__ float se[ASSIGN_WARPS];
@@ -127,6 +128,7 @@ __global__ void k_assign_pick(const float* __restrict__ cos, const int32_t* __re
                               float alpha,
                               int32_t* pi, float* mass, uint32_t* mbits, TraceView tv,
                               uint32_t* status) {
+  grid_dep_wait();
   extern __shared__ int sS[];  // the support of the image, staged once per block
   const int b = blockIdx.y;
   const TextGeom tg = text_geom(toff, b, B, Tmax, status);
@@ -191,13 +193,13 @@ cudaError_t launch_assign(const Dims& dm, const gmc_params& p, Scratch& s, const
   cudaError_t e0;
   if ((e0 = set_smem_limit((const void*)k_assign_gap, smem)) != cudaSuccess) return e0;
   if ((e0 = set_smem_limit((const void*)k_assign_pick, smem)) != cudaSuccess) return e0;
-  k_assign_gap<<<grid, 32 * ASSIGN_WARPS, smem, st>>>(
+  launch_k(k_assign_gap, grid, 32 * ASSIGN_WARPS, smem, st, 1,
       s.cos, s.support, s.slot, dm.toff, dm.B, dm.N, dm.K, dm.T, dm.H, s.omega, s.zn2, s.sigma,
       s.W2, s.ebar, s.epart, s.delta, s.dpart, s.nA, p.gate_scale, p.gate_pow, s.tick2, s.gatev,
       s.status);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  k_assign_pick<<<grid, 32 * ASSIGN_WARPS, smem, st>>>(
+  launch_k(k_assign_pick, grid, 32 * ASSIGN_WARPS, smem, st, 1,
       s.cos, s.support, s.slot, s.delta, s.gatev, s.ebar, dm.toff, dm.B, dm.N, dm.K, dm.T,
       dm.gh, dm.gw, p.gate_pow, p.ambig_margin, p.assign_spatial_w, p.tau_s,
       p.pop_strength, s.pi, s.mass, s.mbits, tv, s.status);

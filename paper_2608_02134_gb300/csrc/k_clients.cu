@@ -65,6 +65,7 @@ __global__ void __launch_bounds__(256, 4) k_build_clients(
     const float* __restrict__ cos, const int32_t* toff, int B, int N, int Tmax, int H, int M,
     int gh, int gw, int L, float beta_G, float beta_V, float beta_S, float tau_v, float tau_s,
     float wq, float fx_scale, int check, float* C, long long* u0, uint32_t* status) {
+  grid_dep_wait();
   __shared__ RowInfo ri[ROWS_PER_BLOCK];
   const int b = blockIdx.y;
   const TextGeom tg = text_geom(toff, b, B, Tmax, status);
@@ -170,7 +171,7 @@ __global__ void __launch_bounds__(256, 4) k_build_clients(
 cudaError_t launch_build_clients(const Dims& dm, const gmc_params& p, int fx_exp, Scratch& s,
                                  cudaStream_t st) {
   dim3 grid(ceil_div(dm.M, ROWS_PER_BLOCK), dm.B);
-  k_build_clients<<<grid, 32 * ROWS_PER_BLOCK, 0, st>>>(
+  launch_k(k_build_clients, grid, 32 * ROWS_PER_BLOCK, 0, st, 1,
       s.A, s.rs, s.nRS, s.zn2, s.sigma, s.omega, s.cos, dm.toff, dm.B, dm.N, dm.T, dm.H, dm.M, dm.gh,
       dm.gw, dm.L, p.beta_G, p.beta_V, p.beta_S, p.tau_v, p.tau_s, p.terminal_q_weight,
       ldexpf(1.f, fx_exp), p.check_mode, s.C, s.u0, s.status);
@@ -183,6 +184,7 @@ cudaError_t launch_build_clients(const Dims& dm, const gmc_params& p, int fx_exp
 // ---------------------------------------------------------------------------
 __global__ void k_sel_total(const float* __restrict__ C, int M, int N, int nblk, double* part,
                             uint32_t* status) {
+  grid_dep_wait();
   __shared__ double red[32];
   const int b = blockIdx.y;
   const size_t n = (size_t)M * N;
@@ -202,6 +204,7 @@ __global__ void k_sel_total(const float* __restrict__ C, int M, int N, int nblk,
 }
 
 __global__ void k_sel_exp(const double* part, int nblk, int B, int32_t* fexp) {
+  grid_dep_wait();
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= B) return;
   double tot = 0.0;
@@ -213,6 +216,7 @@ __global__ void k_sel_exp(const double* part, int nblk, int B, int32_t* fexp) {
 
 __global__ void __launch_bounds__(256) k_sel_colsum(const float* __restrict__ C, int M, int N,
                                                     const int32_t* fexp, long long* u0) {
+  grid_dep_wait();
   const int b = blockIdx.y;
   const int r0 = blockIdx.x * ROWS_PER_BLOCK;
   const int nrows = min(ROWS_PER_BLOCK, M - r0);
@@ -229,12 +233,12 @@ __global__ void __launch_bounds__(256) k_sel_colsum(const float* __restrict__ C,
 }
 
 cudaError_t launch_select_prep(const float* C, int B, int M, int N, Scratch& s, cudaStream_t st) {
-  k_sel_total<<<dim3(s.nSel, B), 256, 0, st>>>(C, M, N, s.nSel, s.selpart, s.status);
+  launch_k(k_sel_total, dim3(s.nSel, B), 256, 0, st, 1, C, M, N, s.nSel, s.selpart, s.status);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  k_sel_exp<<<ceil_div(B, 128), 128, 0, st>>>(s.selpart, s.nSel, B, s.fexp);
+  launch_k(k_sel_exp, ceil_div(B, 128), 128, 0, st, 1, s.selpart, s.nSel, B, s.fexp);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  k_sel_colsum<<<dim3(ceil_div(M, ROWS_PER_BLOCK), B), 256, 0, st>>>(C, M, N, s.fexp, s.u0);
+  launch_k(k_sel_colsum, dim3(ceil_div(M, ROWS_PER_BLOCK), B), 256, 0, st, 1, C, M, N, s.fexp, s.u0);
   return cudaGetLastError();
 }
 

@@ -18,6 +18,7 @@ __global__ void __launch_bounds__(256) k_gram_simt(const Tin* __restrict__ hidde
                                                    const float* __restrict__ rn,
                                                    const int32_t* toff, int B, int N, int K,
                                                    int Tmax, int D, float* cos, uint32_t* status) {
+  grid_dep_wait();
   __shared__ float As[GK][GT + 4];
   __shared__ float Bs[GK][GT + 4];
   const int b = blockIdx.z;
@@ -67,11 +68,11 @@ __global__ void __launch_bounds__(256) k_gram_simt(const Tin* __restrict__ hidde
 cudaError_t launch_gram_simt(const Dims& dm, const void* hidden, Scratch& s, cudaStream_t st) {
   dim3 grid(ceil_div(dm.N, GT), ceil_div(dm.N, GT), dm.B);
   if (dm.dtype == GMC_BF16)
-    k_gram_simt<__nv_bfloat16><<<grid, 256, 0, st>>>((const __nv_bfloat16*)hidden, s.rn, dm.toff,
+    launch_k(k_gram_simt<__nv_bfloat16>, grid, 256, 0, st, 1, (const __nv_bfloat16*)hidden, s.rn, dm.toff,
                                                      dm.B, dm.N, dm.K, dm.T, dm.D, s.cos,
                                                      s.status);
   else
-    k_gram_simt<float><<<grid, 256, 0, st>>>((const float*)hidden, s.rn, dm.toff, dm.B, dm.N,
+    launch_k(k_gram_simt<float>, grid, 256, 0, st, 1, (const float*)hidden, s.rn, dm.toff, dm.B, dm.N,
                                              dm.K, dm.T, dm.D, s.cos, s.status);
   return cudaGetLastError();
 }

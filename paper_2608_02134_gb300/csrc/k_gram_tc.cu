@@ -52,6 +52,7 @@ constexpr size_t GRAM_SMEM = 1024 + 2 * STAGES * TILE_BYTES + sizeof(GramCtl);
 __global__ void __launch_bounds__(GRAM_THREADS, 1)
     k_gram_tc(const __grid_constant__ CUtensorMap tmap, const int32_t* toff, int B, int N,
               int Tmax, int D, const float* __restrict__ rn, float* cos, uint32_t* status) {
+  grid_dep_wait();
   extern __shared__ uint8_t sm_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -272,13 +273,16 @@ cudaError_t launch_gram_tc(const Dims& dm, const void* hidden, Scratch& s, cudaS
   cfg.blockDim = dim3(GRAM_THREADS);
   cfg.dynamicSmemBytes = GRAM_SMEM;
   cfg.stream = st;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 2;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // see grid_dep_wait
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, k_gram_tc, map, dm.toff, dm.B, dm.N, dm.T, dm.D,
                             (const float*)s.rn, s.cos, s.status);
 }

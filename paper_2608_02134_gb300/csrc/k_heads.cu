@@ -35,6 +35,7 @@ __global__ void k_head_stats(const float* __restrict__ A, const float* __restric
                              const float* __restrict__ sigma, const int32_t* toff, int B, int N,
                              int Tmax, int H, float wq, double* hgpart, int nHG, float* W2,
                              uint32_t* status) {
+  grid_dep_wait();
   extern __shared__ float sm_hs[];
   const int b = blockIdx.y;
   const TextGeom tg = text_geom(toff, b, B, Tmax, status);
@@ -172,6 +173,7 @@ __device__ __forceinline__ void warp_argbest(double& v, int& idx, bool want_max)
 __global__ void k_hg_reduce(const double* __restrict__ hgpart, int nHG, int B, int H,
                             const float* __restrict__ rs, int nRS, const int32_t* toff,
                             int Tmax, double* HG) {
+  grid_dep_wait();
   const int w = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   const int HH = H * H, HE = HH + H;
   if (w >= B * HE) return;
@@ -194,6 +196,7 @@ __global__ void k_head_cluster(const double* __restrict__ HGred,
                                const int32_t* toff, int B, int N, int Tmax, int H,
                                int max_clusters, float head_eps, float* omega,
                                TraceView tv, uint32_t* status) {
+  grid_dep_wait();
   extern __shared__ double sm_hc[];
   const int b = blockIdx.x;
   const TextGeom tg = text_geom(toff, b, B, Tmax, status);
@@ -331,18 +334,18 @@ cudaError_t launch_heads(const Dims& dm, const gmc_params& p, Scratch& s, const 
                 sizeof(unsigned short) * (nhb * (nhb + 1) / 2) + 16;
   cudaError_t e = set_smem_limit((const void*)k_head_stats, smem);
   if (e != cudaSuccess) return e;
-  k_head_stats<<<dim3(s.nHG, dm.B), 512, smem, st>>>(s.A, s.Z, s.sigma, dm.toff, dm.B, dm.N, dm.T,
+  launch_k(k_head_stats, dim3(s.nHG, dm.B), 512, smem, st, 1, s.A, s.Z, s.sigma, dm.toff, dm.B, dm.N, dm.T,
                                                      H, p.terminal_q_weight, s.hgpart, s.nHG,
                                                      s.W2, s.status);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   const int warps = dm.B * (H * H + H);
-  k_hg_reduce<<<ceil_div(warps * 32, 256), 256, 0, st>>>(s.hgpart, s.nHG, dm.B, H, s.rs, s.nRS,
+  launch_k(k_hg_reduce, ceil_div(warps * 32, 256), 256, 0, st, 1, s.hgpart, s.nHG, dm.B, H, s.rs, s.nRS,
                                                          dm.toff, dm.T, s.HG);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   size_t smem2 = sizeof(double) * (2 * (size_t)H * H + 3 * H + 2 * GMC_MAX_HEADS) +
                  sizeof(int) * (H + 2 * GMC_MAX_HEADS);
   if ((e = set_smem_limit((const void*)k_head_cluster, smem2)) != cudaSuccess) return e;
-  k_head_cluster<<<dm.B, 256, smem2, st>>>(s.HG, dm.toff, dm.B, dm.N, dm.T, H,
+  launch_k(k_head_cluster, dm.B, 256, smem2, st, 1, s.HG, dm.toff, dm.B, dm.N, dm.T, H,
                                           p.max_head_clusters, p.head_eps, s.omega, tv, s.status);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   return cudaGetLastError();

@@ -18,6 +18,7 @@ __global__ void k_message(const Tin* __restrict__ keys, const Tin* __restrict__ 
                           const float* __restrict__ zn2, const float* __restrict__ sigma,
                           const int32_t* toff, int B, int N, int K, int Tmax, int H, int Hkv,
                           int d, float* A, float* rs, uint32_t* status) {
+  grid_dep_wait();
   extern __shared__ float sm_msg[];  // [d] query, then [N + Tmax] scores
   __shared__ float red[32];
   const int t = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
@@ -70,12 +71,12 @@ cudaError_t launch_message(const Dims& dm, const void* keys, const void* queries
   cudaError_t e;
   if (dm.dtype == GMC_BF16) {
     if ((e = set_smem_limit((const void*)k_message<__nv_bfloat16>, smem)) != cudaSuccess) return e;
-    k_message<__nv_bfloat16><<<grid, 256, smem, st>>>(
+    launch_k(k_message<__nv_bfloat16>, grid, 256, smem, st, 1,
         (const __nv_bfloat16*)keys, (const __nv_bfloat16*)queries, s.zn2, s.sigma, dm.toff, dm.B,
         dm.N, dm.K, dm.T, dm.H, dm.Hkv, dm.d, s.A, s.rs, s.status);
   } else {
     if ((e = set_smem_limit((const void*)k_message<float>, smem)) != cudaSuccess) return e;
-    k_message<float><<<grid, 256, smem, st>>>((const float*)keys, (const float*)queries, s.zn2,
+    launch_k(k_message<float>, grid, 256, smem, st, 1, (const float*)keys, (const float*)queries, s.zn2,
                                               s.sigma, dm.toff, dm.B, dm.N, dm.K, dm.T, dm.H,
                                               dm.Hkv, dm.d, s.A, s.rs, s.status);
   }

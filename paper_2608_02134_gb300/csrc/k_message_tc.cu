@@ -113,6 +113,7 @@ __device__ __forceinline__ void epi_barrier() {
 __global__ void k_pack_q(const __nv_bfloat16* __restrict__ queries, const int32_t* toff, int B,
                          int Tmax, int H, int Hkv, int d, int RQ, __nv_bfloat16* Qp,
                          uint32_t* status) {
+  grid_dep_wait();
   const int b = blockIdx.z, g = blockIdx.y;
   const TextGeom tg = text_geom(toff, b, B, Tmax, status);
   const int grp = H / Hkv;
@@ -137,6 +138,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                  int mode, int kt_per, int nsplit, float2* part,
                  const float* __restrict__ zn2, const float* __restrict__ sigma, float* A,
                  float* rs, uint32_t* status) {
+  grid_dep_wait();
   extern __shared__ uint8_t sm_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -356,6 +358,7 @@ __global__ void __launch_bounds__(FT_THREADS, 1)
                     const int32_t* toff, int B, int N, int Tmax, int H, int Hkv, int d, int RQ,
                     int kt_per, int nsplit, uint32_t tmem_cols, const float* __restrict__ zn2,
                     const float* __restrict__ sigma, float* A, float* rs, uint32_t* status) {
+  grid_dep_wait();
   extern __shared__ uint8_t sm_raw[];
   cg::cluster_group cluster = cg::this_cluster();
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) &
@@ -579,7 +582,7 @@ int message_splits(const Dims& dm) {
 cudaError_t launch_message_tc(const Dims& dm, const void* keys, const void* queries, Scratch& s,
                               cudaStream_t st) {
   const int RQ = message_rq(dm);
-  k_pack_q<<<dim3(ceil_div(RQ, 8), dm.Hkv, dm.B), 256, 0, st>>>(
+  launch_k(k_pack_q, dim3(ceil_div(RQ, 8), dm.Hkv, dm.B), 256, 0, st, 1,
       (const __nv_bfloat16*)queries, dm.toff, dm.B, dm.T, dm.H, dm.Hkv, dm.d, RQ, s.Qp, s.status);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
@@ -608,7 +611,7 @@ cudaError_t launch_message_tc(const Dims& dm, const void* keys, const void* quer
     cfg.blockDim = dim3(FT_THREADS);
     cfg.dynamicSmemBytes = fsmem;
     cfg.stream = st;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = 1;
     attr[0].val.clusterDim.y = 1;
@@ -616,14 +619,18 @@ cudaError_t launch_message_tc(const Dims& dm, const void* keys, const void* quer
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     int ncl = 0;
-    if (cudaOccupancyMaxActiveClusters(&ncl, (void*)k_message_fused, &cfg) == cudaSuccess && ncl > 0)
+    if (cudaOccupancyMaxActiveClusters(&ncl, (void*)k_message_fused, &cfg) == cudaSuccess && ncl > 0) {
+      attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // see grid_dep_wait
+      attr[1].val.programmaticStreamSerializationAllowed = 1;
+      cfg.numAttrs = 2;
       return cudaLaunchKernelEx(&cfg, k_message_fused, qmap, kmap, dm.toff, dm.B, dm.N, dm.T, dm.H,
                                 dm.Hkv, dm.d, RQ, sp.kt_per, sp.n, cols, (const float*)s.zn2,
                                 (const float*)s.sigma, s.A, s.rs, s.status);
+    }
     cudaGetLastError();  // no co-resident cluster: the two launches below
   }
   for (int mode = 0; mode < 2; ++mode) {
-    k_message_tc<<<grid, THREADS, smem, st>>>(qmap, kmap, dm.toff, dm.B, dm.N, dm.T, dm.H, dm.Hkv,
+    launch_k(k_message_tc, grid, THREADS, smem, st, 1, qmap, kmap, dm.toff, dm.B, dm.N, dm.T, dm.H, dm.Hkv,
                                               dm.d, RQ, mode, sp.kt_per, sp.n, s.mpart, s.zn2,
                                               s.sigma, s.A, s.rs, s.status);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;

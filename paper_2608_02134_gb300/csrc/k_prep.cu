@@ -16,6 +16,7 @@ template <typename Tin>
 __global__ void k_rownorm(const Tin* __restrict__ hidden, const int32_t* toff, int B, int N,
                           int K, int Tmax, int D, float norm_eps, float* rn, float* rmsh,
                           uint32_t* status) {
+  grid_dep_wait();
   const int b = blockIdx.y;
   const TextGeom tg = text_geom(toff, b, B, Tmax, status);
   if (tg.T == 0) return;
@@ -58,6 +59,7 @@ __global__ void __launch_bounds__(256) k_probe(
     int K, int Tmax, int H, int Hkv, int d, float lambda_mass, float eps_mass, float* Z,
     float* zn2, float* sigpart, int nP, float* sigma, uint32_t* tick, long long* u0,
     uint32_t* status) {
+  grid_dep_wait();
   extern __shared__ float4 sm_probe4[];
   __shared__ int last;
   const int b = blockIdx.z, g = blockIdx.y, pb = blockIdx.x;
@@ -138,6 +140,7 @@ __global__ void k_identity(const Tin* __restrict__ hidden, const Tin* __restrict
                            const int32_t* __restrict__ pos, const int32_t* toff, int B, int N,
                            int Tmax, int D, int HD, int32_t* out_idx, Tin* out_hidden,
                            Tin* out_kv, int32_t* out_pos, uint32_t* status) {
+  grid_dep_wait();
   const int b = blockIdx.y, r = blockIdx.x;
   const TextGeom tg = text_geom(toff, b, B, Tmax, status);
   if (tg.T == 0 || r >= N + tg.T) return;
@@ -161,11 +164,11 @@ cudaError_t launch_rownorm(const Dims& dm, const void* hidden, float norm_eps, S
                            cudaStream_t st) {
   dim3 grid(ceil_div(dm.N, ROWS_PER_BLOCK), dm.B);
   if (dm.dtype == GMC_BF16)
-    k_rownorm<__nv_bfloat16><<<grid, 32 * ROWS_PER_BLOCK, 0, st>>>(
+    launch_k(k_rownorm<__nv_bfloat16>, grid, 32 * ROWS_PER_BLOCK, 0, st, 1,
         (const __nv_bfloat16*)hidden, dm.toff, dm.B, dm.N, dm.K, dm.T, dm.D, norm_eps, s.rn,
         s.rmsh, s.status);
   else
-    k_rownorm<float><<<grid, 32 * ROWS_PER_BLOCK, 0, st>>>((const float*)hidden, dm.toff, dm.B,
+    launch_k(k_rownorm<float>, grid, 32 * ROWS_PER_BLOCK, 0, st, 1, (const float*)hidden, dm.toff, dm.B,
                                                            dm.N, dm.K, dm.T, dm.D, norm_eps, s.rn,
                                                            s.rmsh, s.status);
   return cudaGetLastError();
@@ -175,11 +178,11 @@ cudaError_t launch_rms_rows(const Dims& dm, const void* hidden, float* rmsh, uin
                             cudaStream_t st) {
   dim3 grid(ceil_div(dm.N, ROWS_PER_BLOCK), dm.B);
   if (dm.dtype == GMC_BF16)
-    k_rownorm<__nv_bfloat16><<<grid, 32 * ROWS_PER_BLOCK, 0, st>>>(
+    launch_k(k_rownorm<__nv_bfloat16>, grid, 32 * ROWS_PER_BLOCK, 0, st, 1,
         (const __nv_bfloat16*)hidden, dm.toff, dm.B, dm.N, dm.K, dm.T, dm.D, 1e-12f, nullptr,
         rmsh, status);
   else
-    k_rownorm<float><<<grid, 32 * ROWS_PER_BLOCK, 0, st>>>((const float*)hidden, dm.toff, dm.B,
+    launch_k(k_rownorm<float>, grid, 32 * ROWS_PER_BLOCK, 0, st, 1, (const float*)hidden, dm.toff, dm.B,
                                                            dm.N, dm.K, dm.T, dm.D, 1e-12f,
                                                            nullptr, rmsh, status);
   return cudaGetLastError();
@@ -195,12 +198,12 @@ cudaError_t launch_probe(const Dims& dm, const void* keys, const float* W, const
   cudaError_t e;
   if (dm.dtype == GMC_BF16) {
     if ((e = set_smem_limit((const void*)k_probe<__nv_bfloat16>, smem)) != cudaSuccess) return e;
-    k_probe<__nv_bfloat16><<<grid, 256, smem, st>>>(
+    launch_k(k_probe<__nv_bfloat16>, grid, 256, smem, st, 1,
         (const __nv_bfloat16*)keys, W, dm.toff, dm.B, dm.N, dm.K, dm.T, dm.H, dm.Hkv, dm.d,
         p.lambda_mass, p.eps_mass, s.Z, s.zn2, s.sigpart, s.nP, s.sigma, s.tick, s.u0, s.status);
   } else {
     if ((e = set_smem_limit((const void*)k_probe<float>, smem)) != cudaSuccess) return e;
-    k_probe<float><<<grid, 256, smem, st>>>((const float*)keys, W, dm.toff, dm.B, dm.N, dm.K,
+    launch_k(k_probe<float>, grid, 256, smem, st, 1, (const float*)keys, W, dm.toff, dm.B, dm.N, dm.K,
                                             dm.T, dm.H, dm.Hkv, dm.d, p.lambda_mass, p.eps_mass,
                                             s.Z, s.zn2, s.sigpart, s.nP, s.sigma, s.tick,
                                             s.u0, s.status);
@@ -214,11 +217,11 @@ cudaError_t launch_identity(const Dims& dm, const void* hidden, const void* keys
   dim3 grid(dm.N + dm.T, dm.B);
   const int HD = dm.Hkv * dm.d;
   if (dm.dtype == GMC_BF16)
-    k_identity<__nv_bfloat16><<<grid, 128, 0, st>>>(
+    launch_k(k_identity<__nv_bfloat16>, grid, 128, 0, st, 1,
         (const __nv_bfloat16*)hidden, (const __nv_bfloat16*)keys, pos, dm.toff, dm.B, dm.N, dm.T,
         dm.D, HD, out_idx, (__nv_bfloat16*)out_hidden, (__nv_bfloat16*)out_kv, out_pos, status);
   else
-    k_identity<float><<<grid, 128, 0, st>>>((const float*)hidden, (const float*)keys, pos,
+    launch_k(k_identity<float>, grid, 128, 0, st, 1, (const float*)hidden, (const float*)keys, pos,
                                             dm.toff, dm.B, dm.N, dm.T, dm.D, HD, out_idx,
                                             (float*)out_hidden, (float*)out_kv, out_pos, status);
   return cudaGetLastError();

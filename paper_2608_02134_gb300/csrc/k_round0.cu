@@ -24,6 +24,7 @@ __global__ void __launch_bounds__(512) k_r0_pool(const long long* __restrict__ u
                                                    int P, const int32_t* toff, int Tmax,
                                                    int32_t* pool0, int32_t* info, long long* s0,
                                                    long long* u1, long long* fv, uint32_t* status) {
+  grid_dep_wait();
   extern __shared__ __align__(16) char sm_r0p[];
   const int b = blockIdx.x;
   // the accumulators of the next two kernels start at zero
@@ -55,6 +56,7 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_rho(
     const float* __restrict__ C, int B, int N, int Mstride, int H, int L2, const int32_t* toff,
     int Tmax, int uniform_rows, const int32_t* __restrict__ pool0, const int32_t* __restrict__ info,
     int P, float resp_temp, float resp_eps, int fx_exp, const int32_t* fexp, long long* s0) {
+  grid_dep_wait();
   __shared__ int pool[GMC_MAX_POOL];
   __shared__ long long sblk[GMC_MAX_POOL];
   const int b = blockIdx.y;
@@ -110,6 +112,7 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_filter(
     int32_t* info, const long long* __restrict__ s0, int P, int bsz, int fx_exp,
     const int32_t* fexp, long long* u1, float* bcov, int32_t* cnt, long long* fv,
     int32_t* order, TraceView tv) {
+  grid_dep_wait();
   __shared__ int pool[GMC_MAX_POOL];
   __shared__ long long sc[GMC_MAX_POOL];
   __shared__ int batch[GMC_MAX_POOL];
@@ -252,16 +255,16 @@ cudaError_t launch_round0(const R0State& r0, int B, int N, int K, int M, const i
   const size_t smem = sizeof(int) * (sel::HBINS + N + 32 + 8 + 2 * P) + (size_t)N + 64;
   if ((e = set_smem_limit((const void*)k_r0_pool, smem)) != cudaSuccess) return e;
   const int uniform = (H == 0);
-  k_r0_pool<<<B, 512, smem, st>>>(u0, B, N, P, uniform ? nullptr : toff, T, r0.pool, r0.info,
+  launch_k(k_r0_pool, B, 512, smem, st, 1, u0, B, N, P, uniform ? nullptr : toff, T, r0.pool, r0.info,
                                   r0.s0, r0.u1, r0.fv, status);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   dim3 grid(ceil_div(M, R0_ROWS), B);
-  k_r0_rho<<<grid, 32 * R0_ROWS, 0, st>>>(C, B, N, M, H, L2, toff, T, uniform, r0.pool, r0.info,
+  launch_k(k_r0_rho, grid, 32 * R0_ROWS, 0, st, 1, C, B, N, M, H, L2, toff, T, uniform, r0.pool, r0.info,
                                           P, p.resp_temp, p.resp_eps, fx_exp, fexp, r0.s0);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   const size_t fsm = sizeof(unsigned long long) * (size_t)N;
   if ((e = set_smem_limit((const void*)k_r0_filter, fsm)) != cudaSuccess) return e;
-  k_r0_filter<<<grid, 32 * R0_ROWS, fsm, st>>>(C, scol, B, N, K, M, H, L2, toff, T, uniform, r0.pool,
+  launch_k(k_r0_filter, grid, 32 * R0_ROWS, fsm, st, 1, C, scol, B, N, K, M, H, L2, toff, T, uniform, r0.pool,
                                              r0.info, r0.s0, P, p.batch_b, fx_exp, fexp, r0.u1,
                                              r0.bcov, r0.cnt, r0.fv, order, tv);
   return cudaGetLastError();

@@ -190,6 +190,7 @@ __device__ __forceinline__ int group_sum(int v, unsigned gm) {
 }  // namespace
 
 __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
+  grid_dep_wait();
   extern __shared__ __align__(16) char sm_sel[];
   cg::cluster_group cluster = cg::this_cluster();
   const int CS = (int)cluster.num_blocks();
@@ -880,7 +881,7 @@ cudaError_t launch_select(const R0State& r0, int B, int N, int K, int M, const i
     cfg.blockDim = dim3(SEL_THREADS);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = st;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = CS;
     attr[0].val.clusterDim.y = 1;
@@ -893,6 +894,9 @@ cudaError_t launch_select(const R0State& r0, int B, int N, int K, int M, const i
       cudaGetLastError();
       continue;
     }
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // see grid_dep_wait
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.numAttrs = 2;
     return cudaLaunchKernelEx(&cfg, k_select, a);
   }
   return cudaErrorInvalidConfiguration;

@@ -101,6 +101,7 @@ __global__ void __launch_bounds__(TR_THREADS, 7) k_transport(
     const uint32_t* __restrict__ mbits, const int32_t* toff, int B, int N, int K, int Tmax, int D,
     int HD, int S, float rms_eps, int check, int32_t* out_idx, Tin* out_hidden, Tin* out_kv,
     int32_t* out_pos, uint32_t* status) {
+  grid_dep_wait();
   constexpr int NW = TR_THREADS / 32;
   constexpr int NM = TR_WIN * NW;  // 32-token masks per window
   static_assert(NM * 32 == TR_WIN * TR_THREADS, "one mask per 32 tokens of a window");
@@ -346,13 +347,16 @@ cudaError_t launch_transport(const Dims& dm, const gmc_params& p, const void* hi
   cfg.blockDim = dim3(TR_THREADS);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = st;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = S;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // see grid_dep_wait
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.numAttrs = 2;
   if (dm.dtype == GMC_BF16) {
     using T = __nv_bfloat16;
     return cudaLaunchKernelEx(&cfg, k_transport<T>, (const T*)hidden, (const T*)keys, pos, support,

@@ -150,6 +150,37 @@ cudaError_t set_smem_limit(const void* func, size_t bytes);
 }  // namespace gmc
 
 namespace gmc {
+// Launch `kernel` on `st` with programmatic stream serialization: it may be
+// scheduled while the previous kernel on the stream is still running, and its
+// first statement (grid_dep_wait) orders every memory access after that
+// kernel.  cluster_x > 1 adds a thread-block cluster of that size along x.
+template <typename... P, typename... A>
+cudaError_t launch_k(void (*kernel)(P...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                     int cluster_x, A... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[2];
+  int n = 0;
+  attr[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[n].val.programmaticStreamSerializationAllowed = 1;
+  ++n;
+  if (cluster_x > 1) {
+    attr[n].id = cudaLaunchAttributeClusterDimension;
+    attr[n].val.clusterDim.x = cluster_x;
+    attr[n].val.clusterDim.y = 1;
+    attr[n].val.clusterDim.z = 1;
+    ++n;
+  }
+  cfg.attrs = attr;
+  cfg.numAttrs = n;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+}  // namespace gmc
+
+namespace gmc {
 cudaError_t launch_gram_simt(const Dims&, const void* hidden, Scratch&, cudaStream_t);
 cudaError_t launch_gram_tc(const Dims&, const void* hidden, Scratch&, cudaStream_t);
 bool gram_tc_supported(const Dims&);
