@@ -144,6 +144,8 @@ R0State carve_round0(Carver& c, size_t B, size_t N, size_t M) {
   r.info = c.take<int32_t>(B * 4);
   r.s0 = c.take<long long>(B * GMC_MAX_POOL);
   r.u1 = c.take<long long>(B * N);
+  r.u2 = c.take<long long>(B * N);
+  r.ugain = SPARSE_GPU_ROUNDS % 2 == 0 ? r.u1 : r.u2;
   r.bcov = c.take<float>(B * M);
   r.cnt = c.take<int32_t>(B * M);
   r.fv = c.take<long long>(B * 4);
@@ -409,7 +411,7 @@ int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* 
     GMC_TRY(cudaStreamWaitEvent(st, sd->join, 0));
   }
   GMC_STAGE("clients", 1, launch_build_clients(dm, p, fx, s, st));
-  GMC_STAGE("round0", 3,
+  GMC_STAGE("round0", 3 + 3 * SPARSE_GPU_ROUNDS,
             launch_round0(r0, dm.B, N, Ke, dm.M, dm.toff, H, T, p.landmarks * p.landmarks, p, fx,
                           nullptr, s.C, s.scol, s.u0, s.order, s.status, tv, st));
   GMC_STAGE("select", 1,
@@ -484,7 +486,7 @@ int gmc_select(const float* clients, int B, int M, int N, int K, const gmc_param
                         s.order, s.status, tv, st));
   GMC_TRY(launch_select(r0, B, N, K, M, nullptr, 0, 1, 0, p, 0, s.fexp, s.C, s.scol, s.u0,
                         s.order, s.support, s.slot, out_idx, s.status, tv, st));
-  g_launches += 7;
+  g_launches += 7 + 3 * SPARSE_GPU_ROUNDS;
   return GMC_OK;
 }
 

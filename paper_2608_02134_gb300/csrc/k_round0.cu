@@ -8,8 +8,20 @@
 //               b_m = max over the batch, and the row's survivors
 //               {i : Cbar_mi > b_m} compacted in place; the next round's gains
 //               are summed in fixed point (global atomics).
-// Every reduction is an integer sum, so the result does not depend on the
-// order blocks run in.  The cluster kernel (k_select) continues from round 1.
+// The next SPARSE_GPU_ROUNDS rounds run the same three steps over the survivor
+// lists left in place by the previous round (row m: values Cbar[m][0..cnt_m),
+// tokens scol[m][0..cnt_m), ascending):
+//   k_rg_pool   the pool of the current gains among the unselected tokens;
+//   k_rg_rho    warp per row: the row's pool entries are found through a
+//               token -> pool slot table; pool tokens without a survivor in
+//               the row have R = 0 and count exp(0) = 1 in its denominator;
+//   k_rg_filter warp per row: batch, coverage over the batch's entries, the
+//               survivors compacted in place, the next gains.
+// While many survivors remain, a whole-GPU round is cheaper than a round of
+// the cluster kernel (16 SMs).  Every reduction is an integer sum, so the
+// result does not depend on the order blocks run in.  The cluster kernel
+// (k_select) continues from the first round not done here; info[b] carries the
+// pool size, the tokens selected so far and the rounds done.
 #include "common.cuh"
 #include "kernels.cuh"
 #include "select_common.cuh"
@@ -27,10 +39,15 @@ __global__ void __launch_bounds__(512) k_r0_pool(const long long* __restrict__ u
   grid_dep_wait();
   extern __shared__ __align__(16) char sm_r0p[];
   const int b = blockIdx.x;
-  // the accumulators of the next two kernels start at zero
+  // the accumulators of the next two kernels start at zero; nothing selected yet
   for (int k = threadIdx.x; k < P; k += blockDim.x) s0[(size_t)b * P + k] = 0;
   for (int j = threadIdx.x; j < N; j += blockDim.x) u1[(size_t)b * N + j] = 0;
   if (threadIdx.x < 4) fv[(size_t)b * 4 + threadIdx.x] = 0;
+  if (threadIdx.x == 0) {
+    info[b * 4 + 1] = 0;
+    info[b * 4 + 2] = 0;
+    info[b * 4 + 3] = 0;
+  }
   if (toff && text_geom(toff, b, B, Tmax, nullptr).T == 0) {
     if (threadIdx.x == 0) info[b * 4] = 0;
     return;
@@ -149,7 +166,10 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_filter(
   __syncthreads();
   if (blockIdx.x == 0) {  // record the first batch once per image
     for (int q = threadIdx.x; q < nb; q += blockDim.x) order[(size_t)b * K + q] = batch[q];
-    if (threadIdx.x == 0) info[b * 4 + 1] = nb;
+    if (threadIdx.x == 0) {
+      info[b * 4 + 1] = nb;  // selected so far
+      info[b * 4 + 2] = 1;   // rounds done
+    }
     if (tv.base) {
       int32_t* tp = tv.at<int32_t>(b, tv.off_pool);
       for (int k = threadIdx.x; k < tv.pool_size; k += blockDim.x) tp[k] = k < Pt ? pool[k] : -1;
@@ -245,6 +265,217 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_filter(
     if (uacc[j]) atomicAdd(&ub[j], uacc[j]);
 }
 
+// ---- sparse rounds on the whole GPU -------------------------------------------
+
+__global__ void __launch_bounds__(512) k_rg_pool(const long long* __restrict__ ucur,
+                                                   long long* unext, int B, int N, int K, int P,
+                                                   const int32_t* toff, int Tmax,
+                                                   const int32_t* __restrict__ order,
+                                                   int32_t* pool0, int32_t* info, long long* sc,
+                                                   TraceView tv) {
+  grid_dep_wait();
+  extern __shared__ __align__(16) char sm_rgp[];
+  const int b = blockIdx.x;
+  for (int k = threadIdx.x; k < P; k += blockDim.x) sc[(size_t)b * P + k] = 0;
+  for (int j = threadIdx.x; j < N; j += blockDim.x) unext[(size_t)b * N + j] = 0;
+  const int S = info[b * 4 + 1], rd = info[b * 4 + 2];
+  // nothing to do here once the budget is met or when the first round found
+  // no gain: the cluster kernel handles those cases
+  const bool skip = (toff && text_geom(toff, b, B, Tmax, nullptr).T == 0) || rd == 0 || S >= K;
+  if (skip) {
+    if (threadIdx.x == 0) info[b * 4] = 0;
+    return;
+  }
+  sel::PoolScratch w;
+  char* p = sm_rgp;
+  w.hist = reinterpret_cast<int*>(p);       p += sizeof(int) * sel::HBINS;
+  w.bnd = reinterpret_cast<int*>(p);        p += sizeof(int) * N;
+  w.wsum = reinterpret_cast<int*>(p);       p += sizeof(int) * 32;
+  w.scal = reinterpret_cast<int*>(p);       p += sizeof(int) * 8;
+  int* pool = reinterpret_cast<int*>(p);    p += sizeof(int) * P;
+  w.tmp = reinterpret_cast<int*>(p);        p += sizeof(int) * P;
+  unsigned char* self = reinterpret_cast<unsigned char*>(p);
+  for (int j = threadIdx.x; j < N; j += blockDim.x) self[j] = 0;
+  for (int h = threadIdx.x; h < sel::HBINS; h += blockDim.x) w.hist[h] = 0;
+  __syncthreads();
+  for (int q = threadIdx.x; q < S; q += blockDim.x) self[order[(size_t)b * K + q]] = 1;
+  __syncthreads();
+  const int Pt = sel::select_pool(ucur + (size_t)b * N, self, N, P, w, pool, nullptr);
+  for (int k = threadIdx.x; k < P; k += blockDim.x) pool0[(size_t)b * P + k] = k < Pt ? pool[k] : -1;
+  if (threadIdx.x == 0) {
+    info[b * 4] = Pt;
+    info[b * 4 + 3] = S;
+  }
+  if (tv.base && Pt > 0) {
+    int32_t* tp = tv.at<int32_t>(b, tv.off_pool) + (size_t)rd * tv.pool_size;
+    for (int k = threadIdx.x; k < tv.pool_size; k += blockDim.x) tp[k] = k < Pt ? pool[k] : -1;
+  }
+}
+
+__global__ void __launch_bounds__(32 * R0_ROWS) k_rg_rho(
+    const float* __restrict__ C, const uint16_t* __restrict__ scol,
+    const float* __restrict__ bcov, const int32_t* __restrict__ cnt, int B, int N, int Mstride,
+    int H, int L2, const int32_t* toff, int Tmax, int uniform_rows,
+    const int32_t* __restrict__ pool0, const int32_t* __restrict__ info, int P, float resp_temp,
+    float resp_eps, int fx_exp, const int32_t* fexp, long long* sc) {
+  grid_dep_wait();
+  __shared__ long long sblk[GMC_MAX_POOL];
+  __shared__ int fslot[R0_ROWS][GMC_MAX_POOL];  // a row's pool entries: slot and residual
+  __shared__ float fres[R0_ROWS][GMC_MAX_POOL];
+  extern __shared__ short pslot[];              // [N] pool slot of every token or -1
+  const int b = blockIdx.y;
+  const int Pt = info[b * 4];
+  if (Pt == 0) return;
+  int Mb = Mstride;
+  if (!uniform_rows) Mb = H * text_geom(toff, b, B, Tmax, nullptr).T + N + L2;
+  const int m0 = blockIdx.x * R0_ROWS;
+  if (m0 >= Mb) return;
+  const float fxs = ldexpf(1.f, fexp ? fexp[b] : fx_exp);
+  for (int j = threadIdx.x; j < N; j += blockDim.x) pslot[j] = -1;
+  for (int k = threadIdx.x; k < P; k += blockDim.x) sblk[k] = 0;
+  __syncthreads();
+  for (int k = threadIdx.x; k < Pt; k += blockDim.x) pslot[pool0[(size_t)b * P + k]] = (short)k;
+  __syncthreads();
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, m = m0 + w;
+  if (m < Mb) {
+    const size_t row = (size_t)b * Mstride + m;
+    const int n = cnt[row];
+    const float bm = bcov[row];
+    const float* vals = C + row * N;
+    const uint16_t* cols = scol + row * N;
+    const unsigned lt = sel::lanemask_lt();
+    int nf = 0;
+    float rmax = 0.f;
+    for (int e0 = 0; e0 < n; e0 += 32) {
+      const int e = e0 + lane;
+      int ps = -1;
+      float R = 0.f;
+      if (e < n) {
+        ps = pslot[cols[e]];
+        if (ps >= 0) R = vals[e] - bm;  // > 0: a survivor exceeds its coverage
+      }
+      const unsigned bal = __ballot_sync(FULL, ps >= 0);
+      if (ps >= 0) {
+        const int at = nf + __popc(bal & lt);
+        fslot[w][at] = ps;
+        fres[w][at] = R;
+        rmax = fmaxf(rmax, R);
+      }
+      nf += __popc(bal);
+    }
+    rmax = warp_max(rmax);
+    __syncwarp();
+    if (nf > 0) {
+      const float tau = resp_temp * rmax + resp_eps;
+      float z = 0.f;
+      for (int q = lane; q < nf; q += 32) z += expf(fres[w][q] / tau);
+      z = warp_sum(z) + (float)(Pt - nf);  // pool tokens without a survivor here: exp(0)
+      const float invz = 1.f / z;
+      for (int q = lane; q < nf; q += 32) {
+        const float R = fres[w][q];
+        atomicAdd((unsigned long long*)&sblk[fslot[w][q]],
+                  (unsigned long long)to_fix(expf(R / tau) * invz * R, fxs));
+      }
+    }
+  }
+  __syncthreads();
+  for (int k = threadIdx.x; k < Pt; k += blockDim.x)
+    if (sblk[k]) atomicAdd((unsigned long long*)&sc[(size_t)b * P + k], (unsigned long long)sblk[k]);
+}
+
+__global__ void __launch_bounds__(32 * R0_ROWS) k_rg_filter(
+    float* C, uint16_t* scol, int B, int N, int K, int Mstride, int H, int L2,
+    const int32_t* toff, int Tmax, int uniform_rows, const int32_t* __restrict__ pool0,
+    int32_t* info, const long long* __restrict__ sc0, int P, int bsz, int fx_exp,
+    const int32_t* fexp, long long* unext, float* bcov, int32_t* cnt, int32_t* order,
+    TraceView tv) {
+  grid_dep_wait();
+  __shared__ int pool[GMC_MAX_POOL];
+  __shared__ long long sc[GMC_MAX_POOL];
+  __shared__ int batch[GMC_MAX_POOL];
+  extern __shared__ unsigned long long uacc[];  // [N] then the batch flags [N] (bytes)
+  unsigned char* inb = reinterpret_cast<unsigned char*>(uacc + N);
+  const int b = blockIdx.y;
+  const int Pt = info[b * 4];
+  if (Pt == 0) return;
+  int Mb = Mstride;
+  if (!uniform_rows) Mb = H * text_geom(toff, b, B, Tmax, nullptr).T + N + L2;
+  const int m0 = blockIdx.x * R0_ROWS;
+  if (m0 >= Mb) return;
+  const int S = info[b * 4 + 3], rd = info[b * 4 + 2];
+  const float fxs = ldexpf(1.f, fexp ? fexp[b] : fx_exp);
+  const int nb = min(bsz, min(Pt, K - S));
+  for (int k = threadIdx.x; k < Pt; k += blockDim.x) {
+    pool[k] = pool0[(size_t)b * P + k];
+    sc[k] = sc0[(size_t)b * P + k];
+  }
+  for (int j = threadIdx.x; j < N; j += blockDim.x) {
+    uacc[j] = 0;
+    inb[j] = 0;
+  }
+  __syncthreads();
+  {
+    const int lane = threadIdx.x & 31, gl = lane & 7;
+    const unsigned gm = 0xFFu << (lane & 24);
+    for (int k = threadIdx.x >> 3; k < Pt; k += blockDim.x >> 3) {  // 8 lanes per pool token
+      const int rank = sel::group_score_rank(sc, pool, Pt, k, gl, gm);
+      if (gl == 0 && rank < nb) batch[rank] = pool[k];
+    }
+  }
+  __syncthreads();
+  for (int q = threadIdx.x; q < nb; q += blockDim.x) inb[batch[q]] = 1;
+  if (blockIdx.x == 0) {  // record the batch once per image
+    for (int q = threadIdx.x; q < nb; q += blockDim.x) order[(size_t)b * K + S + q] = batch[q];
+    if (threadIdx.x == 0) {
+      info[b * 4 + 1] = S + nb;
+      info[b * 4 + 2] = rd + 1;
+      if (tv.base) tv.at<int32_t>(b, tv.off_round_end)[rd] = S + nb;
+    }
+  }
+  __syncthreads();
+  const int lane = threadIdx.x & 31, m = m0 + (threadIdx.x >> 5);
+  if (m < Mb) {
+    const size_t row = (size_t)b * Mstride + m;
+    const int n = cnt[row];
+    float* vals = C + row * N;
+    uint16_t* cols = scol + row * N;
+    float bnew = bcov[row];
+    for (int e = lane; e < n; e += 32)
+      if (inb[cols[e]]) bnew = fmaxf(bnew, vals[e]);
+    bnew = warp_max(bnew);
+    const long long fb_new = to_fix(bnew, fxs);
+    const unsigned lt = sel::lanemask_lt();
+    int wr = 0;
+    for (int e0 = 0; e0 < n; e0 += 32) {
+      const int e = e0 + lane;
+      float c = 0.f;
+      int j = 0;
+      if (e < n) {
+        c = vals[e];
+        j = cols[e];
+      }
+      const bool keep = e < n && c > bnew;
+      const unsigned bal = __ballot_sync(FULL, keep);
+      __syncwarp();  // the chunk is read before any survivor moves down into it
+      if (keep) {
+        const int pos = wr + __popc(bal & lt);
+        vals[pos] = c;
+        cols[pos] = (uint16_t)j;
+        atomicAdd(&uacc[j], (unsigned long long)(to_fix(c, fxs) - fb_new));
+      }
+      wr += __popc(bal);
+    }
+    if (lane == 0) {
+      bcov[row] = bnew;
+      cnt[row] = wr;
+    }
+  }
+  __syncthreads();
+  unsigned long long* ub = reinterpret_cast<unsigned long long*>(unext + (size_t)b * N);
+  for (int j = threadIdx.x; j < N; j += blockDim.x)
+    if (uacc[j]) atomicAdd(&ub[j], uacc[j]);
+}
+
 cudaError_t launch_round0(const R0State& r0, int B, int N, int K, int M, const int32_t* toff,
                           int H, int T, int L2, const gmc_params& p, int fx_exp,
                           const int32_t* fexp, float* C, uint16_t* scol, const long long* u0,
@@ -267,7 +498,31 @@ cudaError_t launch_round0(const R0State& r0, int B, int N, int K, int M, const i
   launch_k(k_r0_filter, grid, 32 * R0_ROWS, fsm, st, 1, C, scol, B, N, K, M, H, L2, toff, T, uniform, r0.pool,
                                              r0.info, r0.s0, P, p.batch_b, fx_exp, fexp, r0.u1,
                                              r0.bcov, r0.cnt, r0.fv, order, tv);
-  return cudaGetLastError();
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  // sparse rounds: gains alternate between u1 and u2
+  const size_t psm = smem;  // the pool kernel's layout is round 0's
+  if ((e = set_smem_limit((const void*)k_rg_pool, psm)) != cudaSuccess) return e;
+  const size_t rsm = sizeof(short) * (size_t)N;
+  if ((e = set_smem_limit((const void*)k_rg_rho, rsm)) != cudaSuccess) return e;
+  const size_t gsm = sizeof(unsigned long long) * (size_t)N + (size_t)N;
+  if ((e = set_smem_limit((const void*)k_rg_filter, gsm)) != cudaSuccess) return e;
+  for (int rr = 1; rr <= SPARSE_GPU_ROUNDS; ++rr) {
+    long long* ucur = rr % 2 == 1 ? r0.u1 : r0.u2;
+    long long* unext = rr % 2 == 1 ? r0.u2 : r0.u1;
+    launch_k(k_rg_pool, B, 512, psm, st, 1, (const long long*)ucur, unext, B, N, K, P,
+             uniform ? nullptr : toff, T, (const int32_t*)order, r0.pool, r0.info, r0.s0, tv);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    launch_k(k_rg_rho, grid, 32 * R0_ROWS, rsm, st, 1, (const float*)C, (const uint16_t*)scol,
+             (const float*)r0.bcov, (const int32_t*)r0.cnt, B, N, M, H, L2, toff, T, uniform,
+             (const int32_t*)r0.pool, (const int32_t*)r0.info, P, p.resp_temp, p.resp_eps, fx_exp,
+             fexp, r0.s0);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    launch_k(k_rg_filter, grid, 32 * R0_ROWS, gsm, st, 1, C, scol, B, N, K, M, H, L2, toff, T,
+             uniform, (const int32_t*)r0.pool, r0.info, (const long long*)r0.s0, P, p.batch_b,
+             fx_exp, fexp, unext, r0.bcov, r0.cnt, order, tv);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  }
+  return cudaSuccess;
 }
 
 }  // namespace gmc

@@ -225,14 +225,16 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
   float* Cimg = a.C + (size_t)b * a.Mstride * N;
   uint16_t* Simg = a.scol + (size_t)b * a.Mstride * N;
 
-  // state after the first round (k_round0.cu); a first round with an empty
-  // pool leaves the gains of the empty support and nothing selected
-  const int Pt0 = valid ? a.r0.info[b * 4] : 0;
-  const int nb0 = Pt0 > 0 ? a.r0.info[b * 4 + 1] : 0;
+  // state after the rounds run on the whole GPU (k_round0.cu); a first round
+  // with an empty pool leaves the gains of the empty support and nothing
+  // selected
+  const int rd0 = valid ? a.r0.info[b * 4 + 2] : 0;  // rounds done
+  const int Pt0 = rd0;                                // > 0: the rounds left survivor lists
+  const int nb0 = rd0 > 0 ? a.r0.info[b * 4 + 1] : 0;  // tokens selected so far
   for (int j = threadIdx.x; j < N; j += blockDim.x) {
     s.u_lo[j] = 0;
     s.u_hi[j] = 0;
-    s.u_full[j] = Pt0 > 0 ? a.r0.u1[(size_t)b * N + j] : a.u0[(size_t)b * N + j];
+    s.u_full[j] = rd0 > 0 ? a.r0.ugain[(size_t)b * N + j] : a.u0[(size_t)b * N + j];
     s.poolslot[j] = -1;
     s.sel[j] = 0;
   }
@@ -357,7 +359,7 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
   if (Pt0 > 0) migrate();
 
   const int rounds_max = (K + a.bsz - 1) / a.bsz + 1;
-  int S_count = nb0, rnd = Pt0 > 0 ? 1 : 0, filled = 0;
+  int S_count = nb0, rnd = rd0, filled = 0;
   const int sub = lane / G, gl = lane % G;
   const int gid = wid * (32 / G) + sub, ngrp = nw * (32 / G);  // 8-lane groups of the block
   const unsigned gm = 0xFFu << (sub * G);

@@ -89,12 +89,19 @@ cudaError_t launch_gram(const Dims&, const void* hidden, Scratch&, cudaStream_t)
 cudaError_t launch_build_clients(const Dims&, const gmc_params&, int fx_exp, Scratch&,
                                  cudaStream_t);
 // State left by the first (dense) selection round, run over the whole GPU.
+// Rounds of the solver run on the whole GPU before the cluster kernel takes
+// over: the dense first round, then this many sparse rounds.
+constexpr int SPARSE_GPU_ROUNDS = 2;
+
 struct R0State {
-  int32_t* pool;   // [B][P]  first-round pool (-1 padded)
-  int32_t* info;   // [B][4]  pool size, batch size
-  long long* s0;   // [B][P]  first-round scores (fixed point)
-  long long* u1;   // [B][N]  second-round gains (fixed point)
-  float* bcov;     // [B][M]  coverage b_m after the first batch
+  int32_t* pool;   // [B][P]  pool of the current whole-GPU round (-1 padded)
+  int32_t* info;   // [B][4]  pool size of the current round, tokens selected so far,
+                   //         rounds done, tokens selected before the current round
+  long long* s0;   // [B][P]  scores of the current round (fixed point)
+  long long* u1;   // [B][N]  gains (fixed point), written by rounds 0, 2, ...
+  long long* u2;   // [B][N]  gains written by rounds 1, 3, ...
+  long long* ugain;  // u1 or u2: the gains the cluster kernel starts from
+  float* bcov;     // [B][M]  coverage b_m after the last whole-GPU round
   int32_t* cnt;    // [B][M]  survivors per row (lists in place over Cbar / scol)
   long long* fv;   // [B][4]  F_b(V) per bank (fixed point)
 };
