@@ -91,7 +91,7 @@ cudaError_t launch_build_clients(const Dims&, const gmc_params&, int fx_exp, Scr
 // State left by the first (dense) selection round, run over the whole GPU.
 // Rounds of the solver run on the whole GPU before the cluster kernel takes
 // over: the dense first round, then this many sparse rounds.
-constexpr int SPARSE_GPU_ROUNDS = 2;
+constexpr int SPARSE_GPU_ROUNDS = 8;
 
 struct R0State {
   int32_t* pool;   // [B][P]  pool of the current whole-GPU round (-1 padded)
