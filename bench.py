@@ -147,6 +147,11 @@ class ClockSampler:
 # ---------------------------------------------------------------------------
 # roofline bookkeeping (algorithmic work per stage, per call)
 # ---------------------------------------------------------------------------
+# sparse solver rounds run as whole-GPU kernels after the dense first one
+# (SPARSE_GPU_ROUNDS in the library's kernels.cuh)
+WIDE_ROUNDS = 8
+
+
 def stage_work(wl) -> dict:
     """Algorithmic bytes / flops each stage must move or compute for one call."""
     B, N, H, Hkv, d, D, K = wl.B, wl.N, wl.H, wl.Hkv, wl.d, wl.D, wl.K
@@ -157,11 +162,13 @@ def stage_work(wl) -> dict:
     w["gram"] = ("tensor", B * 2.0 * N * N * D)                        # the N x N cosine block
     w["message"] = ("hbm", B * (H * Tm * N * 4 + 2 * (N + Tm) * Hkv * d * es + Tm * H * d * es))
     w["clients"] = ("hbm", B * (M * N * 4 + H * Tm * N * 4 + N * N * 4))
-    # selection: one read of the M x N clients per round; the dense first round
-    # is its own stage, the rounds after it are k_select's
+    # selection: one read of the M x N clients per round.  Stage "rounds_gpu"
+    # runs the dense first round and the next WIDE_ROUNDS sparse rounds as
+    # whole-GPU kernels; stage "select" (the cluster kernel) runs the rest.
     rounds = -(-K // 16)
-    w["round0"] = ("hbm", B * (M * N * 4.0))
-    w["select"] = ("hbm", B * (rounds - 1) * (M * N * 4.0))
+    wide = min(rounds, 1 + WIDE_ROUNDS)
+    w["rounds_gpu"] = ("hbm", B * wide * (M * N * 4.0))
+    w["select"] = ("hbm", B * max(1, rounds - wide) * (M * N * 4.0))
     w["transport"] = ("hbm", B * ((N + Tm) * D * es + (K + Tm) * D * es
                                   + 2 * (K + Tm) * 2 * Hkv * d * es + 2 * 3 * (K + Tm) * 4 + 3 * N * 4))
     w["heads"] = ("hbm", B * (H * Tm * N * 4))

@@ -411,7 +411,7 @@ int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* 
     GMC_TRY(cudaStreamWaitEvent(st, sd->join, 0));
   }
   GMC_STAGE("clients", 1, launch_build_clients(dm, p, fx, s, st));
-  GMC_STAGE("round0", 3 + 3 * SPARSE_GPU_ROUNDS,
+  GMC_STAGE("rounds_gpu", 3 + 3 * SPARSE_GPU_ROUNDS,
             launch_round0(r0, dm.B, N, Ke, dm.M, dm.toff, H, T, p.landmarks * p.landmarks, p, fx,
                           nullptr, s.C, s.scol, s.u0, s.order, s.status, tv, st));
   GMC_STAGE("select", 1,
