@@ -47,7 +47,8 @@ __global__ void k_head_stats(const float* __restrict__ A, const float* __restric
   float* Abuf = sm_hs;                          // [2][Hp][HG_RS], rows >= H stay zero
   float* acc = Abuf + 2 * (size_t)Hp * HG_RS;   // [2][npairs][HG_TOK], one per block half
   float* w2 = acc + 2 * (size_t)npairs * HG_TOK;  // [2][H][HG_TOK]
-  unsigned short* tiles = reinterpret_cast<unsigned short*>(w2 + 2 * H * HG_TOK);  // [ntiles]
+  float4* zs = reinterpret_cast<float4*>(w2 + 2 * H * HG_TOK);  // [H][HG_TOK] probe values
+  unsigned short* tiles = reinterpret_cast<unsigned short*>(zs + H * HG_TOK);  // [ntiles]
   const int i0 = blockIdx.x * HG_TOK;
   for (int p = threadIdx.x; p < 2 * npairs * HG_TOK; p += blockDim.x) acc[p] = 0.f;
   for (int p = threadIdx.x; p < 2 * H * HG_TOK; p += blockDim.x) w2[p] = 0.f;
@@ -60,15 +61,42 @@ __global__ void k_head_stats(const float* __restrict__ A, const float* __restric
     for (int hb = 0; hb < nhb; ++hb)
       for (int gb = hb; gb < nhb; ++gb) tiles[p++] = (unsigned short)(hb * 256 + gb);
   }
-  // Queries in pairs of HG_TC-chunks: both are staged with cp.async, then the
-  // two halves of the block work on one chunk each into their own sums.
+  // the block's probe values Z_h[i] for every head (used by the output step)
+  for (int q = threadIdx.x; q < H * HG_TOK; q += blockDim.x) {
+    const int h = q / HG_TOK, i = i0 + q % HG_TOK;
+    zs[q] = i < N ? reinterpret_cast<const float4*>(Z)[((size_t)b * H + h) * N + i]
+                  : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+  // Queries in pairs of HG_TC-chunks: both are staged, then the two halves of
+  // the block work on one chunk each into their own sums.  The HG_TOK tokens
+  // of one (head, query) row are read as 16-byte loads when the rows of A
+  // start on 16 bytes (N % 4 == 0) and the block is not the ragged last one
+  // (the padded shared rows are not 16-byte aligned, so these go through
+  // registers); otherwise as 4-byte cp.async copies.
+  const bool vec = (N & 3) == 0 && i0 + HG_TOK <= N;
   auto stage = [&](int t0, float* buf) {
     const int tc = min(HG_TC, Tb - t0);
-    for (int idx = threadIdx.x; idx < H * HG_TC * HG_TOK; idx += blockDim.x) {
-      const int h = idx / (HG_TC * HG_TOK), tt = (idx / HG_TOK) % HG_TC, ii = idx % HG_TOK;
-      const bool in = tt < tc && i0 + ii < N;
-      const float* src = in ? A + (((size_t)b * H + h) * Tmax + t0 + tt) * N + i0 + ii : A;
-      cp_async4(buf + h * HG_RS + tt * HG_TOK + ii, src, in);
+    if (vec) {
+      constexpr int V = HG_TOK / 4;  // 16-byte pieces per row
+      for (int idx = threadIdx.x; idx < H * HG_TC * V; idx += blockDim.x) {
+        const int h = idx / (HG_TC * V), tt = (idx / V) % HG_TC, v = idx % V;
+        float* dst = buf + h * HG_RS + tt * HG_TOK + 4 * v;
+        float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (tt < tc)
+          x = *reinterpret_cast<const float4*>(A + (((size_t)b * H + h) * Tmax + t0 + tt) * N + i0 +
+                                               4 * v);
+        dst[0] = x.x;
+        dst[1] = x.y;
+        dst[2] = x.z;
+        dst[3] = x.w;
+      }
+    } else {
+      for (int idx = threadIdx.x; idx < H * HG_TC * HG_TOK; idx += blockDim.x) {
+        const int h = idx / (HG_TC * HG_TOK), tt = (idx / HG_TOK) % HG_TC, ii = idx % HG_TOK;
+        const bool in = tt < tc && i0 + ii < N;
+        const float* src = in ? A + (((size_t)b * H + h) * Tmax + t0 + tt) * N + i0 + ii : A;
+        cp_async4(buf + h * HG_RS + tt * HG_TOK + ii, src, in);
+      }
     }
     cp_async_commit();
   };
@@ -136,8 +164,8 @@ __global__ void k_head_stats(const float* __restrict__ A, const float* __restric
     for (int ii = 0; ii < HG_TOK; ++ii) {
       const int i = i0 + ii;
       if (i >= N) break;
-      const float4 zh = reinterpret_cast<const float4*>(Z)[((size_t)b * H + h) * N + i];
-      const float4 zg = reinterpret_cast<const float4*>(Z)[((size_t)b * H + g) * N + i];
+      const float4 zh = zs[h * HG_TOK + ii];
+      const float4 zg = zs[g * HG_TOK + ii];
       const float w = fmaf(zh.x, zg.x, fmaf(zh.y, zg.y, fmaf(zh.z, zg.z, fmaf(zh.w, zg.w, sh * sgv))));
       v = fmaf(w, acc[pi * HG_TOK + ii] + acc[((size_t)npairs + pi) * HG_TOK + ii], v);
     }
@@ -331,7 +359,7 @@ cudaError_t launch_heads(const Dims& dm, const gmc_params& p, Scratch& s, const 
   const int nhb = (H + HG_HB - 1) / HG_HB;
   size_t smem = sizeof(float) * (2 * (size_t)nhb * HG_HB * HG_RS + 2 * (size_t)npairs * HG_TOK +
                                  2 * H * HG_TOK) +
-                sizeof(unsigned short) * (nhb * (nhb + 1) / 2) + 16;
+                sizeof(float4) * H * HG_TOK + sizeof(unsigned short) * (nhb * (nhb + 1) / 2) + 16;
   cudaError_t e = set_smem_limit((const void*)k_head_stats, smem);
   if (e != cudaSuccess) return e;
   launch_k(k_head_stats, dim3(s.nHG, dm.B), 512, smem, st, 1, s.A, s.Z, s.sigma, dm.toff, dm.B, dm.N, dm.T,
