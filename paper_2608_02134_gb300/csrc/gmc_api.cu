@@ -95,12 +95,13 @@ size_t carve_compress(const Dims& dm, Scratch* s, char* base, R0State* r0s = nul
   t.nA = ceil_div(dm.N, ASSIGN_WARPS);
   t.nE = t.nA;  // energy block sums come from the assignment gap kernel
   t.nSel = 0;
-  // status word, one probe and one assignment ticket per image, then the
-  // carrier membership bitmaps: one block, zeroed by one memset per call
-  t.status = c.take<uint32_t>(4 + 2 * B + B * K * (size_t)ceil_div(dm.N, 32));
+  // status word, the probe, head-Gram and assignment tickets of every image,
+  // then the carrier membership bitmaps: one block, zeroed by one memset per call
+  t.status = c.take<uint32_t>(4 + 3 * B + B * K * (size_t)ceil_div(dm.N, 32));
   t.tick = t.status + 4;
   t.tick2 = t.tick + B;
-  t.mbits = t.tick2 + B;
+  t.tick3 = t.tick2 + B;
+  t.mbits = t.tick3 + B;
   t.gatev = c.take<float>(B * 4);
   t.A = c.take<float>(B * H * T * N);
   t.nRS = message_splits(dm);
@@ -380,7 +381,7 @@ int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* 
   std::lock_guard<std::mutex> lk(g_prof.mu);
   // status, tickets, membership bitmaps
   GMC_TRY(cudaMemsetAsync(
-      s.status, 0, sizeof(uint32_t) * (4 + 2 * dm.B + (size_t)dm.B * dm.K * ceil_div(dm.N, 32)),
+      s.status, 0, sizeof(uint32_t) * (4 + 3 * dm.B + (size_t)dm.B * dm.K * ceil_div(dm.N, 32)),
       st));
   if (Ke == N) {  // K = N returns the unmodified execution
     GMC_TRY(launch_identity(dm, hidden, keys, pos_ids, out_idx, out_hidden, out_kv, out_pos,
@@ -394,7 +395,7 @@ int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* 
     GMC_STAGE("rownorm", 1, launch_rownorm(dm, hidden, p.norm_eps, s, st));
     GMC_STAGE("probe", 1, launch_probe(dm, keys, vo_probe, p, s, st));
     GMC_STAGE("message", message_tc_supported(dm) ? 3 : 1, launch_message(dm, keys, queries, s, st));
-    GMC_STAGE("heads", 3, launch_heads(dm, p, s, tv, st));
+    GMC_STAGE("heads", 2, launch_heads(dm, p, s, tv, st));
     GMC_STAGE("gram", 1, launch_gram(dm, hidden, s, st));
   } else {
     // row norms and the cosine Gram run beside probe -> message -> heads
@@ -407,7 +408,7 @@ int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* 
     GMC_TRY(cudaEventRecord(sd->join, sd->st));
     GMC_STAGE("probe", 1, launch_probe(dm, keys, vo_probe, p, s, st));
     GMC_STAGE("message", message_tc_supported(dm) ? 3 : 1, launch_message(dm, keys, queries, s, st));
-    GMC_STAGE("heads", 3, launch_heads(dm, p, s, tv, st));
+    GMC_STAGE("heads", 2, launch_heads(dm, p, s, tv, st));
     GMC_TRY(cudaStreamWaitEvent(st, sd->join, 0));
   }
   GMC_STAGE("clients", 1, launch_build_clients(dm, p, fx, s, st));

@@ -178,15 +178,13 @@ __global__ void k_head_stats(const float* __restrict__ A, const float* __restric
   }
 }
 
-// One block per image: reduce the Gram, then one warp runs farthest-first
-// clustering and the head weights (two heads per lane, H <= 64).
 // Ties: the first centre is the lowest-index largest pattern, each next centre
 // the lowest-index head of smallest max-cosine, and a head joins the earliest
 // centre among equally similar ones.
-__device__ __forceinline__ void warp_argbest(double& v, int& idx, bool want_max) {
+__device__ __forceinline__ void warp_argbest(float& v, int& idx, bool want_max) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
-    const double ov = __shfl_xor_sync(FULL, v, o);
+    const float ov = __shfl_xor_sync(FULL, v, o);
     const int oi = __shfl_xor_sync(FULL, idx, o);
     const bool better = want_max ? (ov > v || (ov == v && oi < idx))
                                  : (ov < v || (ov == v && oi < idx));
@@ -194,68 +192,34 @@ __device__ __forceinline__ void warp_argbest(double& v, int& idx, bool want_max)
   }
 }
 
-// The pattern Gram: sum of the token-block partials, one warp per (image, entry),
-// lanes over the blocks (fixed order, so the sum is reproducible).  Further
-// warps sum every head's atom norms sum_t rs[h,t] (rs in nRS parts per query).
-// HG[b] holds the H*H Gram followed by the H atom-norm totals.
-__global__ void k_hg_reduce(const double* __restrict__ hgpart, int nHG, int B, int H,
-                            const float* __restrict__ rs, int nRS, const int32_t* toff,
-                            int Tmax, double* HG) {
-  grid_dep_wait();
-  const int w = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
-  const int HH = H * H, HE = HH + H;
-  if (w >= B * HE) return;
-  const int b = w / HE, p = w % HE;
-  double s = 0.0;
-  if (p < HH) {
-    for (int k = lane; k < nHG; k += 32) s += hgpart[((size_t)b * nHG + k) * HH + p];
-  } else {
-    const int h = p - HH;
-    const TextGeom tg = text_geom(toff, b, B, Tmax, nullptr);
-    const float* r = rs + ((size_t)b * H + h) * nRS * Tmax;
-    for (int k = lane; k < nRS * Tmax; k += 32)
-      if (k % Tmax < tg.T) s += r[k];
-  }
-  s = warp_sum(s);
-  if (lane == 0) HG[(size_t)b * HE + p] = s;
-}
-
-__global__ void k_head_cluster(const double* __restrict__ HGred,
-                               const int32_t* toff, int B, int N, int Tmax, int H,
-                               int max_clusters, float head_eps, float* omega,
-                               TraceView tv, uint32_t* status) {
-  grid_dep_wait();
-  extern __shared__ double sm_hc[];
-  const int b = blockIdx.x;
-  const TextGeom tg = text_geom(toff, b, B, Tmax, status);
-  if (tg.T == 0) return;
+// Farthest-first head clusters and head weights of image b from its reduced
+// pattern Gram (fp64 sums, read past L1: other blocks wrote them).  The
+// cosines, dispersions and weights are fp32: the weights enter as
+// 1 / (dispersion + head_eps) with head_eps = 0.05 by default, far above the
+// fp32 rounding of a cosine.  One block of 256 threads, one warp for the
+// centres (two heads per lane, H <= 64).
+__device__ void cluster_heads(const double* hgb, int b, int T, int N, int H, int max_clusters,
+                              float head_eps, float* omega, const TraceView& tv, float* sm) {
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-  double* HG = sm_hc;                   // [H*H]
-  double* cs = HG + H * H;              // [H*H] pattern cosines
-  double* pre = cs + H * H;             // [H]   pattern norm / mean atom norm
-  double* dot = pre + H;                // [H]   1/||U_h||, later h's cosine sum in its cluster
-  double* inv = dot + H;                // [H]   1 / (dispersion + eps)
-  double* csum = inv + H;               // [GMC_MAX_HEADS] 1 / norm of a cluster's sum
-  double* isum = csum + GMC_MAX_HEADS;  // [GMC_MAX_HEADS]
+  float* cs = sm;                       // [H*H] pattern cosines
+  float* pre = cs + H * H;              // [H]   pattern norm / mean atom norm
+  float* dot = pre + H;                 // [H]   1/||U_h||, later h's cosine sum in its cluster
+  float* inv = dot + H;                 // [H]   1 / (dispersion + eps)
+  float* csum = inv + H;                // [GMC_MAX_HEADS] 1 / norm of a cluster's sum
+  float* isum = csum + GMC_MAX_HEADS;   // [GMC_MAX_HEADS]
   int* asg = reinterpret_cast<int*>(isum + GMC_MAX_HEADS);  // [H] cluster of every head
   int* cent = asg + H;                  // [GMC_MAX_HEADS] centres
   int* ccnt = cent + GMC_MAX_HEADS;     // [GMC_MAX_HEADS] cluster sizes
-  const double* hgb = HGred + (size_t)b * (H * H + H);
-  for (int p = threadIdx.x; p < H * H; p += blockDim.x) HG[p] = hgb[p];
-  for (int h = threadIdx.x; h < H; h += blockDim.x) pre[h] = hgb[H * H + h];  // sum_t rs[h,t]
-  __syncthreads();
   for (int h = threadIdx.x; h < H; h += blockDim.x) {
-    const double mean = pre[h] / ((double)tg.T * N);
-    pre[h] = (mean > 0.0 && HG[h * H + h] > 0.0) ? sqrt(HG[h * H + h]) / mean : 0.0;
-  }
-  for (int h = threadIdx.x; h < H; h += blockDim.x) {  // 1 / ||U_h||, 0 for a zero pattern
-    const double a = HG[h * H + h];
-    dot[h] = a > 0.0 ? 1.0 / sqrt(a) : 0.0;
+    const double a = __ldcg(&hgb[h * H + h]);
+    const double mean = __ldcg(&hgb[H * H + h]) / ((double)T * N);  // sum_t rs[h,t] / (T N)
+    pre[h] = (mean > 0.0 && a > 0.0) ? (float)(sqrt(a) / mean) : 0.f;
+    dot[h] = a > 0.0 ? (float)(1.0 / sqrt(a)) : 0.f;  // 1 / ||U_h||, 0 for a zero pattern
   }
   __syncthreads();
   for (int p = threadIdx.x; p < H * H; p += blockDim.x) {
     const int h = p / H, g = p % H;
-    cs[p] = HG[p] * dot[h] * dot[g];
+    cs[p] = (float)__ldcg(&hgb[p]) * dot[h] * dot[g];
   }
   __syncthreads();
   const int nc = min(max_clusters, H);
@@ -263,7 +227,7 @@ __global__ void k_head_cluster(const double* __restrict__ HGred,
     const int h0 = lane, h1 = lane + 32;
     bool c0 = false, c1 = false;  // is h0 / h1 a centre
     {
-      double v = -1.0;
+      float v = -1.f;
       int idx = -1;
       if (h0 < H) { v = pre[h0]; idx = h0; }
       if (h1 < H && (idx < 0 || pre[h1] > v)) { v = pre[h1]; idx = h1; }
@@ -274,13 +238,13 @@ __global__ void k_head_cluster(const double* __restrict__ HGred,
     }
     __syncwarp();
     for (int c = 1; c < nc; ++c) {
-      double v = 0.0;
+      float v = 0.f;
       int idx = -1;
       for (int q = 0; q < 2; ++q) {
         const int h = q ? h1 : h0;
         if (h >= H || (q ? c1 : c0)) continue;
-        double mc = -INFINITY;
-        for (int k = 0; k < c; ++k) mc = fmax(mc, cs[h * H + cent[k]]);
+        float mc = -INFINITY;
+        for (int k = 0; k < c; ++k) mc = fmaxf(mc, cs[h * H + cent[k]]);
         if (idx < 0 || mc < v) { v = mc; idx = h; }
       }
       warp_argbest(v, idx, false);
@@ -302,7 +266,7 @@ __global__ void k_head_cluster(const double* __restrict__ HGred,
   // sums over heads as warp trees (two heads per lane, fixed order)
   const int nw = blockDim.x >> 5;
   for (int h = wid; h < H; h += nw) {
-    double d = 0.0;
+    float d = 0.f;
     if (lane < H && asg[lane] == asg[h]) d += cs[h * H + lane];
     if (lane + 32 < H && asg[lane + 32] == asg[h]) d += cs[h * H + lane + 32];
     d = warp_sum(d);
@@ -311,25 +275,25 @@ __global__ void k_head_cluster(const double* __restrict__ HGred,
   __syncthreads();
   // ||sum_{g in k} u_g||^2 (in cosine units) = sum over the cluster's dot values
   for (int k = wid; k < nc; k += nw) {
-    double sk = 0.0;
+    float sk = 0.f;
     int n = 0;
     if (lane < H && asg[lane] == k) { sk += dot[lane]; ++n; }
     if (lane + 32 < H && asg[lane + 32] == k) { sk += dot[lane + 32]; ++n; }
     sk = warp_sum(sk);
     n = warp_sum_int(n);
     if (lane == 0) {
-      csum[k] = sk > 0.0 ? 1.0 / sqrt(sk) : 0.0;  // 1 / ||sum_{g in k} u_g||
+      csum[k] = sk > 0.f ? rsqrtf(sk) : 0.f;  // 1 / ||sum_{g in k} u_g||
       ccnt[k] = n;
     }
   }
   __syncthreads();
   for (int h = threadIdx.x; h < H; h += blockDim.x) {
-    const double dh = 1.0 - dot[h] * csum[asg[h]];
-    inv[h] = 1.0 / (dh + head_eps);
+    const float dh = 1.f - dot[h] * csum[asg[h]];
+    inv[h] = 1.f / (dh + head_eps);
   }
   __syncthreads();
   for (int k = wid; k < nc; k += nw) {
-    double sk = 0.0;
+    float sk = 0.f;
     if (lane < H && asg[lane] == k) sk += inv[lane];
     if (lane + 32 < H && asg[lane + 32] == k) sk += inv[lane + 32];
     sk = warp_sum(sk);
@@ -339,7 +303,7 @@ __global__ void k_head_cluster(const double* __restrict__ HGred,
   int C = 0;
   for (int k = 0; k < nc; ++k) C += ccnt[k] > 0;
   for (int h = threadIdx.x; h < H; h += blockDim.x) {
-    const float w = (float)(inv[h] / isum[asg[h]] / C);
+    const float w = inv[h] / isum[asg[h]] / (float)C;
     omega[(size_t)b * H + h] = w;
     if (tv.base) {
       tv.at<int32_t>(b, tv.off_head_assign)[h] = asg[h];
@@ -351,6 +315,49 @@ __global__ void k_head_cluster(const double* __restrict__ HGred,
     int32_t* tc = tv.at<int32_t>(b, tv.off_centres);
     for (int k = threadIdx.x; k < max_clusters; k += blockDim.x) tc[k] = k < nc ? cent[k] : -1;
   }
+}
+
+// The pattern Gram of image blockIdx.y: sum of the token-block partials, one
+// warp per entry, lanes over the blocks (fixed order, so the sum is
+// reproducible); further warps sum every head's atom norms sum_t rs[h,t] (rs
+// in nRS parts per query).  HG[b] holds the H*H Gram followed by the H
+// atom-norm totals.  The image's last block to finish (ticket zeroed with the
+// status word) clusters the heads.
+__global__ void __launch_bounds__(256) k_hg_reduce(const double* __restrict__ hgpart, int nHG,
+                                                     int B, int N, int H,
+                                                     const float* __restrict__ rs, int nRS,
+                                                     const int32_t* toff, int Tmax, double* HG,
+                                                     uint32_t* tick, int max_clusters,
+                                                     float head_eps, float* omega, TraceView tv,
+                                                     uint32_t* status) {
+  grid_dep_wait();
+  extern __shared__ float sm_hc[];
+  __shared__ int last;
+  const int lane = threadIdx.x & 31, b = blockIdx.y;
+  const int HH = H * H, HE = HH + H;
+  const TextGeom tg = text_geom(toff, b, B, Tmax, status);
+  if (tg.T == 0) return;  // uniform over the image
+  const int p = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (p < HE) {
+    double s = 0.0;
+    if (p < HH) {
+      for (int k = lane; k < nHG; k += 32) s += hgpart[((size_t)b * nHG + k) * HH + p];
+    } else {
+      const int h = p - HH;
+      const float* r = rs + ((size_t)b * H + h) * nRS * Tmax;
+      for (int k = lane; k < nRS * Tmax; k += 32)
+        if (k % Tmax < tg.T) s += r[k];
+    }
+    s = warp_sum(s);
+    if (lane == 0) HG[(size_t)b * HE + p] = s;
+  }
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) last = atomicAdd(&tick[b], 1u) == gridDim.x - 1;
+  __syncthreads();
+  if (!last) return;
+  __threadfence();
+  cluster_heads(HG + (size_t)b * HE, b, tg.T, N, H, max_clusters, head_eps, omega, tv, sm_hc);
 }
 
 cudaError_t launch_heads(const Dims& dm, const gmc_params& p, Scratch& s, const TraceView& tv,
@@ -366,16 +373,12 @@ cudaError_t launch_heads(const Dims& dm, const gmc_params& p, Scratch& s, const 
                                                      H, p.terminal_q_weight, s.hgpart, s.nHG,
                                                      s.W2, s.status);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  const int warps = dm.B * (H * H + H);
-  launch_k(k_hg_reduce, ceil_div(warps * 32, 256), 256, 0, st, 1, s.hgpart, s.nHG, dm.B, H, s.rs, s.nRS,
-                                                         dm.toff, dm.T, s.HG);
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  size_t smem2 = sizeof(double) * (2 * (size_t)H * H + 3 * H + 2 * GMC_MAX_HEADS) +
-                 sizeof(int) * (H + 2 * GMC_MAX_HEADS);
-  if ((e = set_smem_limit((const void*)k_head_cluster, smem2)) != cudaSuccess) return e;
-  launch_k(k_head_cluster, dm.B, 256, smem2, st, 1, s.HG, dm.toff, dm.B, dm.N, dm.T, H,
-                                          p.max_head_clusters, p.head_eps, s.omega, tv, s.status);
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  const size_t smem2 = sizeof(float) * ((size_t)H * H + 3 * H + 2 * GMC_MAX_HEADS) +
+                       sizeof(int) * (H + 2 * GMC_MAX_HEADS);
+  if ((e = set_smem_limit((const void*)k_hg_reduce, smem2)) != cudaSuccess) return e;
+  launch_k(k_hg_reduce, dim3(ceil_div(H * H + H, 8), dm.B), 256, smem2, st, 1,
+           (const double*)s.hgpart, s.nHG, dm.B, dm.N, H, (const float*)s.rs, s.nRS, dm.toff, dm.T,
+           s.HG, s.tick3, p.max_head_clusters, p.head_eps, s.omega, tv, s.status);
   return cudaGetLastError();
 }
 

@@ -45,6 +45,7 @@ struct Scratch {
   float* sigpart;    // [B][nP][H]     block partials of ||Z_h||_F^2
   uint32_t* tick;    // [B]            last-block tickets of the probe (zeroed with status)
   uint32_t* tick2;   // [B]            last-block tickets of the assignment gap pass (same)
+  uint32_t* tick3;   // [B]            last-block tickets of the head-Gram reduction (same)
   float* gatev;      // [B][4]         Delta_bar, s_x, mean message energy
   float* sigma;      // [B][H]         mass coordinate sigma_h
   double* hgpart;    // [B][nHG][H*H]  block partials of the head-pattern Gram
