@@ -59,8 +59,10 @@ struct MsgCtl {
 // 32-column quarter w/4 of every tile), then the TMA producer and MMA warps.
 constexpr int FE_WARPS = 16, FT_THREADS = 32 * (FE_WARPS + 2);
 
-// Control block of the fused kernel: barriers and this CTA's per-row
-// statistics, read by the other CTAs of the cluster.
+constexpr int FUSED_MAX_CLUSTER = 8;  // portable cluster size
+
+// Control block of the fused kernel: barriers, this CTA's per-row statistics
+// and the statistics of every split of the cluster.
 struct FusedCtl {
   uint64_t qfull;
   uint64_t full[STAGES];
@@ -71,15 +73,24 @@ struct FusedCtl {
   float stat_m[4][BM];
   float stat_l[4][BM];
   float rsum[4][BM];
-  float cl_m[BM];  // the split's statistics per query row, for the whole cluster
-  float cl_l[BM];
+  // every split's statistics per query row (base-2 max, sum), written into
+  // each CTA of the cluster by the split that owns them
+  float all_m[FUSED_MAX_CLUSTER][BM];
+  float all_l[FUSED_MAX_CLUSTER][BM];
 };
 
 __device__ __forceinline__ void fused_epi_barrier() {
   asm volatile("bar.sync 1, %0;" ::"n"(FE_WARPS * 32) : "memory");
 }
 constexpr int FUSED_MAX_TILES = 4;     // key tiles a CTA keeps in TMEM (4 x 128 columns)
-constexpr int FUSED_MAX_CLUSTER = 8;   // portable cluster size
+constexpr int FUSED_STAGE_BYTES = FE_WARPS * 32 * 32 * 4;  // one 32 x 32 fp32 tile per warp
+
+// Bytes before the control block: the operand tiles (query tile and key ring)
+// while the MMAs run, then the epilogue warps' staging tiles.
+__host__ __device__ inline size_t fused_region_bytes(int nkb) {
+  const size_t ops = (size_t)nkb * TILE_BYTES * (1 + STAGES);
+  return ops > (size_t)FUSED_STAGE_BYTES ? ops : (size_t)FUSED_STAGE_BYTES;
+}
 
 struct MsgSplit {
   int kt_per;  // key tiles per split
@@ -366,13 +377,19 @@ __global__ void __launch_bounds__(FT_THREADS, 1)
   const int nkb = d / BK;
   uint8_t* Qs = base;
   uint8_t* Ks = base + (size_t)nkb * TILE_BYTES;
-  FusedCtl* ctl = reinterpret_cast<FusedCtl*>(base + (size_t)nkb * TILE_BYTES * (1 + STAGES));
+  FusedCtl* ctl = reinterpret_cast<FusedCtl*>(base + fused_region_bytes(nkb));
+  // g_h(i) of the CTA's query heads and visual keys, [head - j_lo][key - c0*BM]
+  float* gs = reinterpret_cast<float*>(ctl + 1);
+  const int gstr = kt_per * BM + 1;  // odd row stride: rows of different heads in distinct banks
 
   const int b = blockIdx.z / nsplit, split = (int)cluster.block_rank(), g = blockIdx.y,
             tile = blockIdx.x;
   const TextGeom tg = text_geom(toff, b, B, Tmax, status);
   const int grp = H / Hkv;
   if (tg.T == 0 || tile * BM >= grp * tg.T) return;  // uniform over the cluster (same b, tile)
+  // cluster barrier phase 1: this CTA has started (its shared memory may be
+  // written by the others once every CTA has arrived)
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
   const int Tb = tg.T;
   const int nkt = ceil_div(N + Tb, BM);
   const int c0 = split * kt_per, c1 = min(nkt, c0 + kt_per);
@@ -402,7 +419,7 @@ __global__ void __launch_bounds__(FT_THREADS, 1)
   tc::fence_after_sync();
   const uint32_t tmem = ctl->tmem;
   const long long deadline = clock64() + WAIT_CYCLES;
-  const float scale = rsqrtf((float)d);
+  const float c2 = rsqrtf((float)d) * 1.44269504f;  // 1/sqrt(d) in base-2 units (log2 e)
   const int quarter = warp & 3, cq = (warp >> 2) & 3;  // lane quarter, column quarter
   const int r = quarter * 32 + lane;  // tile row == TMEM lane (epilogue warps)
   const int R = tile * BM + r;
@@ -466,32 +483,55 @@ __global__ void __launch_bounds__(FT_THREADS, 1)
     __syncwarp();
   }
 
-  // ---- epilogue warps: this split's statistics -------------------------------
+  asm volatile("barrier.cluster.wait.aligned;" ::: "memory");  // every CTA has started
+
+  // ---- epilogue warps: g_h(i) for the CTA's heads and visual keys (while the
+  // MMAs run), then this split's statistics -----------------------------------
+  const int j_lo = tile * BM / Tb, j_hi = (min(grp * Tb, tile * BM + BM) - 1) / Tb;
+  const int key0 = c0 * BM, nvis = max(0, min(c1 * BM, N) - key0);
+  if (warp < FE_WARPS) {
+    for (int e = threadIdx.x; e < (j_hi - j_lo + 1) * nvis; e += FE_WARPS * 32) {
+      const int jj = e / nvis, kk = e % nvis, hh = g * grp + j_lo + jj;
+      const float sg = sigma[(size_t)b * H + hh];
+      gs[jj * gstr + kk] = sqrtf(zn2[((size_t)b * H + hh) * N + key0 + kk] + sg * sg);
+    }
+  }
   bool ok = true;
+  float mtile[FUSED_MAX_TILES];  // per 32-column block: the max its exponentials are taken at
   if (warp < FE_WARPS) {
     ok = tc::mbar_wait(&ctl->accdone, 0, deadline);
     ok = __all_sync(FULL, ok && !ctl->abort);
     tc::fence_after_sync();
     float m = -INFINITY, l = 0.f;
-    for (int it = 0; ok && it < iters; ++it) {
+#pragma unroll
+    for (int it = 0; it < FUSED_MAX_TILES; ++it) {
+      mtile[it] = -INFINITY;
+      if (!ok || it >= iters) continue;  // uniform over the warp
       float v[32];
-      tc::tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(it * BM + cq * 32), v);
+      const uint32_t ta = tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(it * BM + cq * 32);
+      tc::tmem_ld32(ta, v);
       const int k0 = (c0 + it) * BM + cq * 32;
-      float mt = -INFINITY;
+      float vmax = -INFINITY;
+#pragma unroll
+      for (int q = 0; q < 32; ++q)
+        if (k0 + q < kvis) vmax = fmaxf(vmax, v[q]);
+      // exp(x) = 2^(x log2 e): logits s = v / sqrt(d) in base-2 units are
+      // v * c2; 2^(v c2 - mt) replaces the logits in TMEM and the write pass
+      // rescales it (c2 > 0, so the block max of v c2 is vmax c2)
+      const float mt = vmax * c2;
+      float lt = 0.f;
 #pragma unroll
       for (int q = 0; q < 32; ++q) {
-        v[q] *= scale;
-        if (k0 + q < kvis) mt = fmaxf(mt, v[q]);
+        v[q] = (vmax > -INFINITY && k0 + q < kvis) ? exp2f(fmaf(v[q], c2, -mt)) : 0.f;
+        lt += v[q];
       }
-      if (mt > -INFINITY) {
+      tc::tmem_st32(ta, v);
+      if (vmax > -INFINITY) {
         const float mn = fmaxf(m, mt);
-        float acc = l * expf(m - mn);
-#pragma unroll
-        for (int q = 0; q < 32; ++q)
-          if (k0 + q < kvis) acc += expf(v[q] - mn);
-        l = acc;
+        l = l * exp2f(m - mn) + lt * exp2f(mt - mn);
         m = mn;
       }
+      mtile[it] = vmax > -INFINITY ? mt : -INFINITY;
     }
     ctl->stat_m[cq][r] = m;
     ctl->stat_l[cq][r] = l;
@@ -504,58 +544,67 @@ __global__ void __launch_bounds__(FT_THREADS, 1)
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
         const float mq = ctl->stat_m[q][r];
-        if (mq > -INFINITY) Lc += ctl->stat_l[q][r] * expf(mq - Mc);
+        if (mq > -INFINITY) Lc += ctl->stat_l[q][r] * exp2f(mq - Mc);
       }
-      ctl->cl_m[r] = Mc;
-      ctl->cl_l[r] = Lc;
+      for (int q = 0; q < nsplit; ++q) {  // into every CTA of the cluster, this split's slot
+        cluster.map_shared_rank(&ctl->all_m[split][0], q)[r] = Mc;
+        cluster.map_shared_rank(&ctl->all_l[split][0], q)[r] = Lc;
+      }
     }
   }
-  cluster.sync();  // every split's statistics are published
+  cluster.sync();  // every split's statistics are in every CTA (release / acquire)
 
   if (warp < FE_WARPS) {
     // merge the splits in a fixed order, then the normalised visual columns
     float M = -INFINITY, L = 0.f;
-    for (int q = 0; q < nsplit; ++q) M = fmaxf(M, cluster.map_shared_rank(ctl->cl_m, q)[r]);
+    for (int q = 0; q < nsplit; ++q) M = fmaxf(M, ctl->all_m[q][r]);
     for (int q = 0; q < nsplit; ++q) {
-      const float mq = cluster.map_shared_rank(ctl->cl_m, q)[r];
-      if (mq > -INFINITY) L += cluster.map_shared_rank(ctl->cl_l, q)[r] * expf(mq - M);
+      const float mq = ctl->all_m[q][r];
+      if (mq > -INFINITY) L += ctl->all_l[q][r] * exp2f(mq - M);
     }
     const float invL = 1.f / L;
-    const float sg = sigma[(size_t)b * H + h];
-    const float sg2 = sg * sg;
-    const float* zr = zn2 + ((size_t)b * H + h) * N;
-    float* arow = A + (((size_t)b * H + h) * Tmax + t) * N;
+    const float* grow = gs + (valid ? j - j_lo : 0) * gstr;
+    float* stg = reinterpret_cast<float*>(base) + warp * 32 * 32;  // the operands are consumed
     float rsum = 0.f;
-    for (int it = 0; ok && it < iters; ++it) {
+#pragma unroll
+    for (int it = 0; it < FUSED_MAX_TILES; ++it) {
+      if (!ok || it >= iters) continue;  // uniform over the warp
       const int k0 = (c0 + it) * BM + cq * 32;
       if (k0 >= N) continue;  // uniform over the warp
       float v[32];
-      // warp-collective: every lane loads, valid rows use it
       tc::tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(it * BM + cq * 32), v);
-      if (!valid) continue;
-      const int nv = min(32, N - k0);
-      if (nv == 32 && (N & 3) == 0) {
+      const float f = mtile[it] > -INFINITY ? exp2f(mtile[it] - M) * invL : 0.f;
+      const int nv = min(32, N - k0), kk0 = k0 - key0;
 #pragma unroll
-        for (int q = 0; q < 32; q += 4) {
-          const float4 z = *reinterpret_cast<const float4*>(zr + k0 + q);
-          float4 o;
-          o.x = expf(v[q] * scale - M) * invL;
-          o.y = expf(v[q + 1] * scale - M) * invL;
-          o.z = expf(v[q + 2] * scale - M) * invL;
-          o.w = expf(v[q + 3] * scale - M) * invL;
-          *reinterpret_cast<float4*>(arow + k0 + q) = o;
-          rsum = fmaf(o.x, sqrtf(z.x + sg2), rsum);
-          rsum = fmaf(o.y, sqrtf(z.y + sg2), rsum);
-          rsum = fmaf(o.z, sqrtf(z.z + sg2), rsum);
-          rsum = fmaf(o.w, sqrtf(z.w + sg2), rsum);
-        }
-      } else {
-        for (int q = 0; q < nv; ++q) {
-          const float p = expf(v[q] * scale - M) * invL;
-          arow[k0 + q] = p;
-          rsum = fmaf(p, sqrtf(zr[k0 + q] + sg2), rsum);
+      for (int q = 0; q < 32; ++q) {
+        v[q] *= f;
+        if (q < nv) rsum = fmaf(v[q], grow[kk0 + q], rsum);
+      }
+      // transpose through shared memory: row = lane going in, eight lanes per
+      // 128-byte row segment going out (16-byte chunks XOR-swizzled by row)
+#pragma unroll
+      for (int c4 = 0; c4 < 8; ++c4)
+        *reinterpret_cast<float4*>(stg + lane * 32 + ((c4 ^ (lane & 7)) << 2)) =
+            make_float4(v[4 * c4], v[4 * c4 + 1], v[4 * c4 + 2], v[4 * c4 + 3]);
+      __syncwarp();
+      const int c4 = lane & 7, col = k0 + 4 * c4;
+#pragma unroll
+      for (int rr = 0; rr < 32; rr += 4) {
+        const int row = rr + (lane >> 3);
+        const float4 o = *reinterpret_cast<const float4*>(stg + row * 32 + ((c4 ^ (row & 7)) << 2));
+        const int Rw = tile * BM + quarter * 32 + row;
+        if (Rw >= grp * Tb || col >= N) continue;
+        float* arow = A + (((size_t)b * H + g * grp + Rw / Tb) * Tmax + Rw % Tb) * N;
+        if ((N & 3) == 0 && col + 4 <= N) {
+          *reinterpret_cast<float4*>(arow + col) = o;
+        } else {
+          arow[col] = o.x;
+          if (col + 1 < N) arow[col + 1] = o.y;
+          if (col + 2 < N) arow[col + 2] = o.z;
+          if (col + 3 < N) arow[col + 3] = o.w;
         }
       }
+      __syncwarp();  // the next block reuses the staging tile
     }
     ctl->rsum[cq][r] = rsum;
     fused_epi_barrier();
@@ -564,8 +613,9 @@ __global__ void __launch_bounds__(FT_THREADS, 1)
           ((ctl->rsum[0][r] + ctl->rsum[1][r]) + ctl->rsum[2][r]) + ctl->rsum[3][r];
   }
   if (threadIdx.x == 0 && ctl->abort) set_status(status, GMC_STATUS_TIMEOUT);
+  // no CTA touches another's shared memory after the cluster barrier
   tc::fence_before_sync();
-  cluster.sync();  // the other CTAs have read this CTA's statistics
+  __syncthreads();
   if (warp == 0) tc::tmem_dealloc(tmem, tmem_cols);
 }
 
@@ -601,10 +651,11 @@ cudaError_t launch_message_tc(const Dims& dm, const void* keys, const void* quer
   if ((e = set_smem_limit((const void*)k_message_tc, smem)) != cudaSuccess) return e;
   const MsgSplit sp = msg_split(dm.B, dm.Hkv, RQ, dm.N, dm.T);
   dim3 grid(RQ / BM, dm.Hkv, dm.B * sp.n);
-  if (sp.kt_per <= FUSED_MAX_TILES && sp.n <= FUSED_MAX_CLUSTER) {
+  const size_t fsmem = 1024 + fused_region_bytes(nkb) + sizeof(FusedCtl) +
+                       sizeof(float) * (size_t)(dm.H / dm.Hkv) * (sp.kt_per * BM + 1);
+  if (sp.kt_per <= FUSED_MAX_TILES && sp.n <= FUSED_MAX_CLUSTER && fsmem <= 227 * 1024) {
     uint32_t cols = 32;
     while (cols < (uint32_t)(sp.kt_per * BM)) cols *= 2;
-    const size_t fsmem = 1024 + (size_t)nkb * TILE_BYTES * (1 + STAGES) + sizeof(FusedCtl);
     if ((e = set_smem_limit((const void*)k_message_fused, fsmem)) != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = grid;

@@ -74,32 +74,64 @@ __global__ void __launch_bounds__(256) k_probe(
   float* Vs = reinterpret_cast<float*>(Ws + grp * (d + 1));  // [PR_TOK][d + 1] (padded rows)
   float* zs = Vs + PR_TOK * (d + 1);                         // [PR_TOK][grp]
   const float4* W4 = reinterpret_cast<const float4*>(W) + (size_t)g * grp * d;
+  // W_h rows by cp.async, the values through registers four loads at a time:
+  // every copy of the block is in flight before the first one lands
   for (int idx = threadIdx.x; idx < grp * d; idx += blockDim.x)
-    Ws[(idx / d) * (d + 1) + idx % d] = W4[idx];
+    cp_async16(&Ws[(idx / d) * (d + 1) + idx % d], &W4[idx]);
+  cp_async_commit();
   constexpr int VE = 16 / sizeof(Tin);  // elements per 16-byte load
-  for (int idx = threadIdx.x; idx < PR_TOK * d / VE; idx += blockDim.x) {
-    const int ii = idx / (d / VE), k = (idx % (d / VE)) * VE, i = i0 + ii;
-    uint4 raw = make_uint4(0, 0, 0, 0);
-    if (i < N) raw = *reinterpret_cast<const uint4*>(keys + sq.value_row(i, HD) + (size_t)g * d + k);
-    const Tin* e = reinterpret_cast<const Tin*>(&raw);
+  const int nld = PR_TOK * d / VE;
+  for (int idx0 = 0; idx0 < nld; idx0 += 4 * (int)blockDim.x) {  // uniform over the block
+    uint4 raw[4];
 #pragma unroll
-    for (int q = 0; q < VE; ++q) Vs[ii * (d + 1) + k + q] = to_f32(e[q]);
+    for (int u = 0; u < 4; ++u) {
+      const int idx = idx0 + u * (int)blockDim.x + (int)threadIdx.x;
+      const int ii = idx / (d / VE), k = (idx % (d / VE)) * VE, i = i0 + ii;
+      raw[u] = make_uint4(0, 0, 0, 0);
+      if (idx < nld && i < N)
+        raw[u] = *reinterpret_cast<const uint4*>(keys + sq.value_row(i, HD) + (size_t)g * d + k);
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int idx = idx0 + u * (int)blockDim.x + (int)threadIdx.x;
+      if (idx >= nld) continue;
+      const int ii = idx / (d / VE), k = (idx % (d / VE)) * VE;
+      const Tin* e = reinterpret_cast<const Tin*>(&raw[u]);
+#pragma unroll
+      for (int q = 0; q < VE; ++q) Vs[ii * (d + 1) + k + q] = to_f32(e[q]);
+    }
   }
+  cp_async_wait<0>();
   __syncthreads();
   for (int task = threadIdx.x; task < PR_TOK * grp; task += blockDim.x) {
     const int ii = task / grp, jh = task % grp, i = i0 + ii;
     const float* v = Vs + ii * (d + 1);
     const float4* w = Ws + jh * (d + 1);
-    float z0 = 0.f, z1 = 0.f, z2 = 0.f, z3 = 0.f;
-#pragma unroll 4
-    for (int k = 0; k < d; ++k) {
-      const float x = v[k];
-      const float4 c = w[k];
-      z0 = fmaf(x, c.x, z0);
-      z1 = fmaf(x, c.y, z1);
-      z2 = fmaf(x, c.z, z2);
-      z3 = fmaf(x, c.w, z3);
+    // four coordinates loaded ahead of their FMAs; even and odd k accumulate
+    // apart and are added once at the end (d is a multiple of 4)
+    float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f, b0 = 0.f, b1 = 0.f, b2 = 0.f, b3 = 0.f;
+#pragma unroll 2
+    for (int k = 0; k < d; k += 4) {
+      float x[4];
+      float4 c[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        x[u] = v[k + u];
+        c[u] = w[k + u];
+      }
+#pragma unroll
+      for (int u = 0; u < 4; u += 2) {
+        a0 = fmaf(x[u], c[u].x, a0);
+        a1 = fmaf(x[u], c[u].y, a1);
+        a2 = fmaf(x[u], c[u].z, a2);
+        a3 = fmaf(x[u], c[u].w, a3);
+        b0 = fmaf(x[u + 1], c[u + 1].x, b0);
+        b1 = fmaf(x[u + 1], c[u + 1].y, b1);
+        b2 = fmaf(x[u + 1], c[u + 1].z, b2);
+        b3 = fmaf(x[u + 1], c[u + 1].w, b3);
+      }
     }
+    const float z0 = a0 + b0, z1 = a1 + b1, z2 = a2 + b2, z3 = a3 + b3;
     const float n2 = z0 * z0 + z1 * z1 + z2 * z2 + z3 * z3;
     if (i < N) {
       const size_t o = ((size_t)b * H + g * grp + jh) * N + i;
@@ -109,10 +141,17 @@ __global__ void __launch_bounds__(256) k_probe(
     zs[ii * grp + jh] = i < N ? n2 : 0.f;
   }
   __syncthreads();
-  for (int jh = threadIdx.x; jh < grp; jh += blockDim.x) {
+  // per head of the group: eight threads sum every eighth token, a fixed
+  // shuffle tree adds the eight
+  for (int jh0 = 0; jh0 < grp; jh0 += (int)blockDim.x / 8) {  // uniform over the block
+    const int jh = jh0 + (int)threadIdx.x / 8, pt = threadIdx.x & 7;
     float sacc = 0.f;
-    for (int ii = 0; ii < PR_TOK; ++ii) sacc += zs[ii * grp + jh];  // fixed order
-    sigpart[((size_t)b * nP + pb) * H + g * grp + jh] = sacc;
+    if (jh < grp)
+      for (int ii = pt; ii < PR_TOK; ii += 8) sacc += zs[ii * grp + jh];
+    sacc += __shfl_xor_sync(FULL, sacc, 4);
+    sacc += __shfl_xor_sync(FULL, sacc, 2);
+    sacc += __shfl_xor_sync(FULL, sacc, 1);
+    if (jh < grp && pt == 0) sigpart[((size_t)b * nP + pb) * H + g * grp + jh] = sacc;
   }
   __threadfence();
   __syncthreads();
@@ -120,16 +159,24 @@ __global__ void __launch_bounds__(256) k_probe(
   __syncthreads();
   if (!last) return;
   __threadfence();
-  // the image's partials: loaded by the whole block, summed per head in a fixed order
-  float* ps = Vs;  // reuse: nP * H floats (the host sizes this region for both uses)
-  for (int q = threadIdx.x; q < nP * H; q += blockDim.x)
-    ps[q] = __ldcg(&sigpart[(size_t)b * nP * H + q]);
-  __syncthreads();
-  for (int h = threadIdx.x; h < H; h += blockDim.x) {
-    double sacc = 0.0;
-    for (int q = 0; q < nP; ++q) sacc += (double)ps[q * H + h];
-    const float fro = (float)sqrt(sacc);
-    sigma[(size_t)b * H + h] = sqrtf(lambda_mass) * fmaxf(fro / sqrtf((float)N * 4.f), eps_mass);
+  // the image's partials: eight threads per head sum every eighth partial
+  // (read past L1: other blocks wrote them), a fixed shuffle tree adds the
+  // eight (fp32: the partials are fp32 sums already)
+  const float* sp = sigpart + (size_t)b * nP * H;
+  const int part = threadIdx.x & 7;
+  for (int h0 = 0; h0 < H; h0 += (int)blockDim.x / 8) {  // uniform over the block
+    const int h = h0 + (int)threadIdx.x / 8;
+    float sacc = 0.f;
+    if (h < H) {
+#pragma unroll 4
+      for (int q = part; q < nP; q += 8) sacc += __ldcg(&sp[(size_t)q * H + h]);
+    }
+    sacc += __shfl_xor_sync(FULL, sacc, 4);
+    sacc += __shfl_xor_sync(FULL, sacc, 2);
+    sacc += __shfl_xor_sync(FULL, sacc, 1);
+    if (h < H && part == 0)
+      sigma[(size_t)b * H + h] =
+          sqrtf(lambda_mass) * fmaxf(sqrtf(sacc) / sqrtf((float)N * 4.f), eps_mass);
   }
 }
 
@@ -193,8 +240,7 @@ cudaError_t launch_probe(const Dims& dm, const void* keys, const float* W, const
   const int grp = dm.H / dm.Hkv;
   dim3 grid(s.nP, dm.Hkv, dm.B);
   const size_t smem = sizeof(float4) * grp * (dm.d + 1) +
-                      sizeof(float) * (std::max((size_t)PR_TOK * (dm.d + 1), (size_t)s.nP * dm.H) +
-                                       (size_t)PR_TOK * grp);
+                      sizeof(float) * ((size_t)PR_TOK * (dm.d + 1) + (size_t)PR_TOK * grp);
   cudaError_t e;
   if (dm.dtype == GMC_BF16) {
     if ((e = set_smem_limit((const void*)k_probe<__nv_bfloat16>, smem)) != cudaSuccess) return e;
