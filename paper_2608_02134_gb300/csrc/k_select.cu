@@ -258,16 +258,29 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
     for (int m = m0; m < m1; ++m) wsum += cgl[m] + 16;
     int W = 0;
     int run = block_exclusive_scan(wsum, s.wsum, &W);
-    for (int m = m0; m < m1; ++m) {
-      const int wm = cgl[m] + 16;
-      // CTA c starts after the row where the preceding weight reaches c*W/CS
-      for (int c = 1; c < CS; ++c) {
-        const long long tgt = (long long)c * W / CS;
-        if (run < tgt && run + wm >= tgt) atomicMin(&s.rowb[c], m + 1);
+    // CTA c starts after the row where the preceding weight reaches c*W/CS;
+    // the CS - 1 targets are computed once (the histogram is zero again
+    // before its first use)
+    long long* tgt = reinterpret_cast<long long*>(s.hist);
+    if (threadIdx.x >= 1 && (int)threadIdx.x < CS) tgt[threadIdx.x] = (long long)threadIdx.x * W / CS;
+    __syncthreads();
+    // a target inside this thread's weight range (run, run + wsum] lies in one
+    // of its rows: only then are the rows walked
+    for (int c = 1; c < CS; ++c) {
+      const long long t = tgt[c];
+      if (!(run < t && run + wsum >= t)) continue;
+      long long at = run;
+      for (int m = m0; m < m1; ++m) {
+        const int wm = cgl[m] + 16;
+        if (at < t && at + wm >= t) {
+          atomicMin(&s.rowb[c], m + 1);
+          break;
+        }
+        at += wm;
       }
-      run += wm;
     }
     __syncthreads();
+    if (threadIdx.x < 2 * SEL_MAX_CS) s.hist[threadIdx.x] = 0;
     if (threadIdx.x == 0) {
       s.rowb[0] = 0;
       int prev = 0, ok = 1;
@@ -308,17 +321,47 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
   // the schedule; nothing computed from it does (integer and max reductions).
   auto migrate = [&]() {
     if (!s.scal[SC_GLOBAL] || nrows >= DEADROW) return;  // row ids are stored in 16 bits
+    // entry offsets of the rows (contiguous rows per thread), then every entry
+    // of the CTA handled by one thread: all its global loads are in flight at once
+    const int rper = (nrows + blockDim.x - 1) / blockDim.x;
+    const int q0 = min(nrows, (int)threadIdx.x * rper), q1 = min(nrows, q0 + rper);
     int mine = 0;
-    for (int q = threadIdx.x; q < nrows; q += blockDim.x) mine += s.cnt[q];
+    for (int q = q0; q < q1; ++q) mine += s.cnt[q];
     int tot = 0;
-    block_exclusive_scan(mine, s.wsum, &tot);
+    int at = block_exclusive_scan(mine, s.wsum, &tot);
     if (tot > a.cap) return;  // uniform over the block
+    int* rp = reinterpret_cast<int*>(s.bfix);  // [nrows + 1]; bfix is set at the end
+    for (int q = q0; q < q1; ++q) {
+      rp[q] = at;
+      at += s.cnt[q];
+    }
+    if (threadIdx.x == 0) rp[nrows] = tot;
     for (int j = threadIdx.x; j < N; j += blockDim.x) s.bnd[j] = 0;
     __syncthreads();
-    for (int q = wid; q < nrows; q += nw) {
-      const uint16_t* gc = Simg + (size_t)(mlo + q) * N;
-      const int n = s.cnt[q];
-      for (int k = lane; k < n; k += 32) atomicAdd(&s.bnd[gc[k]], 1);
+    // row of entry e: the last q with rp[q] <= e
+    auto row_of = [&](int e) {
+      int lo = 0, hi = nrows;  // rp[lo] <= e < rp[hi]
+      while (hi - lo > 1) {
+        const int mid = (lo + hi) >> 1;
+        if (rp[mid] <= e) lo = mid; else hi = mid;
+      }
+      return lo;
+    };
+    constexpr int MU = 4;  // entries per thread in flight
+    for (int e0 = threadIdx.x; e0 < tot; e0 += MU * blockDim.x) {
+      int jj[MU];
+#pragma unroll
+      for (int u = 0; u < MU; ++u) {
+        const int e = e0 + u * (int)blockDim.x;
+        jj[u] = -1;
+        if (e < tot) {
+          const int q = row_of(e);
+          jj[u] = Simg[(size_t)(mlo + q) * N + (e - rp[q])];
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < MU; ++u)
+        if (jj[u] >= 0) atomicAdd(&s.bnd[jj[u]], 1);
     }
     __syncthreads();
     {
@@ -326,28 +369,43 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
       const int j0 = min(N, (int)threadIdx.x * per), j1 = min(N, j0 + per);
       int c = 0;
       for (int j = j0; j < j1; ++j) c += s.bnd[j];
-      int at = block_exclusive_scan(c, s.wsum, nullptr);
+      int at2 = block_exclusive_scan(c, s.wsum, nullptr);
       for (int j = j0; j < j1; ++j) {
         const int n = s.bnd[j];
-        s.cstart[j] = at;
-        s.bnd[j] = at;  // fill cursor of token j
-        at += n;
+        s.cstart[j] = at2;
+        s.bnd[j] = at2;  // fill cursor of token j
+        at2 += n;
       }
       if (threadIdx.x == 0) s.cstart[N] = tot;
     }
     __syncthreads();
-    for (int q = wid; q < nrows; q += nw) {
-      const float* gv = Cimg + (size_t)(mlo + q) * N;
-      const uint16_t* gc = Simg + (size_t)(mlo + q) * N;
-      const int n = s.cnt[q];
-      for (int k = lane; k < n; k += 32) {
-        const int j = gc[k];
-        const int pos = atomicAdd(&s.bnd[j], 1);
-        s.svals[pos] = gv[k];
-        s.scols[pos] = (uint16_t)j;
-        s.srows[pos] = (uint16_t)q;
+    for (int e0 = threadIdx.x; e0 < tot; e0 += MU * blockDim.x) {
+      int jj[MU], qq[MU];
+      float vv[MU];
+#pragma unroll
+      for (int u = 0; u < MU; ++u) {
+        const int e = e0 + u * (int)blockDim.x;
+        jj[u] = -1;
+        qq[u] = 0;
+        vv[u] = 0.f;
+        if (e < tot) {
+          const int q = row_of(e);
+          const size_t g = (size_t)(mlo + q) * N + (e - rp[q]);
+          qq[u] = q;
+          jj[u] = Simg[g];
+          vv[u] = Cimg[g];
+        }
       }
+#pragma unroll
+      for (int u = 0; u < MU; ++u)
+        if (jj[u] >= 0) {
+          const int pos = atomicAdd(&s.bnd[jj[u]], 1);
+          s.svals[pos] = vv[u];
+          s.scols[pos] = (uint16_t)jj[u];
+          s.srows[pos] = (uint16_t)qq[u];
+        }
     }
+    __syncthreads();  // rp (over bfix) is no longer read
     for (int q = threadIdx.x; q < nrows; q += blockDim.x) s.bfix[q] = to_fix(s.bcov[q], fxs);
     __syncthreads();
     if (threadIdx.x == 0) {
@@ -783,21 +841,23 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
   }
   cluster.sync();
   if (r != 0) return;
-  if (wid == 0) {
+  {  // the support in ascending token order: contiguous tokens per thread, one block scan
+    const int per = (N + blockDim.x - 1) / blockDim.x;
+    const int j0 = min(N, (int)threadIdx.x * per), j1 = min(N, j0 + per);
+    int c = 0;
+    for (int j = j0; j < j1; ++j) c += s.sel[j] ? 1 : 0;
     int cnt = 0;
-    for (int base = 0; base < N; base += 32) {
-      const int j = base + lane;
-      const bool on = j < N && s.sel[j];
-      const unsigned m = __ballot_sync(FULL, on);
-      const int pos = cnt + __popc(m & lanemask_lt());
-      if (j < N) a.slot[(size_t)b * N + j] = on ? pos : -1;
+    int pos = block_exclusive_scan(c, s.wsum, &cnt);
+    for (int j = j0; j < j1; ++j) {
+      const bool on = s.sel[j] != 0;
+      a.slot[(size_t)b * N + j] = on ? pos : -1;
       if (on && pos < K) {
         a.support[(size_t)b * K + pos] = j;
         if (a.out_idx) a.out_idx[(size_t)b * K + pos] = j;
       }
-      cnt += __popc(m);
+      pos += on ? 1 : 0;
     }
-    if (lane == 0 && cnt != K) set_status(a.status, GMC_STATUS_INTERNAL);
+    if (threadIdx.x == 0 && cnt != K) set_status(a.status, GMC_STATUS_INTERNAL);
   }
   if (a.tv.base) {
     if (threadIdx.x == 0) {
