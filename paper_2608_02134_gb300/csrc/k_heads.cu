@@ -37,9 +37,11 @@ __global__ void k_head_stats(const float* __restrict__ A, const float* __restric
                              uint32_t* status) {
   grid_dep_wait();
   extern __shared__ float sm_hs[];
+  __shared__ float sgm[GMC_MAX_HEADS];  // sigma_h of the image
   const int b = blockIdx.y;
   const TextGeom tg = text_geom(toff, b, B, Tmax, status);
   if (tg.T == 0) return;
+  for (int h = threadIdx.x; h < H; h += blockDim.x) sgm[h] = sigma[(size_t)b * H + h];
   const int Tb = tg.T;
   const int npairs = H * (H + 1) / 2;
   const int nhb = (H + HG_HB - 1) / HG_HB, Hp = nhb * HG_HB;
@@ -159,7 +161,7 @@ __global__ void k_head_stats(const float* __restrict__ A, const float* __restric
     const int h = p / H, g = p % H;
     if (h > g) continue;
     const int pi = pair_index(h, g, H);
-    const float sh = sigma[(size_t)b * H + h], sgv = sigma[(size_t)b * H + g];
+    const float sh = sgm[h], sgv = sgm[g];
     float v = 0.f;
     for (int ii = 0; ii < HG_TOK; ++ii) {
       const int i = i0 + ii;
@@ -211,10 +213,10 @@ __device__ void cluster_heads(const double* hgb, int b, int T, int N, int H, int
   int* cent = asg + H;                  // [GMC_MAX_HEADS] centres
   int* ccnt = cent + GMC_MAX_HEADS;     // [GMC_MAX_HEADS] cluster sizes
   for (int h = threadIdx.x; h < H; h += blockDim.x) {
-    const double a = __ldcg(&hgb[h * H + h]);
-    const double mean = __ldcg(&hgb[H * H + h]) / ((double)T * N);  // sum_t rs[h,t] / (T N)
-    pre[h] = (mean > 0.0 && a > 0.0) ? (float)(sqrt(a) / mean) : 0.f;
-    dot[h] = a > 0.0 ? (float)(1.0 / sqrt(a)) : 0.f;  // 1 / ||U_h||, 0 for a zero pattern
+    const float a = (float)__ldcg(&hgb[h * H + h]);
+    const float mean = (float)__ldcg(&hgb[H * H + h]) / ((float)T * (float)N);  // sum_t rs / (T N)
+    pre[h] = (mean > 0.f && a > 0.f) ? sqrtf(a) / mean : 0.f;
+    dot[h] = a > 0.f ? 1.f / sqrtf(a) : 0.f;  // 1 / ||U_h||, 0 for a zero pattern
   }
   __syncthreads();
   for (int p = threadIdx.x; p < H * H; p += blockDim.x) {
@@ -226,6 +228,8 @@ __device__ void cluster_heads(const double* hgb, int b, int T, int N, int H, int
   if (wid == 0) {  // farthest-first centres, two heads per lane (H <= 64)
     const int h0 = lane, h1 = lane + 32;
     bool c0 = false, c1 = false;  // is h0 / h1 a centre
+    float mc0 = -INFINITY, mc1 = -INFINITY;  // largest cosine of h0 / h1 to a centre
+    int newest;                              // the latest centre (the same in every lane)
     {
       float v = -1.f;
       int idx = -1;
@@ -235,23 +239,24 @@ __device__ void cluster_heads(const double* hgb, int b, int T, int N, int H, int
       if (lane == 0) cent[0] = idx;
       c0 = (h0 == idx);
       c1 = (h1 == idx);
+      newest = idx;
     }
-    __syncwarp();
     for (int c = 1; c < nc; ++c) {
+      if (h0 < H) mc0 = fmaxf(mc0, cs[h0 * H + newest]);
+      if (h1 < H) mc1 = fmaxf(mc1, cs[h1 * H + newest]);
       float v = 0.f;
       int idx = -1;
       for (int q = 0; q < 2; ++q) {
         const int h = q ? h1 : h0;
         if (h >= H || (q ? c1 : c0)) continue;
-        float mc = -INFINITY;
-        for (int k = 0; k < c; ++k) mc = fmaxf(mc, cs[h * H + cent[k]]);
+        const float mc = q ? mc1 : mc0;
         if (idx < 0 || mc < v) { v = mc; idx = h; }
       }
       warp_argbest(v, idx, false);
       if (lane == 0) cent[c] = idx;
       c0 |= (h0 == idx);
       c1 |= (h1 == idx);
-      __syncwarp();
+      newest = idx;
     }
   }
   __syncthreads();

@@ -346,22 +346,31 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_rg_rho(
     const unsigned lt = sel::lanemask_lt();
     int nf = 0;
     float rmax = 0.f;
-    for (int e0 = 0; e0 < n; e0 += 32) {
-      const int e = e0 + lane;
-      int ps = -1;
-      float R = 0.f;
-      if (e < n) {
-        ps = pslot[cols[e]];
-        if (ps >= 0) R = vals[e] - bm;  // > 0: a survivor exceeds its coverage
+    constexpr int RU = 4;  // chunks of 32 entries whose loads are in flight together
+    for (int e00 = 0; e00 < n; e00 += 32 * RU) {
+      int ps[RU];
+      float R[RU];
+#pragma unroll
+      for (int u = 0; u < RU; ++u) {
+        const int e = e00 + 32 * u + lane;
+        ps[u] = e < n ? (int)cols[e] : -1;
       }
-      const unsigned bal = __ballot_sync(FULL, ps >= 0);
-      if (ps >= 0) {
-        const int at = nf + __popc(bal & lt);
-        fslot[w][at] = ps;
-        fres[w][at] = R;
-        rmax = fmaxf(rmax, R);
+#pragma unroll
+      for (int u = 0; u < RU; ++u) {
+        if (ps[u] >= 0) ps[u] = pslot[ps[u]];
+        R[u] = ps[u] >= 0 ? vals[e00 + 32 * u + lane] - bm : 0.f;  // > 0: exceeds its coverage
       }
-      nf += __popc(bal);
+#pragma unroll
+      for (int u = 0; u < RU; ++u) {
+        const unsigned bal = __ballot_sync(FULL, ps[u] >= 0);
+        if (ps[u] >= 0) {
+          const int at = nf + __popc(bal & lt);
+          fslot[w][at] = ps[u];
+          fres[w][at] = R[u];
+          rmax = fmaxf(rmax, R[u]);
+        }
+        nf += __popc(bal);
+      }
     }
     rmax = warp_max(rmax);
     __syncwarp();
@@ -439,31 +448,52 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_rg_filter(
     const int n = cnt[row];
     float* vals = C + row * N;
     uint16_t* cols = scol + row * N;
+    // The list is walked FU chunks of 32 entries at a time, every load of the
+    // chunks issued before the first use (and, below, before any survivor is
+    // written back in place: a chunk's survivors land below its end).
+    constexpr int FU = 4;
     float bnew = bcov[row];
-    for (int e = lane; e < n; e += 32)
-      if (inb[cols[e]]) bnew = fmaxf(bnew, vals[e]);
+    for (int e00 = 0; e00 < n; e00 += 32 * FU) {
+      int jj[FU];
+#pragma unroll
+      for (int u = 0; u < FU; ++u) {
+        const int e = e00 + 32 * u + lane;
+        jj[u] = e < n ? (int)cols[e] : -1;
+      }
+#pragma unroll
+      for (int u = 0; u < FU; ++u)
+        if (jj[u] >= 0 && inb[jj[u]]) bnew = fmaxf(bnew, vals[e00 + 32 * u + lane]);
+    }
     bnew = warp_max(bnew);
     const long long fb_new = to_fix(bnew, fxs);
     const unsigned lt = sel::lanemask_lt();
     int wr = 0;
-    for (int e0 = 0; e0 < n; e0 += 32) {
-      const int e = e0 + lane;
-      float c = 0.f;
-      int j = 0;
-      if (e < n) {
-        c = vals[e];
-        j = cols[e];
+    for (int e00 = 0; e00 < n; e00 += 32 * FU) {
+      float cc[FU];
+      int jj[FU];
+#pragma unroll
+      for (int u = 0; u < FU; ++u) {
+        const int e = e00 + 32 * u + lane;
+        cc[u] = 0.f;
+        jj[u] = 0;
+        if (e < n) {
+          cc[u] = vals[e];
+          jj[u] = cols[e];
+        }
       }
-      const bool keep = e < n && c > bnew;
-      const unsigned bal = __ballot_sync(FULL, keep);
-      __syncwarp();  // the chunk is read before any survivor moves down into it
-      if (keep) {
-        const int pos = wr + __popc(bal & lt);
-        vals[pos] = c;
-        cols[pos] = (uint16_t)j;
-        atomicAdd(&uacc[j], (unsigned long long)(to_fix(c, fxs) - fb_new));
+      __syncwarp();  // the chunks are read before any survivor moves down into them
+#pragma unroll
+      for (int u = 0; u < FU; ++u) {
+        const bool keep = e00 + 32 * u + lane < n && cc[u] > bnew;
+        const unsigned bal = __ballot_sync(FULL, keep);
+        if (keep) {
+          const int pos = wr + __popc(bal & lt);
+          vals[pos] = cc[u];
+          cols[pos] = (uint16_t)jj[u];
+          atomicAdd(&uacc[jj[u]], (unsigned long long)(to_fix(cc[u], fxs) - fb_new));
+        }
+        wr += __popc(bal);
       }
-      wr += __popc(bal);
     }
     if (lane == 0) {
       bcov[row] = bnew;
