@@ -46,6 +46,40 @@ Readings taken where the paper is silent or ambiguous:
   * Transport blend tau_j = 1 (appendix form); rms(u) = sqrt(mean u^2),
     epsilon 1e-6.
 
+Pins (tests/test_oracle_pins.py; the paper prints no worked numeric example,
+so every function is pinned by a closed form, an invariant, a bound of the
+paper, a hand-worked case or brute force on tiny inputs, never by itself):
+  * budget: the totality rule on every (K_r, N) corner.
+  * message_slice: explicit per-element loops; causal keys and the native
+    (not renormalised) visual mass; one query is a plain softmax.
+  * orthonormal_probe / probe_values: orthonormal columns; rotation
+    invariance of ||Z||; the sigma floor closed form (V = 0 => P^G prop. to A).
+  * atom_norms / grounded_clients: a hand example; a zero-energy row is
+    inactive.
+  * query_weights: the terminal query counts double, weights sum to one.
+  * head_patterns / head_clusters: identical heads form one cluster with
+    uniform weights; orthogonal families get equal cluster mass; a
+    hand-worked farthest-first case; weights follow 1 / (dispersion + eps).
+  * message_energy: closed form and the uniform fallback.
+  * cosine_matrix / appearance_clients: the Gibbs modal ratio.
+  * grid_coords / landmark_coords / spatial_clients: normalised cell centres,
+    landmark-grid ratios.
+  * client_matrix / bank_saturation: bank masses and effective shares, row
+    masses from head and query weights.
+  * facility_value: Eq. (7) coverage-to-quantization bound; monotone and
+    submodular by brute force.
+  * select_support / stable_top / batched_certificate: Eq. (6) certificate and
+    the greedy (1 - 1/e) bound against brute-force optima; exact cardinality;
+    the zero-gain fill; a hand-worked responsibility round
+    (tests/golden/responsibility_round.txt); trivial supports.
+  * assign_population: cosine nearest neighbour when s_x = 0; the gap-gate
+    closed form and Eq. (cond-assignment-bound); one representative.
+  * population_weights / transport / rms: positivity, mass and first-moment
+    conservation (Eq. (cond-population-moment)), centroid optimality
+    (Eq. (cond-centroid-optimum)), RMS restoration and its bound.
+  * compaction_rows / compress: K = N identity; end-to-end invariants on the
+    tiny configuration.
+
 Discrete choices (pool, batch, head centres, assignment) are recorded together
 with the fp64 values that decide them.  Every choice can also be *forced*
 (``forced=`` arguments): the oracle then continues from the given choice

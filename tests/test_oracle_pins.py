@@ -555,3 +555,91 @@ def test_identity_when_K_equals_N():
     np.testing.assert_array_equal(res.out_pos, im.pos)
     wl2, im2, res2 = _tiny_result(K=1000)
     assert res2.identity and res2.K == 64
+
+
+# --------------------------------------------------------------------------
+# direct pins of the helper steps (each also runs inside the steps above)
+# --------------------------------------------------------------------------
+def test_head_patterns_hand_example_and_scale_invariance():
+    # Eq. (cond-head-pattern): atoms u_i^{h,t} = A[h,t,i] [Z_h[i]; sigma_h],
+    # divided by their mean norm over all (t, i).
+    # head 0: one atom [3, 4] (norm 5) and a zero atom -> mean norm 2.5,
+    #         U_0 = [1.2, 1.6, 0, 0], ||U_0|| = 2;
+    # head 1: atoms [0, 0.5] twice -> mean norm 0.5, U_1 = [0, 1, 0, 1], ||U_1|| = sqrt 2;
+    # head 2: no attention -> the zero pattern.
+    A = np.array([[[1.0, 0.0]], [[0.5, 0.5]], [[0.0, 0.0]]])
+    Z = np.array([[[3.0], [0.0]], [[0.0], [0.0]], [[1.0], [1.0]]])
+    sigma = np.array([4.0, 1.0, 1.0])
+    cos, pre, _ = O.head_patterns(A, Z, sigma)
+    np.testing.assert_allclose(pre, [2.0, math.sqrt(2.0), 0.0], atol=1e-15)
+    np.testing.assert_allclose(cos[0, 1], 1.6 / (2.0 * math.sqrt(2.0)), rtol=1e-14)
+    np.testing.assert_allclose(np.diag(cos)[:2], [1.0, 1.0], rtol=1e-14)
+    assert cos[2, 2] == 0.0 and cos[0, 2] == 0.0
+    # the mean-norm normalisation makes a pattern blind to the scale of A_h
+    A2 = A.copy()
+    A2[0] *= 7.0
+    cos2, pre2, _ = O.head_patterns(A2, Z, sigma)
+    np.testing.assert_allclose(cos2, cos, rtol=1e-13, atol=1e-15)
+    np.testing.assert_allclose(pre2, pre, rtol=1e-13, atol=1e-15)
+
+
+def test_client_matrix_row_masses_and_layout():
+    # Eq. (cond-coverage): every active row of a bank carries its bank's mass;
+    # the client matrix stacks grounded rows (h, t) h-major, appearance rows,
+    # then the landmark rows.
+    H, T, N, L = 2, 3, 5, 4
+    g = rng(3)
+    PG = g.random((H, T, N))
+    PG /= PG.sum(axis=2, keepdims=True)
+    active = np.ones((H, T), dtype=bool)
+    active[1, 2] = False
+    PG[1, 2] = 0.0
+    omega = np.array([0.25, 0.75])
+    nu = O.query_weights(T, P)
+    PV = g.random((N, N))
+    PV /= PV.sum(axis=1, keepdims=True)
+    PS = g.random((L, N))
+    PS /= PS.sum(axis=1, keepdims=True)
+    cm = O.client_matrix(PG, active, omega, nu, PV, PS, P)
+    assert cm.C.shape == (H * T + N + L, N)
+    rows = cm.C.sum(axis=1)
+    for h in range(H):
+        for t in range(T):
+            want = P["beta_G"] * omega[h] * nu[t] if active[h, t] else 0.0
+            assert rows[h * T + t] == pytest.approx(want, rel=1e-13, abs=1e-15)
+    np.testing.assert_allclose(rows[H * T:H * T + N], P["beta_V"] / N, rtol=1e-13)
+    np.testing.assert_allclose(rows[H * T + N:], P["beta_S"] / L, rtol=1e-13)
+    # grounded row (1, 0) is P^G_{1,0} scaled, column for column
+    np.testing.assert_allclose(cm.C[1 * T + 0] / rows[1 * T + 0], PG[1, 0], rtol=1e-13)
+
+
+def test_stable_top_matches_brute_force_with_ties():
+    g = rng(4)
+    for _ in range(50):
+        n = int(g.integers(1, 12))
+        vals = g.integers(0, 4, n).astype(float)   # many ties
+        ids = g.permutation(100)[:n]
+        k = int(g.integers(0, n + 1))
+        pairs = sorted(zip(vals, ids), key=lambda x: (-x[0], x[1]))
+        want = [int(i) for _, i in pairs[:k]]
+        assert [int(i) for i in O.stable_top(vals, ids, k)] == want
+
+
+def test_rms_and_unit_states_closed_forms():
+    assert O.rms(np.array([3.0, 4.0])) == pytest.approx(math.sqrt(12.5), rel=1e-15)
+    assert O.rms(np.full(7, -2.5)) == pytest.approx(2.5, rel=1e-15)
+    h = np.array([[3.0, 4.0, 0.0], [0.0, 0.0, 0.0], [1e-3, 0.0, 0.0]])
+    x = O.unit_states(h, P)
+    np.testing.assert_allclose(x[0], [0.6, 0.8, 0.0], rtol=1e-15)
+    np.testing.assert_array_equal(x[1], 0.0)                     # eps keeps a zero row zero
+    np.testing.assert_allclose(x[2], [1.0, 0.0, 0.0], rtol=1e-15)
+    # cosines of scaled states are those of the states
+    np.testing.assert_allclose(O.cosine_matrix(5.0 * h, P), O.cosine_matrix(h, P), rtol=1e-14)
+
+
+def test_compaction_rows_index_map():
+    # Appendix "Index map and physical token accounting": kept visual rows in
+    # ascending source order, then every text row, K + T rows in all.
+    rows = O.compaction_rows(np.array([1, 4, 6]), N=8, T=3)
+    np.testing.assert_array_equal(rows, [1, 4, 6, 8, 9, 10])
+    assert O.compaction_rows(np.array([], dtype=np.int64), N=4, T=0).size == 0
