@@ -157,6 +157,8 @@ size_t gmc_workspace_size(const gmc_problem* prob, int N, int T, int H, int d, i
  *
  * Limits: 1 <= N <= GMC_MAX_N, N == grid_h*grid_w, T >= 1, 1 <= H <= GMC_MAX_HEADS,
  * H % Hkv == 0, d <= 1024 and D <= 8192, d a multiple of 8 (bf16) or 4 (fp32),
+ * and H <= 56 in this build (the head-pattern statistics of one token block
+ * must fit a block's 227 KB of shared memory; GMC_ERR_UNSUPPORTED above),
  * D a multiple of 8.  hidden/keys/queries/vo_probe/out_hidden/out_kv must be
  * 16-byte aligned, trace 16-byte aligned.
  */

@@ -321,7 +321,7 @@ const char* gmc_version(void) { return "gmc 0.1.0 sm_103a"; }
 
 size_t gmc_workspace_size(const gmc_problem* prob, int N, int T, int H, int d, int D, int K) {
   if (check_problem(prob, N, T, d, D) != GMC_OK || H < 1 || H > GMC_MAX_HEADS ||
-      H % prob->Hkv != 0)
+      H % prob->Hkv != 0 || !heads_supported(H))
     return 0;
   gmc_params p;
   gmc_default_params(&p);
@@ -353,7 +353,7 @@ int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* 
   int rc = check_problem(prob, N, T, d, D);
   if (rc != GMC_OK) return rc;
   if (H < 1 || H % prob->Hkv != 0) return GMC_ERR_ARG;
-  if (H > GMC_MAX_HEADS) return GMC_ERR_UNSUPPORTED;
+  if (H > GMC_MAX_HEADS || !heads_supported(H)) return GMC_ERR_UNSUPPORTED;
   gmc_params p;
   if (params) p = *params; else gmc_default_params(&p);
   if (!params_ok(p)) return GMC_ERR_ARG;

@@ -365,13 +365,25 @@ __global__ void __launch_bounds__(256) k_hg_reduce(const double* __restrict__ hg
   cluster_heads(HG + (size_t)b * HE, b, tg.T, N, H, max_clusters, head_eps, omega, tv, sm_hc);
 }
 
+// Dynamic shared memory of k_head_stats for H heads: both staged query
+// chunks, both halves' pair sums and query-weighted squares, the probe values
+// and the tile list.
+static size_t head_stats_smem(int H) {
+  const int npairs = H * (H + 1) / 2;
+  const int nhb = (H + HG_HB - 1) / HG_HB;
+  return sizeof(float) * (2 * (size_t)nhb * HG_HB * HG_RS + 2 * (size_t)npairs * HG_TOK +
+                          2 * H * HG_TOK) +
+         sizeof(float4) * H * HG_TOK + sizeof(unsigned short) * (nhb * (nhb + 1) / 2) + 16;
+}
+
+// Whether the head statistics of H heads fit one block's shared memory
+// (227 KB on sm_103a): H <= 56.
+bool heads_supported(int H) { return H >= 1 && head_stats_smem(H) <= 227 * 1024; }
+
 cudaError_t launch_heads(const Dims& dm, const gmc_params& p, Scratch& s, const TraceView& tv,
                          cudaStream_t st) {
-  const int H = dm.H, npairs = H * (H + 1) / 2;
-  const int nhb = (H + HG_HB - 1) / HG_HB;
-  size_t smem = sizeof(float) * (2 * (size_t)nhb * HG_HB * HG_RS + 2 * (size_t)npairs * HG_TOK +
-                                 2 * H * HG_TOK) +
-                sizeof(float4) * H * HG_TOK + sizeof(unsigned short) * (nhb * (nhb + 1) / 2) + 16;
+  const int H = dm.H;
+  const size_t smem = head_stats_smem(H);
   cudaError_t e = set_smem_limit((const void*)k_head_stats, smem);
   if (e != cudaSuccess) return e;
   launch_k(k_head_stats, dim3(s.nHG, dm.B), 512, smem, st, 1, s.A, s.Z, s.sigma, dm.toff, dm.B, dm.N, dm.T,

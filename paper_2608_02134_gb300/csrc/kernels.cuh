@@ -86,6 +86,7 @@ cudaError_t launch_probe(const Dims&, const void* keys, const float* W, const gm
 cudaError_t launch_message(const Dims&, const void* keys, const void* queries, Scratch&,
                            cudaStream_t);
 cudaError_t launch_heads(const Dims&, const gmc_params&, Scratch&, const TraceView&, cudaStream_t);
+bool heads_supported(int H);  // the head statistics of H heads fit a block (H <= 56)
 cudaError_t launch_gram(const Dims&, const void* hidden, Scratch&, cudaStream_t);
 cudaError_t launch_build_clients(const Dims&, const gmc_params&, int fx_exp, Scratch&,
                                  cudaStream_t);

@@ -64,6 +64,9 @@ def test_workspace_and_trace_sizing(gmc):
     assert gmc.workspace_size(pr32, 1296, 64, 28, 128, 3584, 257) > 31 * ws
     assert gmc.workspace_size(gmc.problem(1, 36, 35, 4, 1), 1296, 64, 28, 128, 3584, 257) == 0
     assert gmc.workspace_size(pr, 1296, 64, 30, 128, 3584, 257) == 0      # H % Hkv != 0
+    # head statistics of one token block must fit shared memory: H <= 56
+    assert gmc.workspace_size(pr, 1296, 64, 56, 128, 3584, 257) > 0
+    assert gmc.workspace_size(pr, 1296, 64, 60, 128, 3584, 257) == 0
     L = gmc.trace_layout(pr, gmc.default_params(), 1296, 64, 28, 257)
     assert L.rounds_max == 17 + 1 and L.pool_size == 64
     assert L.off_order >= 64 and L.bytes_per_image % 16 == 0
@@ -92,6 +95,7 @@ def test_argument_validation(gmc):
     assert _compress_rc(gmc, H=6) == gmc.GMC_ERR_ARG                      # H % Hkv
     assert _compress_rc(gmc, T=0) == gmc.GMC_ERR_ARG
     assert _compress_rc(gmc, H=128, prob=gmc.problem(1, 8, 8, 4, 0)) == gmc.GMC_ERR_UNSUPPORTED
+    assert _compress_rc(gmc, H=60, prob=gmc.problem(1, 8, 8, 4, 0)) == gmc.GMC_ERR_UNSUPPORTED
     assert _compress_rc(gmc, D=250) == gmc.GMC_ERR_UNSUPPORTED           # D % 8
     assert _compress_rc(gmc, ws_bytes=1024) == gmc.GMC_ERR_WORKSPACE
     bad = gmc.default_params(batch_b=64, pool_mult=4)                    # pool 256 > GMC_MAX_POOL
