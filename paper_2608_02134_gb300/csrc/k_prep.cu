@@ -1,7 +1,5 @@
 // Per-token preparation: boundary-state norms, probe values and the mass
 // coordinate, and the K = N identity copy.
-#include <algorithm>
-
 #include "common.cuh"
 #include "kernels.cuh"
 
