@@ -45,6 +45,12 @@ Readings taken where the paper is silent or ambiguous:
     support has one element.
   * Transport blend tau_j = 1 (appendix form); rms(u) = sqrt(mean u^2),
     epsilon 1e-6.
+  * Historical message views (optional): the configuration table's
+    "current/history mass 0.5/0.5" is read as a current-view grounded mass
+    beta_G = 0.5 and a history mass beta_hist = 0.5 shared equally by the
+    completed views; each view carries its own layer's queries, keys, values
+    and probe W = O_h P; omega_h and nu_t weight every view's rows; the
+    message energy is the current view's only.
 
 Pins (tests/test_oracle_pins.py; the paper prints no worked numeric example,
 so every function is pinned by a closed form, an invariant, a bound of the
@@ -79,6 +85,11 @@ paper, a hand-worked case or brute force on tiny inputs, never by itself):
     (Eq. (cond-centroid-optimum)), RMS restoration and its bound.
   * compaction_rows / compress: K = N identity; end-to-end invariants on the
     tiny configuration.
+  * view_patterns / client_matrix_views / compress(history=...): the
+    multi-view pattern Gram equals the beta-weighted sum of single-view
+    pattern Grams; duplicated views keep the single-view cosines and head
+    weights; no history or zero history mass leaves the step unchanged; each
+    view's rows carry its mass; the energy stays the current view's.
 
 Discrete choices (pool, batch, head centres, assignment) are recorded together
 with the fp64 values that decide them.  Every choice can also be *forced*
@@ -100,7 +111,8 @@ DEFAULTS = dict(
     probe_rank=4,            # rank-4 probe
     lambda_mass=1.0,         # lambda_mass = 1
     eps_mass=1e-8,           # epsilon_mass = 1e-8
-    beta_G=0.5,              # current-view grounded mass (history views not built)
+    beta_G=0.5,              # current-view grounded mass
+    beta_hist=0.5,           # historical-view grounded mass, split equally over the views
     beta_V=0.5,              # appearance mass
     beta_S=0.25,             # spatial mass
     tau_v=0.2,               # appearance temperature
@@ -257,6 +269,34 @@ def head_patterns(A: np.ndarray, Z: np.ndarray, sigma: np.ndarray):
     return unit @ unit.T, pre, unit
 
 
+def view_patterns(views):
+    """Eq. (cond-head-pattern) over message views.
+
+    ``views`` lists (A, Z, sigma, beta) per view (current first).  U_h^v
+    collects the atoms of head h in view v divided by their mean norm (the
+    zero vector when every atom is zero); the pattern is
+    concat_v [sqrt(beta_v) vec(U_h^v)] divided by its norm.  Returns the
+    pattern cosine matrix [H, H], the pre-normalisation norms [H] and the unit
+    patterns.
+    """
+    H = views[0][0].shape[0]
+    rows = [[] for _ in range(H)]
+    for A, Z, sigma, beta in views:
+        _, T, N = A.shape
+        for h in range(H):
+            zs = np.concatenate([Z[h], np.full((N, 1), sigma[h])], axis=1)     # [N, r+1]
+            atoms = A[h][:, :, None] * zs[None, :, :]                          # [T, N, r+1]
+            mean_norm = float(np.mean(np.sqrt(np.sum(atoms * atoms, axis=2))))
+            Uv = atoms.reshape(-1) / mean_norm if mean_norm > 0 else np.zeros(atoms.size)
+            rows[h].append(math.sqrt(beta) * Uv)
+    U = np.stack([np.concatenate(r) for r in rows])
+    pre = np.sqrt(np.sum(U * U, axis=1))
+    unit = np.zeros_like(U)
+    nz = pre > 0
+    unit[nz] = U[nz] / pre[nz][:, None]
+    return unit @ unit.T, pre, unit
+
+
 @dataclass
 class HeadClusters:
     centres: list           # centre heads in the order farthest-first chose them
@@ -268,7 +308,8 @@ class HeadClusters:
     n_clusters: int
 
 
-def head_clusters(A, Z, sigma, p, forced_centres=None, forced_assign=None) -> HeadClusters:
+def head_clusters(A, Z, sigma, p, forced_centres=None, forced_assign=None,
+                  views=None) -> HeadClusters:
     """Farthest-first cosine clustering and Eq. (cond-head-weight).
 
     First centre: the largest pre-normalisation pattern.  Then, until
@@ -276,9 +317,10 @@ def head_clusters(A, Z, sigma, p, forced_centres=None, forced_assign=None) -> He
     to the existing centres is smallest.  Each head joins its most similar
     centre.  omega_h = (1/C) (d_h + eps)^-1 / sum_{g in c(h)} (d_g + eps)^-1
     with C the number of nonempty clusters and d_h = 1 - u_h^T mu_c, mu_c the
-    normalised mean pattern of the cluster.
+    normalised mean pattern of the cluster.  With ``views`` (see
+    view_patterns) the patterns span every message view.
     """
-    cos, pre, unit = head_patterns(A, Z, sigma)
+    cos, pre, unit = head_patterns(A, Z, sigma) if views is None else view_patterns(views)
     H = cos.shape[0]
     n_c = min(p["max_head_clusters"], H)
     if forced_centres is not None:
@@ -379,6 +421,7 @@ class ClientMatrix:
     C: np.ndarray                # [M, N] preweighted clients Cbar
     banks: dict                  # bank name -> slice of rows
     active: np.ndarray           # [M] active-row indicator a_m
+    views: dict = None           # message view -> slice of its grounded rows
 
 
 def client_matrix(PG, activeG, omega, nu, PV, PS, p) -> ClientMatrix:
@@ -397,6 +440,35 @@ def client_matrix(PG, activeG, omega, nu, PV, PS, p) -> ClientMatrix:
              "spatial": slice(H * T + N, H * T + N + PS.shape[0])}
     active = np.concatenate([activeG.reshape(-1), np.ones(N, bool), np.ones(PS.shape[0], bool)])
     return ClientMatrix(C, banks, active)
+
+
+def client_matrix_views(PGs, actives, betas, omega, nu, PV, PS, p) -> ClientMatrix:
+    """Eq. (cond-coverage) with message views: the grounded rows of every view
+    (view v, h, t) h-major within the view, views in order (current first),
+    then appearance rows, then landmarks.
+
+    Grounded row (v, h, t): beta_v * omega_h * nu_t * a_{v,h,t} * P^G_{v,h,t}.
+    The bank "grounded" spans every view's rows; ``views[v]`` each view's block.
+    """
+    blocks, act = [], []
+    views = {}
+    at = 0
+    for v, (PG, a, beta) in enumerate(zip(PGs, actives, betas)):
+        H, T, N = PG.shape
+        w = beta * omega[:, None] * nu[None, :] * a
+        blocks.append((w[:, :, None] * PG).reshape(H * T, N))
+        act.append(a.reshape(-1))
+        views[v] = slice(at, at + H * T)
+        at += H * T
+    N = PV.shape[0]
+    G = np.concatenate(blocks, axis=0)
+    V = (p["beta_V"] / N) * PV
+    S = (p["beta_S"] / PS.shape[0]) * PS
+    C = np.concatenate([G, V, S], axis=0)
+    banks = {"grounded": slice(0, at), "appearance": slice(at, at + N),
+             "spatial": slice(at + N, at + N + PS.shape[0])}
+    active = np.concatenate(act + [np.ones(N, bool), np.ones(PS.shape[0], bool)])
+    return ClientMatrix(C, banks, active, views)
 
 
 def facility_value(C: np.ndarray, S) -> float:
@@ -662,14 +734,22 @@ class Result:
     out_hidden: np.ndarray = None  # float64 compact hidden (transported visual rows, text rows)
     out_kv: np.ndarray = None      # [2, K+T, Hkv, d]
     out_pos: np.ndarray = None     # [3, K+T]
+    history: list = None           # per historical view: (A, Z, sigma, unorm, PG, active)
 
 
-def compress(hidden, Kall, Vall, Q, pos, W, gh, gw, K_r, p=None, forced=None) -> Result:
+def compress(hidden, Kall, Vall, Q, pos, W, gh, gw, K_r, p=None, forced=None,
+             history=None) -> Result:
     """Grounded Message Coreset compression of one image boundary.
 
     hidden [N+T, D], Kall/Vall [N+T, Hkv, d], Q [T, H, d], pos [3, N+T],
     W [H, d, r].  ``forced`` may hold "centres", "head_assign", "rounds",
     "pi" to follow choices made elsewhere (see the module docstring).
+    ``history`` (optional) lists completed historical message views, each a
+    dict with that layer's text queries "Q" [T, H, d], keys "K" and values
+    "V" [N+T, Hkv, d] and probe "W" [H, d, r] (Appendix "Native message
+    clients"): every view adds its own grounded rows, the head patterns span
+    all views, the views share beta_hist equally, and the message energy stays
+    the current view's (Eq. (cond-grounded-energy)).
     """
     p = p or params()
     forced = forced or {}
@@ -688,13 +768,29 @@ def compress(hidden, Kall, Vall, Q, pos, W, gh, gw, K_r, p=None, forced=None) ->
     res.unorm = atom_norms(res.A, res.Z, res.sigma)
     res.PG, res.activeG = grounded_clients(res.unorm)
     res.nu = query_weights(T, p)
+    views = None
+    if history is not None:
+        res.history = []
+        views = [(res.A, res.Z, res.sigma, p["beta_G"])]
+        for view in history:
+            A_v = message_slice(view["Q"], view["K"], N)
+            Z_v, s_v = probe_values(view["V"][:N], view["W"], H, p)
+            un_v = atom_norms(A_v, Z_v, s_v)
+            PG_v, act_v = grounded_clients(un_v)
+            res.history.append((A_v, Z_v, s_v, un_v, PG_v, act_v))
+            views.append((A_v, Z_v, s_v, p["beta_hist"] / len(history)))
     res.heads = head_clusters(res.A, res.Z, res.sigma, p,
-                              forced.get("centres"), forced.get("head_assign"))
+                              forced.get("centres"), forced.get("head_assign"), views=views)
     res.e, res.ebar = message_energy(res.unorm, res.heads.omega, res.nu)
     res.cos = cosine_matrix(hvis, p)
     PV = appearance_clients(res.cos, p)
     PS = spatial_clients(gh, gw, p)
-    res.clients = client_matrix(res.PG, res.activeG, res.heads.omega, res.nu, PV, PS, p)
+    if history is None:
+        res.clients = client_matrix(res.PG, res.activeG, res.heads.omega, res.nu, PV, PS, p)
+    else:
+        res.clients = client_matrix_views(
+            [res.PG] + [hv[4] for hv in res.history], [res.activeG] + [hv[5] for hv in res.history],
+            [v[3] for v in views], res.heads.omega, res.nu, PV, PS, p)
     res.selection = select_support(res.clients.C, K, p, forced=forced.get("rounds"))
     res.support = res.selection.support
     res.assignment = assign_population(res.cos, res.support, gh, gw, p, forced.get("pi"))

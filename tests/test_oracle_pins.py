@@ -643,3 +643,96 @@ def test_compaction_rows_index_map():
     rows = O.compaction_rows(np.array([1, 4, 6]), N=8, T=3)
     np.testing.assert_array_equal(rows, [1, 4, 6, 8, 9, 10])
     assert O.compaction_rows(np.array([], dtype=np.int64), N=4, T=0).size == 0
+
+
+# --------------------------------------------------------------------------
+# historical message views (Appendix "Native message clients": every view is a
+# separate client collection; Eq. (cond-head-pattern) concatenates the views)
+# --------------------------------------------------------------------------
+def _tiny_with_history(n_views=2, beta_hist=None, same_as_current=False, seed=7):
+    from paper_2608_02134_gb300 import workloads
+    wl = workloads.make("tiny")
+    im = wl.image(0)
+    f = lambda a: np.asarray(a, dtype=np.float64)
+    g = rng(seed)
+    T, H, d = im.queries.shape
+    hist = []
+    for _ in range(n_views):
+        if same_as_current:
+            hist.append(dict(Q=f(im.queries), K=f(im.keys), V=f(im.values), W=f(wl.probe())))
+        else:
+            hist.append(dict(Q=g.standard_normal(im.queries.shape),
+                             K=g.standard_normal(im.keys.shape),
+                             V=g.standard_normal(im.values.shape),
+                             W=g.standard_normal(wl.probe().shape) / math.sqrt(wl.D)))
+    p = O.params() if beta_hist is None else O.params(beta_hist=beta_hist)
+    args = (f(im.hidden), f(im.keys), f(im.values), f(im.queries), im.pos, f(wl.probe()),
+            wl.gh, wl.gw, wl.K, p)
+    return wl, O.compress(*args), O.compress(*args, history=hist), p
+
+
+def test_view_patterns_combine_single_view_patterns():
+    # blocks of the concatenated pattern are orthogonal, so
+    # <u_h, u_g> = sum_v beta_v <U_h^v, U_g^v> with <U_h^v, U_g^v> = cos_v pre_v pre_v
+    g = rng(11)
+    H, T, N, r = 3, 2, 5, 4
+    views = []
+    for beta in (0.5, 0.2, 0.3):
+        A = g.random((H, T, N))
+        A /= A.sum(axis=2, keepdims=True)
+        views.append((A, g.standard_normal((H, N, r)), g.random(H) + 0.1, beta))
+    cos, pre, _ = O.view_patterns(views)
+    dot = np.zeros((H, H))
+    for A, Z, sigma, beta in views:
+        c1, p1, _ = O.head_patterns(A, Z, sigma)
+        dot += beta * c1 * np.outer(p1, p1)
+    np.testing.assert_allclose(pre, np.sqrt(np.diag(dot)), rtol=1e-12)
+    np.testing.assert_allclose(cos, dot / np.outer(pre, pre), rtol=1e-12)
+
+
+def test_duplicate_views_keep_the_single_view_patterns():
+    g = rng(12)
+    H, T, N = 4, 3, 6
+    A = g.random((H, T, N))
+    Z = g.standard_normal((H, N, 4))
+    sigma = g.random(H) + 0.1
+    c1, p1, _ = O.head_patterns(A, Z, sigma)
+    cos, pre, _ = O.view_patterns([(A, Z, sigma, 0.5), (A, Z, sigma, 0.25), (A, Z, sigma, 0.25)])
+    np.testing.assert_allclose(cos, c1, rtol=1e-12, atol=1e-15)
+    np.testing.assert_allclose(pre, p1, rtol=1e-12)        # sqrt(0.5 + 0.25 + 0.25) = 1
+
+
+def test_no_history_and_zero_history_mass_leave_the_step_unchanged():
+    wl, base, empty, _ = _tiny_with_history(n_views=0)
+    np.testing.assert_array_equal(empty.support, base.support)
+    np.testing.assert_allclose(empty.heads.omega, base.heads.omega, rtol=1e-12)
+    np.testing.assert_allclose(empty.clients.C, base.clients.C, rtol=1e-12, atol=1e-18)
+    wl, base, zero, _ = _tiny_with_history(n_views=2, beta_hist=0.0)
+    np.testing.assert_array_equal(zero.support, base.support)
+    np.testing.assert_allclose(zero.heads.omega, base.heads.omega, rtol=1e-12)
+    assert not zero.clients.C[zero.clients.views[1]].any()
+
+
+def test_history_views_add_client_blocks_with_their_masses():
+    wl, base, res, p = _tiny_with_history(n_views=2)
+    H, T = wl.H, int(wl.T[0])
+    cm = res.clients
+    assert cm.C.shape[0] == 3 * H * T + wl.N + p["landmarks"] ** 2
+    masses = [p["beta_G"], p["beta_hist"] / 2, p["beta_hist"] / 2]
+    for v, beta in enumerate(masses):
+        blk = cm.C[cm.views[v]]
+        assert blk.shape == (H * T, wl.N)
+        act = [res.activeG] + [hv[5] for hv in res.history]
+        want = beta * np.outer(res.heads.omega, res.nu) * act[v]
+        np.testing.assert_allclose(blk.sum(axis=1), want.reshape(-1), rtol=1e-12, atol=1e-18)
+    # the message energy stays the current view's (Eq. (cond-grounded-energy))
+    e, _ = O.message_energy(res.unorm, res.heads.omega, res.nu)
+    np.testing.assert_allclose(res.e, e, rtol=1e-14)
+    S = res.support
+    assert S.size == wl.K and np.all(np.diff(S) > 0)
+
+
+def test_duplicated_current_view_as_history_keeps_head_weights():
+    wl, base, res, _ = _tiny_with_history(n_views=2, same_as_current=True)
+    np.testing.assert_array_equal(res.heads.centres, base.heads.centres)
+    np.testing.assert_allclose(res.heads.omega, base.heads.omega, rtol=1e-12)
