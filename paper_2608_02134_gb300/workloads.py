@@ -31,6 +31,12 @@ has i.i.d. N(0,1/D) entries, and is drawn that way from seed 0.
 Positions: M-RoPE visual (0, r, c), text s+k on all three rows with
 s = max(gh, gw); 1-D layouts use (i, i, i) and N+k.
 Seeds: numpy default_rng(1000 + workload index), one substream per image.
+
+Historical message views (``history_view``): the text queries, keys, values
+and probe of an earlier layer for the same image, drawn from their own
+substreams (seed, image, 1 + view) and probe seed (0, 1 + view), so the
+boundary tensors above do not change.  Where the image has object regions,
+the view's visual keys follow the same regions with fresh region centres.
 """
 
 from __future__ import annotations
@@ -69,6 +75,7 @@ class Image:
     queries: np.ndarray   # [T, H, d]
     pos: np.ndarray       # [3, N+T] int32
     T: int
+    region: np.ndarray = None  # [N] object region of every visual token (region workloads)
 
 
 @dataclass
@@ -162,9 +169,27 @@ class Workload:
             pos[:, :N] = np.arange(N)
             pos[:, N:] = N + np.arange(T)
         img = Image(self._round(hidden), self._round(keys), self._round(values),
-                    self._round(queries), pos, T)
+                    self._round(queries), pos, T,
+                    region if self.structure.startswith("regions") else None)
         self._cache[b] = img
         return img
+
+    def history_view(self, b: int, v: int) -> dict:
+        """Historical view v of image b: Q [T, H, d], K and V [N+T, Hkv, d],
+        W [H, d, 4] (rounded like the boundary tensors)."""
+        im = self.image(b)
+        rng = np.random.default_rng([self.seed, b, 1 + v])
+        N, T, H, Hkv, d = self.N, self.T[b], self.H, self.Hkv, self.d
+        f32 = np.float32
+        q = rng.standard_normal((T, H, d), dtype=f32)
+        k = rng.standard_normal((N + T, Hkv, d), dtype=f32)
+        val = rng.standard_normal((N + T, Hkv, d), dtype=f32)
+        if im.region is not None:
+            kap = rng.standard_normal((int(im.region.max()) + 1, Hkv, d), dtype=f32)
+            k[:N] = kap[im.region] + f32(0.3) * rng.standard_normal((N, Hkv, d), dtype=f32)
+        w = (np.random.default_rng([0, 1 + v]).standard_normal((H, d, 4), dtype=f32)
+             / f32(np.sqrt(self.D))).astype(f32)
+        return dict(Q=self._round(q), K=self._round(k), V=self._round(val), W=w)
 
     def text_offsets(self) -> np.ndarray:
         return np.concatenate([[0], np.cumsum(self.T)]).astype(np.int32)

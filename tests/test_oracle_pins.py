@@ -649,22 +649,17 @@ def test_compaction_rows_index_map():
 # historical message views (Appendix "Native message clients": every view is a
 # separate client collection; Eq. (cond-head-pattern) concatenates the views)
 # --------------------------------------------------------------------------
-def _tiny_with_history(n_views=2, beta_hist=None, same_as_current=False, seed=7):
+def _tiny_with_history(n_views=2, beta_hist=None, same_as_current=False):
     from paper_2608_02134_gb300 import workloads
     wl = workloads.make("tiny")
     im = wl.image(0)
     f = lambda a: np.asarray(a, dtype=np.float64)
-    g = rng(seed)
-    T, H, d = im.queries.shape
     hist = []
     for _ in range(n_views):
         if same_as_current:
             hist.append(dict(Q=f(im.queries), K=f(im.keys), V=f(im.values), W=f(wl.probe())))
         else:
-            hist.append(dict(Q=g.standard_normal(im.queries.shape),
-                             K=g.standard_normal(im.keys.shape),
-                             V=g.standard_normal(im.values.shape),
-                             W=g.standard_normal(wl.probe().shape) / math.sqrt(wl.D)))
+            hist.append({k: f(a) for k, a in wl.history_view(0, len(hist)).items()})
     p = O.params() if beta_hist is None else O.params(beta_hist=beta_hist)
     args = (f(im.hidden), f(im.keys), f(im.values), f(im.queries), im.pos, f(wl.probe()),
             wl.gh, wl.gw, wl.K, p)
