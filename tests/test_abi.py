@@ -118,3 +118,11 @@ def test_select_and_transport_validation(gmc):
     assert lib.gmc_transport(ctypes.byref(pr), None, fake, fake, fake, fake, fake, fake, 20, 3, 8,
                              16, 0, fake, fake, fake, fake, fake, 1 << 30, None) == gmc.GMC_ERR_ARG
     assert lib.gmc_read_status(None, None, None) == gmc.GMC_ERR_ARG
+
+
+def test_binding_raises_without_the_library(gmc, monkeypatch, tmp_path):
+    """No fallback: a missing libgmc.so is an error, not a silent CPU path."""
+    monkeypatch.setattr(gmc, "_lib", None)
+    monkeypatch.setattr(gmc, "LIB_PATH", str(tmp_path / "libgmc.so"))
+    with pytest.raises(RuntimeError, match="missing"):
+        gmc.lib()
