@@ -351,7 +351,9 @@ def run_gmc(args):
             cpu = {"value": round(o["boundaries"] / o["seconds"], 6), "unit": UNIT, "cores": cores,
                    "kind": "oracle",
                    "sample": f"{o['boundaries']} boundaries of the {args.workload} workload (about 10 s "
-                             f"of CPU work: {o['seconds']:.2f} s), fp64 numpy oracle"}
+                             f"of CPU work: {o['seconds']:.2f} s), fp64 numpy oracle, one boundary "
+                             f"at a time; its matrix products use up to {cores} BLAS threads, the "
+                             f"rest runs on one core"}
         except Exception as e:  # keep the GPU line even if the host run fails
             cpu = {"value": None, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": f"failed: {e}"}
 
@@ -405,7 +407,9 @@ def run_reference(args):
         "config": workload_config(wl) | {"parallelism": "host cores",
                                          "boundaries_per_step": 1},
         "cpu_baseline": {"value": round(value, 6), "unit": UNIT, "cores": cores, "kind": "oracle",
-                         "sample": f"one boundary of the {args.workload} workload per step"},
+                         "sample": f"one boundary of the {args.workload} workload per step; "
+                                   f"matrix products on up to {cores} BLAS threads, the rest on "
+                                   f"one core"},
         "e2e": {"value": round(value, 6), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
