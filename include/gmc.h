@@ -74,6 +74,7 @@ typedef struct CUstream_st* gmc_stream_t; /* identical to cudaStream_t */
 #define GMC_MAX_N 8192            /* visual tokens per image */
 #define GMC_MAX_POOL 128          /* pool_mult * batch_b */
 #define GMC_MAX_HEADS 64          /* H */
+#define GMC_MAX_VIEWS 4           /* message views: the current one and up to 3 historical ones */
 
 /*
  * Method constants.  gmc_default_params() fills the values of the paper's
@@ -127,6 +128,27 @@ typedef struct gmc_problem {
 size_t gmc_workspace_size(const gmc_problem* prob, int N, int T, int H, int d, int D, int K);
 
 /*
+ * Completed historical message views (appendix "Native message clients"):
+ * earlier layers' text queries, keys/values and value-output probes of the
+ * same images.  Each view adds its own grounded client rows (beta_hist is
+ * shared equally by the views; the current view keeps params->beta_G), the
+ * head patterns concatenate every view (Eq. (cond-head-pattern)), and the
+ * message energy stays the current view's.  Every pointer has the layout of
+ * the corresponding gmc_compress argument.
+ */
+typedef struct gmc_views {
+  int n;                                     /* historical views, 0 .. GMC_MAX_VIEWS-1 */
+  float beta_hist;                           /* their total grounded mass (0.5) */
+  const void* keys[GMC_MAX_VIEWS - 1];       /* per view: keys then values, as `keys` */
+  const void* queries[GMC_MAX_VIEWS - 1];    /* per view: text queries, as `queries` */
+  const float* vo_probe[GMC_MAX_VIEWS - 1];  /* per view: W_h = O_h P of that layer */
+} gmc_views;
+
+/* Workspace of gmc_compress_views with n_views historical views (0 on invalid arguments). */
+size_t gmc_workspace_size_views(const gmc_problem* prob, int n_views, int N, int T, int H, int d,
+                                int D, int K);
+
+/*
  * gmc_compress -- one GMC boundary compression per image (Algorithm 1, steps 2-6).
  *
  * Let Tb = T_b, Rb = N + T_b, Kb = K (after the budget rule), with per-image
@@ -167,6 +189,14 @@ int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* 
                  const float* vo_probe, int N, int T, int H, int d, int D, int K,
                  int32_t* out_idx, void* out_hidden, void* out_kv, int32_t* out_pos,
                  void* workspace, size_t ws_bytes, void* trace, gmc_stream_t stream);
+
+/* gmc_compress with historical message views (views NULL or n == 0: gmc_compress). */
+int gmc_compress_views(const gmc_problem* prob, const gmc_params* params, const gmc_views* views,
+                       const void* hidden, const void* keys, const void* queries,
+                       const int32_t* pos_ids, const float* vo_probe, int N, int T, int H, int d,
+                       int D, int K, int32_t* out_idx, void* out_hidden, void* out_kv,
+                       int32_t* out_pos, void* workspace, size_t ws_bytes, void* trace,
+                       gmc_stream_t stream);
 
 /*
  * Diagnostics trace (optional).  Image b's record starts at byte

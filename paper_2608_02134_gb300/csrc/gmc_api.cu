@@ -73,17 +73,24 @@ int check_problem(const gmc_problem* prob, int N, int T, int d, int D) {
 bool aligned(const void* p, size_t a) { return ((uintptr_t)p % a) == 0; }
 
 Dims make_dims(const gmc_problem* prob, const gmc_params& p, int N, int T, int H, int d, int D,
-               int K) {
+               int K, int V = 1) {
   Dims dm;
   dm.B = prob->B; dm.N = N; dm.T = T; dm.H = H; dm.Hkv = prob->Hkv; dm.d = d; dm.D = D;
   dm.K = K; dm.gh = prob->grid_h; dm.gw = prob->grid_w; dm.L = p.landmarks;
-  dm.M = H * T + N + p.landmarks * p.landmarks;
+  dm.V = V;
+  dm.M = V * H * T + N + p.landmarks * p.landmarks;
   dm.dtype = prob->dtype;
   dm.toff = prob->text_offsets;
   return dm;
 }
 
 R0State carve_round0(Carver& c, size_t B, size_t N, size_t M);
+
+// Words of the per-call zeroed status block: status, probe tickets (per
+// view), assignment tickets, head-Gram tickets (per view), membership bitmaps.
+size_t status_words(const Dims& dm) {
+  return 4 + (2 * (size_t)dm.V + 1) * dm.B + (size_t)dm.B * dm.K * ceil_div(dm.N, 32);
+}
 
 // Workspace of gmc_compress.  base == nullptr only measures.
 size_t carve_compress(const Dims& dm, Scratch* s, char* base, R0State* r0s = nullptr) {
@@ -95,25 +102,40 @@ size_t carve_compress(const Dims& dm, Scratch* s, char* base, R0State* r0s = nul
   t.nA = ceil_div(dm.N, ASSIGN_WARPS);
   t.nE = t.nA;  // energy block sums come from the assignment gap kernel
   t.nSel = 0;
-  // status word, the probe, head-Gram and assignment tickets of every image,
-  // then the carrier membership bitmaps: one block, zeroed by one memset per call
-  t.status = c.take<uint32_t>(4 + 3 * B + B * K * (size_t)ceil_div(dm.N, 32));
+  const size_t V = dm.V;
+  t.V = dm.V;
+  t.B = dm.B;
+  // status word, the probe (per view), assignment and head-Gram (per view)
+  // tickets of every image, then the carrier membership bitmaps: one block,
+  // zeroed by one memset per call
+  t.status = c.take<uint32_t>(status_words(dm));
   t.tick = t.status + 4;
-  t.tick2 = t.tick + B;
+  t.tick2 = t.tick + V * B;
   t.tick3 = t.tick2 + B;
-  t.mbits = t.tick3 + B;
+  t.mbits = t.tick3 + V * B;
   t.gatev = c.take<float>(B * 4);
-  t.A = c.take<float>(B * H * T * N);
   t.nRS = message_splits(dm);
-  t.rs = c.take<float>(B * H * (size_t)t.nRS * T);
-  t.mpart = c.take<float2>(B * dm.Hkv * (size_t)message_rq(dm) * t.nRS);
-  t.Z = c.take<float>(B * H * N * 4);
-  t.zn2 = c.take<float>(B * H * N);
-  t.sigpart = c.take<float>(B * t.nP * H);
-  t.sigma = c.take<float>(B * H);
-  t.hgpart = c.take<double>(B * t.nHG * H * H);
-  t.HG = c.take<double>(B * (H * H + H));
-  t.W2 = c.take<float>(B * H * N);
+  t.vA = B * H * T * N;
+  t.vrs = B * H * (size_t)t.nRS * T;
+  t.vmp = B * dm.Hkv * (size_t)message_rq(dm) * t.nRS;
+  t.vZ = B * H * N * 4;
+  t.vzn = B * H * N;
+  t.vsp = B * t.nP * H;
+  t.vsg = B * H;
+  t.vhp = B * t.nHG * H * H;
+  t.vHG = B * (H * H + H);
+  t.vW2 = B * H * N;
+  t.vQp = B * dm.Hkv * (size_t)message_rq(dm) * dm.d;
+  t.A = c.take<float>(V * t.vA);
+  t.rs = c.take<float>(V * t.vrs);
+  t.mpart = c.take<float2>(V * t.vmp);
+  t.Z = c.take<float>(V * t.vZ);
+  t.zn2 = c.take<float>(V * t.vzn);
+  t.sigpart = c.take<float>(V * t.vsp);
+  t.sigma = c.take<float>(V * t.vsg);
+  t.hgpart = c.take<double>(V * t.vhp);
+  t.HG = c.take<double>(V * t.vHG);
+  t.W2 = c.take<float>(V * t.vW2);
   t.omega = c.take<float>(B * H);
   t.ebar = c.take<float>(B * N);
   t.rn = c.take<float>(B * N);
@@ -132,7 +154,7 @@ size_t carve_compress(const Dims& dm, Scratch* s, char* base, R0State* r0s = nul
   t.mass = c.take<float>(B * N);
   t.selpart = nullptr;
   t.fexp = nullptr;
-  t.Qp = c.take<__nv_bfloat16>(B * dm.Hkv * (size_t)message_rq(dm) * dm.d);
+  t.Qp = c.take<__nv_bfloat16>(V * t.vQp);
   if (s) *s = t;
   R0State r0 = carve_round0(c, B, N, M);
   if (r0s && base) *r0s = r0;
@@ -319,14 +341,19 @@ const char* gmc_error_string(int code) {
 
 const char* gmc_version(void) { return "gmc 0.1.0 sm_103a"; }
 
-size_t gmc_workspace_size(const gmc_problem* prob, int N, int T, int H, int d, int D, int K) {
+size_t gmc_workspace_size_views(const gmc_problem* prob, int n_views, int N, int T, int H, int d,
+                                int D, int K) {
   if (check_problem(prob, N, T, d, D) != GMC_OK || H < 1 || H > GMC_MAX_HEADS ||
-      H % prob->Hkv != 0 || !heads_supported(H))
+      H % prob->Hkv != 0 || !heads_supported(H) || n_views < 0 || n_views > GMC_MAX_VIEWS - 1)
     return 0;
   gmc_params p;
   gmc_default_params(&p);
-  const Dims dm = make_dims(prob, p, N, T, H, d, D, effective_K(K, N));
+  const Dims dm = make_dims(prob, p, N, T, H, d, D, effective_K(K, N), 1 + n_views);
   return carve_compress(dm, nullptr, nullptr);
+}
+
+size_t gmc_workspace_size(const gmc_problem* prob, int N, int T, int H, int d, int D, int K) {
+  return gmc_workspace_size_views(prob, 0, N, T, H, d, D, K);
 }
 
 int gmc_get_trace_layout(const gmc_problem* prob, const gmc_params* params, int N, int T, int H,
@@ -345,11 +372,12 @@ size_t gmc_trace_size(const gmc_problem* prob, const gmc_params* params, int N, 
   return (size_t)prob->B * L.bytes_per_image;
 }
 
-int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* hidden,
-                 const void* keys, const void* queries, const int32_t* pos_ids,
-                 const float* vo_probe, int N, int T, int H, int d, int D, int K,
-                 int32_t* out_idx, void* out_hidden, void* out_kv, int32_t* out_pos,
-                 void* workspace, size_t ws_bytes, void* trace, gmc_stream_t stream_) {
+static int compress_impl(const gmc_problem* prob, const gmc_params* params,
+                         const gmc_views* views, const void* hidden, const void* keys,
+                         const void* queries, const int32_t* pos_ids, const float* vo_probe,
+                         int N, int T, int H, int d, int D, int K, int32_t* out_idx,
+                         void* out_hidden, void* out_kv, int32_t* out_pos, void* workspace,
+                         size_t ws_bytes, void* trace, gmc_stream_t stream_) {
   int rc = check_problem(prob, N, T, d, D);
   if (rc != GMC_OK) return rc;
   if (H < 1 || H % prob->Hkv != 0) return GMC_ERR_ARG;
@@ -364,8 +392,26 @@ int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* 
       !aligned(vo_probe, 16) || !aligned(out_hidden, 16) || !aligned(out_kv, 16) ||
       !aligned(workspace, ALIGN) || (trace && !aligned(trace, 16)))
     return GMC_ERR_ARG;
+  // message views: view 0 is the call's own, then the historical ones
+  const int nh = views ? views->n : 0;
+  if (nh < 0 || nh > GMC_MAX_VIEWS - 1) return GMC_ERR_ARG;
+  if (nh > 0 && !(views->beta_hist >= 0.f)) return GMC_ERR_ARG;
+  const int V = 1 + nh;
+  const void* vkeys[GMC_MAX_VIEWS] = {keys};
+  const void* vqueries[GMC_MAX_VIEWS] = {queries};
+  const float* vprobe[GMC_MAX_VIEWS] = {vo_probe};
+  float vbeta[GMC_MAX_VIEWS] = {p.beta_G};
+  for (int v = 1; v < V; ++v) {
+    vkeys[v] = views->keys[v - 1];
+    vqueries[v] = views->queries[v - 1];
+    vprobe[v] = views->vo_probe[v - 1];
+    vbeta[v] = views->beta_hist / (float)nh;
+    if (!vkeys[v] || !vqueries[v] || !vprobe[v] || !aligned(vkeys[v], 16) ||
+        !aligned(vqueries[v], 16) || !aligned(vprobe[v], 16))
+      return GMC_ERR_ARG;
+  }
   const int Ke = effective_K(K, N);
-  const Dims dm = make_dims(prob, p, N, T, H, d, D, Ke);
+  const Dims dm = make_dims(prob, p, N, T, H, d, D, Ke, V);
   Scratch s;
   R0State r0;
   const size_t need = carve_compress(dm, &s, (char*)workspace, &r0);
@@ -380,22 +426,59 @@ int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* 
   }
   std::lock_guard<std::mutex> lk(g_prof.mu);
   // status, tickets, membership bitmaps
-  GMC_TRY(cudaMemsetAsync(
-      s.status, 0, sizeof(uint32_t) * (4 + 3 * dm.B + (size_t)dm.B * dm.K * ceil_div(dm.N, 32)),
-      st));
+  GMC_TRY(cudaMemsetAsync(s.status, 0, sizeof(uint32_t) * status_words(dm), st));
   if (Ke == N) {  // K = N returns the unmodified execution
     GMC_TRY(launch_identity(dm, hidden, keys, pos_ids, out_idx, out_hidden, out_kv, out_pos,
                             s.status, st));
     g_launches += 1;
     return GMC_OK;
   }
-  const int fx = fixed_point_exponent((double)p.beta_G + p.beta_V + p.beta_S);
+  double mass = (double)p.beta_G + p.beta_V + p.beta_S;
+  if (nh > 0) mass += views->beta_hist;
+  const int fx = fixed_point_exponent(mass);
+  Scratch sv[GMC_MAX_VIEWS];
+  ViewRows vr{};
+  ViewGrams vg{};
+  vr.n = vg.n = V;
+  for (int v = 0; v < V; ++v) {
+    sv[v] = s.view(v);
+    vr.A[v] = sv[v].A;
+    vr.rs[v] = sv[v].rs;
+    vr.zn2[v] = sv[v].zn2;
+    vr.sigma[v] = sv[v].sigma;
+    vr.beta[v] = vg.beta[v] = vbeta[v];
+    vg.HG[v] = sv[v].HG;
+  }
+  // every view's probe and message slice; the historical views' head Grams,
+  // then the current view's, whose last block clusters the heads over all views
+  auto probes = [&]() -> cudaError_t {
+    for (int v = 0; v < V; ++v) {
+      const cudaError_t e = launch_probe(dm, vkeys[v], vprobe[v], p, sv[v], st);
+      if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
+  };
+  auto messages = [&]() -> cudaError_t {
+    for (int v = 0; v < V; ++v) {
+      const cudaError_t e = launch_message(dm, vkeys[v], vqueries[v], sv[v], st);
+      if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
+  };
+  auto heads = [&]() -> cudaError_t {
+    for (int v = 1; v < V; ++v) {
+      const cudaError_t e = launch_heads(dm, p, sv[v], tv, st, 0, nullptr);
+      if (e != cudaSuccess) return e;
+    }
+    return launch_heads(dm, p, sv[0], tv, st, 1, V > 1 ? &vg : nullptr);
+  };
+  const int msg_k = (message_tc_supported(dm) ? 3 : 1) * V;
   GMC_TRY(g_prof.begin(st));  // k_probe zeroes the column sums u0 of the client build
   if (g_prof.on) {  // stage timing: every stage in turn on the caller's stream
     GMC_STAGE("rownorm", 1, launch_rownorm(dm, hidden, p.norm_eps, s, st));
-    GMC_STAGE("probe", 1, launch_probe(dm, keys, vo_probe, p, s, st));
-    GMC_STAGE("message", message_tc_supported(dm) ? 3 : 1, launch_message(dm, keys, queries, s, st));
-    GMC_STAGE("heads", 2, launch_heads(dm, p, s, tv, st));
+    GMC_STAGE("probe", V, probes());
+    GMC_STAGE("message", msg_k, messages());
+    GMC_STAGE("heads", 2 * V, heads());
     GMC_STAGE("gram", 1, launch_gram(dm, hidden, s, st));
   } else {
     // row norms and the cosine Gram run beside probe -> message -> heads
@@ -406,17 +489,19 @@ int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* 
     GMC_STAGE("rownorm", 1, launch_rownorm(dm, hidden, p.norm_eps, s, sd->st));
     GMC_STAGE("gram", 1, launch_gram(dm, hidden, s, sd->st));
     GMC_TRY(cudaEventRecord(sd->join, sd->st));
-    GMC_STAGE("probe", 1, launch_probe(dm, keys, vo_probe, p, s, st));
-    GMC_STAGE("message", message_tc_supported(dm) ? 3 : 1, launch_message(dm, keys, queries, s, st));
-    GMC_STAGE("heads", 2, launch_heads(dm, p, s, tv, st));
+    GMC_STAGE("probe", V, probes());
+    GMC_STAGE("message", msg_k, messages());
+    GMC_STAGE("heads", 2 * V, heads());
     GMC_TRY(cudaStreamWaitEvent(st, sd->join, 0));
   }
-  GMC_STAGE("clients", 1, launch_build_clients(dm, p, fx, s, st));
+  // every view's grounded rows count as head rows of the client layout
+  const int HV = H * V;
+  GMC_STAGE("clients", 1, launch_build_clients(dm, p, fx, s, vr, st));
   GMC_STAGE("rounds_gpu", 3 + 3 * SPARSE_GPU_ROUNDS,
-            launch_round0(r0, dm.B, N, Ke, dm.M, dm.toff, H, T, p.landmarks * p.landmarks, p, fx,
+            launch_round0(r0, dm.B, N, Ke, dm.M, dm.toff, HV, T, p.landmarks * p.landmarks, p, fx,
                           nullptr, s.C, s.scol, s.u0, s.order, s.status, tv, st));
   GMC_STAGE("select", 1,
-            launch_select(r0, dm.B, N, Ke, dm.M, dm.toff, H, T, p.landmarks * p.landmarks, p, fx,
+            launch_select(r0, dm.B, N, Ke, dm.M, dm.toff, HV, T, p.landmarks * p.landmarks, p, fx,
                           nullptr, s.C, s.scol, s.u0, s.order, s.support, s.slot, nullptr, s.status,
                           tv, st));
   GMC_STAGE("assign", 2, launch_assign(dm, p, s, tv, st));
@@ -425,6 +510,27 @@ int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* 
                              s.mbits, out_idx, out_hidden, out_kv, out_pos, s.status, st));
   g_prof.valid = g_prof.on;
   return GMC_OK;
+}
+
+int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* hidden,
+                 const void* keys, const void* queries, const int32_t* pos_ids,
+                 const float* vo_probe, int N, int T, int H, int d, int D, int K,
+                 int32_t* out_idx, void* out_hidden, void* out_kv, int32_t* out_pos,
+                 void* workspace, size_t ws_bytes, void* trace, gmc_stream_t stream_) {
+  return compress_impl(prob, params, nullptr, hidden, keys, queries, pos_ids, vo_probe, N, T, H,
+                       d, D, K, out_idx, out_hidden, out_kv, out_pos, workspace, ws_bytes, trace,
+                       stream_);
+}
+
+int gmc_compress_views(const gmc_problem* prob, const gmc_params* params, const gmc_views* views,
+                       const void* hidden, const void* keys, const void* queries,
+                       const int32_t* pos_ids, const float* vo_probe, int N, int T, int H, int d,
+                       int D, int K, int32_t* out_idx, void* out_hidden, void* out_kv,
+                       int32_t* out_pos, void* workspace, size_t ws_bytes, void* trace,
+                       gmc_stream_t stream_) {
+  return compress_impl(prob, params, views, hidden, keys, queries, pos_ids, vo_probe, N, T, H, d,
+                       D, K, out_idx, out_hidden, out_kv, out_pos, workspace, ws_bytes, trace,
+                       stream_);
 }
 
 // ---------------------------------------------------------------------------

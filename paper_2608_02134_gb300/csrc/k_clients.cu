@@ -1,8 +1,11 @@
 // Client matrix Cbar (appendix Eq. (cond-coverage)) and its column sums.
 //
 // Rows of image b, in this order:
-//   grounded   (h, t), h-major:  beta_G * omega_h * nu_t * ||u_i^{h,t}|| / sum_j ||u_j^{h,t}||
-//              (zero when the row has no energy: an inactive client)
+//   grounded   (v, h, t), view-major then h-major:
+//              beta_v * omega_h * nu_t * ||u_i^{v,h,t}|| / sum_j ||u_j^{v,h,t}||
+//              (v = 0 the current view with beta_G, then the historical views
+//              sharing beta_hist; zero when the row has no energy: an inactive
+//              client)
 //   appearance m = 0..N-1:       beta_V / N * softmax_i(cos_mi / tau_v)
 //   spatial    l = 0..L*L-1:     beta_S / L^2 * softmax_i(-||p_i - l_l||^2 / tau_s)
 // with p_i = ((r+.5)/gh, (c+.5)/gw) and landmarks ((a+.5)/L, (b+.5)/L).
@@ -60,17 +63,16 @@ __device__ __forceinline__ void row_softmax_stats(const float* row, int N, float
 }
 
 __global__ void __launch_bounds__(256, 4) k_build_clients(
-    const float* __restrict__ A, const float* __restrict__ rs, int nRS, const float* __restrict__ zn2,
-    const float* __restrict__ sigma, const float* __restrict__ omega,
+    const ViewRows vw, int nRS, const float* __restrict__ omega,
     const float* __restrict__ cos, const int32_t* toff, int B, int N, int Tmax, int H, int M,
-    int gh, int gw, int L, float beta_G, float beta_V, float beta_S, float tau_v, float tau_s,
+    int gh, int gw, int L, float beta_V, float beta_S, float tau_v, float tau_s,
     float wq, float fx_scale, int check, float* C, long long* u0, uint32_t* status) {
   grid_dep_wait();
   __shared__ RowInfo ri[ROWS_PER_BLOCK];
   const int b = blockIdx.y;
   const TextGeom tg = text_geom(toff, b, B, Tmax, status);
   if (tg.T == 0) return;
-  const int Tb = tg.T, MG = H * Tb, Mb = MG + N + L * L;
+  const int Tb = tg.T, MG = vw.n * H * Tb, Mb = MG + N + L * L;
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const int r0 = blockIdx.x * ROWS_PER_BLOCK;
   if (r0 >= Mb) return;
@@ -78,15 +80,16 @@ __global__ void __launch_bounds__(256, 4) k_build_clients(
     const int m = r0 + w;
     RowInfo inf{-1, nullptr, nullptr, 0.f, 0.f, 0.f, 0.f, 0.f};
     if (m < MG) {
-      const int h = m / Tb, t = m % Tb;
+      const int v = m / (H * Tb), hm = m - v * H * Tb;  // view, then (h, t) h-major
+      const int h = hm / Tb, t = hm % Tb;
       float rsv = 0.f;  // parts over key splits, fixed order
-      for (int q = 0; q < nRS; ++q) rsv += rs[(((size_t)b * H + h) * nRS + q) * Tmax + t];
+      for (int q = 0; q < nRS; ++q) rsv += vw.rs[v][(((size_t)b * H + h) * nRS + q) * Tmax + t];
       const float nu = (t == Tb - 1 ? wq : 1.f) / ((float)(Tb - 1) + wq);
-      const float sg = sigma[(size_t)b * H + h];
+      const float sg = vw.sigma[v][(size_t)b * H + h];
       inf.kind = 0;
-      inf.x = A + (((size_t)b * H + h) * Tmax + t) * N;
-      inf.z = zn2 + ((size_t)b * H + h) * N;
-      inf.scale = rsv > 0.f ? beta_G * omega[(size_t)b * H + h] * nu / rsv : 0.f;
+      inf.x = vw.A[v] + (((size_t)b * H + h) * Tmax + t) * N;
+      inf.z = vw.zn2[v] + ((size_t)b * H + h) * N;
+      inf.scale = rsv > 0.f ? vw.beta[v] * omega[(size_t)b * H + h] * nu / rsv : 0.f;
       inf.sg2 = sg * sg;
     } else if (m < MG + N) {
       const int a = m - MG;
@@ -169,11 +172,11 @@ __global__ void __launch_bounds__(256, 4) k_build_clients(
 }
 
 cudaError_t launch_build_clients(const Dims& dm, const gmc_params& p, int fx_exp, Scratch& s,
-                                 cudaStream_t st) {
+                                 const ViewRows& views, cudaStream_t st) {
   dim3 grid(ceil_div(dm.M, ROWS_PER_BLOCK), dm.B);
   launch_k(k_build_clients, grid, 32 * ROWS_PER_BLOCK, 0, st, 1,
-      s.A, s.rs, s.nRS, s.zn2, s.sigma, s.omega, s.cos, dm.toff, dm.B, dm.N, dm.T, dm.H, dm.M, dm.gh,
-      dm.gw, dm.L, p.beta_G, p.beta_V, p.beta_S, p.tau_v, p.tau_s, p.terminal_q_weight,
+      views, s.nRS, s.omega, s.cos, dm.toff, dm.B, dm.N, dm.T, dm.H, dm.M, dm.gh,
+      dm.gw, dm.L, p.beta_V, p.beta_S, p.tau_v, p.tau_s, p.terminal_q_weight,
       ldexpf(1.f, fx_exp), p.check_mode, s.C, s.u0, s.status);
   return cudaGetLastError();
 }

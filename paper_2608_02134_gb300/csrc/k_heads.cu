@@ -201,7 +201,8 @@ __device__ __forceinline__ void warp_argbest(float& v, int& idx, bool want_max) 
 // fp32 rounding of a cosine.  One block of 256 threads, one warp for the
 // centres (two heads per lane, H <= 64).
 __device__ void cluster_heads(const double* hgb, int b, int T, int N, int H, int max_clusters,
-                              float head_eps, float* omega, const TraceView& tv, float* sm) {
+                              float head_eps, float* omega, const TraceView& tv, float* sm,
+                              const ViewGrams& vg) {
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
   float* cs = sm;                       // [H*H] pattern cosines
   float* pre = cs + H * H;              // [H]   pattern norm / mean atom norm
@@ -212,18 +213,48 @@ __device__ void cluster_heads(const double* hgb, int b, int T, int N, int H, int
   int* asg = reinterpret_cast<int*>(isum + GMC_MAX_HEADS);  // [H] cluster of every head
   int* cent = asg + H;                  // [GMC_MAX_HEADS] centres
   int* ccnt = cent + GMC_MAX_HEADS;     // [GMC_MAX_HEADS] cluster sizes
-  for (int h = threadIdx.x; h < H; h += blockDim.x) {
-    const float a = (float)__ldcg(&hgb[h * H + h]);
-    const float mean = (float)__ldcg(&hgb[H * H + h]) / ((float)T * (float)N);  // sum_t rs / (T N)
-    pre[h] = (mean > 0.f && a > 0.f) ? sqrtf(a) / mean : 0.f;
-    dot[h] = a > 0.f ? 1.f / sqrtf(a) : 0.f;  // 1 / ||U_h||, 0 for a zero pattern
+  const float TN = (float)T * (float)N;
+  if (vg.n > 1) {
+    // patterns over the views (Eq. (cond-head-pattern)): with U_h^v the view's
+    // atoms over their mean norm m_v[h] = sum_t rs_v[h,t] / (T N),
+    // <u_h, u_g> = sum_v beta_v G_v[h][g] / (m_v[h] m_v[g])
+    const int HE = H * H + H;
+    for (int h = threadIdx.x; h < H; h += blockDim.x) {
+      float a = 0.f;
+      for (int v = 0; v < vg.n; ++v) {
+        const double* hv = vg.HG[v] + (size_t)b * HE;
+        const float m = (float)__ldcg(&hv[H * H + h]) / TN;
+        if (m > 0.f) a += vg.beta[v] * (float)__ldcg(&hv[h * H + h]) / (m * m);
+      }
+      pre[h] = a > 0.f ? sqrtf(a) : 0.f;
+      dot[h] = a > 0.f ? 1.f / sqrtf(a) : 0.f;
+    }
+    __syncthreads();
+    for (int p = threadIdx.x; p < H * H; p += blockDim.x) {
+      const int h = p / H, g = p % H;
+      float x = 0.f;
+      for (int v = 0; v < vg.n; ++v) {
+        const double* hv = vg.HG[v] + (size_t)b * HE;
+        const float mh = (float)__ldcg(&hv[H * H + h]) / TN, mg = (float)__ldcg(&hv[H * H + g]) / TN;
+        if (mh > 0.f && mg > 0.f) x += vg.beta[v] * (float)__ldcg(&hv[p]) / (mh * mg);
+      }
+      cs[p] = x * dot[h] * dot[g];
+    }
+    __syncthreads();
+  } else {
+    for (int h = threadIdx.x; h < H; h += blockDim.x) {
+      const float a = (float)__ldcg(&hgb[h * H + h]);
+      const float mean = (float)__ldcg(&hgb[H * H + h]) / TN;  // sum_t rs / (T N)
+      pre[h] = (mean > 0.f && a > 0.f) ? sqrtf(a) / mean : 0.f;
+      dot[h] = a > 0.f ? 1.f / sqrtf(a) : 0.f;  // 1 / ||U_h||, 0 for a zero pattern
+    }
+    __syncthreads();
+    for (int p = threadIdx.x; p < H * H; p += blockDim.x) {
+      const int h = p / H, g = p % H;
+      cs[p] = (float)__ldcg(&hgb[p]) * dot[h] * dot[g];
+    }
+    __syncthreads();
   }
-  __syncthreads();
-  for (int p = threadIdx.x; p < H * H; p += blockDim.x) {
-    const int h = p / H, g = p % H;
-    cs[p] = (float)__ldcg(&hgb[p]) * dot[h] * dot[g];
-  }
-  __syncthreads();
   const int nc = min(max_clusters, H);
   if (wid == 0) {  // farthest-first centres, two heads per lane (H <= 64)
     const int h0 = lane, h1 = lane + 32;
@@ -334,6 +365,7 @@ __global__ void __launch_bounds__(256) k_hg_reduce(const double* __restrict__ hg
                                                      const int32_t* toff, int Tmax, double* HG,
                                                      uint32_t* tick, int max_clusters,
                                                      float head_eps, float* omega, TraceView tv,
+                                                     int cluster, const ViewGrams vg,
                                                      uint32_t* status) {
   grid_dep_wait();
   extern __shared__ float sm_hc[];
@@ -360,9 +392,9 @@ __global__ void __launch_bounds__(256) k_hg_reduce(const double* __restrict__ hg
   __syncthreads();
   if (threadIdx.x == 0) last = atomicAdd(&tick[b], 1u) == gridDim.x - 1;
   __syncthreads();
-  if (!last) return;
+  if (!last || !cluster) return;  // a historical view's Gram waits for the current view's call
   __threadfence();
-  cluster_heads(HG + (size_t)b * HE, b, tg.T, N, H, max_clusters, head_eps, omega, tv, sm_hc);
+  cluster_heads(HG + (size_t)b * HE, b, tg.T, N, H, max_clusters, head_eps, omega, tv, sm_hc, vg);
 }
 
 // Dynamic shared memory of k_head_stats for H heads: both staged query
@@ -381,7 +413,7 @@ static size_t head_stats_smem(int H) {
 bool heads_supported(int H) { return H >= 1 && head_stats_smem(H) <= 227 * 1024; }
 
 cudaError_t launch_heads(const Dims& dm, const gmc_params& p, Scratch& s, const TraceView& tv,
-                         cudaStream_t st) {
+                         cudaStream_t st, int cluster, const ViewGrams* views) {
   const int H = dm.H;
   const size_t smem = head_stats_smem(H);
   cudaError_t e = set_smem_limit((const void*)k_head_stats, smem);
@@ -395,7 +427,8 @@ cudaError_t launch_heads(const Dims& dm, const gmc_params& p, Scratch& s, const 
   if ((e = set_smem_limit((const void*)k_hg_reduce, smem2)) != cudaSuccess) return e;
   launch_k(k_hg_reduce, dim3(ceil_div(H * H + H, 8), dm.B), 256, smem2, st, 1,
            (const double*)s.hgpart, s.nHG, dm.B, dm.N, H, (const float*)s.rs, s.nRS, dm.toff, dm.T,
-           s.HG, s.tick3, p.max_head_clusters, p.head_eps, s.omega, tv, s.status);
+           s.HG, s.tick3, p.max_head_clusters, p.head_eps, s.omega, tv, cluster,
+           views ? *views : ViewGrams{}, s.status);
   return cudaGetLastError();
 }
 

@@ -12,9 +12,12 @@
 namespace gmc {
 
 // Shapes of one call; every per-image buffer is strided by T (= T_max).
+constexpr int MAX_VIEWS = 4;  // message views: the current one and up to 3 historical ones
+
 struct Dims {
   int B, N, T, H, Hkv, d, D, K, gh, gw, L;  // L = landmarks per side
-  int M;                                    // H*T + N + L*L: client rows per image (max)
+  int V;                                    // message views (1: the current view only)
+  int M;                                    // V*H*T + N + L*L: client rows per image (max)
   int dtype;                                // GMC_F32 / GMC_BF16
   const int32_t* toff;                      // device text offsets or nullptr
 };
@@ -32,6 +35,26 @@ struct TraceView {
   template <typename T> __device__ __forceinline__ T* at(int b, size_t off) const {
     return reinterpret_cast<T*>(rec(b) + off);
   }
+};
+
+// The grounded rows' inputs of every message view (view 0 = current), by value
+// to the client builder: row (v, h, t) of image b is
+// beta[v] * omega_h * nu_t * ||u_i^{v,h,t}|| / sum_j ||u_j^{v,h,t}||.
+struct ViewRows {
+  int n;
+  const float* A[MAX_VIEWS];
+  const float* rs[MAX_VIEWS];
+  const float* zn2[MAX_VIEWS];
+  const float* sigma[MAX_VIEWS];
+  float beta[MAX_VIEWS];
+};
+
+// The head-pattern Grams of every view for the clustering (view 0 = current):
+// HG[v] holds [B][H*H + H] (Gram, then sum_t rs[h,t] per head).
+struct ViewGrams {
+  int n;
+  const double* HG[MAX_VIEWS];
+  float beta[MAX_VIEWS];
 };
 
 // Device scratch carved out of the caller's workspace.
@@ -72,6 +95,18 @@ struct Scratch {
   int32_t* fexp;     // [B]            select-path fixed-point exponents
   __nv_bfloat16* Qp; // [B][Hkv][RQ][d] packed text queries of each KV group (tcgen05 path)
   int nP, nHG, nA, nSel, nE, nRS;
+  // Message views: A, rs, mpart, Z, zn2, sigpart, sigma, hgpart, HG, W2, Qp, the
+  // probe tickets (tick) and the head-Gram tickets (tick3) hold V consecutive
+  // per-view blocks; the pointers above address view 0 (the current view).
+  int V, B;
+  size_t vA, vrs, vmp, vZ, vzn, vsp, vsg, vhp, vHG, vW2, vQp;  // elements per view
+  Scratch view(int v) const {
+    Scratch t = *this;
+    t.A += v * vA; t.rs += v * vrs; t.mpart += v * vmp; t.Z += v * vZ; t.zn2 += v * vzn;
+    t.sigpart += v * vsp; t.sigma += v * vsg; t.hgpart += v * vhp; t.HG += v * vHG;
+    t.W2 += v * vW2; t.Qp += v * vQp; t.tick += (size_t)v * B; t.tick3 += (size_t)v * B;
+    return t;
+  }
 };
 
 constexpr int ROWS_PER_BLOCK = 8;  // rownorm / probe / client builder blocks
@@ -85,10 +120,12 @@ cudaError_t launch_probe(const Dims&, const void* keys, const float* W, const gm
                          cudaStream_t);
 cudaError_t launch_message(const Dims&, const void* keys, const void* queries, Scratch&,
                            cudaStream_t);
-cudaError_t launch_heads(const Dims&, const gmc_params&, Scratch&, const TraceView&, cudaStream_t);
+cudaError_t launch_heads(const Dims&, const gmc_params&, Scratch&, const TraceView&, cudaStream_t,
+                         int cluster = 1, const ViewGrams* views = nullptr);
 bool heads_supported(int H);  // the head statistics of H heads fit a block (H <= 56)
 cudaError_t launch_gram(const Dims&, const void* hidden, Scratch&, cudaStream_t);
 cudaError_t launch_build_clients(const Dims&, const gmc_params&, int fx_exp, Scratch&,
+                                 const ViewRows& views,
                                  cudaStream_t);
 // State left by the first (dense) selection round, run over the whole GPU.
 // Rounds of the solver run on the whole GPU before the cluster kernel takes

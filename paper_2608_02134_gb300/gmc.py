@@ -27,7 +27,9 @@ EXPORTS = (
     "gmc_transport_workspace_size", "gmc_transport", "gmc_read_status", "gmc_error_string",
     "gmc_version", "gmc_profile_enable", "gmc_profile_read", "gmc_launch_count",
     "gmc_transport_noalloc", "gmc_cosine_workspace_size", "gmc_cosine",
+    "gmc_workspace_size_views", "gmc_compress_views",
 )
+MAX_VIEWS = 4
 
 
 class Params(ctypes.Structure):
@@ -49,6 +51,13 @@ class Params(ctypes.Structure):
 class Problem(ctypes.Structure):
     _fields_ = [("B", ctypes.c_int), ("grid_h", ctypes.c_int), ("grid_w", ctypes.c_int),
                 ("Hkv", ctypes.c_int), ("dtype", ctypes.c_int), ("text_offsets", ctypes.c_void_p)]
+
+
+class Views(ctypes.Structure):
+    _fields_ = [("n", ctypes.c_int), ("beta_hist", ctypes.c_float),
+                ("keys", ctypes.c_void_p * (MAX_VIEWS - 1)),
+                ("queries", ctypes.c_void_p * (MAX_VIEWS - 1)),
+                ("vo_probe", ctypes.c_void_p * (MAX_VIEWS - 1))]
 
 
 class TraceHeader(ctypes.Structure):
@@ -87,6 +96,11 @@ def lib() -> ctypes.CDLL:
     L.gmc_compress.argtypes = [PP, P, vp, vp, vp, vp, vp, i, i, i, i, i, i, vp, vp, vp, vp, vp,
                                sz, vp, vp]
     L.gmc_compress.restype = i
+    L.gmc_workspace_size_views.argtypes = [PP, i, i, i, i, i, i, i]
+    L.gmc_workspace_size_views.restype = sz
+    L.gmc_compress_views.argtypes = [PP, P, ctypes.POINTER(Views), vp, vp, vp, vp, vp, i, i, i, i,
+                                     i, i, vp, vp, vp, vp, vp, sz, vp, vp]
+    L.gmc_compress_views.restype = i
     L.gmc_get_trace_layout.argtypes = [PP, P, i, i, i, i, ctypes.POINTER(TraceLayout)]
     L.gmc_get_trace_layout.restype = i
     L.gmc_trace_size.argtypes = [PP, P, i, i, i, i]
@@ -181,6 +195,31 @@ def compress(prob: Problem, params: Params, hidden, keys, queries, pos_ids, vo_p
         _stream(stream)))
 
 
+def views(keys, queries, vo_probe, beta_hist=0.5) -> Views:
+    """Historical message views from per-view device tensors (keys, queries, probes)."""
+    v = Views()
+    v.n = len(keys)
+    v.beta_hist = beta_hist
+    for k in range(v.n):
+        v.keys[k], v.queries[k], v.vo_probe[k] = _ptr(keys[k]), _ptr(queries[k]), _ptr(vo_probe[k])
+    return v
+
+
+def workspace_size_views(prob: Problem, n_views, N, T, H, d, D, K) -> int:
+    return int(lib().gmc_workspace_size_views(ctypes.byref(prob), n_views, N, T, H, d, D, K))
+
+
+def compress_views(prob: Problem, params: Params, vw: Views, hidden, keys, queries, pos_ids,
+                   vo_probe, N, T, H, d, D, K, out_idx, out_hidden, out_kv, out_pos, workspace,
+                   trace=None, stream=None):
+    """gmc_compress_views on device tensors (see include/gmc.h)."""
+    _check(lib().gmc_compress_views(
+        ctypes.byref(prob), ctypes.byref(params), ctypes.byref(vw), _ptr(hidden), _ptr(keys),
+        _ptr(queries), _ptr(pos_ids), _ptr(vo_probe), N, T, H, d, D, K, _ptr(out_idx),
+        _ptr(out_hidden), _ptr(out_kv), _ptr(out_pos), _ptr(workspace), workspace.numel(),
+        _ptr(trace), _stream(stream)))
+
+
 def select(clients, B, M, N, K, params: Params, out_idx, workspace, trace=None, stream=None):
     _check(lib().gmc_select(_ptr(clients), B, M, N, K, ctypes.byref(params), _ptr(out_idx),
                             _ptr(workspace), workspace.numel(), _ptr(trace), _stream(stream)))
@@ -272,7 +311,7 @@ class Compressor:
     """
 
     def __init__(self, B, grid_h, grid_w, T, H, Hkv, d, D, K, dtype, text_lengths=None,
-                 params: Params | None = None, trace=False, device="cuda"):
+                 params: Params | None = None, trace=False, device="cuda", n_views=0):
         self.B, self.gh, self.gw, self.T, self.H, self.Hkv, self.d, self.D = B, grid_h, grid_w, T, H, Hkv, d, D
         self.N = grid_h * grid_w
         self.Kr = K
@@ -288,7 +327,8 @@ class Compressor:
             off.append(off[-1] + t)
         self.offsets = torch.tensor(off, dtype=torch.int32, device=device) if text_lengths is not None else None
         self.prob = problem(B, grid_h, grid_w, Hkv, dtype, self.offsets)
-        ws = workspace_size(self.prob, self.N, T, H, d, D, K)
+        self.n_views = n_views
+        ws = workspace_size_views(self.prob, n_views, self.N, T, H, d, D, K)
         if ws == 0:
             raise GMCError("invalid problem for gmc_workspace_size")
         self.workspace = alloc_workspace(ws, device)
@@ -304,10 +344,21 @@ class Compressor:
             self.layout = trace_layout(self.prob, self.params, self.N, T, H, K)
             self.trace = torch.zeros(B * self.layout.bytes_per_image, dtype=torch.uint8, device=device)
 
-    def run(self, hidden, keys, queries, pos_ids, vo_probe, stream=None):
-        compress(self.prob, self.params, hidden, keys, queries, pos_ids, vo_probe, self.N, self.T,
-                 self.H, self.d, self.D, self.Kr, self.out_idx, self.out_hidden, self.out_kv,
-                 self.out_pos, self.workspace, self.trace, stream)
+    def run(self, hidden, keys, queries, pos_ids, vo_probe, stream=None, history=None,
+            beta_hist=0.5):
+        """history: None, or (keys, queries, vo_probe) lists of the historical views."""
+        if history is None:
+            compress(self.prob, self.params, hidden, keys, queries, pos_ids, vo_probe, self.N,
+                     self.T, self.H, self.d, self.D, self.Kr, self.out_idx, self.out_hidden,
+                     self.out_kv, self.out_pos, self.workspace, self.trace, stream)
+        else:
+            if len(history[0]) > self.n_views:
+                raise GMCError("more historical views than the workspace was sized for")
+            vw = views(*history, beta_hist=beta_hist)
+            compress_views(self.prob, self.params, vw, hidden, keys, queries, pos_ids, vo_probe,
+                           self.N, self.T, self.H, self.d, self.D, self.Kr, self.out_idx,
+                           self.out_hidden, self.out_kv, self.out_pos, self.workspace, self.trace,
+                           stream)
         return Outputs(self.out_idx, self.out_hidden, self.out_kv, self.out_pos, self.K, self.trace,
                        self.layout)
 

@@ -191,6 +191,18 @@ class Workload:
              / f32(np.sqrt(self.D))).astype(f32)
         return dict(Q=self._round(q), K=self._round(k), V=self._round(val), W=w)
 
+    def history_abi_arrays(self, v: int) -> dict:
+        """Historical view v of every image in the C-ABI layout of gmc_views:
+        keys [B][2][N+T_b][Hkv][d] (K then V), queries [B][T_b][H][d], vo_probe."""
+        kv, q = [], []
+        for b in range(self.B):
+            hv = self.history_view(b, v)
+            kv.append(np.stack([hv["K"], hv["V"]]).reshape(-1))
+            q.append(hv["Q"].reshape(-1))
+        conv = bf16_bits if self.dtype == "bf16" else (lambda a: np.ascontiguousarray(a, np.float32))
+        return dict(keys=conv(np.concatenate(kv)), queries=conv(np.concatenate(q)),
+                    vo_probe=self.history_view(0, v)["W"])
+
     def text_offsets(self) -> np.ndarray:
         return np.concatenate([[0], np.cumsum(self.T)]).astype(np.int32)
 

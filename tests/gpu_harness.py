@@ -23,6 +23,7 @@ class GpuRun:
     pos: np.ndarray
     status: int
     traces: list
+    n_hist: int = 0
 
 
 def to_device(wl: workloads.Workload, device="cuda"):
@@ -38,12 +39,26 @@ def to_device(wl: workloads.Workload, device="cuda"):
     return out
 
 
-def run(wl: workloads.Workload, params=None, trace=True, inputs=None) -> GpuRun:
+def _dev(a, device="cuda"):
+    t = torch.from_numpy(np.ascontiguousarray(a))
+    if a.dtype == np.uint16:
+        t = t.view(torch.int16).view(torch.bfloat16)
+    return t.to(device)
+
+
+def run(wl: workloads.Workload, params=None, trace=True, inputs=None, n_hist=0) -> GpuRun:
     dt = gmc.GMC_BF16 if wl.dtype == "bf16" else gmc.GMC_F32
     inp = inputs or to_device(wl)
     comp = gmc.Compressor(wl.B, wl.gh, wl.gw, wl.T_max, wl.H, wl.Hkv, wl.d, wl.D, wl.K, dt,
-                          text_lengths=wl.T if wl.ragged else None, params=params, trace=trace)
-    out = comp.run(inp["hidden"], inp["keys"], inp["queries"], inp["pos_ids"], inp["vo_probe"])
+                          text_lengths=wl.T if wl.ragged else None, params=params, trace=trace,
+                          n_views=n_hist)
+    history = None
+    if n_hist:
+        hv = [wl.history_abi_arrays(v) for v in range(n_hist)]
+        history = ([_dev(h["keys"]) for h in hv], [_dev(h["queries"]) for h in hv],
+                   [_dev(h["vo_probe"]) for h in hv])
+    out = comp.run(inp["hidden"], inp["keys"], inp["queries"], inp["pos_ids"], inp["vo_probe"],
+                   history=history)
     torch.cuda.synchronize()
     status = comp.status()
     hid = out.hidden.float().cpu().numpy().astype(np.float64)
@@ -54,7 +69,7 @@ def run(wl: workloads.Workload, params=None, trace=True, inputs=None) -> GpuRun:
         traces = parity.parse_trace(out.trace.cpu().numpy(), out.layout, wl.B, comp.K, wl.H, wl.N,
                                     comp.params.max_head_clusters)
     return GpuRun(wl, comp, out.idx.cpu().numpy(), hid, raw, out.kv.float().cpu().numpy(),
-                  out.pos.cpu().numpy(), status, traces)
+                  out.pos.cpu().numpy(), status, traces, n_hist)
 
 
 def oracle_params(p: gmc.Params) -> dict:
@@ -91,8 +106,11 @@ def compare_image(g: GpuRun, b: int, hidden_tol: float) -> ImageReport:
     nc = min(p["max_head_clusters"], H)
     forced = dict(centres=tr.centres[:nc].tolist(), head_assign=tr.head_assign.tolist(),
                   rounds=tr.forced_rounds(), pi=tr.pi)
+    history = None
+    if g.n_hist:
+        history = [{k: f(a) for k, a in wl.history_view(b, v).items()} for v in range(g.n_hist)]
     res = O.compress(f(im.hidden), f(im.keys), f(im.values), f(im.queries), im.pos, f(wl.probe()),
-                     wl.gh, wl.gw, wl.K, p, forced=forced)
+                     wl.gh, wl.gw, wl.K, p, forced=forced, history=history)
     dec = parity.Decisions()
     tag = f"{wl.name}[b={b}]"
     parity.check_heads(res.heads, dec, tag)

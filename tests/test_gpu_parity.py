@@ -127,3 +127,33 @@ def test_deterministic_repeat():
     b = GH.run(wl, inputs=inp)
     assert np.array_equal(a.idx, b.idx)
     assert np.array_equal(a.hidden_raw, b.hidden_raw)
+
+
+def test_history_views_small_bf16():
+    """Two completed historical message views (each with its own queries, keys, values, probe)."""
+    from paper_2608_02134_gb300 import workloads
+    from tests import gpu_harness as GH
+    wl = workloads.make("qwen", gh=12, gw=12, T=20, D=64, H=8, Hkv=2, K=30)
+    _check(GH.run(wl, n_hist=2), [0], TOL_BF16)
+
+
+def test_history_views_tiny_fp32_ragged_batch():
+    from paper_2608_02134_gb300 import workloads
+    from tests import gpu_harness as GH
+    wl = workloads.make("tiny", B=2, T=[8, 5], K=16)
+    _check(GH.run(wl, n_hist=1), [0, 1], TOL_F32)
+
+
+def test_history_views_qwen_shape():
+    """The deployed two-view setting (current view + two completed views) at the Qwen shape."""
+    from paper_2608_02134_gb300 import workloads
+    from tests import gpu_harness as GH
+    wl = workloads.make("qwen")
+    _check(GH.run(wl, n_hist=2), [0], TOL_BF16)
+
+
+def test_history_views_llava_shape():
+    from paper_2608_02134_gb300 import workloads
+    from tests import gpu_harness as GH
+    wl = workloads.make("llava", K=128)
+    _check(GH.run(wl, n_hist=2), [0], TOL_BF16)
