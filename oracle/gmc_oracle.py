@@ -79,10 +79,15 @@ paper, a hand-worked case or brute force on tiny inputs, never by itself):
     the zero-gain fill; a hand-worked responsibility round
     (tests/golden/responsibility_round.txt); trivial supports.
   * assign_population: cosine nearest neighbour when s_x = 0; the gap-gate
-    closed form and Eq. (cond-assignment-bound); one representative.
+    closed form and Eq. (cond-assignment-bound); one representative; a
+    hand-worked case at s_x = 1 - 1/e where the spatial term, its ambiguity
+    gate and the grid coordinates each decide one representative
+    (tests/golden/assignment_spatial_gate.txt).
   * population_weights / transport / rms: positivity, mass and first-moment
     conservation (Eq. (cond-population-moment)), centroid optimality
-    (Eq. (cond-centroid-optimum)), RMS restoration and its bound.
+    (Eq. (cond-centroid-optimum)), RMS restoration and its bound; energies,
+    weights and a two-cluster transport worked by hand at s_x = 1 - 1/e
+    (tests/golden/population_transport.txt).
   * compaction_rows / compress: K = N identity; end-to-end invariants on the
     tiny configuration.
   * view_patterns / client_matrix_views / compress(history=...): the

@@ -470,6 +470,46 @@ def test_assignment_single_representative_and_no_discard():
     assert b.delta_bar == 0.0 and b.s_x == 0.0 and np.all(b.pi == np.arange(9))
 
 
+def test_assignment_spatial_gate_hand_example():
+    """Eq. (cond-assignment) and (cond-population-gate) worked by hand
+    (tests/golden/assignment_spatial_gate.txt): the spatial term, its gate and
+    the grid coordinates each decide one token's representative."""
+    from tests.golden_cases import load_case
+    c = load_case("assignment_spatial_gate.txt")
+    N = c["gh"] * c["gw"]
+    S = np.array(c["S"])
+    cos = np.eye(N)
+    for i, row in c["cos_to_S"].items():
+        cos[int(i), S] = row
+        cos[S, int(i)] = row
+    a = O.assign_population(cos, S, c["gh"], c["gw"], P)
+    assert a.delta_bar == pytest.approx(c["delta_bar"], rel=1e-12)
+    assert a.s_x == pytest.approx(c["s_x"], rel=1e-12)
+    for i, g in c["g"].items():
+        assert a.g[int(i)] == pytest.approx(g, rel=1e-10)
+    for i, kap in c["kappa"].items():
+        assert a.kappa_best[int(i)] == pytest.approx(max(kap), rel=1e-12)
+        assert a.kappa_chosen[int(i)] == pytest.approx(max(kap), rel=1e-12)
+    assert a.pi.tolist() == c["pi"]
+
+
+def test_population_weights_and_transport_hand_example():
+    """Eq. (cond-grounded-energy), (cond-population-gate) and (cond-transport)
+    worked by hand (tests/golden/population_transport.txt) at s_x = 1 - 1/e."""
+    from tests.golden_cases import load_case
+    c = load_case("population_transport.txt")
+    e = np.array(c["energy"])
+    e_o, ebar = O.message_energy(e[None, None, :], np.ones(1), np.ones(1))
+    np.testing.assert_allclose(e_o, e, rtol=1e-15)
+    np.testing.assert_allclose(ebar, c["ebar"], rtol=1e-15)
+    np.testing.assert_allclose(O.population_weights(ebar, c["s_x"], P), c["m"], rtol=1e-14)
+    tr = O.transport(np.array(c["h"]), np.array(c["S"]), np.array(c["pi"]),
+                     np.array(c["m_transport"]), P)
+    np.testing.assert_allclose(tr.mass, c["M"], rtol=1e-15)
+    np.testing.assert_allclose(tr.centroid, c["centroid"], rtol=1e-15, atol=1e-15)
+    np.testing.assert_allclose(tr.restored, c["restored"], rtol=1e-13, atol=1e-15)
+
+
 # --------------------------------------------------------------------------
 # a10 transport: Eq. (5), (cond-population-moment), (cond-centroid-optimum), (cond-rms-bound)
 # --------------------------------------------------------------------------
