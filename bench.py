@@ -159,7 +159,9 @@ def stage_work(wl) -> dict:
     Tm = sum(wl.T) / B
     M = H * Tm + N + 256
     w = {}
-    w["gram"] = ("tensor", B * 2.0 * N * N * D)                        # the N x N cosine block
+    # the cosine Gram: the method needs the symmetric half, 2 * N(N+1)/2 * D
+    # flops (the kernel issues the 128 x 128 tiles on and above the diagonal)
+    w["gram"] = ("tensor", B * 1.0 * N * (N + 1) * D)
     w["message"] = ("hbm", B * (H * Tm * N * 4 + 2 * (N + Tm) * Hkv * d * es + Tm * H * d * es))
     w["clients"] = ("hbm", B * (M * N * 4 + H * Tm * N * 4 + N * N * 4))
     # selection: one read of the M x N clients per round.  Stage "rounds_gpu"

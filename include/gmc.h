@@ -302,9 +302,11 @@ int gmc_transport(const gmc_problem* prob, const gmc_params* params, const void*
  *   - Larger problems (B * N > GMC_NOALLOC_MAX_ROWS) are rejected with
  *     GMC_ERR_UNSUPPORTED before anything is launched.
  *   - It calls no cudaMalloc, cudaFree or other allocating routine.
- *   - The first call made with a given device current looks up the array's
- *     device address (cudaGetSymbolAddress) and caches it; make that first
- *     call before any stream capture that includes this entry point.
+ *   - The first call made in a CUDA context (normally the device's primary
+ *     context) looks up the array's device address (cudaGetSymbolAddress)
+ *     and caches it for that context; make that first call before any
+ *     stream capture that includes this entry point.  After cudaDeviceReset
+ *     the new primary context gets a fresh look-up on its first call.
  *   - All calls share the one array.  Calls that overlap on the GPU (other
  *     streams, other host threads) race on it; serialise them.  The status
  *     word is cleared at the start of every call; the rest is overwritten.
@@ -320,6 +322,38 @@ int gmc_transport_noalloc(const gmc_problem* prob, const gmc_params* params, con
                           const int32_t* assign, const float* weights, int N, int T, int d, int D,
                           int K, int32_t* out_idx, void* out_hidden, void* out_kv,
                           int32_t* out_pos, uint32_t* device_status, gmc_stream_t stream);
+
+/*
+ * gmc_clients -- the client matrix alone (steps 1 of gmc_compress): grounded
+ * message clients (Sec. 3.2, Eq. (1)-(2); appendix Eq. (cond-native-message)
+ * .. (cond-head-weight)), appearance and spatial clients (appendix Eq.
+ * (cond-aux-clients), (cond-coverage)), written to out_clients as
+ * float[B][M][N] with M = (1 + views->n) * H * T + N + landmarks^2.  Image b's
+ * rows: grounded (view, head, text query) view-major then head-major for its
+ * own T_b, then N appearance rows, then landmarks^2 spatial rows; rows past
+ * that (ragged images) are left unspecified.  Arguments, workspace (sized by
+ * gmc_workspace_size / gmc_workspace_size_views) and trace are those of
+ * gmc_compress_views (views may be NULL); the trace receives the head
+ * clustering fields.  The selection, assignment, transport and compaction do
+ * not run.  Returns GMC_OK or a GMC_ERR_* code.
+ */
+int gmc_clients(const gmc_problem* prob, const gmc_params* params, const gmc_views* views,
+                const void* hidden, const void* keys, const void* queries, const int32_t* pos_ids,
+                const float* vo_probe, int N, int T, int H, int d, int D, int K,
+                float* out_clients, void* workspace, size_t ws_bytes, void* trace,
+                gmc_stream_t stream);
+
+/*
+ * gmc_selftest_bounded_wait -- checks the failure path of the bounded device
+ * waits (no counterpart in the paper).  A one-block kernel waits, with the
+ * library's clock-bounded mbarrier wait, on a barrier phase that nothing ever
+ * completes; after `cycles` SM clocks (0 .. 4e9) it sets GMC_STATUS_TIMEOUT
+ * in the status word at the start of `workspace` (256-byte aligned, >= 4
+ * bytes; cleared first) and returns.  The context stays usable.  Read the
+ * bit with gmc_read_status.  Returns GMC_OK, GMC_ERR_ARG or GMC_ERR_CUDA.
+ */
+int gmc_selftest_bounded_wait(long long cycles, void* workspace, size_t ws_bytes,
+                              gmc_stream_t stream);
 
 /*
  * Synchronise `stream`, then copy the device status word of `workspace`

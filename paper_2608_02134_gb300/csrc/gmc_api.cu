@@ -27,23 +27,6 @@ cudaError_t set_smem_limit(const void* func, size_t bytes) {
   return e;
 }
 
-}  // namespace gmc
-
-namespace {
-
-constexpr size_t ALIGN = 256;
-constexpr int MAX_N_BUILD = 8192;
-
-struct Carver {
-  char* base;
-  size_t off = 0;
-  template <typename T> T* take(size_t count) {
-    const size_t at = off;
-    off += (count * sizeof(T) + ALIGN - 1) & ~(ALIGN - 1);
-    return base ? reinterpret_cast<T*>(base + at) : nullptr;
-  }
-};
-
 bool params_ok(const gmc_params& p) {
   return p.batch_b >= 1 && p.pool_mult >= 1 && p.pool_mult * p.batch_b <= GMC_MAX_POOL &&
          p.resp_temp > 0.f && p.resp_eps >= 0.f && p.tau_v > 0.f && p.tau_s > 0.f &&
@@ -55,20 +38,36 @@ bool params_ok(const gmc_params& p) {
          p.rms_eps >= 0.f && p.norm_eps > 0.f && (p.check_mode == 0 || p.check_mode == 1);
 }
 
-int effective_K(int K, int N) { return K < 1 ? 1 : (K > N ? N : K); }
-
-// Shape checks shared by gmc_compress / gmc_transport.
+// Shape checks shared by gmc_compress / gmc_transport / gmc_transport_noalloc.
 int check_problem(const gmc_problem* prob, int N, int T, int d, int D) {
   if (!prob) return GMC_ERR_ARG;
   if (prob->B < 1 || prob->grid_h < 1 || prob->grid_w < 1 || N < 1 ||
       (long long)prob->grid_h * prob->grid_w != N || T < 1 || d < 1 || D < 1 || prob->Hkv < 1)
     return GMC_ERR_ARG;
   if (prob->dtype != GMC_F32 && prob->dtype != GMC_BF16) return GMC_ERR_ARG;
-  if (N > MAX_N_BUILD || D > 8192 || d > 1024) return GMC_ERR_UNSUPPORTED;
+  if (N > GMC_MAX_N || D > 8192 || d > 1024) return GMC_ERR_UNSUPPORTED;
   if (prob->dtype == GMC_BF16 && (d % 8 != 0 || D % 8 != 0)) return GMC_ERR_UNSUPPORTED;
   if (prob->dtype == GMC_F32 && (d % 4 != 0 || D % 8 != 0)) return GMC_ERR_UNSUPPORTED;
   return GMC_OK;
 }
+
+}  // namespace gmc
+
+namespace {
+
+constexpr size_t ALIGN = 256;
+
+struct Carver {
+  char* base;
+  size_t off = 0;
+  template <typename T> T* take(size_t count) {
+    const size_t at = off;
+    off += (count * sizeof(T) + ALIGN - 1) & ~(ALIGN - 1);
+    return base ? reinterpret_cast<T*>(base + at) : nullptr;
+  }
+};
+
+int effective_K(int K, int N) { return K < 1 ? 1 : (K > N ? N : K); }
 
 bool aligned(const void* p, size_t a) { return ((uintptr_t)p % a) == 0; }
 
@@ -372,12 +371,15 @@ size_t gmc_trace_size(const gmc_problem* prob, const gmc_params* params, int N, 
   return (size_t)prob->B * L.bytes_per_image;
 }
 
+// The whole step, or (out_clients != nullptr) its steps up to the client
+// matrix, copied into out_clients.
 static int compress_impl(const gmc_problem* prob, const gmc_params* params,
                          const gmc_views* views, const void* hidden, const void* keys,
                          const void* queries, const int32_t* pos_ids, const float* vo_probe,
                          int N, int T, int H, int d, int D, int K, int32_t* out_idx,
                          void* out_hidden, void* out_kv, int32_t* out_pos, void* workspace,
-                         size_t ws_bytes, void* trace, gmc_stream_t stream_) {
+                         size_t ws_bytes, void* trace, gmc_stream_t stream_,
+                         float* out_clients = nullptr) {
   int rc = check_problem(prob, N, T, d, D);
   if (rc != GMC_OK) return rc;
   if (H < 1 || H % prob->Hkv != 0) return GMC_ERR_ARG;
@@ -385,9 +387,10 @@ static int compress_impl(const gmc_problem* prob, const gmc_params* params,
   gmc_params p;
   if (params) p = *params; else gmc_default_params(&p);
   if (!params_ok(p)) return GMC_ERR_ARG;
-  if (!hidden || !keys || !queries || !pos_ids || !vo_probe || !out_idx || !out_hidden ||
-      !out_kv || !out_pos || !workspace)
+  if (!hidden || !keys || !queries || !pos_ids || !vo_probe || !workspace ||
+      (!out_clients && (!out_idx || !out_hidden || !out_kv || !out_pos)))
     return GMC_ERR_ARG;
+  if (out_clients && !aligned(out_clients, 16)) return GMC_ERR_ARG;
   if (!aligned(hidden, 16) || !aligned(keys, 16) || !aligned(queries, 16) ||
       !aligned(vo_probe, 16) || !aligned(out_hidden, 16) || !aligned(out_kv, 16) ||
       !aligned(workspace, ALIGN) || (trace && !aligned(trace, 16)))
@@ -427,7 +430,7 @@ static int compress_impl(const gmc_problem* prob, const gmc_params* params,
   std::lock_guard<std::mutex> lk(g_prof.mu);
   // status, tickets, membership bitmaps
   GMC_TRY(cudaMemsetAsync(s.status, 0, sizeof(uint32_t) * status_words(dm), st));
-  if (Ke == N) {  // K = N returns the unmodified execution
+  if (Ke == N && !out_clients) {  // K = N returns the unmodified execution
     GMC_TRY(launch_identity(dm, hidden, keys, pos_ids, out_idx, out_hidden, out_kv, out_pos,
                             s.status, st));
     g_launches += 1;
@@ -497,6 +500,11 @@ static int compress_impl(const gmc_problem* prob, const gmc_params* params,
   // every view's grounded rows count as head rows of the client layout
   const int HV = H * V;
   GMC_STAGE("clients", 1, launch_build_clients(dm, p, fx, s, vr, st));
+  if (out_clients) {  // staged call: the client matrix, before selection compacts it in place
+    GMC_TRY(cudaMemcpyAsync(out_clients, s.C, sizeof(float) * dm.B * (size_t)dm.M * N,
+                            cudaMemcpyDeviceToDevice, st));
+    return GMC_OK;
+  }
   GMC_STAGE("rounds_gpu", 3 + 3 * SPARSE_GPU_ROUNDS,
             launch_round0(r0, dm.B, N, Ke, dm.M, dm.toff, HV, T, p.landmarks * p.landmarks, p, fx,
                           nullptr, s.C, s.scol, s.u0, s.order, s.status, tv, st));
@@ -533,6 +541,17 @@ int gmc_compress_views(const gmc_problem* prob, const gmc_params* params, const 
                        stream_);
 }
 
+int gmc_clients(const gmc_problem* prob, const gmc_params* params, const gmc_views* views,
+                const void* hidden, const void* keys, const void* queries, const int32_t* pos_ids,
+                const float* vo_probe, int N, int T, int H, int d, int D, int K,
+                float* out_clients, void* workspace, size_t ws_bytes, void* trace,
+                gmc_stream_t stream_) {
+  if (!out_clients) return GMC_ERR_ARG;
+  return compress_impl(prob, params, views, hidden, keys, queries, pos_ids, vo_probe, N, T, H, d,
+                       D, K, nullptr, nullptr, nullptr, nullptr, workspace, ws_bytes, trace,
+                       stream_, out_clients);
+}
+
 // ---------------------------------------------------------------------------
 // gmc_select
 // ---------------------------------------------------------------------------
@@ -558,7 +577,7 @@ static size_t carve_select(int B, int M, int N, int K, Scratch* s, char* base,
 
 size_t gmc_select_workspace_size(int B, int M, int N, int K, const gmc_params* params) {
   (void)params;
-  if (B < 1 || M < 1 || N < 1 || N > MAX_N_BUILD || K < 1 || K > N) return 0;
+  if (B < 1 || M < 1 || N < 1 || N > GMC_MAX_N || K < 1 || K > N) return 0;
   return carve_select(B, M, N, K, nullptr, nullptr);
 }
 
@@ -567,7 +586,7 @@ int gmc_select(const float* clients, int B, int M, int N, int K, const gmc_param
                gmc_stream_t stream_) {
   if (!clients || !out_idx || !workspace || B < 1 || M < 1 || N < 1 || K < 1 || K > N)
     return GMC_ERR_ARG;
-  if (N > MAX_N_BUILD) return GMC_ERR_UNSUPPORTED;
+  if (N > GMC_MAX_N) return GMC_ERR_UNSUPPORTED;
   if (!aligned(workspace, ALIGN) || (trace && !aligned(trace, 16))) return GMC_ERR_ARG;
   gmc_params p;
   if (params) p = *params; else gmc_default_params(&p);

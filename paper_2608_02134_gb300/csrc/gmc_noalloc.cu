@@ -13,8 +13,13 @@
 // The array is a file-scope __device__ variable, so every GPU that loads
 // libgmc.so holds it (GMC_NOALLOC_MAX_ROWS floats + 256 bytes) until the
 // process exits.  In host code its name is only a host-side stand-in; the
-// device address is fetched with cudaGetSymbolAddress once per device (on
-// the first call made with that device current) and cached.
+// device address is fetched with cudaGetSymbolAddress on the first call made
+// in a given CUDA context (the device's primary context, or whichever
+// context is current) and cached for that context.  A context that replaces
+// it -- for example the new primary context after cudaDeviceReset -- gets
+// its own look-up on its first call.
+#include <cuda.h>  // CUcontext: the cache key (the driver entry point is found at run time)
+
 #include <mutex>
 
 #include "common.cuh"
@@ -31,22 +36,55 @@ static __device__ __align__(256) unsigned char
 
 constexpr int kMaxDevices = 256;
 std::mutex g_setup_mu;
-void* g_scratch_addr[kMaxDevices] = {};
+struct CachedAddress {
+  CUcontext ctx;  // context the address belongs to
+  void* addr;
+};
+CachedAddress g_scratch_addr[kMaxDevices] = {};
 
-// Device address of the scratch array on the current device.
+using CtxGetCurrentFn = CUresult (*)(CUcontext*);
+
+// cuCtxGetCurrent through the runtime's driver entry point table (the
+// library does not link libcuda directly).  nullptr if unavailable.
+CtxGetCurrentFn ctx_get_current() {
+  static CtxGetCurrentFn fn = [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) !=
+            cudaSuccess ||
+        q != cudaDriverEntryPointSuccess) {
+      cudaGetLastError();
+      return (CtxGetCurrentFn) nullptr;
+    }
+    return reinterpret_cast<CtxGetCurrentFn>(p);
+  }();
+  return fn;
+}
+
+// Device address of the scratch array in the current context: looked up by
+// the first call in a context (cudaGetSymbolAddress also creates the device's
+// primary context if none is current yet), reused while that context stays
+// current.  Without the driver entry point every call looks it up.
 cudaError_t scratch_address(void** out) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
   std::lock_guard<std::mutex> lk(g_setup_mu);
-  if (!g_scratch_addr[dev]) {
+  CUcontext ctx = nullptr;
+  const CtxGetCurrentFn get = ctx_get_current();
+  const bool known = get && get(&ctx) == CUDA_SUCCESS && ctx != nullptr;
+  CachedAddress& c = g_scratch_addr[dev];
+  if (!known || !c.addr || c.ctx != ctx) {
     void* p = nullptr;
     e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
     if (e != cudaSuccess) return e;
-    g_scratch_addr[dev] = p;
+    // the look-up made the device's primary context current if none was
+    if (get && !known && get(&ctx) != CUDA_SUCCESS) ctx = nullptr;
+    c.addr = p;
+    c.ctx = ctx;
   }
-  *out = g_scratch_addr[dev];
+  *out = c.addr;
   return cudaSuccess;
 }
 
@@ -61,17 +99,14 @@ extern "C" int gmc_transport_noalloc(const gmc_problem* prob, const gmc_params* 
                                      int d, int D, int K, int32_t* out_idx, void* out_hidden,
                                      void* out_kv, int32_t* out_pos, uint32_t* device_status,
                                      gmc_stream_t stream_) {
-  if (!prob || prob->B < 1 || prob->grid_h < 1 || prob->grid_w < 1 || prob->Hkv < 1 || N < 1 ||
-      (long long)prob->grid_h * prob->grid_w != N || T < 1 || d < 1 || D < 1 || K < 1 || K > N)
-    return GMC_ERR_ARG;
-  if (prob->dtype != GMC_F32 && prob->dtype != GMC_BF16) return GMC_ERR_ARG;
+  // the checks of gmc_transport, plus the size of the fixed scratch
+  const int rc = check_problem(prob, N, T, d, D);
+  if (rc != GMC_OK) return rc;
+  if (K < 1 || K > N) return GMC_ERR_ARG;
   if ((long long)prob->B * N > GMC_NOALLOC_MAX_ROWS) return GMC_ERR_UNSUPPORTED;
-  if (N > GMC_MAX_N || D > 8192 || d > 1024 || D % 8 != 0 ||
-      d % (prob->dtype == GMC_BF16 ? 8 : 4) != 0)
-    return GMC_ERR_UNSUPPORTED;
   gmc_params p;
   if (params) p = *params; else gmc_default_params(&p);
-  if (!(p.rms_eps >= 0.f)) return GMC_ERR_ARG;
+  if (!params_ok(p)) return GMC_ERR_ARG;
   if (!hidden || !keys || !pos_ids || !support || !assign || !weights || !out_idx ||
       !out_hidden || !out_kv || !out_pos)
     return GMC_ERR_ARG;

@@ -170,6 +170,10 @@ __global__ void k_assign_pick(const float* __restrict__ cos, const int32_t* __re
       const int ok = __shfl_xor_sync(FULL, bk, o);
       if (ob > best || (ob == best && ok < bk)) { best = ob; bk = ok; }
     }
+    if (bk >= K) {  // no comparable value (non-finite cosines): the first carrier
+      bk = 0;
+      if (lane == 0) set_status(status, GMC_STATUS_NONFINITE);
+    }
     choice = S[bk];
   }
   if (lane == 0) {

@@ -14,7 +14,7 @@
 //   k_rg_pool   the pool of the current gains among the unselected tokens;
 //   k_rg_rho    warp per row: the row's pool entries are found through a
 //               token -> pool slot table; pool tokens without a survivor in
-//               the row have R = 0 and count exp(0) = 1 in its denominator;
+//               the row have R = 0 and still count in its softmax denominator;
 //   k_rg_filter warp per row: batch, coverage over the batch's entries, the
 //               survivors compacted in place, the next gains.
 // While many survivors remain, a whole-GPU round is cheaper than a round of
@@ -104,18 +104,21 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_rho(
     rmax = warp_max(rmax);
     npool = warp_sum_int(npool);
     if (npool > 0) {
+      // softmax of R / tau shifted by its largest logit rmax / tau: every
+      // exponential is at most 1, whatever resp_temp
       const float tau = resp_temp * rmax + resp_eps;
+      const float e0 = expf(-rmax / tau);  // a pool token with R = 0
       float z = 0.f;
 #pragma unroll
       for (int u = 0; u < GMC_MAX_POOL / 32; ++u)
-        if (Rd[u] > 0.f) z += expf(Rd[u] / tau);
-      z = warp_sum(z) + (float)(Pt - npool);
+        if (Rd[u] > 0.f) z += expf((Rd[u] - rmax) / tau);
+      z = warp_sum(z) + (float)(Pt - npool) * e0;
       const float invz = 1.f / z;
 #pragma unroll
       for (int u = 0; u < GMC_MAX_POOL / 32; ++u)
         if (Rd[u] > 0.f)
           atomicAdd((unsigned long long*)&sblk[lane + 32 * u],
-                    (unsigned long long)to_fix(expf(Rd[u] / tau) * invz * Rd[u], fxs));
+                    (unsigned long long)to_fix(expf((Rd[u] - rmax) / tau) * invz * Rd[u], fxs));
     }
   }
   __syncthreads();
@@ -375,15 +378,17 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_rg_rho(
     rmax = warp_max(rmax);
     __syncwarp();
     if (nf > 0) {
+      // softmax shifted by the largest logit (exponentials at most 1)
       const float tau = resp_temp * rmax + resp_eps;
+      const float e0 = expf(-rmax / tau);  // pool tokens without a survivor here: R = 0
       float z = 0.f;
-      for (int q = lane; q < nf; q += 32) z += expf(fres[w][q] / tau);
-      z = warp_sum(z) + (float)(Pt - nf);  // pool tokens without a survivor here: exp(0)
+      for (int q = lane; q < nf; q += 32) z += expf((fres[w][q] - rmax) / tau);
+      z = warp_sum(z) + (float)(Pt - nf) * e0;
       const float invz = 1.f / z;
       for (int q = lane; q < nf; q += 32) {
         const float R = fres[w][q];
         atomicAdd((unsigned long long*)&sblk[fslot[w][q]],
-                  (unsigned long long)to_fix(expf(R / tau) * invz * R, fxs));
+                  (unsigned long long)to_fix(expf((R - rmax) / tau) * invz * R, fxs));
       }
     }
   }

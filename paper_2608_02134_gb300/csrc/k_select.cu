@@ -14,8 +14,9 @@
 // each client row keeps only its "survivors" {i : Cbar_mi > b_m}, compacted in
 // place, and later rounds touch only those.  This is exact, not an
 // approximation: the skipped entries are exactly the zero residuals.  (A pool
-// member with R_mi = 0 still counts exp(0) = 1 in row m's softmax
-// denominator; the kernel adds those terms explicitly.)  Survivor lists start
+// member with R_mi = 0 still counts in row m's softmax denominator; the
+// kernel adds those terms explicitly.  Every softmax is shifted by its row's
+// largest logit, so no exponential exceeds 1 for any temperature.)  Survivor lists start
 // in global memory (in place over Cbar, row-major, processed by 8-lane groups)
 // and move into the CTA's shared memory as soon as they all fit there, sorted
 // by token ("flat mode"): then the responsibilities and the coverage update
@@ -484,15 +485,17 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
         }
       }
       __syncthreads();
-      // softmax denominators, exact in 2^-40
+      // softmax denominators shifted by the row's largest logit (every term at
+      // most 1, so at most 2^40 * pool size), exact in 2^-40
       for (int k = gid; k < Pt; k += ngrp) {
         const int j = s.pool[k];
         for (int p = s.cstart[j] + gl; p < s.cstart[j + 1]; p += G) {
           const int q = s.srows[p];
           if (q == DEADROW) continue;
-          const float tau = a.resp_temp * __int_as_float(s.rmaxb[q]) + a.resp_eps;
-          atomicAdd(&s.z64[q],
-                    (unsigned long long)to_fix(expf((s.svals[p] - s.bcov[q]) / tau), z_one));
+          const float rmax = __int_as_float(s.rmaxb[q]);
+          const float tau = a.resp_temp * rmax + a.resp_eps;
+          atomicAdd(&s.z64[q], (unsigned long long)to_fix(
+                                   expf(((s.svals[p] - s.bcov[q]) - rmax) / tau), z_one));
         }
       }
       __syncthreads();
@@ -503,10 +506,13 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
         for (int p = s.cstart[j] + gl; p < s.cstart[j + 1]; p += G) {
           const int q = s.srows[p];
           if (q == DEADROW) continue;
-          const float tau = a.resp_temp * __int_as_float(s.rmaxb[q]) + a.resp_eps;
-          const float z = fix_to_float(s.z64[q]) * z_inv + (float)(Pt - s.npl[q]);
+          const float rmax = __int_as_float(s.rmaxb[q]);
+          const float tau = a.resp_temp * rmax + a.resp_eps;
+          // pool tokens without an entry in row q have R = 0
+          const float z =
+              fix_to_float(s.z64[q]) * z_inv + (float)(Pt - s.npl[q]) * expf(-rmax / tau);
           const float R = s.svals[p] - s.bcov[q];
-          acc += (unsigned long long)to_fix(expf(R / tau) / z * R, fxs);
+          acc += (unsigned long long)to_fix(expf((R - rmax) / tau) / z * R, fxs);
         }
 #pragma unroll
         for (int o = G / 2; o > 0; o >>= 1) acc += __shfl_xor_sync(gm, acc, o);
@@ -558,17 +564,18 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
       const bool any_spill = __any_sync(gm, spill);
       ncache = mine < PCL ? mine : PCL;
       if (npool > 0) {
+        // softmax shifted by the row's largest logit (exponentials at most 1)
         const float tau = a.resp_temp * rmax + a.resp_eps;
         float z = 0.f;
         if (!any_spill) {
 #pragma unroll
           for (int t = 0; t < PCL; ++t)
-            if (t < ncache) z += expf((cv[t] - bm) / tau);
+            if (t < ncache) z += expf(((cv[t] - bm) - rmax) / tau);
         } else {
           for (int k = gl; k < n; k += G)
-            if (s.poolslot[cols[k]] >= 0) z += expf((vals[k] - bm) / tau);
+            if (s.poolslot[cols[k]] >= 0) z += expf(((vals[k] - bm) - rmax) / tau);
         }
-        z = group_sum(z, gm) + (float)(Pt - npool);
+        z = group_sum(z, gm) + (float)(Pt - npool) * expf(-rmax / tau);  // R = 0 entries
         const float invz = 1.f / z;
         if (!any_spill) {
 #pragma unroll
@@ -576,7 +583,7 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
             if (t < ncache) {
               const float R = cv[t] - bm;
               atomicAdd(&s.sw[wid * Pt + cs[t]],
-                        (unsigned long long)to_fix(expf(R / tau) * invz * R, fxs));
+                        (unsigned long long)to_fix(expf((R - rmax) / tau) * invz * R, fxs));
             }
         } else {
           for (int k = gl; k < n; k += G) {
@@ -584,7 +591,7 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
             if (ps >= 0) {
               const float R = vals[k] - bm;
               atomicAdd(&s.sw[wid * Pt + ps],
-                        (unsigned long long)to_fix(expf(R / tau) * invz * R, fxs));
+                        (unsigned long long)to_fix(expf((R - rmax) / tau) * invz * R, fxs));
             }
           }
         }

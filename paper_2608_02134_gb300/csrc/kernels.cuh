@@ -190,6 +190,14 @@ struct SeqIdx {
 }  // namespace gmc
 
 namespace gmc {
+// Argument checks shared by the entry points (gmc_api.cu): every parameter in
+// its documented range; the problem's shape within this build's limits
+// (GMC_OK, GMC_ERR_ARG or GMC_ERR_UNSUPPORTED).
+bool params_ok(const gmc_params& p);
+int check_problem(const gmc_problem* prob, int N, int T, int d, int D);
+}  // namespace gmc
+
+namespace gmc {
 // Raise a kernel's dynamic shared-memory limit when a launch needs more than
 // the 48 KB default (idempotent; remembers the largest value set per kernel).
 cudaError_t set_smem_limit(const void* func, size_t bytes);

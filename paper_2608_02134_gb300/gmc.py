@@ -27,7 +27,7 @@ EXPORTS = (
     "gmc_transport_workspace_size", "gmc_transport", "gmc_read_status", "gmc_error_string",
     "gmc_version", "gmc_profile_enable", "gmc_profile_read", "gmc_launch_count",
     "gmc_transport_noalloc", "gmc_cosine_workspace_size", "gmc_cosine",
-    "gmc_workspace_size_views", "gmc_compress_views",
+    "gmc_workspace_size_views", "gmc_compress_views", "gmc_clients", "gmc_selftest_bounded_wait",
 )
 MAX_VIEWS = 4
 
@@ -133,6 +133,11 @@ def lib() -> ctypes.CDLL:
     L.gmc_cosine_workspace_size.restype = sz
     L.gmc_cosine.argtypes = [PP, P, vp, i, i, i, vp, vp, sz, vp]
     L.gmc_cosine.restype = i
+    L.gmc_clients.argtypes = [PP, P, ctypes.POINTER(Views), vp, vp, vp, vp, vp, i, i, i, i, i, i,
+                              vp, vp, sz, vp, vp]
+    L.gmc_clients.restype = i
+    L.gmc_selftest_bounded_wait.argtypes = [ctypes.c_longlong, vp, sz, vp]
+    L.gmc_selftest_bounded_wait.restype = i
     _lib = L
     return L
 
@@ -218,6 +223,21 @@ def compress_views(prob: Problem, params: Params, vw: Views, hidden, keys, queri
         _ptr(queries), _ptr(pos_ids), _ptr(vo_probe), N, T, H, d, D, K, _ptr(out_idx),
         _ptr(out_hidden), _ptr(out_kv), _ptr(out_pos), _ptr(workspace), workspace.numel(),
         _ptr(trace), _stream(stream)))
+
+
+def clients(prob: Problem, params: Params, vw: Views | None, hidden, keys, queries, pos_ids,
+            vo_probe, N, T, H, d, D, K, out_clients, workspace, trace=None, stream=None):
+    """gmc_clients: the client matrix alone, float[B][M][N] into out_clients (see include/gmc.h)."""
+    _check(lib().gmc_clients(
+        ctypes.byref(prob), ctypes.byref(params), ctypes.byref(vw) if vw is not None else None,
+        _ptr(hidden), _ptr(keys), _ptr(queries), _ptr(pos_ids), _ptr(vo_probe), N, T, H, d, D, K,
+        _ptr(out_clients), _ptr(workspace), workspace.numel(), _ptr(trace), _stream(stream)))
+
+
+def selftest_bounded_wait(cycles: int, workspace, stream=None):
+    """gmc_selftest_bounded_wait: a device wait that nothing ends, bounded by `cycles` clocks."""
+    _check(lib().gmc_selftest_bounded_wait(cycles, _ptr(workspace), workspace.numel(),
+                                           _stream(stream)))
 
 
 def select(clients, B, M, N, K, params: Params, out_idx, workspace, trace=None, stream=None):
