@@ -148,8 +148,9 @@ class ClockSampler:
 # roofline bookkeeping (algorithmic work per stage, per call)
 # ---------------------------------------------------------------------------
 # sparse solver rounds run as whole-GPU kernels after the dense first one
-# (SPARSE_GPU_ROUNDS in the library's kernels.cuh)
-WIDE_ROUNDS = 8
+# (sparse_gpu_rounds(N) in the library's kernels.cuh)
+def wide_rounds(N: int) -> int:
+    return 8 if N > 2048 else 4
 
 
 def stage_work(wl) -> dict:
@@ -165,10 +166,10 @@ def stage_work(wl) -> dict:
     w["message"] = ("hbm", B * (H * Tm * N * 4 + 2 * (N + Tm) * Hkv * d * es + Tm * H * d * es))
     w["clients"] = ("hbm", B * (M * N * 4 + H * Tm * N * 4 + N * N * 4))
     # selection: one read of the M x N clients per round.  Stage "rounds_gpu"
-    # runs the dense first round and the next WIDE_ROUNDS sparse rounds as
+    # runs the dense first round and the next wide_rounds(N) sparse rounds as
     # whole-GPU kernels; stage "select" (the cluster kernel) runs the rest.
     rounds = -(-K // 16)
-    wide = min(rounds, 1 + WIDE_ROUNDS)
+    wide = min(rounds, 1 + wide_rounds(N))
     w["rounds_gpu"] = ("hbm", B * wide * (M * N * 4.0))
     w["select"] = ("hbm", B * max(1, rounds - wide) * (M * N * 4.0))
     w["transport"] = ("hbm", B * ((N + Tm) * D * es + (K + Tm) * D * es

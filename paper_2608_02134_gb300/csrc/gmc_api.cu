@@ -167,7 +167,7 @@ R0State carve_round0(Carver& c, size_t B, size_t N, size_t M) {
   r.s0 = c.take<long long>(B * GMC_MAX_POOL);
   r.u1 = c.take<long long>(B * N);
   r.u2 = c.take<long long>(B * N);
-  r.ugain = SPARSE_GPU_ROUNDS % 2 == 0 ? r.u1 : r.u2;
+  r.ugain = sparse_gpu_rounds((int)N) % 2 == 0 ? r.u1 : r.u2;
   r.bcov = c.take<float>(B * M);
   r.cnt = c.take<int32_t>(B * M);
   r.fv = c.take<long long>(B * 4);
@@ -505,7 +505,7 @@ static int compress_impl(const gmc_problem* prob, const gmc_params* params,
                             cudaMemcpyDeviceToDevice, st));
     return GMC_OK;
   }
-  GMC_STAGE("rounds_gpu", 3 + 3 * SPARSE_GPU_ROUNDS,
+  GMC_STAGE("rounds_gpu", 3 + 3 * sparse_gpu_rounds(N),
             launch_round0(r0, dm.B, N, Ke, dm.M, dm.toff, HV, T, p.landmarks * p.landmarks, p, fx,
                           nullptr, s.C, s.scol, s.u0, s.order, s.status, tv, st));
   GMC_STAGE("select", 1,
@@ -612,7 +612,7 @@ int gmc_select(const float* clients, int B, int M, int N, int K, const gmc_param
                         s.order, s.status, tv, st));
   GMC_TRY(launch_select(r0, B, N, K, M, nullptr, 0, 1, 0, p, 0, s.fexp, s.C, s.scol, s.u0,
                         s.order, s.support, s.slot, out_idx, s.status, tv, st));
-  g_launches += 7 + 3 * SPARSE_GPU_ROUNDS;
+  g_launches += 7 + 3 * sparse_gpu_rounds(N);
   return GMC_OK;
 }
 

@@ -8,7 +8,7 @@
 //               b_m = max over the batch, and the row's survivors
 //               {i : Cbar_mi > b_m} compacted in place; the next round's gains
 //               are summed in fixed point (global atomics).
-// The next SPARSE_GPU_ROUNDS rounds run the same three steps over the survivor
+// The next sparse_gpu_rounds(N) rounds run the same three steps over the survivor
 // lists left in place by the previous round (row m: values Cbar[m][0..cnt_m),
 // tokens scol[m][0..cnt_m), ascending):
 //   k_rg_pool   the pool of the current gains among the unselected tokens;
@@ -29,7 +29,24 @@
 namespace gmc {
 
 namespace {
-constexpr int R0_ROWS = 8;  // rows per block (one warp each)
+constexpr int R0_ROWS = 8;  // warps per block; the responsibility kernels take one row per warp
+// The filters take `rpw` rows per warp (rows m0 + w + R0_ROWS * i).  More rows
+// per block mean fewer global atomics for the next gains (one per block and
+// column) but less parallelism: one row per warp is faster while the blocks
+// fit on the GPU at once, four when there are many more blocks than that.
+int filter_rows_per_warp(int B, int M) {
+  static int sms = 0;
+  if (sms == 0) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+      cudaGetLastError();
+      sms = 152;
+    }
+  }
+  const long long blocks = (long long)B * ceil_div(M, R0_ROWS);
+  return blocks > 32LL * sms ? 4 : 1;
+}
 }
 
 __global__ void __launch_bounds__(512) k_r0_pool(const long long* __restrict__ u0, int B, int N,
@@ -54,17 +71,24 @@ __global__ void __launch_bounds__(512) k_r0_pool(const long long* __restrict__ u
   }
   sel::PoolScratch w;
   char* p = sm_r0p;
+  long long* ug = reinterpret_cast<long long*>(p);  p += sizeof(long long) * (size_t)N;
   w.hist = reinterpret_cast<int*>(p);       p += sizeof(int) * sel::HBINS;
   w.bnd = reinterpret_cast<int*>(p);        p += sizeof(int) * N;
   w.wsum = reinterpret_cast<int*>(p);       p += sizeof(int) * 32;
   w.scal = reinterpret_cast<int*>(p);       p += sizeof(int) * 8;
+  w.coarse = reinterpret_cast<int*>(p);     p += sizeof(int) * sel::CBINS;
   int* pool = reinterpret_cast<int*>(p);    p += sizeof(int) * P;
-  w.tmp = reinterpret_cast<int*>(p);        p += sizeof(int) * P;
+  w.key = reinterpret_cast<short*>(p);     p += sizeof(short) * (size_t)N;
+  w.pk = reinterpret_cast<unsigned char*>(p); p += (size_t)N;
   unsigned char* selz = reinterpret_cast<unsigned char*>(p);
-  for (int j = threadIdx.x; j < N; j += blockDim.x) selz[j] = 0;
+  for (int j = threadIdx.x; j < N; j += blockDim.x) {
+    selz[j] = 0;
+    ug[j] = u0[(size_t)b * N + j];  // the gains in shared memory: select_pool reads them often
+  }
   for (int h = threadIdx.x; h < sel::HBINS; h += blockDim.x) w.hist[h] = 0;
+  if (threadIdx.x < sel::CBINS) w.coarse[threadIdx.x] = 0;
   __syncthreads();
-  const int Pt = sel::select_pool(u0 + (size_t)b * N, selz, N, P, w, pool, nullptr);
+  const int Pt = sel::select_pool(ug, selz, N, P, w, pool, nullptr);
   for (int k = threadIdx.x; k < P; k += blockDim.x) pool0[(size_t)b * P + k] = k < Pt ? pool[k] : -1;
   if (threadIdx.x == 0) info[b * 4] = Pt;
 }
@@ -131,7 +155,7 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_filter(
     const int32_t* toff, int Tmax, int uniform_rows, const int32_t* __restrict__ pool0,
     int32_t* info, const long long* __restrict__ s0, int P, int bsz, int fx_exp,
     const int32_t* fexp, long long* u1, float* bcov, int32_t* cnt, long long* fv,
-    int32_t* order, TraceView tv) {
+    int32_t* order, int rpw, TraceView tv) {
   grid_dep_wait();
   __shared__ int pool[GMC_MAX_POOL];
   __shared__ long long sc[GMC_MAX_POOL];
@@ -147,7 +171,7 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_filter(
     MG = H * text_geom(toff, b, B, Tmax, nullptr).T;
     Mb = MG + N + L2;
   }
-  const int m0 = blockIdx.x * R0_ROWS;
+  const int m0 = blockIdx.x * R0_ROWS * rpw;
   if (m0 >= Mb) return;
   const float fxs = ldexpf(1.f, fexp ? fexp[b] : fx_exp);
   const int nb = min(bsz, min(Pt, K));
@@ -179,8 +203,10 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_filter(
       if (threadIdx.x == 0) tv.at<int32_t>(b, tv.off_round_end)[0] = nb;
     }
   }
-  const int lane = threadIdx.x & 31, m = m0 + (threadIdx.x >> 5);
-  if (m < Mb) {
+  const int lane = threadIdx.x & 31;
+  for (int ir = 0; ir < rpw; ++ir) {
+    const int m = m0 + (threadIdx.x >> 5) + R0_ROWS * ir;
+    if (m >= Mb) break;
     float* vals = C + ((size_t)b * Mstride + m) * N;
     uint16_t* cols = scol + ((size_t)b * Mstride + m) * N;
     float bnew = 0.f;
@@ -189,6 +215,7 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_filter(
     const long long fb_new = to_fix(bnew, fxs);
     int w = 0;
     float rowmax = 0.f;
+    const unsigned lt = sel::lanemask_lt();
     if ((N & 3) == 0) {
       // 32 lanes x 8 float4 = 1024 columns per step; all loads issued before any
       // survivor is written back in place
@@ -206,20 +233,16 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_filter(
         for (int u = 0; u < 8; ++u) {
           const int k4 = base4 + u * 32 + lane;
           const float c4[4] = {buf[u].x, buf[u].y, buf[u].z, buf[u].w};
-          int kc = 0;
+          // survivors before this lane's: one ballot per element of the float4
+          int pre = 0, tot = 0;
 #pragma unroll
           for (int e2 = 0; e2 < 4; ++e2) {
             rowmax = fmaxf(rowmax, c4[e2]);
-            kc += (k4 < n4 && c4[e2] > bnew);
+            const unsigned bal = __ballot_sync(FULL, k4 < n4 && c4[e2] > bnew);
+            pre += __popc(bal & lt);
+            tot += __popc(bal);
           }
-          int pre = kc;
-#pragma unroll
-          for (int o = 1; o < 32; o <<= 1) {
-            const int y = __shfl_up_sync(FULL, pre, o);
-            if (lane >= o) pre += y;
-          }
-          const int tot = __shfl_sync(FULL, pre, 31);
-          int pos = w + pre - kc;
+          int pos = w + pre;
           if (k4 < n4) {
 #pragma unroll
             for (int e2 = 0; e2 < 4; ++e2)
@@ -291,19 +314,26 @@ __global__ void __launch_bounds__(512) k_rg_pool(const long long* __restrict__ u
   }
   sel::PoolScratch w;
   char* p = sm_rgp;
+  long long* ug = reinterpret_cast<long long*>(p);  p += sizeof(long long) * (size_t)N;
   w.hist = reinterpret_cast<int*>(p);       p += sizeof(int) * sel::HBINS;
   w.bnd = reinterpret_cast<int*>(p);        p += sizeof(int) * N;
   w.wsum = reinterpret_cast<int*>(p);       p += sizeof(int) * 32;
   w.scal = reinterpret_cast<int*>(p);       p += sizeof(int) * 8;
+  w.coarse = reinterpret_cast<int*>(p);     p += sizeof(int) * sel::CBINS;
   int* pool = reinterpret_cast<int*>(p);    p += sizeof(int) * P;
-  w.tmp = reinterpret_cast<int*>(p);        p += sizeof(int) * P;
+  w.key = reinterpret_cast<short*>(p);     p += sizeof(short) * (size_t)N;
+  w.pk = reinterpret_cast<unsigned char*>(p); p += (size_t)N;
   unsigned char* self = reinterpret_cast<unsigned char*>(p);
-  for (int j = threadIdx.x; j < N; j += blockDim.x) self[j] = 0;
+  for (int j = threadIdx.x; j < N; j += blockDim.x) {
+    self[j] = 0;
+    ug[j] = ucur[(size_t)b * N + j];  // the gains in shared memory: select_pool reads them often
+  }
   for (int h = threadIdx.x; h < sel::HBINS; h += blockDim.x) w.hist[h] = 0;
+  if (threadIdx.x < sel::CBINS) w.coarse[threadIdx.x] = 0;
   __syncthreads();
   for (int q = threadIdx.x; q < S; q += blockDim.x) self[order[(size_t)b * K + q]] = 1;
   __syncthreads();
-  const int Pt = sel::select_pool(ucur + (size_t)b * N, self, N, P, w, pool, nullptr);
+  const int Pt = sel::select_pool(ug, self, N, P, w, pool, nullptr);
   for (int k = threadIdx.x; k < P; k += blockDim.x) pool0[(size_t)b * P + k] = k < Pt ? pool[k] : -1;
   if (threadIdx.x == 0) {
     info[b * 4] = Pt;
@@ -401,7 +431,7 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_rg_filter(
     float* C, uint16_t* scol, int B, int N, int K, int Mstride, int H, int L2,
     const int32_t* toff, int Tmax, int uniform_rows, const int32_t* __restrict__ pool0,
     int32_t* info, const long long* __restrict__ sc0, int P, int bsz, int fx_exp,
-    const int32_t* fexp, long long* unext, float* bcov, int32_t* cnt, int32_t* order,
+    const int32_t* fexp, long long* unext, float* bcov, int32_t* cnt, int32_t* order, int rpw,
     TraceView tv) {
   grid_dep_wait();
   __shared__ int pool[GMC_MAX_POOL];
@@ -414,7 +444,7 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_rg_filter(
   if (Pt == 0) return;
   int Mb = Mstride;
   if (!uniform_rows) Mb = H * text_geom(toff, b, B, Tmax, nullptr).T + N + L2;
-  const int m0 = blockIdx.x * R0_ROWS;
+  const int m0 = blockIdx.x * R0_ROWS * rpw;
   if (m0 >= Mb) return;
   const int S = info[b * 4 + 3], rd = info[b * 4 + 2];
   const float fxs = ldexpf(1.f, fexp ? fexp[b] : fx_exp);
@@ -447,8 +477,10 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_rg_filter(
     }
   }
   __syncthreads();
-  const int lane = threadIdx.x & 31, m = m0 + (threadIdx.x >> 5);
-  if (m < Mb) {
+  const int lane = threadIdx.x & 31;
+  for (int ir = 0; ir < rpw; ++ir) {
+    const int m = m0 + (threadIdx.x >> 5) + R0_ROWS * ir;
+    if (m >= Mb) break;
     const size_t row = (size_t)b * Mstride + m;
     const int n = cnt[row];
     float* vals = C + row * N;
@@ -518,7 +550,9 @@ cudaError_t launch_round0(const R0State& r0, int B, int N, int K, int M, const i
                           cudaStream_t st) {
   const int P = p.pool_mult * p.batch_b;
   cudaError_t e;
-  const size_t smem = sizeof(int) * (sel::HBINS + N + 32 + 8 + 2 * P) + (size_t)N + 64;
+  const size_t smem =
+      sizeof(long long) * (size_t)N + sizeof(int) * (sel::HBINS + N + 32 + 8 + sel::CBINS + P) +
+      4 * (size_t)N + 64;
   if ((e = set_smem_limit((const void*)k_r0_pool, smem)) != cudaSuccess) return e;
   const int uniform = (H == 0);
   launch_k(k_r0_pool, B, 512, smem, st, 1, u0, B, N, P, uniform ? nullptr : toff, T, r0.pool, r0.info,
@@ -530,9 +564,11 @@ cudaError_t launch_round0(const R0State& r0, int B, int N, int K, int M, const i
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   const size_t fsm = sizeof(unsigned long long) * (size_t)N;
   if ((e = set_smem_limit((const void*)k_r0_filter, fsm)) != cudaSuccess) return e;
-  launch_k(k_r0_filter, grid, 32 * R0_ROWS, fsm, st, 1, C, scol, B, N, K, M, H, L2, toff, T, uniform, r0.pool,
+  const int rpw = filter_rows_per_warp(B, M);
+  const dim3 fgrid(ceil_div(M, R0_ROWS * rpw), B);
+  launch_k(k_r0_filter, fgrid, 32 * R0_ROWS, fsm, st, 1, C, scol, B, N, K, M, H, L2, toff, T, uniform, r0.pool,
                                              r0.info, r0.s0, P, p.batch_b, fx_exp, fexp, r0.u1,
-                                             r0.bcov, r0.cnt, r0.fv, order, tv);
+                                             r0.bcov, r0.cnt, r0.fv, order, rpw, tv);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   // sparse rounds: gains alternate between u1 and u2
   const size_t psm = smem;  // the pool kernel's layout is round 0's
@@ -541,7 +577,7 @@ cudaError_t launch_round0(const R0State& r0, int B, int N, int K, int M, const i
   if ((e = set_smem_limit((const void*)k_rg_rho, rsm)) != cudaSuccess) return e;
   const size_t gsm = sizeof(unsigned long long) * (size_t)N + (size_t)N;
   if ((e = set_smem_limit((const void*)k_rg_filter, gsm)) != cudaSuccess) return e;
-  for (int rr = 1; rr <= SPARSE_GPU_ROUNDS; ++rr) {
+  for (int rr = 1; rr <= sparse_gpu_rounds(N); ++rr) {
     long long* ucur = rr % 2 == 1 ? r0.u1 : r0.u2;
     long long* unext = rr % 2 == 1 ? r0.u2 : r0.u1;
     launch_k(k_rg_pool, B, 512, psm, st, 1, (const long long*)ucur, unext, B, N, K, P,
@@ -552,9 +588,9 @@ cudaError_t launch_round0(const R0State& r0, int B, int N, int K, int M, const i
              (const int32_t*)r0.pool, (const int32_t*)r0.info, P, p.resp_temp, p.resp_eps, fx_exp,
              fexp, r0.s0);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    launch_k(k_rg_filter, grid, 32 * R0_ROWS, gsm, st, 1, C, scol, B, N, K, M, H, L2, toff, T,
+    launch_k(k_rg_filter, fgrid, 32 * R0_ROWS, gsm, st, 1, C, scol, B, N, K, M, H, L2, toff, T,
              uniform, (const int32_t*)r0.pool, r0.info, (const long long*)r0.s0, P, p.batch_b,
-             fx_exp, fexp, unext, r0.bcov, r0.cnt, order, tv);
+             fx_exp, fexp, unext, r0.bcov, r0.cnt, order, rpw, tv);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
   return cudaSuccess;

@@ -29,15 +29,20 @@
 // Parallel layout.  The CS CTAs of a cluster split the client rows; each CTA
 // keeps its rows' coverage b_m, survivor counts and lists.  Gains and scores
 // are summed in 64-bit fixed point, so every reduction (shared-memory atomics
-// inside a CTA, distributed-shared-memory loads / atomics across the cluster)
-// is exact and order-independent: the solver is deterministic.  Per round:
-//   gains: each CTA reduces one slice of tokens over the cluster and
-//          broadcasts it, so every CTA holds the full gain vector;
-//   pool:  every CTA selects the same pool locally (histogram + exact tie
-//          ranking), slots numbered in ascending token order;
-//   scores: pushed into every CTA by atomics; every CTA picks the same batch.
-// Three cluster barriers per round; all control decisions are derived from
-// data every CTA holds identically, so all CTAs run the same barriers.
+// inside a CTA, distributed-shared-memory atomics across the cluster) is
+// exact and order-independent: the solver is deterministic.  Per round:
+//   pool:   every CTA selects the same pool from the full gain vector
+//           (histogram + exact tie ranking, see select_pool);
+//   scores: every CTA adds its rows' responsibility-weighted residuals into
+//           the score array of every CTA of the cluster; every CTA then picks
+//           the same batch;
+//   gains:  every CTA adds its rows' residuals for the next round into the
+//           owner of each token (token j belongs to CTA j / ceil(N / CS)); after
+//           the barrier every CTA reads the full gain vector from the owners.
+//           The owners' buffers alternate between rounds, so a buffer is
+//           cleared only after every CTA has read it.
+// Two cluster barriers per round; all control decisions are derived from data
+// every CTA holds identically, so all CTAs run the same barriers.
 #include <cooperative_groups.h>
 
 #include "common.cuh"
@@ -83,18 +88,20 @@ struct SelArgs {
 };
 
 struct SelSmem {
-  unsigned* u_lo;       // [N]  this CTA's partial gains of the next round, low 32 bits
-  unsigned* u_hi;       // [N]  high 32 bits (carries included)
+  unsigned long long* gacc;  // [NB][SL] next-round gains of the tokens this CTA owns,
+                             // summed by every CTA of the cluster (NB = 2 buffers
+                             // used by alternate rounds when CS > 1, else 1)
   long long* u_full;    // [N]  gains of the current round (every CTA)
   int* hist;            // [HBINS]
+  int* coarse;          // [CBINS]
+  unsigned char* pk;    // [N]  select_pool: boundary tokens that enter
+  short* key;           // [N]  select_pool: bucket of every token
   int* bnd;             // [N]  tokens in the boundary histogram bin
-  int* tmp;             // [P]  pool tokens in arrival order (select_pool)
   unsigned char* sel;   // [N]
   short* poolslot;      // [N]  pool slot of a token or -1
   int* pool;            // [P]
-  long long* s_acc;     // [P]  cluster-wide scores
+  long long* s_acc;     // [P]  cluster-wide scores, pushed by every CTA
   unsigned long long* sw;  // [SEL_WARPS][P] per-warp partial scores
-  long long* s_part;    // [P]  this CTA's scores, read by the whole cluster
   int* batch;           // [P]
   int* inb;             // [P]
   int* wsum;            // [32] scan scratch
@@ -106,7 +113,6 @@ struct SelSmem {
   int* bnb;             // [RPC] flat mode: bits of the row's largest batch value
   long long* bfix;      // [RPC] flat mode: coverage in fixed point
   int* cstart;          // [N+1] flat mode: first entry of every token
-  int* rowb;            // [SEL_MAX_CS + 1] first client row of every CTA of the cluster
   long long* fb;        // [8]  F_S[3], F_V[3] (fixed point)
   int* scal;            // [16] Bstar, c_hi, Pt, nbnd, cursor, global rows left
   float* svals;         // [cap]
@@ -116,7 +122,8 @@ struct SelSmem {
 
 enum { SC_BSTAR = 0, SC_CHI, SC_PT, SC_NBND, SC_CURSOR, SC_GLOBAL, SC_NEED };
 
-__host__ __device__ inline size_t sel_fixed_bytes(int N, int P, int RPC, SelSmem* o, char* base) {
+__host__ __device__ inline size_t sel_fixed_bytes(int N, int P, int RPC, int gwords, SelSmem* o,
+                                                  char* base) {
   size_t off = 0;
   auto take = [&](size_t bytes) {
     size_t at = off;
@@ -124,18 +131,18 @@ __host__ __device__ inline size_t sel_fixed_bytes(int N, int P, int RPC, SelSmem
     return base ? base + at : nullptr;
   };
   char* p;
-  p = take(sizeof(unsigned) * N);   if (o) o->u_lo = (unsigned*)p;
-  p = take(sizeof(unsigned) * N);   if (o) o->u_hi = (unsigned*)p;
+  p = take(sizeof(unsigned long long) * gwords);  if (o) o->gacc = (unsigned long long*)p;
   p = take(sizeof(long long) * N);  if (o) o->u_full = (long long*)p;
   p = take(sizeof(int) * HBINS);    if (o) o->hist = (int*)p;
+  p = take(sizeof(int) * sel::CBINS);  if (o) o->coarse = (int*)p;
+  p = take(N);                      if (o) o->pk = (unsigned char*)p;
+  p = take(sizeof(short) * N);      if (o) o->key = (short*)p;
   p = take(sizeof(int) * N);        if (o) o->bnd = (int*)p;
-  p = take(sizeof(int) * P);        if (o) o->tmp = (int*)p;
   p = take(N);                      if (o) o->sel = (unsigned char*)p;
   p = take(sizeof(short) * N);      if (o) o->poolslot = (short*)p;
   p = take(sizeof(int) * P);        if (o) o->pool = (int*)p;
   p = take(sizeof(long long) * P);  if (o) o->s_acc = (long long*)p;
   p = take(sizeof(unsigned long long) * SEL_WARPS * P);  if (o) o->sw = (unsigned long long*)p;
-  p = take(sizeof(long long) * P);  if (o) o->s_part = (long long*)p;
   p = take(sizeof(int) * P);        if (o) o->batch = (int*)p;
   p = take(sizeof(int) * P);        if (o) o->inb = (int*)p;
   p = take(sizeof(int) * 32);       if (o) o->wsum = (int*)p;
@@ -147,28 +154,26 @@ __host__ __device__ inline size_t sel_fixed_bytes(int N, int P, int RPC, SelSmem
   p = take(sizeof(int) * RPC);      if (o) o->bnb = (int*)p;
   p = take(sizeof(long long) * RPC);  if (o) o->bfix = (long long*)p;
   p = take(sizeof(int) * (N + 1));  if (o) o->cstart = (int*)p;
-  p = take(sizeof(int) * (SEL_MAX_CS + 1));  if (o) o->rowb = (int*)p;
   p = take(sizeof(long long) * 8);  if (o) o->fb = (long long*)p;
   p = take(sizeof(int) * 16);       if (o) o->scal = (int*)p;
   return off;
 }
 
+// Fire-and-forget 64-bit add into the shared memory of CTA `rank` of the
+// cluster at the offset of local shared-memory address `local` (no value is
+// returned, so the issuing thread does not wait for the remote round trip;
+// the next cluster barrier orders it before every later read).
+__device__ __forceinline__ void red_add_cluster(const void* local, int rank,
+                                                unsigned long long v) {
+  const uint32_t la = (uint32_t)__cvta_generic_to_shared(local);
+  uint32_t ra;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(ra) : "r"(la), "r"(rank));
+  asm volatile("red.shared::cluster.add.u64 [%0], %1;" ::"r"(ra), "l"(v) : "memory");
+}
+
 using sel::key_before;
 using sel::lanemask_lt;
 using sel::block_exclusive_scan;
-
-// Exact 64-bit fixed-point add into shared memory as two 32-bit atomics: the
-// low word wraps and its carry goes to the high word, so the pair always holds
-// the exact sum, whatever the order of the additions.
-__device__ __forceinline__ void add_fix(unsigned* lo, unsigned* hi, unsigned long long v) {
-  const unsigned vl = (unsigned)v, vh = (unsigned)(v >> 32);
-  const unsigned old = atomicAdd(lo, vl);
-  const unsigned up = vh + ((old + vl) < old ? 1u : 0u);
-  if (up) atomicAdd(hi, up);
-}
-__device__ __forceinline__ long long get_fix(const unsigned* lo, const unsigned* hi) {
-  return (long long)(((unsigned long long)*hi << 32) | *lo);
-}
 
 // Reductions inside an aligned group of G = 8 lanes (mask `gm`).
 constexpr int G = 8;
@@ -213,11 +218,12 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
     Mb = MG + N + a.L2;
   }
   const int RPC = a.rpc;  // capacity of the per-row arrays of one CTA
+  // token j's next-round gain is summed in CTA j / SL (its owner)
   const int SL = (N + CS - 1) / CS;
-  const int jlo = r * SL, jhi = min(N, jlo + SL);
+  const int NB = CS > 1 ? 2 : 1;
 
   SelSmem s;
-  const size_t fixed = sel_fixed_bytes(N, P, RPC, &s, sm_sel);
+  const size_t fixed = sel_fixed_bytes(N, P, RPC, NB * SL, &s, sm_sel);
   s.svals = reinterpret_cast<float*>(sm_sel + fixed);
   s.scols = reinterpret_cast<uint16_t*>(sm_sel + fixed + sizeof(float) * (size_t)a.cap);
   s.srows = s.scols + a.cap;
@@ -233,78 +239,27 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
   const int Pt0 = rd0;                                // > 0: the rounds left survivor lists
   const int nb0 = rd0 > 0 ? a.r0.info[b * 4 + 1] : 0;  // tokens selected so far
   for (int j = threadIdx.x; j < N; j += blockDim.x) {
-    s.u_lo[j] = 0;
-    s.u_hi[j] = 0;
     s.u_full[j] = rd0 > 0 ? a.r0.ugain[(size_t)b * N + j] : a.u0[(size_t)b * N + j];
     s.poolslot[j] = -1;
     s.sel[j] = 0;
   }
   for (int k = threadIdx.x; k < P; k += blockDim.x) s.s_acc[k] = 0;
+  for (int q = threadIdx.x; q < NB * SL; q += blockDim.x) s.gacc[q] = 0;
   for (int h = threadIdx.x; h < HBINS; h += blockDim.x) s.hist[h] = 0;  // select_pool keeps it zero
+  if (threadIdx.x < sel::CBINS) s.coarse[threadIdx.x] = 0;
   if (threadIdx.x < 8) s.fb[threadIdx.x] = 0;
   if (threadIdx.x < 16) s.scal[threadIdx.x] = 0;
   if (threadIdx.x == 0) s.scal[SC_GLOBAL] = 1;
-  // Rows are split over the cluster so every CTA holds about the same number
-  // of survivors (weight: survivors + 16 per row); every CTA computes the same
-  // split.  Without a first round, or if a part would exceed RPC rows, the
-  // rows are split evenly.
-  if (threadIdx.x <= SEL_MAX_CS) s.rowb[threadIdx.x] = Mb;
+  // Rows are dealt to the CTAs in turn (CTA r holds rows r, r + CS, ...):
+  // every CTA gets the same mix of grounded, appearance and spatial rows and
+  // of the image's regions, so the work of every phase is about even.
   __syncthreads();
-  bool balanced = false;
-  if (Pt0 > 0 && CS > 1) {
-    const int chunk = (Mb + blockDim.x - 1) / blockDim.x;
-    const int m0 = min(Mb, (int)threadIdx.x * chunk), m1 = min(Mb, m0 + chunk);
-    const int32_t* cgl = a.r0.cnt + (size_t)b * a.Mstride;
-    int wsum = 0;
-    for (int m = m0; m < m1; ++m) wsum += cgl[m] + 16;
-    int W = 0;
-    int run = block_exclusive_scan(wsum, s.wsum, &W);
-    // CTA c starts after the row where the preceding weight reaches c*W/CS;
-    // the CS - 1 targets are computed once (the histogram is zero again
-    // before its first use)
-    long long* tgt = reinterpret_cast<long long*>(s.hist);
-    if (threadIdx.x >= 1 && (int)threadIdx.x < CS) tgt[threadIdx.x] = (long long)threadIdx.x * W / CS;
-    __syncthreads();
-    // a target inside this thread's weight range (run, run + wsum] lies in one
-    // of its rows: only then are the rows walked
-    for (int c = 1; c < CS; ++c) {
-      const long long t = tgt[c];
-      if (!(run < t && run + wsum >= t)) continue;
-      long long at = run;
-      for (int m = m0; m < m1; ++m) {
-        const int wm = cgl[m] + 16;
-        if (at < t && at + wm >= t) {
-          atomicMin(&s.rowb[c], m + 1);
-          break;
-        }
-        at += wm;
-      }
-    }
-    __syncthreads();
-    if (threadIdx.x < 2 * SEL_MAX_CS) s.hist[threadIdx.x] = 0;
-    if (threadIdx.x == 0) {
-      s.rowb[0] = 0;
-      int prev = 0, ok = 1;
-      for (int c = 1; c <= CS; ++c) {
-        int bc = c < CS ? s.rowb[c] : Mb;
-        if (bc < prev) bc = prev;
-        if (c < CS) s.rowb[c] = bc;
-        if (bc - prev > RPC) ok = 0;
-        prev = bc;
-      }
-      s.scal[SC_NEED] = ok;
-    }
-    __syncthreads();
-    balanced = s.scal[SC_NEED] != 0;
-  }
-  const int even = (Mb + CS - 1) / CS;
-  const int mlo = balanced ? s.rowb[r] : min(Mb, r * even);
-  const int mhi = balanced ? (r + 1 < CS ? s.rowb[r + 1] : Mb) : min(Mb, mlo + even);
-  const int nrows = max(0, mhi - mlo);
+  const int nrows = Mb > r ? (Mb - r + CS - 1) / CS : 0;
+  auto grow = [&](int q) { return q * CS + r; };  // client row of local row q
   for (int q = threadIdx.x; q < RPC; q += blockDim.x) {
     const bool have = Pt0 > 0 && q < nrows;
-    s.bcov[q] = have ? a.r0.bcov[(size_t)b * a.Mstride + mlo + q] : 0.f;
-    s.cnt[q] = have ? a.r0.cnt[(size_t)b * a.Mstride + mlo + q] : 0;
+    s.bcov[q] = have ? a.r0.bcov[(size_t)b * a.Mstride + grow(q)] : 0.f;
+    s.cnt[q] = have ? a.r0.cnt[(size_t)b * a.Mstride + grow(q)] : 0;
     s.bfix[q] = 0;
     s.rmaxb[q] = 0;
     s.npl[q] = 0;
@@ -357,7 +312,7 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
         jj[u] = -1;
         if (e < tot) {
           const int q = row_of(e);
-          jj[u] = Simg[(size_t)(mlo + q) * N + (e - rp[q])];
+          jj[u] = Simg[(size_t)grow(q) * N + (e - rp[q])];
         }
       }
 #pragma unroll
@@ -391,7 +346,7 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
         vv[u] = 0.f;
         if (e < tot) {
           const int q = row_of(e);
-          const size_t g = (size_t)(mlo + q) * N + (e - rp[q]);
+          const size_t g = (size_t)grow(q) * N + (e - rp[q]);
           qq[u] = q;
           jj[u] = Simg[g];
           vv[u] = Cimg[g];
@@ -418,6 +373,17 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
   if (Pt0 > 0) migrate();
 
   const int rounds_max = (K + a.bsz - 1) / a.bsz + 1;
+  // add v to token j's gain for the round after `rnd` at the token's owner
+  // (exact: 64-bit integer atomics, order-independent)
+  auto gain_add = [&](int j, unsigned long long v, int rnd_now) {
+    const int o = j / SL;
+    unsigned long long* at = s.gacc + (rnd_now & (NB - 1)) * SL + (j - o * SL);
+    if (CS > 1) red_add_cluster(at, o, v); else atomicAdd(at, v);
+  };
+  // add v to pool slot k's score in every CTA of the cluster
+  auto score_push = [&](int k, unsigned long long v, int c0, int cstep) {
+    for (int c = c0; c < CS; c += cstep) red_add_cluster(s.s_acc + k, c, v);
+  };
   int S_count = nb0, rnd = rd0, filled = 0;
   const int sub = lane / G, gl = lane % G;
   const int gid = wid * (32 / G) + sub, ngrp = nw * (32 / G);  // 8-lane groups of the block
@@ -429,7 +395,7 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
       break;
     }
     // ---- pool of this round ------------------------------------------------------
-    sel::PoolScratch pw{s.hist, s.bnd, s.tmp, s.wsum, s.scal + 8};
+    sel::PoolScratch pw{s.hist, s.coarse, s.bnd, s.key, s.pk, s.wsum, s.scal + 8};
     const int Pt = sel::select_pool(s.u_full, s.sel, N, P, pw, s.pool, s.poolslot);
     if (Pt == 0) {
       // Zero-gain remainder: fill in ascending source order (F unchanged).
@@ -499,7 +465,8 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
         }
       }
       __syncthreads();
-      // s_k = sum_m rho_mk R_mk: one group owns pool slot k, so its sum is this CTA's score
+      // s_k = sum_m rho_mk R_mk: one group owns pool slot k and adds its sum
+      // into every CTA's scores
       for (int k = gid; k < Pt; k += ngrp) {
         const int j = s.pool[k];
         unsigned long long acc = 0;
@@ -516,7 +483,7 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
         }
 #pragma unroll
         for (int o = G / 2; o > 0; o >>= 1) acc += __shfl_xor_sync(gm, acc, o);
-        if (gl == 0) s.s_part[k] = (long long)acc;
+        if (acc) score_push(k, acc, gl, G);  // the group's lanes share the CTAs
       }
     }
     if (!flat) {
@@ -527,8 +494,8 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
       const int q = q0 + sub;
       const int n = q < nrows ? s.cnt[q] : 0;
       const float bm = q < nrows ? s.bcov[q] : 0.f;
-      const float* vals = Cimg + (size_t)(mlo + q) * N;
-      const uint16_t* cols = Simg + (size_t)(mlo + q) * N;
+      const float* vals = Cimg + (size_t)grow(q) * N;
+      const uint16_t* cols = Simg + (size_t)grow(q) * N;
       float rmax = 0.f;
       int npool = 0, ncache = 0, mine = 0;  // mine: pool entries this lane saw
       float cv[PCL] = {};
@@ -600,22 +567,17 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
     }
     __syncthreads();
     if (!flat)
-      for (int k = threadIdx.x; k < Pt; k += blockDim.x) {
+      for (int q = threadIdx.x; q < Pt * CS; q += blockDim.x) {  // (slot, target CTA) pairs
+        const int k = q / CS, c = q - k * CS;
         unsigned long long v = 0;
         for (int w2 = 0; w2 < SEL_WARPS; ++w2) v += s.sw[w2 * Pt + k];
-        s.s_part[k] = (long long)v;
+        if (v) score_push(k, v, c, CS);
       }
-    cluster.sync();  // every CTA's scores are complete
-    for (int k = threadIdx.x; k < Pt; k += blockDim.x) {
-      long long v[SEL_MAX_CS];
-#pragma unroll
-      for (int c = 0; c < SEL_MAX_CS; ++c) v[c] = c < CS ? cluster.map_shared_rank(s.s_part, c)[k] : 0;
-      long long t = 0;
-#pragma unroll
-      for (int c = 0; c < SEL_MAX_CS; ++c) t += v[c];
-      s.s_acc[k] = t;
-    }
-    __syncthreads();
+    cluster.sync();  // every CTA's scores have reached every CTA's s_acc
+    // nobody reads the gain buffer of the previous round any more (it was read
+    // before this round's pool): clear this CTA's part of it for the next round
+    if (CS > 1)
+      for (int q = threadIdx.x; q < SL; q += blockDim.x) s.gacc[((rnd + 1) & 1) * SL + q] = 0;
 
     // ---- batch, coverage update, survivor filter, next gains ------------------
     const int nb = min(a.bsz, min(Pt, K - S_count));
@@ -677,7 +639,7 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
           if (qq[u] == DEADROW) continue;
           if (cc[u] > s.bcov[qq[u]]) {
             if (jj[u] != jc) {
-              if (acc) add_fix(&s.u_lo[jc], &s.u_hi[jc], acc);
+              if (acc) gain_add(jc, acc, rnd);
               if (nj) atomicAdd(&s.bnd[jc], nj);
               jc = jj[u];
               acc = 0;
@@ -691,7 +653,7 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
           }
         }
       }
-      if (acc) add_fix(&s.u_lo[jc], &s.u_hi[jc], acc);
+      if (acc) gain_add(jc, acc, rnd);
       if (nj) atomicAdd(&s.bnd[jc], nj);
       // Once fewer than 60% of the entries are live, drop the dead ones: the
       // live entries move down in order (token-major order is kept) and the
@@ -757,8 +719,8 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
       const int q = q0 + sub;
       const int n = q < nrows ? s.cnt[q] : 0;
       const float bm = q < nrows ? s.bcov[q] : 0.f;
-      float* vals = Cimg + (size_t)(mlo + q) * N;
-      uint16_t* cols = Simg + (size_t)(mlo + q) * N;
+      float* vals = Cimg + (size_t)grow(q) * N;
+      uint16_t* cols = Simg + (size_t)grow(q) * N;
       float bnew = bm;
       for (int k0 = gl; k0 < n; k0 += UNR * G) {
         int cc[UNR];
@@ -797,8 +759,7 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
             const int pos = w + __popc(msk & lt);
             vals[pos] = c[u];
             cols[pos] = (uint16_t)jj[u];
-            add_fix(&s.u_lo[jj[u]], &s.u_hi[jj[u]],
-                    (unsigned long long)(to_fix(c[u], fxs) - fb_new));
+            gain_add(jj[u], (unsigned long long)(to_fix(c[u], fxs) - fb_new), rnd);
           }
           w += __popc(msk);
         }
@@ -818,27 +779,30 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
     S_count += nb;
     ++rnd;
     if (S_count >= K) break;
-    cluster.sync();  // every CTA's gain partials are complete
+    cluster.sync();  // every contribution to the new gains has reached its owner
 
-    // ---- gains of the next round: reduce this CTA's token slice, broadcast it ----
-    for (int j = jlo + threadIdx.x; j < jhi; j += blockDim.x) {
-      long long t = 0;
-      for (int c = 0; c < CS; ++c)
-        t += get_fix(cluster.map_shared_rank(s.u_lo, c) + j, cluster.map_shared_rank(s.u_hi, c) + j);
-      for (int c = 0; c < CS; ++c) cluster.map_shared_rank(s.u_full, c)[j] = t;
-    }
-    cluster.sync();  // full gains everywhere; partials no longer read
-    for (int j = threadIdx.x; j < N; j += blockDim.x) {
-      s.u_lo[j] = 0;
-      s.u_hi[j] = 0;
+    // ---- gains of the next round, read from their owners ----------------------
+    {
+      const unsigned long long* gb = s.gacc + ((rnd - 1) & (NB - 1)) * SL;
+      for (int j = threadIdx.x; j < N; j += blockDim.x) {
+        const int o = j / SL;
+        const unsigned long long* at = gb + (j - o * SL);
+        s.u_full[j] = (long long)*(CS > 1 ? cluster.map_shared_rank(at, o) : at);
+      }
+      if (CS == 1) {  // a single CTA reuses its one buffer at once
+        __syncthreads();
+        for (int q = threadIdx.x; q < SL; q += blockDim.x) s.gacc[q] = 0;
+      }
+      __syncthreads();
     }
   }
 
   // ---- final: coverage per bank, sorted support, trace ---------------------
   {
     long long f0 = 0, f1 = 0, f2 = 0;
-    for (int m = mlo + threadIdx.x; m < mhi; m += blockDim.x) {
-      const long long v = to_fix(s.bcov[m - mlo], fxs);
+    for (int q = threadIdx.x; q < nrows; q += blockDim.x) {
+      const int m = grow(q);
+      const long long v = to_fix(s.bcov[q], fxs);
       if (m < MG) f0 += v; else if (m < MG + N) f1 += v; else f2 += v;
     }
     long long* fb0 = cluster.map_shared_rank(s.fb, 0);
@@ -926,19 +890,11 @@ cudaError_t launch_select(const R0State& r0, int B, int N, int K, int M, const i
   int CS = 1;
   while (CS * 2 <= SEL_MAX_CS && (long long)B * CS * 2 <= g_num_sms) CS *= 2;
   for (; CS >= 1; CS /= 2) {
-    // Row capacity of one CTA: room for a balanced split that gives a CTA up to
-    // 2x its even share of rows while leaving space for 16K survivor entries;
-    // else the even share alone.
-    const int even = (M + CS - 1) / CS;
-    int RPC = 0;
-    size_t fixed = 0;
-    for (int f = 2; f >= 1; f /= 2) {
-      RPC = min(M, f * even);
-      fixed = sel_fixed_bytes(N, a.P, RPC, nullptr, nullptr);
-      if (fixed + 8 * 16384 + 16 <= SMEM_LIMIT || (f == 1 && fixed + 1024 <= SMEM_LIMIT)) break;
-      RPC = 0;
-    }
-    if (RPC == 0) continue;
+    // Row capacity of one CTA: rows are dealt in turn, so ceil(M / CS) each
+    const int RPC = (M + CS - 1) / CS;
+    const int gwords = (CS > 1 ? 2 : 1) * ((N + CS - 1) / CS);
+    const size_t fixed = sel_fixed_bytes(N, a.P, RPC, gwords, nullptr, nullptr);
+    if (fixed + 1024 > SMEM_LIMIT) continue;
     a.rpc = RPC;
     // the rest of the shared memory holds survivor entries (value, token, row: 8 bytes)
     a.cap = (int)((SMEM_LIMIT - fixed - 16) / 8);

@@ -129,8 +129,11 @@ cudaError_t launch_build_clients(const Dims&, const gmc_params&, int fx_exp, Scr
                                  cudaStream_t);
 // State left by the first (dense) selection round, run over the whole GPU.
 // Rounds of the solver run on the whole GPU before the cluster kernel takes
-// over: the dense first round, then this many sparse rounds.
-constexpr int SPARSE_GPU_ROUNDS = 8;
+// over: the dense first round, then sparse_gpu_rounds(N) sparse rounds (an
+// even count: the cluster kernel starts from the gains in u1).  Larger images
+// keep more survivors per round, so more rounds stay on the whole GPU; the
+// counts were chosen by measurement.
+__host__ __device__ inline int sparse_gpu_rounds(int N) { return N > 2048 ? 8 : 4; }
 
 struct R0State {
   int32_t* pool;   // [B][P]  pool of the current whole-GPU round (-1 padded)

@@ -56,12 +56,15 @@ __device__ inline int block_exclusive_scan(int v, int* wsum, int* total) {
 }
 
 // Shared-memory scratch of select_pool.
+constexpr int CBINS = 64;       // coarse bins: the binary exponent of a gain
 struct PoolScratch {
-  int* hist;  // [HBINS], all zero on entry and on return
-  int* bnd;   // [N]
-  int* tmp;   // [P]  pool tokens in arrival order
-  int* wsum;  // [32]
-  int* scal;  // [5]
+  int* hist;           // [HBINS] fine bins, all zero on entry and on return
+  int* coarse;         // [CBINS] coarse bins, all zero on entry and on return
+  int* bnd;            // [N]  tokens of the boundary bin, ascending
+  short* key;          // [N]  bucket of every token (-1: not a candidate)
+  unsigned char* pk;   // [N]  boundary tokens that enter the pool
+  int* wsum;           // [32]
+  int* scal;           // [8]
 };
 
 // Warp-aggregated append: every lane with `want` gets a distinct index from
@@ -87,110 +90,157 @@ __device__ __forceinline__ int group_rank_of(const int* a, int n, int x, int gl,
 }
 
 // Pool of one round: the min(P, #{u_i > 0}) tokens with sel[i] == 0 of largest
-// gain u (fixed point), ties to the lower index.  A histogram over an
-// exponent/mantissa bucket finds the boundary bucket; tokens inside it are
-// ranked exactly.  Pool tokens arrive in any order and take the slot of their
-// rank by token index, so slots ascend with the token: pool[0..Pt).
-// poolslot (optional) receives the slot of every pool token.  Returns Pt.
-// Every thread of the block must call it (blockDim a multiple of 32, N
-// rounded up to the block is walked by whole warps); the result does not
-// depend on thread scheduling.
+// gain u (fixed point), ties to the lower index.  pool[0..Pt) lists the tokens
+// above the boundary bucket (below) by index, then the boundary bucket's
+// entering tokens by index; poolslot (optional) receives the slot of every
+// pool token.  The slots are a deterministic function of the gains, the same
+// in every block that calls this with the same data.  Returns Pt.
+//
+// Every gain gets an 11-bit bucket (exponent, 5 mantissa bits; monotone in u).
+// One pass counts the buckets and their exponents (64 coarse bins, counted
+// once per warp and exponent); every warp then finds the boundary bucket
+// holding the P-th largest gain from the coarse bins and the 32 fine bins of
+// one exponent.  Warp w owns 32-token chunks [w * nc, (w + 1) * nc) (lane =
+// token within a chunk, so every shared access is conflict-free); ballots
+// order the tokens above the boundary bucket and those inside it by index,
+// and one scan of the per-warp counts places them: no shared counter,
+// nothing that depends on thread scheduling.  Tokens inside the boundary
+// bucket are ranked exactly by (u desc, index asc).
+// Every thread of the block must call it; blockDim is a multiple of 32.
 __device__ inline int select_pool(const long long* u, const unsigned char* sel, int N, int P,
                                   PoolScratch w, int* pool, short* poolslot) {
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
-  if (threadIdx.x < 5) w.scal[threadIdx.x] = 0;
-  for (int j = threadIdx.x; j < N; j += blockDim.x) {
-    const long long v = u[j];
-    if (!sel[j] && v > 0) atomicAdd(&w.hist[gain_bucket(v)], 1);
+  const int nc = (N + 32 * nw - 1) / (32 * nw);  // chunks per warp
+  const unsigned lt = lanemask_lt();
+  // 1. bucket of every candidate (-1: selected or zero gain), histograms
+  for (int c = 0; c < nc; ++c) {
+    const int j = (wid * nc + c) * 32 + lane;
+    int kb = -1;
+    if (j < N) {
+      const long long v = u[j];
+      if (!sel[j] && v > 0) {
+        kb = gain_bucket(v);
+        atomicAdd(&w.hist[kb], 1);
+      }
+      w.key[j] = (short)kb;
+    }
+    // exponents: one atomic per warp and distinct exponent
+    const int e = kb >= 0 ? kb >> 5 : -1;
+    const unsigned same = __match_any_sync(FULL, e);
+    if (e >= 0 && (same & lt) == 0) atomicAdd(&w.coarse[e], __popc(same));
   }
   __syncthreads();
+  // 2. boundary bucket, found by every warp alike: coarse bins from the top,
+  //    then the fine bins of the boundary exponent
+  int bstar, above, Pt;
   {
-    // Every thread owns a contiguous range of buckets (zeroed again here); the
-    // thread whose range holds the P-th largest candidate finds the boundary
-    // bucket inside it.
-    const int per = (HBINS + blockDim.x - 1) / blockDim.x;
-    const int h0 = min(HBINS, (int)threadIdx.x * per), h1 = min(HBINS, h0 + per);
-    int part = 0;
-    for (int h = h0; h < h1; ++h) part += w.hist[h];
-    int x = part;  // inclusive prefix within the warp
+    const int hi = CBINS - 1 - 2 * lane;  // this lane's two coarse bins: hi, hi - 1
+    const int c0 = w.coarse[hi], c1 = w.coarse[hi - 1];
+    int incl = c0 + c1;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
-      const int y = __shfl_up_sync(FULL, x, o);
-      if (lane >= o) x += y;
+      const int y = __shfl_up_sync(FULL, incl, o);
+      if (lane >= o) incl += y;
     }
-    if (lane == 31) w.wsum[wid] = x;
-    __syncthreads();
-    int t = lane < nw ? w.wsum[lane] : 0;  // warp totals, prefix over warps by shuffles
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int y = __shfl_up_sync(FULL, t, o);
-      if (lane >= o) t += y;
-    }
-    const int npos = __shfl_sync(FULL, t, 31);
-    const int wbefore = wid > 0 ? __shfl_sync(FULL, t, wid - 1) : 0;
-    const int above = npos - (wbefore + x);  // candidates in higher buckets
+    const int npos = __shfl_sync(FULL, incl, 31);
     if (npos <= P) {
-      if (threadIdx.x == 0) {
-        w.scal[0] = -1;    // every candidate is in the pool
-        w.scal[1] = npos;  // count above the boundary bucket
-        w.scal[2] = npos;  // pool size
+      bstar = -1;    // every candidate is in the pool
+      above = npos;  // tokens above the boundary bucket
+      Pt = npos;
+    } else {
+      const unsigned reach = __ballot_sync(FULL, incl >= P);
+      const int L = __ffs(reach) - 1;  // first lane whose prefix reaches P
+      int excl = __shfl_sync(FULL, incl - c0 - c1, L);
+      const int l0 = __shfl_sync(FULL, c0, L);
+      int cb = CBINS - 1 - 2 * L;
+      if (excl + l0 < P) {
+        excl += l0;
+        cb -= 1;
       }
-    } else if (above < P && above + part >= P) {
-      int cum = above;
-      int bstar = h0;
-      for (int h = h1 - 1; h >= h0; --h) {
-        const int hc = w.hist[h];
-        if (cum + hc >= P) { bstar = h; break; }
-        cum += hc;
+      const int f = cb * 32 + 31 - lane;  // fine bins of that exponent, top first
+      const int fc = w.hist[f];
+      int fi = fc;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(FULL, fi, o);
+        if (lane >= o) fi += y;
       }
-      w.scal[0] = bstar;
-      w.scal[1] = cum;
-      w.scal[2] = P;
+      const int Lf = __ffs(__ballot_sync(FULL, excl + fi >= P)) - 1;
+      bstar = __shfl_sync(FULL, f, Lf);               // boundary bucket
+      above = __shfl_sync(FULL, excl + fi - fc, Lf);  // tokens in higher buckets
+      Pt = P;
     }
-    for (int h = h0; h < h1; ++h) w.hist[h] = 0;
   }
+  // 3. tokens above / inside the boundary bucket, by index: per-warp counts,
+  //    one scan, then the placements (tmp: above, bnd: boundary bucket)
+  int cu = 0, ca = 0;
+  for (int c = 0; c < nc; ++c) {
+    const int j = (wid * nc + c) * 32 + lane;
+    const int kb = j < N ? w.key[j] : -1;
+    cu += __popc(__ballot_sync(FULL, kb > bstar));
+    ca += __popc(__ballot_sync(FULL, kb >= 0 && kb == bstar));
+  }
+  if (lane == 0) w.wsum[wid] = (cu << 16) | ca;  // cu, ca < 2^15: N <= 8192
   __syncthreads();
-  const int Pt = w.scal[2];
-  const int bstar = w.scal[0];
-  if (Pt > 0) {
-    for (int j0 = wid * 32; j0 < N; j0 += nw * 32) {  // whole warps: aggregated appends
-      const int j = j0 + lane;
-      int k = -1;
-      if (j < N) {
-        const long long v = u[j];
-        if (!sel[j] && v > 0) k = gain_bucket(v);
+  // every warp has read the histograms: clear the bins this thread counted
+  for (int c = 0; c < nc; ++c) {
+    const int j = (wid * nc + c) * 32 + lane;
+    const int kb = j < N ? w.key[j] : -1;
+    if (kb >= 0) {
+      w.hist[kb] = 0;
+      w.coarse[kb >> 5] = 0;
+    }
+  }
+  int pre, nb;
+  {
+    const int x = lane < nw ? w.wsum[lane] : 0;
+    int incl = x;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(FULL, incl, o);
+      if (lane >= o) incl += y;
+    }
+    pre = __shfl_sync(FULL, incl - x, wid);  // this warp's offsets (packed)
+    nb = __shfl_sync(FULL, incl, 31) & 0xFFFF;
+  }
+  int pu = pre >> 16, pa = pre & 0xFFFF;
+  for (int c = 0; c < nc; ++c) {
+    const int j = (wid * nc + c) * 32 + lane;
+    const int kb = j < N ? w.key[j] : -1;
+    const bool up = kb > bstar, at = kb >= 0 && kb == bstar;
+    const unsigned bu = __ballot_sync(FULL, up), ba = __ballot_sync(FULL, at);
+    if (up) {
+      const int slot = pu + __popc(bu & lt);
+      pool[slot] = j;
+      if (poolslot) poolslot[j] = (short)slot;
+    }
+    if (at) w.bnd[pa + __popc(ba & lt)] = j;
+    pu += __popc(bu);
+    pa += __popc(ba);
+  }
+  if (bstar >= 0) {
+    __syncthreads();
+    // 4. the boundary bucket's tokens that enter, ranked exactly by (u desc,
+    //    index asc); they take the slots after the tokens above, by index
+    const int need = Pt - above;
+    for (int q = threadIdx.x; q < nb; q += blockDim.x) {
+      const int j = w.bnd[q];
+      const long long v = u[j];
+      int rank = 0;
+      for (int q2 = 0; q2 < nb; ++q2) {
+        const int j2 = w.bnd[q2];
+        rank += key_before(u[j2], j2, v, j);
       }
-      const bool up = k > bstar, at = k >= 0 && k == bstar;
-      const int pu = warp_append(up, &w.scal[4]);
-      const int pb = warp_append(at, &w.scal[3]);
-      if (up) w.tmp[pu] = j;
-      if (at) w.bnd[pb] = j;
+      w.pk[q] = rank < need;
     }
     __syncthreads();
-    if (bstar >= 0) {
-      const int nb = w.scal[3], need = Pt - w.scal[1];
-      for (int q = threadIdx.x; q < nb; q += blockDim.x) {
-        const int j = w.bnd[q];
-        const long long v = u[j];
-        int rank = 0;
-        for (int q2 = 0; q2 < nb; ++q2) {
-          const int j2 = w.bnd[q2];
-          rank += key_before(u[j2], j2, v, j);
-        }
-        if (rank < need) w.tmp[w.scal[1] + rank] = j;  // after the tokens above the bucket
-      }
-    }
-    __syncthreads();
-    // slot = rank by token index: one 8-lane group per pool token
-    const int gl = lane & 7;
-    const unsigned gm = 0xFFu << (lane & 24);
-    for (int k0 = threadIdx.x >> 3; k0 < Pt; k0 += blockDim.x >> 3) {
-      const int j = w.tmp[k0];
-      const int slot = group_rank_of(w.tmp, Pt, j, gl, gm);
-      if (gl == 0) {
-        pool[slot] = j;
-        if (poolslot) poolslot[j] = (short)slot;
-      }
+    for (int q = threadIdx.x; q < nb; q += blockDim.x) {
+      if (!w.pk[q]) continue;
+      int before = 0;
+      for (int q2 = 0; q2 < q; ++q2) before += w.pk[q2];
+      const int j = w.bnd[q];
+      pool[above + before] = j;
+      if (poolslot) poolslot[j] = (short)(above + before);
     }
   }
   __syncthreads();
