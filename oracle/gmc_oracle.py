@@ -90,6 +90,9 @@ paper, a hand-worked case or brute force on tiny inputs, never by itself):
     (tests/golden/population_transport.txt).
   * compaction_rows / compress: K = N identity; end-to-end invariants on the
     tiny configuration.
+  * gather_prefix_kv: the gathered prefix rows are the source rows at the
+    compaction index map, bit for bit, layer by layer (brute force), and the
+    identity budget returns every layer unchanged.
   * view_patterns / client_matrix_views / compress(history=...): the
     multi-view pattern Gram equals the beta-weighted sum of single-view
     pattern Grams; duplicated views keep the single-view cosines and head
@@ -711,6 +714,20 @@ def compaction_rows(S_sorted: np.ndarray, N: int, T: int) -> np.ndarray:
     return np.concatenate([np.asarray(S_sorted, dtype=np.int64), N + np.arange(T)])
 
 
+def gather_prefix_kv(prefix, rows: np.ndarray):
+    """Cached path: the dense K/V of prefix layers 0..p-1 at the kept sequence rows.
+
+    Appendix "Index map and physical token accounting": the prompt K/V of the
+    blocks before the boundary are gathered, unchanged, at the retained
+    sequence indices (selected visual rows ascending, then every text row);
+    only layers from the boundary on see transported states.  `prefix` lists
+    (K_l, V_l), each [N+T, Hkv, d]; returns [p, 2, len(rows), Hkv, d].
+    """
+    if not prefix:
+        return np.zeros((0, 2, rows.size, 0, 0))
+    return np.stack([np.stack([K_l[rows], V_l[rows]]) for K_l, V_l in prefix])
+
+
 # ---------------------------------------------------------------------------
 # Whole step (Algorithm 1, steps 2-6) for one image
 # ---------------------------------------------------------------------------
@@ -739,11 +756,12 @@ class Result:
     out_hidden: np.ndarray = None  # float64 compact hidden (transported visual rows, text rows)
     out_kv: np.ndarray = None      # [2, K+T, Hkv, d]
     out_pos: np.ndarray = None     # [3, K+T]
+    out_prefix_kv: np.ndarray = None  # [p, 2, K+T, Hkv, d] dense prefix layers at the kept rows
     history: list = None           # per historical view: (A, Z, sigma, unorm, PG, active)
 
 
 def compress(hidden, Kall, Vall, Q, pos, W, gh, gw, K_r, p=None, forced=None,
-             history=None) -> Result:
+             history=None, prefix=None) -> Result:
     """Grounded Message Coreset compression of one image boundary.
 
     hidden [N+T, D], Kall/Vall [N+T, Hkv, d], Q [T, H, d], pos [3, N+T],
@@ -755,6 +773,9 @@ def compress(hidden, Kall, Vall, Q, pos, W, gh, gw, K_r, p=None, forced=None,
     clients"): every view adds its own grounded rows, the head patterns span
     all views, the views share beta_hist equally, and the message energy stays
     the current view's (Eq. (cond-grounded-energy)).
+    ``prefix`` (optional) lists the dense prefix layers' (K, V), each
+    [N+T, Hkv, d]; ``out_prefix_kv`` then holds them at the kept rows
+    (``gather_prefix_kv``).
     """
     p = p or params()
     forced = forced or {}
@@ -765,7 +786,8 @@ def compress(hidden, Kall, Vall, Q, pos, W, gh, gw, K_r, p=None, forced=None,
         rows = np.arange(N + T)
         return Result(K=K, identity=True, support=np.arange(N), rows=rows,
                       out_hidden=np.array(hidden, dtype=np.float64),
-                      out_kv=np.stack([Kall, Vall]), out_pos=np.array(pos))
+                      out_kv=np.stack([Kall, Vall]), out_pos=np.array(pos),
+                      out_prefix_kv=gather_prefix_kv(prefix, rows))
     res = Result(K=K, identity=False)
     hvis = hidden[:N]
     res.A = message_slice(Q, Kall, N)
@@ -805,4 +827,5 @@ def compress(hidden, Kall, Vall, Q, pos, W, gh, gw, K_r, p=None, forced=None,
     res.out_hidden = np.concatenate([res.transport.restored, hidden[N:]], axis=0)
     res.out_kv = np.stack([Kall[res.rows], Vall[res.rows]])
     res.out_pos = np.asarray(pos)[:, res.rows]
+    res.out_prefix_kv = gather_prefix_kv(prefix, res.rows)
     return res

@@ -37,6 +37,8 @@ and probe of an earlier layer for the same image, drawn from their own
 substreams (seed, image, 1 + view) and probe seed (0, 1 + view), so the
 boundary tensors above do not change.  Where the image has object regions,
 the view's visual keys follow the same regions with fresh region centres.
+Dense prefix layers (``prefix_kv``): keys and values of the layers before the
+boundary, N(0, 1) from substreams (seed, image, 100 + layer).
 """
 
 from __future__ import annotations
@@ -202,6 +204,25 @@ class Workload:
         conv = bf16_bits if self.dtype == "bf16" else (lambda a: np.ascontiguousarray(a, np.float32))
         return dict(keys=conv(np.concatenate(kv)), queries=conv(np.concatenate(q)),
                     vo_probe=self.history_view(0, v)["W"])
+
+    def prefix_kv(self, b: int, layer: int) -> dict:
+        """Keys and values [N+T, Hkv, d] of dense prefix layer `layer` of image b
+        (the cached path keeps them at the kept rows), from their own substream
+        (seed, image, 100 + layer); N(0, 1), rounded like the boundary tensors."""
+        rng = np.random.default_rng([self.seed, b, 100 + layer])
+        shape = (self.N + self.T[b], self.Hkv, self.d)
+        return dict(K=self._round(rng.standard_normal(shape, dtype=np.float32)),
+                    V=self._round(rng.standard_normal(shape, dtype=np.float32)))
+
+    def prefix_abi_arrays(self, layer: int) -> np.ndarray:
+        """Prefix layer `layer` of every image in the C-ABI layout of `keys`:
+        [B][2][N+T_b][Hkv][d], K then V."""
+        kv = []
+        for b in range(self.B):
+            pk = self.prefix_kv(b, layer)
+            kv.append(np.stack([pk["K"], pk["V"]]).reshape(-1))
+        conv = bf16_bits if self.dtype == "bf16" else (lambda a: np.ascontiguousarray(a, np.float32))
+        return conv(np.concatenate(kv))
 
     def text_offsets(self) -> np.ndarray:
         return np.concatenate([[0], np.cumsum(self.T)]).astype(np.int32)

@@ -771,3 +771,34 @@ def test_duplicated_current_view_as_history_keeps_head_weights():
     wl, base, res, _ = _tiny_with_history(n_views=2, same_as_current=True)
     np.testing.assert_array_equal(res.heads.centres, base.heads.centres)
     np.testing.assert_allclose(res.heads.omega, base.heads.omega, rtol=1e-12)
+
+
+# --------------------------------------------------------------------------
+# Cached path: dense prefix layers at the kept rows (appendix "Index map and
+# physical token accounting")
+# --------------------------------------------------------------------------
+def test_prefix_kv_gather_is_the_index_map_layer_by_layer():
+    from paper_2608_02134_gb300 import workloads
+    wl = workloads.make("tiny", K=20, T=6)
+    im = wl.image(0)
+    f = lambda a: np.asarray(a, dtype=np.float64)
+    prefix = [(f(wl.prefix_kv(0, l)["K"]), f(wl.prefix_kv(0, l)["V"])) for l in range(3)]
+    res = O.compress(f(im.hidden), f(im.keys), f(im.values), f(im.queries), im.pos,
+                     f(wl.probe()), wl.gh, wl.gw, wl.K, prefix=prefix)
+    N, T = wl.N, 6
+    kept = list(res.support) + list(range(N, N + T))          # brute force, row by row
+    assert res.out_prefix_kv.shape == (3, 2, wl.K + T, wl.Hkv, wl.d)
+    for l, (Kl, Vl) in enumerate(prefix):
+        for r, src in enumerate(kept):
+            assert np.array_equal(res.out_prefix_kv[l, 0, r], Kl[src])
+            assert np.array_equal(res.out_prefix_kv[l, 1, r], Vl[src])
+    # the boundary layer's own K/V follow the same map
+    assert np.array_equal(res.out_kv[0], f(im.keys)[kept])
+    # identity budget: every prefix layer unchanged
+    idn = O.compress(f(im.hidden), f(im.keys), f(im.values), f(im.queries), im.pos,
+                     f(wl.probe()), wl.gh, wl.gw, wl.N, prefix=prefix)
+    for l, (Kl, Vl) in enumerate(prefix):
+        assert np.array_equal(idn.out_prefix_kv[l, 0], Kl) and np.array_equal(idn.out_prefix_kv[l, 1], Vl)
+    none = O.compress(f(im.hidden), f(im.keys), f(im.values), f(im.queries), im.pos,
+                      f(wl.probe()), wl.gh, wl.gw, wl.K)
+    assert none.out_prefix_kv.shape[0] == 0
