@@ -75,6 +75,7 @@ typedef struct CUstream_st* gmc_stream_t; /* identical to cudaStream_t */
 #define GMC_MAX_POOL 128          /* pool_mult * batch_b */
 #define GMC_MAX_HEADS 64          /* H */
 #define GMC_MAX_VIEWS 4           /* message views: the current one and up to 3 historical ones */
+#define GMC_MAX_PREFIX_LAYERS 64  /* dense prefix layers gathered by gmc_compress_ex */
 
 /*
  * Method constants.  gmc_default_params() fills the values of the paper's
@@ -197,6 +198,35 @@ int gmc_compress_views(const gmc_problem* prob, const gmc_params* params, const 
                        int D, int K, int32_t* out_idx, void* out_hidden, void* out_kv,
                        int32_t* out_pos, void* workspace, size_t ws_bytes, void* trace,
                        gmc_stream_t stream);
+
+/*
+ * Dense prefix layers for the cached path (appendix "Index map and physical
+ * token accounting"): the prompt K/V that blocks 0 .. p-1 already computed are
+ * kept, unchanged, at the retained sequence rows -- the selected visual rows
+ * in ascending order, then every text row, the rows out_kv uses -- while the
+ * boundary layer and the layers after it see the transported states.  Layer
+ * l's input has the layout of `keys` ([B][2][N+T_b][Hkv][d], K then V) and
+ * its output the layout of `out_kv` ([B][2][K+T_b][Hkv][d]); the gather is
+ * bit-exact and runs in the same kernel as the compaction.
+ */
+typedef struct gmc_prefix_kv {
+  int n_layers;                              /* p, 0 .. GMC_MAX_PREFIX_LAYERS */
+  const void* keys[GMC_MAX_PREFIX_LAYERS];   /* per layer: device input, as `keys` */
+  void* out_kv[GMC_MAX_PREFIX_LAYERS];       /* per layer: device output, as `out_kv` */
+} gmc_prefix_kv;
+
+/*
+ * gmc_compress_ex -- gmc_compress with historical message views and dense
+ * prefix layers (either may be NULL; both NULL is gmc_compress).  Workspace:
+ * gmc_workspace_size_views with views->n (the prefix layers need none).  The
+ * prefix outputs may not alias any input or other output.
+ */
+int gmc_compress_ex(const gmc_problem* prob, const gmc_params* params, const gmc_views* views,
+                    const gmc_prefix_kv* prefix, const void* hidden, const void* keys,
+                    const void* queries, const int32_t* pos_ids, const float* vo_probe, int N,
+                    int T, int H, int d, int D, int K, int32_t* out_idx, void* out_hidden,
+                    void* out_kv, int32_t* out_pos, void* workspace, size_t ws_bytes,
+                    void* trace, gmc_stream_t stream);
 
 /*
  * Diagnostics trace (optional).  Image b's record starts at byte

@@ -374,7 +374,8 @@ size_t gmc_trace_size(const gmc_problem* prob, const gmc_params* params, int N, 
 // The whole step, or (out_clients != nullptr) its steps up to the client
 // matrix, copied into out_clients.
 static int compress_impl(const gmc_problem* prob, const gmc_params* params,
-                         const gmc_views* views, const void* hidden, const void* keys,
+                         const gmc_views* views, const gmc_prefix_kv* prefix,
+                         const void* hidden, const void* keys,
                          const void* queries, const int32_t* pos_ids, const float* vo_probe,
                          int N, int T, int H, int d, int D, int K, int32_t* out_idx,
                          void* out_hidden, void* out_kv, int32_t* out_pos, void* workspace,
@@ -413,6 +414,18 @@ static int compress_impl(const gmc_problem* prob, const gmc_params* params,
         !aligned(vqueries[v], 16) || !aligned(vprobe[v], 16))
       return GMC_ERR_ARG;
   }
+  // dense prefix layers (cached path), gathered with the compaction
+  PrefixKV pf{};
+  if (prefix && !out_clients) {
+    if (prefix->n_layers < 0 || prefix->n_layers > GMC_MAX_PREFIX_LAYERS) return GMC_ERR_ARG;
+    pf.n = prefix->n_layers;
+    for (int l = 0; l < pf.n; ++l) {
+      pf.keys[l] = prefix->keys[l];
+      pf.out[l] = prefix->out_kv[l];
+      if (!pf.keys[l] || !pf.out[l] || !aligned(pf.keys[l], 16) || !aligned(pf.out[l], 16))
+        return GMC_ERR_ARG;
+    }
+  }
   const int Ke = effective_K(K, N);
   const Dims dm = make_dims(prob, p, N, T, H, d, D, Ke, V);
   Scratch s;
@@ -432,7 +445,7 @@ static int compress_impl(const gmc_problem* prob, const gmc_params* params,
   GMC_TRY(cudaMemsetAsync(s.status, 0, sizeof(uint32_t) * status_words(dm), st));
   if (Ke == N && !out_clients) {  // K = N returns the unmodified execution
     GMC_TRY(launch_identity(dm, hidden, keys, pos_ids, out_idx, out_hidden, out_kv, out_pos,
-                            s.status, st));
+                            s.status, st, &pf));
     g_launches += 1;
     return GMC_OK;
   }
@@ -515,7 +528,7 @@ static int compress_impl(const gmc_problem* prob, const gmc_params* params,
   GMC_STAGE("assign", 2, launch_assign(dm, p, s, tv, st));
   GMC_STAGE("transport", 1,
             launch_transport(dm, p, hidden, keys, pos_ids, s.support, s.pi, s.mass, s.rmsh,
-                             s.mbits, out_idx, out_hidden, out_kv, out_pos, s.status, st));
+                             s.mbits, out_idx, out_hidden, out_kv, out_pos, s.status, st, &pf));
   g_prof.valid = g_prof.on;
   return GMC_OK;
 }
@@ -525,9 +538,9 @@ int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* 
                  const float* vo_probe, int N, int T, int H, int d, int D, int K,
                  int32_t* out_idx, void* out_hidden, void* out_kv, int32_t* out_pos,
                  void* workspace, size_t ws_bytes, void* trace, gmc_stream_t stream_) {
-  return compress_impl(prob, params, nullptr, hidden, keys, queries, pos_ids, vo_probe, N, T, H,
-                       d, D, K, out_idx, out_hidden, out_kv, out_pos, workspace, ws_bytes, trace,
-                       stream_);
+  return compress_impl(prob, params, nullptr, nullptr, hidden, keys, queries, pos_ids, vo_probe,
+                       N, T, H, d, D, K, out_idx, out_hidden, out_kv, out_pos, workspace,
+                       ws_bytes, trace, stream_);
 }
 
 int gmc_compress_views(const gmc_problem* prob, const gmc_params* params, const gmc_views* views,
@@ -536,9 +549,20 @@ int gmc_compress_views(const gmc_problem* prob, const gmc_params* params, const 
                        int D, int K, int32_t* out_idx, void* out_hidden, void* out_kv,
                        int32_t* out_pos, void* workspace, size_t ws_bytes, void* trace,
                        gmc_stream_t stream_) {
-  return compress_impl(prob, params, views, hidden, keys, queries, pos_ids, vo_probe, N, T, H, d,
-                       D, K, out_idx, out_hidden, out_kv, out_pos, workspace, ws_bytes, trace,
-                       stream_);
+  return compress_impl(prob, params, views, nullptr, hidden, keys, queries, pos_ids, vo_probe, N,
+                       T, H, d, D, K, out_idx, out_hidden, out_kv, out_pos, workspace, ws_bytes,
+                       trace, stream_);
+}
+
+int gmc_compress_ex(const gmc_problem* prob, const gmc_params* params, const gmc_views* views,
+                    const gmc_prefix_kv* prefix, const void* hidden, const void* keys,
+                    const void* queries, const int32_t* pos_ids, const float* vo_probe, int N,
+                    int T, int H, int d, int D, int K, int32_t* out_idx, void* out_hidden,
+                    void* out_kv, int32_t* out_pos, void* workspace, size_t ws_bytes,
+                    void* trace, gmc_stream_t stream_) {
+  return compress_impl(prob, params, views, prefix, hidden, keys, queries, pos_ids, vo_probe, N,
+                       T, H, d, D, K, out_idx, out_hidden, out_kv, out_pos, workspace, ws_bytes,
+                       trace, stream_);
 }
 
 int gmc_clients(const gmc_problem* prob, const gmc_params* params, const gmc_views* views,
@@ -547,9 +571,9 @@ int gmc_clients(const gmc_problem* prob, const gmc_params* params, const gmc_vie
                 float* out_clients, void* workspace, size_t ws_bytes, void* trace,
                 gmc_stream_t stream_) {
   if (!out_clients) return GMC_ERR_ARG;
-  return compress_impl(prob, params, views, hidden, keys, queries, pos_ids, vo_probe, N, T, H, d,
-                       D, K, nullptr, nullptr, nullptr, nullptr, workspace, ws_bytes, trace,
-                       stream_, out_clients);
+  return compress_impl(prob, params, views, nullptr, hidden, keys, queries, pos_ids, vo_probe, N,
+                       T, H, d, D, K, nullptr, nullptr, nullptr, nullptr, workspace, ws_bytes,
+                       trace, stream_, out_clients);
 }
 
 // ---------------------------------------------------------------------------

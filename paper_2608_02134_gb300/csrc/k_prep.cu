@@ -184,7 +184,7 @@ template <typename Tin>
 __global__ void k_identity(const Tin* __restrict__ hidden, const Tin* __restrict__ keys,
                            const int32_t* __restrict__ pos, const int32_t* toff, int B, int N,
                            int Tmax, int D, int HD, int32_t* out_idx, Tin* out_hidden,
-                           Tin* out_kv, int32_t* out_pos, uint32_t* status) {
+                           Tin* out_kv, int32_t* out_pos, uint32_t* status, PrefixKV pf) {
   grid_dep_wait();
   const int b = blockIdx.y, r = blockIdx.x;
   const TextGeom tg = text_geom(toff, b, B, Tmax, status);
@@ -201,6 +201,14 @@ __global__ void k_identity(const Tin* __restrict__ hidden, const Tin* __restrict
     uint4* kd = reinterpret_cast<uint4*>(out_kv + sq.out_kv_row(w, r, HD));
     for (int k = threadIdx.x; k < nkv; k += blockDim.x) kd[k] = ks[k];
   }
+  for (int l = 0; l < pf.n; ++l)  // dense prefix layers: unchanged as well
+    for (int w = 0; w < 2; ++w) {
+      const Tin* kl = static_cast<const Tin*>(pf.keys[l]);
+      const uint4* ks = reinterpret_cast<const uint4*>(
+          kl + (w == 0 ? sq.key_row(r, HD) : sq.value_row(r, HD)));
+      uint4* kd = reinterpret_cast<uint4*>(static_cast<Tin*>(pf.out[l]) + sq.out_kv_row(w, r, HD));
+      for (int k = threadIdx.x; k < nkv; k += blockDim.x) kd[k] = ks[k];
+    }
   if (threadIdx.x < 3) out_pos[sq.out_pos(threadIdx.x, r)] = pos[sq.pos(threadIdx.x, r)];
   if (threadIdx.x == 0 && r < N) out_idx[(size_t)b * N + r] = r;
 }
@@ -257,17 +265,20 @@ cudaError_t launch_probe(const Dims& dm, const void* keys, const float* W, const
 
 cudaError_t launch_identity(const Dims& dm, const void* hidden, const void* keys,
                             const int32_t* pos, int32_t* out_idx, void* out_hidden, void* out_kv,
-                            int32_t* out_pos, uint32_t* status, cudaStream_t st) {
+                            int32_t* out_pos, uint32_t* status, cudaStream_t st,
+                            const PrefixKV* prefix) {
   dim3 grid(dm.N + dm.T, dm.B);
   const int HD = dm.Hkv * dm.d;
+  PrefixKV pf{};
+  if (prefix) pf = *prefix;
   if (dm.dtype == GMC_BF16)
     launch_k(k_identity<__nv_bfloat16>, grid, 128, 0, st, 1,
         (const __nv_bfloat16*)hidden, (const __nv_bfloat16*)keys, pos, dm.toff, dm.B, dm.N, dm.T,
-        dm.D, HD, out_idx, (__nv_bfloat16*)out_hidden, (__nv_bfloat16*)out_kv, out_pos, status);
+        dm.D, HD, out_idx, (__nv_bfloat16*)out_hidden, (__nv_bfloat16*)out_kv, out_pos, status, pf);
   else
     launch_k(k_identity<float>, grid, 128, 0, st, 1, (const float*)hidden, (const float*)keys, pos,
                                             dm.toff, dm.B, dm.N, dm.T, dm.D, HD, out_idx,
-                                            (float*)out_hidden, (float*)out_kv, out_pos, status);
+                                            (float*)out_hidden, (float*)out_kv, out_pos, status, pf);
   return cudaGetLastError();
 }
 

@@ -9,7 +9,8 @@
 // and is written to compact row k.  Members are summed in ascending source
 // order, so the result does not depend on scheduling.  Text rows, K/V rows
 // and position ids are gathered bit-exactly at the kept sequence rows
-// [support ascending ; N .. N+T_b-1].
+// [support ascending ; N .. N+T_b-1], and so are the K/V rows of the dense
+// prefix layers when the caller passes them (the cached path).
 #include "common.cuh"
 #include "kernels.cuh"
 
@@ -100,7 +101,7 @@ __global__ void __launch_bounds__(TR_THREADS, 7) k_transport(
     const float* __restrict__ mass, const float* __restrict__ rmsh,
     const uint32_t* __restrict__ mbits, const int32_t* toff, int B, int N, int K, int Tmax, int D,
     int HD, int S, float rms_eps, int check, int32_t* out_idx, Tin* out_hidden, Tin* out_kv,
-    int32_t* out_pos, uint32_t* status) {
+    int32_t* out_pos, uint32_t* status, PrefixKV pf) {
   grid_dep_wait();
   constexpr int NW = TR_THREADS / 32;
   constexpr int NM = TR_WIN * NW;  // 32-token masks per window
@@ -175,6 +176,25 @@ __global__ void __launch_bounds__(TR_THREADS, 7) k_transport(
       *kv_dst(dst, q) = *kv_src(src, q);
     if (part == 0 && threadIdx.x < 3) out_pos[sq.out_pos(threadIdx.x, dst)] = stpos[slot][threadIdx.x];
   };
+  // the dense prefix layers' K/V of kept row src, written to output row dst;
+  // the loads of PL layers are in flight together
+  auto copy_prefix = [&](int src, int dst) {
+    constexpr int PL = 8;
+    for (int l0 = 0; l0 < pf.n; l0 += PL)
+      for (int q = part * TR_THREADS + threadIdx.x; q < 2 * nkv; q += S * TR_THREADS) {
+        const int wv = q >= nkv, e = q - wv * nkv;
+        const size_t ro = wv == 0 ? sq.key_row(src, HD) : sq.value_row(src, HD);
+        const size_t wo = sq.out_kv_row(wv, dst, HD);
+        uint4 v[PL];
+#pragma unroll
+        for (int u = 0; u < PL; ++u)
+          if (l0 + u < pf.n)
+            v[u] = reinterpret_cast<const uint4*>(static_cast<const Tin*>(pf.keys[l0 + u]) + ro)[e];
+#pragma unroll
+        for (int u = 0; u < PL; ++u)
+          if (l0 + u < pf.n) reinterpret_cast<uint4*>(static_cast<Tin*>(pf.out[l0 + u]) + wo)[e] = v[u];
+      }
+  };
   // this CTA's slice of D, in 8-element chunks
   const int nch = D / TR_VEC, cper = ceil_div(nch, S);
   const int c = part * cper + threadIdx.x;
@@ -201,8 +221,12 @@ __global__ void __launch_bounds__(TR_THREADS, 7) k_transport(
         for (int q = 0; q < U; ++q) dp[q] = stage[q][threadIdx.x];
       }
       flush_kv_pos(N + r, K + r, 0);
+      copy_prefix(N + r, K + r);
     }
-    if (car) flush_kv_pos(j, r, 1);
+    if (car) {
+      flush_kv_pos(j, r, 1);
+      copy_prefix(j, r);
+    }
   };
   if (!car) {
     flush_all();
@@ -338,8 +362,11 @@ cudaError_t launch_transport(const Dims& dm, const gmc_params& p, const void* hi
                              const void* keys, const int32_t* pos, const int32_t* support,
                              const int32_t* pi, const float* mass, const float* rmsh,
                              const uint32_t* mbits, int32_t* out_idx, void* out_hidden,
-                             void* out_kv, int32_t* out_pos, uint32_t* status, cudaStream_t st) {
+                             void* out_kv, int32_t* out_pos, uint32_t* status, cudaStream_t st,
+                             const PrefixKV* prefix) {
   const int S = transport_split(dm.D);
+  PrefixKV pf{};
+  if (prefix) pf = *prefix;
   const int HD = dm.Hkv * dm.d;
   // mbits: the carrier membership bitmaps, or nullptr to scan the assignment
   cudaLaunchConfig_t cfg = {};
@@ -362,13 +389,13 @@ cudaError_t launch_transport(const Dims& dm, const gmc_params& p, const void* hi
     return cudaLaunchKernelEx(&cfg, k_transport<T>, (const T*)hidden, (const T*)keys, pos, support,
                               pi, mass, rmsh, mbits, (const int32_t*)dm.toff, dm.B, dm.N, dm.K, dm.T,
                               dm.D, HD, S, p.rms_eps, p.check_mode, out_idx, (T*)out_hidden,
-                              (T*)out_kv, out_pos, status);
+                              (T*)out_kv, out_pos, status, pf);
   }
   return cudaLaunchKernelEx(&cfg, k_transport<float>, (const float*)hidden, (const float*)keys,
                             pos, support, pi, mass, rmsh, mbits, (const int32_t*)dm.toff, dm.B,
                             dm.N,
                             dm.K, dm.T, dm.D, HD, S, p.rms_eps, p.check_mode, out_idx,
-                            (float*)out_hidden, (float*)out_kv, out_pos, status);
+                            (float*)out_hidden, (float*)out_kv, out_pos, status, pf);
 }
 
 }  // namespace gmc

@@ -57,6 +57,14 @@ struct ViewGrams {
   float beta[MAX_VIEWS];
 };
 
+// Dense prefix layers gathered at the kept rows with the compaction (passed
+// by value to the transport and identity kernels; n = 0: none).
+struct PrefixKV {
+  int n;
+  const void* keys[GMC_MAX_PREFIX_LAYERS];
+  void* out[GMC_MAX_PREFIX_LAYERS];
+};
+
 // Device scratch carved out of the caller's workspace.
 struct Scratch {
   uint32_t* status;
@@ -163,10 +171,10 @@ cudaError_t launch_transport(const Dims&, const gmc_params&, const void* hidden,
                              const int32_t* pos, const int32_t* support, const int32_t* pi,
                              const float* mass, const float* rmsh, const uint32_t* mbits,
                              int32_t* out_idx, void* out_hidden, void* out_kv, int32_t* out_pos,
-                             uint32_t* status, cudaStream_t);
+                             uint32_t* status, cudaStream_t, const PrefixKV* prefix = nullptr);
 cudaError_t launch_identity(const Dims&, const void* hidden, const void* keys, const int32_t* pos,
                             int32_t* out_idx, void* out_hidden, void* out_kv, int32_t* out_pos,
-                            uint32_t* status, cudaStream_t);
+                            uint32_t* status, cudaStream_t, const PrefixKV* prefix = nullptr);
 cudaError_t launch_rms_rows(const Dims&, const void* hidden, float* rmsh, uint32_t* status,
                             cudaStream_t);
 

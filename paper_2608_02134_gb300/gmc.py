@@ -28,8 +28,10 @@ EXPORTS = (
     "gmc_version", "gmc_profile_enable", "gmc_profile_read", "gmc_launch_count",
     "gmc_transport_noalloc", "gmc_cosine_workspace_size", "gmc_cosine",
     "gmc_workspace_size_views", "gmc_compress_views", "gmc_clients", "gmc_selftest_bounded_wait",
+    "gmc_compress_ex",
 )
 MAX_VIEWS = 4
+MAX_PREFIX_LAYERS = 64
 
 
 class Params(ctypes.Structure):
@@ -58,6 +60,12 @@ class Views(ctypes.Structure):
                 ("keys", ctypes.c_void_p * (MAX_VIEWS - 1)),
                 ("queries", ctypes.c_void_p * (MAX_VIEWS - 1)),
                 ("vo_probe", ctypes.c_void_p * (MAX_VIEWS - 1))]
+
+
+class PrefixKV(ctypes.Structure):
+    _fields_ = [("n_layers", ctypes.c_int),
+                ("keys", ctypes.c_void_p * MAX_PREFIX_LAYERS),
+                ("out_kv", ctypes.c_void_p * MAX_PREFIX_LAYERS)]
 
 
 class TraceHeader(ctypes.Structure):
@@ -133,6 +141,9 @@ def lib() -> ctypes.CDLL:
     L.gmc_cosine_workspace_size.restype = sz
     L.gmc_cosine.argtypes = [PP, P, vp, i, i, i, vp, vp, sz, vp]
     L.gmc_cosine.restype = i
+    L.gmc_compress_ex.argtypes = [PP, P, ctypes.POINTER(Views), ctypes.POINTER(PrefixKV), vp, vp,
+                                  vp, vp, vp, i, i, i, i, i, i, vp, vp, vp, vp, vp, sz, vp, vp]
+    L.gmc_compress_ex.restype = i
     L.gmc_clients.argtypes = [PP, P, ctypes.POINTER(Views), vp, vp, vp, vp, vp, i, i, i, i, i, i,
                               vp, vp, sz, vp, vp]
     L.gmc_clients.restype = i
@@ -208,6 +219,29 @@ def views(keys, queries, vo_probe, beta_hist=0.5) -> Views:
     for k in range(v.n):
         v.keys[k], v.queries[k], v.vo_probe[k] = _ptr(keys[k]), _ptr(queries[k]), _ptr(vo_probe[k])
     return v
+
+
+def prefix_kv(keys, outs) -> PrefixKV:
+    """Dense prefix layers from per-layer device tensors (inputs as `keys`, outputs as `out_kv`)."""
+    if len(keys) != len(outs) or len(keys) > MAX_PREFIX_LAYERS:
+        raise GMCError("prefix layers: one output per input, at most 64")
+    pf = PrefixKV()
+    pf.n_layers = len(keys)
+    for l, (k, o) in enumerate(zip(keys, outs)):
+        pf.keys[l], pf.out_kv[l] = _ptr(k), _ptr(o)
+    return pf
+
+
+def compress_ex(prob: Problem, params: Params, vw, pf, hidden, keys, queries, pos_ids, vo_probe,
+                N, T, H, d, D, K, out_idx, out_hidden, out_kv, out_pos, workspace, trace=None,
+                stream=None):
+    """gmc_compress_ex on device tensors (vw, pf: Views / PrefixKV or None; see include/gmc.h)."""
+    _check(lib().gmc_compress_ex(
+        ctypes.byref(prob), ctypes.byref(params), ctypes.byref(vw) if vw is not None else None,
+        ctypes.byref(pf) if pf is not None else None, _ptr(hidden), _ptr(keys), _ptr(queries),
+        _ptr(pos_ids), _ptr(vo_probe), N, T, H, d, D, K, _ptr(out_idx), _ptr(out_hidden),
+        _ptr(out_kv), _ptr(out_pos), _ptr(workspace), workspace.numel(), _ptr(trace),
+        _stream(stream)))
 
 
 def workspace_size_views(prob: Problem, n_views, N, T, H, d, D, K) -> int:
@@ -365,9 +399,21 @@ class Compressor:
             self.trace = torch.zeros(B * self.layout.bytes_per_image, dtype=torch.uint8, device=device)
 
     def run(self, hidden, keys, queries, pos_ids, vo_probe, stream=None, history=None,
-            beta_hist=0.5):
-        """history: None, or (keys, queries, vo_probe) lists of the historical views."""
-        if history is None:
+            beta_hist=0.5, prefix=None):
+        """history: None, or (keys, queries, vo_probe) lists of the historical views;
+        prefix: None, or the dense prefix layers' K/V tensors (layout of `keys`),
+        gathered into self.out_prefix (one tensor per layer, layout of out_kv)."""
+        if prefix is not None:
+            if history is not None and len(history[0]) > self.n_views:
+                raise GMCError("more historical views than the workspace was sized for")
+            if getattr(self, "out_prefix", None) is None or len(self.out_prefix) != len(prefix):
+                self.out_prefix = [torch.empty_like(self.out_kv) for _ in prefix]
+            vw = views(*history, beta_hist=beta_hist) if history is not None else None
+            compress_ex(self.prob, self.params, vw, prefix_kv(prefix, self.out_prefix), hidden,
+                        keys, queries, pos_ids, vo_probe, self.N, self.T, self.H, self.d, self.D,
+                        self.Kr, self.out_idx, self.out_hidden, self.out_kv, self.out_pos,
+                        self.workspace, self.trace, stream)
+        elif history is None:
             compress(self.prob, self.params, hidden, keys, queries, pos_ids, vo_probe, self.N,
                      self.T, self.H, self.d, self.D, self.Kr, self.out_idx, self.out_hidden,
                      self.out_kv, self.out_pos, self.workspace, self.trace, stream)

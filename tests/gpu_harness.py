@@ -24,6 +24,7 @@ class GpuRun:
     status: int
     traces: list
     n_hist: int = 0
+    prefix: list = None     # per dense prefix layer: gathered K/V (float64 values), layout of kv
 
 
 def to_device(wl: workloads.Workload, device="cuda"):
@@ -46,7 +47,8 @@ def _dev(a, device="cuda"):
     return t.to(device)
 
 
-def run(wl: workloads.Workload, params=None, trace=True, inputs=None, n_hist=0) -> GpuRun:
+def run(wl: workloads.Workload, params=None, trace=True, inputs=None, n_hist=0,
+        n_prefix=0) -> GpuRun:
     dt = gmc.GMC_BF16 if wl.dtype == "bf16" else gmc.GMC_F32
     inp = inputs or to_device(wl)
     comp = gmc.Compressor(wl.B, wl.gh, wl.gw, wl.T_max, wl.H, wl.Hkv, wl.d, wl.D, wl.K, dt,
@@ -57,8 +59,9 @@ def run(wl: workloads.Workload, params=None, trace=True, inputs=None, n_hist=0) 
         hv = [wl.history_abi_arrays(v) for v in range(n_hist)]
         history = ([_dev(h["keys"]) for h in hv], [_dev(h["queries"]) for h in hv],
                    [_dev(h["vo_probe"]) for h in hv])
+    prefix = [_dev(wl.prefix_abi_arrays(l)) for l in range(n_prefix)] if n_prefix else None
     out = comp.run(inp["hidden"], inp["keys"], inp["queries"], inp["pos_ids"], inp["vo_probe"],
-                   history=history)
+                   history=history, prefix=prefix)
     torch.cuda.synchronize()
     status = comp.status()
     hid = out.hidden.float().cpu().numpy().astype(np.float64)
@@ -68,8 +71,9 @@ def run(wl: workloads.Workload, params=None, trace=True, inputs=None, n_hist=0) 
     if trace:
         traces = parity.parse_trace(out.trace.cpu().numpy(), out.layout, wl.B, comp.K, wl.H, wl.N,
                                     comp.params.max_head_clusters)
+    pref = [t.float().cpu().numpy() for t in comp.out_prefix] if n_prefix else None
     return GpuRun(wl, comp, out.idx.cpu().numpy(), hid, raw, out.kv.float().cpu().numpy(),
-                  out.pos.cpu().numpy(), status, traces, n_hist)
+                  out.pos.cpu().numpy(), status, traces, n_hist, pref)
 
 
 def oracle_params(p: gmc.Params) -> dict:
@@ -109,8 +113,12 @@ def compare_image(g: GpuRun, b: int, hidden_tol: float) -> ImageReport:
     history = None
     if g.n_hist:
         history = [{k: f(a) for k, a in wl.history_view(b, v).items()} for v in range(g.n_hist)]
+    prefix = None
+    if g.prefix:
+        prefix = [(f(wl.prefix_kv(b, l)["K"]), f(wl.prefix_kv(b, l)["V"]))
+                  for l in range(len(g.prefix))]
     res = O.compress(f(im.hidden), f(im.keys), f(im.values), f(im.queries), im.pos, f(wl.probe()),
-                     wl.gh, wl.gw, wl.K, p, forced=forced, history=history)
+                     wl.gh, wl.gw, wl.K, p, forced=forced, history=history, prefix=prefix)
     dec = parity.Decisions()
     tag = f"{wl.name}[b={b}]"
     parity.check_heads(res.heads, dec, tag)
@@ -130,6 +138,11 @@ def compare_image(g: GpuRun, b: int, hidden_tol: float) -> ImageReport:
     kvo = g.kv[2 * o:2 * (o + K + T)].reshape(2, K + T, wl.Hkv, wl.d)
     if not np.array_equal(kvo, res.out_kv):
         dec.failures.append(f"{tag} compact K/V rows differ")
+    if g.prefix:
+        for l, pl in enumerate(g.prefix):
+            got = pl[2 * o:2 * (o + K + T)].reshape(2, K + T, wl.Hkv, wl.d)
+            if not np.array_equal(got, res.out_prefix_kv[l]):
+                dec.failures.append(f"{tag} prefix layer {l} K/V rows differ")
     pos = g.pos[3 * o:3 * (o + K + T)].reshape(3, K + T)
     if not np.array_equal(pos, res.out_pos):
         dec.failures.append(f"{tag} position ids differ")

@@ -179,3 +179,31 @@ def test_responsibility_temperature(resp_temp):
     wl = workloads.make("qwen", gh=18, gw=18, T=24, D=128, H=8, Hkv=2, K=60)
     g = GH.run(wl, params=gmc.default_params(resp_temp=resp_temp))
     _check(g, [0], TOL_BF16)
+
+
+def test_prefix_layers_qwen_shape():
+    """Cached path: two dense prefix layers gathered bit-exactly at the kept rows."""
+    from paper_2608_02134_gb300 import workloads
+    from tests import gpu_harness as GH
+    wl = workloads.make("qwen")
+    _check(GH.run(wl, n_prefix=2), [0], TOL_BF16)
+
+
+def test_prefix_layers_ragged_batch_with_views():
+    from paper_2608_02134_gb300 import workloads
+    from tests import gpu_harness as GH
+    wl = workloads.make("qwen", B=3, T=[20, 7, 33], gh=12, gw=12, D=64, H=8, Hkv=2, K=30)
+    _check(GH.run(wl, n_prefix=9, n_hist=2), [0, 1, 2], TOL_BF16)
+
+
+def test_prefix_layers_fp32_and_identity():
+    from paper_2608_02134_gb300 import workloads
+    from tests import gpu_harness as GH
+    wl = workloads.make("tiny")
+    _check(GH.run(wl, n_prefix=1), [0], TOL_F32)
+    wl2 = workloads.make("tiny", K=64)                        # K = N: every layer unchanged
+    g = GH.run(wl2, trace=False, n_prefix=3)
+    for l in range(3):
+        pk = wl2.prefix_kv(0, l)
+        ref = np.stack([pk["K"], pk["V"]]).reshape(-1).astype(np.float64)
+        assert np.array_equal(g.prefix[l].reshape(-1), ref)
