@@ -45,6 +45,10 @@ Readings taken where the paper is silent or ambiguous:
     support has one element.
   * Transport blend tau_j = 1 (appendix form); rms(u) = sqrt(mean u^2),
     epsilon 1e-6.
+  * Multi-image prompts: I images of equal grids lie one after another in
+    the visual segment; coordinates, landmarks and the assignment's spatial
+    term use each image's own grid; the seed round picks one max-gain token
+    per image before the responsibility rounds.
   * Historical message views (optional): the configuration table's
     "current/history mass 0.5/0.5" is read as a current-view grounded mass
     beta_G = 0.5 and a history mass beta_hist = 0.5 shared equally by the
@@ -90,6 +94,13 @@ paper, a hand-worked case or brute force on tiny inputs, never by itself):
     (tests/golden/population_transport.txt).
   * compaction_rows / compress: K = N identity; end-to-end invariants on the
     tiny configuration.
+  * multi-image prompts (image_index and the n_images arguments): each
+    image's appearance block is the single-image bank of that image and zero
+    elsewhere; spatial landmarks repeat per image, block-diagonal; the seeds
+    are every image's best singleton gain (brute force) and a budget below
+    the image count keeps exactly them; clusters never cross images and the
+    gap uses same-image carriers only (brute force); two copies of one image
+    assign exactly like the image alone; one image is the single-image path.
   * gather_prefix_kv: the gathered prefix rows are the source rows at the
     compaction index map, bit for bit, layer by layer (brute force), and the
     identity budget returns every layer unchanged.
@@ -390,9 +401,22 @@ def cosine_matrix(hvis: np.ndarray, p: dict) -> np.ndarray:
     return x @ x.T
 
 
-def appearance_clients(cos: np.ndarray, p: dict) -> np.ndarray:
-    """P^V_m(i) proportional to exp(x_m^T x_i / tau_v), each row normalised.  [N, N]."""
+def image_index(N: int, n_images: int = 1) -> np.ndarray:
+    """Image I_i of every visual token: n_images equal grids laid out one after
+    another (tokens [k N/I, (k+1) N/I) belong to image k)."""
+    return np.arange(N) // (N // n_images)
+
+
+def appearance_clients(cos: np.ndarray, p: dict, n_images: int = 1) -> np.ndarray:
+    """P^V_m(i) proportional to exp(x_m^T x_i / tau_v), each row normalised.  [N, N].
+
+    With several images a row covers the tokens of its own image only
+    (appendix "Appearance and spatial clients", last paragraphs).
+    """
     logits = cos / p["tau_v"]
+    if n_images > 1:
+        img = image_index(cos.shape[0], n_images)
+        logits = np.where(img[:, None] == img[None, :], logits, -np.inf)
     logits = logits - logits.max(axis=1, keepdims=True)
     E = np.exp(logits)
     return E / E.sum(axis=1, keepdims=True)
@@ -410,15 +434,27 @@ def landmark_coords(n: int) -> np.ndarray:
     return np.stack([(a + 0.5) / n, (b + 0.5) / n], axis=1)
 
 
-def spatial_clients(gh: int, gw: int, p: dict) -> np.ndarray:
-    """P^S_l(i) proportional to exp(-||p_i - l_l||^2 / tau_s), rows normalised (one image)."""
+def spatial_clients(gh: int, gw: int, p: dict, n_images: int = 1) -> np.ndarray:
+    """P^S_l(i) proportional to 1[I_i = I_l] exp(-||p_i - l_l||^2 / tau_s), rows normalised.
+
+    Every image has its own landmark grid in its normalised coordinates
+    (Eq. (cond-aux-clients)): rows (image k, landmark l), k-major, each over
+    image k's tokens.  [n_images * L^2, n_images * gh * gw].
+    """
     P = grid_coords(gh, gw)
     Lm = landmark_coords(p["landmarks"])
     d2 = np.sum((Lm[:, None, :] - P[None, :, :]) ** 2, axis=2)
     logits = -d2 / p["tau_s"]
     logits = logits - logits.max(axis=1, keepdims=True)
     E = np.exp(logits)
-    return E / E.sum(axis=1, keepdims=True)
+    one = E / E.sum(axis=1, keepdims=True)
+    if n_images == 1:
+        return one
+    L2, Ng = one.shape
+    out = np.zeros((n_images * L2, n_images * Ng))
+    for k in range(n_images):
+        out[k * L2:(k + 1) * L2, k * Ng:(k + 1) * Ng] = one
+    return out
 
 
 # ---------------------------------------------------------------------------
@@ -508,6 +544,7 @@ class SelectRound:
     F_before: float
     F_after: float
     U: float                   # sum of the K largest remaining singleton gains
+    seed: bool = False         # multi-image seed round: one max-gain token per image
 
 
 @dataclass
@@ -521,7 +558,8 @@ class Selection:
         return np.array(sorted(self.order), dtype=np.int64)
 
 
-def select_support(C: np.ndarray, K: int, p: dict, forced=None, mode: str = "responsibility") -> Selection:
+def select_support(C: np.ndarray, K: int, p: dict, forced=None, mode: str = "responsibility",
+                   n_images: int = 1) -> Selection:
     """Deployed batched solver until |S| = K.
 
     Round t (support S_t, b_m = max_{j in S_t} C_mj, b = 0 for S empty):
@@ -538,6 +576,11 @@ def select_support(C: np.ndarray, K: int, p: dict, forced=None, mode: str = "res
     empty pool and its filled tokens as batch).  When given, the oracle
     computes its own values, records them, then continues with the forced
     choice.
+
+    n_images > 1: S starts with the token of largest singleton gain of every
+    image (ties to the lowest index), recorded as a first "seed" round whose
+    pool and batch are those tokens (Sec. 3.3; appendix "Batched
+    complementary support"; Algorithm 1 step 3).
     """
     M, N = C.shape
     bsz = p["batch_b"] if mode == "responsibility" else 1
@@ -547,6 +590,19 @@ def select_support(C: np.ndarray, K: int, p: dict, forced=None, mode: str = "res
     sel = Selection(order=[], K=K)
     ids = np.arange(N)
     rnd = 0
+    if n_images > 1:
+        u = C.sum(axis=0)  # S empty: every client value is a residual
+        img = image_index(N, n_images)
+        own = np.array([int(stable_top(u[img == k], ids[img == k], 1)[0]) for k in range(n_images)])
+        f = forced[0] if forced is not None else None
+        seeds = np.asarray(f[1], dtype=np.int64) if f is not None else own
+        selected[seeds] = True
+        sel.order.extend(int(i) for i in seeds)
+        bm = C[:, seeds].max(axis=1)
+        remaining = np.sort(u)[::-1]
+        sel.rounds.append(SelectRound(u, own, own, u[own], own, seeds, False, 0.0,
+                                      float(bm.sum()), float(remaining[:K].sum()), seed=True))
+        rnd = 1
     while len(sel.order) < K:
         R = np.maximum(C - bm[:, None], 0.0)
         u = R.sum(axis=0)
@@ -632,7 +688,7 @@ class Assignment:
 
 
 def assign_population(cos: np.ndarray, S: np.ndarray, gh: int, gw: int, p: dict,
-                      forced_pi=None) -> Assignment:
+                      forced_pi=None, n_images: int = 1) -> Assignment:
     """pi(i) = argmax_{j in S} cos_ij + lambda_p s_x g_i exp(-||p_i - p_j||^2 / tau_s).
 
     Selected tokens represent themselves.  delta_i is the gap between the
@@ -640,31 +696,36 @@ def assign_population(cos: np.ndarray, S: np.ndarray, gh: int, gw: int, p: dict,
     its mean over discarded tokens (0 when none is discarded);
     s_x = 1 - exp[-(Delta_bar / gate_scale)^gate_pow];
     g_i = exp[-(delta_i / ambig_margin)^gate_pow].  Ties go to the lowest j.
+    With several images, token i's candidates S_i are the selected tokens of
+    its own image, and both the gap and the coordinates are within that image.
     """
     N = cos.shape[0]
     S = np.asarray(S, dtype=np.int64)
     in_S = np.zeros(N, bool)
     in_S[S] = True
     disc = np.flatnonzero(~in_S)
+    img = image_index(N, n_images)
+    compat = {int(i): S[img[S] == img[i]] for i in disc}  # S_i: same-image carriers
     delta = np.zeros(N)
     for i in disc:
-        v = np.sort(cos[i, S])[::-1]
+        v = np.sort(cos[i, compat[int(i)]])[::-1]
         delta[i] = v[0] - v[1] if v.size > 1 else 0.0
     delta_bar = float(delta[disc].mean()) if disc.size else 0.0
     s_x = 1.0 - math.exp(-((delta_bar / p["gate_scale"]) ** p["gate_pow"]))
     g = np.exp(-((delta / p["ambig_margin"]) ** p["gate_pow"]))
-    P = grid_coords(gh, gw)
-    slot = {int(j): k for k, j in enumerate(S)}
+    P = np.tile(grid_coords(gh, gw), (n_images, 1))  # coordinates in each token's own grid
     pi = np.arange(N)
     kb = np.zeros(N)
     kc = np.zeros(N)
     for i in disc:
-        d2 = np.sum((P[S] - P[i]) ** 2, axis=1)
-        kappa = cos[i, S] + p["assign_spatial_w"] * s_x * g[i] * np.exp(-d2 / p["tau_s"])
-        j = int(stable_top(kappa, S, 1)[0])
+        Si = compat[int(i)]
+        d2 = np.sum((P[Si] - P[i]) ** 2, axis=1)
+        kappa = cos[i, Si] + p["assign_spatial_w"] * s_x * g[i] * np.exp(-d2 / p["tau_s"])
+        j = int(stable_top(kappa, Si, 1)[0])
         pi[i] = j if forced_pi is None else int(forced_pi[i])
         kb[i] = kappa.max()
-        kc[i] = kappa[slot[int(pi[i])]] if int(pi[i]) in slot else -np.inf
+        hit = np.flatnonzero(Si == pi[i])
+        kc[i] = kappa[hit[0]] if hit.size else -np.inf
     if forced_pi is not None:
         pi[S] = np.asarray(forced_pi)[S]
     return Assignment(pi, delta, delta_bar, s_x, g, kb, kc)
@@ -761,7 +822,7 @@ class Result:
 
 
 def compress(hidden, Kall, Vall, Q, pos, W, gh, gw, K_r, p=None, forced=None,
-             history=None, prefix=None) -> Result:
+             history=None, prefix=None, n_images: int = 1) -> Result:
     """Grounded Message Coreset compression of one image boundary.
 
     hidden [N+T, D], Kall/Vall [N+T, Hkv, d], Q [T, H, d], pos [3, N+T],
@@ -773,15 +834,18 @@ def compress(hidden, Kall, Vall, Q, pos, W, gh, gw, K_r, p=None, forced=None,
     clients"): every view adds its own grounded rows, the head patterns span
     all views, the views share beta_hist equally, and the message energy stays
     the current view's (Eq. (cond-grounded-energy)).
+    ``n_images`` > 1: a multi-image prompt whose visual segment holds that many
+    images of gh x gw tokens one after another (budget, seeds, banks and
+    assignment per image as the paper states; see the functions above).
     ``prefix`` (optional) lists the dense prefix layers' (K, V), each
     [N+T, Hkv, d]; ``out_prefix_kv`` then holds them at the kept rows
     (``gather_prefix_kv``).
     """
     p = p or params()
     forced = forced or {}
-    N = gh * gw
+    N = gh * gw * n_images
     T, H, d = Q.shape
-    K = budget(K_r, N)
+    K = budget(K_r, N, n_images)
     if K == N:   # K = N returns the unmodified execution
         rows = np.arange(N + T)
         return Result(K=K, identity=True, support=np.arange(N), rows=rows,
@@ -810,17 +874,19 @@ def compress(hidden, Kall, Vall, Q, pos, W, gh, gw, K_r, p=None, forced=None,
                               forced.get("centres"), forced.get("head_assign"), views=views)
     res.e, res.ebar = message_energy(res.unorm, res.heads.omega, res.nu)
     res.cos = cosine_matrix(hvis, p)
-    PV = appearance_clients(res.cos, p)
-    PS = spatial_clients(gh, gw, p)
+    PV = appearance_clients(res.cos, p, n_images)
+    PS = spatial_clients(gh, gw, p, n_images)
     if history is None:
         res.clients = client_matrix(res.PG, res.activeG, res.heads.omega, res.nu, PV, PS, p)
     else:
         res.clients = client_matrix_views(
             [res.PG] + [hv[4] for hv in res.history], [res.activeG] + [hv[5] for hv in res.history],
             [v[3] for v in views], res.heads.omega, res.nu, PV, PS, p)
-    res.selection = select_support(res.clients.C, K, p, forced=forced.get("rounds"))
+    res.selection = select_support(res.clients.C, K, p, forced=forced.get("rounds"),
+                                   n_images=n_images)
     res.support = res.selection.support
-    res.assignment = assign_population(res.cos, res.support, gh, gw, p, forced.get("pi"))
+    res.assignment = assign_population(res.cos, res.support, gh, gw, p, forced.get("pi"),
+                                       n_images)
     res.m = population_weights(res.ebar, res.assignment.s_x, p)
     res.transport = transport(hvis, res.support, res.assignment.pi, res.m, p)
     res.rows = compaction_rows(res.support, N, T)

@@ -23,6 +23,9 @@ no benchmark image, prompt or checkpoint is used):
            w_i ~ N(0,I_32), and 200 seeded rows replaced by fresh N(0,I_D).
   serving  32 independent qwen-shaped images, T_b ~ U[16,256] (seeded),
            K=257 each, one call.
+  multi    one prompt with two qwen-shaped images (N = 2 x 1296, each 36x36,
+           one after the other), T=64, K=514 (20%), bf16; every image drawn
+           like a qwen image from its own substream (seed, 0, 1000 + image).
 
 Values are drawn in fp32; bf16 workloads round them once to bf16 (round to
 nearest even) and every consumer reads the rounded values.  Values V ~ N(0,1).
@@ -54,7 +57,10 @@ WORKLOADS = {
     "qwen": (2, 1, 36, 36, 64, 28, 4, 128, 3584, 257, "bf16", "regions+detail", "mrope"),
     "doc": (3, 1, 64, 64, 128, 28, 4, 128, 3584, 410, "bf16", "lowrank", "mrope"),
     "serving": (4, 32, 36, 36, None, 28, 4, 128, 3584, 257, "bf16", "regions+detail", "mrope"),
+    # multi-image prompt: two qwen-shaped images (2 x 36 x 36 visual tokens) before the text
+    "multi": (5, 1, 36, 36, 64, 28, 4, 128, 3584, 514, "bf16", "regions+detail", "mrope"),
 }
+IMAGES = {"multi": 2}  # images per boundary (1 when absent)
 
 
 def round_to_bf16(x: np.ndarray) -> np.ndarray:
@@ -96,11 +102,17 @@ class Workload:
     dtype: str
     structure: str
     positions: str
+    I: int = 1  # images per boundary (a multi-image prompt when > 1)
     _cache: dict = field(default_factory=dict, repr=False)
 
     @property
-    def N(self) -> int:
+    def Ng(self) -> int:
+        """Visual tokens of one image (its grid)."""
         return self.gh * self.gw
+
+    @property
+    def N(self) -> int:
+        return self.gh * self.gw * self.I
 
     @property
     def T_max(self) -> int:
@@ -124,8 +136,65 @@ class Workload:
         x = np.asarray(x, dtype=np.float32)
         return round_to_bf16(x) if self.dtype == "bf16" else x
 
+    def _visual(self, rng, f32):
+        """One image's visual hidden rows, keys, values and regions (multi-image
+        prompts), drawn like the single-image rows below."""
+        Ng, D, Hkv, d = self.Ng, self.D, self.Hkv, self.d
+        hidden = rng.standard_normal((Ng, D), dtype=f32)
+        keys = rng.standard_normal((Ng, Hkv, d), dtype=f32)
+        values = rng.standard_normal((Ng, Hkv, d), dtype=f32)
+        region = None
+        if self.structure.startswith("regions"):
+            n_reg = 8
+            seeds = rng.choice(Ng, size=n_reg, replace=False)
+            sr, sc = np.divmod(seeds, self.gw)
+            r, c = np.divmod(np.arange(Ng), self.gw)
+            dist = (r[:, None] - sr[None, :]) ** 2 + (c[:, None] - sc[None, :]) ** 2
+            region = np.argmin(dist, axis=1)
+            mu = rng.standard_normal((n_reg, D), dtype=f32)
+            kap = rng.standard_normal((n_reg, Hkv, d), dtype=f32)
+            hidden = mu[region] + f32(0.3) * rng.standard_normal((Ng, D), dtype=f32)
+            keys = kap[region] + f32(0.3) * rng.standard_normal((Ng, Hkv, d), dtype=f32)
+            if self.structure == "regions+detail":
+                typical = float(np.mean(np.linalg.norm(hidden, axis=1)))
+                for k in range(n_reg):
+                    members = np.flatnonzero(region == k)
+                    pick = rng.choice(members, size=min(2, members.size), replace=False)
+                    for i in pick:
+                        v = rng.standard_normal(D, dtype=f32)
+                        hidden[i] = f32(5.0 * typical) * v / np.linalg.norm(v)
+        return hidden, keys, values, region
+
+    def _multi_image(self, b: int) -> Image:
+        f32 = np.float32
+        rng = np.random.default_rng([self.seed, b])
+        T, D, H, Hkv, d = self.T[b], self.D, self.H, self.Hkv, self.d
+        parts = [self._visual(np.random.default_rng([self.seed, b, 1000 + k]), f32)
+                 for k in range(self.I)]
+        hidden = np.concatenate([p[0] for p in parts] + [rng.standard_normal((T, D), dtype=f32)])
+        keys = np.concatenate([p[1] for p in parts] + [rng.standard_normal((T, Hkv, d), dtype=f32)])
+        values = np.concatenate([p[2] for p in parts] +
+                                [rng.standard_normal((T, Hkv, d), dtype=f32)])
+        queries = rng.standard_normal((T, H, d), dtype=f32)
+        region = None
+        if parts[0][3] is not None:  # regions numbered per image, distinct across images
+            region = np.concatenate([p[3] + 8 * k for k, p in enumerate(parts)])
+        N, Ng, s = self.N, self.Ng, max(self.gh, self.gw)
+        pos = np.empty((3, N + T), dtype=np.int32)
+        r, c = np.divmod(np.arange(Ng), self.gw)
+        for k in range(self.I):  # M-RoPE: image k at temporal index k*s
+            pos[0, k * Ng:(k + 1) * Ng] = k * s
+            pos[1, k * Ng:(k + 1) * Ng] = k * s + r
+            pos[2, k * Ng:(k + 1) * Ng] = k * s + c
+        pos[:, N:] = self.I * s + np.arange(T)
+        return Image(self._round(hidden), self._round(keys), self._round(values),
+                     self._round(queries), pos, T, region)
+
     def image(self, b: int) -> Image:
         if b in self._cache:
+            return self._cache[b]
+        if self.I > 1:
+            self._cache[b] = self._multi_image(b)
             return self._cache[b]
         rng = np.random.default_rng([self.seed, b])
         N, T, D, H, Hkv, d = self.N, self.T[b], self.D, self.H, self.Hkv, self.d
@@ -258,6 +327,7 @@ def make(name: str, K: int | None = None, B: int | None = None, T: int | list | 
     d = shape.pop("d", d)
     D = shape.pop("D", D)
     dtype = shape.pop("dtype", dtype)
+    n_img = shape.pop("I", IMAGES.get(name, 1))
     structure = shape.pop("structure", structure)
     if shape:
         raise KeyError(f"unknown workload fields {sorted(shape)}")
@@ -270,4 +340,4 @@ def make(name: str, K: int | None = None, B: int | None = None, T: int | list | 
     elif isinstance(T, int):
         T = [T] * B
     return Workload(name, idx, B, gh, gw, list(T), H, Hkv, d, D, K0 if K is None else K,
-                    dtype, structure, positions)
+                    dtype, structure, positions, n_img)

@@ -802,3 +802,139 @@ def test_prefix_kv_gather_is_the_index_map_layer_by_layer():
     none = O.compress(f(im.hidden), f(im.keys), f(im.values), f(im.queries), im.pos,
                       f(wl.probe()), wl.gh, wl.gw, wl.K)
     assert none.out_prefix_kv.shape[0] == 0
+
+
+# --------------------------------------------------------------------------
+# Multi-image prompts (Sec. 3.1 budget, Sec. 3.3 seeding, appendix Eq.
+# (cond-aux-clients) with 1[I_i = I_m], same-image assignment)
+# --------------------------------------------------------------------------
+def _multi_case(I=3, gh=4, gw=5, D=6, seed=80):
+    r = rng(seed)
+    N = I * gh * gw
+    h = r.standard_normal((N, D))
+    return h, N
+
+
+def test_multi_image_appearance_rows_stay_in_their_image():
+    I, gh, gw = 3, 4, 5
+    h, N = _multi_case(I, gh, gw)
+    cos = O.cosine_matrix(h, P)
+    PV = O.appearance_clients(cos, P, n_images=I)
+    Ng = gh * gw
+    for k in range(I):
+        blk = slice(k * Ng, (k + 1) * Ng)
+        # each image's block is the single-image bank of that image alone
+        np.testing.assert_allclose(PV[blk, blk], O.appearance_clients(cos[blk, blk], P), rtol=1e-13)
+        off = np.ones(N, bool)
+        off[blk] = False
+        assert np.all(PV[blk][:, off] == 0.0)
+    np.testing.assert_allclose(PV.sum(axis=1), 1.0, rtol=1e-13)
+
+
+def test_multi_image_spatial_landmarks_per_image():
+    I, gh, gw = 2, 6, 6
+    PS = O.spatial_clients(gh, gw, P, n_images=I)
+    one = O.spatial_clients(gh, gw, P)
+    L2, Ng = one.shape
+    assert PS.shape == (I * L2, I * Ng)
+    for k in range(I):
+        for k2 in range(I):
+            blk = PS[k * L2:(k + 1) * L2, k2 * Ng:(k2 + 1) * Ng]
+            if k == k2:
+                np.testing.assert_array_equal(blk, one)
+            else:
+                assert np.all(blk == 0.0)
+    # bank mass: beta_S shared by all I * L^2 rows
+    hvis = rng(81).standard_normal((I * Ng, 5))
+    cm = O.client_matrix(np.zeros((1, 1, I * Ng)), np.zeros((1, 1), bool), np.ones(1), np.ones(1),
+                         O.appearance_clients(O.cosine_matrix(hvis, P), P, I), PS, P)
+    assert cm.C[cm.banks["spatial"]].sum() == pytest.approx(P["beta_S"], rel=1e-13)
+
+
+def test_multi_image_seeds_are_each_images_best_singleton():
+    I, Ng, M = 3, 12, 40
+    C = _rand_C(M, I * Ng, 82)
+    u = C.sum(axis=0)
+    sel = O.select_support(C, 10, P, n_images=I)
+    seed = sel.rounds[0]
+    assert seed.seed and list(seed.batch) == sel.order[:I]
+    for k in range(I):   # brute force: largest column sum of image k, lowest index on ties
+        best = max(range(k * Ng, (k + 1) * Ng), key=lambda i: (u[i], -i))
+        assert sel.order[k] == best
+    assert len(sel.order) == 10 and len(set(sel.order)) == 10
+    # a budget below the image count: one carrier per image, the seeds
+    assert O.budget(2, I * Ng, I) == I
+    sel2 = O.select_support(C, O.budget(2, I * Ng, I), P, n_images=I)
+    assert sel2.order == sel.order[:I]
+    # a single image: no seed round, the plain solver
+    s1 = O.select_support(C, 10, P)
+    assert not s1.rounds[0].seed
+
+
+def test_multi_image_assignment_is_same_image():
+    I, gh, gw = 3, 4, 5
+    h, N = _multi_case(I, gh, gw, seed=83)
+    Ng = gh * gw
+    cos = O.cosine_matrix(h, P)
+    S = np.array([1, 7, 22, 33, 41, 55])   # image 0: 1, 7; image 1: 22, 33; image 2: 41, 55
+    a = O.assign_population(cos, S, gh, gw, P, n_images=I)
+    img = np.arange(N) // Ng
+    assert np.all(img[a.pi] == img)          # clusters never cross images
+    assert np.all(a.pi[S] == S)
+    for i in range(N):                        # the gap over same-image carriers only
+        if i in S:
+            continue
+        Si = S[img[S] == img[i]]
+        v = sorted(cos[i, Si], reverse=True)
+        assert a.delta[i] == pytest.approx(v[0] - v[1], abs=1e-15)
+    # a plain nearest neighbour when the gate is closed, within the image
+    b = O.assign_population(cos, S, gh, gw, O.params(gate_scale=1e9), n_images=I)
+    for i in range(N):
+        if i not in S:
+            Si = S[img[S] == img[i]]
+            assert b.pi[i] == Si[int(np.argmax(cos[i, Si]))]
+
+
+def test_multi_image_compress_invariants():
+    from paper_2608_02134_gb300 import workloads
+    wl = workloads.make("tiny", I=2, gh=6, gw=6, T=5, K=9)
+    im = wl.image(0)
+    f = lambda a: np.asarray(a, dtype=np.float64)
+    res = O.compress(f(im.hidden), f(im.keys), f(im.values), f(im.queries), im.pos,
+                     f(wl.probe()), wl.gh, wl.gw, wl.K, n_images=2)
+    N, Ng = wl.N, wl.Ng
+    img = np.arange(N) // Ng
+    assert res.K == 9 and res.support.size == 9
+    assert set(img[res.support]) == {0, 1}
+    assert np.all(img[res.assignment.pi] == img)
+    # transport conserves each image's population mass
+    for k in range(2):
+        Sk = res.support[img[res.support] == k]
+        slot = np.searchsorted(res.support, Sk)
+        assert res.transport.mass[slot].sum() == pytest.approx(res.m[img == k].sum(), rel=1e-12)
+    # one image is the single-image path
+    wl1 = workloads.make("tiny")
+    im1 = wl1.image(0)
+    r1 = O.compress(f(im1.hidden), f(im1.keys), f(im1.values), f(im1.queries), im1.pos,
+                    f(wl1.probe()), wl1.gh, wl1.gw, wl1.K, n_images=1)
+    r0 = O.compress(f(im1.hidden), f(im1.keys), f(im1.values), f(im1.queries), im1.pos,
+                    f(wl1.probe()), wl1.gh, wl1.gw, wl1.K)
+    assert np.array_equal(r1.support, r0.support) and np.array_equal(r1.out_hidden, r0.out_hidden)
+
+
+def test_multi_image_assignment_uses_each_images_own_grid():
+    """Two copies of one image with mirrored supports assign exactly like the
+    single image: same gaps, gate and kappa (coordinates are per image grid)."""
+    gh, gw, Ng = 4, 5, 20
+    h0 = rng(84).standard_normal((Ng, 3))
+    S0 = np.array([2, 9, 13, 18])
+    single = O.assign_population(O.cosine_matrix(h0, P), S0, gh, gw, P)
+    assert single.s_x > 0.5 and np.max(single.g[np.setdiff1d(np.arange(Ng), S0)]) > 0.1
+    h = np.concatenate([h0, h0])
+    both = O.assign_population(O.cosine_matrix(h, P), np.concatenate([S0, S0 + Ng]), gh, gw, P,
+                               n_images=2)
+    assert both.s_x == pytest.approx(single.s_x, rel=1e-13)
+    for k in range(2):
+        blk = slice(k * Ng, (k + 1) * Ng)
+        np.testing.assert_array_equal(both.pi[blk], single.pi + k * Ng)
+        np.testing.assert_allclose(both.kappa_best[blk], single.kappa_best, rtol=1e-13)
