@@ -117,12 +117,21 @@ void gmc_default_params(gmc_params* p);
  * functions.
  */
 typedef struct gmc_problem {
-  int B;                       /* images in the call, >= 1 */
-  int grid_h, grid_w;          /* source grid of every image; N == grid_h * grid_w */
+  int B;                       /* boundaries (prompts) in the call, >= 1 */
+  int grid_h, grid_w;          /* source grid of every image; N == images * grid_h * grid_w */
   int Hkv;                     /* key/value heads; H % Hkv == 0, query head h reads h / (H/Hkv) */
   int dtype;                   /* GMC_F32 or GMC_BF16 */
   const int32_t* text_offsets; /* DEVICE int32[B+1]: offsets[0] = 0, T_b = offsets[b+1]-offsets[b],
                                   1 <= T_b <= T; or NULL: every image has exactly T text tokens */
+  int images;                  /* images of every prompt, 0 or 1 = one (Sec. 3.1 I): the visual
+                                  segment holds them one after another, grid_h x grid_w tokens
+                                  each in raster order; the budget is min(N, max(K, images)), the
+                                  support starts with each image's best singleton-gain token,
+                                  appearance and spatial clients (one landmark grid per image)
+                                  cover their own image, and every token is assigned to a
+                                  carrier of its own image (appendix "Appearance and spatial
+                                  clients", "Batched complementary support", Eq.
+                                  (cond-assignment)).  gmc_transport* ignore it. */
 } gmc_problem;
 
 /* Bytes of workspace gmc_compress needs for this problem (0 on invalid arguments). */

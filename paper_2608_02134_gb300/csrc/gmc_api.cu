@@ -41,8 +41,10 @@ bool params_ok(const gmc_params& p) {
 // Shape checks shared by gmc_compress / gmc_transport / gmc_transport_noalloc.
 int check_problem(const gmc_problem* prob, int N, int T, int d, int D) {
   if (!prob) return GMC_ERR_ARG;
+  const int I = prob->images < 1 ? 1 : prob->images;  // images per prompt
   if (prob->B < 1 || prob->grid_h < 1 || prob->grid_w < 1 || N < 1 ||
-      (long long)prob->grid_h * prob->grid_w != N || T < 1 || d < 1 || D < 1 || prob->Hkv < 1)
+      (long long)prob->grid_h * prob->grid_w * I != N || T < 1 || d < 1 || D < 1 ||
+      prob->Hkv < 1)
     return GMC_ERR_ARG;
   if (prob->dtype != GMC_F32 && prob->dtype != GMC_BF16) return GMC_ERR_ARG;
   if (N > GMC_MAX_N || D > 8192 || d > 1024) return GMC_ERR_UNSUPPORTED;
@@ -67,7 +69,12 @@ struct Carver {
   }
 };
 
-int effective_K(int K, int N) { return K < 1 ? 1 : (K > N ? N : K); }
+// K = min{N, max{K_r, I}} (Sec. 3.1); K_r < 1 asks for the minimum
+int effective_K(int K, int N, int I = 1) {
+  const int k = K < I ? I : K;
+  return k < 1 ? 1 : (k > N ? N : k);
+}
+int images_of(const gmc_problem* prob) { return prob->images < 1 ? 1 : prob->images; }
 
 bool aligned(const void* p, size_t a) { return ((uintptr_t)p % a) == 0; }
 
@@ -77,7 +84,8 @@ Dims make_dims(const gmc_problem* prob, const gmc_params& p, int N, int T, int H
   dm.B = prob->B; dm.N = N; dm.T = T; dm.H = H; dm.Hkv = prob->Hkv; dm.d = d; dm.D = D;
   dm.K = K; dm.gh = prob->grid_h; dm.gw = prob->grid_w; dm.L = p.landmarks;
   dm.V = V;
-  dm.M = V * H * T + N + p.landmarks * p.landmarks;
+  dm.I = images_of(prob);
+  dm.M = V * H * T + N + dm.I * p.landmarks * p.landmarks;
   dm.dtype = prob->dtype;
   dm.toff = prob->text_offsets;
   return dm;
@@ -180,10 +188,12 @@ int fixed_point_exponent(double total) {
   return e < -60 ? -60 : (e > 120 ? 120 : e);
 }
 
-int fill_trace_layout(int B, const gmc_params& p, int N, int H, int K, gmc_trace_layout* o) {
+int fill_trace_layout(int B, const gmc_params& p, int N, int H, int K, gmc_trace_layout* o,
+                      int images = 1) {
   if (B < 1 || N < 1 || H < 0 || K < 1) return GMC_ERR_ARG;
   gmc_trace_layout L{};
-  L.rounds_max = (K + p.batch_b - 1) / p.batch_b + 1;
+  // responsibility rounds, a zero-gain fill, and a seed round for several images
+  L.rounds_max = (K + p.batch_b - 1) / p.batch_b + 1 + (images > 1 ? 1 : 0);
   L.pool_size = p.pool_mult * p.batch_b;
   size_t off = sizeof(gmc_trace_header);
   auto take = [&](size_t bytes) {
@@ -347,7 +357,8 @@ size_t gmc_workspace_size_views(const gmc_problem* prob, int n_views, int N, int
     return 0;
   gmc_params p;
   gmc_default_params(&p);
-  const Dims dm = make_dims(prob, p, N, T, H, d, D, effective_K(K, N), 1 + n_views);
+  const Dims dm =
+      make_dims(prob, p, N, T, H, d, D, effective_K(K, N, images_of(prob)), 1 + n_views);
   return carve_compress(dm, nullptr, nullptr);
 }
 
@@ -361,7 +372,8 @@ int gmc_get_trace_layout(const gmc_problem* prob, const gmc_params* params, int 
   gmc_params p;
   if (params) p = *params; else gmc_default_params(&p);
   if (!params_ok(p)) return GMC_ERR_ARG;
-  return fill_trace_layout(prob->B, p, N, H, effective_K(K, N), out);
+  return fill_trace_layout(prob->B, p, N, H, effective_K(K, N, images_of(prob)), out,
+                           images_of(prob));
 }
 
 size_t gmc_trace_size(const gmc_problem* prob, const gmc_params* params, int N, int T, int H,
@@ -426,7 +438,7 @@ static int compress_impl(const gmc_problem* prob, const gmc_params* params,
         return GMC_ERR_ARG;
     }
   }
-  const int Ke = effective_K(K, N);
+  const int Ke = effective_K(K, N, images_of(prob));
   const Dims dm = make_dims(prob, p, N, T, H, d, D, Ke, V);
   Scratch s;
   R0State r0;
@@ -436,7 +448,7 @@ static int compress_impl(const gmc_problem* prob, const gmc_params* params,
   gmc_trace_layout L;
   TraceView tv{};
   if (trace) {
-    fill_trace_layout(dm.B, p, N, H, Ke, &L);
+    fill_trace_layout(dm.B, p, N, H, Ke, &L, dm.I);
     tv = make_trace_view(trace, L);
     GMC_TRY(cudaMemsetAsync(trace, 0, (size_t)dm.B * L.bytes_per_image, st));
   }
@@ -518,13 +530,13 @@ static int compress_impl(const gmc_problem* prob, const gmc_params* params,
                             cudaMemcpyDeviceToDevice, st));
     return GMC_OK;
   }
+  const int LS = dm.I * p.landmarks * p.landmarks;  // spatial rows: a landmark grid per image
   GMC_STAGE("rounds_gpu", 3 + 3 * sparse_gpu_rounds(N),
-            launch_round0(r0, dm.B, N, Ke, dm.M, dm.toff, HV, T, p.landmarks * p.landmarks, p, fx,
-                          nullptr, s.C, s.scol, s.u0, s.order, s.status, tv, st));
+            launch_round0(r0, dm.B, N, Ke, dm.M, dm.toff, HV, T, LS, p, fx, nullptr, s.C, s.scol,
+                          s.u0, s.order, s.status, tv, st, dm.I));
   GMC_STAGE("select", 1,
-            launch_select(r0, dm.B, N, Ke, dm.M, dm.toff, HV, T, p.landmarks * p.landmarks, p, fx,
-                          nullptr, s.C, s.scol, s.u0, s.order, s.support, s.slot, nullptr, s.status,
-                          tv, st));
+            launch_select(r0, dm.B, N, Ke, dm.M, dm.toff, HV, T, LS, p, fx, nullptr, s.C, s.scol,
+                          s.u0, s.order, s.support, s.slot, nullptr, s.status, tv, st, dm.I));
   GMC_STAGE("assign", 2, launch_assign(dm, p, s, tv, st));
   GMC_STAGE("transport", 1,
             launch_transport(dm, p, hidden, keys, pos_ids, s.support, s.pi, s.mass, s.rmsh,

@@ -125,7 +125,7 @@ extern "C" int gmc_transport_noalloc(const gmc_problem* prob, const gmc_params* 
   Dims dm;
   dm.B = prob->B; dm.N = N; dm.T = T; dm.H = 0; dm.Hkv = prob->Hkv; dm.d = d; dm.D = D;
   dm.K = K; dm.gh = prob->grid_h; dm.gw = prob->grid_w; dm.L = p.landmarks;
-  dm.V = 1; dm.M = N; dm.dtype = prob->dtype; dm.toff = prob->text_offsets;
+  dm.V = 1; dm.I = 1; dm.M = N; dm.dtype = prob->dtype; dm.toff = prob->text_offsets;
   if ((e = cudaMemsetAsync(status, 0, sizeof(uint32_t), st)) != cudaSuccess ||
       (e = launch_rms_rows(dm, hidden, rmsh, status, st)) != cudaSuccess ||
       (e = launch_transport(dm, p, hidden, keys, pos_ids, support, assign, weights, rmsh,

@@ -6,7 +6,9 @@
 //   s_x = 1 - exp(-(Delta_bar / gate_scale)^gate_pow)
 //   g_i = exp(-(delta_i / ambig_margin)^gate_pow)
 //   pi(i) = argmax_{j in S} cos_ij + lambda_p s_x g_i exp(-||p_i - p_j||^2 / tau_s)
-// (ties to the lowest j); selected tokens represent themselves.  The
+// (ties to the lowest j); selected tokens represent themselves.  With I > 1
+// images per prompt (Ng = N / I tokens each, one after another) token i's
+// candidates, its gap and its coordinates are those of its own image.  The
 // population weights are m_i = (1 - alpha s_x) + alpha s_x ebar_i.  Token i
 // also sets bit i of its carrier's membership bitmap (atomicOr: the bitmap
 // does not depend on the order of the writes), which the transport reads
@@ -28,7 +30,8 @@ __global__ void k_assign_gap(const float* __restrict__ cos, const int32_t* __res
                              const float* __restrict__ zn2, const float* __restrict__ sigma,
                              const float* __restrict__ W2, float* energy, float* epart,
                              float* delta, double* dpart, int nA, float gate_scale,
-                             float gate_pow, uint32_t* tick, float* gatev, uint32_t* status) {
+                             float gate_pow, int I, uint32_t* tick, float* gatev,
+                             uint32_t* status) {
   grid_dep_wait();
   __shared__ double sd[ASSIGN_WARPS];
   __shared__ int sc[ASSIGN_WARPS];
@@ -58,11 +61,16 @@ __global__ void k_assign_gap(const float* __restrict__ cos, const int32_t* __res
   if (i < N && slot[(size_t)b * N + i] < 0) {
     const float* row = cos + ((size_t)b * N + i) * N;
     const int32_t* S = sS;
+    const int Ng = N / I, img = i / Ng;
     float m1 = -INFINITY, m2 = -INFINITY;
+    int ncomp = 0;  // carriers of token i's image
     for (int k = lane; k < K; k += 32) {
+      if (S[k] / Ng != img) continue;
+      ++ncomp;
       const float v = row[S[k]];
       if (v > m1) { m2 = m1; m1 = v; } else if (v > m2) { m2 = v; }
     }
+    ncomp = warp_sum_int(ncomp);
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
       const float b1 = __shfl_xor_sync(FULL, m1, o), b2 = __shfl_xor_sync(FULL, m2, o);
@@ -70,7 +78,7 @@ __global__ void k_assign_gap(const float* __restrict__ cos, const int32_t* __res
       m2 = fmaxf(fminf(m1, b1), fmaxf(m2, b2));
       m1 = hi;
     }
-    const float d = K > 1 ? m1 - m2 : 0.f;
+    const float d = ncomp > 1 ? m1 - m2 : 0.f;
     if (lane == 0) delta[(size_t)b * N + i] = d;
     dv = d;
     dc = 1;
@@ -125,7 +133,7 @@ __global__ void k_assign_pick(const float* __restrict__ cos, const int32_t* __re
                               const float* __restrict__ gatev, const float* __restrict__ energy,
                               const int32_t* toff, int B, int N, int K, int Tmax, int gh, int gw,
                               float gate_pow, float ambig_margin, float lambda_p, float tau_s,
-                              float alpha,
+                              float alpha, int I,
                               int32_t* pi, float* mass, uint32_t* mbits, TraceView tv,
                               uint32_t* status) {
   grid_dep_wait();
@@ -150,16 +158,19 @@ __global__ void k_assign_pick(const float* __restrict__ cos, const int32_t* __re
   if (slot[(size_t)b * N + i] < 0) {
     const float gi = expf(-powf(delta[(size_t)b * N + i] / ambig_margin, gate_pow));
     const float coef = lambda_p * sx * gi;
-    const float piy = ((i / gw) + 0.5f) / gh, pix = ((i % gw) + 0.5f) / gw;
+    const int Ng = N / I, img = i / Ng, il = i - img * Ng;  // coordinates in its own grid
+    const float piy = ((il / gw) + 0.5f) / gh, pix = ((il % gw) + 0.5f) / gw;
     const float* row = cos + ((size_t)b * N + i) * N;
     const int32_t* S = sS;
     float best = -INFINITY;
     int bk = 0x7fffffff;
     for (int k = lane; k < K; k += 32) {
       const int j = S[k];
+      if (j / Ng != img) continue;  // a carrier of another image
       float v = row[j];
       if (coef > 0.f) {
-        const float dy = ((j / gw) + 0.5f) / gh - piy, dx = ((j % gw) + 0.5f) / gw - pix;
+        const int jl = j - img * Ng;
+        const float dy = ((jl / gw) + 0.5f) / gh - piy, dx = ((jl % gw) + 0.5f) / gw - pix;
         v += coef * expf(-(dy * dy + dx * dx) / tau_s);
       }
       if (v > best) { best = v; bk = k; }  // k ascending within a lane: first max kept
@@ -170,8 +181,13 @@ __global__ void k_assign_pick(const float* __restrict__ cos, const int32_t* __re
       const int ok = __shfl_xor_sync(FULL, bk, o);
       if (ob > best || (ob == best && ok < bk)) { best = ob; bk = ok; }
     }
-    if (bk >= K) {  // no comparable value (non-finite cosines): the first carrier
-      bk = 0;
+    if (bk >= K) {  // no comparable value (non-finite cosines): the image's first carrier
+      int first = K;
+      for (int k = lane; k < K; k += 32)
+        if (S[k] / Ng == img) { first = k; break; }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) first = min(first, __shfl_xor_sync(FULL, first, o));
+      bk = first < K ? first : 0;
       if (lane == 0) set_status(status, GMC_STATUS_NONFINITE);
     }
     choice = S[bk];
@@ -199,14 +215,14 @@ cudaError_t launch_assign(const Dims& dm, const gmc_params& p, Scratch& s, const
   if ((e0 = set_smem_limit((const void*)k_assign_pick, smem)) != cudaSuccess) return e0;
   launch_k(k_assign_gap, grid, 32 * ASSIGN_WARPS, smem, st, 1,
       s.cos, s.support, s.slot, dm.toff, dm.B, dm.N, dm.K, dm.T, dm.H, s.omega, s.zn2, s.sigma,
-      s.W2, s.ebar, s.epart, s.delta, s.dpart, s.nA, p.gate_scale, p.gate_pow, s.tick2, s.gatev,
-      s.status);
+      s.W2, s.ebar, s.epart, s.delta, s.dpart, s.nA, p.gate_scale, p.gate_pow, dm.I, s.tick2,
+      s.gatev, s.status);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   launch_k(k_assign_pick, grid, 32 * ASSIGN_WARPS, smem, st, 1,
       s.cos, s.support, s.slot, s.delta, s.gatev, s.ebar, dm.toff, dm.B, dm.N, dm.K, dm.T,
       dm.gh, dm.gw, p.gate_pow, p.ambig_margin, p.assign_spatial_w, p.tau_s,
-      p.pop_strength, s.pi, s.mass, s.mbits, tv, s.status);
+      p.pop_strength, dm.I, s.pi, s.mass, s.mbits, tv, s.status);
   return cudaGetLastError();
 }
 

@@ -7,8 +7,12 @@
 //              sharing beta_hist; zero when the row has no energy: an inactive
 //              client)
 //   appearance m = 0..N-1:       beta_V / N * softmax_i(cos_mi / tau_v)
-//   spatial    l = 0..L*L-1:     beta_S / L^2 * softmax_i(-||p_i - l_l||^2 / tau_s)
-// with p_i = ((r+.5)/gh, (c+.5)/gw) and landmarks ((a+.5)/L, (b+.5)/L).
+//   spatial    l = 0..I*L*L-1:   beta_S / (I L^2) * softmax_i(-||p_i - l_l||^2 / tau_s)
+// with p_i = ((r+.5)/gh, (c+.5)/gw) and landmarks ((a+.5)/L, (b+.5)/L).  A
+// prompt with I > 1 images holds them one after another (Ng = gh * gw tokens
+// each): an appearance row and the landmark grid of image k (rows k L^2 ..)
+// cover image k's tokens only, in that image's own coordinates; grounded rows
+// cover every visual token.
 // The spatial softmax separates over the grid: ||p_i - l||^2 = dy_r^2 + dx_c^2,
 // so its smallest distance is min dy^2 + min dx^2 and its normaliser is
 // (sum_r exp(-dy_r^2 / tau_s)) (sum_c exp(-dx_c^2 / tau_s)) (each factor
@@ -30,6 +34,7 @@ struct RowInfo {
   float shift;     // appearance: row max of the cosine; spatial: smallest distance^2
   float sg2;       // grounded: sigma_h^2
   float ly, lx;    // spatial: landmark coordinates
+  int lo, hi;      // columns the row covers (its image; every column for grounded rows)
 };
 
 // Online (max, sum of exp((x - max) / tau)) of a row, one lane's share: 8
@@ -66,19 +71,20 @@ __global__ void __launch_bounds__(256, 4) k_build_clients(
     const ViewRows vw, int nRS, const float* __restrict__ omega,
     const float* __restrict__ cos, const int32_t* toff, int B, int N, int Tmax, int H, int M,
     int gh, int gw, int L, float beta_V, float beta_S, float tau_v, float tau_s,
-    float wq, float fx_scale, int check, float* C, long long* u0, uint32_t* status) {
+    float wq, float fx_scale, int check, int I, float* C, long long* u0, uint32_t* status) {
   grid_dep_wait();
   __shared__ RowInfo ri[ROWS_PER_BLOCK];
   const int b = blockIdx.y;
   const TextGeom tg = text_geom(toff, b, B, Tmax, status);
   if (tg.T == 0) return;
-  const int Tb = tg.T, MG = vw.n * H * Tb, Mb = MG + N + L * L;
+  const int Tb = tg.T, MG = vw.n * H * Tb, Mb = MG + N + I * L * L;
+  const int Ng = N / I;  // tokens of one image
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const int r0 = blockIdx.x * ROWS_PER_BLOCK;
   if (r0 >= Mb) return;
   {
     const int m = r0 + w;
-    RowInfo inf{-1, nullptr, nullptr, 0.f, 0.f, 0.f, 0.f, 0.f};
+    RowInfo inf{-1, nullptr, nullptr, 0.f, 0.f, 0.f, 0.f, 0.f, 0, N};
     if (m < MG) {
       const int v = m / (H * Tb), hm = m - v * H * Tb;  // view, then (h, t) h-major
       const int h = hm / Tb, t = hm % Tb;
@@ -94,14 +100,19 @@ __global__ void __launch_bounds__(256, 4) k_build_clients(
     } else if (m < MG + N) {
       const int a = m - MG;
       const float* row = cos + ((size_t)b * N + a) * N;
+      inf.lo = (a / Ng) * Ng;  // the row's own image
+      inf.hi = inf.lo + Ng;
       float mx, z;
-      row_softmax_stats(row, N, 1.f / tau_v, lane, mx, z);
+      row_softmax_stats(row + inf.lo, Ng, 1.f / tau_v, lane, mx, z);
       inf.kind = 1;
       inf.x = row;
       inf.scale = beta_V / ((float)N * z);
       inf.shift = mx;
     } else if (m < Mb) {
-      const int l = m - MG - N;
+      const int lg = m - MG - N;
+      const int l = lg % (L * L);  // landmark of image lg / L^2
+      inf.lo = (lg / (L * L)) * Ng;
+      inf.hi = inf.lo + Ng;
       const int la = l / L, lb = l % L;
       const float ly = (la + 0.5f) / L, lx = (lb + 0.5f) / L;
       float mny = INFINITY, mnx = INFINITY;
@@ -127,7 +138,7 @@ __global__ void __launch_bounds__(256, 4) k_build_clients(
       zy = warp_sum(zy);
       zx = warp_sum(zx);
       inf.kind = 2;
-      inf.scale = beta_S / ((float)(L * L) * (zy * zx));
+      inf.scale = beta_S / ((float)(I * L * L) * (zy * zx));
       inf.shift = mny + mnx;
       inf.ly = ly;
       inf.lx = lx;
@@ -139,8 +150,8 @@ __global__ void __launch_bounds__(256, 4) k_build_clients(
   const float itv = 1.f / tau_v, its = 1.f / tau_s;
   for (int j = threadIdx.x; j < N; j += blockDim.x) {
     long long colsum = 0;
-    const int jr = j / gw;
-    const float py = (jr + 0.5f) / gh, px = ((j - jr * gw) + 0.5f) / gw;
+    const int jl = j % Ng, jr = jl / gw;  // position in its own image's grid
+    const float py = (jr + 0.5f) / gh, px = ((jl - jr * gw) + 0.5f) / gw;
     // every row's operands are loaded before any is used
     float xv[ROWS_PER_BLOCK], zv[ROWS_PER_BLOCK];
 #pragma unroll
@@ -154,7 +165,9 @@ __global__ void __launch_bounds__(256, 4) k_build_clients(
       if (q >= nrows) break;
       const RowInfo& inf = ri[q];
       float v = 0.f;
-      if (inf.kind == 0) {
+      if (j < inf.lo || j >= inf.hi) {
+        v = 0.f;  // another image's token
+      } else if (inf.kind == 0) {
         v = xv[q] * sqrtf(zv[q] + inf.sg2) * inf.scale;
       } else if (inf.kind == 1) {
         v = expf((xv[q] - inf.shift) * itv) * inf.scale;
@@ -177,7 +190,7 @@ cudaError_t launch_build_clients(const Dims& dm, const gmc_params& p, int fx_exp
   launch_k(k_build_clients, grid, 32 * ROWS_PER_BLOCK, 0, st, 1,
       views, s.nRS, s.omega, s.cos, dm.toff, dm.B, dm.N, dm.T, dm.H, dm.M, dm.gh,
       dm.gw, dm.L, p.beta_V, p.beta_S, p.tau_v, p.tau_s, p.terminal_q_weight,
-      ldexpf(1.f, fx_exp), p.check_mode, s.C, s.u0, s.status);
+      ldexpf(1.f, fx_exp), p.check_mode, dm.I, s.C, s.u0, s.status);
   return cudaGetLastError();
 }
 

@@ -50,7 +50,7 @@ int filter_rows_per_warp(int B, int M) {
 }
 
 __global__ void __launch_bounds__(512) k_r0_pool(const long long* __restrict__ u0, int B, int N,
-                                                   int P, const int32_t* toff, int Tmax,
+                                                   int P, const int32_t* toff, int Tmax, int I,
                                                    int32_t* pool0, int32_t* info, long long* s0,
                                                    long long* u1, long long* fv, uint32_t* status) {
   grid_dep_wait();
@@ -88,6 +88,34 @@ __global__ void __launch_bounds__(512) k_r0_pool(const long long* __restrict__ u
   for (int h = threadIdx.x; h < sel::HBINS; h += blockDim.x) w.hist[h] = 0;
   if (threadIdx.x < sel::CBINS) w.coarse[threadIdx.x] = 0;
   __syncthreads();
+  if (I > 1) {
+    // several images: the first round only seeds S with each image's token of
+    // largest singleton gain (ties to the lower index), one warp per image;
+    // the filter takes them as its batch
+    const int lane = threadIdx.x & 31, Ng = N / I;
+    for (int k = threadIdx.x >> 5; k < I; k += blockDim.x >> 5) {
+      long long bv = -1;
+      int bj = 0x7fffffff;
+      for (int j = k * Ng + lane; j < (k + 1) * Ng; j += 32)
+        if (ug[j] > bv) {  // j ascending within a lane: the first maximum is kept
+          bv = ug[j];
+          bj = j;
+        }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const long long ov = __shfl_xor_sync(FULL, bv, o);
+        const int oj = __shfl_xor_sync(FULL, bj, o);
+        if (ov > bv || (ov == bv && oj < bj)) {
+          bv = ov;
+          bj = oj;
+        }
+      }
+      if (lane == 0) pool0[(size_t)b * P + k] = bj;
+    }
+    for (int k = I + threadIdx.x; k < P; k += blockDim.x) pool0[(size_t)b * P + k] = -1;
+    if (threadIdx.x == 0) info[b * 4] = I;
+    return;
+  }
   const int Pt = sel::select_pool(ug, selz, N, P, w, pool, nullptr);
   for (int k = threadIdx.x; k < P; k += blockDim.x) pool0[(size_t)b * P + k] = k < Pt ? pool[k] : -1;
   if (threadIdx.x == 0) info[b * 4] = Pt;
@@ -96,8 +124,9 @@ __global__ void __launch_bounds__(512) k_r0_pool(const long long* __restrict__ u
 __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_rho(
     const float* __restrict__ C, int B, int N, int Mstride, int H, int L2, const int32_t* toff,
     int Tmax, int uniform_rows, const int32_t* __restrict__ pool0, const int32_t* __restrict__ info,
-    int P, float resp_temp, float resp_eps, int fx_exp, const int32_t* fexp, long long* s0) {
+    int P, float resp_temp, float resp_eps, int fx_exp, const int32_t* fexp, int I, long long* s0) {
   grid_dep_wait();
+  if (I > 1) return;  // a seed round: no responsibilities
   __shared__ int pool[GMC_MAX_POOL];
   __shared__ long long sblk[GMC_MAX_POOL];
   const int b = blockIdx.y;
@@ -155,7 +184,7 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_filter(
     const int32_t* toff, int Tmax, int uniform_rows, const int32_t* __restrict__ pool0,
     int32_t* info, const long long* __restrict__ s0, int P, int bsz, int fx_exp,
     const int32_t* fexp, long long* u1, float* bcov, int32_t* cnt, long long* fv,
-    int32_t* order, int rpw, TraceView tv) {
+    int32_t* order, int rpw, int I, TraceView tv) {
   grid_dep_wait();
   __shared__ int pool[GMC_MAX_POOL];
   __shared__ long long sc[GMC_MAX_POOL];
@@ -174,7 +203,7 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_filter(
   const int m0 = blockIdx.x * R0_ROWS * rpw;
   if (m0 >= Mb) return;
   const float fxs = ldexpf(1.f, fexp ? fexp[b] : fx_exp);
-  const int nb = min(bsz, min(Pt, K));
+  const int nb = I > 1 ? Pt : min(bsz, min(Pt, K));  // a seed round takes its whole pool
   for (int k = threadIdx.x; k < Pt; k += blockDim.x) {
     pool[k] = pool0[(size_t)b * P + k];
     sc[k] = s0[(size_t)b * P + k];
@@ -186,7 +215,7 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_filter(
     const int lane = threadIdx.x & 31, gl = lane & 7;
     const unsigned gm = 0xFFu << (lane & 24);
     for (int k = threadIdx.x >> 3; k < Pt; k += blockDim.x >> 3) {  // 8 lanes per pool token
-      const int rank = sel::group_score_rank(sc, pool, Pt, k, gl, gm);
+      const int rank = I > 1 ? k : sel::group_score_rank(sc, pool, Pt, k, gl, gm);
       if (gl == 0 && rank < nb) batch[rank] = pool[k];
     }
   }
@@ -547,7 +576,7 @@ cudaError_t launch_round0(const R0State& r0, int B, int N, int K, int M, const i
                           int H, int T, int L2, const gmc_params& p, int fx_exp,
                           const int32_t* fexp, float* C, uint16_t* scol, const long long* u0,
                           int32_t* order, uint32_t* status, const TraceView& tv,
-                          cudaStream_t st) {
+                          cudaStream_t st, int I) {
   const int P = p.pool_mult * p.batch_b;
   cudaError_t e;
   const size_t smem =
@@ -555,12 +584,12 @@ cudaError_t launch_round0(const R0State& r0, int B, int N, int K, int M, const i
       4 * (size_t)N + 64;
   if ((e = set_smem_limit((const void*)k_r0_pool, smem)) != cudaSuccess) return e;
   const int uniform = (H == 0);
-  launch_k(k_r0_pool, B, 512, smem, st, 1, u0, B, N, P, uniform ? nullptr : toff, T, r0.pool, r0.info,
+  launch_k(k_r0_pool, B, 512, smem, st, 1, u0, B, N, P, uniform ? nullptr : toff, T, I, r0.pool, r0.info,
                                   r0.s0, r0.u1, r0.fv, status);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   dim3 grid(ceil_div(M, R0_ROWS), B);
   launch_k(k_r0_rho, grid, 32 * R0_ROWS, 0, st, 1, C, B, N, M, H, L2, toff, T, uniform, r0.pool, r0.info,
-                                          P, p.resp_temp, p.resp_eps, fx_exp, fexp, r0.s0);
+                                          P, p.resp_temp, p.resp_eps, fx_exp, fexp, I, r0.s0);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   const size_t fsm = sizeof(unsigned long long) * (size_t)N;
   if ((e = set_smem_limit((const void*)k_r0_filter, fsm)) != cudaSuccess) return e;
@@ -568,7 +597,7 @@ cudaError_t launch_round0(const R0State& r0, int B, int N, int K, int M, const i
   const dim3 fgrid(ceil_div(M, R0_ROWS * rpw), B);
   launch_k(k_r0_filter, fgrid, 32 * R0_ROWS, fsm, st, 1, C, scol, B, N, K, M, H, L2, toff, T, uniform, r0.pool,
                                              r0.info, r0.s0, P, p.batch_b, fx_exp, fexp, r0.u1,
-                                             r0.bcov, r0.cnt, r0.fv, order, rpw, tv);
+                                             r0.bcov, r0.cnt, r0.fv, order, rpw, I, tv);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   // sparse rounds: gains alternate between u1 and u2
   const size_t psm = smem;  // the pool kernel's layout is round 0's

@@ -82,6 +82,7 @@ struct SelArgs {
   int32_t* out_idx;
   uint32_t* status;
   TraceView tv;
+  int images;           // images per prompt (> 1: the first round seeded one token per image)
   int cap;              // survivor entries that fit in shared memory
   int rpc;              // rows one CTA can own
   R0State r0;           // state after the first round
@@ -372,7 +373,7 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
   };
   if (Pt0 > 0) migrate();
 
-  const int rounds_max = (K + a.bsz - 1) / a.bsz + 1;
+  const int rounds_max = (K + a.bsz - 1) / a.bsz + 1 + (a.images > 1 ? 1 : 0);
   // add v to token j's gain for the round after `rnd` at the token's owner
   // (exact: 64-bit integer atomics, order-independent)
   auto gain_add = [&](int j, unsigned long long v, int rnd_now) {
@@ -860,7 +861,7 @@ cudaError_t launch_select(const R0State& r0, int B, int N, int K, int M, const i
                           const gmc_params& p, int fx_exp, const int32_t* fexp, float* C,
                           uint16_t* scol, const long long* u0, int32_t* order, int32_t* support,
                           int32_t* slot, int32_t* out_idx, uint32_t* status, const TraceView& tv,
-                          cudaStream_t st) {
+                          cudaStream_t st, int I) {
   cudaError_t e;
   if (g_num_sms == 0) {
     int dev = 0;
@@ -887,6 +888,7 @@ cudaError_t launch_select(const R0State& r0, int B, int N, int K, int M, const i
   a.status = status;
   a.tv = tv;
   a.r0 = r0;
+  a.images = I;
   int CS = 1;
   while (CS * 2 <= SEL_MAX_CS && (long long)B * CS * 2 <= g_num_sms) CS *= 2;
   for (; CS >= 1; CS /= 2) {

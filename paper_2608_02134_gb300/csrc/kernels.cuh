@@ -17,7 +17,8 @@ constexpr int MAX_VIEWS = 4;  // message views: the current one and up to 3 hist
 struct Dims {
   int B, N, T, H, Hkv, d, D, K, gh, gw, L;  // L = landmarks per side
   int V;                                    // message views (1: the current view only)
-  int M;                                    // V*H*T + N + L*L: client rows per image (max)
+  int I;                                    // images per prompt (N = I * gh * gw)
+  int M;                                    // V*H*T + N + I*L*L: client rows per prompt (max)
   int dtype;                                // GMC_F32 / GMC_BF16
   const int32_t* toff;                      // device text offsets or nullptr
 };
@@ -158,12 +159,12 @@ struct R0State {
 cudaError_t launch_round0(const R0State&, int B, int N, int K, int M, const int32_t* toff, int H,
                           int T, int L2, const gmc_params&, int fx_exp, const int32_t* fexp,
                           float* C, uint16_t* scol, const long long* u0, int32_t* order,
-                          uint32_t* status, const TraceView&, cudaStream_t);
+                          uint32_t* status, const TraceView&, cudaStream_t, int I = 1);
 cudaError_t launch_select(const R0State&, int B, int N, int K, int M, const int32_t* toff, int H, int T, int L2,
                           const gmc_params&, int fx_exp, const int32_t* fexp_per_image, float* C,
                           uint16_t* scol, const long long* u0, int32_t* order, int32_t* support,
                           int32_t* slot, int32_t* out_idx, uint32_t* status, const TraceView&,
-                          cudaStream_t);
+                          cudaStream_t, int I = 1);
 cudaError_t launch_select_prep(const float* C, int B, int M, int N, Scratch&, cudaStream_t);
 cudaError_t launch_assign(const Dims&, const gmc_params&, Scratch&, const TraceView&,
                           cudaStream_t);

@@ -52,7 +52,8 @@ class Params(ctypes.Structure):
 
 class Problem(ctypes.Structure):
     _fields_ = [("B", ctypes.c_int), ("grid_h", ctypes.c_int), ("grid_w", ctypes.c_int),
-                ("Hkv", ctypes.c_int), ("dtype", ctypes.c_int), ("text_offsets", ctypes.c_void_p)]
+                ("Hkv", ctypes.c_int), ("dtype", ctypes.c_int), ("text_offsets", ctypes.c_void_p),
+                ("images", ctypes.c_int)]
 
 
 class Views(ctypes.Structure):
@@ -181,8 +182,9 @@ def _stream(stream):
     return ctypes.c_void_p(s.cuda_stream)
 
 
-def problem(B, grid_h, grid_w, Hkv, dtype, text_offsets=None) -> Problem:
-    return Problem(B, grid_h, grid_w, Hkv, dtype, None if text_offsets is None else text_offsets.data_ptr())
+def problem(B, grid_h, grid_w, Hkv, dtype, text_offsets=None, images=1) -> Problem:
+    return Problem(B, grid_h, grid_w, Hkv, dtype,
+                   None if text_offsets is None else text_offsets.data_ptr(), images)
 
 
 def workspace_size(prob: Problem, N, T, H, d, D, K) -> int:
@@ -365,11 +367,12 @@ class Compressor:
     """
 
     def __init__(self, B, grid_h, grid_w, T, H, Hkv, d, D, K, dtype, text_lengths=None,
-                 params: Params | None = None, trace=False, device="cuda", n_views=0):
+                 params: Params | None = None, trace=False, device="cuda", n_views=0, images=1):
         self.B, self.gh, self.gw, self.T, self.H, self.Hkv, self.d, self.D = B, grid_h, grid_w, T, H, Hkv, d, D
-        self.N = grid_h * grid_w
+        self.images = images
+        self.N = grid_h * grid_w * images
         self.Kr = K
-        self.K = min(self.N, max(1, K))
+        self.K = min(self.N, max(images, K))
         self.dtype = dtype
         self.tdt = torch.bfloat16 if dtype == GMC_BF16 else torch.float32
         self.params = params or default_params()
@@ -380,7 +383,7 @@ class Compressor:
         for t in lens:
             off.append(off[-1] + t)
         self.offsets = torch.tensor(off, dtype=torch.int32, device=device) if text_lengths is not None else None
-        self.prob = problem(B, grid_h, grid_w, Hkv, dtype, self.offsets)
+        self.prob = problem(B, grid_h, grid_w, Hkv, dtype, self.offsets, images)
         self.n_views = n_views
         ws = workspace_size_views(self.prob, n_views, self.N, T, H, d, D, K)
         if ws == 0:

@@ -53,7 +53,7 @@ def run(wl: workloads.Workload, params=None, trace=True, inputs=None, n_hist=0,
     inp = inputs or to_device(wl)
     comp = gmc.Compressor(wl.B, wl.gh, wl.gw, wl.T_max, wl.H, wl.Hkv, wl.d, wl.D, wl.K, dt,
                           text_lengths=wl.T if wl.ragged else None, params=params, trace=trace,
-                          n_views=n_hist)
+                          n_views=n_hist, images=wl.I)
     history = None
     if n_hist:
         hv = [wl.history_abi_arrays(v) for v in range(n_hist)]
@@ -118,7 +118,8 @@ def compare_image(g: GpuRun, b: int, hidden_tol: float) -> ImageReport:
         prefix = [(f(wl.prefix_kv(b, l)["K"]), f(wl.prefix_kv(b, l)["V"]))
                   for l in range(len(g.prefix))]
     res = O.compress(f(im.hidden), f(im.keys), f(im.values), f(im.queries), im.pos, f(wl.probe()),
-                     wl.gh, wl.gw, wl.K, p, forced=forced, history=history, prefix=prefix)
+                     wl.gh, wl.gw, wl.K, p, forced=forced, history=history, prefix=prefix,
+                     n_images=wl.I)
     dec = parity.Decisions()
     tag = f"{wl.name}[b={b}]"
     parity.check_heads(res.heads, dec, tag)

@@ -135,6 +135,20 @@ def check_selection(sel: O.Selection, P: int, dec: Decisions, tag=""):
         u = r.gains
         free = np.flatnonzero(~selected)
         dec.checked += 1
+        if getattr(r, "seed", False):
+            # multi-image seed round: every image's token of largest singleton gain
+            I = len(r.batch)
+            Ng = N // I
+            for k, jk in enumerate(np.asarray(r.batch)):
+                ids = np.arange(k * Ng, (k + 1) * Ng)
+                ok, exact = valid_topk(u[ids], ids, [int(jk)], 1)
+                if not ok:
+                    dec.failures.append(f"{tag} seed of image {k}: {int(jk)} is not its best gain")
+                elif not exact:
+                    dec.near_ties.append(f"{tag} seed of image {k}")
+            dec.exact += 1
+            selected[r.batch] = True
+            continue
         if r.fill:
             # valid only when every remaining gain is (near) zero; ascending order
             if u[free].max(initial=0.0) > TOL * scale0:

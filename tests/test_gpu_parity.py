@@ -207,3 +207,28 @@ def test_prefix_layers_fp32_and_identity():
         pk = wl2.prefix_kv(0, l)
         ref = np.stack([pk["K"], pk["V"]]).reshape(-1).astype(np.float64)
         assert np.array_equal(g.prefix[l].reshape(-1), ref)
+
+
+def test_multi_image_prompt_qwen_shape():
+    """Two Qwen-shaped images in one prompt: seeds, image-restricted banks, same-image clusters."""
+    from paper_2608_02134_gb300 import workloads
+    from tests import gpu_harness as GH
+    wl = workloads.make("multi")
+    g = GH.run(wl)
+    _check(g, [0], TOL_BF16)
+    img = np.arange(wl.N) // wl.Ng
+    pi = g.traces[0].pi
+    assert np.all(img[pi] == img)
+
+
+@pytest.mark.parametrize("I,K", [(3, 24), (4, 2)])
+def test_multi_image_small_shapes(I, K):
+    """Three and four images (K below the image count: one carrier each), ragged text, fp32 and bf16."""
+    from paper_2608_02134_gb300 import workloads
+    from tests import gpu_harness as GH
+    wl = workloads.make("tiny", I=I, gh=6, gw=7, B=2, T=[5, 9], K=K)
+    g = GH.run(wl)
+    _check(g, [0, 1], TOL_F32)
+    assert g.comp.K == max(K, I)
+    wl2 = workloads.make("qwen", I=I, gh=8, gw=8, T=12, D=64, H=8, Hkv=2, K=K)
+    _check(GH.run(wl2), [0], TOL_BF16)
