@@ -250,13 +250,16 @@ typedef struct gmc_trace_header {
   float delta_bar;    /* mean best-minus-second-best selected cosine over discarded tokens */
   float F_S[3];       /* F_b(S) for the grounded, appearance, spatial banks */
   float F_V[3];       /* F_b(V) */
-  float c_B;          /* batched certificate 1 - prod_t (1 - q_t) (Eq. (6)) */
+  float c_B;          /* batched certificate 1 - prod_t (1 - q_t) over the rounds with U_t > 0,
+                         q_t = [F(S_t u B_t) - F(S_t)] / U_t, U_t the sum of the K largest
+                         singleton gains of unselected tokens (Sec. 4.1 Eq. (6); appendix Eq.
+                         (cond-batched-bound)), from the round gains and coverage below */
   int32_t reserved[3];
 } gmc_trace_header;
 
 typedef struct gmc_trace_layout {
   size_t bytes_per_image; /* the record size; gmc_trace_size() = B * bytes_per_image */
-  int rounds_max;         /* ceil(K / batch_b) + 1 */
+  int rounds_max;         /* ceil(K / batch_b) + 1, + 1 for prompts of several images */
   int pool_size;          /* pool_mult * batch_b */
   /* byte offsets inside one record */
   size_t off_order;       /* int32[K]   indices in the order they entered the support */
@@ -269,6 +272,9 @@ typedef struct gmc_trace_layout {
   size_t off_pi;          /* int32[N]   representative of every visual token */
   size_t off_ebar;        /* float[N]   normalised message energy */
   size_t off_mass;        /* float[N]   population weights m_i */
+  size_t off_gains;       /* int64[rounds_max][N]  singleton gains at the start of each round,
+                             fixed point (scale 2^e, e = 61 - ceil(log2(total bank mass))) */
+  size_t off_cover;       /* int64[rounds_max]  F(S) after each round, same fixed point */
 } gmc_trace_layout;
 
 /* Fill *out for this problem.  Returns GMC_OK or GMC_ERR_ARG. */

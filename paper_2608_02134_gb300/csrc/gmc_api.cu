@@ -171,7 +171,7 @@ size_t carve_compress(const Dims& dm, Scratch* s, char* base, R0State* r0s = nul
 R0State carve_round0(Carver& c, size_t B, size_t N, size_t M) {
   R0State r;
   r.pool = c.take<int32_t>(B * GMC_MAX_POOL);
-  r.info = c.take<int32_t>(B * 4);
+  r.info = c.take<int32_t>(B * INFO_W);
   r.s0 = c.take<long long>(B * GMC_MAX_POOL);
   r.u1 = c.take<long long>(B * N);
   r.u2 = c.take<long long>(B * N);
@@ -210,6 +210,8 @@ int fill_trace_layout(int B, const gmc_params& p, int N, int H, int K, gmc_trace
   L.off_pi = take(4 * (size_t)N);
   L.off_ebar = take(4 * (size_t)N);
   L.off_mass = take(4 * (size_t)N);
+  L.off_gains = take(8 * (size_t)L.rounds_max * N);
+  L.off_cover = take(8 * (size_t)L.rounds_max);
   L.bytes_per_image = (off + 15) & ~(size_t)15;
   *o = L;
   return GMC_OK;
@@ -228,6 +230,8 @@ TraceView make_trace_view(void* trace, const gmc_trace_layout& L) {
   tv.off_pi = L.off_pi;
   tv.off_ebar = L.off_ebar;
   tv.off_mass = L.off_mass;
+  tv.off_gains = L.off_gains;
+  tv.off_cover = L.off_cover;
   tv.rounds_max = L.rounds_max;
   tv.pool_size = L.pool_size;
   return tv;

@@ -52,7 +52,8 @@ int filter_rows_per_warp(int B, int M) {
 __global__ void __launch_bounds__(512) k_r0_pool(const long long* __restrict__ u0, int B, int N,
                                                    int P, const int32_t* toff, int Tmax, int I,
                                                    int32_t* pool0, int32_t* info, long long* s0,
-                                                   long long* u1, long long* fv, uint32_t* status) {
+                                                   long long* u1, long long* fv, uint32_t* status,
+                                                   TraceView tv) {
   grid_dep_wait();
   extern __shared__ __align__(16) char sm_r0p[];
   const int b = blockIdx.x;
@@ -61,12 +62,13 @@ __global__ void __launch_bounds__(512) k_r0_pool(const long long* __restrict__ u
   for (int j = threadIdx.x; j < N; j += blockDim.x) u1[(size_t)b * N + j] = 0;
   if (threadIdx.x < 4) fv[(size_t)b * 4 + threadIdx.x] = 0;
   if (threadIdx.x == 0) {
-    info[b * 4 + 1] = 0;
-    info[b * 4 + 2] = 0;
-    info[b * 4 + 3] = 0;
+    info[b * INFO_W + 1] = 0;
+    info[b * INFO_W + 2] = 0;
+    info[b * INFO_W + 3] = 0;
+    info[b * INFO_W + 4] = 0;
   }
   if (toff && text_geom(toff, b, B, Tmax, nullptr).T == 0) {
-    if (threadIdx.x == 0) info[b * 4] = 0;
+    if (threadIdx.x == 0) info[b * INFO_W] = 0;
     return;
   }
   sel::PoolScratch w;
@@ -84,6 +86,7 @@ __global__ void __launch_bounds__(512) k_r0_pool(const long long* __restrict__ u
   for (int j = threadIdx.x; j < N; j += blockDim.x) {
     selz[j] = 0;
     ug[j] = u0[(size_t)b * N + j];  // the gains in shared memory: select_pool reads them often
+    if (tv.base) tv.gains(b, 0, N)[j] = ug[j];
   }
   for (int h = threadIdx.x; h < sel::HBINS; h += blockDim.x) w.hist[h] = 0;
   if (threadIdx.x < sel::CBINS) w.coarse[threadIdx.x] = 0;
@@ -113,12 +116,12 @@ __global__ void __launch_bounds__(512) k_r0_pool(const long long* __restrict__ u
       if (lane == 0) pool0[(size_t)b * P + k] = bj;
     }
     for (int k = I + threadIdx.x; k < P; k += blockDim.x) pool0[(size_t)b * P + k] = -1;
-    if (threadIdx.x == 0) info[b * 4] = I;
+    if (threadIdx.x == 0) info[b * INFO_W] = I;
     return;
   }
   const int Pt = sel::select_pool(ug, selz, N, P, w, pool, nullptr);
   for (int k = threadIdx.x; k < P; k += blockDim.x) pool0[(size_t)b * P + k] = k < Pt ? pool[k] : -1;
-  if (threadIdx.x == 0) info[b * 4] = Pt;
+  if (threadIdx.x == 0) info[b * INFO_W] = Pt;
 }
 
 __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_rho(
@@ -130,7 +133,7 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_rho(
   __shared__ int pool[GMC_MAX_POOL];
   __shared__ long long sblk[GMC_MAX_POOL];
   const int b = blockIdx.y;
-  const int Pt = info[b * 4];
+  const int Pt = info[b * INFO_W];
   if (Pt == 0) return;
   int Mb = Mstride;
   if (!uniform_rows) Mb = H * text_geom(toff, b, B, Tmax, nullptr).T + N + L2;
@@ -193,7 +196,7 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_filter(
   // the block's contributions to the next gains, one global atomic per column at the end
   extern __shared__ unsigned long long uacc[];  // [N]
   const int b = blockIdx.y;
-  const int Pt = info[b * 4];
+  const int Pt = info[b * INFO_W];
   if (Pt == 0) return;
   int Mb = Mstride, MG = Mstride;
   if (!uniform_rows) {
@@ -223,8 +226,8 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_filter(
   if (blockIdx.x == 0) {  // record the first batch once per image
     for (int q = threadIdx.x; q < nb; q += blockDim.x) order[(size_t)b * K + q] = batch[q];
     if (threadIdx.x == 0) {
-      info[b * 4 + 1] = nb;  // selected so far
-      info[b * 4 + 2] = 1;   // rounds done
+      info[b * INFO_W + 1] = nb;  // selected so far
+      info[b * INFO_W + 2] = 1;   // rounds done
     }
     if (tv.base) {
       int32_t* tp = tv.at<int32_t>(b, tv.off_pool);
@@ -310,6 +313,7 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_filter(
       cnt[(size_t)b * Mstride + m] = w;
       const int bank = m < MG ? 0 : (m < MG + N ? 1 : 2);
       atomicAdd((unsigned long long*)&fb[bank], (unsigned long long)to_fix(rowmax, fxs));
+      if (tv.base) atomicAdd(tv.cover(b, 0), (unsigned long long)fb_new);  // F after the round
     }
   }
   __syncthreads();
@@ -333,12 +337,12 @@ __global__ void __launch_bounds__(512) k_rg_pool(const long long* __restrict__ u
   const int b = blockIdx.x;
   for (int k = threadIdx.x; k < P; k += blockDim.x) sc[(size_t)b * P + k] = 0;
   for (int j = threadIdx.x; j < N; j += blockDim.x) unext[(size_t)b * N + j] = 0;
-  const int S = info[b * 4 + 1], rd = info[b * 4 + 2];
+  const int S = info[b * INFO_W + 1], rd = info[b * INFO_W + 2];
   // nothing to do here once the budget is met or when the first round found
   // no gain: the cluster kernel handles those cases
   const bool skip = (toff && text_geom(toff, b, B, Tmax, nullptr).T == 0) || rd == 0 || S >= K;
   if (skip) {
-    if (threadIdx.x == 0) info[b * 4] = 0;
+    if (threadIdx.x == 0) info[b * INFO_W] = 0;
     return;
   }
   sel::PoolScratch w;
@@ -356,6 +360,7 @@ __global__ void __launch_bounds__(512) k_rg_pool(const long long* __restrict__ u
   for (int j = threadIdx.x; j < N; j += blockDim.x) {
     self[j] = 0;
     ug[j] = ucur[(size_t)b * N + j];  // the gains in shared memory: select_pool reads them often
+    if (tv.base) tv.gains(b, rd, N)[j] = ug[j];
   }
   for (int h = threadIdx.x; h < sel::HBINS; h += blockDim.x) w.hist[h] = 0;
   if (threadIdx.x < sel::CBINS) w.coarse[threadIdx.x] = 0;
@@ -365,8 +370,9 @@ __global__ void __launch_bounds__(512) k_rg_pool(const long long* __restrict__ u
   const int Pt = sel::select_pool(ug, self, N, P, w, pool, nullptr);
   for (int k = threadIdx.x; k < P; k += blockDim.x) pool0[(size_t)b * P + k] = k < Pt ? pool[k] : -1;
   if (threadIdx.x == 0) {
-    info[b * 4] = Pt;
-    info[b * 4 + 3] = S;
+    info[b * INFO_W] = Pt;
+    info[b * INFO_W + 3] = S;
+    info[b * INFO_W + 4] = rd;
   }
   if (tv.base && Pt > 0) {
     int32_t* tp = tv.at<int32_t>(b, tv.off_pool) + (size_t)rd * tv.pool_size;
@@ -386,7 +392,7 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_rg_rho(
   __shared__ float fres[R0_ROWS][GMC_MAX_POOL];
   extern __shared__ short pslot[];              // [N] pool slot of every token or -1
   const int b = blockIdx.y;
-  const int Pt = info[b * 4];
+  const int Pt = info[b * INFO_W];
   if (Pt == 0) return;
   int Mb = Mstride;
   if (!uniform_rows) Mb = H * text_geom(toff, b, B, Tmax, nullptr).T + N + L2;
@@ -469,13 +475,13 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_rg_filter(
   extern __shared__ unsigned long long uacc[];  // [N] then the batch flags [N] (bytes)
   unsigned char* inb = reinterpret_cast<unsigned char*>(uacc + N);
   const int b = blockIdx.y;
-  const int Pt = info[b * 4];
+  const int Pt = info[b * INFO_W];
   if (Pt == 0) return;
   int Mb = Mstride;
   if (!uniform_rows) Mb = H * text_geom(toff, b, B, Tmax, nullptr).T + N + L2;
   const int m0 = blockIdx.x * R0_ROWS * rpw;
   if (m0 >= Mb) return;
-  const int S = info[b * 4 + 3], rd = info[b * 4 + 2];
+  const int S = info[b * INFO_W + 3], rd = info[b * INFO_W + 4];
   const float fxs = ldexpf(1.f, fexp ? fexp[b] : fx_exp);
   const int nb = min(bsz, min(Pt, K - S));
   for (int k = threadIdx.x; k < Pt; k += blockDim.x) {
@@ -500,8 +506,8 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_rg_filter(
   if (blockIdx.x == 0) {  // record the batch once per image
     for (int q = threadIdx.x; q < nb; q += blockDim.x) order[(size_t)b * K + S + q] = batch[q];
     if (threadIdx.x == 0) {
-      info[b * 4 + 1] = S + nb;
-      info[b * 4 + 2] = rd + 1;
+      info[b * INFO_W + 1] = S + nb;
+      info[b * INFO_W + 2] = rd + 1;
       if (tv.base) tv.at<int32_t>(b, tv.off_round_end)[rd] = S + nb;
     }
   }
@@ -564,6 +570,7 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_rg_filter(
     if (lane == 0) {
       bcov[row] = bnew;
       cnt[row] = wr;
+      if (tv.base) atomicAdd(tv.cover(b, rd), (unsigned long long)fb_new);  // F after the round
     }
   }
   __syncthreads();
@@ -585,7 +592,7 @@ cudaError_t launch_round0(const R0State& r0, int B, int N, int K, int M, const i
   if ((e = set_smem_limit((const void*)k_r0_pool, smem)) != cudaSuccess) return e;
   const int uniform = (H == 0);
   launch_k(k_r0_pool, B, 512, smem, st, 1, u0, B, N, P, uniform ? nullptr : toff, T, I, r0.pool, r0.info,
-                                  r0.s0, r0.u1, r0.fv, status);
+                                  r0.s0, r0.u1, r0.fv, status, tv);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   dim3 grid(ceil_div(M, R0_ROWS), B);
   launch_k(k_r0_rho, grid, 32 * R0_ROWS, 0, st, 1, C, B, N, M, H, L2, toff, T, uniform, r0.pool, r0.info,

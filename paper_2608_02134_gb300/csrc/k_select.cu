@@ -236,9 +236,9 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
   // state after the rounds run on the whole GPU (k_round0.cu); a first round
   // with an empty pool leaves the gains of the empty support and nothing
   // selected
-  const int rd0 = valid ? a.r0.info[b * 4 + 2] : 0;  // rounds done
+  const int rd0 = valid ? a.r0.info[b * INFO_W + 2] : 0;  // rounds done
   const int Pt0 = rd0;                                // > 0: the rounds left survivor lists
-  const int nb0 = rd0 > 0 ? a.r0.info[b * 4 + 1] : 0;  // tokens selected so far
+  const int nb0 = rd0 > 0 ? a.r0.info[b * INFO_W + 1] : 0;  // tokens selected so far
   for (int j = threadIdx.x; j < N; j += blockDim.x) {
     s.u_full[j] = rd0 > 0 ? a.r0.ugain[(size_t)b * N + j] : a.u0[(size_t)b * N + j];
     s.poolslot[j] = -1;
@@ -395,6 +395,8 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
       if (threadIdx.x == 0) set_status(a.status, GMC_STATUS_INTERNAL);
       break;
     }
+    if (r == 0 && a.tv.base)  // certificate input: the gains this round starts from
+      for (int j = threadIdx.x; j < N; j += blockDim.x) a.tv.gains(b, rnd, N)[j] = s.u_full[j];
     // ---- pool of this round ------------------------------------------------------
     sel::PoolScratch pw{s.hist, s.coarse, s.bnd, s.key, s.pk, s.wsum, s.scal + 8};
     const int Pt = sel::select_pool(s.u_full, s.sel, N, P, pw, s.pool, s.poolslot);
@@ -772,6 +774,13 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
     }
     }
     __syncthreads();
+    if (a.tv.base) {  // certificate input: F(S) after this round, this CTA's rows
+      long long f = 0;
+      for (int q = threadIdx.x; q < nrows; q += blockDim.x) f += to_fix(s.bcov[q], fxs);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) f += __shfl_xor_sync(FULL, f, o);
+      if (lane == 0 && f) atomicAdd(a.tv.cover(b, rnd), (unsigned long long)f);
+    }
     for (int k = threadIdx.x; k < Pt; k += blockDim.x) {
       s.poolslot[s.pool[k]] = -1;
       s.s_acc[k] = 0;
@@ -842,7 +851,6 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
         hd->F_S[q] = (float)((double)s.fb[q] * inv);
         hd->F_V[q] = (float)((double)a.r0.fv[(size_t)b * 4 + q] * inv);
       }
-      hd->c_B = -1.f;  // not computed by this build
     }
     int32_t* to = a.tv.at<int32_t>(b, a.tv.off_order);
     for (int q = threadIdx.x; q < K; q += blockDim.x) to[q] = a.order[(size_t)b * K + q];
@@ -853,6 +861,97 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
          q < (size_t)a.tv.rounds_max * a.tv.pool_size; q += blockDim.x)
       tp[q] = -1;
   }
+}
+
+// Batched certificate (Sec. 4.1 Eq. (6); appendix Eq. (cond-batched-bound)),
+// computed only for the diagnostics trace from what the solver recorded there:
+// round t's gains u^t and F(S) after it.  U_t, the sum of the K largest gains
+// of the tokens not selected before round t, comes from the K-th largest gain
+// theta (binary search on the fixed-point value, counting on the whole
+// block): U_t = sum_{u > theta} u + (K - #{u > theta}) theta, exactly.
+// c_B = 1 - prod_t (1 - q_t) over the rounds with U_t > 0,
+// q_t = (F_t - F_{t-1}) / U_t.  One block per image.
+__global__ void __launch_bounds__(256) k_certificate(int N, int K, TraceView tv) {
+  grid_dep_wait();
+  extern __shared__ __align__(16) char sm_cert[];
+  long long* g = reinterpret_cast<long long*>(sm_cert);               // [N]
+  unsigned char* done = reinterpret_cast<unsigned char*>(g + N);      // [N] selected before t
+  __shared__ long long red[8];
+  __shared__ unsigned long long red2[8];
+  const int b = blockIdx.x;
+  gmc_trace_header* hd = tv.header(b);
+  const int R = hd->rounds;
+  const int32_t* order = tv.at<int32_t>(b, tv.off_order);
+  const int32_t* rend = tv.at<int32_t>(b, tv.off_round_end);
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  for (int j = threadIdx.x; j < N; j += blockDim.x) done[j] = 0;
+  // block sum of (count, value) over the unselected tokens with g > x (or >= x)
+  auto count_ge = [&](long long x) {
+    long long c = 0;
+    for (int j = threadIdx.x; j < N; j += blockDim.x) c += (!done[j] && g[j] >= x);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(FULL, c, o);
+    __syncthreads();
+    if (lane == 0) red[wid] = c;
+    __syncthreads();
+    long long t = 0;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += red[w];
+    return t;
+  };
+  double prod = 1.0, Fprev = 0.0;
+  const double inv = 1.0;  // q_t is a ratio of two fixed-point values: the scale cancels
+  for (int t = 0; t < R; ++t) {
+    __syncthreads();
+    const int before = t > 0 ? rend[t - 1] : 0;
+    for (int q = threadIdx.x; q < before; q += blockDim.x) done[order[q]] = 1;
+    const long long* gt = tv.gains(b, t, N);
+    for (int j = threadIdx.x; j < N; j += blockDim.x) g[j] = gt[j] < 0 ? 0 : gt[j];
+    __syncthreads();
+    // theta = the largest x with #{u >= x} >= K (0 when fewer than K tokens
+    // remain).  Every gain is at most the fixed-point total mass, below 2^62, so
+    // the search range [0, 2^62] halves in at most 63 steps
+    long long lo = 0, hi = 1LL << 62;
+    if (count_ge(0) >= K) {
+      for (int it = 0; it < 64 && lo < hi; ++it) {
+        const long long mid = lo + (hi - lo + 1) / 2;
+        if (count_ge(mid) >= K) lo = mid; else hi = mid - 1;
+      }
+    }
+    const long long theta = lo;
+    // sum and count of the gains above theta
+    unsigned long long sv = 0;
+    long long cv = 0;
+    for (int j = threadIdx.x; j < N; j += blockDim.x)
+      if (!done[j] && g[j] > theta) {
+        sv += (unsigned long long)g[j];
+        ++cv;
+      }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      sv += __shfl_xor_sync(FULL, sv, o);
+      cv += __shfl_xor_sync(FULL, cv, o);
+    }
+    __syncthreads();
+    if (lane == 0) {
+      red2[wid] = sv;
+      red[wid] = cv;
+    }
+    __syncthreads();
+    unsigned long long S = 0;
+    long long C = 0;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) {
+      S += red2[w];
+      C += red[w];
+    }
+    const long long remain = count_ge(0);
+    const double U = remain >= K ? (double)S + (double)(K - C) * (double)theta : (double)S;
+    const double F = (double)*tv.cover(b, t) * inv;
+    if (U > 0.0) {
+      prod *= 1.0 - (F - Fprev) / U;
+      Fprev = F;
+    }
+  }
+  if (threadIdx.x == 0) hd->c_B = (float)(1.0 - prod);
 }
 
 static int g_num_sms = 0;
@@ -924,7 +1023,12 @@ cudaError_t launch_select(const R0State& r0, int B, int N, int K, int M, const i
     attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // see grid_dep_wait
     attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.numAttrs = 2;
-    return cudaLaunchKernelEx(&cfg, k_select, a);
+    if ((e = cudaLaunchKernelEx(&cfg, k_select, a)) != cudaSuccess || !tv.base) return e;
+    // diagnostics trace: the batched certificate from the recorded rounds
+    const size_t csm = (sizeof(long long) + 1) * (size_t)N;
+    if ((e = set_smem_limit((const void*)k_certificate, csm)) != cudaSuccess) return e;
+    launch_k(k_certificate, B, 256, csm, st, 1, N, K, tv);
+    return cudaGetLastError();
   }
   return cudaErrorInvalidConfiguration;
 }

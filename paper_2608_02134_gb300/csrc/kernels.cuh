@@ -27,7 +27,7 @@ struct Dims {
 struct TraceView {
   char* base;  // nullptr: no trace
   size_t stride, off_order, off_round_end, off_pool, off_centres, off_head_assign, off_omega,
-      off_pi, off_ebar, off_mass;
+      off_pi, off_ebar, off_mass, off_gains, off_cover;
   int rounds_max, pool_size;
   __device__ __forceinline__ char* rec(int b) const { return base + (size_t)b * stride; }
   __device__ __forceinline__ gmc_trace_header* header(int b) const {
@@ -35,6 +35,13 @@ struct TraceView {
   }
   template <typename T> __device__ __forceinline__ T* at(int b, size_t off) const {
     return reinterpret_cast<T*>(rec(b) + off);
+  }
+  // round rd's gains row and F(S) slot (certificate inputs)
+  __device__ __forceinline__ long long* gains(int b, int rd, int N) const {
+    return at<long long>(b, off_gains) + (size_t)rd * N;
+  }
+  __device__ __forceinline__ unsigned long long* cover(int b, int rd) const {
+    return at<unsigned long long>(b, off_cover) + rd;
   }
 };
 
@@ -144,10 +151,16 @@ cudaError_t launch_build_clients(const Dims&, const gmc_params&, int fx_exp, Scr
 // counts were chosen by measurement.
 __host__ __device__ inline int sparse_gpu_rounds(int N) { return N > 2048 ? 8 : 4; }
 
+// per-image words of R0State::info
+constexpr int INFO_W = 8;
+
 struct R0State {
   int32_t* pool;   // [B][P]  pool of the current whole-GPU round (-1 padded)
-  int32_t* info;   // [B][4]  pool size of the current round, tokens selected so far,
-                   //         rounds done, tokens selected before the current round
+  int32_t* info;   // [B][INFO_W]  pool size of the current round, tokens selected so far,
+                   //         rounds done, tokens selected before the current round,
+                   //         rounds done before the current round (the last two are
+                   //         snapshots the pool kernel takes, read by every filter block
+                   //         while block 0 advances the running counts)
   long long* s0;   // [B][P]  scores of the current round (fixed point)
   long long* u1;   // [B][N]  gains (fixed point), written by rounds 0, 2, ...
   long long* u2;   // [B][N]  gains written by rounds 1, 3, ...

@@ -82,7 +82,8 @@ class TraceLayout(ctypes.Structure):
                 ("off_round_end", ctypes.c_size_t), ("off_pool", ctypes.c_size_t),
                 ("off_centres", ctypes.c_size_t), ("off_head_assign", ctypes.c_size_t),
                 ("off_omega", ctypes.c_size_t), ("off_pi", ctypes.c_size_t),
-                ("off_ebar", ctypes.c_size_t), ("off_mass", ctypes.c_size_t)]
+                ("off_ebar", ctypes.c_size_t), ("off_mass", ctypes.c_size_t),
+                ("off_gains", ctypes.c_size_t), ("off_cover", ctypes.c_size_t)]
 
 
 _lib = None

@@ -79,6 +79,7 @@ class ImageTrace:
     delta_bar: float
     F_S: list
     F_V: list
+    c_B: float
     order: np.ndarray
     round_end: np.ndarray
     pool: np.ndarray
@@ -113,6 +114,7 @@ def parse_trace(buf: np.ndarray, layout, B: int, K: int, H: int, N: int, max_clu
         R, P = layout.rounds_max, layout.pool_size
         out.append(ImageTrace(
             hd.K, hd.rounds, hd.n_clusters, hd.filled, hd.s_x, hd.delta_bar, list(hd.F_S), list(hd.F_V),
+            hd.c_B,
             arr(layout.off_order, K, np.int32), arr(layout.off_round_end, R, np.int32),
             arr(layout.off_pool, R * P, np.int32).reshape(R, P),
             arr(layout.off_centres, max_clusters, np.int32), arr(layout.off_head_assign, H, np.int32),

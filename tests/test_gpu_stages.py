@@ -59,6 +59,9 @@ def _check_select(C, K, **pk):
         assert traces[b].K == K and traces[b].rounds == len(sel.rounds)
         fs = O.facility_value(C64, sel.support)
         assert abs(traces[b].F_S[0] - fs) <= 1e-5 * max(fs, 1e-30)
+        # batched certificate Eq. (6) along the same rounds
+        assert abs(traces[b].c_B - O.batched_certificate(sel)) <= 1e-4, (traces[b].c_B,
+                                                                          O.batched_certificate(sel))
     assert not fails, "\n".join(fails[:10])
     return idx, traces, ties
 
