@@ -55,6 +55,12 @@ Readings taken where the paper is silent or ambiguous:
     completed views; each view carries its own layer's queries, keys, values
     and probe W = O_h P; omega_h and nu_t weight every view's rows; the
     message energy is the current view's only.
+  * Long prefixes (bounded appearance bank): the rank-r Rademacher map R
+    [r, D] (+-1 entries, numpy default_rng(104729), an input like the probe)
+    acts on the raw boundary state and the result is normalised,
+    x~_i = R h_i / ||R h_i||; the M_V = min(N, 4096) clients are the tokens
+    floor(m N / M_V); their rows carry beta_V / M_V; the assignment uses the
+    cosines of the unprojected states against the support only.
 
 Pins (tests/test_oracle_pins.py; the paper prints no worked numeric example,
 so every function is pinned by a closed form, an invariant, a bound of the
@@ -109,6 +115,15 @@ paper, a hand-worked case or brute force on tiny inputs, never by itself):
     pattern Grams; duplicated views keep the single-view cosines and head
     weights; no history or zero history mass leaves the step unchanged; each
     view's rows carry its mass; the energy stays the current view's.
+  * bounded_client_tokens / projected_states / bounded_appearance_clients /
+    support_cosines / compress(long_prefix=...): uniform spacing (count,
+    first token, gaps of floor or ceil N/M_V); under an orthogonal +-1 map
+    (a signed, column-permuted Sylvester-Hadamard matrix, D = r) projected
+    cosines equal the exact ones, so every bounded row is the exact bank's
+    row of its client token and, with M_V >= N, the whole step equals the
+    exact-bank step; a null-space component of R leaves x~ unchanged; a
+    Johnson-Lindenstrauss bound on random maps; support-column cosines give
+    the full-matrix assignment; appearance rows carry beta_V / M_V each.
 
 Discrete choices (pool, batch, head centres, assignment) are recorded together
 with the fp64 values that decide them.  Every choice can also be *forced*
@@ -422,6 +437,48 @@ def appearance_clients(cos: np.ndarray, p: dict, n_images: int = 1) -> np.ndarra
     return E / E.sum(axis=1, keepdims=True)
 
 
+# ---------------------------------------------------------------------------
+# Long prefixes: the bounded appearance bank (appendix "Appearance and spatial
+# clients", last paragraph, and the cost paragraphs after Algorithm 1; Table
+# "Shared GMC configuration", long-prefix row: rank 128, M_V <= 4096, b = 512)
+# ---------------------------------------------------------------------------
+def bounded_client_tokens(N: int, max_clients: int) -> np.ndarray:
+    """The M_V = min(N, max_clients) uniformly spaced source tokens that act as
+    appearance clients: c(m) = floor(m N / M_V), m = 0 .. M_V - 1 (every
+    token when N <= max_clients)."""
+    MV = min(N, max_clients)
+    return (np.arange(MV, dtype=np.int64) * N) // MV
+
+
+def projected_states(hvis: np.ndarray, R: np.ndarray, p: dict) -> np.ndarray:
+    """Appearance states under the fixed rank-r Rademacher map R [r, D]:
+    y_i = R h_i, x~_i = y_i / max(||y_i||, eps).  [N, r].  Normalising after
+    the map makes x~ independent of R's scale (1 or 1/sqrt(r))."""
+    y = hvis @ R.T
+    n = np.sqrt(np.sum(y * y, axis=1))
+    return y / np.maximum(n, p["norm_eps"])[:, None]
+
+
+def bounded_appearance_clients(xt: np.ndarray, clients: np.ndarray, p: dict,
+                               n_images: int = 1) -> np.ndarray:
+    """Row m: P^V_m(i) proportional to exp(x~_{c(m)}^T x~_i / tau_v) over every
+    token i of client c(m)'s image, normalised.  [M_V, N]."""
+    logits = (xt[clients] @ xt.T) / p["tau_v"]
+    if n_images > 1:
+        img = image_index(xt.shape[0], n_images)
+        logits = np.where(img[clients][:, None] == img[None, :], logits, -np.inf)
+    logits = logits - logits.max(axis=1, keepdims=True)
+    E = np.exp(logits)
+    return E / E.sum(axis=1, keepdims=True)
+
+
+def support_cosines(hvis: np.ndarray, S_sorted: np.ndarray, p: dict) -> np.ndarray:
+    """cos(h_i, h_j) for every token i and selected j: [N, K], column k the
+    k-th selected token (the N x K product the assignment needs)."""
+    x = unit_states(hvis, p)
+    return x @ x[np.asarray(S_sorted, dtype=np.int64)].T
+
+
 def grid_coords(gh: int, gw: int) -> np.ndarray:
     """Normalised source coordinates p_i = ((r+0.5)/gh, (c+0.5)/gw), i = r*gw + c."""
     r, c = np.divmod(np.arange(gh * gw), gw)
@@ -472,17 +529,20 @@ def client_matrix(PG, activeG, omega, nu, PV, PS, p) -> ClientMatrix:
     """Stack the three banks: rows (h, t) h-major, then appearance rows m, then landmarks l.
 
     Grounded row (h, t): beta_G * omega_h * nu_t * a_{h,t} * P^G_{h,t}.
-    Appearance row m: (beta_V / N) P^V_m.  Spatial row l: (beta_S / M_S) P^S_l.
+    Appearance row m: (beta_V / M_V) P^V_m, M_V = N on the exact bank (every
+    token a client) or the bounded bank's client count.  Spatial row l:
+    (beta_S / M_S) P^S_l.
     """
     H, T, N = PG.shape
+    MV = PV.shape[0]
     wG = p["beta_G"] * omega[:, None] * nu[None, :] * activeG
     G = (wG[:, :, None] * PG).reshape(H * T, N)
-    V = (p["beta_V"] / N) * PV
+    V = (p["beta_V"] / MV) * PV
     S = (p["beta_S"] / PS.shape[0]) * PS
     C = np.concatenate([G, V, S], axis=0)
-    banks = {"grounded": slice(0, H * T), "appearance": slice(H * T, H * T + N),
-             "spatial": slice(H * T + N, H * T + N + PS.shape[0])}
-    active = np.concatenate([activeG.reshape(-1), np.ones(N, bool), np.ones(PS.shape[0], bool)])
+    banks = {"grounded": slice(0, H * T), "appearance": slice(H * T, H * T + MV),
+             "spatial": slice(H * T + MV, H * T + MV + PS.shape[0])}
+    active = np.concatenate([activeG.reshape(-1), np.ones(MV, bool), np.ones(PS.shape[0], bool)])
     return ClientMatrix(C, banks, active)
 
 
@@ -504,14 +564,14 @@ def client_matrix_views(PGs, actives, betas, omega, nu, PV, PS, p) -> ClientMatr
         act.append(a.reshape(-1))
         views[v] = slice(at, at + H * T)
         at += H * T
-    N = PV.shape[0]
+    MV = PV.shape[0]  # appearance clients (N on the exact bank)
     G = np.concatenate(blocks, axis=0)
-    V = (p["beta_V"] / N) * PV
+    V = (p["beta_V"] / MV) * PV
     S = (p["beta_S"] / PS.shape[0]) * PS
     C = np.concatenate([G, V, S], axis=0)
-    banks = {"grounded": slice(0, at), "appearance": slice(at, at + N),
-             "spatial": slice(at + N, at + N + PS.shape[0])}
-    active = np.concatenate(act + [np.ones(N, bool), np.ones(PS.shape[0], bool)])
+    banks = {"grounded": slice(0, at), "appearance": slice(at, at + MV),
+             "spatial": slice(at + MV, at + MV + PS.shape[0])}
+    active = np.concatenate(act + [np.ones(MV, bool), np.ones(PS.shape[0], bool)])
     return ClientMatrix(C, banks, active, views)
 
 
@@ -688,7 +748,7 @@ class Assignment:
 
 
 def assign_population(cos: np.ndarray, S: np.ndarray, gh: int, gw: int, p: dict,
-                      forced_pi=None, n_images: int = 1) -> Assignment:
+                      forced_pi=None, n_images: int = 1, support_cols: bool = False) -> Assignment:
     """pi(i) = argmax_{j in S} cos_ij + lambda_p s_x g_i exp(-||p_i - p_j||^2 / tau_s).
 
     Selected tokens represent themselves.  delta_i is the gap between the
@@ -698,9 +758,16 @@ def assign_population(cos: np.ndarray, S: np.ndarray, gh: int, gw: int, p: dict,
     g_i = exp[-(delta_i / ambig_margin)^gate_pow].  Ties go to the lowest j.
     With several images, token i's candidates S_i are the selected tokens of
     its own image, and both the gap and the coordinates are within that image.
+    support_cols: ``cos`` is [N, |S|], column k holding the cosines with the
+    k-th token of S (``support_cosines``), instead of [N, N].
     """
     N = cos.shape[0]
     S = np.asarray(S, dtype=np.int64)
+    if support_cols:
+        colof = {int(j): k for k, j in enumerate(S)}
+        cos_at = lambda i, js: cos[i, [colof[int(j)] for j in js]]  # noqa: E731
+    else:
+        cos_at = lambda i, js: cos[i, js]  # noqa: E731
     in_S = np.zeros(N, bool)
     in_S[S] = True
     disc = np.flatnonzero(~in_S)
@@ -708,7 +775,7 @@ def assign_population(cos: np.ndarray, S: np.ndarray, gh: int, gw: int, p: dict,
     compat = {int(i): S[img[S] == img[i]] for i in disc}  # S_i: same-image carriers
     delta = np.zeros(N)
     for i in disc:
-        v = np.sort(cos[i, compat[int(i)]])[::-1]
+        v = np.sort(cos_at(i, compat[int(i)]))[::-1]
         delta[i] = v[0] - v[1] if v.size > 1 else 0.0
     delta_bar = float(delta[disc].mean()) if disc.size else 0.0
     s_x = 1.0 - math.exp(-((delta_bar / p["gate_scale"]) ** p["gate_pow"]))
@@ -720,7 +787,7 @@ def assign_population(cos: np.ndarray, S: np.ndarray, gh: int, gw: int, p: dict,
     for i in disc:
         Si = compat[int(i)]
         d2 = np.sum((P[Si] - P[i]) ** 2, axis=1)
-        kappa = cos[i, Si] + p["assign_spatial_w"] * s_x * g[i] * np.exp(-d2 / p["tau_s"])
+        kappa = cos_at(i, Si) + p["assign_spatial_w"] * s_x * g[i] * np.exp(-d2 / p["tau_s"])
         j = int(stable_top(kappa, Si, 1)[0])
         pi[i] = j if forced_pi is None else int(forced_pi[i])
         kb[i] = kappa.max()
@@ -819,10 +886,13 @@ class Result:
     out_pos: np.ndarray = None     # [3, K+T]
     out_prefix_kv: np.ndarray = None  # [p, 2, K+T, Hkv, d] dense prefix layers at the kept rows
     history: list = None           # per historical view: (A, Z, sigma, unorm, PG, active)
+    xt: np.ndarray = None          # long prefixes: projected appearance states [N, r]
+    clients_V: np.ndarray = None   # long prefixes: tokens of the appearance clients [M_V]
+    cos_support: np.ndarray = None  # long prefixes: support cosines [N, K]
 
 
 def compress(hidden, Kall, Vall, Q, pos, W, gh, gw, K_r, p=None, forced=None,
-             history=None, prefix=None, n_images: int = 1) -> Result:
+             history=None, prefix=None, n_images: int = 1, long_prefix=None) -> Result:
     """Grounded Message Coreset compression of one image boundary.
 
     hidden [N+T, D], Kall/Vall [N+T, Hkv, d], Q [T, H, d], pos [3, N+T],
@@ -840,6 +910,14 @@ def compress(hidden, Kall, Vall, Q, pos, W, gh, gw, K_r, p=None, forced=None,
     ``prefix`` (optional) lists the dense prefix layers' (K, V), each
     [N+T, Hkv, d]; ``out_prefix_kv`` then holds them at the kept rows
     (``gather_prefix_kv``).
+    ``long_prefix`` (optional) selects the bounded appearance bank of long
+    prefixes: a dict with the Rademacher map "R" [r, D] and "max_clients".
+    The appearance clients are then the uniformly spaced tokens of
+    ``bounded_client_tokens`` over the projected states, and the assignment
+    reads only the N x K support cosines (``support_cosines``); ``cos`` is
+    None and ``cos_support`` holds them.  The responsibility batch b comes
+    from ``p`` as always (the long-prefix row of the configuration table uses
+    b = 512).
     """
     p = p or params()
     forced = forced or {}
@@ -873,8 +951,13 @@ def compress(hidden, Kall, Vall, Q, pos, W, gh, gw, K_r, p=None, forced=None,
     res.heads = head_clusters(res.A, res.Z, res.sigma, p,
                               forced.get("centres"), forced.get("head_assign"), views=views)
     res.e, res.ebar = message_energy(res.unorm, res.heads.omega, res.nu)
-    res.cos = cosine_matrix(hvis, p)
-    PV = appearance_clients(res.cos, p, n_images)
+    if long_prefix is None:
+        res.cos = cosine_matrix(hvis, p)
+        PV = appearance_clients(res.cos, p, n_images)
+    else:
+        res.xt = projected_states(hvis, np.asarray(long_prefix["R"], dtype=np.float64), p)
+        res.clients_V = bounded_client_tokens(N, int(long_prefix["max_clients"]))
+        PV = bounded_appearance_clients(res.xt, res.clients_V, p, n_images)
     PS = spatial_clients(gh, gw, p, n_images)
     if history is None:
         res.clients = client_matrix(res.PG, res.activeG, res.heads.omega, res.nu, PV, PS, p)
@@ -885,8 +968,13 @@ def compress(hidden, Kall, Vall, Q, pos, W, gh, gw, K_r, p=None, forced=None,
     res.selection = select_support(res.clients.C, K, p, forced=forced.get("rounds"),
                                    n_images=n_images)
     res.support = res.selection.support
-    res.assignment = assign_population(res.cos, res.support, gh, gw, p, forced.get("pi"),
-                                       n_images)
+    if long_prefix is None:
+        res.assignment = assign_population(res.cos, res.support, gh, gw, p, forced.get("pi"),
+                                           n_images)
+    else:
+        res.cos_support = support_cosines(hvis, res.support, p)
+        res.assignment = assign_population(res.cos_support, res.support, gh, gw, p,
+                                           forced.get("pi"), n_images, support_cols=True)
     res.m = population_weights(res.ebar, res.assignment.s_x, p)
     res.transport = transport(hvis, res.support, res.assignment.pi, res.m, p)
     res.rows = compaction_rows(res.support, N, T)

@@ -26,6 +26,13 @@ no benchmark image, prompt or checkpoint is used):
   multi    one prompt with two qwen-shaped images (N = 2 x 1296, each 36x36,
            one after the other), T=64, K=514 (20%), bf16; every image drawn
            like a qwen image from its own substream (seed, 0, 1000 + image).
+  longdoc  the paper's long-prefix document path: qwen dims, N=15876
+           (126x126), T=128, K=4096, bf16, drawn like doc (rank-32
+           background, isolated rows at doc's density: 775 of them); bounded
+           appearance bank with rank 128, at most 4096 clients, b = 512.
+  longsmall a small long-prefix case for parity: N=1600 (40x40), T=16, H=4,
+           Hkv=2, d=64, D=256, K=320, bf16, drawn like doc (80 isolated
+           rows); rank 128, at most 512 clients, b = 64 (pool 256).
 
 Values are drawn in fp32; bf16 workloads round them once to bf16 (round to
 nearest even) and every consumer reads the rounded values.  Values V ~ N(0,1).
@@ -42,6 +49,9 @@ boundary tensors above do not change.  Where the image has object regions,
 the view's visual keys follow the same regions with fresh region centres.
 Dense prefix layers (``prefix_kv``): keys and values of the layers before the
 boundary, N(0, 1) from substreams (seed, image, 100 + layer).
+Long-prefix Rademacher map (``rademacher``): r x D entries +-1 with equal
+probability from numpy default_rng(104729) (the seed of the paper's
+configuration table), an input of both the CUDA path and the oracle.
 """
 
 from __future__ import annotations
@@ -59,8 +69,24 @@ WORKLOADS = {
     "serving": (4, 32, 36, 36, None, 28, 4, 128, 3584, 257, "bf16", "regions+detail", "mrope"),
     # multi-image prompt: two qwen-shaped images (2 x 36 x 36 visual tokens) before the text
     "multi": (5, 1, 36, 36, 64, 28, 4, 128, 3584, 514, "bf16", "regions+detail", "mrope"),
+    # long prefixes: the bounded appearance bank (LONG_PREFIX below)
+    "longdoc": (6, 1, 126, 126, 128, 28, 4, 128, 3584, 4096, "bf16", "lowrank", "mrope"),
+    "longsmall": (7, 1, 40, 40, 16, 4, 2, 64, 256, 320, "bf16", "lowrank", "mrope"),
 }
 IMAGES = {"multi": 2}  # images per boundary (1 when absent)
+# bounded appearance bank of the long-prefix workloads: projection rank, most
+# appearance clients, responsibility batch b (pool 4b)
+LONG_PREFIX = {
+    "longdoc": dict(rank=128, max_clients=4096, batch_b=512),
+    "longsmall": dict(rank=128, max_clients=512, batch_b=64),
+}
+
+
+def rademacher(D: int, rank: int = 128, seed: int = 104729) -> np.ndarray:
+    """The fixed rank x D Rademacher map of the long-prefix appearance bank:
+    entries -1 or +1 with equal probability, fp32 (exact in bf16)."""
+    rng = np.random.default_rng(seed)
+    return (rng.integers(0, 2, size=(rank, D)).astype(np.float32) * 2.0 - 1.0).astype(np.float32)
 
 
 def round_to_bf16(x: np.ndarray) -> np.ndarray:
@@ -226,7 +252,8 @@ class Workload:
             Bm = rng.standard_normal((D, 32), dtype=f32) / f32(np.sqrt(32.0))
             w = rng.standard_normal((N, 32), dtype=f32)
             hidden[:N] = w @ Bm.T
-            iso = rng.choice(N, size=min(200, N), replace=False)
+            # isolated high-innovation rows: 200 per 4096 tokens
+            iso = rng.choice(N, size=min(int(round(200 * N / 4096)), N), replace=False)
             hidden[iso] = rng.standard_normal((iso.size, D), dtype=f32)
         pos = np.empty((3, N + T), dtype=np.int32)
         if self.positions == "mrope":

@@ -938,3 +938,126 @@ def test_multi_image_assignment_uses_each_images_own_grid():
         blk = slice(k * Ng, (k + 1) * Ng)
         np.testing.assert_array_equal(both.pi[blk], single.pi + k * Ng)
         np.testing.assert_allclose(both.kappa_best[blk], single.kappa_best, rtol=1e-13)
+
+
+# --------------------------------------------------------------------------
+# Long prefixes: the bounded appearance bank (appendix "Appearance and
+# spatial clients", last paragraph; Table "Shared GMC configuration",
+# long-prefix row)
+# --------------------------------------------------------------------------
+def _orthogonal_pm1(n: int, seed: int) -> np.ndarray:
+    """A +-1 matrix with R R^T = R^T R = n I that is not symmetric: a
+    Sylvester-Hadamard matrix with permuted, sign-flipped columns."""
+    from scipy.linalg import hadamard
+    r = rng(seed)
+    return (hadamard(n)[:, r.permutation(n)] * r.choice([-1.0, 1.0], size=n)[None, :]).astype(float)
+
+
+def test_bounded_client_tokens_are_uniformly_spaced():
+    np.testing.assert_array_equal(O.bounded_client_tokens(1296, 4096), np.arange(1296))
+    for N, M in [(15876, 4096), (1600, 512), (4097, 4096), (10, 3)]:
+        c = O.bounded_client_tokens(N, M)
+        assert c.size == M and c[0] == 0 and c[-1] < N
+        gaps = np.diff(c)
+        assert set(gaps.tolist()) <= {N // M, -(-N // M)}
+        assert len(set(c.tolist())) == M
+
+
+def test_projected_cosines_equal_exact_under_an_orthogonal_map():
+    """R R^T = n I preserves inner products up to the factor n, which the
+    normalisation removes: projected cosines are the exact cosines."""
+    D = 64
+    R = _orthogonal_pm1(D, 3)
+    assert not np.array_equal(R, R.T)
+    h = rng(4).standard_normal((30, D)) * rng(5).uniform(0.1, 10, size=(30, 1))
+    xt = O.projected_states(h, R, P)
+    np.testing.assert_allclose(xt @ xt.T, O.cosine_matrix(h, P), atol=1e-13)
+    np.testing.assert_allclose(np.linalg.norm(xt, axis=1), 1.0, rtol=1e-14)
+
+
+def test_projected_states_ignore_the_maps_null_space_and_scale():
+    r, D = 8, 40
+    R = rng(6).choice([-1.0, 1.0], size=(r, D))
+    h = rng(7).standard_normal((12, D))
+    # a component in the null space of R (orthogonal to every row of R)
+    q, _ = np.linalg.qr(R.T)                       # [D, r]: the row space of R
+    v = rng(8).standard_normal((12, D))
+    v -= (v @ q) @ q.T
+    np.testing.assert_allclose(O.projected_states(h + 5 * v, R, P), O.projected_states(h, R, P),
+                               atol=1e-12)
+    np.testing.assert_allclose(O.projected_states(h, R / math.sqrt(r), P),
+                               O.projected_states(h, R, P), atol=1e-14)
+
+
+def test_random_rademacher_cosines_obey_a_johnson_lindenstrauss_bound():
+    """Rank 128 keeps cosines of random states within a few 1/sqrt(128)."""
+    D, r = 512, 128
+    R = rng(9).choice([-1.0, 1.0], size=(r, D))
+    h = rng(10).standard_normal((40, D))
+    h[20:] = h[:20] + 0.5 * rng(11).standard_normal((20, D))  # correlated pairs too
+    err = np.abs(O.projected_states(h, R, P) @ O.projected_states(h, R, P).T - O.cosine_matrix(h, P))
+    assert err.max() < 0.45 and err.mean() < 0.12
+
+
+def test_bounded_rows_are_the_exact_rows_of_their_client_tokens():
+    """Under an orthogonal map every bounded appearance row is the exact
+    bank's row of its client token, for one image and per image."""
+    D, N = 32, 60
+    R = _orthogonal_pm1(D, 12)
+    h = rng(13).standard_normal((N, D))
+    for n_img in (1, 2):
+        exact = O.appearance_clients(O.cosine_matrix(h, P), P, n_img)
+        c = O.bounded_client_tokens(N, 17)
+        bounded = O.bounded_appearance_clients(O.projected_states(h, R, P), c, P, n_img)
+        assert bounded.shape == (17, N)
+        np.testing.assert_allclose(bounded, exact[c], rtol=1e-11, atol=1e-300)
+
+
+def test_bounded_bank_rows_carry_beta_v_over_m_v():
+    H, T, N, MV = 2, 3, 20, 7
+    PG = rng(14).uniform(size=(H, T, N))
+    PG /= PG.sum(axis=2, keepdims=True)
+    PV = rng(15).uniform(size=(MV, N))
+    PV /= PV.sum(axis=1, keepdims=True)
+    PS = O.spatial_clients(4, 5, P)
+    cm = O.client_matrix(PG, np.ones((H, T), bool), np.full(H, 0.5), np.full(T, 1 / 3), PV, PS, P)
+    assert cm.C.shape == (H * T + MV + PS.shape[0], N)
+    rows = cm.C[cm.banks["appearance"]].sum(axis=1)
+    np.testing.assert_allclose(rows, P["beta_V"] / MV, rtol=1e-14)
+    assert cm.C[cm.banks["spatial"]].sum() == pytest.approx(P["beta_S"], rel=1e-13)
+
+
+def test_support_column_cosines_give_the_full_matrix_assignment():
+    gh, gw = 5, 6
+    h = rng(16).standard_normal((gh * gw, 7))
+    S = np.array([1, 4, 11, 17, 22, 29])
+    full = O.assign_population(O.cosine_matrix(h, P), S, gh, gw, P)
+    cols = O.support_cosines(h, S, P)
+    np.testing.assert_allclose(cols, O.cosine_matrix(h, P)[:, S], atol=1e-15)
+    part = O.assign_population(cols, S, gh, gw, P, support_cols=True)
+    np.testing.assert_array_equal(part.pi, full.pi)
+    np.testing.assert_allclose(part.delta, full.delta, atol=1e-15)
+    assert part.s_x == full.s_x
+
+
+def test_long_prefix_step_equals_the_exact_step_under_an_orthogonal_map():
+    """With an orthogonal +-1 map of rank D and every token a client, the
+    bounded-bank step is the exact-bank step (same support, assignment and
+    outputs); with fewer clients it keeps its invariants."""
+    from paper_2608_02134_gb300 import workloads
+    wl = workloads.make("tiny")
+    im = wl.image(0)
+    f = lambda a: np.asarray(a, dtype=np.float64)  # noqa: E731
+    args = (f(im.hidden), f(im.keys), f(im.values), f(im.queries), im.pos, f(wl.probe()),
+            wl.gh, wl.gw, wl.K)
+    R = _orthogonal_pm1(wl.D, 17)
+    exact = O.compress(*args)
+    bounded = O.compress(*args, long_prefix=dict(R=R, max_clients=wl.N))
+    np.testing.assert_array_equal(bounded.support, exact.support)
+    np.testing.assert_array_equal(bounded.assignment.pi, exact.assignment.pi)
+    np.testing.assert_allclose(bounded.out_hidden, exact.out_hidden, rtol=1e-12, atol=1e-12)
+    few = O.compress(*args, long_prefix=dict(R=R, max_clients=16))
+    assert few.clients.banks["appearance"].stop - few.clients.banks["appearance"].start == 16
+    assert few.support.size == wl.K and np.all(np.diff(few.support) > 0)
+    assert few.transport.mass.sum() == pytest.approx(few.m.sum(), rel=1e-12)
+    assert np.all(np.isin(few.assignment.pi, few.support))
