@@ -76,6 +76,9 @@ typedef struct CUstream_st* gmc_stream_t; /* identical to cudaStream_t */
 #define GMC_MAX_HEADS 64          /* H */
 #define GMC_MAX_VIEWS 4           /* message views: the current one and up to 3 historical ones */
 #define GMC_MAX_PREFIX_LAYERS 64  /* dense prefix layers gathered by gmc_compress_ex */
+#define GMC_MAX_N_LONG 16384      /* visual tokens per image on the long-prefix path */
+#define GMC_MAX_POOL_WIDE 4096    /* pool_mult * batch_b on the long-prefix path and gmc_select */
+#define GMC_MAX_RANK 256          /* rows of the long-prefix Rademacher map */
 
 /*
  * Method constants.  gmc_default_params() fills the values of the paper's
@@ -238,6 +241,62 @@ int gmc_compress_ex(const gmc_problem* prob, const gmc_params* params, const gmc
                     void* trace, gmc_stream_t stream);
 
 /*
+ * Long prefixes: the bounded appearance bank (appendix "Appearance and spatial
+ * clients", last paragraph; the cost notes after Algorithm 1; Table "Shared
+ * GMC configuration", long-prefix row: rank 128, Rademacher seed 104729,
+ * M_V <= 4096, b = 512).  The appearance states are the boundary states under a
+ * fixed rank-r map R with entries +-1, normalised after the map:
+ * x~_i = R h_i / max(||R h_i||, norm_eps).  The appearance clients are the
+ * M_V = min(N, max_clients) uniformly spaced tokens c(m) = floor(m N / M_V);
+ * row m is softmax_i(x~_{c(m)} . x~_i / tau_v), beta_V / M_V each.  The
+ * assignment uses the cosines of the unprojected states against the support
+ * only (an N x K product), and every solver round runs on the whole GPU.
+ */
+typedef struct gmc_long_prefix {
+  int rank;                /* r, a multiple of 8, 8 .. GMC_MAX_RANK (128 in the paper) */
+  int max_clients;         /* M_V cap, >= 1 (4096 in the paper) */
+  const void* rademacher;  /* DEVICE bf16 [r][D], entries -1 or +1 (exact in bf16); 16-byte
+                              aligned; read only */
+} gmc_long_prefix;
+
+/* Workspace of gmc_compress_long with n_views historical views (0 on invalid
+ * arguments).  Unlike gmc_workspace_size it depends on params (the pool size). */
+size_t gmc_workspace_size_long(const gmc_problem* prob, const gmc_params* params,
+                               const gmc_long_prefix* lp, int n_views, int N, int T, int H, int d,
+                               int D, int K);
+
+/*
+ * gmc_compress_long -- gmc_compress_ex with the bounded appearance bank of long
+ * prefixes (lp must not be NULL; views and prefix may be NULL).  Arguments,
+ * layouts, outputs and the trace are those of gmc_compress_ex; the trace's
+ * appearance bank values F_S[1] / F_V[1] are the bounded bank's.  params may
+ * set pool_mult * batch_b up to GMC_MAX_POOL_WIDE (the paper's b = 512 gives a
+ * pool of 2048).
+ * Limits: bf16 states, one image per prompt (images 0 or 1), 128 <= N <=
+ * GMC_MAX_N_LONG, and the limits of gmc_compress otherwise; GMC_ERR_UNSUPPORTED
+ * beyond them, GMC_ERR_ARG for a NULL, misaligned or out-of-range lp.
+ */
+int gmc_compress_long(const gmc_problem* prob, const gmc_params* params,
+                      const gmc_long_prefix* lp, const gmc_views* views,
+                      const gmc_prefix_kv* prefix, const void* hidden, const void* keys,
+                      const void* queries, const int32_t* pos_ids, const float* vo_probe, int N,
+                      int T, int H, int d, int D, int K, int32_t* out_idx, void* out_hidden,
+                      void* out_kv, int32_t* out_pos, void* workspace, size_t ws_bytes,
+                      void* trace, gmc_stream_t stream);
+
+/*
+ * gmc_clients_long -- gmc_clients with the bounded appearance bank: out_clients
+ * receives float[B][M][N] with M = (1 + views->n) * H * T + M_V + landmarks^2
+ * (grounded rows, then the M_V appearance rows, then the spatial rows).
+ * Workspace: gmc_workspace_size_long.
+ */
+int gmc_clients_long(const gmc_problem* prob, const gmc_params* params, const gmc_long_prefix* lp,
+                     const gmc_views* views, const void* hidden, const void* keys,
+                     const void* queries, const int32_t* pos_ids, const float* vo_probe, int N,
+                     int T, int H, int d, int D, int K, float* out_clients, void* workspace,
+                     size_t ws_bytes, void* trace, gmc_stream_t stream);
+
+/*
  * Diagnostics trace (optional).  Image b's record starts at byte
  * b * gmc_trace_size(...) / B.  All fields are 4-byte words.
  */
@@ -293,7 +352,9 @@ size_t gmc_trace_size(const gmc_problem* prob, const gmc_params* params, int N, 
  *   trace    NULL or B records laid out as gmc_get_trace_layout with H = 0
  *            (order, round_end, pool and the header's K / rounds / filled are written)
  * 1 <= K <= N <= GMC_MAX_N, M >= 1.  The clients are copied into the workspace
- * first, so `clients` is never written.
+ * first, so `clients` is never written.  A pool pool_mult * batch_b above
+ * GMC_MAX_POOL (up to GMC_MAX_POOL_WIDE) runs every round on the whole GPU, the
+ * solver of gmc_compress_long, and allows N up to GMC_MAX_N_LONG.
  */
 size_t gmc_select_workspace_size(int B, int M, int N, int K, const gmc_params* params);
 int gmc_select(const float* clients, int B, int M, int N, int K, const gmc_params* params,

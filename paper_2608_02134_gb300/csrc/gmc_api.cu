@@ -27,8 +27,8 @@ cudaError_t set_smem_limit(const void* func, size_t bytes) {
   return e;
 }
 
-bool params_ok(const gmc_params& p) {
-  return p.batch_b >= 1 && p.pool_mult >= 1 && p.pool_mult * p.batch_b <= GMC_MAX_POOL &&
+bool params_ok(const gmc_params& p, int max_pool) {
+  return p.batch_b >= 1 && p.pool_mult >= 1 && (long long)p.pool_mult * p.batch_b <= max_pool &&
          p.resp_temp > 0.f && p.resp_eps >= 0.f && p.tau_v > 0.f && p.tau_s > 0.f &&
          p.beta_G >= 0.f && p.beta_V >= 0.f && p.beta_S >= 0.f && p.landmarks >= 1 &&
          p.landmarks <= 64 && p.max_head_clusters >= 1 &&
@@ -39,7 +39,7 @@ bool params_ok(const gmc_params& p) {
 }
 
 // Shape checks shared by gmc_compress / gmc_transport / gmc_transport_noalloc.
-int check_problem(const gmc_problem* prob, int N, int T, int d, int D) {
+int check_problem(const gmc_problem* prob, int N, int T, int d, int D, int max_n) {
   if (!prob) return GMC_ERR_ARG;
   const int I = prob->images < 1 ? 1 : prob->images;  // images per prompt
   if (prob->B < 1 || prob->grid_h < 1 || prob->grid_w < 1 || N < 1 ||
@@ -47,7 +47,7 @@ int check_problem(const gmc_problem* prob, int N, int T, int d, int D) {
       prob->Hkv < 1)
     return GMC_ERR_ARG;
   if (prob->dtype != GMC_F32 && prob->dtype != GMC_BF16) return GMC_ERR_ARG;
-  if (N > GMC_MAX_N || D > 8192 || d > 1024) return GMC_ERR_UNSUPPORTED;
+  if (N > max_n || D > 8192 || d > 1024) return GMC_ERR_UNSUPPORTED;
   if (prob->dtype == GMC_BF16 && (d % 8 != 0 || D % 8 != 0)) return GMC_ERR_UNSUPPORTED;
   if (prob->dtype == GMC_F32 && (d % 4 != 0 || D % 8 != 0)) return GMC_ERR_UNSUPPORTED;
   return GMC_OK;
@@ -69,6 +69,19 @@ struct Carver {
   }
 };
 
+// The long-prefix path: bf16 states, one image per prompt, at least one full
+// 128-row tile of visual tokens, a rank that keeps the split states' rows
+// 16-byte aligned, a device map.
+int check_long_prefix(const gmc_problem* prob, const gmc_long_prefix* lp) {
+  if (!lp->rademacher || ((uintptr_t)lp->rademacher % 16) != 0 || lp->rank < 8 ||
+      lp->rank % 8 != 0 || lp->max_clients < 1)
+    return GMC_ERR_ARG;
+  if (lp->rank > GMC_MAX_RANK || prob->dtype != GMC_BF16 || (prob->images > 1) ||
+      prob->grid_h * prob->grid_w < 128)
+    return GMC_ERR_UNSUPPORTED;
+  return GMC_OK;
+}
+
 // K = min{N, max{K_r, I}} (Sec. 3.1); K_r < 1 asks for the minimum
 int effective_K(int K, int N, int I = 1) {
   const int k = K < I ? I : K;
@@ -85,10 +98,46 @@ Dims make_dims(const gmc_problem* prob, const gmc_params& p, int N, int T, int H
   dm.K = K; dm.gh = prob->grid_h; dm.gw = prob->grid_w; dm.L = p.landmarks;
   dm.V = V;
   dm.I = images_of(prob);
-  dm.M = V * H * T + N + dm.I * p.landmarks * p.landmarks;
+  dm.MV = N;
+  dm.rank = 0;
+  dm.M = V * H * T + dm.MV + dm.I * p.landmarks * p.landmarks;
   dm.dtype = prob->dtype;
   dm.toff = prob->text_offsets;
   return dm;
+}
+
+// Long prefixes: the bounded appearance bank has min(N, max_clients) rows.
+Dims long_dims(Dims dm, const gmc_params& p, const gmc_long_prefix& lp) {
+  dm.MV = lp.max_clients < dm.N ? lp.max_clients : dm.N;
+  dm.rank = lp.rank;
+  dm.M = dm.V * dm.H * dm.T + dm.MV + dm.I * p.landmarks * p.landmarks;
+  return dm;
+}
+
+// Scratch of the long-prefix path and its wide solver (carved after the rest).
+struct LongScratch {
+  float* Y;             // [B][N][r]   projected states R h_i
+  __nv_bfloat16* Xa;    // [B][N][3r]  [hi | hi | lo] of the unit projected states
+  __nv_bfloat16* Xb;    // [B][N][3r]  [hi | lo | hi]
+  __nv_bfloat16* XaC;   // [B][MV][3r] Xa at the appearance clients
+  float* app;           // [B][MV][N]  projected cosines of the appearance clients
+  __nv_bfloat16* Hs;    // [B][K][D]   selected visual rows
+  float* rnS;           // [B][K]      their reciprocal norms
+  float* cs;            // [B][N][K]   support cosines
+  WideState w;
+};
+
+void carve_wide(Carver& c, size_t B, size_t N, size_t M, size_t P, WideState* w) {
+  w->pool = c.take<int32_t>(B * P);
+  w->sc = c.take<long long>(B * P);
+  w->batch = c.take<int32_t>(B * P);
+  w->stamp = c.take<int32_t>(B * N);
+  w->info = c.take<int32_t>(B * INFO_W);
+  w->u1 = c.take<long long>(B * N);
+  w->u2 = c.take<long long>(B * N);
+  w->bcov = c.take<float>(B * M);
+  w->cnt = c.take<int32_t>(B * M);
+  w->fv = c.take<long long>(B * 4);
 }
 
 R0State carve_round0(Carver& c, size_t B, size_t N, size_t M);
@@ -100,7 +149,8 @@ size_t status_words(const Dims& dm) {
 }
 
 // Workspace of gmc_compress.  base == nullptr only measures.
-size_t carve_compress(const Dims& dm, Scratch* s, char* base, R0State* r0s = nullptr) {
+size_t carve_compress(const Dims& dm, Scratch* s, char* base, R0State* r0s = nullptr,
+                      LongScratch* ls = nullptr, int pool = 0) {
   Carver c{base};
   Scratch t{};
   const size_t B = dm.B, N = dm.N, H = dm.H, T = dm.T, M = dm.M, K = dm.K;
@@ -147,7 +197,7 @@ size_t carve_compress(const Dims& dm, Scratch* s, char* base, R0State* r0s = nul
   t.ebar = c.take<float>(B * N);
   t.rn = c.take<float>(B * N);
   t.rmsh = c.take<float>(B * N);
-  t.cos = c.take<float>(B * N * N);
+  t.cos = dm.rank ? nullptr : c.take<float>(B * N * N);
   t.C = c.take<float>(B * M * N);
   t.scol = c.take<uint16_t>(B * M * N);
   t.u0 = c.take<long long>(B * N);
@@ -163,6 +213,21 @@ size_t carve_compress(const Dims& dm, Scratch* s, char* base, R0State* r0s = nul
   t.fexp = nullptr;
   t.Qp = c.take<__nv_bfloat16>(V * t.vQp);
   if (s) *s = t;
+  if (dm.rank) {  // long prefixes: bounded bank, support cosines, wide solver
+    LongScratch l{};
+    const size_t r = dm.rank, MV = dm.MV;
+    l.Y = c.take<float>(B * N * r);
+    l.Xa = c.take<__nv_bfloat16>(B * N * 3 * r);
+    l.Xb = c.take<__nv_bfloat16>(B * N * 3 * r);
+    l.XaC = c.take<__nv_bfloat16>(B * MV * 3 * r);
+    l.app = c.take<float>(B * MV * N);
+    l.Hs = c.take<__nv_bfloat16>(B * K * dm.D);
+    l.rnS = c.take<float>(B * K);
+    l.cs = c.take<float>(B * N * K);
+    carve_wide(c, B, N, M, (size_t)pool, &l.w);
+    if (ls && base) *ls = l;
+    return c.off;
+  }
   R0State r0 = carve_round0(c, B, N, M);
   if (r0s && base) *r0s = r0;
   return c.off;
@@ -375,7 +440,7 @@ int gmc_get_trace_layout(const gmc_problem* prob, const gmc_params* params, int 
   if (!prob || !out || T < 1) return GMC_ERR_ARG;
   gmc_params p;
   if (params) p = *params; else gmc_default_params(&p);
-  if (!params_ok(p)) return GMC_ERR_ARG;
+  if (!params_ok(p, GMC_MAX_POOL_WIDE)) return GMC_ERR_ARG;
   return fill_trace_layout(prob->B, p, N, H, effective_K(K, N, images_of(prob)), out,
                            images_of(prob));
 }
@@ -396,14 +461,18 @@ static int compress_impl(const gmc_problem* prob, const gmc_params* params,
                          int N, int T, int H, int d, int D, int K, int32_t* out_idx,
                          void* out_hidden, void* out_kv, int32_t* out_pos, void* workspace,
                          size_t ws_bytes, void* trace, gmc_stream_t stream_,
-                         float* out_clients = nullptr) {
-  int rc = check_problem(prob, N, T, d, D);
+                         float* out_clients = nullptr, const gmc_long_prefix* lp = nullptr) {
+  int rc = check_problem(prob, N, T, d, D, lp ? GMC_MAX_N_LONG : GMC_MAX_N);
   if (rc != GMC_OK) return rc;
   if (H < 1 || H % prob->Hkv != 0) return GMC_ERR_ARG;
   if (H > GMC_MAX_HEADS || !heads_supported(H)) return GMC_ERR_UNSUPPORTED;
   gmc_params p;
   if (params) p = *params; else gmc_default_params(&p);
-  if (!params_ok(p)) return GMC_ERR_ARG;
+  if (!params_ok(p, lp ? GMC_MAX_POOL_WIDE : GMC_MAX_POOL)) return GMC_ERR_ARG;
+  if (lp) {
+    rc = check_long_prefix(prob, lp);
+    if (rc != GMC_OK) return rc;
+  }
   if (!hidden || !keys || !queries || !pos_ids || !vo_probe || !workspace ||
       (!out_clients && (!out_idx || !out_hidden || !out_kv || !out_pos)))
     return GMC_ERR_ARG;
@@ -443,10 +512,13 @@ static int compress_impl(const gmc_problem* prob, const gmc_params* params,
     }
   }
   const int Ke = effective_K(K, N, images_of(prob));
-  const Dims dm = make_dims(prob, p, N, T, H, d, D, Ke, V);
+  Dims dm = make_dims(prob, p, N, T, H, d, D, Ke, V);
+  if (lp) dm = long_dims(dm, p, *lp);
   Scratch s;
   R0State r0;
-  const size_t need = carve_compress(dm, &s, (char*)workspace, &r0);
+  LongScratch ls{};
+  const size_t need =
+      carve_compress(dm, &s, (char*)workspace, &r0, &ls, p.pool_mult * p.batch_b);
   if (ws_bytes < need) return GMC_ERR_WORKSPACE;
   cudaStream_t st = (cudaStream_t)stream_;
   gmc_trace_layout L;
@@ -506,12 +578,40 @@ static int compress_impl(const gmc_problem* prob, const gmc_params* params,
   };
   const int msg_k = (message_tc_supported(dm) ? 3 : 1) * V;
   GMC_TRY(g_prof.begin(st));  // k_probe zeroes the column sums u0 of the client build
+  // the appearance branch: cosine Gram, or on long prefixes the projection,
+  // the split unit states and the bounded bank's cosines
+  auto project = [&](cudaStream_t q) -> cudaError_t {
+    GemmArgs g{};
+    g.B = dm.B; g.M = N; g.Nn = dm.rank; g.Kd = D;
+    g.a_img = N; g.b_img = 0; g.a_text = 1; g.b_text = 0;
+    g.toff = dm.toff; g.Tmax = T;
+    g.C = ls.Y; g.c_img = (long long)N * dm.rank; g.ldc = dm.rank;
+    g.status = s.status;
+    cudaError_t e = launch_gemm_tc(g, hidden, (long long)dm.B * (N + T), D, lp->rademacher,
+                                   dm.rank, D, q);
+    if (e != cudaSuccess) return e;
+    return launch_lp_norm(dm, p.norm_eps, ls.Y, ls.Xa, ls.Xb, ls.XaC, s.status, q);
+  };
+  auto app_cos = [&](cudaStream_t q) -> cudaError_t {
+    GemmArgs g{};
+    g.B = dm.B; g.M = dm.MV; g.Nn = N; g.Kd = 3 * dm.rank;
+    g.a_img = dm.MV; g.b_img = N; g.toff = dm.toff; g.Tmax = T;
+    g.C = ls.app; g.c_img = (long long)dm.MV * N; g.ldc = N;
+    g.status = s.status;
+    return launch_gemm_tc(g, ls.XaC, (long long)dm.B * dm.MV, 3 * dm.rank, ls.Xb,
+                          (long long)dm.B * N, 3 * dm.rank, q);
+  };
   if (g_prof.on) {  // stage timing: every stage in turn on the caller's stream
     GMC_STAGE("rownorm", 1, launch_rownorm(dm, hidden, p.norm_eps, s, st));
     GMC_STAGE("probe", V, probes());
     GMC_STAGE("message", msg_k, messages());
     GMC_STAGE("heads", 2 * V, heads());
-    GMC_STAGE("gram", 1, launch_gram(dm, hidden, s, st));
+    if (lp) {
+      GMC_STAGE("project", 2, project(st));
+      GMC_STAGE("app_cos", 1, app_cos(st));
+    } else {
+      GMC_STAGE("gram", 1, launch_gram(dm, hidden, s, st));
+    }
   } else {
     // row norms and the cosine Gram run beside probe -> message -> heads
     SideStream* sd = nullptr;
@@ -519,7 +619,12 @@ static int compress_impl(const gmc_problem* prob, const gmc_params* params,
     GMC_TRY(cudaEventRecord(sd->fork, st));
     GMC_TRY(cudaStreamWaitEvent(sd->st, sd->fork, 0));
     GMC_STAGE("rownorm", 1, launch_rownorm(dm, hidden, p.norm_eps, s, sd->st));
-    GMC_STAGE("gram", 1, launch_gram(dm, hidden, s, sd->st));
+    if (lp) {
+      GMC_STAGE("project", 2, project(sd->st));
+      GMC_STAGE("app_cos", 1, app_cos(sd->st));
+    } else {
+      GMC_STAGE("gram", 1, launch_gram(dm, hidden, s, sd->st));
+    }
     GMC_TRY(cudaEventRecord(sd->join, sd->st));
     GMC_STAGE("probe", V, probes());
     GMC_STAGE("message", msg_k, messages());
@@ -528,13 +633,47 @@ static int compress_impl(const gmc_problem* prob, const gmc_params* params,
   }
   // every view's grounded rows count as head rows of the client layout
   const int HV = H * V;
-  GMC_STAGE("clients", 1, launch_build_clients(dm, p, fx, s, vr, st));
+  GMC_STAGE("clients", 1, launch_build_clients(dm, p, fx, s, vr, lp ? ls.app : s.cos, st));
   if (out_clients) {  // staged call: the client matrix, before selection compacts it in place
     GMC_TRY(cudaMemcpyAsync(out_clients, s.C, sizeof(float) * dm.B * (size_t)dm.M * N,
                             cudaMemcpyDeviceToDevice, st));
     return GMC_OK;
   }
   const int LS = dm.I * p.landmarks * p.landmarks;  // spatial rows: a landmark grid per image
+  if (lp) {
+    WideGeom wg{};
+    wg.B = dm.B; wg.N = N; wg.K = Ke; wg.Mstride = dm.M;
+    wg.HV = HV; wg.Tmax = T; wg.MV = dm.MV; wg.L2 = LS;
+    wg.toff = dm.toff; wg.uniform = 0;
+    GMC_STAGE("select", 4 * wide_rounds(Ke, p) + 1,
+              launch_wide_select(ls.w, wg, p, fx, nullptr, s.C, s.scol, s.u0, s.order, s.support,
+                                 s.slot, nullptr, s.status, tv, st));
+    if (tv.base) {
+      GMC_TRY(launch_certificate(dm.B, N, Ke, tv, st));
+      g_launches += 1;
+    }
+    // the N x K support cosines of the assignment (Eq. (cond-assignment))
+    auto support_cos = [&]() -> cudaError_t {
+      cudaError_t e = launch_gather_support(dm, hidden, s.support, s.rn, ls.Hs, ls.rnS, s.status, st);
+      if (e != cudaSuccess) return e;
+      GemmArgs g{};
+      g.B = dm.B; g.M = N; g.Nn = Ke; g.Kd = D;
+      g.a_img = N; g.b_img = Ke; g.a_text = 1; g.b_text = 0;
+      g.toff = dm.toff; g.Tmax = T;
+      g.rscale = s.rn; g.cscale = ls.rnS;
+      g.C = ls.cs; g.c_img = (long long)N * Ke; g.ldc = Ke;
+      g.status = s.status;
+      return launch_gemm_tc(g, hidden, (long long)dm.B * (N + T), D, ls.Hs, (long long)dm.B * Ke,
+                            D, st);
+    };
+    GMC_STAGE("support_cos", 2, support_cos());
+    GMC_STAGE("assign", 2, launch_assign(dm, p, s, tv, st, ls.cs));
+    GMC_STAGE("transport", 1,
+              launch_transport(dm, p, hidden, keys, pos_ids, s.support, s.pi, s.mass, s.rmsh,
+                               s.mbits, out_idx, out_hidden, out_kv, out_pos, s.status, st, &pf));
+    g_prof.valid = g_prof.on;
+    return GMC_OK;
+  }
   GMC_STAGE("rounds_gpu", 3 + 3 * sparse_gpu_rounds(N),
             launch_round0(r0, dm.B, N, Ke, dm.M, dm.toff, HV, T, LS, p, fx, nullptr, s.C, s.scol,
                           s.u0, s.order, s.status, tv, st, dm.I));
@@ -581,6 +720,45 @@ int gmc_compress_ex(const gmc_problem* prob, const gmc_params* params, const gmc
                        trace, stream_);
 }
 
+size_t gmc_workspace_size_long(const gmc_problem* prob, const gmc_params* params,
+                               const gmc_long_prefix* lp, int n_views, int N, int T, int H, int d,
+                               int D, int K) {
+  if (!lp || check_problem(prob, N, T, d, D, GMC_MAX_N_LONG) != GMC_OK ||
+      check_long_prefix(prob, lp) != GMC_OK || H < 1 || H > GMC_MAX_HEADS ||
+      H % prob->Hkv != 0 || !heads_supported(H) || n_views < 0 || n_views > GMC_MAX_VIEWS - 1)
+    return 0;
+  gmc_params p;
+  if (params) p = *params; else gmc_default_params(&p);
+  if (!params_ok(p, GMC_MAX_POOL_WIDE)) return 0;
+  Dims dm = make_dims(prob, p, N, T, H, d, D, effective_K(K, N, images_of(prob)), 1 + n_views);
+  dm = long_dims(dm, p, *lp);
+  return carve_compress(dm, nullptr, nullptr, nullptr, nullptr, p.pool_mult * p.batch_b);
+}
+
+int gmc_compress_long(const gmc_problem* prob, const gmc_params* params,
+                      const gmc_long_prefix* lp, const gmc_views* views,
+                      const gmc_prefix_kv* prefix, const void* hidden, const void* keys,
+                      const void* queries, const int32_t* pos_ids, const float* vo_probe, int N,
+                      int T, int H, int d, int D, int K, int32_t* out_idx, void* out_hidden,
+                      void* out_kv, int32_t* out_pos, void* workspace, size_t ws_bytes,
+                      void* trace, gmc_stream_t stream_) {
+  if (!lp) return GMC_ERR_ARG;
+  return compress_impl(prob, params, views, prefix, hidden, keys, queries, pos_ids, vo_probe, N,
+                       T, H, d, D, K, out_idx, out_hidden, out_kv, out_pos, workspace, ws_bytes,
+                       trace, stream_, nullptr, lp);
+}
+
+int gmc_clients_long(const gmc_problem* prob, const gmc_params* params, const gmc_long_prefix* lp,
+                     const gmc_views* views, const void* hidden, const void* keys,
+                     const void* queries, const int32_t* pos_ids, const float* vo_probe, int N,
+                     int T, int H, int d, int D, int K, float* out_clients, void* workspace,
+                     size_t ws_bytes, void* trace, gmc_stream_t stream_) {
+  if (!out_clients || !lp) return GMC_ERR_ARG;
+  return compress_impl(prob, params, views, nullptr, hidden, keys, queries, pos_ids, vo_probe, N,
+                       T, H, d, D, K, nullptr, nullptr, nullptr, nullptr, workspace, ws_bytes,
+                       trace, stream_, out_clients, lp);
+}
+
 int gmc_clients(const gmc_problem* prob, const gmc_params* params, const gmc_views* views,
                 const void* hidden, const void* keys, const void* queries, const int32_t* pos_ids,
                 const float* vo_probe, int N, int T, int H, int d, int D, int K,
@@ -596,7 +774,7 @@ int gmc_clients(const gmc_problem* prob, const gmc_params* params, const gmc_vie
 // gmc_select
 // ---------------------------------------------------------------------------
 static size_t carve_select(int B, int M, int N, int K, Scratch* s, char* base,
-                           R0State* r0s = nullptr) {
+                           R0State* r0s = nullptr, int wide_pool = 0, WideState* ws = nullptr) {
   Carver c{base};
   Scratch t{};
   t.nSel = 64;
@@ -610,15 +788,30 @@ static size_t carve_select(int B, int M, int N, int K, Scratch* s, char* base,
   t.selpart = c.take<double>((size_t)B * t.nSel);
   t.fexp = c.take<int32_t>((size_t)B);
   if (s) *s = t;
+  if (wide_pool > 0) {  // pools above GMC_MAX_POOL: the wide solver's state
+    WideState w{};
+    carve_wide(c, (size_t)B, (size_t)N, (size_t)M, (size_t)wide_pool, &w);
+    if (ws && base) *ws = w;
+    return c.off;
+  }
   R0State r0 = carve_round0(c, (size_t)B, (size_t)N, (size_t)M);
   if (r0s && base) *r0s = r0;
   return c.off;
 }
 
+// gmc_select runs the wide solver when the pool exceeds GMC_MAX_POOL
+static int select_wide_pool(const gmc_params& p) {
+  const int P = p.pool_mult * p.batch_b;
+  return P > GMC_MAX_POOL ? P : 0;
+}
+
 size_t gmc_select_workspace_size(int B, int M, int N, int K, const gmc_params* params) {
-  (void)params;
-  if (B < 1 || M < 1 || N < 1 || N > GMC_MAX_N || K < 1 || K > N) return 0;
-  return carve_select(B, M, N, K, nullptr, nullptr);
+  gmc_params p;
+  if (params) p = *params; else gmc_default_params(&p);
+  if (!params_ok(p, GMC_MAX_POOL_WIDE)) return 0;
+  const int wp = select_wide_pool(p);
+  if (B < 1 || M < 1 || N < 1 || N > (wp ? GMC_MAX_N_LONG : GMC_MAX_N) || K < 1 || K > N) return 0;
+  return carve_select(B, M, N, K, nullptr, nullptr, nullptr, wp);
 }
 
 int gmc_select(const float* clients, int B, int M, int N, int K, const gmc_params* params,
@@ -626,14 +819,16 @@ int gmc_select(const float* clients, int B, int M, int N, int K, const gmc_param
                gmc_stream_t stream_) {
   if (!clients || !out_idx || !workspace || B < 1 || M < 1 || N < 1 || K < 1 || K > N)
     return GMC_ERR_ARG;
-  if (N > GMC_MAX_N) return GMC_ERR_UNSUPPORTED;
   if (!aligned(workspace, ALIGN) || (trace && !aligned(trace, 16))) return GMC_ERR_ARG;
   gmc_params p;
   if (params) p = *params; else gmc_default_params(&p);
-  if (!params_ok(p)) return GMC_ERR_ARG;
+  if (!params_ok(p, GMC_MAX_POOL_WIDE)) return GMC_ERR_ARG;
+  const int wp = select_wide_pool(p);
+  if (N > (wp ? GMC_MAX_N_LONG : GMC_MAX_N)) return GMC_ERR_UNSUPPORTED;
   Scratch s;
   R0State r0;
-  const size_t need = carve_select(B, M, N, K, &s, (char*)workspace, &r0);
+  WideState w{};
+  const size_t need = carve_select(B, M, N, K, &s, (char*)workspace, &r0, wp, &w);
   if (ws_bytes < need) return GMC_ERR_WORKSPACE;
   cudaStream_t st = (cudaStream_t)stream_;
   TraceView tv{};
@@ -648,6 +843,20 @@ int gmc_select(const float* clients, int B, int M, int N, int K, const gmc_param
                           cudaMemcpyDeviceToDevice, st));
   GMC_TRY(cudaMemsetAsync(s.u0, 0, sizeof(long long) * B * (size_t)N, st));
   GMC_TRY(launch_select_prep(s.C, B, M, N, s, st));
+  if (wp) {
+    WideGeom wg{};
+    wg.B = B; wg.N = N; wg.K = K; wg.Mstride = M;
+    wg.HV = 0; wg.Tmax = 1; wg.MV = 0; wg.L2 = 0;
+    wg.toff = nullptr; wg.uniform = 1;
+    GMC_TRY(launch_wide_select(w, wg, p, 0, s.fexp, s.C, s.scol, s.u0, s.order, s.support, s.slot,
+                               out_idx, s.status, tv, st));
+    g_launches += 3 + 4 * wide_rounds(K, p) + 1;
+    if (tv.base) {
+      GMC_TRY(launch_certificate(B, N, K, tv, st));
+      g_launches += 1;
+    }
+    return GMC_OK;
+  }
   GMC_TRY(launch_round0(r0, B, N, K, M, nullptr, 0, 1, 0, p, 0, s.fexp, s.C, s.scol, s.u0,
                         s.order, s.status, tv, st));
   GMC_TRY(launch_select(r0, B, N, K, M, nullptr, 0, 1, 0, p, 0, s.fexp, s.C, s.scol, s.u0,

@@ -13,6 +13,9 @@
 // also sets bit i of its carrier's membership bitmap (atomicOr: the bitmap
 // does not depend on the order of the writes), which the transport reads
 // instead of scanning the whole assignment.
+// The cosines come from the N x N matrix at the support's columns, or (cs
+// mode, long prefixes) from the N x K support cosines, column k holding the
+// k-th selected token: the same values, read as contiguous rows.
 #include "common.cuh"
 #include "kernels.cuh"
 
@@ -24,7 +27,8 @@ namespace gmc {
 // lanes over the heads, and per-block sums of e (the mean normalises ebar in pass 2).
 // The last block of an image to finish (ticket) adds the block partials in a
 // fixed order and stores Delta_bar, s_x and the mean energy for pass 2.
-__global__ void k_assign_gap(const float* __restrict__ cos, const int32_t* __restrict__ support,
+__global__ void k_assign_gap(const float* __restrict__ cos, int cs_mode,
+                             const int32_t* __restrict__ support,
                              const int32_t* __restrict__ slot, const int32_t* toff, int B, int N,
                              int K, int Tmax, int H, const float* __restrict__ omega,
                              const float* __restrict__ zn2, const float* __restrict__ sigma,
@@ -59,7 +63,7 @@ __global__ void k_assign_gap(const float* __restrict__ cos, const int32_t* __res
   double dv = 0.0;
   int dc = 0;
   if (i < N && slot[(size_t)b * N + i] < 0) {
-    const float* row = cos + ((size_t)b * N + i) * N;
+    const float* row = cos + ((size_t)b * N + i) * (cs_mode ? K : N);
     const int32_t* S = sS;
     const int Ng = N / I, img = i / Ng;
     float m1 = -INFINITY, m2 = -INFINITY;
@@ -67,7 +71,7 @@ __global__ void k_assign_gap(const float* __restrict__ cos, const int32_t* __res
     for (int k = lane; k < K; k += 32) {
       if (S[k] / Ng != img) continue;
       ++ncomp;
-      const float v = row[S[k]];
+      const float v = row[cs_mode ? k : S[k]];
       if (v > m1) { m2 = m1; m1 = v; } else if (v > m2) { m2 = v; }
     }
     ncomp = warp_sum_int(ncomp);
@@ -128,7 +132,8 @@ __global__ void k_assign_gap(const float* __restrict__ cos, const int32_t* __res
 }
 
 // Pass 2: s_x, the gated spatial assignment, and the population weights.
-__global__ void k_assign_pick(const float* __restrict__ cos, const int32_t* __restrict__ support,
+__global__ void k_assign_pick(const float* __restrict__ cos, int cs_mode,
+                              const int32_t* __restrict__ support,
                               const int32_t* __restrict__ slot, const float* __restrict__ delta,
                               const float* __restrict__ gatev, const float* __restrict__ energy,
                               const int32_t* toff, int B, int N, int K, int Tmax, int gh, int gw,
@@ -160,14 +165,14 @@ __global__ void k_assign_pick(const float* __restrict__ cos, const int32_t* __re
     const float coef = lambda_p * sx * gi;
     const int Ng = N / I, img = i / Ng, il = i - img * Ng;  // coordinates in its own grid
     const float piy = ((il / gw) + 0.5f) / gh, pix = ((il % gw) + 0.5f) / gw;
-    const float* row = cos + ((size_t)b * N + i) * N;
+    const float* row = cos + ((size_t)b * N + i) * (cs_mode ? K : N);
     const int32_t* S = sS;
     float best = -INFINITY;
     int bk = 0x7fffffff;
     for (int k = lane; k < K; k += 32) {
       const int j = S[k];
       if (j / Ng != img) continue;  // a carrier of another image
-      float v = row[j];
+      float v = row[cs_mode ? k : j];
       if (coef > 0.f) {
         const int jl = j - img * Ng;
         const float dy = ((jl / gw) + 0.5f) / gh - piy, dx = ((jl % gw) + 0.5f) / gw - pix;
@@ -207,20 +212,22 @@ __global__ void k_assign_pick(const float* __restrict__ cos, const int32_t* __re
 }
 
 cudaError_t launch_assign(const Dims& dm, const gmc_params& p, Scratch& s, const TraceView& tv,
-                          cudaStream_t st) {
+                          cudaStream_t st, const float* cs) {
+  const float* src = cs ? cs : s.cos;
+  const int cs_mode = cs ? 1 : 0;
   dim3 grid(s.nA, dm.B);
   const size_t smem = sizeof(int) * (size_t)dm.K;
   cudaError_t e0;
   if ((e0 = set_smem_limit((const void*)k_assign_gap, smem)) != cudaSuccess) return e0;
   if ((e0 = set_smem_limit((const void*)k_assign_pick, smem)) != cudaSuccess) return e0;
   launch_k(k_assign_gap, grid, 32 * ASSIGN_WARPS, smem, st, 1,
-      s.cos, s.support, s.slot, dm.toff, dm.B, dm.N, dm.K, dm.T, dm.H, s.omega, s.zn2, s.sigma,
+      src, cs_mode, s.support, s.slot, dm.toff, dm.B, dm.N, dm.K, dm.T, dm.H, s.omega, s.zn2, s.sigma,
       s.W2, s.ebar, s.epart, s.delta, s.dpart, s.nA, p.gate_scale, p.gate_pow, dm.I, s.tick2,
       s.gatev, s.status);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   launch_k(k_assign_pick, grid, 32 * ASSIGN_WARPS, smem, st, 1,
-      s.cos, s.support, s.slot, s.delta, s.gatev, s.ebar, dm.toff, dm.B, dm.N, dm.K, dm.T,
+      src, cs_mode, s.support, s.slot, s.delta, s.gatev, s.ebar, dm.toff, dm.B, dm.N, dm.K, dm.T,
       dm.gh, dm.gw, p.gate_pow, p.ambig_margin, p.assign_spatial_w, p.tau_s,
       p.pop_strength, dm.I, s.pi, s.mass, s.mbits, tv, s.status);
   return cudaGetLastError();

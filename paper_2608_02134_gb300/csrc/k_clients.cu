@@ -6,7 +6,10 @@
 //              (v = 0 the current view with beta_G, then the historical views
 //              sharing beta_hist; zero when the row has no energy: an inactive
 //              client)
-//   appearance m = 0..N-1:       beta_V / N * softmax_i(cos_mi / tau_v)
+//   appearance m = 0..MV-1:      beta_V / MV * softmax_i(app_mi / tau_v), where
+//                                app is the N x N cosine matrix (MV = N, exact
+//                                bank) or the bounded bank's M_V x N projected
+//                                cosines x~_{c(m)} . x~_i (long prefixes)
 //   spatial    l = 0..I*L*L-1:   beta_S / (I L^2) * softmax_i(-||p_i - l_l||^2 / tau_s)
 // with p_i = ((r+.5)/gh, (c+.5)/gw) and landmarks ((a+.5)/L, (b+.5)/L).  A
 // prompt with I > 1 images holds them one after another (Ng = gh * gw tokens
@@ -69,7 +72,7 @@ __device__ __forceinline__ void row_softmax_stats(const float* row, int N, float
 
 __global__ void __launch_bounds__(256, 4) k_build_clients(
     const ViewRows vw, int nRS, const float* __restrict__ omega,
-    const float* __restrict__ cos, const int32_t* toff, int B, int N, int Tmax, int H, int M,
+    const float* __restrict__ app, int MV, const int32_t* toff, int B, int N, int Tmax, int H, int M,
     int gh, int gw, int L, float beta_V, float beta_S, float tau_v, float tau_s,
     float wq, float fx_scale, int check, int I, float* C, long long* u0, uint32_t* status) {
   grid_dep_wait();
@@ -77,7 +80,7 @@ __global__ void __launch_bounds__(256, 4) k_build_clients(
   const int b = blockIdx.y;
   const TextGeom tg = text_geom(toff, b, B, Tmax, status);
   if (tg.T == 0) return;
-  const int Tb = tg.T, MG = vw.n * H * Tb, Mb = MG + N + I * L * L;
+  const int Tb = tg.T, MG = vw.n * H * Tb, Mb = MG + MV + I * L * L;
   const int Ng = N / I;  // tokens of one image
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const int r0 = blockIdx.x * ROWS_PER_BLOCK;
@@ -97,19 +100,19 @@ __global__ void __launch_bounds__(256, 4) k_build_clients(
       inf.z = vw.zn2[v] + ((size_t)b * H + h) * N;
       inf.scale = rsv > 0.f ? vw.beta[v] * omega[(size_t)b * H + h] * nu / rsv : 0.f;
       inf.sg2 = sg * sg;
-    } else if (m < MG + N) {
+    } else if (m < MG + MV) {
       const int a = m - MG;
-      const float* row = cos + ((size_t)b * N + a) * N;
-      inf.lo = (a / Ng) * Ng;  // the row's own image
+      const float* row = app + ((size_t)b * MV + a) * N;
+      inf.lo = (a / Ng) * Ng;  // the row's own image (one image when the bank is bounded)
       inf.hi = inf.lo + Ng;
       float mx, z;
       row_softmax_stats(row + inf.lo, Ng, 1.f / tau_v, lane, mx, z);
       inf.kind = 1;
       inf.x = row;
-      inf.scale = beta_V / ((float)N * z);
+      inf.scale = beta_V / ((float)MV * z);
       inf.shift = mx;
     } else if (m < Mb) {
-      const int lg = m - MG - N;
+      const int lg = m - MG - MV;
       const int l = lg % (L * L);  // landmark of image lg / L^2
       inf.lo = (lg / (L * L)) * Ng;
       inf.hi = inf.lo + Ng;
@@ -185,10 +188,10 @@ __global__ void __launch_bounds__(256, 4) k_build_clients(
 }
 
 cudaError_t launch_build_clients(const Dims& dm, const gmc_params& p, int fx_exp, Scratch& s,
-                                 const ViewRows& views, cudaStream_t st) {
+                                 const ViewRows& views, const float* app, cudaStream_t st) {
   dim3 grid(ceil_div(dm.M, ROWS_PER_BLOCK), dm.B);
   launch_k(k_build_clients, grid, 32 * ROWS_PER_BLOCK, 0, st, 1,
-      views, s.nRS, s.omega, s.cos, dm.toff, dm.B, dm.N, dm.T, dm.H, dm.M, dm.gh,
+      views, s.nRS, s.omega, app, dm.MV, dm.toff, dm.B, dm.N, dm.T, dm.H, dm.M, dm.gh,
       dm.gw, dm.L, p.beta_V, p.beta_S, p.tau_v, p.tau_s, p.terminal_q_weight,
       ldexpf(1.f, fx_exp), p.check_mode, dm.I, s.C, s.u0, s.status);
   return cudaGetLastError();

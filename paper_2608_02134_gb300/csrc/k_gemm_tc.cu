@@ -1,0 +1,230 @@
+// General C = diag(r) (A B^T) diag(c) on the tcgen05 tensor cores (bf16 operands,
+// fp32 accumulation in tensor memory, fp32 output): the dense contractions of
+// the long-prefix path.
+//
+//   * the fixed rank-r Rademacher projection of the boundary states, y_i = R h_i
+//     (A = visual hidden rows, B = R, no scaling);
+//   * the bounded appearance bank's cosines x~_{c(m)} . x~_i over the projected
+//     unit states (A, B = the states split into bf16 hi/lo terms, laid out so
+//     one product over 3r columns sums hi.hi + hi.lo + lo.hi);
+//   * the N x K support cosines of the assignment, cos(h_i, h_{S_k}) (A =
+//     visual hidden rows, B = the selected rows gathered, scaled by the
+//     reciprocal norms of both).
+// (Appendix "Appearance and spatial clients", last paragraph; the cost notes
+// after Algorithm 1: the bounded bank and the chunked N x K assignment product.)
+//
+// One CTA computes one 128 x BN output tile (BN = 128 or 256, one TMEM column
+// per output column).  Warp 0 / lane 0 streams 64-wide K slices of the A and B
+// row blocks with TMA (128-byte swizzle) through a 4-stage mbarrier ring; warp
+// 1 / lane 0 issues tcgen05.mma (M = 128, N = BN, K = 16).  Then all 8 warps
+// drain TMEM: warp w reads lane quarter w % 4 and half w / 4 of the columns in
+// 32-column chunks, applies the row and column scales and stores each chunk
+// through a padded 32 x 32 shared-memory transpose, so every store
+// instruction writes one 128-byte row segment.  Ragged edges: TMA fills K
+// columns past the operands' extents with zeros.  The last row block of an
+// operand with at least one full tile of rows is shifted inward (start M - 128,
+// likewise Nn - BN) so every box lies inside the image's own rows -- the
+// hidden states' visual rows are followed by text rows whose count only the
+// device knows -- and stores only the rows and columns the previous tile does
+// not own; a smaller operand reads zeros past its declared rows.  Every mbarrier wait is bounded (about two seconds);
+// on timeout the kernel records GMC_STATUS_TIMEOUT, drains its copies and
+// frees its tensor memory.
+#include "common.cuh"
+#include "kernels.cuh"
+#include "tc.cuh"
+
+namespace gmc {
+
+namespace {
+constexpr int GM = 128, GK = 64, GSTAGES = 4;
+constexpr int G_THREADS = 256;
+constexpr int GA_BYTES = GM * GK * 2;  // 16 KiB per stage
+constexpr long long G_WAIT = 4000000000LL;
+
+struct GemmCtl {
+  uint64_t full[GSTAGES];
+  uint64_t empty[GSTAGES];
+  uint64_t done;
+  uint32_t tmem;
+  volatile int abort;
+};
+
+template <int BN> constexpr size_t gemm_smem() {
+  return 1024 + (size_t)GSTAGES * (GA_BYTES + BN * GK * 2) + sizeof(GemmCtl) + sizeof(float) * (GM + BN);
+}
+}  // namespace
+
+template <int BN>
+__global__ void __launch_bounds__(G_THREADS, 1)
+    k_gemm_tc(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap bmap,
+              GemmArgs g) {
+  grid_dep_wait();
+  constexpr int B_BYTES = BN * GK * 2;
+  extern __shared__ uint8_t sm_raw[];
+  uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* tilesA = base;
+  uint8_t* tilesB = base + GSTAGES * GA_BYTES;
+  GemmCtl* ctl = reinterpret_cast<GemmCtl*>(base + GSTAGES * (GA_BYTES + B_BYTES));
+  float* rs = reinterpret_cast<float*>(ctl + 1);  // [GM] row scales of the tile
+  float* cs = rs + GM;                            // [BN] column scales
+
+  const int b = blockIdx.z;
+  const int n0 = blockIdx.x * BN, m0 = blockIdx.y * GM;
+  // the tile as loaded: shifted inward at the ragged end
+  const int ml = g.M >= GM ? min(m0, g.M - GM) : m0;
+  const int nl = g.Nn >= BN ? min(n0, g.Nn - BN) : n0;
+  int arow = (int)((long long)b * g.a_img), brow = (int)((long long)b * g.b_img);
+  if (g.a_text || g.b_text) {
+    const TextGeom tg = text_geom(g.toff, b, g.B, g.Tmax, g.status);
+    if (tg.T == 0) return;  // uniform over the block
+    if (g.a_text) arow += tg.off;
+    if (g.b_text) brow += tg.off;
+  }
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nk = ceil_div(g.Kd, GK);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < GSTAGES; ++s) {
+      tc::mbar_init(&ctl->full[s], 1);
+      tc::mbar_init(&ctl->empty[s], 1);
+    }
+    tc::mbar_init(&ctl->done, 1);
+    ctl->abort = 0;
+    tc::fence_mbar_init();
+    tc::prefetch_tmap(&amap);
+    tc::prefetch_tmap(&bmap);
+  }
+  if (warp == 0) {
+    tc::tmem_alloc(&ctl->tmem, BN);
+    tc::tmem_relinquish();
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = ctl->tmem;
+  const long long deadline = clock64() + G_WAIT;
+  int issued = 0;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      for (int kb = 0; kb < nk; ++kb) {
+        const int s = kb % GSTAGES;
+        const uint32_t ph = (uint32_t)(kb / GSTAGES) & 1u;
+        if (kb >= GSTAGES && !tc::mbar_wait(&ctl->empty[s], ph ^ 1u, deadline)) {
+          ctl->abort = 1;
+          break;
+        }
+        if (ctl->abort) break;
+        tc::mbar_arrive_expect_tx(&ctl->full[s], GA_BYTES + B_BYTES);
+        tc::tma_load_2d(tilesA + s * GA_BYTES, &amap, kb * GK, arow + ml, &ctl->full[s]);
+        tc::tma_load_2d(tilesB + s * B_BYTES, &bmap, kb * GK, brow + nl, &ctl->full[s]);
+        ++issued;
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc = tc::idesc_bf16_f32(GM, BN);
+      for (int kb = 0; kb < nk; ++kb) {
+        const int s = kb % GSTAGES;
+        const uint32_t ph = (uint32_t)(kb / GSTAGES) & 1u;
+        if (!tc::mbar_wait(&ctl->full[s], ph, deadline)) {
+          ctl->abort = 1;
+          break;
+        }
+        tc::fence_after_sync();
+        const uint64_t ad = tc::desc_sw128_kmajor(tilesA + s * GA_BYTES);
+        const uint64_t bd = tc::desc_sw128_kmajor(tilesB + s * B_BYTES);
+#pragma unroll
+        for (int kk = 0; kk < GK / 16; ++kk)
+          tc::mma_bf16(tmem, ad + 2 * kk, bd + 2 * kk, idesc, (kb | kk) != 0);
+        tc::mma_commit(&ctl->empty[s]);
+      }
+      tc::mma_commit(&ctl->done);  // also on abort, so the epilogue wakes up
+    }
+    __syncwarp();
+  } else {
+    // scales of the tile's rows and columns (1 where none is given)
+    for (int q = threadIdx.x - 64; q < GM + BN; q += G_THREADS - 64) {
+      float v = 1.f;
+      if (q < GM) {
+        const int m = ml + q;
+        if (g.rscale && m < g.M) v = g.rscale[(size_t)b * g.M + m];
+        rs[q] = v;
+      } else {
+        const int n = nl + q - GM;
+        if (g.cscale && n < g.Nn) v = g.cscale[(size_t)b * g.Nn + n];
+        cs[q - GM] = v;
+      }
+    }
+  }
+
+  bool ok = tc::mbar_wait(&ctl->done, 0, deadline) && !ctl->abort;
+  ok = __syncthreads_and(ok);  // also publishes the scales
+  tc::fence_after_sync();
+  if (ok && nk > 0) {
+    const int quarter = warp & 3, half = warp >> 2;
+    const int row = quarter * 32 + lane;  // this thread's TMEM lane = tile row
+    const float r = rs[row];
+    // the operand ring is idle now: a padded 32 x 33 staging block per warp
+    float* st = reinterpret_cast<float*>(tilesA) + warp * (32 * 33);
+    const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
+    float* Cimg = g.C + (size_t)b * g.c_img;
+#pragma unroll 1
+    for (int c = 0; c < BN / 64; ++c) {
+      const int cl = half * (BN / 2) + c * 32;  // first column of the chunk, within the tile
+      float v[32];
+      tc::tmem_ld32(trow + (uint32_t)cl, v);
+#pragma unroll
+      for (int q = 0; q < 32; ++q) st[lane * 33 + q] = v[q] * r * cs[cl + q];
+      __syncwarp();
+      const int col = nl + cl + lane;
+      const bool col_ok = col >= n0 && col < g.Nn;  // owned by this tile
+#pragma unroll 4
+      for (int rr = 0; rr < 32; ++rr) {
+        const int m = ml + quarter * 32 + rr;
+        if (m >= m0 && m < g.M && col_ok) Cimg[(size_t)m * g.ldc + col] = st[rr * 33 + lane];
+      }
+      __syncwarp();
+    }
+  }
+  if (!ok && threadIdx.x == 0) set_status(g.status, GMC_STATUS_TIMEOUT);
+  if (warp == 0 && lane == 0 && !ok) {
+    // drain TMA copies still in flight into this CTA's shared memory
+    const long long d2 = clock64() + G_WAIT;
+    for (int kb = (issued > GSTAGES ? issued - GSTAGES : 0); kb < issued; ++kb)
+      if (!tc::mbar_wait(&ctl->full[kb % GSTAGES], (uint32_t)(kb / GSTAGES) & 1u, d2)) break;
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  if (warp == 0) tc::tmem_dealloc(tmem, BN);
+}
+
+// ---------------------------------------------------------------------------
+// host side
+// ---------------------------------------------------------------------------
+template <int BN>
+static cudaError_t launch_gemm_bn(const GemmArgs& g, const void* A, long long a_rows, int lda,
+                                  const void* Bm, long long b_rows, int ldb, cudaStream_t st) {
+  CUtensorMap am, bm;
+  cudaError_t e = make_tmap_bf16(&am, A, (uint64_t)g.Kd, (uint64_t)a_rows, (uint64_t)lda, GM);
+  if (e != cudaSuccess) return e;
+  if ((e = make_tmap_bf16(&bm, Bm, (uint64_t)g.Kd, (uint64_t)b_rows, (uint64_t)ldb, BN)) !=
+      cudaSuccess)
+    return e;
+  const size_t smem = gemm_smem<BN>();
+  if ((e = set_smem_limit((const void*)k_gemm_tc<BN>, smem)) != cudaSuccess) return e;
+  const dim3 grid(ceil_div(g.Nn, BN), ceil_div(g.M, GM), g.B);
+  launch_k(k_gemm_tc<BN>, grid, G_THREADS, smem, st, 1, am, bm, g);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gemm_tc(const GemmArgs& g, const void* A, long long a_rows, int lda,
+                           const void* Bm, long long b_rows, int ldb, cudaStream_t st) {
+  if (g.M < 1 || g.Nn < 1 || g.Kd < 1 || g.B < 1) return cudaErrorInvalidValue;
+  if (g.Nn <= 128) return launch_gemm_bn<128>(g, A, a_rows, lda, Bm, b_rows, ldb, st);
+  return launch_gemm_bn<256>(g, A, a_rows, lda, Bm, b_rows, ldb, st);
+}
+
+}  // namespace gmc

@@ -1025,12 +1025,17 @@ cudaError_t launch_select(const R0State& r0, int B, int N, int K, int M, const i
     cfg.numAttrs = 2;
     if ((e = cudaLaunchKernelEx(&cfg, k_select, a)) != cudaSuccess || !tv.base) return e;
     // diagnostics trace: the batched certificate from the recorded rounds
-    const size_t csm = (sizeof(long long) + 1) * (size_t)N;
-    if ((e = set_smem_limit((const void*)k_certificate, csm)) != cudaSuccess) return e;
-    launch_k(k_certificate, B, 256, csm, st, 1, N, K, tv);
-    return cudaGetLastError();
+    return launch_certificate(B, N, K, tv, st);
   }
   return cudaErrorInvalidConfiguration;
+}
+
+cudaError_t launch_certificate(int B, int N, int K, const TraceView& tv, cudaStream_t st) {
+  const size_t csm = (sizeof(long long) + 1) * (size_t)N;
+  cudaError_t e;
+  if ((e = set_smem_limit((const void*)k_certificate, csm)) != cudaSuccess) return e;
+  launch_k(k_certificate, B, 256, csm, st, 1, N, K, tv);
+  return cudaGetLastError();
 }
 
 }  // namespace gmc

@@ -2,6 +2,7 @@
 // translation units.  Nothing here is exported from libgmc.so.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stddef.h>
@@ -18,9 +19,11 @@ struct Dims {
   int B, N, T, H, Hkv, d, D, K, gh, gw, L;  // L = landmarks per side
   int V;                                    // message views (1: the current view only)
   int I;                                    // images per prompt (N = I * gh * gw)
-  int M;                                    // V*H*T + N + I*L*L: client rows per prompt (max)
+  int MV;                                   // appearance rows: N (exact bank) or the bounded bank's M_V
+  int M;                                    // V*H*T + MV + I*L*L: client rows per prompt (max)
   int dtype;                                // GMC_F32 / GMC_BF16
   const int32_t* toff;                      // device text offsets or nullptr
+  int rank;                                 // long prefixes: rows r of the Rademacher map (0: exact bank)
 };
 
 // Trace record layout passed by value to kernels (byte offsets, 0 = absent).
@@ -140,8 +143,10 @@ cudaError_t launch_heads(const Dims&, const gmc_params&, Scratch&, const TraceVi
                          int cluster = 1, const ViewGrams* views = nullptr);
 bool heads_supported(int H);  // the head statistics of H heads fit a block (H <= 56)
 cudaError_t launch_gram(const Dims&, const void* hidden, Scratch&, cudaStream_t);
+// app: the appearance rows' cosines, [B][MV][N] (the exact bank passes the
+// N x N cosine matrix, MV = N)
 cudaError_t launch_build_clients(const Dims&, const gmc_params&, int fx_exp, Scratch&,
-                                 const ViewRows& views,
+                                 const ViewRows& views, const float* app,
                                  cudaStream_t);
 // State left by the first (dense) selection round, run over the whole GPU.
 // Rounds of the solver run on the whole GPU before the cluster kernel takes
@@ -179,8 +184,12 @@ cudaError_t launch_select(const R0State&, int B, int N, int K, int M, const int3
                           int32_t* slot, int32_t* out_idx, uint32_t* status, const TraceView&,
                           cudaStream_t, int I = 1);
 cudaError_t launch_select_prep(const float* C, int B, int M, int N, Scratch&, cudaStream_t);
+// Batched certificate c_B of the trace from the recorded rounds (one block per image).
+cudaError_t launch_certificate(int B, int N, int K, const TraceView&, cudaStream_t);
+// cs: nullptr (cosines read from the N x N matrix at the support's columns) or
+// the support cosines [B][N][K], column k holding the k-th selected token
 cudaError_t launch_assign(const Dims&, const gmc_params&, Scratch&, const TraceView&,
-                          cudaStream_t);
+                          cudaStream_t, const float* cs = nullptr);
 cudaError_t launch_transport(const Dims&, const gmc_params&, const void* hidden, const void* keys,
                              const int32_t* pos, const int32_t* support, const int32_t* pi,
                              const float* mass, const float* rmsh, const uint32_t* mbits,
@@ -218,8 +227,8 @@ namespace gmc {
 // Argument checks shared by the entry points (gmc_api.cu): every parameter in
 // its documented range; the problem's shape within this build's limits
 // (GMC_OK, GMC_ERR_ARG or GMC_ERR_UNSUPPORTED).
-bool params_ok(const gmc_params& p);
-int check_problem(const gmc_problem* prob, int N, int T, int d, int D);
+bool params_ok(const gmc_params& p, int max_pool = GMC_MAX_POOL);
+int check_problem(const gmc_problem* prob, int N, int T, int d, int D, int max_n = GMC_MAX_N);
 }  // namespace gmc
 
 namespace gmc {
@@ -268,4 +277,66 @@ cudaError_t launch_message_tc(const Dims&, const void* keys, const void* queries
 bool message_tc_supported(const Dims&);
 int message_rq(const Dims&);  // packed query rows per (image, KV group)
 int message_splits(const Dims&);  // key splits of the message slice (parts of rs)
+}  // namespace gmc
+
+namespace gmc {
+// C = diag(rscale) (A B^T) diag(cscale) on the tensor cores (k_gemm_tc.cu):
+// A and B bf16, K-major rows of Kd elements; C fp32.  Image b's A rows start at
+// row b * a_img (+ the image's text offset when a_text: the hidden layout, b*N +
+// off_b) of A's tensor map, its B rows likewise; its C block at b * c_img.
+struct GemmArgs {
+  int B, M, Nn, Kd;          // images, rows, columns, contraction length
+  long long a_img, b_img;    // operand rows between images (0: shared by every image)
+  int a_text, b_text;        // add the image's text offset to the A / B row
+  const int32_t* toff;       // text offsets (nullptr: uniform Tmax)
+  int Tmax;
+  const float* rscale;       // [B][M] or nullptr
+  const float* cscale;       // [B][Nn] or nullptr
+  float* C;                  // output
+  long long c_img, ldc;      // elements between images / rows of C
+  uint32_t* status;
+};
+// a_rows / b_rows: rows declared in the operand's tensor map (reads past them
+// return zeros); lda / ldb: row pitch in elements (a multiple of 8).
+cudaError_t launch_gemm_tc(const GemmArgs&, const void* A, long long a_rows, int lda,
+                           const void* Bm, long long b_rows, int ldb, cudaStream_t);
+cudaError_t make_tmap_bf16(CUtensorMap* map, const void* base, uint64_t row_elems, uint64_t rows,
+                           uint64_t pitch_elems, uint32_t box_rows);
+
+// Long prefixes (k_longprefix.cu): the projected unit states split into bf16
+// hi/lo terms (Xa = [hi|hi|lo], Xb = [hi|lo|hi], XaC = Xa at the M_V uniformly
+// spaced client tokens floor(m N / M_V)), and the selected rows gathered for
+// the support cosines.
+cudaError_t launch_lp_norm(const Dims&, float norm_eps, const float* Y, __nv_bfloat16* Xa,
+                           __nv_bfloat16* Xb, __nv_bfloat16* XaC, uint32_t* status, cudaStream_t);
+cudaError_t launch_gather_support(const Dims&, const void* hidden, const int32_t* support,
+                                  const float* rn, __nv_bfloat16* Hs, float* rnS, uint32_t* status,
+                                  cudaStream_t);
+
+// Wide selection (k_wide.cu): every round of the batched responsibility solver
+// on the whole GPU, for pools above GMC_MAX_POOL and visual counts above
+// GMC_MAX_N (the long-prefix path: b = 512, N = 15,876).
+struct WideState {
+  int32_t* pool;    // [B][P]   pool of the current round (-1 padded)
+  long long* sc;    // [B][P]   its scores (fixed point)
+  int32_t* batch;   // [B][P]   the current round's batch, in score order
+  int32_t* stamp;   // [B][N]   1 + the round a token entered the support (0: not yet)
+  int32_t* info;    // [B][INFO_W] as R0State::info
+  long long* u1;    // [B][N]   gains written by rounds 0, 2, ...
+  long long* u2;    // [B][N]   gains written by rounds 1, 3, ...
+  float* bcov;      // [B][M]   coverage b_m
+  int32_t* cnt;     // [B][M]   survivors per row
+  long long* fv;    // [B][4]   F_b(V) per bank (fixed point)
+};
+struct WideGeom {
+  int B, N, K, Mstride;  // client rows per image (stride)
+  int HV, Tmax, MV, L2;  // grounded rows per text token, appearance rows, spatial rows
+  const int32_t* toff;
+  int uniform;           // gmc_select: every image has Mstride rows, all in bank 0
+};
+int wide_rounds(int K, const gmc_params&);  // whole-GPU rounds launched: ceil(K / b)
+cudaError_t launch_wide_select(const WideState&, const WideGeom&, const gmc_params&, int fx_exp,
+                               const int32_t* fexp, float* C, uint16_t* scol, const long long* u0,
+                               int32_t* order, int32_t* support, int32_t* slot, int32_t* out_idx,
+                               uint32_t* status, const TraceView&, cudaStream_t);
 }  // namespace gmc

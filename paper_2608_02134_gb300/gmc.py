@@ -28,7 +28,7 @@ EXPORTS = (
     "gmc_version", "gmc_profile_enable", "gmc_profile_read", "gmc_launch_count",
     "gmc_transport_noalloc", "gmc_cosine_workspace_size", "gmc_cosine",
     "gmc_workspace_size_views", "gmc_compress_views", "gmc_clients", "gmc_selftest_bounded_wait",
-    "gmc_compress_ex",
+    "gmc_compress_ex", "gmc_workspace_size_long", "gmc_compress_long", "gmc_clients_long",
 )
 MAX_VIEWS = 4
 MAX_PREFIX_LAYERS = 64
@@ -67,6 +67,11 @@ class PrefixKV(ctypes.Structure):
     _fields_ = [("n_layers", ctypes.c_int),
                 ("keys", ctypes.c_void_p * MAX_PREFIX_LAYERS),
                 ("out_kv", ctypes.c_void_p * MAX_PREFIX_LAYERS)]
+
+
+class LongPrefix(ctypes.Structure):
+    _fields_ = [("rank", ctypes.c_int), ("max_clients", ctypes.c_int),
+                ("rademacher", ctypes.c_void_p)]
 
 
 class TraceHeader(ctypes.Structure):
@@ -149,6 +154,15 @@ def lib() -> ctypes.CDLL:
     L.gmc_clients.argtypes = [PP, P, ctypes.POINTER(Views), vp, vp, vp, vp, vp, i, i, i, i, i, i,
                               vp, vp, sz, vp, vp]
     L.gmc_clients.restype = i
+    LP = ctypes.POINTER(LongPrefix)
+    L.gmc_workspace_size_long.argtypes = [PP, P, LP, i, i, i, i, i, i, i]
+    L.gmc_workspace_size_long.restype = sz
+    L.gmc_compress_long.argtypes = [PP, P, LP, ctypes.POINTER(Views), ctypes.POINTER(PrefixKV), vp,
+                                    vp, vp, vp, vp, i, i, i, i, i, i, vp, vp, vp, vp, vp, sz, vp, vp]
+    L.gmc_compress_long.restype = i
+    L.gmc_clients_long.argtypes = [PP, P, LP, ctypes.POINTER(Views), vp, vp, vp, vp, vp, i, i, i,
+                                   i, i, i, vp, vp, sz, vp, vp]
+    L.gmc_clients_long.restype = i
     L.gmc_selftest_bounded_wait.argtypes = [ctypes.c_longlong, vp, sz, vp]
     L.gmc_selftest_bounded_wait.restype = i
     _lib = L
@@ -271,6 +285,41 @@ def clients(prob: Problem, params: Params, vw: Views | None, hidden, keys, queri
         _ptr(out_clients), _ptr(workspace), workspace.numel(), _ptr(trace), _stream(stream)))
 
 
+def long_prefix(rademacher, max_clients=4096) -> LongPrefix:
+    """The bounded appearance bank of long prefixes: rademacher is the device
+    bf16 [r][D] map (entries +-1), max_clients the M_V cap."""
+    return LongPrefix(int(rademacher.shape[0]), int(max_clients), rademacher.data_ptr())
+
+
+def workspace_size_long(prob: Problem, params: Params, lp: LongPrefix, n_views, N, T, H, d, D,
+                        K) -> int:
+    return int(lib().gmc_workspace_size_long(ctypes.byref(prob), ctypes.byref(params),
+                                             ctypes.byref(lp), n_views, N, T, H, d, D, K))
+
+
+def compress_long(prob: Problem, params: Params, lp: LongPrefix, vw, pf, hidden, keys, queries,
+                  pos_ids, vo_probe, N, T, H, d, D, K, out_idx, out_hidden, out_kv, out_pos,
+                  workspace, trace=None, stream=None):
+    """gmc_compress_long on device tensors (vw, pf: Views / PrefixKV or None; see include/gmc.h)."""
+    _check(lib().gmc_compress_long(
+        ctypes.byref(prob), ctypes.byref(params), ctypes.byref(lp),
+        ctypes.byref(vw) if vw is not None else None, ctypes.byref(pf) if pf is not None else None,
+        _ptr(hidden), _ptr(keys), _ptr(queries), _ptr(pos_ids), _ptr(vo_probe), N, T, H, d, D, K,
+        _ptr(out_idx), _ptr(out_hidden), _ptr(out_kv), _ptr(out_pos), _ptr(workspace),
+        workspace.numel(), _ptr(trace), _stream(stream)))
+
+
+def clients_long(prob: Problem, params: Params, lp: LongPrefix, vw, hidden, keys, queries,
+                 pos_ids, vo_probe, N, T, H, d, D, K, out_clients, workspace, trace=None,
+                 stream=None):
+    """gmc_clients_long: the client matrix with the bounded appearance bank."""
+    _check(lib().gmc_clients_long(
+        ctypes.byref(prob), ctypes.byref(params), ctypes.byref(lp),
+        ctypes.byref(vw) if vw is not None else None, _ptr(hidden), _ptr(keys), _ptr(queries),
+        _ptr(pos_ids), _ptr(vo_probe), N, T, H, d, D, K, _ptr(out_clients), _ptr(workspace),
+        workspace.numel(), _ptr(trace), _stream(stream)))
+
+
 def selftest_bounded_wait(cycles: int, workspace, stream=None):
     """gmc_selftest_bounded_wait: a device wait that nothing ends, bounded by `cycles` clocks."""
     _check(lib().gmc_selftest_bounded_wait(cycles, _ptr(workspace), workspace.numel(),
@@ -368,7 +417,8 @@ class Compressor:
     """
 
     def __init__(self, B, grid_h, grid_w, T, H, Hkv, d, D, K, dtype, text_lengths=None,
-                 params: Params | None = None, trace=False, device="cuda", n_views=0, images=1):
+                 params: Params | None = None, trace=False, device="cuda", n_views=0, images=1,
+                 long_prefix: LongPrefix | None = None):
         self.B, self.gh, self.gw, self.T, self.H, self.Hkv, self.d, self.D = B, grid_h, grid_w, T, H, Hkv, d, D
         self.images = images
         self.N = grid_h * grid_w * images
@@ -386,7 +436,12 @@ class Compressor:
         self.offsets = torch.tensor(off, dtype=torch.int32, device=device) if text_lengths is not None else None
         self.prob = problem(B, grid_h, grid_w, Hkv, dtype, self.offsets, images)
         self.n_views = n_views
-        ws = workspace_size_views(self.prob, n_views, self.N, T, H, d, D, K)
+        self.long_prefix = long_prefix
+        if long_prefix is not None:
+            ws = workspace_size_long(self.prob, self.params, long_prefix, n_views, self.N, T, H, d,
+                                     D, K)
+        else:
+            ws = workspace_size_views(self.prob, n_views, self.N, T, H, d, D, K)
         if ws == 0:
             raise GMCError("invalid problem for gmc_workspace_size")
         self.workspace = alloc_workspace(ws, device)
@@ -407,7 +462,20 @@ class Compressor:
         """history: None, or (keys, queries, vo_probe) lists of the historical views;
         prefix: None, or the dense prefix layers' K/V tensors (layout of `keys`),
         gathered into self.out_prefix (one tensor per layer, layout of out_kv)."""
-        if prefix is not None:
+        if history is not None and len(history[0]) > self.n_views:
+            raise GMCError("more historical views than the workspace was sized for")
+        if self.long_prefix is not None:
+            pf = None
+            if prefix is not None:
+                if getattr(self, "out_prefix", None) is None or len(self.out_prefix) != len(prefix):
+                    self.out_prefix = [torch.empty_like(self.out_kv) for _ in prefix]
+                pf = prefix_kv(prefix, self.out_prefix)
+            vw = views(*history, beta_hist=beta_hist) if history is not None else None
+            compress_long(self.prob, self.params, self.long_prefix, vw, pf, hidden, keys, queries,
+                          pos_ids, vo_probe, self.N, self.T, self.H, self.d, self.D, self.Kr,
+                          self.out_idx, self.out_hidden, self.out_kv, self.out_pos,
+                          self.workspace, self.trace, stream)
+        elif prefix is not None:
             if history is not None and len(history[0]) > self.n_views:
                 raise GMCError("more historical views than the workspace was sized for")
             if getattr(self, "out_prefix", None) is None or len(self.out_prefix) != len(prefix):

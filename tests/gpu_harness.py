@@ -25,6 +25,7 @@ class GpuRun:
     traces: list
     n_hist: int = 0
     prefix: list = None     # per dense prefix layer: gathered K/V (float64 values), layout of kv
+    long_prefix: dict = None  # bounded appearance bank: {"R": map [r, D], "max_clients": M_V cap}
 
 
 def to_device(wl: workloads.Workload, device="cuda"):
@@ -47,13 +48,30 @@ def _dev(a, device="cuda"):
     return t.to(device)
 
 
+def long_prefix_of(wl: workloads.Workload):
+    """The long-prefix workloads' bounded bank: (oracle dict, batch b) or (None, None)."""
+    cfg = workloads.LONG_PREFIX.get(wl.name)
+    if cfg is None:
+        return None, None
+    R = workloads.rademacher(wl.D, cfg["rank"])
+    return {"R": R, "max_clients": cfg["max_clients"]}, cfg["batch_b"]
+
+
 def run(wl: workloads.Workload, params=None, trace=True, inputs=None, n_hist=0,
         n_prefix=0) -> GpuRun:
     dt = gmc.GMC_BF16 if wl.dtype == "bf16" else gmc.GMC_F32
     inp = inputs or to_device(wl)
+    lpo, lpb = long_prefix_of(wl)
+    lp = None
+    if lpo is not None:
+        if params is None:
+            params = gmc.default_params(batch_b=lpb)
+        R = torch.from_numpy(lpo["R"]).to(torch.bfloat16).cuda()
+        lp = gmc.long_prefix(R, lpo["max_clients"])
+        lp._keep = R  # the map stays alive as long as the struct that points to it
     comp = gmc.Compressor(wl.B, wl.gh, wl.gw, wl.T_max, wl.H, wl.Hkv, wl.d, wl.D, wl.K, dt,
                           text_lengths=wl.T if wl.ragged else None, params=params, trace=trace,
-                          n_views=n_hist, images=wl.I)
+                          n_views=n_hist, images=wl.I, long_prefix=lp)
     history = None
     if n_hist:
         hv = [wl.history_abi_arrays(v) for v in range(n_hist)]
@@ -73,7 +91,7 @@ def run(wl: workloads.Workload, params=None, trace=True, inputs=None, n_hist=0,
                                     comp.params.max_head_clusters)
     pref = [t.float().cpu().numpy() for t in comp.out_prefix] if n_prefix else None
     return GpuRun(wl, comp, out.idx.cpu().numpy(), hid, raw, out.kv.float().cpu().numpy(),
-                  out.pos.cpu().numpy(), status, traces, n_hist, pref)
+                  out.pos.cpu().numpy(), status, traces, n_hist, pref, lpo)
 
 
 def oracle_params(p: gmc.Params) -> dict:
@@ -119,7 +137,7 @@ def compare_image(g: GpuRun, b: int, hidden_tol: float) -> ImageReport:
                   for l in range(len(g.prefix))]
     res = O.compress(f(im.hidden), f(im.keys), f(im.values), f(im.queries), im.pos, f(wl.probe()),
                      wl.gh, wl.gw, wl.K, p, forced=forced, history=history, prefix=prefix,
-                     n_images=wl.I)
+                     n_images=wl.I, long_prefix=g.long_prefix)
     dec = parity.Decisions()
     tag = f"{wl.name}[b={b}]"
     parity.check_heads(res.heads, dec, tag)

@@ -126,3 +126,61 @@ def test_binding_raises_without_the_library(gmc, monkeypatch, tmp_path):
     monkeypatch.setattr(gmc, "LIB_PATH", str(tmp_path / "libgmc.so"))
     with pytest.raises(RuntimeError, match="missing"):
         gmc.lib()
+
+
+def _long_rc(gmc, prob, lp, params=None, ws_bytes=1 << 40, **shape):
+    lib = gmc.lib()
+    sh = dict(N=1600, T=16, H=4, d=64, D=256, K=320)
+    sh.update(shape)
+    fake = ctypes.c_void_p(1 << 20)
+    return lib.gmc_compress_long(ctypes.byref(prob), params, ctypes.byref(lp) if lp else None,
+                                 None, None, fake, fake, fake, fake, fake, sh["N"], sh["T"],
+                                 sh["H"], sh["d"], sh["D"], sh["K"], fake, fake, fake, fake,
+                                 fake, ws_bytes, None, None)
+
+
+def test_long_prefix_sizing_and_validation(gmc):
+    """gmc_compress_long: the bounded bank's limits (bf16, one image, N >= 128,
+    rank a multiple of 8 up to GMC_MAX_RANK, N up to GMC_MAX_N_LONG, pools up
+    to GMC_MAX_POOL_WIDE)."""
+    assert ctypes.sizeof(gmc.LongPrefix) == 16
+    lp = gmc.LongPrefix(128, 4096, 1 << 20)
+    pr = gmc.problem(1, 126, 126, 4, gmc.GMC_BF16)
+    p = gmc.default_params(batch_b=512)
+    N = 126 * 126
+    ws = gmc.workspace_size_long(pr, p, lp, 0, N, 128, 28, 128, 3584, 4096)
+    # the client matrix with M_V = 4096 appearance rows, and the N x K support cosines
+    M = 28 * 128 + 4096 + 256
+    assert ws >= M * N * 4 + N * 4096 * 4
+    # no N x N cosine matrix: far below what the exact bank would need
+    assert ws < M * N * 6 + N * N * 4
+    assert gmc.workspace_size_long(pr, gmc.default_params(), lp, 0, N, 128, 28, 128, 3584,
+                                   4096) > 0
+    assert gmc.workspace_size_long(pr, p, lp, 0, N, 128, 28, 128, 3584, 4096) > \
+        gmc.workspace_size_long(pr, gmc.default_params(), lp, 0, N, 128, 28, 128, 3584, 4096)
+    small = gmc.problem(1, 40, 40, 2, gmc.GMC_BF16)
+    lps = gmc.LongPrefix(128, 512, 1 << 20)
+    p64 = gmc.default_params(batch_b=64)
+    assert _long_rc(gmc, small, lps, ctypes.byref(p64), ws_bytes=1024) == gmc.GMC_ERR_WORKSPACE
+    assert _long_rc(gmc, small, None, ctypes.byref(p64)) == gmc.GMC_ERR_ARG
+    assert _long_rc(gmc, small, gmc.LongPrefix(12, 512, 1 << 20), ctypes.byref(p64)) == gmc.GMC_ERR_ARG
+    assert _long_rc(gmc, small, gmc.LongPrefix(128, 0, 1 << 20), ctypes.byref(p64)) == gmc.GMC_ERR_ARG
+    assert _long_rc(gmc, small, gmc.LongPrefix(128, 512, 0), ctypes.byref(p64)) == gmc.GMC_ERR_ARG
+    assert _long_rc(gmc, small, gmc.LongPrefix(264, 512, 1 << 20), ctypes.byref(p64)) == \
+        gmc.GMC_ERR_UNSUPPORTED                                             # rank > 256
+    assert _long_rc(gmc, gmc.problem(1, 40, 40, 2, gmc.GMC_F32), lps, ctypes.byref(p64)) == \
+        gmc.GMC_ERR_UNSUPPORTED                                             # bf16 only
+    assert _long_rc(gmc, gmc.problem(1, 8, 8, 2, gmc.GMC_BF16), lps, ctypes.byref(p64),
+                    N=64) == gmc.GMC_ERR_UNSUPPORTED                        # N < 128
+    assert _long_rc(gmc, gmc.problem(1, 40, 40, 2, gmc.GMC_BF16, images=2), lps,
+                    ctypes.byref(p64), N=3200) == gmc.GMC_ERR_UNSUPPORTED   # one image
+    assert _long_rc(gmc, gmc.problem(1, 130, 130, 2, gmc.GMC_BF16), lps, ctypes.byref(p64),
+                    N=16900) == gmc.GMC_ERR_UNSUPPORTED                     # N > 16384
+    big = gmc.default_params(batch_b=2048, pool_mult=4)                     # pool 8192 > 4096
+    assert _long_rc(gmc, small, lps, ctypes.byref(big)) == gmc.GMC_ERR_ARG
+    # the standard entry point keeps its limits
+    assert _compress_rc(gmc, prob=pr, N=N, T=128, H=28, d=128, D=3584, K=4096) == \
+        gmc.GMC_ERR_UNSUPPORTED
+    # gmc_select accepts wide pools (every round on the whole GPU) and longer N with them
+    assert gmc.select_workspace_size(1, 500, 12000, 1500, p) > 500 * 12000 * 6
+    assert gmc.select_workspace_size(1, 500, 12000, 1500, gmc.default_params()) == 0
