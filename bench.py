@@ -10,6 +10,10 @@ D=3584, K=257, bf16), synthetic seeded tensors.  Inputs are resident in HBM;
 L2 is flushed (a 512 MiB write) before every timed step.  Under torchrun every
 rank compresses its own boundaries (independent replicas, weak scaling).
 
+--workload longdoc runs the long-prefix document path instead (N=15876 on
+126x126, T=128, K=4096, bounded appearance bank of rank 128 with at most 4096
+clients, b=512) through gmc_compress_long.
+
 --impl reference times the fp64 CPU oracle on the host cores on the same
 workload (one boundary per step); rank 0 only.
 """
@@ -47,6 +51,28 @@ METRIC = "compressed boundaries/sec (us/boundary) at Qwen2.5-VL-7B shape; % HBM 
 UNIT = "boundaries/s"
 
 
+def long_prefix_cfg(wl):
+    """(rademacher map, max_clients, batch_b) of a long-prefix workload, else None."""
+    from paper_2608_02134_gb300 import workloads
+    cfg = workloads.LONG_PREFIX.get(wl.name)
+    if cfg is None:
+        return None
+    return workloads.rademacher(wl.D, cfg["rank"]), cfg["max_clients"], cfg["batch_b"]
+
+
+def oracle_step(wl, k: int):
+    """One oracle boundary of the workload (image k % B)."""
+    import numpy as np
+    from oracle import gmc_oracle as O
+    f = lambda a: np.asarray(a, dtype=np.float64)
+    im = wl.image(k % wl.B)
+    lp = long_prefix_cfg(wl)
+    p = O.params(batch_b=lp[2]) if lp else O.params()
+    long_prefix = {"R": f(lp[0]), "max_clients": lp[1]} if lp else None
+    O.compress(f(im.hidden), f(im.keys), f(im.values), f(im.queries), im.pos, f(wl.probe()),
+               wl.gh, wl.gw, wl.K, p, long_prefix=long_prefix)
+
+
 def workload_config(wl) -> dict:
     return {"workload": f"{wl.name}: B={wl.B} N={wl.N} ({wl.gh}x{wl.gw}) T={'ragged' if wl.ragged else wl.T_max} "
                         f"H={wl.H} Hkv={wl.Hkv} d={wl.d} D={wl.D} K={wl.K} {wl.dtype}",
@@ -58,18 +84,13 @@ def workload_config(wl) -> dict:
 # ---------------------------------------------------------------------------
 def oracle_sample(name: str, n: int, min_seconds: float = 10.0) -> dict:
     """Oracle boundaries of the workload until min_seconds of CPU work (at most n)."""
-    import numpy as np
-    from oracle import gmc_oracle as O
     from paper_2608_02134_gb300 import workloads
     wl = workloads.make(name)
-    f = lambda a: np.asarray(a, dtype=np.float64)
     t = 0.0
     k = 0
     while k < n and (k == 0 or t < min_seconds):
-        im = wl.image(k % wl.B)
         t0 = time.perf_counter()
-        O.compress(f(im.hidden), f(im.keys), f(im.values), f(im.queries), im.pos, f(wl.probe()),
-                   wl.gh, wl.gw, wl.K)
+        oracle_step(wl, k)
         t += time.perf_counter() - t0
         k += 1
     return {"seconds": t, "boundaries": k}
@@ -158,8 +179,25 @@ def stage_work(wl) -> dict:
     B, N, H, Hkv, d, D, K = wl.B, wl.N, wl.H, wl.Hkv, wl.d, wl.D, wl.K
     es = 2 if wl.dtype == "bf16" else 4
     Tm = sum(wl.T) / B
-    M = H * Tm + N + 256
+    lp = long_prefix_cfg(wl)
+    MV = min(N, lp[1]) if lp else N
+    M = H * Tm + MV + 256
     w = {}
+    if lp:  # long prefixes: bounded bank, wide solver, N x K support cosines
+        r = lp[0].shape[0]
+        w["project"] = ("hbm", B * (N * D * es + N * r * 4.0 + 2 * 2 * N * 3 * r + MV * 3 * r * 2))
+        w["app_cos"] = ("hbm", B * (MV * N * 4.0 + (MV + N) * 3 * r * 2))
+        w["support_cos"] = ("tensor", B * 2.0 * N * K * D)
+        w["select"] = ("hbm", B * -(-K // lp[2]) * (M * N * 4.0))
+        w["clients"] = ("hbm", B * (M * N * 4 + H * Tm * N * 4 + MV * N * 4.0))
+        w["assign"] = ("hbm", B * (N * K * 4.0))
+        w["message"] = ("hbm", B * (H * Tm * N * 4 + 2 * (N + Tm) * Hkv * d * es + Tm * H * d * es))
+        w["transport"] = ("hbm", B * ((N + Tm) * D * es + (K + Tm) * D * es
+                                      + 2 * (K + Tm) * 2 * Hkv * d * es + 2 * 3 * (K + Tm) * 4 + 3 * N * 4))
+        w["heads"] = ("hbm", B * (H * Tm * N * 4))
+        w["probe"] = ("hbm", B * N * Hkv * d * es)
+        w["rownorm"] = ("hbm", B * N * D * es)
+        return w
     # the cosine Gram: the method needs the symmetric half, 2 * N(N+1)/2 * D
     # flops (the kernel issues the 128 x 128 tiles on and above the diagonal)
     w["gram"] = ("tensor", B * 1.0 * N * (N + 1) * D)
@@ -249,8 +287,15 @@ def run_gmc(args):
             t = t.view(torch.int16).view(torch.bfloat16)
         host[k] = t.pin_memory()
     inp = {k: v.to(dev) for k, v in host.items()}
+    lpc = long_prefix_cfg(wl)
+    lp, params = None, None
+    if lpc:
+        rmap = torch.from_numpy(lpc[0]).to(torch.bfloat16).to(dev)
+        lp = gmc.long_prefix(rmap, lpc[1])
+        params = gmc.default_params(batch_b=lpc[2])
     comp = gmc.Compressor(wl.B, wl.gh, wl.gw, wl.T_max, wl.H, wl.Hkv, wl.d, wl.D, wl.K, dt,
-                          text_lengths=wl.T if wl.ragged else None, device=dev)
+                          text_lengths=wl.T if wl.ragged else None, device=dev, params=params,
+                          long_prefix=lp)
     flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)
 
@@ -387,16 +432,12 @@ def run_reference(args):
     if rank != 0:
         return
     import numpy as np  # noqa: F401  (thread count fixed by the environment set in main)
-    from oracle import gmc_oracle as O
     from paper_2608_02134_gb300 import workloads
     wl = workloads.make(args.workload)
-    f = lambda a: np.asarray(a, dtype=np.float64)
     times = []
     for k in range(max(args.warmup, 0) + args.steps):
-        im = wl.image(k % wl.B)
         t0 = time.perf_counter()
-        O.compress(f(im.hidden), f(im.keys), f(im.values), f(im.queries), im.pos, f(wl.probe()),
-                   wl.gh, wl.gw, wl.K)
+        oracle_step(wl, k)
         if k >= args.warmup:
             times.append(time.perf_counter() - t0)
     sec = sum(times) / len(times)
