@@ -10,8 +10,12 @@
 //   * the N x K support cosines of the assignment, cos(h_i, h_{S_k}) (A =
 //     visual hidden rows, B = the selected rows gathered, scaled by the
 //     reciprocal norms of both).
+//   * the cosine Gram of the boundary states for large or batched problems
+//     (symmetric mode: A = B = the visual rows, scaled by their reciprocal
+//     norms; only tiles on or above the diagonal are computed).
 // (Appendix "Appearance and spatial clients", last paragraph; the cost notes
-// after Algorithm 1: the bounded bank and the chunked N x K assignment product.)
+// after Algorithm 1: the bounded bank and the chunked N x K assignment product;
+// Eq. (cond-aux-clients), (cond-assignment) for the cosines.)
 //
 // One CTA computes one 128 x BN output tile (BN = 128 or 256, one TMEM column
 // per output column).  Warp 0 / lane 0 streams 64-wide K slices of the A and B
@@ -26,9 +30,14 @@
 // likewise Nn - BN) so every box lies inside the image's own rows -- the
 // hidden states' visual rows are followed by text rows whose count only the
 // device knows -- and stores only the rows and columns the previous tile does
-// not own; a smaller operand reads zeros past its declared rows.  Every mbarrier wait is bounded (about two seconds);
-// on timeout the kernel records GMC_STATUS_TIMEOUT, drains its copies and
-// frees its tensor memory.
+// not own; a smaller operand reads zeros past its declared rows.  Symmetric
+// mode (M == Nn, A and B the same rows): the grid enumerates the tiles that
+// hold an entry with j >= i; a tile stores its own entries and, from
+// registers (coalesced over the lanes), the mirror C[j][i] of each entry
+// j > i whose own tile is not computed -- every entry is written exactly
+// once, so the result does not depend on the order of the stores.  Every
+// mbarrier wait is bounded (about two seconds); on timeout the kernel records
+// GMC_STATUS_TIMEOUT, drains its copies and frees its tensor memory.
 #include "common.cuh"
 #include "kernels.cuh"
 #include "tc.cuh"
@@ -48,6 +57,16 @@ struct GemmCtl {
   uint32_t tmem;
   volatile int abort;
 };
+
+// Symmetric mode: tile (I, J) (rows 128 I.., columns BN J..) is computed when it
+// holds an entry with j >= i.
+template <int BN> __host__ __device__ __forceinline__ bool sym_tile(int I, int J) {
+  return BN * J + BN - 1 >= GM * I;
+}
+template <int BN> __host__ __device__ __forceinline__ int sym_first_col(int I) {
+  const int x = GM * I - (BN - 1);
+  return x <= 0 ? 0 : (x + BN - 1) / BN;
+}
 
 template <int BN> constexpr size_t gemm_smem() {
   return 1024 + (size_t)GSTAGES * (GA_BYTES + BN * GK * 2) + sizeof(GemmCtl) + sizeof(float) * (GM + BN);
@@ -70,7 +89,18 @@ __global__ void __launch_bounds__(G_THREADS, 1)
   float* cs = rs + GM;                            // [BN] column scales
 
   const int b = blockIdx.z;
-  const int n0 = blockIdx.x * BN, m0 = blockIdx.y * GM;
+  int tI = blockIdx.y, tJ = blockIdx.x;
+  if (g.sym) {  // blockIdx.x enumerates the computed tiles, row block by row block
+    const int nJ = ceil_div(g.Nn, BN);
+    int t = blockIdx.x;
+    tI = 0;
+    while (t >= nJ - sym_first_col<BN>(tI)) {
+      t -= nJ - sym_first_col<BN>(tI);
+      ++tI;
+    }
+    tJ = sym_first_col<BN>(tI) + t;
+  }
+  const int n0 = tJ * BN, m0 = tI * GM;
   // the tile as loaded: shifted inward at the ragged end
   const int ml = g.M >= GM ? min(m0, g.M - GM) : m0;
   const int nl = g.Nn >= BN ? min(n0, g.Nn - BN) : n0;
@@ -177,7 +207,20 @@ __global__ void __launch_bounds__(G_THREADS, 1)
       float v[32];
       tc::tmem_ld32(trow + (uint32_t)cl, v);
 #pragma unroll
-      for (int q = 0; q < 32; ++q) st[lane * 33 + q] = v[q] * r * cs[cl + q];
+      for (int q = 0; q < 32; ++q) {
+        v[q] *= r * cs[cl + q];
+        st[lane * 33 + q] = v[q];
+      }
+      if (g.sym) {  // mirrors of owned entries j > i whose own tile is not computed
+        const int i = ml + row;
+        const bool own_i = i >= m0 && i < g.M;
+#pragma unroll 4
+        for (int q = 0; q < 32; ++q) {
+          const int j = nl + cl + q;
+          if (own_i && j >= n0 && j < g.Nn && j > i && !sym_tile<BN>(j / GM, i / BN))
+            Cimg[(size_t)j * g.ldc + i] = v[q];
+        }
+      }
       __syncwarp();
       const int col = nl + cl + lane;
       const bool col_ok = col >= n0 && col < g.Nn;  // owned by this tile
@@ -215,14 +258,27 @@ static cudaError_t launch_gemm_bn(const GemmArgs& g, const void* A, long long a_
     return e;
   const size_t smem = gemm_smem<BN>();
   if ((e = set_smem_limit((const void*)k_gemm_tc<BN>, smem)) != cudaSuccess) return e;
-  const dim3 grid(ceil_div(g.Nn, BN), ceil_div(g.M, GM), g.B);
+  dim3 grid(ceil_div(g.Nn, BN), ceil_div(g.M, GM), g.B);
+  if (g.sym) grid = dim3(gemm_sym_ctas(g.M, 1), 1, g.B);  // the computed tiles of every image
   launch_k(k_gemm_tc<BN>, grid, G_THREADS, smem, st, 1, am, bm, g);
   return cudaGetLastError();
+}
+
+int gemm_sym_ctas(int N, int B) {  // symmetric Grams use 128 x 256 tiles (N > 128)
+  int nt = 0;
+  for (int I = 0; I < ceil_div(N, GM); ++I) nt += ceil_div(N, 256) - sym_first_col<256>(I);
+  return nt * B;
 }
 
 cudaError_t launch_gemm_tc(const GemmArgs& g, const void* A, long long a_rows, int lda,
                            const void* Bm, long long b_rows, int ldb, cudaStream_t st) {
   if (g.M < 1 || g.Nn < 1 || g.Kd < 1 || g.B < 1) return cudaErrorInvalidValue;
+  if (g.sym && (g.M != g.Nn || g.Nn <= 128)) return cudaErrorInvalidValue;
+  // an operand addressed from the hidden states (a_text / b_text) must hold a
+  // full box of rows, so the shifted last box stays inside the image's visual
+  // rows (the buffer may end right after the last image's text rows)
+  if ((g.a_text && g.M < GM) || (g.b_text && g.Nn < (g.Nn <= 128 ? 128 : 256)))
+    return cudaErrorInvalidValue;
   if (g.Nn <= 128) return launch_gemm_bn<128>(g, A, a_rows, lda, Bm, b_rows, ldb, st);
   return launch_gemm_bn<256>(g, A, a_rows, lda, Bm, b_rows, ldb, st);
 }

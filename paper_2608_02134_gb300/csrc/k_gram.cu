@@ -78,10 +78,35 @@ cudaError_t launch_gram_simt(const Dims& dm, const void* hidden, Scratch& s, cud
 }
 
 cudaError_t launch_gram(const Dims& dm, const void* hidden, Scratch& s, cudaStream_t st) {
-  // bf16 states with at least one full 128-row tile: tcgen05 (k_gram_tc.cu);
-  // fp32 states (exact fp32 products) and tiny grids: the CUDA-core kernel above.
-  if (gram_tc_supported(dm)) return launch_gram_tc(dm, hidden, s, st);
-  return launch_gram_simt(dm, hidden, s, st);
+  // bf16 states with at least one full 128-row tile: tcgen05.  Problems whose
+  // 128 x 256 tiles on or above the diagonal fill the GPU at least once (the
+  // document page, serving batches) run the general kernel in symmetric mode
+  // (k_gemm_tc.cu); a single smaller image runs the split-contraction Gram of
+  // k_gram_tc.cu, which keeps more SMs busy at that size.  fp32 states (exact
+  // fp32 products) and tiny grids: the CUDA-core kernel above.
+  if (!gram_tc_supported(dm)) return launch_gram_simt(dm, hidden, s, st);
+  static int sms = 0;
+  if (sms == 0) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+      cudaGetLastError();
+      sms = 152;
+    }
+  }
+  if (dm.N >= 256 && gemm_sym_ctas(dm.N, dm.B) >= sms) {
+    GemmArgs g{};
+    g.B = dm.B; g.M = dm.N; g.Nn = dm.N; g.Kd = dm.D;
+    g.a_img = dm.N; g.b_img = dm.N; g.a_text = 1; g.b_text = 1;
+    g.toff = dm.toff; g.Tmax = dm.T;
+    g.rscale = s.rn; g.cscale = s.rn;
+    g.C = s.cos; g.c_img = (long long)dm.N * dm.N; g.ldc = dm.N;
+    g.status = s.status;
+    g.sym = 1;
+    const long long rows = (long long)dm.B * (dm.N + dm.T);
+    return launch_gemm_tc(g, hidden, rows, dm.D, hidden, rows, dm.D, st);
+  }
+  return launch_gram_tc(dm, hidden, s, st);
 }
 
 }  // namespace gmc

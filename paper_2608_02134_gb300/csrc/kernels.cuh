@@ -295,7 +295,10 @@ struct GemmArgs {
   float* C;                  // output
   long long c_img, ldc;      // elements between images / rows of C
   uint32_t* status;
+  int sym;                   // 1: C symmetric (A, B the same rows, M == Nn > 128): tiles on
+                             // or above the diagonal computed, the rest mirrored
 };
+int gemm_sym_ctas(int N, int B);  // CTAs of the symmetric mode for N x N Grams of B images
 // a_rows / b_rows: rows declared in the operand's tensor map (reads past them
 // return zeros); lda / ldb: row pitch in elements (a multiple of 8).
 cudaError_t launch_gemm_tc(const GemmArgs&, const void* A, long long a_rows, int lda,

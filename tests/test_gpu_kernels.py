@@ -27,6 +27,10 @@ def _cos_ref(h64: torch.Tensor) -> torch.Tensor:
     (2, 12, 12, 128, [9, 1], torch.bfloat16),      # 2 x 2 tiles, 16-row ragged edge, T_b = 1
     (1, 13, 11, 256, [4], torch.bfloat16),         # N % 4 != 0: CUDA-core path
     (1, 10, 10, 40, [3], torch.float32),           # CUDA-core path
+    # the general kernel's symmetric mode (its tiles fill the GPU at least once):
+    (1, 64, 64, 256, [17], torch.bfloat16),        # document page grid, 128 x 256 tiles
+    (6, 36, 36, 640, [64, 3, 40, 1, 64, 16], torch.bfloat16),  # a batch, ragged text
+    (4, 50, 50, 200, [8, 8, 8, 8], torch.bfloat16),  # ragged row and column tiles, D % 64 != 0
 ])
 def test_cosine_matches_fp64_reference(B, gh, gw, D, tlens, dtype):
     from paper_2608_02134_gb300 import gmc
