@@ -272,7 +272,7 @@ size_t gmc_workspace_size_long(const gmc_problem* prob, const gmc_params* params
  * appearance bank values F_S[1] / F_V[1] are the bounded bank's.  params may
  * set pool_mult * batch_b up to GMC_MAX_POOL_WIDE (the paper's b = 512 gives a
  * pool of 2048).
- * Limits: bf16 states, one image per prompt (images 0 or 1), 128 <= N <=
+ * Limits: bf16 states, one image per prompt (images 0 or 1), 256 <= N <=
  * GMC_MAX_N_LONG, and the limits of gmc_compress otherwise; GMC_ERR_UNSUPPORTED
  * beyond them, GMC_ERR_ARG for a NULL, misaligned or out-of-range lp.
  */

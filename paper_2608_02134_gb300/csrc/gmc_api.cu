@@ -69,15 +69,15 @@ struct Carver {
   }
 };
 
-// The long-prefix path: bf16 states, one image per prompt, at least one full
-// 128-row tile of visual tokens, a rank that keeps the split states' rows
-// 16-byte aligned, a device map.
+// The long-prefix path: bf16 states, one image per prompt, at least 256 visual
+// tokens (a full 128 x 256 tile of the support cosines), a rank that keeps the
+// split states' rows 16-byte aligned, a device map.
 int check_long_prefix(const gmc_problem* prob, const gmc_long_prefix* lp) {
   if (!lp->rademacher || ((uintptr_t)lp->rademacher % 16) != 0 || lp->rank < 8 ||
       lp->rank % 8 != 0 || lp->max_clients < 1)
     return GMC_ERR_ARG;
   if (lp->rank > GMC_MAX_RANK || prob->dtype != GMC_BF16 || (prob->images > 1) ||
-      prob->grid_h * prob->grid_w < 128)
+      prob->grid_h * prob->grid_w < 256)
     return GMC_ERR_UNSUPPORTED;
   return GMC_OK;
 }
@@ -123,7 +123,7 @@ struct LongScratch {
   float* app;           // [B][MV][N]  projected cosines of the appearance clients
   __nv_bfloat16* Hs;    // [B][K][D]   selected visual rows
   float* rnS;           // [B][K]      their reciprocal norms
-  float* cs;            // [B][N][K]   support cosines
+  float* cs;            // [B][K][N]   support cosines (row k: every token against S_k)
   WideState w;
 };
 
@@ -156,7 +156,7 @@ size_t carve_compress(const Dims& dm, Scratch* s, char* base, R0State* r0s = nul
   const size_t B = dm.B, N = dm.N, H = dm.H, T = dm.T, M = dm.M, K = dm.K;
   t.nP = ceil_div(dm.N, PROBE_TOK);
   t.nHG = ceil_div(dm.N, HG_TOK);
-  t.nA = ceil_div(dm.N, ASSIGN_WARPS);
+  t.nA = assign_blocks(dm.N);
   t.nE = t.nA;  // energy block sums come from the assignment gap kernel
   t.nSel = 0;
   const size_t V = dm.V;
@@ -652,18 +652,20 @@ static int compress_impl(const gmc_problem* prob, const gmc_params* params,
       GMC_TRY(launch_certificate(dm.B, N, Ke, tv, st));
       g_launches += 1;
     }
-    // the N x K support cosines of the assignment (Eq. (cond-assignment))
+    // the support cosines of the assignment (Eq. (cond-assignment)), K x N:
+    // row k holds the cosines of every token with the k-th selected one
     auto support_cos = [&]() -> cudaError_t {
       cudaError_t e = launch_gather_support(dm, hidden, s.support, s.rn, ls.Hs, ls.rnS, s.status, st);
       if (e != cudaSuccess) return e;
       GemmArgs g{};
-      g.B = dm.B; g.M = N; g.Nn = Ke; g.Kd = D;
-      g.a_img = N; g.b_img = Ke; g.a_text = 1; g.b_text = 0;
+      g.B = dm.B; g.M = Ke; g.Nn = N; g.Kd = D;
+      g.a_img = Ke; g.b_img = N; g.a_text = 0; g.b_text = 1;
       g.toff = dm.toff; g.Tmax = T;
-      g.rscale = s.rn; g.cscale = ls.rnS;
-      g.C = ls.cs; g.c_img = (long long)N * Ke; g.ldc = Ke;
+      g.rscale = ls.rnS; g.cscale = s.rn;
+      g.C = ls.cs; g.c_img = (long long)N * Ke; g.ldc = N;
       g.status = s.status;
-      return launch_gemm_tc(g, hidden, (long long)dm.B * (N + T), D, ls.Hs, (long long)dm.B * Ke,
+      g.m_fast = 1;  // the hidden rows (B) are the large operand
+      return launch_gemm_tc(g, ls.Hs, (long long)dm.B * Ke, D, hidden, (long long)dm.B * (N + T),
                             D, st);
     };
     GMC_STAGE("support_cos", 2, support_cos());

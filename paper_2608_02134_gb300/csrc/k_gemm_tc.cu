@@ -7,9 +7,9 @@
 //   * the bounded appearance bank's cosines x~_{c(m)} . x~_i over the projected
 //     unit states (A, B = the states split into bf16 hi/lo terms, laid out so
 //     one product over 3r columns sums hi.hi + hi.lo + lo.hi);
-//   * the N x K support cosines of the assignment, cos(h_i, h_{S_k}) (A =
-//     visual hidden rows, B = the selected rows gathered, scaled by the
-//     reciprocal norms of both).
+//   * the support cosines of the assignment, cos(h_{S_k}, h_i), as K x N rows
+//     (A = the selected rows gathered, B = the visual hidden rows, scaled by
+//     the reciprocal norms of both).
 //   * the cosine Gram of the boundary states for large or batched problems
 //     (symmetric mode: A = B = the visual rows, scaled by their reciprocal
 //     norms; only tiles on or above the diagonal are computed).
@@ -89,7 +89,9 @@ __global__ void __launch_bounds__(G_THREADS, 1)
   float* cs = rs + GM;                            // [BN] column scales
 
   const int b = blockIdx.z;
-  int tI = blockIdx.y, tJ = blockIdx.x;
+  // consecutive CTAs share a B tile (m_fast: the larger operand is B and stays
+  // in L2 while the A tiles stream past it) or an A tile
+  int tI = g.m_fast ? blockIdx.x : blockIdx.y, tJ = g.m_fast ? blockIdx.y : blockIdx.x;
   if (g.sym) {  // blockIdx.x enumerates the computed tiles, row block by row block
     const int nJ = ceil_div(g.Nn, BN);
     int t = blockIdx.x;
@@ -259,6 +261,7 @@ static cudaError_t launch_gemm_bn(const GemmArgs& g, const void* A, long long a_
   const size_t smem = gemm_smem<BN>();
   if ((e = set_smem_limit((const void*)k_gemm_tc<BN>, smem)) != cudaSuccess) return e;
   dim3 grid(ceil_div(g.Nn, BN), ceil_div(g.M, GM), g.B);
+  if (g.m_fast) grid = dim3(ceil_div(g.M, GM), ceil_div(g.Nn, BN), g.B);
   if (g.sym) grid = dim3(gemm_sym_ctas(g.M, 1), 1, g.B);  // the computed tiles of every image
   launch_k(k_gemm_tc<BN>, grid, G_THREADS, smem, st, 1, am, bm, g);
   return cudaGetLastError();
@@ -273,7 +276,7 @@ int gemm_sym_ctas(int N, int B) {  // symmetric Grams use 128 x 256 tiles (N > 1
 cudaError_t launch_gemm_tc(const GemmArgs& g, const void* A, long long a_rows, int lda,
                            const void* Bm, long long b_rows, int ldb, cudaStream_t st) {
   if (g.M < 1 || g.Nn < 1 || g.Kd < 1 || g.B < 1) return cudaErrorInvalidValue;
-  if (g.sym && (g.M != g.Nn || g.Nn <= 128)) return cudaErrorInvalidValue;
+  if (g.sym && (g.M != g.Nn || g.Nn <= 128 || g.m_fast)) return cudaErrorInvalidValue;
   // an operand addressed from the hidden states (a_text / b_text) must hold a
   // full box of rows, so the shifted last box stays inside the image's visual
   // rows (the buffer may end right after the last image's text rows)

@@ -71,7 +71,7 @@ __global__ void __launch_bounds__(512) k_r0_pool(const long long* __restrict__ u
     if (threadIdx.x == 0) info[b * INFO_W] = 0;
     return;
   }
-  sel::PoolScratch w;
+  sel::PoolScratch w{};  // gains in shared memory: no boundary staging
   char* p = sm_r0p;
   long long* ug = reinterpret_cast<long long*>(p);  p += sizeof(long long) * (size_t)N;
   w.hist = reinterpret_cast<int*>(p);       p += sizeof(int) * sel::HBINS;
@@ -345,7 +345,7 @@ __global__ void __launch_bounds__(512) k_rg_pool(const long long* __restrict__ u
     if (threadIdx.x == 0) info[b * INFO_W] = 0;
     return;
   }
-  sel::PoolScratch w;
+  sel::PoolScratch w{};  // gains in shared memory: no boundary staging
   char* p = sm_rgp;
   long long* ug = reinterpret_cast<long long*>(p);  p += sizeof(long long) * (size_t)N;
   w.hist = reinterpret_cast<int*>(p);       p += sizeof(int) * sel::HBINS;

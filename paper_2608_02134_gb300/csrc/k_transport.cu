@@ -25,6 +25,7 @@ constexpr int TR_THREADS = 128;  // threads per CTA
 constexpr int TR_WIN = 16;       // assignments per thread in one membership window
 constexpr int TR_MAXS = 8;       // CTAs per output row (portable cluster size)
 constexpr int TR_KVS = 2;        // K/V 16-B units per thread and row staged asynchronously
+constexpr int TR_FW = 4;         // bitmap words per thread of the single-pass membership scan
 
 // Raw 8-element slices of a row, kept in registers while more member rows are
 // in flight (a cluster can hold dozens of members: each batch is one memory
@@ -93,7 +94,11 @@ inline int transport_split(int D) {
 // assignment kernel wrote one (mbits != nullptr), else built by ballots over
 // the assignment (token base + u * TR_THREADS + tid read by thread tid,
 // coalesced).  The masks' counts, scanned in token order, place every member
-// in ascending source order.
+// in ascending source order.  With a bitmap of at most TR_FW words per
+// thread (N <= 16384), every word is read at once (thread t: words TR_FW t ..)
+// and one scan places all members when they fit one window: long prefixes
+// have thousands of carriers with a few members each, and the windows'
+// barriers would dominate.
 template <typename Tin>
 __global__ void __launch_bounds__(TR_THREADS, 7) k_transport(
     const Tin* __restrict__ hidden, const Tin* __restrict__ keys, const int32_t* __restrict__ pos,
@@ -125,8 +130,18 @@ __global__ void __launch_bounds__(TR_THREADS, 7) k_transport(
   const uint32_t* bits = mbits ? mbits + ((size_t)b * K + r) * nwd : nullptr;
   int pw[TR_WIN];
   uint32_t bw = 0;
+  const bool single = bits && nwd <= TR_FW * TR_THREADS;  // uniform over the cluster
+  uint32_t fw[TR_FW];
+#pragma unroll
+  for (int q = 0; q < TR_FW; ++q) fw[q] = 0u;
   if (car) {
-    if (bits) {
+    if (single) {
+#pragma unroll
+      for (int q = 0; q < TR_FW; ++q) {
+        const int x = TR_FW * (int)threadIdx.x + q;
+        if (x < nwd) fw[q] = bits[x];
+      }
+    } else if (bits) {
       if (threadIdx.x < NM && threadIdx.x < nwd) bw = bits[threadIdx.x];
     } else {
 #pragma unroll
@@ -241,7 +256,72 @@ __global__ void __launch_bounds__(TR_THREADS, 7) k_transport(
 #pragma unroll
   for (int q = 0; q < TR_VEC; ++q) acc[q] = 0.f;
   float Msum = 0.f;
-  for (int base = 0; base < N; base += TR_WIN * TR_THREADS) {
+  // ascending source order; ILP member rows are loaded before any is added
+  auto accumulate = [&](int total) {
+    for (int q0 = 0; q0 < total; q0 += ILP) {
+      Raw8<Tin> raw[ILP];
+      float wg[ILP];
+#pragma unroll
+      for (int u = 0; u < ILP; ++u) {
+        wg[u] = 0.f;
+        if (q0 + u < total) {
+          const int m = members[q0 + u];
+          wg[u] = mass[(size_t)b * N + m];
+          if (active) raw[u].load(hidden + sq.hidden_row(m, D) + e0);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < ILP; ++u)
+        if (q0 + u < total) {
+          Msum += wg[u];
+          if (active) {
+            float v[TR_VEC];
+            raw[u].to_f32(v);
+#pragma unroll
+            for (int t = 0; t < TR_VEC; ++t) acc[t] = fmaf(wg[u], v[t], acc[t]);
+          }
+        }
+    }
+  };
+  bool scanned = false;
+  if (single) {
+    // counts of this thread's words, a block scan in thread (= token) order
+    int c = 0;
+#pragma unroll
+    for (int q = 0; q < TR_FW; ++q) c += __popc(fw[q]);
+    int incl = c;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(FULL, incl, o);
+      if (lane >= o) incl += y;
+    }
+    if (lane == 31) cnt[w] = incl;
+    __syncthreads();
+    int before = 0, total = 0;
+#pragma unroll
+    for (int q = 0; q < NW; ++q) {
+      before += q < w ? cnt[q] : 0;
+      total += cnt[q];
+    }
+    if (total <= TR_WIN * TR_THREADS) {  // uniform over the block
+      int pos = before + incl - c;
+#pragma unroll
+      for (int q = 0; q < TR_FW; ++q) {
+        uint32_t m = fw[q];
+        const int t0 = 32 * (TR_FW * (int)threadIdx.x + q);
+        while (m) {
+          const int bit = __ffs(m) - 1;
+          members[pos++] = (uint16_t)(t0 + bit);
+          m &= m - 1u;
+        }
+      }
+      __syncthreads();
+      accumulate(total);
+      scanned = true;
+    }
+    __syncthreads();  // cnt is reused by the windows
+  }
+  for (int base = 0; base < (scanned ? 0 : N); base += TR_WIN * TR_THREADS) {
     // mask x of the window covers tokens base + 32 x .. base + 32 x + 31
     if (bits) {
       if (threadIdx.x < NM) {
@@ -298,31 +378,7 @@ __global__ void __launch_bounds__(TR_THREADS, 7) k_transport(
     }
     const int total = cnt[TR_WIN * NW];
     __syncthreads();
-    // ascending source order; ILP member rows are loaded before any is added
-    for (int q0 = 0; q0 < total; q0 += ILP) {
-      Raw8<Tin> raw[ILP];
-      float wg[ILP];
-#pragma unroll
-      for (int u = 0; u < ILP; ++u) {
-        wg[u] = 0.f;
-        if (q0 + u < total) {
-          const int m = members[q0 + u];
-          wg[u] = mass[(size_t)b * N + m];
-          if (active) raw[u].load(hidden + sq.hidden_row(m, D) + e0);
-        }
-      }
-#pragma unroll
-      for (int u = 0; u < ILP; ++u)
-        if (q0 + u < total) {
-          Msum += wg[u];
-          if (active) {
-            float v[TR_VEC];
-            raw[u].to_f32(v);
-#pragma unroll
-            for (int t = 0; t < TR_VEC; ++t) acc[t] = fmaf(wg[u], v[t], acc[t]);
-          }
-        }
-    }
+    accumulate(total);
     __syncthreads();  // members and cnt are refilled by the next window
   }
   const float invM = 1.f / Msum;

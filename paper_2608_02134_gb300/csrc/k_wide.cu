@@ -33,6 +33,8 @@
 // launched; a round whose pool is empty, or that starts with the budget met,
 // does nothing.  k_w_final then fills the budget in ascending order if needed,
 // writes the ascending support and the diagnostics.
+#include <algorithm>
+
 #include "common.cuh"
 #include "kernels.cuh"
 #include "select_common.cuh"
@@ -40,8 +42,11 @@
 namespace gmc {
 
 namespace {
-constexpr int WROWS = 8;      // warps (client rows) per responsibility / filter block
+constexpr int WROWS = 8;      // warps (client rows) per responsibility block
+constexpr int FROWS = 16;     // warps per filter block (one block per SM: the next gains of
+                              // N tokens take 8 N bytes of shared memory)
 constexpr int WP_THREADS = 1024;
+constexpr int W_BCAP = 4096;  // boundary-bucket gains the pool kernel stages in shared memory
 
 // Rows of image b: grounded [0, MG), appearance [MG, MG + MV), spatial after;
 // 0 rows for an image whose text offsets are invalid.
@@ -115,7 +120,10 @@ __global__ void __launch_bounds__(WP_THREADS) k_w_pool(WideState w, WideGeom g, 
   int* pool = reinterpret_cast<int*>(p);     p += sizeof(int) * (size_t)P;
   ps.key = reinterpret_cast<short*>(p);      p += sizeof(short) * (size_t)N;
   ps.pk = reinterpret_cast<unsigned char*>(p); p += (size_t)N;
-  unsigned char* selz = reinterpret_cast<unsigned char*>(p);
+  unsigned char* selz = reinterpret_cast<unsigned char*>(p); p += (size_t)N;
+  p = reinterpret_cast<char*>((reinterpret_cast<uintptr_t>(p) + 15) & ~static_cast<uintptr_t>(15));
+  ps.bval = reinterpret_cast<long long*>(p);  // the boundary bucket's gains
+  ps.bcap = min(N, W_BCAP);
   for (int j = threadIdx.x; j < N; j += blockDim.x) {
     selz[j] = 0;
     if (tv.base) tv.gains(b, rd, N)[j] = ucur[j];
@@ -257,6 +265,47 @@ __global__ void __launch_bounds__(WP_THREADS) k_w_batch(WideState w, WideGeom g,
   const int nb = min(bsz, min(Pt, K - S));
   long long* ks = reinterpret_cast<long long*>(sm_wb);   // [NP] scores
   int* kj = reinterpret_cast<int*>(ks + NP);             // [NP] tokens
+  // The batch is the top nb of the pool by (score desc, token asc): the
+  // histogram selection over the pool slots with the tokens as tie-breakers.
+  // Scores of zero are no candidates there; if fewer than nb are positive,
+  // the bitonic sort below orders the whole pool instead.
+  {
+    char* p = reinterpret_cast<char*>(kj + NP);
+    sel::PoolScratch ps{};
+    ps.hist = reinterpret_cast<int*>(p);       p += sizeof(int) * sel::HBINS;
+    ps.bnd = reinterpret_cast<int*>(p);        p += sizeof(int) * (size_t)NP;
+    ps.wsum = reinterpret_cast<int*>(p);       p += sizeof(int) * 32;
+    ps.scal = reinterpret_cast<int*>(p);       p += sizeof(int) * 8;
+    ps.coarse = reinterpret_cast<int*>(p);     p += sizeof(int) * sel::CBINS;
+    int* top = reinterpret_cast<int*>(p);      p += sizeof(int) * (size_t)NP;
+    ps.key = reinterpret_cast<short*>(p);      p += sizeof(short) * (size_t)NP;
+    ps.pk = reinterpret_cast<unsigned char*>(p); p += (size_t)NP;
+    unsigned char* none = reinterpret_cast<unsigned char*>(p);
+    for (int k = threadIdx.x; k < Pt; k += blockDim.x) {
+      ks[k] = w.sc[(size_t)b * P + k];
+      kj[k] = w.pool[(size_t)b * P + k];
+      none[k] = 0;
+    }
+    for (int h = threadIdx.x; h < sel::HBINS; h += blockDim.x) ps.hist[h] = 0;
+    if (threadIdx.x < sel::CBINS) ps.coarse[threadIdx.x] = 0;
+    __syncthreads();
+    const int got = sel::select_pool(ks, none, Pt, nb, ps, top, nullptr, kj);
+    if (got == nb) {  // uniform over the block
+      for (int q = threadIdx.x; q < nb; q += blockDim.x) {
+        const int j = kj[top[q]];
+        w.batch[(size_t)b * P + q] = j;
+        w.stamp[(size_t)b * g.N + j] = rd + 1;
+        order[(size_t)b * K + S + q] = j;
+      }
+      if (threadIdx.x == 0) {
+        info[1] = S + nb;
+        info[2] = rd + 1;
+        if (tv.base) tv.at<int32_t>(b, tv.off_round_end)[rd] = S + nb;
+      }
+      return;
+    }
+    __syncthreads();
+  }
   for (int k = threadIdx.x; k < NP; k += blockDim.x) {
     const bool in = k < Pt;
     ks[k] = in ? w.sc[(size_t)b * P + k] : -1;  // padding sorts after every pool entry
@@ -296,7 +345,7 @@ __global__ void __launch_bounds__(WP_THREADS) k_w_batch(WideState w, WideGeom g,
 
 // ---- coverage update, survivor compaction, next gains ---------------------------------
 template <bool DENSE>
-__global__ void __launch_bounds__(32 * WROWS) k_w_filter(WideState w, WideGeom g, int P, int rnd,
+__global__ void __launch_bounds__(32 * FROWS) k_w_filter(WideState w, WideGeom g, int P, int rnd,
                                                          float* C, uint16_t* scol, int fx_exp,
                                                          const int32_t* fexp, int rpw,
                                                          TraceView tv) {
@@ -308,7 +357,7 @@ __global__ void __launch_bounds__(32 * WROWS) k_w_filter(WideState w, WideGeom g
   if (Pt == 0) return;
   int MG;
   const int Mb = wide_rows(g, b, &MG);
-  const int m0 = blockIdx.x * WROWS * rpw;
+  const int m0 = blockIdx.x * FROWS * rpw;
   if (m0 >= Mb) return;
   const int S = info[3], rd = info[4];
   const int nb = info[1] - S;  // the batch kernel has run: info[1] = S + nb
@@ -323,7 +372,7 @@ __global__ void __launch_bounds__(32 * WROWS) k_w_filter(WideState w, WideGeom g
   const int lane = threadIdx.x & 31;
   const unsigned lt = sel::lanemask_lt();
   for (int ir = 0; ir < rpw; ++ir) {
-    const int m = m0 + (threadIdx.x >> 5) + WROWS * ir;
+    const int m = m0 + (threadIdx.x >> 5) + FROWS * ir;
     if (m >= Mb) break;
     const size_t row = (size_t)b * g.Mstride + m;
     float* vals = C + row * N;
@@ -336,6 +385,50 @@ __global__ void __launch_bounds__(32 * WROWS) k_w_filter(WideState w, WideGeom g
       bnew = warp_max(bnew);
       const long long fb_new = to_fix(bnew, fxs);
       float rowmax = 0.f;
+      if ((N & 3) == 0) {
+        // 8 x 16 bytes per lane in flight; all loads of a step issued before
+        // any survivor is written back in place (survivors land below the
+        // step's end).  Lane l's float4 holds tokens 4 k4 .. 4 k4 + 3, so the
+        // survivors are written lane by lane: ascending token order.
+        const float4* row4 = reinterpret_cast<const float4*>(vals);
+        const int n4 = N >> 2;
+        for (int b4 = 0; b4 < n4; b4 += 32 * 8) {
+          float4 buf[8];
+#pragma unroll
+          for (int u = 0; u < 8; ++u) {
+            const int k4 = b4 + u * 32 + lane;
+            buf[u] = k4 < n4 ? row4[k4] : make_float4(0.f, 0.f, 0.f, 0.f);
+          }
+          __syncwarp();
+#pragma unroll
+          for (int u = 0; u < 8; ++u) {
+            const int k4 = b4 + u * 32 + lane;
+            const float c4[4] = {buf[u].x, buf[u].y, buf[u].z, buf[u].w};
+            int pre = 0, tot = 0;
+#pragma unroll
+            for (int e2 = 0; e2 < 4; ++e2) {
+              rowmax = fmaxf(rowmax, c4[e2]);
+              const unsigned bal = __ballot_sync(FULL, k4 < n4 && c4[e2] > bnew);
+              pre += __popc(bal & lt);
+              tot += __popc(bal);
+            }
+            int pos = wr + pre;
+            if (k4 < n4) {
+#pragma unroll
+              for (int e2 = 0; e2 < 4; ++e2)
+                if (c4[e2] > bnew) {
+                  const int k = 4 * k4 + e2;
+                  vals[pos] = c4[e2];
+                  cols[pos] = (uint16_t)k;
+                  atomicAdd(&uacc[k], (unsigned long long)(to_fix(c4[e2], fxs) - fb_new));
+                  ++pos;
+                }
+            }
+            wr += tot;
+          }
+          __syncwarp();
+        }
+      } else
       // 8 loads per lane in flight; all loads of a step issued before any
       // survivor is written back in place (survivors land below the step's end)
       for (int base = 0; base < N; base += 32 * 8) {
@@ -525,10 +618,13 @@ cudaError_t launch_wide_select(const WideState& w, const WideGeom& g, const gmc_
   int NP = 1;
   while (NP < P) NP <<= 1;
   const size_t psm = sizeof(int) * (sel::HBINS + (size_t)N + 32 + 8 + sel::CBINS + P) +
-                     sizeof(short) * (size_t)N + 2 * (size_t)N + 64;
+                     sizeof(short) * (size_t)N + 2 * (size_t)N + 16 +
+                     sizeof(long long) * (size_t)std::min(N, W_BCAP) + 64;
   const size_t rsm_dense = sizeof(long long) * (size_t)P + sizeof(float) * (size_t)WROWS * P;
   const size_t rsm_sparse = sizeof(long long) * (size_t)P + sizeof(short) * (size_t)N;
-  const size_t bsm = (sizeof(long long) + sizeof(int)) * (size_t)NP;
+  const size_t bsm = (sizeof(long long) + sizeof(int)) * (size_t)NP +
+                     sizeof(int) * (sel::HBINS + 2 * (size_t)NP + 32 + 8 + sel::CBINS) +
+                     sizeof(short) * (size_t)NP + 2 * (size_t)NP + 64;
   const size_t fsm = sizeof(unsigned long long) * (size_t)N;
   if ((e = set_smem_limit((const void*)k_w_pool, psm)) != cudaSuccess) return e;
   if ((e = set_smem_limit((const void*)k_w_rho<true>, rsm_dense)) != cudaSuccess) return e;
@@ -537,10 +633,10 @@ cudaError_t launch_wide_select(const WideState& w, const WideGeom& g, const gmc_
   if ((e = set_smem_limit((const void*)k_w_filter<true>, fsm)) != cudaSuccess) return e;
   if ((e = set_smem_limit((const void*)k_w_filter<false>, fsm)) != cudaSuccess) return e;
   // filters: one row per warp while the blocks fit on the GPU at once, four beyond
-  const long long fblocks = (long long)g.B * ceil_div(g.Mstride, WROWS);
-  const int rpw = fblocks > 8LL * sms ? 4 : 1;
+  const long long fblocks = (long long)g.B * ceil_div(g.Mstride, FROWS);
+  const int rpw = fblocks > 4LL * sms ? 4 : 1;
   const dim3 rgrid(ceil_div(g.Mstride, WROWS), g.B);
-  const dim3 fgrid(ceil_div(g.Mstride, WROWS * rpw), g.B);
+  const dim3 fgrid(ceil_div(g.Mstride, FROWS * rpw), g.B);
   const int R = wide_rounds(g.K, p);
   for (int rnd = 0; rnd < R; ++rnd) {
     launch_k(k_w_pool, g.B, WP_THREADS, psm, st, 1, w, g, P, rnd, u0, (const int32_t*)order, tv);
@@ -555,10 +651,10 @@ cudaError_t launch_wide_select(const WideState& w, const WideGeom& g, const gmc_
     launch_k(k_w_batch, g.B, WP_THREADS, bsm, st, 1, w, g, P, NP, p.batch_b, order, tv);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     if (rnd == 0)
-      launch_k(k_w_filter<true>, fgrid, 32 * WROWS, fsm, st, 1, w, g, P, rnd, C, scol, fx_exp,
+      launch_k(k_w_filter<true>, fgrid, 32 * FROWS, fsm, st, 1, w, g, P, rnd, C, scol, fx_exp,
                fexp, rpw, tv);
     else
-      launch_k(k_w_filter<false>, fgrid, 32 * WROWS, fsm, st, 1, w, g, P, rnd, C, scol, fx_exp,
+      launch_k(k_w_filter<false>, fgrid, 32 * FROWS, fsm, st, 1, w, g, P, rnd, C, scol, fx_exp,
                fexp, rpw, tv);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }

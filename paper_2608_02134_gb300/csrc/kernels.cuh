@@ -130,7 +130,8 @@ struct Scratch {
 
 constexpr int ROWS_PER_BLOCK = 8;  // rownorm / probe / client builder blocks
 constexpr int HG_TOK = 8;          // tokens per head-statistics block
-constexpr int ASSIGN_WARPS = 8;    // tokens per assignment block
+constexpr int ASSIGN_WARPS = 16;   // warps per assignment block (32 tokens, one per lane)
+int assign_blocks(int N);          // assignment blocks per image
 constexpr int PROBE_TOK = 32;       // tokens per probe block
 
 // Launch wrappers.  Each returns the first CUDA error it saw.
@@ -297,6 +298,7 @@ struct GemmArgs {
   uint32_t* status;
   int sym;                   // 1: C symmetric (A, B the same rows, M == Nn > 128): tiles on
                              // or above the diagonal computed, the rest mirrored
+  int m_fast;                // 1: consecutive CTAs walk the row tiles (B is the larger operand)
 };
 int gemm_sym_ctas(int N, int B);  // CTAs of the symmetric mode for N x N Grams of B images
 // a_rows / b_rows: rows declared in the operand's tensor map (reads past them

@@ -65,6 +65,9 @@ struct PoolScratch {
   unsigned char* pk;   // [N]  boundary tokens that enter the pool
   int* wsum;           // [32]
   int* scal;           // [8]
+  long long* bval;     // optional [bcap]: the boundary bucket's gains, staged when the
+                       // gains are in global memory (nullptr: read them in place)
+  int bcap;
 };
 
 // Warp-aggregated append: every lane with `want` gets a distinct index from
@@ -106,9 +109,12 @@ __device__ __forceinline__ int group_rank_of(const int* a, int n, int x, int gl,
 // and one scan of the per-warp counts places them: no shared counter,
 // nothing that depends on thread scheduling.  Tokens inside the boundary
 // bucket are ranked exactly by (u desc, index asc).
+// ids (optional): ties are broken by the lower ids[j] instead of the lower j
+// (the batch kernel ranks pool slots by (score desc, token asc)).
 // Every thread of the block must call it; blockDim is a multiple of 32.
 __device__ inline int select_pool(const long long* u, const unsigned char* sel, int N, int P,
-                                  PoolScratch w, int* pool, short* poolslot) {
+                                  PoolScratch w, int* pool, short* poolslot,
+                                  const int* ids = nullptr) {
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
   const int nc = (N + 32 * nw - 1) / (32 * nw);  // chunks per warp
   const unsigned lt = lanemask_lt();
@@ -223,24 +229,48 @@ __device__ inline int select_pool(const long long* u, const unsigned char* sel, 
     // 4. the boundary bucket's tokens that enter, ranked exactly by (u desc,
     //    index asc); they take the slots after the tokens above, by index
     const int need = Pt - above;
+    const bool staged = w.bval && nb <= w.bcap;  // uniform over the block
+    if (staged) {
+      for (int q = threadIdx.x; q < nb; q += blockDim.x) w.bval[q] = u[w.bnd[q]];
+      __syncthreads();
+    }
     for (int q = threadIdx.x; q < nb; q += blockDim.x) {
       const int j = w.bnd[q];
-      const long long v = u[j];
+      const long long v = staged ? w.bval[q] : u[j];
+      const int id = ids ? ids[j] : j;
       int rank = 0;
       for (int q2 = 0; q2 < nb; ++q2) {
         const int j2 = w.bnd[q2];
-        rank += key_before(u[j2], j2, v, j);
+        rank += key_before(staged ? w.bval[q2] : u[j2], ids ? ids[j2] : j2, v, id);
       }
       w.pk[q] = rank < need;
     }
     __syncthreads();
-    for (int q = threadIdx.x; q < nb; q += blockDim.x) {
-      if (!w.pk[q]) continue;
-      int before = 0;
-      for (int q2 = 0; q2 < q; ++q2) before += w.pk[q2];
-      const int j = w.bnd[q];
-      pool[above + before] = j;
-      if (poolslot) poolslot[j] = (short)(above + before);
+    // slots in index order: each entering token counts the entering ones
+    // before it (a small bucket), or a block scan of the entering flags over
+    // contiguous ranges (a large one: its barriers cost less than the counts)
+    if (nb <= 256) {
+      for (int q = threadIdx.x; q < nb; q += blockDim.x) {
+        if (!w.pk[q]) continue;
+        int before = 0;
+        for (int q2 = 0; q2 < q; ++q2) before += w.pk[q2];
+        const int j = w.bnd[q];
+        pool[above + before] = j;
+        if (poolslot) poolslot[j] = (short)(above + before);
+      }
+    } else {
+      const int per = (nb + (int)blockDim.x - 1) / (int)blockDim.x;
+      const int q0 = min(nb, (int)threadIdx.x * per), q1 = min(nb, q0 + per);
+      int c = 0;
+      for (int q = q0; q < q1; ++q) c += w.pk[q];
+      int before = block_exclusive_scan(c, w.wsum, nullptr);
+      for (int q = q0; q < q1; ++q) {
+        if (!w.pk[q]) continue;
+        const int j = w.bnd[q];
+        pool[above + before] = j;
+        if (poolslot) poolslot[j] = (short)(above + before);
+        ++before;
+      }
     }
   }
   __syncthreads();

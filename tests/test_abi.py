@@ -140,7 +140,7 @@ def _long_rc(gmc, prob, lp, params=None, ws_bytes=1 << 40, **shape):
 
 
 def test_long_prefix_sizing_and_validation(gmc):
-    """gmc_compress_long: the bounded bank's limits (bf16, one image, N >= 128,
+    """gmc_compress_long: the bounded bank's limits (bf16, one image, N >= 256,
     rank a multiple of 8 up to GMC_MAX_RANK, N up to GMC_MAX_N_LONG, pools up
     to GMC_MAX_POOL_WIDE)."""
     assert ctypes.sizeof(gmc.LongPrefix) == 16
@@ -171,7 +171,9 @@ def test_long_prefix_sizing_and_validation(gmc):
     assert _long_rc(gmc, gmc.problem(1, 40, 40, 2, gmc.GMC_F32), lps, ctypes.byref(p64)) == \
         gmc.GMC_ERR_UNSUPPORTED                                             # bf16 only
     assert _long_rc(gmc, gmc.problem(1, 8, 8, 2, gmc.GMC_BF16), lps, ctypes.byref(p64),
-                    N=64) == gmc.GMC_ERR_UNSUPPORTED                        # N < 128
+                    N=64) == gmc.GMC_ERR_UNSUPPORTED                        # N < 256
+    assert _long_rc(gmc, gmc.problem(1, 12, 20, 2, gmc.GMC_BF16), lps, ctypes.byref(p64),
+                    N=240) == gmc.GMC_ERR_UNSUPPORTED
     assert _long_rc(gmc, gmc.problem(1, 40, 40, 2, gmc.GMC_BF16, images=2), lps,
                     ctypes.byref(p64), N=3200) == gmc.GMC_ERR_UNSUPPORTED   # one image
     assert _long_rc(gmc, gmc.problem(1, 130, 130, 2, gmc.GMC_BF16), lps, ctypes.byref(p64),
