@@ -133,7 +133,7 @@ __global__ void __launch_bounds__(WP_THREADS) k_w_pool(WideState w, WideGeom g, 
   __syncthreads();
   for (int q = threadIdx.x; q < S; q += blockDim.x) selz[order[(size_t)b * K + q]] = 1;
   __syncthreads();
-  const int Pt = sel::select_pool(ucur, selz, N, P, ps, pool, nullptr);
+  const int Pt = sel::select_pool<true>(ucur, selz, N, P, ps, pool, nullptr);
   for (int k = threadIdx.x; k < P; k += blockDim.x) w.pool[(size_t)b * P + k] = k < Pt ? pool[k] : -1;
   if (threadIdx.x == 0) {
     info[0] = Pt;
@@ -289,7 +289,7 @@ __global__ void __launch_bounds__(WP_THREADS) k_w_batch(WideState w, WideGeom g,
     for (int h = threadIdx.x; h < sel::HBINS; h += blockDim.x) ps.hist[h] = 0;
     if (threadIdx.x < sel::CBINS) ps.coarse[threadIdx.x] = 0;
     __syncthreads();
-    const int got = sel::select_pool(ks, none, Pt, nb, ps, top, nullptr, kj);
+    const int got = sel::select_pool<true>(ks, none, Pt, nb, ps, top, nullptr, kj);
     if (got == nb) {  // uniform over the block
       for (int q = threadIdx.x; q < nb; q += blockDim.x) {
         const int j = kj[top[q]];

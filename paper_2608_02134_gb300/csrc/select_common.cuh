@@ -25,6 +25,11 @@ __device__ __forceinline__ int gain_bucket(long long u) {
   const unsigned long long top = (unsigned long long)u << lz;     // leading one at bit 63
   return (63 - lz) * 32 + (int)((top >> 58) & 31);
 }
+// The next 11 mantissa bits: within one bucket, monotone in the gain.
+__device__ __forceinline__ int gain_subbucket(long long u) {
+  const unsigned long long top = (unsigned long long)u << __clzll(u);
+  return (int)((top >> 47) & 2047);
+}
 
 // Block-wide exclusive scan of one int per thread (deterministic).  Every
 // thread of the block must call it.
@@ -110,8 +115,11 @@ __device__ __forceinline__ int group_rank_of(const int* a, int n, int x, int gl,
 // nothing that depends on thread scheduling.  Tokens inside the boundary
 // bucket are ranked exactly by (u desc, index asc).
 // ids (optional): ties are broken by the lower ids[j] instead of the lower j
-// (the batch kernel ranks pool slots by (score desc, token asc)).
+// (the batch kernel ranks pool slots by (score desc, token asc)).  REFINE
+// (the wide solver's long prefixes) splits a large boundary bucket once more
+// (below); the standard solvers leave it out, it costs them registers.
 // Every thread of the block must call it; blockDim is a multiple of 32.
+template <bool REFINE = false>
 __device__ inline int select_pool(const long long* u, const unsigned char* sel, int N, int P,
                                   PoolScratch w, int* pool, short* poolslot,
                                   const int* ids = nullptr) {
@@ -228,24 +236,75 @@ __device__ inline int select_pool(const long long* u, const unsigned char* sel, 
     __syncthreads();
     // 4. the boundary bucket's tokens that enter, ranked exactly by (u desc,
     //    index asc); they take the slots after the tokens above, by index
-    const int need = Pt - above;
+    int need = Pt - above;
     const bool staged = w.bval && nb <= w.bcap;  // uniform over the block
     if (staged) {
       for (int q = threadIdx.x; q < nb; q += blockDim.x) w.bval[q] = u[w.bnd[q]];
       __syncthreads();
     }
+    // A large bucket (near-equal gains) is split once more by the next 11
+    // mantissa bits: the tokens of higher sub-buckets enter, those of lower
+    // ones do not, and only the boundary sub-bucket is ranked exactly.
+    // pk[q]: 1 enters, 0 does not, 2 undecided (ranked below).
+    const bool refine = REFINE && nb > 512;  // uniform over the block
+    if (refine) {
+      for (int q = threadIdx.x; q < nb; q += blockDim.x)
+        atomicAdd(&w.hist[gain_subbucket(staged ? w.bval[q] : u[w.bnd[q]])], 1);
+      __syncthreads();
+      if (wid == 0) {  // the sub-bucket holding the need-th largest: 64 bins per lane, top first
+        int cnt = 0;
+        for (int t = 0; t < 64; ++t) cnt += w.hist[2047 - (lane * 64 + t)];
+        int incl = cnt;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const int y = __shfl_up_sync(FULL, incl, o);
+          if (lane >= o) incl += y;
+        }
+        const int L = __ffs(__ballot_sync(FULL, incl >= need)) - 1;  // need <= nb: L >= 0
+        if (lane == L) {
+          int acc = incl - cnt, sb = 2047 - lane * 64;
+          for (int t = 0; t < 64; ++t, --sb) {
+            const int c = w.hist[sb];
+            if (acc + c >= need) break;
+            acc += c;
+          }
+          w.scal[0] = sb;   // boundary sub-bucket
+          w.scal[1] = acc;  // tokens in higher sub-buckets
+        }
+      }
+      __syncthreads();
+      const int sb = w.scal[0];
+      for (int q = threadIdx.x; q < nb; q += blockDim.x) {
+        const int sk = gain_subbucket(staged ? w.bval[q] : u[w.bnd[q]]);
+        w.pk[q] = sk > sb ? 1 : (sk == sb ? 2 : 0);
+      }
+      need -= w.scal[1];
+      __syncthreads();
+    }
     for (int q = threadIdx.x; q < nb; q += blockDim.x) {
+      if (refine && w.pk[q] != 2) continue;
       const int j = w.bnd[q];
       const long long v = staged ? w.bval[q] : u[j];
       const int id = ids ? ids[j] : j;
       int rank = 0;
       for (int q2 = 0; q2 < nb; ++q2) {
+        if (refine && w.pk[q2] != 2) continue;  // only the boundary sub-bucket competes
         const int j2 = w.bnd[q2];
         rank += key_before(staged ? w.bval[q2] : u[j2], ids ? ids[j2] : j2, v, id);
       }
-      w.pk[q] = rank < need;
+      // refine: pk still marks who competes, so the verdict waits in key[q]
+      // (the tokens' bucket keys are no longer read)
+      if (refine) w.key[q] = (short)(rank < need);
+      else w.pk[q] = rank < need;
     }
     __syncthreads();
+    if (refine) {  // the verdicts, and the sub-buckets cleared (every thread has read them)
+      for (int q = threadIdx.x; q < nb; q += blockDim.x) {
+        if (w.pk[q] == 2) w.pk[q] = (unsigned char)w.key[q];
+        w.hist[gain_subbucket(staged ? w.bval[q] : u[w.bnd[q]])] = 0;
+      }
+      __syncthreads();
+    }
     // slots in index order: each entering token counts the entering ones
     // before it (a small bucket), or a block scan of the entering flags over
     // contiguous ranges (a large one: its barriers cost less than the counts)
