@@ -24,6 +24,12 @@
 // The column sums u0_i = sum_m Cbar_mi (the singleton gains of the empty
 // support) are accumulated in 64-bit fixed point, so they are exact sums of
 // the fp32 entries and independent of the order the blocks finish in.
+// A block's eight rows are nearly always of one kind -- eight consecutive
+// queries of one head (which share the factor sqrt(||Z_h[i]||^2 + sigma_h^2)
+// of every column), eight consecutive appearance rows, or eight landmarks:
+// those blocks keep their rows' constants in registers and compute the
+// shared factor once per column; a mixed block takes the generic loop.  Both
+// evaluate the same expressions, so the entries are the same.
 #include "common.cuh"
 #include "kernels.cuh"
 
@@ -148,9 +154,103 @@ __global__ void __launch_bounds__(256, 4) k_build_clients(
     }
     if (lane == 0) ri[w] = inf;
   }
+  __shared__ int umode;  // 0 generic, 1 grounded (one head), 2 appearance, 3 spatial
   __syncthreads();
   const int nrows = min(ROWS_PER_BLOCK, Mb - r0);
   const float itv = 1.f / tau_v, its = 1.f / tau_s;
+  if (threadIdx.x == 0) {
+    int mode = 0;
+    if (nrows == ROWS_PER_BLOCK && !check) {
+      const RowInfo& f = ri[0];
+      bool same = true;
+      for (int q = 1; q < ROWS_PER_BLOCK; ++q) {
+        const RowInfo& g = ri[q];
+        same = same && g.kind == f.kind && g.lo == f.lo && g.hi == f.hi;
+        if (f.kind == 0) same = same && g.z == f.z && g.sg2 == f.sg2 && g.x == f.x + (size_t)q * N;
+        if (f.kind == 1) same = same && g.x == f.x + (size_t)q * N;
+      }
+      if (same && f.kind >= 0) mode = f.kind + 1;
+    }
+    umode = mode;
+  }
+  __syncthreads();
+  const int mode = umode;
+  float* Crow = C + ((size_t)b * M + r0) * N;
+  unsigned long long* ucol = reinterpret_cast<unsigned long long*>(u0 + (size_t)b * N);
+  if (mode == 1) {  // grounded rows of one head: x * sqrt(||Z_h[i]||^2 + sigma_h^2) * scale
+    const float* x0 = ri[0].x;
+    const float* zr = ri[0].z;
+    const float sg2 = ri[0].sg2;
+    float sc[ROWS_PER_BLOCK];
+#pragma unroll
+    for (int q = 0; q < ROWS_PER_BLOCK; ++q) sc[q] = ri[q].scale;
+    for (int j = threadIdx.x; j < N; j += blockDim.x) {
+      float xv[ROWS_PER_BLOCK];
+#pragma unroll
+      for (int q = 0; q < ROWS_PER_BLOCK; ++q) xv[q] = x0[(size_t)q * N + j];
+      const float g = sqrtf(zr[j] + sg2);
+      long long colsum = 0;
+#pragma unroll
+      for (int q = 0; q < ROWS_PER_BLOCK; ++q) {
+        const float v = xv[q] * g * sc[q];
+        Crow[(size_t)q * N + j] = v;
+        colsum += to_fix(v, fx_scale);
+      }
+      if (colsum) atomicAdd(ucol + j, (unsigned long long)colsum);
+    }
+    return;
+  }
+  if (mode == 2) {  // appearance rows: exp((x - row max) / tau_v) * scale on the row's image
+    const float* x0 = ri[0].x;
+    const int lo = ri[0].lo, hi = ri[0].hi;
+    float sh[ROWS_PER_BLOCK], sc[ROWS_PER_BLOCK];
+#pragma unroll
+    for (int q = 0; q < ROWS_PER_BLOCK; ++q) {
+      sh[q] = ri[q].shift;
+      sc[q] = ri[q].scale;
+    }
+    for (int j = threadIdx.x; j < N; j += blockDim.x) {
+      const bool in = j >= lo && j < hi;
+      float xv[ROWS_PER_BLOCK];
+#pragma unroll
+      for (int q = 0; q < ROWS_PER_BLOCK; ++q) xv[q] = in ? x0[(size_t)q * N + j] : 0.f;
+      long long colsum = 0;
+#pragma unroll
+      for (int q = 0; q < ROWS_PER_BLOCK; ++q) {
+        const float v = in ? expf((xv[q] - sh[q]) * itv) * sc[q] : 0.f;
+        Crow[(size_t)q * N + j] = v;
+        colsum += to_fix(v, fx_scale);
+      }
+      if (colsum) atomicAdd(ucol + j, (unsigned long long)colsum);
+    }
+    return;
+  }
+  if (mode == 3) {  // landmark rows: exp((smallest d^2 - ||p_i - l||^2) / tau_s) * scale
+    const int lo = ri[0].lo, hi = ri[0].hi;
+    float sh[ROWS_PER_BLOCK], sc[ROWS_PER_BLOCK], ly[ROWS_PER_BLOCK], lx[ROWS_PER_BLOCK];
+#pragma unroll
+    for (int q = 0; q < ROWS_PER_BLOCK; ++q) {
+      sh[q] = ri[q].shift;
+      sc[q] = ri[q].scale;
+      ly[q] = ri[q].ly;
+      lx[q] = ri[q].lx;
+    }
+    for (int j = threadIdx.x; j < N; j += blockDim.x) {
+      const bool in = j >= lo && j < hi;
+      const int jl = j % Ng, jr = jl / gw;  // position in its own image's grid
+      const float py = (jr + 0.5f) / gh, px = ((jl - jr * gw) + 0.5f) / gw;
+      long long colsum = 0;
+#pragma unroll
+      for (int q = 0; q < ROWS_PER_BLOCK; ++q) {
+        const float dy = py - ly[q], dx = px - lx[q];
+        const float v = in ? expf((sh[q] - (dy * dy + dx * dx)) * its) * sc[q] : 0.f;
+        Crow[(size_t)q * N + j] = v;
+        colsum += to_fix(v, fx_scale);
+      }
+      if (colsum) atomicAdd(ucol + j, (unsigned long long)colsum);
+    }
+    return;
+  }
   for (int j = threadIdx.x; j < N; j += blockDim.x) {
     long long colsum = 0;
     const int jl = j % Ng, jr = jl / gw;  // position in its own image's grid
