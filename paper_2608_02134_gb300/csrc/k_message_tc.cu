@@ -39,7 +39,8 @@ namespace {
 constexpr int BM = 128, BK = 64, STAGES = 2;
 constexpr int SPLIT_TARGET_CTAS = 152;  // one wave of one CTA per SM on a 152-SM GB300
 constexpr int TILE_BYTES = BM * BK * 2;
-constexpr int EPI_WARPS = 8, THREADS = 32 * (EPI_WARPS + 2);
+constexpr int EPI_WARPS = 16, THREADS = 32 * (EPI_WARPS + 2);
+constexpr int EPI_PARTS = EPI_WARPS / 4;  // 32-column parts of a tile (warp w: lane quarter w % 4)
 constexpr long long WAIT_CYCLES = 4000000000LL;
 
 struct MsgCtl {
@@ -50,9 +51,9 @@ struct MsgCtl {
   uint64_t acce[2];
   uint32_t tmem;
   volatile int abort;
-  float stat_m[2][BM];
-  float stat_l[2][BM];
-  float rsum[2][BM];
+  float stat_m[EPI_PARTS][BM];
+  float stat_l[EPI_PARTS][BM];
+  float rsum[EPI_PARTS][BM];
 };
 
 // Fused kernel: 16 epilogue warps (warp w reads TMEM lanes 32*(w%4).. and the
@@ -251,7 +252,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
     __syncwarp();
   } else {  // ---------------- epilogue warps 0..7
-    const int quarter = warp & 3, half = warp >> 2;
+    const int quarter = warp & 3, cpart = warp >> 2;  // TMEM lane quarter, 32-column part
     const int r = quarter * 32 + lane;           // tile row == TMEM lane
     const int R = tile * BM + r;                 // packed row
     const bool valid = R < grp * Tb;
@@ -279,22 +280,21 @@ __global__ void __launch_bounds__(THREADS, 1)
       const int buf = it & 1, c = c0 + it;
       bool ok = tc::mbar_wait(&ctl->accf[buf], (uint32_t)(it >> 1) & 1u, deadline);
       ok = __all_sync(FULL, ok && !ctl->abort);
-      float v[64];
+      float v[32];
       if (ok) {
         tc::fence_after_sync();
-        const uint32_t ta = tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(buf * BM + half * 64);
+        const uint32_t ta = tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(buf * BM + cpart * 32);
         tc::tmem_ld32(ta, v);
-        tc::tmem_ld32(ta + 32, v + 32);
       }
       tc::fence_before_sync();
       __syncwarp();
       if (lane == 0) mbar_arrive(&ctl->acce[buf]);
       if (!ok) continue;
-      const int k0 = c * BM + half * 64;
+      const int k0 = c * BM + cpart * 32;
       if (mode == 0) {  // running max / sum over the visible keys
         float mt = -INFINITY;
 #pragma unroll
-        for (int q = 0; q < 64; ++q) {
+        for (int q = 0; q < 32; ++q) {
           v[q] *= scale;
           if (k0 + q < kvis) mt = fmaxf(mt, v[q]);
         }
@@ -302,16 +302,16 @@ __global__ void __launch_bounds__(THREADS, 1)
           const float mn = fmaxf(m, mt);
           float acc = l * expf(m - mn);
 #pragma unroll
-          for (int q = 0; q < 64; ++q)
+          for (int q = 0; q < 32; ++q)
             if (k0 + q < kvis) acc += expf(v[q] - mn);
           l = acc;
           m = mn;
         }
       } else if (valid && k0 < N) {  // normalised visual columns
-        const int nv = min(64, N - k0);
-        if (nv == 64 && (N & 3) == 0) {
+        const int nv = min(32, N - k0);
+        if (nv == 32 && (N & 3) == 0) {
 #pragma unroll
-          for (int q = 0; q < 64; q += 4) {
+          for (int q = 0; q < 32; q += 4) {
             const float4 z = *reinterpret_cast<const float4*>(zr + k0 + q);
             float4 o;
             o.x = expf(v[q] * scale - M) * invL;
@@ -325,31 +325,43 @@ __global__ void __launch_bounds__(THREADS, 1)
             rsum = fmaf(o.w, sqrtf(z.w + sg2), rsum);
           }
         } else {
-          for (int q = 0; q < nv; ++q) {
-            const float p = expf(v[q] * scale - M) * invL;
-            arow[k0 + q] = p;
-            rsum = fmaf(p, sqrtf(zr[k0 + q] + sg2), rsum);
-          }
+#pragma unroll
+          for (int q = 0; q < 32; ++q)  // unrolled: v stays in registers
+            if (q < nv) {
+              const float p = expf(v[q] * scale - M) * invL;
+              arow[k0 + q] = p;
+              rsum = fmaf(p, sqrtf(zr[k0 + q] + sg2), rsum);
+            }
         }
       }
     }
-    if (mode == 0) {  // combine the two column halves of every row
-      ctl->stat_m[half][r] = m;
-      ctl->stat_l[half][r] = l;
+    if (mode == 0) {  // combine the column parts of every row, in a fixed order
+      ctl->stat_m[cpart][r] = m;
+      ctl->stat_l[cpart][r] = l;
       epi_barrier();
-      if (half == 0 && !ctl->abort) {
-        const float mo = ctl->stat_m[1][r], lo = ctl->stat_l[1][r];
-        const float Mc = fmaxf(m, mo);
-        const float Lc = Mc > -INFINITY ? (m > -INFINITY ? l * expf(m - Mc) : 0.f) +
-                                              (mo > -INFINITY ? lo * expf(mo - Mc) : 0.f)
-                                        : 0.f;
+      if (cpart == 0 && !ctl->abort) {
+        float Mc = -INFINITY;
+#pragma unroll
+        for (int q = 0; q < EPI_PARTS; ++q) Mc = fmaxf(Mc, ctl->stat_m[q][r]);
+        float Lc = 0.f;
+        if (Mc > -INFINITY) {
+#pragma unroll
+          for (int q = 0; q < EPI_PARTS; ++q) {
+            const float mq = ctl->stat_m[q][r];
+            if (mq > -INFINITY) Lc += ctl->stat_l[q][r] * expf(mq - Mc);
+          }
+        }
         prow[split] = make_float2(Mc, Lc);
       }
     } else {
-      ctl->rsum[half][r] = rsum;
+      ctl->rsum[cpart][r] = rsum;
       epi_barrier();
-      if (half == 0 && valid && !ctl->abort)
-        rs[(((size_t)b * H + h) * nsplit + split) * Tmax + t] = rsum + ctl->rsum[1][r];
+      if (cpart == 0 && valid && !ctl->abort) {
+        float sum = 0.f;
+#pragma unroll
+        for (int q = 0; q < EPI_PARTS; ++q) sum += ctl->rsum[q][r];
+        rs[(((size_t)b * H + h) * nsplit + split) * Tmax + t] = sum;
+      }
     }
   }
   if (threadIdx.x == 0 && ctl->abort) set_status(status, GMC_STATUS_TIMEOUT);
