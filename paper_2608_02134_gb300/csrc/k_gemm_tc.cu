@@ -216,7 +216,7 @@ __global__ void __launch_bounds__(G_THREADS, 1)
       if (g.sym) {  // mirrors of owned entries j > i whose own tile is not computed
         const int i = ml + row;
         const bool own_i = i >= m0 && i < g.M;
-#pragma unroll 4
+#pragma unroll  // fully: v stays in registers
         for (int q = 0; q < 32; ++q) {
           const int j = nl + cl + q;
           if (own_i && j >= n0 && j < g.Nn && j > i && !sym_tile<BN>(j / GM, i / BN))
