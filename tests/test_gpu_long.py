@@ -235,3 +235,16 @@ def test_long_doc_full_size_sampled():
         want = p["beta_V"] / MV * e / e.sum()
         got = out[0, a0 + mrow].cpu().numpy().astype(np.float64)
         assert parity.rel_row_err(got[None], want[None]) < 1e-4, mrow
+
+
+def test_long_small_with_views_and_prefix_layers():
+    """gmc_compress_long with a historical message view and two dense prefix
+    layers: the view's grounded rows join the client matrix beside the bounded
+    bank, and the prefix layers' K/V are gathered at the kept rows."""
+    from paper_2608_02134_gb300 import workloads
+    from tests import gpu_harness as GH
+    wl = workloads.make("longsmall")
+    g = GH.run(wl, n_hist=1, n_prefix=2)
+    assert g.status == 0, hex(g.status)
+    rep = GH.compare_image(g, 0, 2e-2)
+    assert not rep.dec.failures, "\n".join(rep.dec.failures[:10])
