@@ -577,7 +577,7 @@ static int compress_impl(const gmc_problem* prob, const gmc_params* params,
     return launch_heads(dm, p, sv[0], tv, st, 1, V > 1 ? &vg : nullptr);
   };
   const int msg_k = (message_tc_supported(dm) ? 3 : 1) * V;
-  GMC_TRY(g_prof.begin(st));  // k_probe zeroes the column sums u0 of the client build
+  GMC_TRY(g_prof.begin(st));  // k_rownorm zeroes the column sums u0 of the client build
   // the appearance branch: cosine Gram, or on long prefixes the projection,
   // the split unit states and the bounded bank's cosines
   auto project = [&](cudaStream_t q) -> cudaError_t {
@@ -625,6 +625,10 @@ static int compress_impl(const gmc_problem* prob, const gmc_params* params,
     } else {
       GMC_STAGE("gram", 1, launch_gram(dm, hidden, s, sd->st));
     }
+    // the appearance and spatial rows need only the cosines: built here,
+    // beside the message slice and the heads
+    GMC_STAGE("clients_aux", 1,
+              launch_build_clients(dm, p, fx, s, vr, lp ? ls.app : s.cos, sd->st, 2));
     GMC_TRY(cudaEventRecord(sd->join, sd->st));
     GMC_STAGE("probe", V, probes());
     GMC_STAGE("message", msg_k, messages());
@@ -633,7 +637,9 @@ static int compress_impl(const gmc_problem* prob, const gmc_params* params,
   }
   // every view's grounded rows count as head rows of the client layout
   const int HV = H * V;
-  GMC_STAGE("clients", 1, launch_build_clients(dm, p, fx, s, vr, lp ? ls.app : s.cos, st));
+  // the grounded rows (every row when stages are timed one after another)
+  GMC_STAGE("clients", 1,
+            launch_build_clients(dm, p, fx, s, vr, lp ? ls.app : s.cos, st, g_prof.on ? 0 : 1));
   if (out_clients) {  // staged call: the client matrix, before selection compacts it in place
     GMC_TRY(cudaMemcpyAsync(out_clients, s.C, sizeof(float) * dm.B * (size_t)dm.M * N,
                             cudaMemcpyDeviceToDevice, st));

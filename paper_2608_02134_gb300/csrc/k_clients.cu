@@ -80,7 +80,8 @@ __global__ void __launch_bounds__(256, 4) k_build_clients(
     const ViewRows vw, int nRS, const float* __restrict__ omega,
     const float* __restrict__ app, int MV, const int32_t* toff, int B, int N, int Tmax, int H, int M,
     int gh, int gw, int L, float beta_V, float beta_S, float tau_v, float tau_s,
-    float wq, float fx_scale, int check, int I, float* C, long long* u0, uint32_t* status) {
+    float wq, float fx_scale, int check, int I, float* C, long long* u0, uint32_t* status,
+    int part) {
   grid_dep_wait();
   __shared__ RowInfo ri[ROWS_PER_BLOCK];
   const int b = blockIdx.y;
@@ -89,12 +90,17 @@ __global__ void __launch_bounds__(256, 4) k_build_clients(
   const int Tb = tg.T, MG = vw.n * H * Tb, Mb = MG + MV + I * L * L;
   const int Ng = N / I;  // tokens of one image
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-  const int r0 = blockIdx.x * ROWS_PER_BLOCK;
-  if (r0 >= Mb) return;
+  // part 0: every row; 1: the grounded rows [0, MG); 2: the appearance and
+  // spatial rows [MG, Mb) (built beside the message slice and the heads)
+  const int rbeg = part == 2 ? MG : 0, rend = part == 1 ? MG : Mb;
+  const int r0 = rbeg + blockIdx.x * ROWS_PER_BLOCK;
+  if (r0 >= rend) return;
   {
     const int m = r0 + w;
     RowInfo inf{-1, nullptr, nullptr, 0.f, 0.f, 0.f, 0.f, 0.f, 0, N};
-    if (m < MG) {
+    if (m >= rend) {
+      // past this launch's rows
+    } else if (m < MG) {
       const int v = m / (H * Tb), hm = m - v * H * Tb;  // view, then (h, t) h-major
       const int h = hm / Tb, t = hm % Tb;
       float rsv = 0.f;  // parts over key splits, fixed order
@@ -156,7 +162,7 @@ __global__ void __launch_bounds__(256, 4) k_build_clients(
   }
   __shared__ int umode;  // 0 generic, 1 grounded (one head), 2 appearance, 3 spatial
   __syncthreads();
-  const int nrows = min(ROWS_PER_BLOCK, Mb - r0);
+  const int nrows = min(ROWS_PER_BLOCK, rend - r0);
   const float itv = 1.f / tau_v, its = 1.f / tau_s;
   if (threadIdx.x == 0) {
     int mode = 0;
@@ -288,12 +294,16 @@ __global__ void __launch_bounds__(256, 4) k_build_clients(
 }
 
 cudaError_t launch_build_clients(const Dims& dm, const gmc_params& p, int fx_exp, Scratch& s,
-                                 const ViewRows& views, const float* app, cudaStream_t st) {
-  dim3 grid(ceil_div(dm.M, ROWS_PER_BLOCK), dm.B);
+                                 const ViewRows& views, const float* app, cudaStream_t st,
+                                 int part) {
+  const int rows = part == 0 ? dm.M
+                 : part == 1 ? dm.V * dm.H * dm.T
+                             : dm.MV + dm.I * dm.L * dm.L;
+  dim3 grid(ceil_div(rows, ROWS_PER_BLOCK), dm.B);
   launch_k(k_build_clients, grid, 32 * ROWS_PER_BLOCK, 0, st, 1,
       views, s.nRS, s.omega, app, dm.MV, dm.toff, dm.B, dm.N, dm.T, dm.H, dm.M, dm.gh,
       dm.gw, dm.L, p.beta_V, p.beta_S, p.tau_v, p.tau_s, p.terminal_q_weight,
-      ldexpf(1.f, fx_exp), p.check_mode, dm.I, s.C, s.u0, s.status);
+      ldexpf(1.f, fx_exp), p.check_mode, dm.I, s.C, s.u0, s.status, part);
   return cudaGetLastError();
 }
 

@@ -13,9 +13,13 @@ namespace gmc {
 template <typename Tin>
 __global__ void k_rownorm(const Tin* __restrict__ hidden, const int32_t* toff, int B, int N,
                           int K, int Tmax, int D, float norm_eps, float* rn, float* rmsh,
-                          uint32_t* status) {
+                          long long* u0, uint32_t* status) {
   grid_dep_wait();
   const int b = blockIdx.y;
+  // the client build's column sums start at zero (this kernel opens the
+  // branch of the path that builds the appearance and spatial rows)
+  if (u0 && threadIdx.x < ROWS_PER_BLOCK && blockIdx.x * ROWS_PER_BLOCK + (int)threadIdx.x < N)
+    u0[(size_t)b * N + blockIdx.x * ROWS_PER_BLOCK + threadIdx.x] = 0;
   const TextGeom tg = text_geom(toff, b, B, Tmax, status);
   if (tg.T == 0) return;
   const int lane = threadIdx.x & 31;
@@ -55,15 +59,11 @@ template <typename Tin>
 __global__ void __launch_bounds__(256) k_probe(
     const Tin* __restrict__ keys, const float* __restrict__ W, const int32_t* toff, int B, int N,
     int K, int Tmax, int H, int Hkv, int d, float lambda_mass, float eps_mass, float* Z,
-    float* zn2, float* sigpart, int nP, float* sigma, uint32_t* tick, long long* u0,
-    uint32_t* status) {
+    float* zn2, float* sigpart, int nP, float* sigma, uint32_t* tick, uint32_t* status) {
   grid_dep_wait();
   extern __shared__ float4 sm_probe4[];
   __shared__ int last;
   const int b = blockIdx.z, g = blockIdx.y, pb = blockIdx.x;
-  // the client build's column sums start at zero (it runs after this kernel)
-  if (u0 && g == 0 && threadIdx.x < PR_TOK && pb * PR_TOK + (int)threadIdx.x < N)
-    u0[(size_t)b * N + pb * PR_TOK + threadIdx.x] = 0;
   const TextGeom tg = text_geom(toff, b, B, Tmax, status);
   if (tg.T == 0) return;  // uniform over the image
   const SeqIdx sq(b, N, K, tg.off, tg.T);
@@ -219,11 +219,11 @@ cudaError_t launch_rownorm(const Dims& dm, const void* hidden, float norm_eps, S
   if (dm.dtype == GMC_BF16)
     launch_k(k_rownorm<__nv_bfloat16>, grid, 32 * ROWS_PER_BLOCK, 0, st, 1,
         (const __nv_bfloat16*)hidden, dm.toff, dm.B, dm.N, dm.K, dm.T, dm.D, norm_eps, s.rn,
-        s.rmsh, s.status);
+        s.rmsh, s.u0, s.status);
   else
     launch_k(k_rownorm<float>, grid, 32 * ROWS_PER_BLOCK, 0, st, 1, (const float*)hidden, dm.toff, dm.B,
                                                            dm.N, dm.K, dm.T, dm.D, norm_eps, s.rn,
-                                                           s.rmsh, s.status);
+                                                           s.rmsh, s.u0, s.status);
   return cudaGetLastError();
 }
 
@@ -233,11 +233,11 @@ cudaError_t launch_rms_rows(const Dims& dm, const void* hidden, float* rmsh, uin
   if (dm.dtype == GMC_BF16)
     launch_k(k_rownorm<__nv_bfloat16>, grid, 32 * ROWS_PER_BLOCK, 0, st, 1,
         (const __nv_bfloat16*)hidden, dm.toff, dm.B, dm.N, dm.K, dm.T, dm.D, 1e-12f, nullptr,
-        rmsh, status);
+        rmsh, nullptr, status);
   else
     launch_k(k_rownorm<float>, grid, 32 * ROWS_PER_BLOCK, 0, st, 1, (const float*)hidden, dm.toff, dm.B,
                                                            dm.N, dm.K, dm.T, dm.D, 1e-12f,
-                                                           nullptr, rmsh, status);
+                                                           nullptr, rmsh, nullptr, status);
   return cudaGetLastError();
 }
 
@@ -252,13 +252,13 @@ cudaError_t launch_probe(const Dims& dm, const void* keys, const float* W, const
     if ((e = set_smem_limit((const void*)k_probe<__nv_bfloat16>, smem)) != cudaSuccess) return e;
     launch_k(k_probe<__nv_bfloat16>, grid, 256, smem, st, 1,
         (const __nv_bfloat16*)keys, W, dm.toff, dm.B, dm.N, dm.K, dm.T, dm.H, dm.Hkv, dm.d,
-        p.lambda_mass, p.eps_mass, s.Z, s.zn2, s.sigpart, s.nP, s.sigma, s.tick, s.u0, s.status);
+        p.lambda_mass, p.eps_mass, s.Z, s.zn2, s.sigpart, s.nP, s.sigma, s.tick, s.status);
   } else {
     if ((e = set_smem_limit((const void*)k_probe<float>, smem)) != cudaSuccess) return e;
     launch_k(k_probe<float>, grid, 256, smem, st, 1, (const float*)keys, W, dm.toff, dm.B, dm.N, dm.K,
                                             dm.T, dm.H, dm.Hkv, dm.d, p.lambda_mass, p.eps_mass,
                                             s.Z, s.zn2, s.sigpart, s.nP, s.sigma, s.tick,
-                                            s.u0, s.status);
+                                            s.status);
   }
   return cudaGetLastError();
 }

@@ -146,9 +146,11 @@ bool heads_supported(int H);  // the head statistics of H heads fit a block (H <
 cudaError_t launch_gram(const Dims&, const void* hidden, Scratch&, cudaStream_t);
 // app: the appearance rows' cosines, [B][MV][N] (the exact bank passes the
 // N x N cosine matrix, MV = N)
+// part: 0 every row, 1 the grounded rows, 2 the appearance and spatial rows
+// (the column sums s.u0 start at zero: k_rownorm clears them)
 cudaError_t launch_build_clients(const Dims&, const gmc_params&, int fx_exp, Scratch&,
                                  const ViewRows& views, const float* app,
-                                 cudaStream_t);
+                                 cudaStream_t, int part = 0);
 // State left by the first (dense) selection round, run over the whole GPU.
 // Rounds of the solver run on the whole GPU before the cluster kernel takes
 // over: the dense first round, then sparse_gpu_rounds(N) sparse rounds (an
