@@ -66,6 +66,7 @@ __global__ void __launch_bounds__(512) k_r0_pool(const long long* __restrict__ u
     info[b * INFO_W + 2] = 0;
     info[b * INFO_W + 3] = 0;
     info[b * INFO_W + 4] = 0;
+    info[b * INFO_W + 5] = -1;  // boundary bucket of the last pool: none yet
   }
   if (toff && text_geom(toff, b, B, Tmax, nullptr).T == 0) {
     if (threadIdx.x == 0) info[b * INFO_W] = 0;
@@ -119,9 +120,13 @@ __global__ void __launch_bounds__(512) k_r0_pool(const long long* __restrict__ u
     if (threadIdx.x == 0) info[b * INFO_W] = I;
     return;
   }
-  const int Pt = sel::select_pool(ug, selz, N, P, w, pool, nullptr);
+  int bstar = -1;
+  const int Pt = sel::select_pool(ug, selz, N, P, w, pool, nullptr, nullptr, &bstar);
   for (int k = threadIdx.x; k < P; k += blockDim.x) pool0[(size_t)b * P + k] = k < Pt ? pool[k] : -1;
-  if (threadIdx.x == 0) info[b * INFO_W] = Pt;
+  if (threadIdx.x == 0) {
+    info[b * INFO_W] = Pt;
+    info[b * INFO_W + 5] = bstar;
+  }
 }
 
 __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_rho(
@@ -347,6 +352,10 @@ __global__ void __launch_bounds__(512) k_rg_pool(const long long* __restrict__ u
   }
   sel::PoolScratch w{};  // gains in shared memory: no boundary staging
   char* p = sm_rgp;
+  sel::WindowScratch ws;
+  ws.win = reinterpret_cast<int*>(p);       p += sizeof(int) * (sel::WBINS + 4);
+  ws.cu = reinterpret_cast<long long*>(p);  p += sizeof(long long) * sel::WCAP;
+  ws.cj = reinterpret_cast<int*>(p);        p += sizeof(int) * sel::WCAP;
   long long* ug = reinterpret_cast<long long*>(p);  p += sizeof(long long) * (size_t)N;
   w.hist = reinterpret_cast<int*>(p);       p += sizeof(int) * sel::HBINS;
   w.bnd = reinterpret_cast<int*>(p);        p += sizeof(int) * N;
@@ -357,19 +366,28 @@ __global__ void __launch_bounds__(512) k_rg_pool(const long long* __restrict__ u
   w.key = reinterpret_cast<short*>(p);     p += sizeof(short) * (size_t)N;
   w.pk = reinterpret_cast<unsigned char*>(p); p += (size_t)N;
   unsigned char* self = reinterpret_cast<unsigned char*>(p);
+  // the gains in shared memory (select_pool reads them often): copied here
+  // without a boundary hint, else by the window pool's first pass
+  int hint = info[b * INFO_W + 5];
+  const long long* ub = ucur + (size_t)b * N;
   for (int j = threadIdx.x; j < N; j += blockDim.x) {
     self[j] = 0;
-    ug[j] = ucur[(size_t)b * N + j];  // the gains in shared memory: select_pool reads them often
-    if (tv.base) tv.gains(b, rd, N)[j] = ug[j];
+    if (hint < 0) ug[j] = ub[j];
   }
   for (int h = threadIdx.x; h < sel::HBINS; h += blockDim.x) w.hist[h] = 0;
   if (threadIdx.x < sel::CBINS) w.coarse[threadIdx.x] = 0;
+  for (int q = threadIdx.x; q < sel::WBINS + 4; q += blockDim.x) ws.win[q] = 0;
   __syncthreads();
   for (int q = threadIdx.x; q < S; q += blockDim.x) self[order[(size_t)b * K + q]] = 1;
   __syncthreads();
-  const int Pt = sel::select_pool(ug, self, N, P, w, pool, nullptr);
+  int Pt = sel::select_pool_window([&](int j) { return ub[j]; }, ug, self, N, P, ws, pool,
+                                   nullptr, &hint);
+  if (Pt < 0) Pt = sel::select_pool(ug, self, N, P, w, pool, nullptr, nullptr, &hint);
+  if (tv.base)
+    for (int j = threadIdx.x; j < N; j += blockDim.x) tv.gains(b, rd, N)[j] = ug[j];
   for (int k = threadIdx.x; k < P; k += blockDim.x) pool0[(size_t)b * P + k] = k < Pt ? pool[k] : -1;
   if (threadIdx.x == 0) {
+    info[b * INFO_W + 5] = hint;
     info[b * INFO_W] = Pt;
     info[b * INFO_W + 3] = S;
     info[b * INFO_W + 4] = rd;
@@ -607,7 +625,8 @@ cudaError_t launch_round0(const R0State& r0, int B, int N, int K, int M, const i
                                              r0.bcov, r0.cnt, r0.fv, order, rpw, I, tv);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   // sparse rounds: gains alternate between u1 and u2
-  const size_t psm = smem;  // the pool kernel's layout is round 0's
+  // the pool kernel's layout is round 0's after the window scratch
+  const size_t psm = smem + sizeof(int) * (sel::WBINS + 4) + 12 * (size_t)sel::WCAP;
   if ((e = set_smem_limit((const void*)k_rg_pool, psm)) != cudaSuccess) return e;
   const size_t rsm = sizeof(short) * (size_t)N;
   if ((e = set_smem_limit((const void*)k_rg_rho, rsm)) != cudaSuccess) return e;

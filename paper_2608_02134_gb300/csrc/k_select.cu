@@ -114,6 +114,9 @@ struct SelSmem {
   int* bnb;             // [RPC] flat mode: bits of the row's largest batch value
   long long* bfix;      // [RPC] flat mode: coverage in fixed point
   int* cstart;          // [N+1] flat mode: first entry of every token
+  int* win;             // [WBINS + 4] select_pool_window: window bins and counters
+  long long* wcu;       // [WCAP] select_pool_window: candidates' gains
+  int* wcj;             // [WCAP] select_pool_window: candidates' tokens
   long long* fb;        // [8]  F_S[3], F_V[3] (fixed point)
   int* scal;            // [16] Bstar, c_hi, Pt, nbnd, cursor, global rows left
   float* svals;         // [cap]
@@ -155,6 +158,9 @@ __host__ __device__ inline size_t sel_fixed_bytes(int N, int P, int RPC, int gwo
   p = take(sizeof(int) * RPC);      if (o) o->bnb = (int*)p;
   p = take(sizeof(long long) * RPC);  if (o) o->bfix = (long long*)p;
   p = take(sizeof(int) * (N + 1));  if (o) o->cstart = (int*)p;
+  p = take(sizeof(int) * (sel::WBINS + 4));  if (o) o->win = (int*)p;
+  p = take(sizeof(long long) * sel::WCAP);   if (o) o->wcu = (long long*)p;
+  p = take(sizeof(int) * sel::WCAP);         if (o) o->wcj = (int*)p;
   p = take(sizeof(long long) * 8);  if (o) o->fb = (long long*)p;
   p = take(sizeof(int) * 16);       if (o) o->scal = (int*)p;
   return off;
@@ -239,6 +245,9 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
   const int rd0 = valid ? a.r0.info[b * INFO_W + 2] : 0;  // rounds done
   const int Pt0 = rd0;                                // > 0: the rounds left survivor lists
   const int nb0 = rd0 > 0 ? a.r0.info[b * INFO_W + 1] : 0;  // tokens selected so far
+  // boundary bucket of the last pool (-1: none; the next pool is then found
+  // over every bucket)
+  int phint = rd0 > 0 ? a.r0.info[b * INFO_W + 5] : -1;
   for (int j = threadIdx.x; j < N; j += blockDim.x) {
     s.u_full[j] = rd0 > 0 ? a.r0.ugain[(size_t)b * N + j] : a.u0[(size_t)b * N + j];
     s.poolslot[j] = -1;
@@ -248,6 +257,7 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
   for (int q = threadIdx.x; q < NB * SL; q += blockDim.x) s.gacc[q] = 0;
   for (int h = threadIdx.x; h < HBINS; h += blockDim.x) s.hist[h] = 0;  // select_pool keeps it zero
   if (threadIdx.x < sel::CBINS) s.coarse[threadIdx.x] = 0;
+  for (int q = threadIdx.x; q < sel::WBINS + 4; q += blockDim.x) s.win[q] = 0;
   if (threadIdx.x < 8) s.fb[threadIdx.x] = 0;
   if (threadIdx.x < 16) s.scal[threadIdx.x] = 0;
   if (threadIdx.x == 0) s.scal[SC_GLOBAL] = 1;
@@ -386,6 +396,34 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
     for (int c = c0; c < CS; c += cstep) red_add_cluster(s.s_acc + k, c, v);
   };
   int S_count = nb0, rnd = rd0, filled = 0;
+  // token j's gain for the round after the last one, at its owner
+  auto gain_at = [&](int j) -> const unsigned long long* {
+    const int o = j / SL;
+    const unsigned long long* at = s.gacc + ((rnd - 1) & (NB - 1)) * SL + (j - o * SL);
+    return CS > 1 ? cluster.map_shared_rank(at, o) : at;
+  };
+  auto read_gains = [&]() {
+    constexpr int GU = 4;  // remote loads in flight per thread
+    for (int j0 = threadIdx.x; j0 < N; j0 += GU * blockDim.x) {
+      unsigned long long v[GU];
+#pragma unroll
+      for (int t = 0; t < GU; ++t) {
+        const int j = j0 + t * (int)blockDim.x;
+        v[t] = j < N ? *gain_at(j) : 0ull;
+      }
+#pragma unroll
+      for (int t = 0; t < GU; ++t) {
+        const int j = j0 + t * (int)blockDim.x;
+        if (j < N) s.u_full[j] = (long long)v[t];
+      }
+    }
+    if (CS == 1) {  // a single CTA reuses its one buffer at once
+      __syncthreads();
+      for (int q = threadIdx.x; q < SL; q += blockDim.x) s.gacc[q] = 0;
+    }
+    __syncthreads();
+  };
+  bool remote_gains = false;  // this round's gains are still at their owners
   const int sub = lane / G, gl = lane % G;
   const int gid = wid * (32 / G) + sub, ngrp = nw * (32 / G);  // 8-lane groups of the block
   const unsigned gm = 0xFFu << (sub * G);
@@ -395,11 +433,24 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
       if (threadIdx.x == 0) set_status(a.status, GMC_STATUS_INTERNAL);
       break;
     }
+    // ---- pool of this round ------------------------------------------------------
+    // (u_full is complete once either pool routine returns)
+    int Pt;
+    if (remote_gains)
+      Pt = sel::select_pool_window([&](int j) { return (long long)*gain_at(j); }, s.u_full, s.sel,
+                                   N, P, sel::WindowScratch{s.win, s.wcu, s.wcj}, s.pool,
+                                   s.poolslot, &phint);
+    else
+      Pt = sel::select_pool_window([&](int j) { return s.u_full[j]; }, s.u_full, s.sel, N, P,
+                                   sel::WindowScratch{s.win, s.wcu, s.wcj}, s.pool, s.poolslot,
+                                   &phint);
+    remote_gains = false;
+    if (Pt < 0) {
+      sel::PoolScratch pw{s.hist, s.coarse, s.bnd, s.key, s.pk, s.wsum, s.scal + 8};
+      Pt = sel::select_pool(s.u_full, s.sel, N, P, pw, s.pool, s.poolslot, nullptr, &phint);
+    }
     if (r == 0 && a.tv.base)  // certificate input: the gains this round starts from
       for (int j = threadIdx.x; j < N; j += blockDim.x) a.tv.gains(b, rnd, N)[j] = s.u_full[j];
-    // ---- pool of this round ------------------------------------------------------
-    sel::PoolScratch pw{s.hist, s.coarse, s.bnd, s.key, s.pk, s.wsum, s.scal + 8};
-    const int Pt = sel::select_pool(s.u_full, s.sel, N, P, pw, s.pool, s.poolslot);
     if (Pt == 0) {
       // Zero-gain remainder: fill in ascending source order (F unchanged).
       const int need = K - S_count;
@@ -792,18 +843,12 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
     cluster.sync();  // every contribution to the new gains has reached its owner
 
     // ---- gains of the next round, read from their owners ----------------------
-    {
-      const unsigned long long* gb = s.gacc + ((rnd - 1) & (NB - 1)) * SL;
-      for (int j = threadIdx.x; j < N; j += blockDim.x) {
-        const int o = j / SL;
-        const unsigned long long* at = gb + (j - o * SL);
-        s.u_full[j] = (long long)*(CS > 1 ? cluster.map_shared_rank(at, o) : at);
-      }
-      if (CS == 1) {  // a single CTA reuses its one buffer at once
-        __syncthreads();
-        for (int q = threadIdx.x; q < SL; q += blockDim.x) s.gacc[q] = 0;
-      }
-      __syncthreads();
+    // With a cluster and a boundary hint the pool's first pass reads them
+    // (remote_gains); otherwise they are copied here.
+    remote_gains = CS > 1;
+    if (!remote_gains || phint < 0) {
+      read_gains();
+      remote_gains = false;
     }
   }
 

@@ -119,10 +119,11 @@ __device__ __forceinline__ int group_rank_of(const int* a, int n, int x, int gl,
 // (the wide solver's long prefixes) splits a large boundary bucket once more
 // (below); the standard solvers leave it out, it costs them registers.
 // Every thread of the block must call it; blockDim is a multiple of 32.
+// bstar_out (optional): the boundary bucket, or -1 when every candidate entered.
 template <bool REFINE = false>
 __device__ inline int select_pool(const long long* u, const unsigned char* sel, int N, int P,
                                   PoolScratch w, int* pool, short* poolslot,
-                                  const int* ids = nullptr) {
+                                  const int* ids = nullptr, int* bstar_out = nullptr) {
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
   const int nc = (N + 32 * nw - 1) / (32 * nw);  // chunks per warp
   const unsigned lt = lanemask_lt();
@@ -333,6 +334,190 @@ __device__ inline int select_pool(const long long* u, const unsigned char* sel, 
     }
   }
   __syncthreads();
+  if (bstar_out) *bstar_out = bstar;
+  return Pt;
+}
+
+// Pool of a later round from a window of buckets below the previous boundary.
+//
+// A round takes its batch out of the candidates and can only lower the other
+// gains (the coverage b_m grows), so the P-th largest gain of the next round is
+// at most the P-th largest of this one: its bucket lies at or below the last
+// boundary bucket `hint`.  One pass loads the gains (load(j), stored into u[j]
+// for later readers), counts the candidates above a window of WBINS buckets
+// that ends WTOP buckets above the hint and histograms the ones inside it;
+// every warp finds the boundary bucket from the window alone.  The tokens in
+// or above the boundary bucket (at most WCAP) are listed in any order and
+// ranked exactly by (u desc, index asc); a pool token's slot is its rank, so
+// the pool is the same in every block that calls this with the same gains and
+// hint.  Three block barriers; a thread's loads of a pass are all issued before
+// its atomics.
+//
+// Returns Pt and sets *hint to the new boundary bucket (-1 once every
+// candidate enters); returns -1 when the boundary is not inside the window or
+// more than WCAP tokens reach it (the caller then runs select_pool on u, which
+// is complete on return).  With *hint < 0 it returns -1 at once and loads
+// nothing.  Every thread gets the same answer.  Every thread of the block must
+// call it.
+constexpr int WBINS = 128;  // window buckets: 4 per lane of one warp
+constexpr int WTOP = 8;     // window buckets above the hint
+constexpr int WCAP = 256;   // candidates ranked exactly
+constexpr int WU = 4;       // tokens a thread handles per pass step
+struct WindowScratch {
+  int* win;        // [WBINS + 4] window bins (top bucket first) and 4 counters;
+                   // all zero on entry and on return
+  long long* cu;   // [WCAP] candidates' gains
+  int* cj;         // [WCAP] candidates' tokens
+};
+
+template <class Load>
+__device__ inline int select_pool_window(Load load, long long* u, const unsigned char* sel, int N,
+                                         int P, WindowScratch w, int* pool, short* poolslot,
+                                         int* hint) {
+  const int lane = threadIdx.x & 31;
+  const int h = *hint;
+  if (h < 0) return -1;  // uniform: every thread holds the same hint
+  const int top = h + WTOP;             // highest window bucket (bin 0)
+  int* cnt = w.win + WBINS;             // 0: above the window, 1: positive, 2: listed
+  const int step = (int)blockDim.x;
+  // 1. gains, window histogram, counts above the window and of positive candidates
+  int npos_w = 0, nabove_w = 0;
+  for (int j0 = (int)threadIdx.x - lane; j0 < N; j0 += WU * step) {  // warp-uniform
+    long long v[WU];
+    unsigned char sl[WU];
+#pragma unroll
+    for (int t = 0; t < WU; ++t) {
+      const int j = j0 + t * step + lane;
+      v[t] = j < N ? load(j) : 0;
+      sl[t] = j < N ? sel[j] : 1;
+    }
+#pragma unroll
+    for (int t = 0; t < WU; ++t) {
+      const int j = j0 + t * step + lane;
+      if (j < N) u[j] = v[t];
+      const int kb = !sl[t] && v[t] > 0 ? gain_bucket(v[t]) : -1;
+      const int bin = top - kb;
+      if (kb >= 0 && bin >= 0 && bin < WBINS) atomicAdd(&w.win[bin], 1);
+      npos_w += __popc(__ballot_sync(FULL, kb >= 0));
+      nabove_w += __popc(__ballot_sync(FULL, kb > top));
+    }
+  }
+  if (lane == 0) {
+    if (nabove_w) atomicAdd(&cnt[0], nabove_w);
+    if (npos_w) atomicAdd(&cnt[1], npos_w);
+  }
+  __syncthreads();
+  // 2. boundary bucket, found by every warp alike
+  const int npos = cnt[1], nabove = cnt[0];
+  int bstar = -1, ncand = npos, Pt = npos;
+  bool miss = false;
+  if (npos > P) {
+    Pt = P;
+    if (nabove >= P) {
+      miss = true;  // the boundary is above the window
+    } else {
+      const int4 c4 = reinterpret_cast<const int4*>(w.win)[lane];  // bins 4 lane .. 4 lane + 3
+      const int s4 = c4.x + c4.y + c4.z + c4.w;
+      int incl = s4;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(FULL, incl, o);
+        if (lane >= o) incl += y;
+      }
+      const int need = P - nabove;
+      const unsigned reach = __ballot_sync(FULL, incl >= need);
+      if (!reach) {
+        miss = true;  // the boundary is below the window
+      } else {
+        const int L = __ffs(reach) - 1;
+        int acc = __shfl_sync(FULL, incl - s4, L);
+        const int b0 = __shfl_sync(FULL, c4.x, L), b1 = __shfl_sync(FULL, c4.y, L);
+        const int b2 = __shfl_sync(FULL, c4.z, L), b3 = __shfl_sync(FULL, c4.w, L);
+        int t = 0;
+        if (acc + b0 < need) {
+          acc += b0;
+          t = 1;
+          if (acc + b1 < need) {
+            acc += b1;
+            t = 2;
+            if (acc + b2 < need) {
+              acc += b2;
+              t = 3;
+            }
+          }
+        }
+        const int bt = t == 0 ? b0 : t == 1 ? b1 : t == 2 ? b2 : b3;
+        bstar = top - (4 * L + t);
+        ncand = nabove + acc + bt;  // every candidate in or above the boundary bucket
+        miss = ncand > WCAP;
+      }
+    }
+  } else {
+    miss = npos > WCAP;
+  }
+  if (miss) {
+    __syncthreads();  // every warp has read the bins
+    for (int q = threadIdx.x; q < WBINS + 4; q += blockDim.x) w.win[q] = 0;
+    __syncthreads();
+    return -1;
+  }
+  // 3. list the candidates in or above the boundary bucket (any order); a
+  //    thread reads back only the gains it stored itself
+  for (int j0 = (int)threadIdx.x - lane; j0 < N; j0 += WU * step) {
+    long long v[WU];
+    unsigned want = 0;
+#pragma unroll
+    for (int t = 0; t < WU; ++t) {
+      const int j = j0 + t * step + lane;
+      v[t] = j < N ? u[j] : 0;
+      if (j < N && !sel[j] && v[t] > 0 && gain_bucket(v[t]) >= bstar) want |= 1u << t;
+    }
+    unsigned bal[WU];
+    int tot = 0;
+#pragma unroll
+    for (int t = 0; t < WU; ++t) {
+      bal[t] = __ballot_sync(FULL, (want >> t) & 1u);
+      tot += __popc(bal[t]);
+    }
+    if (tot) {  // warp-uniform: one atomic per warp and step
+      int base = 0;
+      if (lane == 0) base = atomicAdd(&cnt[2], tot);
+      base = __shfl_sync(FULL, base, 0);
+      const unsigned lt = lanemask_lt();
+#pragma unroll
+      for (int t = 0; t < WU; ++t) {
+        if ((want >> t) & 1u) {
+          const int at = base + __popc(bal[t] & lt);
+          w.cu[at] = v[t];
+          w.cj[at] = j0 + t * step + lane;
+        }
+        base += __popc(bal[t]);
+      }
+    }
+  }
+  __syncthreads();
+  // 4. rank every candidate among them (4 lanes each); slot = rank
+  for (int q = threadIdx.x; q < WBINS + 4; q += blockDim.x) w.win[q] = 0;
+  for (int base = ((int)threadIdx.x - lane) >> 2; base < ncand; base += blockDim.x >> 2) {
+    const int q = base + (lane >> 2), gl = lane & 3;
+    int rank = 0;
+    long long v = 0;
+    int jq = 0;
+    if (q < ncand) {
+      v = w.cu[q];
+      jq = w.cj[q];
+#pragma unroll 4
+      for (int q2 = gl; q2 < ncand; q2 += 4) rank += key_before(w.cu[q2], w.cj[q2], v, jq);
+    }
+    rank += __shfl_xor_sync(FULL, rank, 1);
+    rank += __shfl_xor_sync(FULL, rank, 2);
+    if (q < ncand && gl == 0 && rank < Pt) {
+      pool[rank] = jq;
+      if (poolslot) poolslot[jq] = (short)rank;
+    }
+  }
+  __syncthreads();
+  *hint = Pt == P ? bstar : -1;
   return Pt;
 }
 
