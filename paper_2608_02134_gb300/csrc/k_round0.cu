@@ -341,7 +341,9 @@ __global__ void __launch_bounds__(512) k_rg_pool(const long long* __restrict__ u
   extern __shared__ __align__(16) char sm_rgp[];
   const int b = blockIdx.x;
   for (int k = threadIdx.x; k < P; k += blockDim.x) sc[(size_t)b * P + k] = 0;
-  for (int j = threadIdx.x; j < N; j += blockDim.x) unext[(size_t)b * N + j] = 0;
+  // the next gains start from these: the filter adds only the changes of the
+  // rows whose coverage grows
+  for (int j = threadIdx.x; j < N; j += blockDim.x) unext[(size_t)b * N + j] = ucur[(size_t)b * N + j];
   const int S = info[b * INFO_W + 1], rd = info[b * INFO_W + 2];
   // nothing to do here once the budget is met or when the first round found
   // no gain: the cluster kernel handles those cases
@@ -542,7 +544,8 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_rg_filter(
     // chunks issued before the first use (and, below, before any survivor is
     // written back in place: a chunk's survivors land below its end).
     constexpr int FU = 4;
-    float bnew = bcov[row];
+    const float bold = bcov[row];
+    float bnew = bold;
     for (int e00 = 0; e00 < n; e00 += 32 * FU) {
       int jj[FU];
 #pragma unroll
@@ -556,6 +559,11 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_rg_filter(
     }
     bnew = warp_max(bnew);
     const long long fb_new = to_fix(bnew, fxs);
+    if (!(bnew > bold)) {  // no batch entry above the coverage: row and gains unchanged
+      if (lane == 0 && tv.base) atomicAdd(tv.cover(b, rd), (unsigned long long)fb_new);
+      continue;
+    }
+    const long long fb_old = to_fix(bold, fxs);
     const unsigned lt = sel::lanemask_lt();
     int wr = 0;
     for (int e00 = 0; e00 < n; e00 += 32 * FU) {
@@ -574,13 +582,18 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_rg_filter(
       __syncwarp();  // the chunks are read before any survivor moves down into them
 #pragma unroll
       for (int u = 0; u < FU; ++u) {
-        const bool keep = e00 + 32 * u + lane < n && cc[u] > bnew;
+        const bool in = e00 + 32 * u + lane < n;
+        const bool keep = in && cc[u] > bnew;
         const unsigned bal = __ballot_sync(FULL, keep);
+        // the entry's residual moves from C - b_old to C - b_new, or to zero
+        // (exact: integers modulo 2^64)
+        if (in)
+          atomicAdd(&uacc[jj[u]], (unsigned long long)(keep ? fb_old - fb_new
+                                                             : fb_old - to_fix(cc[u], fxs)));
         if (keep) {
           const int pos = wr + __popc(bal & lt);
           vals[pos] = cc[u];
           cols[pos] = (uint16_t)jj[u];
-          atomicAdd(&uacc[jj[u]], (unsigned long long)(to_fix(cc[u], fxs) - fb_new));
         }
         wr += __popc(bal);
       }

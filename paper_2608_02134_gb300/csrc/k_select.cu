@@ -89,9 +89,10 @@ struct SelArgs {
 };
 
 struct SelSmem {
-  unsigned long long* gacc;  // [NB][SL] next-round gains of the tokens this CTA owns,
-                             // summed by every CTA of the cluster (NB = 2 buffers
-                             // used by alternate rounds when CS > 1, else 1)
+  unsigned long long* gacc;  // [SL] gains of the tokens this CTA owns: every CTA of
+                             // the cluster adds the changes of its rows (
+                             // the buffer is read in a round's pool and changed
+                             // after that round's score barrier)
   long long* u_full;    // [N]  gains of the current round (every CTA)
   int* hist;            // [HBINS]
   int* coarse;          // [CBINS]
@@ -113,6 +114,7 @@ struct SelSmem {
   unsigned long long* z64;  // [RPC] flat mode: softmax denominator (fixed point 2^40)
   int* bnb;             // [RPC] flat mode: bits of the row's largest batch value
   long long* bfix;      // [RPC] flat mode: coverage in fixed point
+  long long* bfold;     // [RPC] flat mode: coverage in fixed point before the round's batch
   int* cstart;          // [N+1] flat mode: first entry of every token
   int* win;             // [WBINS + 4] select_pool_window: window bins and counters
   long long* wcu;       // [WCAP] select_pool_window: candidates' gains
@@ -157,6 +159,7 @@ __host__ __device__ inline size_t sel_fixed_bytes(int N, int P, int RPC, int gwo
   p = take(sizeof(unsigned long long) * RPC); if (o) o->z64 = (unsigned long long*)p;
   p = take(sizeof(int) * RPC);      if (o) o->bnb = (int*)p;
   p = take(sizeof(long long) * RPC);  if (o) o->bfix = (long long*)p;
+  p = take(sizeof(long long) * RPC);  if (o) o->bfold = (long long*)p;
   p = take(sizeof(int) * (N + 1));  if (o) o->cstart = (int*)p;
   p = take(sizeof(int) * (sel::WBINS + 4));  if (o) o->win = (int*)p;
   p = take(sizeof(long long) * sel::WCAP);   if (o) o->wcu = (long long*)p;
@@ -227,10 +230,9 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
   const int RPC = a.rpc;  // capacity of the per-row arrays of one CTA
   // token j's next-round gain is summed in CTA j / SL (its owner)
   const int SL = (N + CS - 1) / CS;
-  const int NB = CS > 1 ? 2 : 1;
 
   SelSmem s;
-  const size_t fixed = sel_fixed_bytes(N, P, RPC, NB * SL, &s, sm_sel);
+  const size_t fixed = sel_fixed_bytes(N, P, RPC, SL, &s, sm_sel);
   s.svals = reinterpret_cast<float*>(sm_sel + fixed);
   s.scols = reinterpret_cast<uint16_t*>(sm_sel + fixed + sizeof(float) * (size_t)a.cap);
   s.srows = s.scols + a.cap;
@@ -254,7 +256,12 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
     s.sel[j] = 0;
   }
   for (int k = threadIdx.x; k < P; k += blockDim.x) s.s_acc[k] = 0;
-  for (int q = threadIdx.x; q < NB * SL; q += blockDim.x) s.gacc[q] = 0;
+  for (int q = threadIdx.x; q < SL; q += blockDim.x) {  // the gains of the tokens this CTA owns
+    const int j = r * SL + q;
+    s.gacc[q] = j < N ? (unsigned long long)(rd0 > 0 ? a.r0.ugain[(size_t)b * N + j]
+                                                     : a.u0[(size_t)b * N + j])
+                      : 0ull;
+  }
   for (int h = threadIdx.x; h < HBINS; h += blockDim.x) s.hist[h] = 0;  // select_pool keeps it zero
   if (threadIdx.x < sel::CBINS) s.coarse[threadIdx.x] = 0;
   for (int q = threadIdx.x; q < sel::WBINS + 4; q += blockDim.x) s.win[q] = 0;
@@ -388,7 +395,7 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
   // (exact: 64-bit integer atomics, order-independent)
   auto gain_add = [&](int j, unsigned long long v, int rnd_now) {
     const int o = j / SL;
-    unsigned long long* at = s.gacc + (rnd_now & (NB - 1)) * SL + (j - o * SL);
+    unsigned long long* at = s.gacc + (j - o * SL);
     if (CS > 1) red_add_cluster(at, o, v); else atomicAdd(at, v);
   };
   // add v to pool slot k's score in every CTA of the cluster
@@ -399,7 +406,7 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
   // token j's gain for the round after the last one, at its owner
   auto gain_at = [&](int j) -> const unsigned long long* {
     const int o = j / SL;
-    const unsigned long long* at = s.gacc + ((rnd - 1) & (NB - 1)) * SL + (j - o * SL);
+    const unsigned long long* at = s.gacc + (j - o * SL);
     return CS > 1 ? cluster.map_shared_rank(at, o) : at;
   };
   auto read_gains = [&]() {
@@ -416,10 +423,6 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
         const int j = j0 + t * (int)blockDim.x;
         if (j < N) s.u_full[j] = (long long)v[t];
       }
-    }
-    if (CS == 1) {  // a single CTA reuses its one buffer at once
-      __syncthreads();
-      for (int q = threadIdx.x; q < SL; q += blockDim.x) s.gacc[q] = 0;
     }
     __syncthreads();
   };
@@ -627,11 +630,8 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
         for (int w2 = 0; w2 < SEL_WARPS; ++w2) v += s.sw[w2 * Pt + k];
         if (v) score_push(k, v, c, CS);
       }
-    cluster.sync();  // every CTA's scores have reached every CTA's s_acc
-    // nobody reads the gain buffer of the previous round any more (it was read
-    // before this round's pool): clear this CTA's part of it for the next round
-    if (CS > 1)
-      for (int q = threadIdx.x; q < SL; q += blockDim.x) s.gacc[((rnd + 1) & 1) * SL + q] = 0;
+    cluster.sync();  // every CTA's scores have reached every CTA's s_acc, and every
+                     // CTA has read this round's gains
 
     // ---- batch, coverage update, survivor filter, next gains ------------------
     const int nb = min(a.bsz, min(Pt, K - S_count));
@@ -662,6 +662,7 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
       for (int q = threadIdx.x; q < nrows; q += blockDim.x) {
         const float bn = fmaxf(s.bcov[q], __int_as_float(s.bnb[q]));
         s.bcov[q] = bn;
+        s.bfold[q] = s.bfix[q];
         s.bfix[q] = to_fix(bn, fxs);
         s.bnb[q] = 0;
         s.rmaxb[q] = 0;
@@ -670,9 +671,12 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
       }
       for (int j = threadIdx.x; j < N; j += blockDim.x) s.bnd[j] = 0;  // live entries per token
       __syncthreads();
-      // survivor filter (dead entries marked in place) and next-round gains: each
-      // thread walks a contiguous slice (an odd length keeps a warp's threads on
-      // distinct banks) and sums every token's residuals in a register
+      // survivor filter (dead entries marked in place) and the changes of the
+      // gains: an entry's residual moves from C - b_old to C - b_new, or to zero
+      // when it dies (exact: integers modulo 2^64; nothing for rows whose
+      // coverage stayed).  Each thread walks a contiguous slice (an odd length
+      // keeps a warp's threads on distinct banks) and sums every token's
+      // changes in a register
       const int tot = s.scal[SC_CURSOR];
       const int per = ((tot + SEL_THREADS - 1) / SEL_THREADS) | 1;
       const int p0s = min(tot, (int)threadIdx.x * per), p1s = min(tot, p0s + per);
@@ -691,18 +695,20 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
 #pragma unroll
         for (int u = 0; u < FU; ++u) {
           if (qq[u] == DEADROW) continue;
-          if (cc[u] > s.bcov[qq[u]]) {
-            if (jj[u] != jc) {
-              if (acc) gain_add(jc, acc, rnd);
-              if (nj) atomicAdd(&s.bnd[jc], nj);
-              jc = jj[u];
-              acc = 0;
-              nj = 0;
-            }
-            acc += (unsigned long long)(to_fix(cc[u], fxs) - s.bfix[qq[u]]);
+          if (jj[u] != jc) {
+            if (acc) gain_add(jc, acc, rnd);
+            if (nj) atomicAdd(&s.bnd[jc], nj);
+            jc = jj[u];
+            acc = 0;
+            nj = 0;
+          }
+          const int q = qq[u];
+          if (cc[u] > s.bcov[q]) {
+            acc += (unsigned long long)(s.bfold[q] - s.bfix[q]);
             ++nj;
             ++mylive;
           } else {
+            acc += (unsigned long long)(s.bfold[q] - to_fix(cc[u], fxs));
             s.srows[p0 + u] = (uint16_t)DEADROW;
           }
         }
@@ -792,9 +798,13 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
         }
       }
       bnew = group_max(bnew, gm);
-      const long long fb_new = to_fix(bnew, fxs);
-      int w = 0;
-      for (int base = 0; base < n; base += UNR * G) {
+      const long long fb_new = to_fix(bnew, fxs), fb_old = to_fix(bm, fxs);
+      // a row whose coverage stayed keeps its list and changes no gain; in the
+      // others an entry's residual moves from C - b_old to C - b_new, or to zero
+      // when it dies (exact: integers modulo 2^64)
+      const int nch = bnew > bm ? n : 0;  // uniform over the group
+      int w = n - nch;
+      for (int base = 0; base < nch; base += UNR * G) {
         float c[UNR];
         int jj[UNR];
 #pragma unroll
@@ -809,11 +819,14 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
           const int k = base + u * G + gl;
           const bool keep = k < n && c[u] > bnew;
           const unsigned msk = __ballot_sync(gm, keep);
+          if (k < n) {
+            const long long d = keep ? fb_old - fb_new : fb_old - to_fix(c[u], fxs);
+            if (d) gain_add(jj[u], (unsigned long long)d, rnd);
+          }
           if (keep) {
             const int pos = w + __popc(msk & lt);
             vals[pos] = c[u];
             cols[pos] = (uint16_t)jj[u];
-            gain_add(jj[u], (unsigned long long)(to_fix(c[u], fxs) - fb_new), rnd);
           }
           w += __popc(msk);
         }
