@@ -19,7 +19,9 @@
 //
 // One CTA computes one 128 x BN output tile (BN = 128 or 256, one TMEM column
 // per output column).  Warp 0 / lane 0 streams 64-wide K slices of the A and B
-// row blocks with TMA (128-byte swizzle) through a 4-stage mbarrier ring; warp
+// row blocks with TMA (128-byte swizzle) through an mbarrier ring of ST stages
+// (4; 2 when the grid holds more tiles than SMs: two CTAs then share an SM and
+// one's epilogue overlaps the other's products); warp
 // 1 / lane 0 issues tcgen05.mma (M = 128, N = BN, K = 16).  Then all 8 warps
 // drain TMEM: warp w reads lane quarter w % 4 and half w / 4 of the columns in
 // 32-column chunks, applies the row and column scales and stores each chunk
@@ -45,7 +47,7 @@
 namespace gmc {
 
 namespace {
-constexpr int GM = 128, GK = 64, GSTAGES = 4;
+constexpr int GM = 128, GK = 64, GSTAGES = 4;  // ring stages: at most GSTAGES
 constexpr int G_THREADS = 256;
 constexpr int GA_BYTES = GM * GK * 2;  // 16 KiB per stage
 constexpr long long G_WAIT = 4000000000LL;
@@ -68,13 +70,13 @@ template <int BN> __host__ __device__ __forceinline__ int sym_first_col(int I) {
   return x <= 0 ? 0 : (x + BN - 1) / BN;
 }
 
-template <int BN> constexpr size_t gemm_smem() {
-  return 1024 + (size_t)GSTAGES * (GA_BYTES + BN * GK * 2) + sizeof(GemmCtl) + sizeof(float) * (GM + BN);
+template <int BN, int ST> constexpr size_t gemm_smem() {
+  return 1024 + (size_t)ST * (GA_BYTES + BN * GK * 2) + sizeof(GemmCtl) + sizeof(float) * (GM + BN);
 }
 }  // namespace
 
-template <int BN>
-__global__ void __launch_bounds__(G_THREADS, 1)
+template <int BN, int ST>
+__global__ void __launch_bounds__(G_THREADS, ST == 2 ? 2 : 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap bmap,
               GemmArgs g) {
   grid_dep_wait();
@@ -83,8 +85,8 @@ __global__ void __launch_bounds__(G_THREADS, 1)
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* tilesA = base;
-  uint8_t* tilesB = base + GSTAGES * GA_BYTES;
-  GemmCtl* ctl = reinterpret_cast<GemmCtl*>(base + GSTAGES * (GA_BYTES + B_BYTES));
+  uint8_t* tilesB = base + ST * GA_BYTES;
+  GemmCtl* ctl = reinterpret_cast<GemmCtl*>(base + ST * (GA_BYTES + B_BYTES));
   float* rs = reinterpret_cast<float*>(ctl + 1);  // [GM] row scales of the tile
   float* cs = rs + GM;                            // [BN] column scales
 
@@ -117,7 +119,7 @@ __global__ void __launch_bounds__(G_THREADS, 1)
   const int nk = ceil_div(g.Kd, GK);
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < GSTAGES; ++s) {
+    for (int s = 0; s < ST; ++s) {
       tc::mbar_init(&ctl->full[s], 1);
       tc::mbar_init(&ctl->empty[s], 1);
     }
@@ -141,9 +143,9 @@ __global__ void __launch_bounds__(G_THREADS, 1)
   if (warp == 0) {
     if (lane == 0) {
       for (int kb = 0; kb < nk; ++kb) {
-        const int s = kb % GSTAGES;
-        const uint32_t ph = (uint32_t)(kb / GSTAGES) & 1u;
-        if (kb >= GSTAGES && !tc::mbar_wait(&ctl->empty[s], ph ^ 1u, deadline)) {
+        const int s = kb % ST;
+        const uint32_t ph = (uint32_t)(kb / ST) & 1u;
+        if (kb >= ST && !tc::mbar_wait(&ctl->empty[s], ph ^ 1u, deadline)) {
           ctl->abort = 1;
           break;
         }
@@ -159,8 +161,8 @@ __global__ void __launch_bounds__(G_THREADS, 1)
     if (lane == 0) {
       const uint32_t idesc = tc::idesc_bf16_f32(GM, BN);
       for (int kb = 0; kb < nk; ++kb) {
-        const int s = kb % GSTAGES;
-        const uint32_t ph = (uint32_t)(kb / GSTAGES) & 1u;
+        const int s = kb % ST;
+        const uint32_t ph = (uint32_t)(kb / ST) & 1u;
         if (!tc::mbar_wait(&ctl->full[s], ph, deadline)) {
           ctl->abort = 1;
           break;
@@ -238,8 +240,8 @@ __global__ void __launch_bounds__(G_THREADS, 1)
   if (warp == 0 && lane == 0 && !ok) {
     // drain TMA copies still in flight into this CTA's shared memory
     const long long d2 = clock64() + G_WAIT;
-    for (int kb = (issued > GSTAGES ? issued - GSTAGES : 0); kb < issued; ++kb)
-      if (!tc::mbar_wait(&ctl->full[kb % GSTAGES], (uint32_t)(kb / GSTAGES) & 1u, d2)) break;
+    for (int kb = (issued > ST ? issued - ST : 0); kb < issued; ++kb)
+      if (!tc::mbar_wait(&ctl->full[kb % ST], (uint32_t)(kb / ST) & 1u, d2)) break;
   }
   tc::fence_before_sync();
   __syncthreads();
@@ -249,6 +251,16 @@ __global__ void __launch_bounds__(G_THREADS, 1)
 // ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
+template <int BN, int ST>
+static cudaError_t launch_gemm_st(const CUtensorMap& am, const CUtensorMap& bm, const GemmArgs& g,
+                                  dim3 grid, cudaStream_t st) {
+  const size_t smem = gemm_smem<BN, ST>();
+  cudaError_t e;
+  if ((e = set_smem_limit((const void*)k_gemm_tc<BN, ST>, smem)) != cudaSuccess) return e;
+  launch_k(k_gemm_tc<BN, ST>, grid, G_THREADS, smem, st, 1, am, bm, g);
+  return cudaGetLastError();
+}
+
 template <int BN>
 static cudaError_t launch_gemm_bn(const GemmArgs& g, const void* A, long long a_rows, int lda,
                                   const void* Bm, long long b_rows, int ldb, cudaStream_t st) {
@@ -258,13 +270,17 @@ static cudaError_t launch_gemm_bn(const GemmArgs& g, const void* A, long long a_
   if ((e = make_tmap_bf16(&bm, Bm, (uint64_t)g.Kd, (uint64_t)b_rows, (uint64_t)ldb, BN)) !=
       cudaSuccess)
     return e;
-  const size_t smem = gemm_smem<BN>();
-  if ((e = set_smem_limit((const void*)k_gemm_tc<BN>, smem)) != cudaSuccess) return e;
   dim3 grid(ceil_div(g.Nn, BN), ceil_div(g.M, GM), g.B);
   if (g.m_fast) grid = dim3(ceil_div(g.M, GM), ceil_div(g.Nn, BN), g.B);
   if (g.sym) grid = dim3(gemm_sym_ctas(g.M, 1), 1, g.B);  // the computed tiles of every image
-  launch_k(k_gemm_tc<BN>, grid, G_THREADS, smem, st, 1, am, bm, g);
-  return cudaGetLastError();
+  static int sms = 0;
+  if (sms == 0 && cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, 0) != cudaSuccess) {
+    cudaGetLastError();
+    sms = 152;
+  }
+  // more tiles than SMs: two CTAs per SM with two stages each
+  if ((long long)grid.x * grid.y * grid.z > sms) return launch_gemm_st<BN, 2>(am, bm, g, grid, st);
+  return launch_gemm_st<BN, GSTAGES>(am, bm, g, grid, st);
 }
 
 int gemm_sym_ctas(int N, int B) {  // symmetric Grams use 128 x 256 tiles (N > 128)
