@@ -63,6 +63,7 @@ constexpr int PCL = 8;     // pool entries a lane keeps in registers (8 lanes x 
 constexpr int DEADROW = 0xFFFF;  // flat mode: row id of an entry whose residual is zero
 constexpr int FU = 4;      // flat mode: entries a thread loads ahead in a walk
 constexpr int CU = 8;      // flat mode: entries a thread moves per compaction chunk
+constexpr int COMPACT_EVERY = 4;  // flat mode: rounds between compactions of the survivor lists
 constexpr size_t SMEM_LIMIT = 227 * 1024;
 
 struct SelArgs {
@@ -715,12 +716,14 @@ __global__ void __launch_bounds__(SEL_THREADS, 1) k_select(SelArgs a) {
       }
       if (acc) gain_add(jc, acc, rnd);
       if (nj) atomicAdd(&s.bnd[jc], nj);
-      // Once fewer than 60% of the entries are live, drop the dead ones: the
-      // live entries move down in order (token-major order is kept) and the
-      // token segments restart at the prefix sums of the live counts.
+      // Every fourth round every CTA drops its dead entries: the live entries
+      // move down in order (token-major order is kept) and the token segments
+      // restart at the prefix sums of the live counts.  The same round in every
+      // CTA: a compaction in one CTA alone would hold the others at the next
+      // cluster barrier.
       int live = 0;
       block_exclusive_scan(mylive, s.wsum, &live);
-      if (live * 5 < tot * 3) {
+      if (rnd % COMPACT_EVERY == 0 && live < tot) {  // live, tot: block-wide values
         {
           const int perj = (N + SEL_THREADS - 1) / SEL_THREADS;
           const int j0 = min(N, (int)threadIdx.x * perj), j1 = min(N, j0 + perj);
