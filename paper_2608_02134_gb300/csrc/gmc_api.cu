@@ -155,7 +155,8 @@ size_t carve_compress(const Dims& dm, Scratch* s, char* base, R0State* r0s = nul
   Scratch t{};
   const size_t B = dm.B, N = dm.N, H = dm.H, T = dm.T, M = dm.M, K = dm.K;
   t.nP = ceil_div(dm.N, PROBE_TOK);
-  t.nHG = ceil_div(dm.N, HG_TOK);
+  t.hgtok = head_tokens(dm.B, dm.N, dm.H);
+  t.nHG = ceil_div(dm.N, t.hgtok);
   t.nA = assign_blocks(dm.N);
   t.nE = t.nA;  // energy block sums come from the assignment gap kernel
   t.nSel = 0;

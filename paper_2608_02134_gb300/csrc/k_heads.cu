@@ -14,8 +14,6 @@
 namespace gmc {
 
 constexpr int HG_TC = 32;                       // queries per staged chunk
-constexpr int HG_RS = HG_TC * HG_TOK + 2;       // row stride of a staged head: 4 rows apart
-                                                // land 8 banks apart
 constexpr int HG_HB = 4;                        // heads per register tile side
 
 __device__ __forceinline__ float query_weight(int t, int Tb, float wq) {
@@ -26,16 +24,19 @@ __device__ __forceinline__ int pair_index(int h, int g, int H) {  // h <= g, h-m
   return h * H - h * (h - 1) / 2 + (g - h);
 }
 
-// Per block: HG_TOK tokens, all head pairs (h <= g).  Writes the block's part
-// of the pattern Gram (an fp32 sum over its HG_TOK tokens, stored as fp64 for
+// Per block: TOK tokens (8, or 9 where that puts one image's blocks in one wave), all head
+// pairs (h <= g).  Writes the block's part
+// of the pattern Gram (an fp32 sum over its TOK tokens, stored as fp64 for
 // the cross-block sum) and W2[h,i] = sum_t nu_t A[h,t,i]^2.  The per-token
 // sums over queries are register tiles of 4 x 4 head pairs: 8 shared loads
 // feed 16 FMAs.
+template <int TOK>
 __global__ void k_head_stats(const float* __restrict__ A, const float* __restrict__ Z,
                              const float* __restrict__ sigma, const int32_t* toff, int B, int N,
                              int Tmax, int H, float wq, double* hgpart, int nHG, float* W2,
                              uint32_t* status) {
   grid_dep_wait();
+  constexpr int RS = HG_TC * TOK + 2;  // row stride of a staged head: 4 rows apart land 8 banks apart
   extern __shared__ float sm_hs[];
   __shared__ float sgm[GMC_MAX_HEADS];  // sigma_h of the image
   const int b = blockIdx.y;
@@ -46,17 +47,17 @@ __global__ void k_head_stats(const float* __restrict__ A, const float* __restric
   const int npairs = H * (H + 1) / 2;
   const int nhb = (H + HG_HB - 1) / HG_HB, Hp = nhb * HG_HB;
   const int ntiles = nhb * (nhb + 1) / 2;
-  float* Abuf = sm_hs;                          // [2][Hp][HG_RS], rows >= H stay zero
-  float* acc = Abuf + 2 * (size_t)Hp * HG_RS;   // [2][npairs][HG_TOK], one per block half
-  float* w2 = acc + 2 * (size_t)npairs * HG_TOK;  // [2][H][HG_TOK]
-  float4* zs = reinterpret_cast<float4*>(w2 + 2 * H * HG_TOK);  // [H][HG_TOK] probe values
-  unsigned short* tiles = reinterpret_cast<unsigned short*>(zs + H * HG_TOK);  // [ntiles]
-  const int i0 = blockIdx.x * HG_TOK;
-  for (int p = threadIdx.x; p < 2 * npairs * HG_TOK; p += blockDim.x) acc[p] = 0.f;
-  for (int p = threadIdx.x; p < 2 * H * HG_TOK; p += blockDim.x) w2[p] = 0.f;
-  for (int p = H * HG_RS + threadIdx.x; p < Hp * HG_RS; p += blockDim.x) {
+  float* Abuf = sm_hs;                          // [2][Hp][RS], rows >= H stay zero
+  float* acc = Abuf + 2 * (size_t)Hp * RS;   // [2][npairs][TOK], one per block half
+  float* w2 = acc + 2 * (size_t)npairs * TOK;  // [2][H][TOK]
+  float4* zs = reinterpret_cast<float4*>(w2 + 2 * H * TOK);  // [H][TOK] probe values
+  unsigned short* tiles = reinterpret_cast<unsigned short*>(zs + H * TOK);  // [ntiles]
+  const int i0 = blockIdx.x * TOK;
+  for (int p = threadIdx.x; p < 2 * npairs * TOK; p += blockDim.x) acc[p] = 0.f;
+  for (int p = threadIdx.x; p < 2 * H * TOK; p += blockDim.x) w2[p] = 0.f;
+  for (int p = H * RS + threadIdx.x; p < Hp * RS; p += blockDim.x) {
     Abuf[p] = 0.f;
-    Abuf[(size_t)Hp * HG_RS + p] = 0.f;
+    Abuf[(size_t)Hp * RS + p] = 0.f;
   }
   if (threadIdx.x == 0) {
     int p = 0;
@@ -64,25 +65,25 @@ __global__ void k_head_stats(const float* __restrict__ A, const float* __restric
       for (int gb = hb; gb < nhb; ++gb) tiles[p++] = (unsigned short)(hb * 256 + gb);
   }
   // the block's probe values Z_h[i] for every head (used by the output step)
-  for (int q = threadIdx.x; q < H * HG_TOK; q += blockDim.x) {
-    const int h = q / HG_TOK, i = i0 + q % HG_TOK;
+  for (int q = threadIdx.x; q < H * TOK; q += blockDim.x) {
+    const int h = q / TOK, i = i0 + q % TOK;
     zs[q] = i < N ? reinterpret_cast<const float4*>(Z)[((size_t)b * H + h) * N + i]
                   : make_float4(0.f, 0.f, 0.f, 0.f);
   }
   // Queries in pairs of HG_TC-chunks: both are staged, then the two halves of
-  // the block work on one chunk each into their own sums.  The HG_TOK tokens
+  // the block work on one chunk each into their own sums.  The TOK tokens
   // of one (head, query) row are read as 16-byte loads when the rows of A
   // start on 16 bytes (N % 4 == 0) and the block is not the ragged last one
   // (the padded shared rows are not 16-byte aligned, so these go through
   // registers); otherwise as 4-byte cp.async copies.
-  const bool vec = (N & 3) == 0 && i0 + HG_TOK <= N;
+  const bool vec = TOK % 4 == 0 && (N & 3) == 0 && i0 + TOK <= N;
   auto stage = [&](int t0, float* buf) {
     const int tc = min(HG_TC, Tb - t0);
     if (vec) {
-      constexpr int V = HG_TOK / 4;  // 16-byte pieces per row
+      constexpr int V = TOK / 4;  // 16-byte pieces per row
       for (int idx = threadIdx.x; idx < H * HG_TC * V; idx += blockDim.x) {
         const int h = idx / (HG_TC * V), tt = (idx / V) % HG_TC, v = idx % V;
-        float* dst = buf + h * HG_RS + tt * HG_TOK + 4 * v;
+        float* dst = buf + h * RS + tt * TOK + 4 * v;
         float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
         if (tt < tc)
           x = *reinterpret_cast<const float4*>(A + (((size_t)b * H + h) * Tmax + t0 + tt) * N + i0 +
@@ -93,32 +94,32 @@ __global__ void k_head_stats(const float* __restrict__ A, const float* __restric
         dst[3] = x.w;
       }
     } else {
-      for (int idx = threadIdx.x; idx < H * HG_TC * HG_TOK; idx += blockDim.x) {
-        const int h = idx / (HG_TC * HG_TOK), tt = (idx / HG_TOK) % HG_TC, ii = idx % HG_TOK;
+      for (int idx = threadIdx.x; idx < H * HG_TC * TOK; idx += blockDim.x) {
+        const int h = idx / (HG_TC * TOK), tt = (idx / TOK) % HG_TC, ii = idx % TOK;
         const bool in = tt < tc && i0 + ii < N;
         const float* src = in ? A + (((size_t)b * H + h) * Tmax + t0 + tt) * N + i0 + ii : A;
-        cp_async4(buf + h * HG_RS + tt * HG_TOK + ii, src, in);
+        cp_async4(buf + h * RS + tt * TOK + ii, src, in);
       }
     }
     cp_async_commit();
   };
   const int hsz = blockDim.x / 2, half = threadIdx.x / hsz, ht = threadIdx.x % hsz;
-  float* accH = acc + (size_t)half * npairs * HG_TOK;
-  float* w2H = w2 + (size_t)half * H * HG_TOK;
+  float* accH = acc + (size_t)half * npairs * TOK;
+  float* w2H = w2 + (size_t)half * H * TOK;
   for (int tp = 0; tp < Tb; tp += 2 * HG_TC) {
     __syncthreads();  // both buffers are free
     stage(tp, Abuf);
-    stage(tp + HG_TC, Abuf + (size_t)Hp * HG_RS);
+    stage(tp + HG_TC, Abuf + (size_t)Hp * RS);
     cp_async_wait<0>();
     __syncthreads();
     const int t0 = tp + half * HG_TC;
     const int tc = max(0, min(HG_TC, Tb - t0));
-    const float* Ablk = Abuf + (size_t)half * Hp * HG_RS;
-    for (int task = ht; task < ntiles * HG_TOK; task += hsz) {
-      const int tile = task / HG_TOK, ii = task % HG_TOK;
+    const float* Ablk = Abuf + (size_t)half * Hp * RS;
+    for (int task = ht; task < ntiles * TOK; task += hsz) {
+      const int tile = task / TOK, ii = task % TOK;
       const int hb = tiles[tile] >> 8, gb = tiles[tile] & 255;
-      const float* ah = Ablk + (size_t)hb * HG_HB * HG_RS + ii;
-      const float* ag = Ablk + (size_t)gb * HG_HB * HG_RS + ii;
+      const float* ah = Ablk + (size_t)hb * HG_HB * RS + ii;
+      const float* ag = Ablk + (size_t)gb * HG_HB * RS + ii;
       float sacc[HG_HB][HG_HB];
 #pragma unroll
       for (int u = 0; u < HG_HB; ++u)
@@ -128,8 +129,8 @@ __global__ void k_head_stats(const float* __restrict__ A, const float* __restric
         float x[HG_HB], y[HG_HB];
 #pragma unroll
         for (int u = 0; u < HG_HB; ++u) {
-          x[u] = ah[u * HG_RS + tt * HG_TOK];
-          y[u] = ag[u * HG_RS + tt * HG_TOK];
+          x[u] = ah[u * RS + tt * TOK];
+          y[u] = ag[u * RS + tt * TOK];
         }
 #pragma unroll
         for (int u = 0; u < HG_HB; ++u)
@@ -141,15 +142,15 @@ __global__ void k_head_stats(const float* __restrict__ A, const float* __restric
 #pragma unroll
         for (int v = 0; v < HG_HB; ++v) {
           const int h = hb * HG_HB + u, g = gb * HG_HB + v;
-          if (h <= g && g < H) accH[pair_index(h, g, H) * HG_TOK + ii] += sacc[u][v];
+          if (h <= g && g < H) accH[pair_index(h, g, H) * TOK + ii] += sacc[u][v];
         }
     }
-    for (int q = ht; q < H * HG_TOK; q += hsz) {
-      const int h = q / HG_TOK, ii = q % HG_TOK;
-      const float* ah = Ablk + h * HG_RS;
+    for (int q = ht; q < H * TOK; q += hsz) {
+      const int h = q / TOK, ii = q % TOK;
+      const float* ah = Ablk + h * RS;
       float sw = 0.f;
       for (int tt = 0; tt < tc; ++tt) {
-        const float a = ah[tt * HG_TOK + ii];
+        const float a = ah[tt * TOK + ii];
         sw = fmaf(query_weight(t0 + tt, Tb, wq) * a, a, sw);
       }
       w2H[q] += sw;
@@ -163,20 +164,20 @@ __global__ void k_head_stats(const float* __restrict__ A, const float* __restric
     const int pi = pair_index(h, g, H);
     const float sh = sgm[h], sgv = sgm[g];
     float v = 0.f;
-    for (int ii = 0; ii < HG_TOK; ++ii) {
+    for (int ii = 0; ii < TOK; ++ii) {
       const int i = i0 + ii;
       if (i >= N) break;
-      const float4 zh = zs[h * HG_TOK + ii];
-      const float4 zg = zs[g * HG_TOK + ii];
+      const float4 zh = zs[h * TOK + ii];
+      const float4 zg = zs[g * TOK + ii];
       const float w = fmaf(zh.x, zg.x, fmaf(zh.y, zg.y, fmaf(zh.z, zg.z, fmaf(zh.w, zg.w, sh * sgv))));
-      v = fmaf(w, acc[pi * HG_TOK + ii] + acc[((size_t)npairs + pi) * HG_TOK + ii], v);
+      v = fmaf(w, acc[pi * TOK + ii] + acc[((size_t)npairs + pi) * TOK + ii], v);
     }
     out[h * H + g] = v;
     out[g * H + h] = v;
   }
-  for (int q = threadIdx.x; q < H * HG_TOK; q += blockDim.x) {
-    const int h = q / HG_TOK, i = i0 + q % HG_TOK;
-    if (i < N) W2[((size_t)b * H + h) * N + i] = w2[q] + w2[H * HG_TOK + q];
+  for (int q = threadIdx.x; q < H * TOK; q += blockDim.x) {
+    const int h = q / TOK, i = i0 + q % TOK;
+    if (i < N) W2[((size_t)b * H + h) * N + i] = w2[q] + w2[H * TOK + q];
   }
 }
 
@@ -400,27 +401,46 @@ __global__ void __launch_bounds__(256) k_hg_reduce(const double* __restrict__ hg
 // Dynamic shared memory of k_head_stats for H heads: both staged query
 // chunks, both halves' pair sums and query-weighted squares, the probe values
 // and the tile list.
-static size_t head_stats_smem(int H) {
+static size_t head_stats_smem(int H, int tok) {
   const int npairs = H * (H + 1) / 2;
   const int nhb = (H + HG_HB - 1) / HG_HB;
-  return sizeof(float) * (2 * (size_t)nhb * HG_HB * HG_RS + 2 * (size_t)npairs * HG_TOK +
-                          2 * H * HG_TOK) +
-         sizeof(float4) * H * HG_TOK + sizeof(unsigned short) * (nhb * (nhb + 1) / 2) + 16;
+  const int rs = HG_TC * tok + 2;
+  return sizeof(float) * (2 * (size_t)nhb * HG_HB * rs + 2 * (size_t)npairs * tok + 2 * H * tok) +
+         sizeof(float4) * H * tok + sizeof(unsigned short) * (nhb * (nhb + 1) / 2) + 16;
+}
+
+int head_tokens(int B, int N, int H) {
+  static int sms = 0;
+  if (sms == 0) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+      cudaGetLastError();
+      sms = 152;
+    }
+  }
+  const long long b8 = (long long)B * ceil_div(N, 8), b9 = (long long)B * ceil_div(N, 9);
+  return b8 > sms && b9 <= sms && head_stats_smem(H, 9) <= 227 * 1024 ? 9 : 8;
 }
 
 // Whether the head statistics of H heads fit one block's shared memory
 // (227 KB on sm_103a): H <= 56.
-bool heads_supported(int H) { return H >= 1 && head_stats_smem(H) <= 227 * 1024; }
+bool heads_supported(int H) { return H >= 1 && head_stats_smem(H, 8) <= 227 * 1024; }
 
 cudaError_t launch_heads(const Dims& dm, const gmc_params& p, Scratch& s, const TraceView& tv,
                          cudaStream_t st, int cluster, const ViewGrams* views) {
   const int H = dm.H;
-  const size_t smem = head_stats_smem(H);
-  cudaError_t e = set_smem_limit((const void*)k_head_stats, smem);
+  const int tok = s.hgtok;
+  const size_t smem = head_stats_smem(H, tok);
+  const void* kf = tok == 9 ? (const void*)k_head_stats<9> : (const void*)k_head_stats<8>;
+  cudaError_t e = set_smem_limit(kf, smem);
   if (e != cudaSuccess) return e;
-  launch_k(k_head_stats, dim3(s.nHG, dm.B), 512, smem, st, 1, s.A, s.Z, s.sigma, dm.toff, dm.B, dm.N, dm.T,
-                                                     H, p.terminal_q_weight, s.hgpart, s.nHG,
-                                                     s.W2, s.status);
+  if (tok == 9)
+    launch_k(k_head_stats<9>, dim3(s.nHG, dm.B), 512, smem, st, 1, s.A, s.Z, s.sigma, dm.toff, dm.B,
+             dm.N, dm.T, H, p.terminal_q_weight, s.hgpart, s.nHG, s.W2, s.status);
+  else
+    launch_k(k_head_stats<8>, dim3(s.nHG, dm.B), 512, smem, st, 1, s.A, s.Z, s.sigma, dm.toff, dm.B,
+             dm.N, dm.T, H, p.terminal_q_weight, s.hgpart, s.nHG, s.W2, s.status);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   const size_t smem2 = sizeof(float) * ((size_t)H * H + 3 * H + 2 * GMC_MAX_HEADS) +
                        sizeof(int) * (H + 2 * GMC_MAX_HEADS);

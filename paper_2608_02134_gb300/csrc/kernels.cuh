@@ -114,6 +114,7 @@ struct Scratch {
   int32_t* fexp;     // [B]            select-path fixed-point exponents
   __nv_bfloat16* Qp; // [B][Hkv][RQ][d] packed text queries of each KV group (tcgen05 path)
   int nP, nHG, nA, nSel, nE, nRS;
+  int hgtok;         // tokens per head-statistics block (nHG = ceil(N / hgtok))
   // Message views: A, rs, mpart, Z, zn2, sigpart, sigma, hgpart, HG, W2, Qp, the
   // probe tickets (tick) and the head-Gram tickets (tick3) hold V consecutive
   // per-view blocks; the pointers above address view 0 (the current view).
@@ -129,7 +130,8 @@ struct Scratch {
 };
 
 constexpr int ROWS_PER_BLOCK = 8;  // rownorm / probe / client builder blocks
-constexpr int HG_TOK = 8;          // tokens per head-statistics block
+int head_tokens(int B, int N, int H);  // tokens per head-statistics block: 8, or 9 where
+                                      // that puts every block in one wave
 constexpr int ASSIGN_WARPS = 16;   // warps per assignment block (32 tokens, one per lane)
 int assign_blocks(int N);          // assignment blocks per image
 constexpr int PROBE_TOK = 32;       // tokens per probe block
