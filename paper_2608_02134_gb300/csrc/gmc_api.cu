@@ -558,7 +558,7 @@ static int compress_impl(const gmc_problem* prob, const gmc_params* params,
   // then the current view's, whose last block clusters the heads over all views
   auto probes = [&]() -> cudaError_t {
     for (int v = 0; v < V; ++v) {
-      const cudaError_t e = launch_probe(dm, vkeys[v], vprobe[v], p, sv[v], st);
+      const cudaError_t e = launch_probe(dm, vkeys[v], vprobe[v], vqueries[v], p, sv[v], st);
       if (e != cudaSuccess) return e;
     }
     return cudaSuccess;
@@ -577,7 +577,7 @@ static int compress_impl(const gmc_problem* prob, const gmc_params* params,
     }
     return launch_heads(dm, p, sv[0], tv, st, 1, V > 1 ? &vg : nullptr);
   };
-  const int msg_k = (message_tc_supported(dm) ? 3 : 1) * V;
+  const int msg_k = (message_tc_supported(dm) ? 2 : 1) * V;  // at most two launches per view
   GMC_TRY(g_prof.begin(st));  // k_rownorm zeroes the column sums u0 of the client build
   // the appearance branch: cosine Gram, or on long prefixes the projection,
   // the split unit states and the bounded bank's cosines

@@ -120,30 +120,6 @@ __device__ __forceinline__ void epi_barrier() {
 }
 }  // namespace
 
-// Q [T_b rows][H][d] of every image -> Qp [B][Hkv][RQ][d], row j*T_b + t of
-// group g holding query head g*grp + j; rows >= grp*T_b are zero.
-__global__ void k_pack_q(const __nv_bfloat16* __restrict__ queries, const int32_t* toff, int B,
-                         int Tmax, int H, int Hkv, int d, int RQ, __nv_bfloat16* Qp,
-                         uint32_t* status) {
-  grid_dep_wait();
-  const int b = blockIdx.z, g = blockIdx.y;
-  const TextGeom tg = text_geom(toff, b, B, Tmax, status);
-  const int grp = H / Hkv;
-  const int lane = threadIdx.x & 31;
-  const int row = blockIdx.x * 8 + (threadIdx.x >> 5);
-  if (row >= RQ) return;
-  uint4* dst = reinterpret_cast<uint4*>(Qp + (((size_t)b * Hkv + g) * RQ + row) * d);
-  const int nv = d / 8;
-  if (tg.T > 0 && row < grp * tg.T) {
-    const int j = row / tg.T, t = row % tg.T;
-    const uint4* src = reinterpret_cast<const uint4*>(
-        queries + ((size_t)tg.off + t) * H * d + (size_t)(g * grp + j) * d);
-    for (int q = lane; q < nv; q += 32) dst[q] = src[q];
-  } else {
-    for (int q = lane; q < nv; q += 32) dst[q] = make_uint4(0, 0, 0, 0);
-  }
-}
-
 __global__ void __launch_bounds__(THREADS, 1)
     k_message_tc(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
                  const int32_t* toff, int B, int N, int Tmax, int H, int Hkv, int d, int RQ,
@@ -641,13 +617,13 @@ int message_splits(const Dims& dm) {
   return message_tc_supported(dm) ? msg_split(dm.B, dm.Hkv, message_rq(dm), dm.N, dm.T).n : 1;
 }
 
+// The packed queries Qp are written by the probe kernel, launched before this
+// one on the same stream (k_prep.cu).
 cudaError_t launch_message_tc(const Dims& dm, const void* keys, const void* queries, Scratch& s,
                               cudaStream_t st) {
+  (void)queries;
   const int RQ = message_rq(dm);
-  launch_k(k_pack_q, dim3(ceil_div(RQ, 8), dm.Hkv, dm.B), 256, 0, st, 1,
-      (const __nv_bfloat16*)queries, dm.toff, dm.B, dm.T, dm.H, dm.Hkv, dm.d, RQ, s.Qp, s.status);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
+  cudaError_t e;
   CUtensorMap qmap, kmap;
   if ((e = make_tmap_bf16(&qmap, s.Qp, dm.d, (uint64_t)dm.B * dm.Hkv * RQ, dm.d, BM)) != cudaSuccess)
     return e;

@@ -53,18 +53,37 @@ __global__ void k_rownorm(const Tin* __restrict__ hidden, const int32_t* toff, i
 // W_h are staged in shared memory, one thread per (token, head) computes the
 // four probe coordinates.  The last block of an image to finish (a ticket per
 // image, zeroed with the status word) sums the partials in a fixed order.
+// With Qp (the tensor-core message slice follows), the blocks of KV group g
+// also write the group's packed text queries first: Qp [B][Hkv][RQ][d], row
+// j*T_b + t holding query head g*grp + j at text position t, rows >= grp*T_b
+// zero (block pb: rows pb, pb + nP, ...).
 constexpr int PR_TOK = PROBE_TOK;
 
 template <typename Tin>
 __global__ void __launch_bounds__(256) k_probe(
     const Tin* __restrict__ keys, const float* __restrict__ W, const int32_t* toff, int B, int N,
     int K, int Tmax, int H, int Hkv, int d, float lambda_mass, float eps_mass, float* Z,
-    float* zn2, float* sigpart, int nP, float* sigma, uint32_t* tick, uint32_t* status) {
+    float* zn2, float* sigpart, int nP, float* sigma, uint32_t* tick,
+    const __nv_bfloat16* __restrict__ queries, int RQ, __nv_bfloat16* Qp, uint32_t* status) {
   grid_dep_wait();
   extern __shared__ float4 sm_probe4[];
   __shared__ int last;
   const int b = blockIdx.z, g = blockIdx.y, pb = blockIdx.x;
   const TextGeom tg = text_geom(toff, b, B, Tmax, status);
+  if (Qp) {
+    const int grp = H / Hkv, nv = d / 8;  // 16-byte pieces per row
+    for (int idx = threadIdx.x;; idx += blockDim.x) {
+      const int row = pb + (idx / nv) * nP, q = idx % nv;
+      if (row >= RQ) break;  // row grows with idx
+      uint4 v = make_uint4(0, 0, 0, 0);
+      if (tg.T > 0 && row < grp * tg.T) {
+        const int j = row / tg.T, t = row % tg.T;
+        v = reinterpret_cast<const uint4*>(queries + ((size_t)tg.off + t) * H * d +
+                                           (size_t)(g * grp + j) * d)[q];
+      }
+      reinterpret_cast<uint4*>(Qp + (((size_t)b * Hkv + g) * RQ + row) * d)[q] = v;
+    }
+  }
   if (tg.T == 0) return;  // uniform over the image
   const SeqIdx sq(b, N, K, tg.off, tg.T);
   const int grp = H / Hkv, HD = Hkv * d, i0 = pb * PR_TOK;
@@ -241,8 +260,12 @@ cudaError_t launch_rms_rows(const Dims& dm, const void* hidden, float* rmsh, uin
   return cudaGetLastError();
 }
 
-cudaError_t launch_probe(const Dims& dm, const void* keys, const float* W, const gmc_params& p,
-                         Scratch& s, cudaStream_t st) {
+cudaError_t launch_probe(const Dims& dm, const void* keys, const float* W, const void* queries,
+                         const gmc_params& p, Scratch& s, cudaStream_t st) {
+  const bool pack = message_tc_supported(dm);  // the packed queries of the tensor-core slice
+  const int RQ = pack ? message_rq(dm) : 0;
+  __nv_bfloat16* Qp = pack ? s.Qp : nullptr;
+  const __nv_bfloat16* q16 = static_cast<const __nv_bfloat16*>(queries);
   const int grp = dm.H / dm.Hkv;
   dim3 grid(s.nP, dm.Hkv, dm.B);
   const size_t smem = sizeof(float4) * grp * (dm.d + 1) +
@@ -252,13 +275,14 @@ cudaError_t launch_probe(const Dims& dm, const void* keys, const float* W, const
     if ((e = set_smem_limit((const void*)k_probe<__nv_bfloat16>, smem)) != cudaSuccess) return e;
     launch_k(k_probe<__nv_bfloat16>, grid, 256, smem, st, 1,
         (const __nv_bfloat16*)keys, W, dm.toff, dm.B, dm.N, dm.K, dm.T, dm.H, dm.Hkv, dm.d,
-        p.lambda_mass, p.eps_mass, s.Z, s.zn2, s.sigpart, s.nP, s.sigma, s.tick, s.status);
+        p.lambda_mass, p.eps_mass, s.Z, s.zn2, s.sigpart, s.nP, s.sigma, s.tick, q16, RQ, Qp,
+        s.status);
   } else {
     if ((e = set_smem_limit((const void*)k_probe<float>, smem)) != cudaSuccess) return e;
     launch_k(k_probe<float>, grid, 256, smem, st, 1, (const float*)keys, W, dm.toff, dm.B, dm.N, dm.K,
                                             dm.T, dm.H, dm.Hkv, dm.d, p.lambda_mass, p.eps_mass,
                                             s.Z, s.zn2, s.sigpart, s.nP, s.sigma, s.tick,
-                                            s.status);
+                                            q16, RQ, Qp, s.status);
   }
   return cudaGetLastError();
 }

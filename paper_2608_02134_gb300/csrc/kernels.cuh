@@ -138,7 +138,8 @@ constexpr int PROBE_TOK = 32;       // tokens per probe block
 
 // Launch wrappers.  Each returns the first CUDA error it saw.
 cudaError_t launch_rownorm(const Dims&, const void* hidden, float norm_eps, Scratch&, cudaStream_t);
-cudaError_t launch_probe(const Dims&, const void* keys, const float* W, const gmc_params&, Scratch&,
+cudaError_t launch_probe(const Dims&, const void* keys, const float* W, const void* queries,
+                         const gmc_params&, Scratch&,
                          cudaStream_t);
 cudaError_t launch_message(const Dims&, const void* keys, const void* queries, Scratch&,
                            cudaStream_t);
