@@ -29,12 +29,14 @@
 namespace gmc {
 
 namespace {
-constexpr int R0_ROWS = 8;  // warps per block; the responsibility kernels take one row per warp
-// The filters take `rpw` rows per warp (rows m0 + w + R0_ROWS * i).  More rows
+// Warps per block of the responsibility and filter kernels (ROWS, a template
+// parameter: 16 for one image, 8 for a batch; the responsibility kernels take
+// one row per warp).  The filters take `rpw` rows per warp (rows m0 + w +
+// ROWS * i).  More rows
 // per block mean fewer global atomics for the next gains (one per block and
 // column) but less parallelism: one row per warp is faster while the blocks
 // fit on the GPU at once, four when there are many more blocks than that.
-int filter_rows_per_warp(int B, int M) {
+int filter_rows_per_warp(int B, int M, int rows) {
   static int sms = 0;
   if (sms == 0) {
     int dev = 0;
@@ -44,7 +46,7 @@ int filter_rows_per_warp(int B, int M) {
       sms = 152;
     }
   }
-  const long long blocks = (long long)B * ceil_div(M, R0_ROWS);
+  const long long blocks = (long long)B * ceil_div(M, rows);
   return blocks > 32LL * sms ? 4 : 1;
 }
 }
@@ -129,7 +131,8 @@ __global__ void __launch_bounds__(512) k_r0_pool(const long long* __restrict__ u
   }
 }
 
-__global__ void __launch_bounds__(32 * R0_ROWS) k_r0_rho(
+template <int ROWS>
+__global__ void __launch_bounds__(32 * ROWS) k_r0_rho(
     const float* __restrict__ C, int B, int N, int Mstride, int H, int L2, const int32_t* toff,
     int Tmax, int uniform_rows, const int32_t* __restrict__ pool0, const int32_t* __restrict__ info,
     int P, float resp_temp, float resp_eps, int fx_exp, const int32_t* fexp, int I, long long* s0) {
@@ -142,7 +145,7 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_rho(
   if (Pt == 0) return;
   int Mb = Mstride;
   if (!uniform_rows) Mb = H * text_geom(toff, b, B, Tmax, nullptr).T + N + L2;
-  const int m0 = blockIdx.x * R0_ROWS;
+  const int m0 = blockIdx.x * ROWS;
   if (m0 >= Mb) return;
   const float fxs = ldexpf(1.f, fexp ? fexp[b] : fx_exp);
   for (int k = threadIdx.x; k < P; k += blockDim.x) {
@@ -187,7 +190,8 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_rho(
     if (sblk[k]) atomicAdd((unsigned long long*)&s0[(size_t)b * P + k], (unsigned long long)sblk[k]);
 }
 
-__global__ void __launch_bounds__(32 * R0_ROWS) k_r0_filter(
+template <int ROWS>
+__global__ void __launch_bounds__(32 * ROWS) k_r0_filter(
     float* C, uint16_t* scol, int B, int N, int K, int Mstride, int H, int L2,
     const int32_t* toff, int Tmax, int uniform_rows, const int32_t* __restrict__ pool0,
     int32_t* info, const long long* __restrict__ s0, int P, int bsz, int fx_exp,
@@ -208,7 +212,7 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_filter(
     MG = H * text_geom(toff, b, B, Tmax, nullptr).T;
     Mb = MG + N + L2;
   }
-  const int m0 = blockIdx.x * R0_ROWS * rpw;
+  const int m0 = blockIdx.x * ROWS * rpw;
   if (m0 >= Mb) return;
   const float fxs = ldexpf(1.f, fexp ? fexp[b] : fx_exp);
   const int nb = I > 1 ? Pt : min(bsz, min(Pt, K));  // a seed round takes its whole pool
@@ -242,7 +246,7 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_r0_filter(
   }
   const int lane = threadIdx.x & 31;
   for (int ir = 0; ir < rpw; ++ir) {
-    const int m = m0 + (threadIdx.x >> 5) + R0_ROWS * ir;
+    const int m = m0 + (threadIdx.x >> 5) + ROWS * ir;
     if (m >= Mb) break;
     float* vals = C + ((size_t)b * Mstride + m) * N;
     uint16_t* cols = scol + ((size_t)b * Mstride + m) * N;
@@ -400,7 +404,8 @@ __global__ void __launch_bounds__(512) k_rg_pool(const long long* __restrict__ u
   }
 }
 
-__global__ void __launch_bounds__(32 * R0_ROWS) k_rg_rho(
+template <int ROWS>
+__global__ void __launch_bounds__(32 * ROWS) k_rg_rho(
     const float* __restrict__ C, const uint16_t* __restrict__ scol,
     const float* __restrict__ bcov, const int32_t* __restrict__ cnt, int B, int N, int Mstride,
     int H, int L2, const int32_t* toff, int Tmax, int uniform_rows,
@@ -408,15 +413,15 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_rg_rho(
     float resp_eps, int fx_exp, const int32_t* fexp, long long* sc) {
   grid_dep_wait();
   __shared__ long long sblk[GMC_MAX_POOL];
-  __shared__ int fslot[R0_ROWS][GMC_MAX_POOL];  // a row's pool entries: slot and residual
-  __shared__ float fres[R0_ROWS][GMC_MAX_POOL];
+  __shared__ int fslot[ROWS][GMC_MAX_POOL];  // a row's pool entries: slot and residual
+  __shared__ float fres[ROWS][GMC_MAX_POOL];
   extern __shared__ short pslot[];              // [N] pool slot of every token or -1
   const int b = blockIdx.y;
   const int Pt = info[b * INFO_W];
   if (Pt == 0) return;
   int Mb = Mstride;
   if (!uniform_rows) Mb = H * text_geom(toff, b, B, Tmax, nullptr).T + N + L2;
-  const int m0 = blockIdx.x * R0_ROWS;
+  const int m0 = blockIdx.x * ROWS;
   if (m0 >= Mb) return;
   const float fxs = ldexpf(1.f, fexp ? fexp[b] : fx_exp);
   for (int j = threadIdx.x; j < N; j += blockDim.x) pslot[j] = -1;
@@ -482,7 +487,8 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_rg_rho(
     if (sblk[k]) atomicAdd((unsigned long long*)&sc[(size_t)b * P + k], (unsigned long long)sblk[k]);
 }
 
-__global__ void __launch_bounds__(32 * R0_ROWS) k_rg_filter(
+template <int ROWS>
+__global__ void __launch_bounds__(32 * ROWS) k_rg_filter(
     float* C, uint16_t* scol, int B, int N, int K, int Mstride, int H, int L2,
     const int32_t* toff, int Tmax, int uniform_rows, const int32_t* __restrict__ pool0,
     int32_t* info, const long long* __restrict__ sc0, int P, int bsz, int fx_exp,
@@ -499,7 +505,7 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_rg_filter(
   if (Pt == 0) return;
   int Mb = Mstride;
   if (!uniform_rows) Mb = H * text_geom(toff, b, B, Tmax, nullptr).T + N + L2;
-  const int m0 = blockIdx.x * R0_ROWS * rpw;
+  const int m0 = blockIdx.x * ROWS * rpw;
   if (m0 >= Mb) return;
   const int S = info[b * INFO_W + 3], rd = info[b * INFO_W + 4];
   const float fxs = ldexpf(1.f, fexp ? fexp[b] : fx_exp);
@@ -534,7 +540,7 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_rg_filter(
   __syncthreads();
   const int lane = threadIdx.x & 31;
   for (int ir = 0; ir < rpw; ++ir) {
-    const int m = m0 + (threadIdx.x >> 5) + R0_ROWS * ir;
+    const int m = m0 + (threadIdx.x >> 5) + ROWS * ir;
     if (m >= Mb) break;
     const size_t row = (size_t)b * Mstride + m;
     const int n = cnt[row];
@@ -610,6 +616,55 @@ __global__ void __launch_bounds__(32 * R0_ROWS) k_rg_filter(
     if (uacc[j]) atomicAdd(&ub[j], uacc[j]);
 }
 
+// The responsibility and filter launches of every whole-GPU round, ROWS rows per block.
+template <int ROWS>
+static cudaError_t launch_rounds_rows(const R0State& r0, int B, int N, int K, int M,
+                                      const int32_t* toff, int H, int T, int L2,
+                                      const gmc_params& p, int fx_exp, const int32_t* fexp,
+                                      float* C, uint16_t* scol, int32_t* order, const TraceView& tv,
+                                      cudaStream_t st, int I, size_t smem) {
+  const int P = p.pool_mult * p.batch_b;
+  const int uniform = (H == 0);
+  cudaError_t e;
+  dim3 grid(ceil_div(M, ROWS), B);
+  launch_k(k_r0_rho<ROWS>, grid, 32 * ROWS, 0, st, 1, C, B, N, M, H, L2, toff, T, uniform, r0.pool,
+           r0.info, P, p.resp_temp, p.resp_eps, fx_exp, fexp, I, r0.s0);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  const size_t fsm = sizeof(unsigned long long) * (size_t)N;
+  if ((e = set_smem_limit((const void*)k_r0_filter<ROWS>, fsm)) != cudaSuccess) return e;
+  const int rpw = filter_rows_per_warp(B, M, ROWS);
+  const dim3 fgrid(ceil_div(M, ROWS * rpw), B);
+  launch_k(k_r0_filter<ROWS>, fgrid, 32 * ROWS, fsm, st, 1, C, scol, B, N, K, M, H, L2, toff, T,
+           uniform, r0.pool, r0.info, r0.s0, P, p.batch_b, fx_exp, fexp, r0.u1, r0.bcov, r0.cnt,
+           r0.fv, order, rpw, I, tv);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  // sparse rounds: gains alternate between u1 and u2
+  // the pool kernel's layout is round 0's after the window scratch
+  const size_t psm = smem + sizeof(int) * (sel::WBINS + 4) + 12 * (size_t)sel::WCAP;
+  if ((e = set_smem_limit((const void*)k_rg_pool, psm)) != cudaSuccess) return e;
+  const size_t rsm = sizeof(short) * (size_t)N;
+  if ((e = set_smem_limit((const void*)k_rg_rho<ROWS>, rsm)) != cudaSuccess) return e;
+  const size_t gsm = sizeof(unsigned long long) * (size_t)N + (size_t)N;
+  if ((e = set_smem_limit((const void*)k_rg_filter<ROWS>, gsm)) != cudaSuccess) return e;
+  for (int rr = 1; rr <= sparse_gpu_rounds(N); ++rr) {
+    long long* ucur = rr % 2 == 1 ? r0.u1 : r0.u2;
+    long long* unext = rr % 2 == 1 ? r0.u2 : r0.u1;
+    launch_k(k_rg_pool, B, 512, psm, st, 1, (const long long*)ucur, unext, B, N, K, P,
+             uniform ? nullptr : toff, T, (const int32_t*)order, r0.pool, r0.info, r0.s0, tv);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    launch_k(k_rg_rho<ROWS>, grid, 32 * ROWS, rsm, st, 1, (const float*)C, (const uint16_t*)scol,
+             (const float*)r0.bcov, (const int32_t*)r0.cnt, B, N, M, H, L2, toff, T, uniform,
+             (const int32_t*)r0.pool, (const int32_t*)r0.info, P, p.resp_temp, p.resp_eps, fx_exp,
+             fexp, r0.s0);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    launch_k(k_rg_filter<ROWS>, fgrid, 32 * ROWS, gsm, st, 1, C, scol, B, N, K, M, H, L2, toff, T,
+             uniform, (const int32_t*)r0.pool, r0.info, (const long long*)r0.s0, P, p.batch_b,
+             fx_exp, fexp, unext, r0.bcov, r0.cnt, order, rpw, tv);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
 cudaError_t launch_round0(const R0State& r0, int B, int N, int K, int M, const int32_t* toff,
                           int H, int T, int L2, const gmc_params& p, int fx_exp,
                           const int32_t* fexp, float* C, uint16_t* scol, const long long* u0,
@@ -625,43 +680,13 @@ cudaError_t launch_round0(const R0State& r0, int B, int N, int K, int M, const i
   launch_k(k_r0_pool, B, 512, smem, st, 1, u0, B, N, P, uniform ? nullptr : toff, T, I, r0.pool, r0.info,
                                   r0.s0, r0.u1, r0.fv, status, tv);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  dim3 grid(ceil_div(M, R0_ROWS), B);
-  launch_k(k_r0_rho, grid, 32 * R0_ROWS, 0, st, 1, C, B, N, M, H, L2, toff, T, uniform, r0.pool, r0.info,
-                                          P, p.resp_temp, p.resp_eps, fx_exp, fexp, I, r0.s0);
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  const size_t fsm = sizeof(unsigned long long) * (size_t)N;
-  if ((e = set_smem_limit((const void*)k_r0_filter, fsm)) != cudaSuccess) return e;
-  const int rpw = filter_rows_per_warp(B, M);
-  const dim3 fgrid(ceil_div(M, R0_ROWS * rpw), B);
-  launch_k(k_r0_filter, fgrid, 32 * R0_ROWS, fsm, st, 1, C, scol, B, N, K, M, H, L2, toff, T, uniform, r0.pool,
-                                             r0.info, r0.s0, P, p.batch_b, fx_exp, fexp, r0.u1,
-                                             r0.bcov, r0.cnt, r0.fv, order, rpw, I, tv);
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  // sparse rounds: gains alternate between u1 and u2
-  // the pool kernel's layout is round 0's after the window scratch
-  const size_t psm = smem + sizeof(int) * (sel::WBINS + 4) + 12 * (size_t)sel::WCAP;
-  if ((e = set_smem_limit((const void*)k_rg_pool, psm)) != cudaSuccess) return e;
-  const size_t rsm = sizeof(short) * (size_t)N;
-  if ((e = set_smem_limit((const void*)k_rg_rho, rsm)) != cudaSuccess) return e;
-  const size_t gsm = sizeof(unsigned long long) * (size_t)N + (size_t)N;
-  if ((e = set_smem_limit((const void*)k_rg_filter, gsm)) != cudaSuccess) return e;
-  for (int rr = 1; rr <= sparse_gpu_rounds(N); ++rr) {
-    long long* ucur = rr % 2 == 1 ? r0.u1 : r0.u2;
-    long long* unext = rr % 2 == 1 ? r0.u2 : r0.u1;
-    launch_k(k_rg_pool, B, 512, psm, st, 1, (const long long*)ucur, unext, B, N, K, P,
-             uniform ? nullptr : toff, T, (const int32_t*)order, r0.pool, r0.info, r0.s0, tv);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    launch_k(k_rg_rho, grid, 32 * R0_ROWS, rsm, st, 1, (const float*)C, (const uint16_t*)scol,
-             (const float*)r0.bcov, (const int32_t*)r0.cnt, B, N, M, H, L2, toff, T, uniform,
-             (const int32_t*)r0.pool, (const int32_t*)r0.info, P, p.resp_temp, p.resp_eps, fx_exp,
-             fexp, r0.s0);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    launch_k(k_rg_filter, fgrid, 32 * R0_ROWS, gsm, st, 1, C, scol, B, N, K, M, H, L2, toff, T,
-             uniform, (const int32_t*)r0.pool, r0.info, (const long long*)r0.s0, P, p.batch_b,
-             fx_exp, fexp, unext, r0.bcov, r0.cnt, order, rpw, tv);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  }
-  return cudaSuccess;
+  // one image: 16 rows per block (fewer, larger blocks finish the rounds
+  // sooner); a batch: 8
+  if (B == 1)
+    return launch_rounds_rows<16>(r0, B, N, K, M, toff, H, T, L2, p, fx_exp, fexp, C, scol, order,
+                                  tv, st, I, smem);
+  return launch_rounds_rows<8>(r0, B, N, K, M, toff, H, T, L2, p, fx_exp, fexp, C, scol, order, tv,
+                               st, I, smem);
 }
 
 }  // namespace gmc
