@@ -348,18 +348,28 @@ def run_gmc(args):
     e2e_steps = min(args.steps, 20)
     eev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
            for _ in range(e2e_steps)]
+    def e2e_step():
+        if lp is None:
+            # gmc_compress_host: the library enqueues the copies, the hidden states'
+            # beside the probe, the message slice and the heads
+            comp.run_host(host, inp, out_host)
+        else:
+            for k in inp:
+                inp[k].copy_(host[k], non_blocking=True)
+            step()
+            out_host["idx"].copy_(comp.out_idx, non_blocking=True)
+            out_host["hidden"].copy_(comp.out_hidden, non_blocking=True)
+            out_host["kv"].copy_(comp.out_kv, non_blocking=True)
+            out_host["pos"].copy_(comp.out_pos, non_blocking=True)
+
+    for _ in range(args.warmup):
+        e2e_step()
     barrier()
     torch.cuda.synchronize(dev)
     for a, b in eev:
         flush.zero_()
         a.record(stream)
-        for k in inp:
-            inp[k].copy_(host[k], non_blocking=True)
-        step()
-        out_host["idx"].copy_(comp.out_idx, non_blocking=True)
-        out_host["hidden"].copy_(comp.out_hidden, non_blocking=True)
-        out_host["kv"].copy_(comp.out_kv, non_blocking=True)
-        out_host["pos"].copy_(comp.out_pos, non_blocking=True)
+        e2e_step()
         b.record(stream)
     torch.cuda.synchronize(dev)
     barrier()

@@ -203,6 +203,46 @@ int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* 
                  int32_t* out_idx, void* out_hidden, void* out_kv, int32_t* out_pos,
                  void* workspace, size_t ws_bytes, void* trace, gmc_stream_t stream);
 
+/*
+ * gmc_compress_host -- gmc_compress from and to HOST memory (a deployment
+ * variant; the paper has no counterpart).  The caller passes its inputs in
+ * page-locked host memory, device buffers to copy them into (the layouts and
+ * alignment of gmc_compress's inputs), the device outputs and page-locked
+ * host buffers for them.  The call enqueues, on `stream` and the library's
+ * side stream:
+ *   - the copies of keys, queries, vo_probe and pos_ids on `stream`;
+ *   - the copy of the hidden states on the side stream, after everything
+ *     enqueued on `stream` before the call (so a previous call that still
+ *     reads `d_hidden` is not overwritten), beside the probe, the message
+ *     slice and the heads, which do not read the hidden states; the row norms
+ *     and the cosine Gram follow it there, and `stream` joins the side stream
+ *     before the first kernel on it that reads them;
+ *   - gmc_compress on the device buffers;
+ *   - the copies of the four outputs back to the host buffers on `stream`.
+ * It returns once that is enqueued: synchronise `stream` before reading the
+ * host outputs or reusing the host inputs.  Byte counts are the caller's
+ * (every input and output of the call, e.g. hidden: (B*N + sum_b T_b) * D *
+ * element size).  Returns GMC_OK or the error gmc_compress returns
+ * (GMC_ERR_ARG also for a NULL pointer or a zero byte count).
+ */
+typedef struct gmc_host_io {
+  /* inputs: page-locked HOST memory, then the DEVICE buffers they are copied to */
+  const void* hidden;    void* d_hidden;    size_t hidden_bytes;
+  const void* keys;      void* d_keys;      size_t keys_bytes;
+  const void* queries;   void* d_queries;   size_t queries_bytes;
+  const int32_t* pos_ids; int32_t* d_pos_ids; size_t pos_ids_bytes;
+  const float* vo_probe; float* d_vo_probe; size_t vo_probe_bytes;
+  /* outputs: DEVICE buffers of gmc_compress, then the page-locked HOST copies */
+  int32_t* d_out_idx;    int32_t* out_idx;  size_t out_idx_bytes;
+  void* d_out_hidden;    void* out_hidden;  size_t out_hidden_bytes;
+  void* d_out_kv;        void* out_kv;      size_t out_kv_bytes;
+  int32_t* d_out_pos;    int32_t* out_pos;  size_t out_pos_bytes;
+} gmc_host_io;
+
+int gmc_compress_host(const gmc_problem* prob, const gmc_params* params, const gmc_host_io* io,
+                      int N, int T, int H, int d, int D, int K, void* workspace, size_t ws_bytes,
+                      void* trace, gmc_stream_t stream);
+
 /* gmc_compress with historical message views (views NULL or n == 0: gmc_compress). */
 int gmc_compress_views(const gmc_problem* prob, const gmc_params* params, const gmc_views* views,
                        const void* hidden, const void* keys, const void* queries,

@@ -351,6 +351,7 @@ Profiler g_prof;
 struct SideStream {
   cudaStream_t st = nullptr;
   cudaEvent_t fork = nullptr, join = nullptr;
+  cudaEvent_t aux = nullptr;  // gmc_compress_host: the hidden states' copy has landed
 };
 SideStream g_side[64];
 
@@ -364,6 +365,7 @@ cudaError_t side_stream(SideStream** out) {
     if ((e = cudaStreamCreateWithFlags(&sd.st, cudaStreamNonBlocking)) != cudaSuccess) return e;
     if ((e = cudaEventCreateWithFlags(&sd.fork, cudaEventDisableTiming)) != cudaSuccess) return e;
     if ((e = cudaEventCreateWithFlags(&sd.join, cudaEventDisableTiming)) != cudaSuccess) return e;
+    if ((e = cudaEventCreateWithFlags(&sd.aux, cudaEventDisableTiming)) != cudaSuccess) return e;
   }
   *out = &sd;
   return cudaSuccess;
@@ -705,6 +707,58 @@ int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* 
   return compress_impl(prob, params, nullptr, nullptr, hidden, keys, queries, pos_ids, vo_probe,
                        N, T, H, d, D, K, out_idx, out_hidden, out_kv, out_pos, workspace,
                        ws_bytes, trace, stream_);
+}
+
+int gmc_compress_host(const gmc_problem* prob, const gmc_params* params, const gmc_host_io* io,
+                      int N, int T, int H, int d, int D, int K, void* workspace, size_t ws_bytes,
+                      void* trace, gmc_stream_t stream_) {
+  if (!prob || !io) return GMC_ERR_ARG;
+  if (!io->hidden || !io->d_hidden || !io->keys || !io->d_keys || !io->queries ||
+      !io->d_queries || !io->pos_ids || !io->d_pos_ids || !io->vo_probe || !io->d_vo_probe ||
+      !io->d_out_idx || !io->out_idx || !io->d_out_hidden || !io->out_hidden || !io->d_out_kv ||
+      !io->out_kv || !io->d_out_pos || !io->out_pos)
+    return GMC_ERR_ARG;
+  if (!io->hidden_bytes || !io->keys_bytes || !io->queries_bytes || !io->pos_ids_bytes ||
+      !io->vo_probe_bytes || !io->out_idx_bytes || !io->out_hidden_bytes || !io->out_kv_bytes ||
+      !io->out_pos_bytes)
+    return GMC_ERR_ARG;
+  // the problem is checked before any copy is enqueued
+  if (gmc_workspace_size(prob, N, T, H, d, D, K) == 0) return GMC_ERR_ARG;
+  cudaStream_t st = (cudaStream_t)stream_;
+  SideStream* sd = nullptr;
+  GMC_TRY(side_stream(&sd));
+  // the hidden states on the side stream, after the caller's earlier work on `stream`
+  GMC_TRY(cudaEventRecord(sd->fork, st));
+  GMC_TRY(cudaStreamWaitEvent(sd->st, sd->fork, 0));
+  GMC_TRY(cudaMemcpyAsync(io->d_hidden, io->hidden, io->hidden_bytes, cudaMemcpyHostToDevice,
+                          sd->st));
+  GMC_TRY(cudaMemcpyAsync(io->d_keys, io->keys, io->keys_bytes, cudaMemcpyHostToDevice, st));
+  GMC_TRY(cudaMemcpyAsync(io->d_queries, io->queries, io->queries_bytes, cudaMemcpyHostToDevice,
+                          st));
+  GMC_TRY(cudaMemcpyAsync(io->d_vo_probe, io->vo_probe, io->vo_probe_bytes,
+                          cudaMemcpyHostToDevice, st));
+  GMC_TRY(cudaMemcpyAsync(io->d_pos_ids, io->pos_ids, io->pos_ids_bytes, cudaMemcpyHostToDevice,
+                          st));
+  // Only the pipelined path reads the hidden states after its side stream has
+  // joined; the identity (K = N) and the stage-timed runs read them on `stream`.
+  const bool pipelined = !g_prof.on && effective_K(K, N, images_of(prob)) != N;
+  if (!pipelined) {
+    GMC_TRY(cudaEventRecord(sd->aux, sd->st));
+    GMC_TRY(cudaStreamWaitEvent(st, sd->aux, 0));
+  }
+  const int rc = compress_impl(prob, params, nullptr, nullptr, io->d_hidden, io->d_keys,
+                               io->d_queries, io->d_pos_ids, io->d_vo_probe, N, T, H, d, D, K,
+                               io->d_out_idx, io->d_out_hidden, io->d_out_kv, io->d_out_pos,
+                               workspace, ws_bytes, trace, stream_);
+  if (rc != GMC_OK) return rc;
+  GMC_TRY(cudaMemcpyAsync(io->out_idx, io->d_out_idx, io->out_idx_bytes, cudaMemcpyDeviceToHost,
+                          st));
+  GMC_TRY(cudaMemcpyAsync(io->out_hidden, io->d_out_hidden, io->out_hidden_bytes,
+                          cudaMemcpyDeviceToHost, st));
+  GMC_TRY(cudaMemcpyAsync(io->out_kv, io->d_out_kv, io->out_kv_bytes, cudaMemcpyDeviceToHost, st));
+  GMC_TRY(cudaMemcpyAsync(io->out_pos, io->d_out_pos, io->out_pos_bytes, cudaMemcpyDeviceToHost,
+                          st));
+  return GMC_OK;
 }
 
 int gmc_compress_views(const gmc_problem* prob, const gmc_params* params, const gmc_views* views,

@@ -29,9 +29,20 @@ EXPORTS = (
     "gmc_transport_noalloc", "gmc_cosine_workspace_size", "gmc_cosine",
     "gmc_workspace_size_views", "gmc_compress_views", "gmc_clients", "gmc_selftest_bounded_wait",
     "gmc_compress_ex", "gmc_workspace_size_long", "gmc_compress_long", "gmc_clients_long",
+    "gmc_compress_host",
 )
 MAX_VIEWS = 4
 MAX_PREFIX_LAYERS = 64
+
+
+class HostIO(ctypes.Structure):
+    """gmc_host_io: (host, device, bytes) for every input, (device, host, bytes) for every output."""
+    _fields_ = ([f for n in ("hidden", "keys", "queries", "pos_ids", "vo_probe")
+                 for f in ((n, ctypes.c_void_p), ("d_" + n, ctypes.c_void_p),
+                           (n + "_bytes", ctypes.c_size_t))] +
+                [f for n in ("out_idx", "out_hidden", "out_kv", "out_pos")
+                 for f in (("d_" + n, ctypes.c_void_p), (n, ctypes.c_void_p),
+                           (n + "_bytes", ctypes.c_size_t))])
 
 
 class Params(ctypes.Structure):
@@ -111,6 +122,9 @@ def lib() -> ctypes.CDLL:
     L.gmc_compress.argtypes = [PP, P, vp, vp, vp, vp, vp, i, i, i, i, i, i, vp, vp, vp, vp, vp,
                                sz, vp, vp]
     L.gmc_compress.restype = i
+    L.gmc_compress_host.argtypes = [PP, P, ctypes.POINTER(HostIO), i, i, i, i, i, i, vp, sz, vp,
+                                    vp]
+    L.gmc_compress_host.restype = i
     L.gmc_workspace_size_views.argtypes = [PP, i, i, i, i, i, i, i]
     L.gmc_workspace_size_views.restype = sz
     L.gmc_compress_views.argtypes = [PP, P, ctypes.POINTER(Views), vp, vp, vp, vp, vp, i, i, i, i,
@@ -226,6 +240,30 @@ def compress(prob: Problem, params: Params, hidden, keys, queries, pos_ids, vo_p
         _ptr(pos_ids), _ptr(vo_probe), N, T, H, d, D, K, _ptr(out_idx), _ptr(out_hidden),
         _ptr(out_kv), _ptr(out_pos), _ptr(workspace), workspace.numel(), _ptr(trace),
         _stream(stream)))
+
+
+def _nbytes(t) -> int:
+    return t.numel() * t.element_size()
+
+
+def compress_host(prob: Problem, params: Params, host_in, dev_in, dev_out, host_out, N, T, H, d,
+                  D, K, workspace, trace=None, stream=None):
+    """gmc_compress_host: inputs from page-locked host tensors through the device
+    tensors `dev_in`, outputs back into page-locked host tensors.  host_in / dev_in:
+    dicts with hidden, keys, queries, pos_ids, vo_probe; dev_out / host_out: dicts
+    with idx, hidden, kv, pos."""
+    io = HostIO()
+    for n in ("hidden", "keys", "queries", "pos_ids", "vo_probe"):
+        setattr(io, n, _ptr(host_in[n]))
+        setattr(io, "d_" + n, _ptr(dev_in[n]))
+        setattr(io, n + "_bytes", _nbytes(host_in[n]))
+    for n, k in (("out_idx", "idx"), ("out_hidden", "hidden"), ("out_kv", "kv"), ("out_pos", "pos")):
+        setattr(io, "d_" + n, _ptr(dev_out[k]))
+        setattr(io, n, _ptr(host_out[k]))
+        setattr(io, n + "_bytes", _nbytes(host_out[k]))
+    _check(lib().gmc_compress_host(ctypes.byref(prob), ctypes.byref(params), ctypes.byref(io), N,
+                                   T, H, d, D, K, _ptr(workspace), workspace.numel(), _ptr(trace),
+                                   _stream(stream)))
 
 
 def views(keys, queries, vo_probe, beta_hist=0.5) -> Views:
@@ -499,6 +537,18 @@ class Compressor:
                            stream)
         return Outputs(self.out_idx, self.out_hidden, self.out_kv, self.out_pos, self.K, self.trace,
                        self.layout)
+
+    def run_host(self, host_in, dev_in, host_out, stream=None):
+        """gmc_compress_host: the inputs in page-locked host tensors (dict: hidden, keys,
+        queries, pos_ids, vo_probe) copied through the device tensors `dev_in`, the outputs
+        (this Compressor's device buffers) copied back into `host_out` (dict: idx, hidden,
+        kv, pos).  Synchronise the stream before reading host_out."""
+        if self.long_prefix is not None:
+            raise GMCError("run_host covers gmc_compress (no long-prefix bank)")
+        compress_host(self.prob, self.params, host_in, dev_in,
+                      {"idx": self.out_idx, "hidden": self.out_hidden, "kv": self.out_kv,
+                       "pos": self.out_pos}, host_out, self.N, self.T, self.H, self.d, self.D,
+                      self.Kr, self.workspace, self.trace, stream)
 
     def status(self, stream=None) -> int:
         return read_status(self.workspace, stream)

@@ -186,3 +186,22 @@ def test_long_prefix_sizing_and_validation(gmc):
     # gmc_select accepts wide pools (every round on the whole GPU) and longer N with them
     assert gmc.select_workspace_size(1, 500, 12000, 1500, p) > 500 * 12000 * 6
     assert gmc.select_workspace_size(1, 500, 12000, 1500, gmc.default_params()) == 0
+
+
+def test_host_io_struct_and_validation(gmc):
+    """gmc_host_io: 9 (pointer, pointer, size) triples; nothing is copied when an
+    argument is missing or the problem is invalid."""
+    assert ctypes.sizeof(gmc.HostIO) == 9 * 3 * 8
+    lib = gmc.lib()
+    pr = gmc.problem(1, 36, 36, 4, gmc.GMC_BF16)
+    p = gmc.default_params()
+    fake = ctypes.c_void_p(1 << 20)
+    assert lib.gmc_compress_host(ctypes.byref(pr), ctypes.byref(p), None, 1296, 64, 28, 128, 3584,
+                                 257, fake, 1 << 30, None, None) == gmc.GMC_ERR_ARG
+    io = gmc.HostIO()
+    assert lib.gmc_compress_host(ctypes.byref(pr), ctypes.byref(p), ctypes.byref(io), 1296, 64, 28,
+                                 128, 3584, 257, fake, 1 << 30, None, None) == gmc.GMC_ERR_ARG
+    for name, _ in gmc.HostIO._fields_:  # every pointer and size set: the problem decides
+        setattr(io, name, 1 << 20)
+    assert lib.gmc_compress_host(ctypes.byref(pr), ctypes.byref(p), ctypes.byref(io), 1295, 64, 28,
+                                 128, 3584, 257, fake, 1 << 30, None, None) == gmc.GMC_ERR_ARG
