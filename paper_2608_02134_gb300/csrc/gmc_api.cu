@@ -565,10 +565,13 @@ static int compress_impl(const gmc_problem* prob, const gmc_params* params,
     }
     return cudaSuccess;
   };
+  int msg_k = 0;  // message-slice launches of the call
   auto messages = [&]() -> cudaError_t {
     for (int v = 0; v < V; ++v) {
-      const cudaError_t e = launch_message(dm, vkeys[v], vqueries[v], sv[v], st);
+      int n = 0;
+      const cudaError_t e = launch_message(dm, vkeys[v], vqueries[v], sv[v], st, &n);
       if (e != cudaSuccess) return e;
+      msg_k += n;
     }
     return cudaSuccess;
   };
@@ -579,7 +582,6 @@ static int compress_impl(const gmc_problem* prob, const gmc_params* params,
     }
     return launch_heads(dm, p, sv[0], tv, st, 1, V > 1 ? &vg : nullptr);
   };
-  const int msg_k = (message_tc_supported(dm) ? 2 : 1) * V;  // at most two launches per view
   GMC_TRY(g_prof.begin(st));  // k_rownorm zeroes the column sums u0 of the client build
   // the appearance branch: cosine Gram, or on long prefixes the projection,
   // the split unit states and the bounded bank's cosines

@@ -62,10 +62,11 @@ __global__ void k_message(const Tin* __restrict__ keys, const Tin* __restrict__ 
 }
 
 cudaError_t launch_message(const Dims& dm, const void* keys, const void* queries, Scratch& s,
-                           cudaStream_t st) {
+                           cudaStream_t st, int* launches) {
   // bf16 with d in {64, 128} and a full 128-key tile: tcgen05 (k_message_tc.cu);
   // fp32 inputs and other shapes: the CUDA-core kernel above.
-  if (message_tc_supported(dm)) return launch_message_tc(dm, keys, queries, s, st);
+  if (message_tc_supported(dm)) return launch_message_tc(dm, keys, queries, s, st, launches);
+  if (launches) *launches = 1;
   dim3 grid(dm.T, dm.H, dm.B);
   size_t smem = sizeof(float) * (dm.d + dm.N + dm.T);
   cudaError_t e;

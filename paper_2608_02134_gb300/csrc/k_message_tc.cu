@@ -620,8 +620,9 @@ int message_splits(const Dims& dm) {
 // The packed queries Qp are written by the probe kernel, launched before this
 // one on the same stream (k_prep.cu).
 cudaError_t launch_message_tc(const Dims& dm, const void* keys, const void* queries, Scratch& s,
-                              cudaStream_t st) {
+                              cudaStream_t st, int* launches) {
   (void)queries;
+  if (launches) *launches = 1;
   const int RQ = message_rq(dm);
   cudaError_t e;
   CUtensorMap qmap, kmap;
@@ -668,6 +669,7 @@ cudaError_t launch_message_tc(const Dims& dm, const void* keys, const void* quer
     }
     cudaGetLastError();  // no co-resident cluster: the two launches below
   }
+  if (launches) *launches = 2;
   for (int mode = 0; mode < 2; ++mode) {
     launch_k(k_message_tc, grid, THREADS, smem, st, 1, qmap, kmap, dm.toff, dm.B, dm.N, dm.T, dm.H, dm.Hkv,
                                               dm.d, RQ, mode, sp.kt_per, sp.n, s.mpart, s.zn2,

@@ -142,7 +142,7 @@ cudaError_t launch_probe(const Dims&, const void* keys, const float* W, const vo
                          const gmc_params&, Scratch&,
                          cudaStream_t);
 cudaError_t launch_message(const Dims&, const void* keys, const void* queries, Scratch&,
-                           cudaStream_t);
+                           cudaStream_t, int* launches = nullptr);
 cudaError_t launch_heads(const Dims&, const gmc_params&, Scratch&, const TraceView&, cudaStream_t,
                          int cluster = 1, const ViewGrams* views = nullptr);
 bool heads_supported(int H);  // the head statistics of H heads fit a block (H <= 56)
@@ -279,7 +279,7 @@ cudaError_t launch_gram_simt(const Dims&, const void* hidden, Scratch&, cudaStre
 cudaError_t launch_gram_tc(const Dims&, const void* hidden, Scratch&, cudaStream_t);
 bool gram_tc_supported(const Dims&);
 cudaError_t launch_message_tc(const Dims&, const void* keys, const void* queries, Scratch&,
-                              cudaStream_t);
+                              cudaStream_t, int* launches = nullptr);
 bool message_tc_supported(const Dims&);
 int message_rq(const Dims&);  // packed query rows per (image, KV group)
 int message_splits(const Dims&);  // key splits of the message slice (parts of rs)
