@@ -127,22 +127,35 @@ __device__ inline int select_pool(const long long* u, const unsigned char* sel, 
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
   const int nc = (N + 32 * nw - 1) / (32 * nw);  // chunks per warp
   const unsigned lt = lanemask_lt();
-  // 1. bucket of every candidate (-1: selected or zero gain), histograms
-  for (int c = 0; c < nc; ++c) {
-    const int j = (wid * nc + c) * 32 + lane;
-    int kb = -1;
-    if (j < N) {
-      const long long v = u[j];
-      if (!sel[j] && v > 0) {
-        kb = gain_bucket(v);
-        atomicAdd(&w.hist[kb], 1);
-      }
-      w.key[j] = (short)kb;
+  // 1. bucket of every candidate (-1: selected or zero gain), histograms; the
+  //    gains of four chunks are loaded before any of their atomics
+  for (int c0 = 0; c0 < nc; c0 += 4) {
+    long long vv[4];
+    bool cand[4];
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+      const int j = (wid * nc + c0 + t) * 32 + lane;
+      const bool in = c0 + t < nc && j < N;
+      vv[t] = in ? u[j] : 0;
+      cand[t] = in && !sel[j];
     }
-    // exponents: one atomic per warp and distinct exponent
-    const int e = kb >= 0 ? kb >> 5 : -1;
-    const unsigned same = __match_any_sync(FULL, e);
-    if (e >= 0 && (same & lt) == 0) atomicAdd(&w.coarse[e], __popc(same));
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+      if (c0 + t >= nc) break;  // uniform over the warp
+      const int j = (wid * nc + c0 + t) * 32 + lane;
+      int kb = -1;
+      if (j < N) {
+        if (cand[t] && vv[t] > 0) {
+          kb = gain_bucket(vv[t]);
+          atomicAdd(&w.hist[kb], 1);
+        }
+        w.key[j] = (short)kb;
+      }
+      // exponents: one atomic per warp and distinct exponent
+      const int e = kb >= 0 ? kb >> 5 : -1;
+      const unsigned same = __match_any_sync(FULL, e);
+      if (e >= 0 && (same & lt) == 0) atomicAdd(&w.coarse[e], __popc(same));
+    }
   }
   __syncthreads();
   // 2. boundary bucket, found by every warp alike: coarse bins from the top,
