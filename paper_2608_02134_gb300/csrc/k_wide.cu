@@ -124,6 +124,9 @@ __global__ void __launch_bounds__(WP_THREADS) k_w_pool(WideState w, WideGeom g, 
   p = reinterpret_cast<char*>((reinterpret_cast<uintptr_t>(p) + 15) & ~static_cast<uintptr_t>(15));
   ps.bval = reinterpret_cast<long long*>(p);  // the boundary bucket's gains
   ps.bcap = min(N, W_BCAP);
+  p += sizeof(long long) * (size_t)ps.bcap;
+  ps.sortbuf = reinterpret_cast<int*>(p);     // and their order
+  ps.scap = W_BCAP;
   for (int j = threadIdx.x; j < N; j += blockDim.x) {
     selz[j] = 0;
     if (tv.base) tv.gains(b, rd, N)[j] = ucur[j];
@@ -280,7 +283,10 @@ __global__ void __launch_bounds__(WP_THREADS) k_w_batch(WideState w, WideGeom g,
     int* top = reinterpret_cast<int*>(p);      p += sizeof(int) * (size_t)NP;
     ps.key = reinterpret_cast<short*>(p);      p += sizeof(short) * (size_t)NP;
     ps.pk = reinterpret_cast<unsigned char*>(p); p += (size_t)NP;
-    unsigned char* none = reinterpret_cast<unsigned char*>(p);
+    unsigned char* none = reinterpret_cast<unsigned char*>(p); p += (size_t)NP;
+    p = reinterpret_cast<char*>((reinterpret_cast<uintptr_t>(p) + 15) & ~static_cast<uintptr_t>(15));
+    ps.sortbuf = reinterpret_cast<int*>(p);  // [NP], NP a power of two
+    ps.scap = NP;
     for (int k = threadIdx.x; k < Pt; k += blockDim.x) {
       ks[k] = w.sc[(size_t)b * P + k];
       kj[k] = w.pool[(size_t)b * P + k];
@@ -619,12 +625,13 @@ cudaError_t launch_wide_select(const WideState& w, const WideGeom& g, const gmc_
   while (NP < P) NP <<= 1;
   const size_t psm = sizeof(int) * (sel::HBINS + (size_t)N + 32 + 8 + sel::CBINS + P) +
                      sizeof(short) * (size_t)N + 2 * (size_t)N + 16 +
-                     sizeof(long long) * (size_t)std::min(N, W_BCAP) + 64;
+                     sizeof(long long) * (size_t)std::min(N, W_BCAP) +
+                     sizeof(int) * (size_t)W_BCAP + 64;
   const size_t rsm_dense = sizeof(long long) * (size_t)P + sizeof(float) * (size_t)WROWS * P;
   const size_t rsm_sparse = sizeof(long long) * (size_t)P + sizeof(short) * (size_t)N;
   const size_t bsm = (sizeof(long long) + sizeof(int)) * (size_t)NP +
                      sizeof(int) * (sel::HBINS + 2 * (size_t)NP + 32 + 8 + sel::CBINS) +
-                     sizeof(short) * (size_t)NP + 2 * (size_t)NP + 64;
+                     sizeof(short) * (size_t)NP + 2 * (size_t)NP + sizeof(int) * (size_t)NP + 80;
   const size_t fsm = sizeof(unsigned long long) * (size_t)N;
   if ((e = set_smem_limit((const void*)k_w_pool, psm)) != cudaSuccess) return e;
   if ((e = set_smem_limit((const void*)k_w_rho<true>, rsm_dense)) != cudaSuccess) return e;

@@ -73,7 +73,11 @@ struct PoolScratch {
   long long* bval;     // optional [bcap]: the boundary bucket's gains, staged when the
                        // gains are in global memory (nullptr: read them in place)
   int bcap;
+  int* sortbuf;        // optional [scap], scap a power of two: a boundary bucket of more
+                       // than SORT_MIN gains is sorted there instead of ranked
+  int scap;
 };
+constexpr int SORT_MIN = 128;
 
 // Warp-aggregated append: every lane with `want` gets a distinct index from
 // *counter (order within the warp by lane).  All lanes of the warp call it.
@@ -256,11 +260,47 @@ __device__ inline int select_pool(const long long* u, const unsigned char* sel, 
       for (int q = threadIdx.x; q < nb; q += blockDim.x) w.bval[q] = u[w.bnd[q]];
       __syncthreads();
     }
-    // A large bucket (near-equal gains) is split once more by the next 11
-    // mantissa bits: the tokens of higher sub-buckets enter, those of lower
-    // ones do not, and only the boundary sub-bucket is ranked exactly.
+    // A large bucket is sorted by (u desc, id asc) (bitonic, in shared
+    // memory) and its first `need` tokens enter.  Otherwise a large bucket
+    // (near-equal gains) is split once more by the next 11 mantissa bits: the
+    // tokens of higher sub-buckets enter, those of lower ones do not, and only
+    // the boundary sub-bucket is ranked exactly.
     // pk[q]: 1 enters, 0 does not, 2 undecided (ranked below).
-    const bool refine = REFINE && nb > 512;  // uniform over the block
+    const bool sorted = w.sortbuf && nb > SORT_MIN && nb <= w.scap;  // uniform over the block
+    const bool refine = REFINE && nb > 512 && !sorted;                        // uniform
+    if (sorted) {
+      int n2 = 1;
+      while (n2 < nb) n2 <<= 1;
+      for (int q = threadIdx.x; q < n2; q += blockDim.x) w.sortbuf[q] = q < nb ? q : -1;
+      __syncthreads();
+      // a before c: c is padding, or (u, id) of a comes first
+      auto before = [&](int a, int c) {
+        if (a < 0) return false;
+        if (c < 0) return true;
+        const int ja = w.bnd[a], jc = w.bnd[c];
+        return key_before(staged ? w.bval[a] : u[ja], ids ? ids[ja] : ja,
+                          staged ? w.bval[c] : u[jc], ids ? ids[jc] : jc);
+      };
+      for (int k = 2; k <= n2; k <<= 1)
+        for (int jj = k >> 1; jj > 0; jj >>= 1) {
+          for (int i = threadIdx.x; i < n2; i += blockDim.x) {
+            const int ixj = i ^ jj;
+            if (ixj > i) {
+              const int a = w.sortbuf[i], c = w.sortbuf[ixj];
+              const bool af = before(a, c);
+              if (((i & k) == 0) != af) {  // out of order for this half's direction
+                w.sortbuf[i] = c;
+                w.sortbuf[ixj] = a;
+              }
+            }
+          }
+          __syncthreads();
+        }
+      for (int q = threadIdx.x; q < nb; q += blockDim.x) w.pk[q] = 0;
+      __syncthreads();
+      for (int q = threadIdx.x; q < need; q += blockDim.x) w.pk[w.sortbuf[q]] = 1;
+      __syncthreads();
+    }
     if (refine) {
       for (int q = threadIdx.x; q < nb; q += blockDim.x)
         atomicAdd(&w.hist[gain_subbucket(staged ? w.bval[q] : u[w.bnd[q]])], 1);
@@ -295,7 +335,7 @@ __device__ inline int select_pool(const long long* u, const unsigned char* sel, 
       need -= w.scal[1];
       __syncthreads();
     }
-    for (int q = threadIdx.x; q < nb; q += blockDim.x) {
+    for (int q = threadIdx.x; q < (sorted ? 0 : nb); q += blockDim.x) {
       if (refine && w.pk[q] != 2) continue;
       const int j = w.bnd[q];
       const long long v = staged ? w.bval[q] : u[j];
