@@ -639,9 +639,11 @@ cudaError_t launch_wide_select(const WideState& w, const WideGeom& g, const gmc_
   if ((e = set_smem_limit((const void*)k_w_batch, bsm)) != cudaSuccess) return e;
   if ((e = set_smem_limit((const void*)k_w_filter<true>, fsm)) != cudaSuccess) return e;
   if ((e = set_smem_limit((const void*)k_w_filter<false>, fsm)) != cudaSuccess) return e;
-  // filters: one row per warp while the blocks fit on the GPU at once, four beyond
+  // filters: one row per warp while the blocks fit on the GPU about twice, four
+  // beyond (each block ends with an atomic per column it touched: fewer, longer
+  // blocks add fewer; 4 measured best on the long-prefix document)
   const long long fblocks = (long long)g.B * ceil_div(g.Mstride, FROWS);
-  const int rpw = fblocks > 4LL * sms ? 4 : 1;
+  const int rpw = fblocks > 2LL * sms ? 4 : 1;
   const dim3 rgrid(ceil_div(g.Mstride, WROWS), g.B);
   const dim3 fgrid(ceil_div(g.Mstride, FROWS * rpw), g.B);
   const int R = wide_rounds(g.K, p);
