@@ -196,6 +196,13 @@ size_t gmc_workspace_size_views(const gmc_problem* prob, int n_views, int N, int
  * must fit a block's 227 KB of shared memory; GMC_ERR_UNSUPPORTED above),
  * D a multiple of 8.  hidden/keys/queries/vo_probe/out_hidden/out_kv must be
  * 16-byte aligned, trace 16-byte aligned.
+ *
+ * Selection runs on one thread-block cluster per image while its state (a
+ * copy of every token's gain, bucket and pool slot, and a share of the M
+ * client rows per CTA) fits a CTA's shared memory; beyond that (with the
+ * default parameters, N above about 7,700 at H = 28 and T = 128) every round runs
+ * on the whole GPU, with the same decisions.  A multi-image prompt
+ * (images > 1) that does not fit the cluster returns GMC_ERR_UNSUPPORTED.
  */
 int gmc_compress(const gmc_problem* prob, const gmc_params* params, const void* hidden,
                  const void* keys, const void* queries, const int32_t* pos_ids,
@@ -394,7 +401,9 @@ size_t gmc_trace_size(const gmc_problem* prob, const gmc_params* params, int N, 
  * 1 <= K <= N <= GMC_MAX_N, M >= 1.  The clients are copied into the workspace
  * first, so `clients` is never written.  A pool pool_mult * batch_b above
  * GMC_MAX_POOL (up to GMC_MAX_POOL_WIDE) runs every round on the whole GPU, the
- * solver of gmc_compress_long, and allows N up to GMC_MAX_N_LONG.
+ * solver of gmc_compress_long, and allows N up to GMC_MAX_N_LONG; so does a
+ * problem whose cluster-solver state does not fit a CTA's shared memory (as in
+ * gmc_compress).
  */
 size_t gmc_select_workspace_size(int B, int M, int N, int K, const gmc_params* params);
 int gmc_select(const float* clients, int B, int M, int N, int K, const gmc_params* params,

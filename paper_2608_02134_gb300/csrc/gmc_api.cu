@@ -231,6 +231,11 @@ size_t carve_compress(const Dims& dm, Scratch* s, char* base, R0State* r0s = nul
   }
   R0State r0 = carve_round0(c, B, N, M);
   if (r0s && base) *r0s = r0;
+  // the wide solver's state, for problems whose cluster-solver state does not
+  // fit one CTA's shared memory (a few words per token and client row)
+  WideState w{};
+  carve_wide(c, B, N, M, GMC_MAX_POOL, &w);
+  if (ls && base) ls->w = w;
   return c.off;
 }
 
@@ -523,6 +528,14 @@ static int compress_impl(const gmc_problem* prob, const gmc_params* params,
   const size_t need =
       carve_compress(dm, &s, (char*)workspace, &r0, &ls, p.pool_mult * p.batch_b);
   if (ws_bytes < need) return GMC_ERR_WORKSPACE;
+  // every selection round on the whole GPU: long prefixes, and problems whose
+  // cluster-solver state (a copy per token and a share of the client rows in
+  // each CTA) does not fit one CTA's shared memory; that solver seeds no
+  // per-image tokens, so a multi-image prompt must fit the cluster solver
+  const bool wide =
+      lp != nullptr || (!out_clients && Ke != N &&
+                        !select_fits(dm.B, N, dm.M, p.pool_mult * p.batch_b));
+  if (wide && dm.I > 1) return GMC_ERR_UNSUPPORTED;
   cudaStream_t st = (cudaStream_t)stream_;
   gmc_trace_layout L;
   TraceView tv{};
@@ -651,7 +664,7 @@ static int compress_impl(const gmc_problem* prob, const gmc_params* params,
     return GMC_OK;
   }
   const int LS = dm.I * p.landmarks * p.landmarks;  // spatial rows: a landmark grid per image
-  if (lp) {
+  if (wide) {
     WideGeom wg{};
     wg.B = dm.B; wg.N = N; wg.K = Ke; wg.Mstride = dm.M;
     wg.HV = HV; wg.Tmax = T; wg.MV = dm.MV; wg.L2 = LS;
@@ -663,6 +676,16 @@ static int compress_impl(const gmc_problem* prob, const gmc_params* params,
       GMC_TRY(launch_certificate(dm.B, N, Ke, tv, st));
       g_launches += 1;
     }
+  } else {
+    GMC_STAGE("rounds_gpu", 3 + 3 * sparse_gpu_rounds(N),
+              launch_round0(r0, dm.B, N, Ke, dm.M, dm.toff, HV, T, LS, p, fx, nullptr, s.C,
+                            s.scol, s.u0, s.order, s.status, tv, st, dm.I));
+    GMC_STAGE("select", 1,
+              launch_select(r0, dm.B, N, Ke, dm.M, dm.toff, HV, T, LS, p, fx, nullptr, s.C,
+                            s.scol, s.u0, s.order, s.support, s.slot, nullptr, s.status, tv, st,
+                            dm.I));
+  }
+  if (lp) {
     // the support cosines of the assignment (Eq. (cond-assignment)), K x N:
     // row k holds the cosines of every token with the k-th selected one
     auto support_cos = [&]() -> cudaError_t {
@@ -687,12 +710,6 @@ static int compress_impl(const gmc_problem* prob, const gmc_params* params,
     g_prof.valid = g_prof.on;
     return GMC_OK;
   }
-  GMC_STAGE("rounds_gpu", 3 + 3 * sparse_gpu_rounds(N),
-            launch_round0(r0, dm.B, N, Ke, dm.M, dm.toff, HV, T, LS, p, fx, nullptr, s.C, s.scol,
-                          s.u0, s.order, s.status, tv, st, dm.I));
-  GMC_STAGE("select", 1,
-            launch_select(r0, dm.B, N, Ke, dm.M, dm.toff, HV, T, LS, p, fx, nullptr, s.C, s.scol,
-                          s.u0, s.order, s.support, s.slot, nullptr, s.status, tv, st, dm.I));
   GMC_STAGE("assign", 2, launch_assign(dm, p, s, tv, st));
   GMC_STAGE("transport", 1,
             launch_transport(dm, p, hidden, keys, pos_ids, s.support, s.pi, s.mass, s.rmsh,
@@ -853,18 +870,20 @@ static size_t carve_select(int B, int M, int N, int K, Scratch* s, char* base,
   t.selpart = c.take<double>((size_t)B * t.nSel);
   t.fexp = c.take<int32_t>((size_t)B);
   if (s) *s = t;
-  if (wide_pool > 0) {  // pools above GMC_MAX_POOL: the wide solver's state
-    WideState w{};
-    carve_wide(c, (size_t)B, (size_t)N, (size_t)M, (size_t)wide_pool, &w);
-    if (ws && base) *ws = w;
-    return c.off;
-  }
+  // the wide solver's state: pools above GMC_MAX_POOL, and problems whose
+  // cluster-solver state does not fit one CTA's shared memory
+  WideState w{};
+  carve_wide(c, (size_t)B, (size_t)N, (size_t)M, (size_t)(wide_pool > 0 ? wide_pool : GMC_MAX_POOL),
+             &w);
+  if (ws && base) *ws = w;
+  if (wide_pool > 0) return c.off;
   R0State r0 = carve_round0(c, (size_t)B, (size_t)N, (size_t)M);
   if (r0s && base) *r0s = r0;
   return c.off;
 }
 
-// gmc_select runs the wide solver when the pool exceeds GMC_MAX_POOL
+// gmc_select runs the wide solver when the pool exceeds GMC_MAX_POOL (and, at
+// run time, when the cluster solver's state does not fit; see select_fits)
 static int select_wide_pool(const gmc_params& p) {
   const int P = p.pool_mult * p.batch_b;
   return P > GMC_MAX_POOL ? P : 0;
@@ -908,7 +927,7 @@ int gmc_select(const float* clients, int B, int M, int N, int K, const gmc_param
                           cudaMemcpyDeviceToDevice, st));
   GMC_TRY(cudaMemsetAsync(s.u0, 0, sizeof(long long) * B * (size_t)N, st));
   GMC_TRY(launch_select_prep(s.C, B, M, N, s, st));
-  if (wp) {
+  if (wp || !select_fits(B, N, M, p.pool_mult * p.batch_b)) {
     WideGeom wg{};
     wg.B = B; wg.N = N; wg.K = K; wg.Mstride = M;
     wg.HV = 0; wg.Tmax = 1; wg.MV = 0; wg.L2 = 0;

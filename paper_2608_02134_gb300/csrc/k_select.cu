@@ -1017,22 +1017,46 @@ __global__ void __launch_bounds__(256) k_certificate(int N, int K, TraceView tv)
 
 static int g_num_sms = 0;
 
+static cudaError_t num_sms() {
+  if (g_num_sms) return cudaSuccess;
+  int dev = 0, n = 0;
+  cudaError_t e;
+  if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+  if ((e = cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+    return e;
+  if ((e = cudaFuncSetAttribute(k_select, cudaFuncAttributeNonPortableClusterSizeAllowed, 1)) !=
+      cudaSuccess)
+    return e;
+  g_num_sms = n;
+  return cudaSuccess;
+}
+
+// The largest cluster launch_select tries (images x CTAs within the SMs) has
+// the smallest per-CTA state; the state of any smaller one is larger.
+static int first_cluster_size(int B) {
+  int CS = 1;
+  while (CS * 2 <= SEL_MAX_CS && (long long)B * CS * 2 <= g_num_sms) CS *= 2;
+  return CS;
+}
+
+bool select_fits(int B, int N, int M, int P) {
+  if (num_sms() != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  const int CS = first_cluster_size(B);
+  const int RPC = (M + CS - 1) / CS;
+  const int gwords = (CS > 1 ? 2 : 1) * ((N + CS - 1) / CS);
+  return sel_fixed_bytes(N, P, RPC, gwords, nullptr, nullptr) + 1024 <= SMEM_LIMIT;
+}
+
 cudaError_t launch_select(const R0State& r0, int B, int N, int K, int M, const int32_t* toff, int H, int T, int L2,
                           const gmc_params& p, int fx_exp, const int32_t* fexp, float* C,
                           uint16_t* scol, const long long* u0, int32_t* order, int32_t* support,
                           int32_t* slot, int32_t* out_idx, uint32_t* status, const TraceView& tv,
                           cudaStream_t st, int I) {
   cudaError_t e;
-  if (g_num_sms == 0) {
-    int dev = 0;
-    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
-    if ((e = cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev)) !=
-        cudaSuccess)
-      return e;
-    if ((e = cudaFuncSetAttribute(k_select, cudaFuncAttributeNonPortableClusterSizeAllowed, 1)) !=
-        cudaSuccess)
-      return e;
-  }
+  if ((e = num_sms()) != cudaSuccess) return e;
   SelArgs a;
   a.B = B; a.N = N; a.K = K; a.Mstride = M; a.H = H; a.Tmax = T; a.L2 = L2;
   a.toff = toff;
@@ -1049,9 +1073,7 @@ cudaError_t launch_select(const R0State& r0, int B, int N, int K, int M, const i
   a.tv = tv;
   a.r0 = r0;
   a.images = I;
-  int CS = 1;
-  while (CS * 2 <= SEL_MAX_CS && (long long)B * CS * 2 <= g_num_sms) CS *= 2;
-  for (; CS >= 1; CS /= 2) {
+  for (int CS = first_cluster_size(B); CS >= 1; CS /= 2) {
     // Row capacity of one CTA: rows are dealt in turn, so ceil(M / CS) each
     const int RPC = (M + CS - 1) / CS;
     const int gwords = (CS > 1 ? 2 : 1) * ((N + CS - 1) / CS);

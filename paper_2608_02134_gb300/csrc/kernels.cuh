@@ -190,6 +190,11 @@ cudaError_t launch_select(const R0State&, int B, int N, int K, int M, const int3
                           int32_t* slot, int32_t* out_idx, uint32_t* status, const TraceView&,
                           cudaStream_t, int I = 1);
 cudaError_t launch_select_prep(const float* C, int B, int M, int N, Scratch&, cudaStream_t);
+// Whether the cluster solver's per-CTA state (a copy of every token's gain,
+// bucket and pool slot, and its share of the client rows) fits one CTA's
+// shared memory for this problem on this device; where it does not, every
+// round runs on the whole GPU (launch_wide_select).
+bool select_fits(int B, int N, int M, int P);
 // Batched certificate c_B of the trace from the recorded rounds (one block per image).
 cudaError_t launch_certificate(int B, int N, int K, const TraceView&, cudaStream_t);
 // cs: nullptr (cosines read from the N x N matrix at the support's columns) or

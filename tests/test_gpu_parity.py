@@ -66,6 +66,29 @@ def test_document_shape():
     _check(GH.run(wl), [0], TOL_BF16)
 
 
+def test_largest_image():
+    """N = GMC_MAX_N (a 128 x 64 page, K = 820): the cluster solver's state
+    does not fit a CTA, so every selection round runs on the whole GPU; every
+    decision is still checked against the oracle."""
+    from paper_2608_02134_gb300 import gmc, workloads
+    from tests import gpu_harness as GH
+    wl = workloads.make("doc", gh=128, gw=64, K=820)
+    assert wl.N == 8192  # GMC_MAX_N
+    g = GH.run(wl)
+    _check(g, [0], TOL_BF16)
+    # the stages of a timed call: no cluster rounds
+    inp = GH.to_device(wl)
+    gmc.profile_enable(True)
+    try:
+        g.comp.run(inp["hidden"], inp["keys"], inp["queries"], inp["pos_ids"], inp["vo_probe"])
+        torch.cuda.synchronize()
+        stages = gmc.profile_read()
+    finally:
+        gmc.profile_enable(False)
+    assert "select" in stages and "rounds_gpu" not in stages, sorted(stages)
+    assert g.comp.status() == 0
+
+
 def test_serving_batch_every_image():
     """32 ragged images in one call; the oracle checks every one of them."""
     from paper_2608_02134_gb300 import workloads

@@ -111,6 +111,18 @@ def test_select_parameters_b1_and_k_equals_n():
     _check_select(C, 60)
 
 
+def test_select_beyond_the_cluster_runs_on_the_whole_gpu():
+    """N = GMC_MAX_N with 4,800 client rows and a 128-token pool: the cluster
+    solver's per-CTA state (a copy per token, 1/16 of the rows) exceeds a
+    CTA's 227 KB, so every round runs on the whole GPU (4 launches a round,
+    then the final one; the prep kernels and the certificate besides)."""
+    from paper_2608_02134_gb300 import gmc
+    B, M, N, K, b = 1, 4800, 8192, 600, 32
+    n0 = gmc.launch_count()
+    _check_select(_structured_clients(B, M, N, 91), K, batch_b=b)
+    assert gmc.launch_count() - n0 == 3 + 4 * (-(-K // b)) + 1 + 1
+
+
 def test_transport_with_oracle_decisions():
     from paper_2608_02134_gb300 import gmc, workloads
     from tests import gpu_harness as GH, parity
