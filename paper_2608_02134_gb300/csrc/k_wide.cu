@@ -79,10 +79,14 @@ __device__ __forceinline__ long long* gains_out(const WideState& w, int rnd) {
 }  // namespace
 
 // ---- pool ------------------------------------------------------------------------
+// win: pools of at most WCAP / 2 tokens take the window pool (the boundary
+// bucket of a round lies at or below the last one), with the gains staged in
+// shared memory; the full histogram pool runs in round 0, when the window
+// misses, and for larger pools.
 __global__ void __launch_bounds__(WP_THREADS) k_w_pool(WideState w, WideGeom g, int P, int rnd,
                                                        const long long* __restrict__ u0,
                                                        const int32_t* __restrict__ order,
-                                                       TraceView tv) {
+                                                       TraceView tv, int win) {
   grid_dep_wait();
   extern __shared__ __align__(16) char sm_wp[];
   const int b = blockIdx.x, N = g.N, K = g.K;
@@ -99,6 +103,7 @@ __global__ void __launch_bounds__(WP_THREADS) k_w_pool(WideState w, WideGeom g, 
   int MG;
   const int Mb = wide_rows(g, b, &MG);
   const int S = rnd == 0 ? 0 : info[1], rd = rnd == 0 ? 0 : info[2];
+  int hint = rnd == 0 || !win ? -1 : info[5];  // the last round's boundary bucket
   __syncthreads();  // every thread has read info before thread 0 rewrites it
   if (rnd == 0 && threadIdx.x == 0) {
     info[1] = 0;
@@ -127,21 +132,38 @@ __global__ void __launch_bounds__(WP_THREADS) k_w_pool(WideState w, WideGeom g, 
   p += sizeof(long long) * (size_t)ps.bcap;
   ps.sortbuf = reinterpret_cast<int*>(p);     // and their order
   ps.scap = W_BCAP;
+  p += sizeof(int) * (size_t)W_BCAP;
+  sel::WindowScratch ws{};
+  long long* ug = nullptr;  // win: the gains, staged for the pool's passes
+  if (win) {
+    p = reinterpret_cast<char*>((reinterpret_cast<uintptr_t>(p) + 15) & ~static_cast<uintptr_t>(15));
+    ug = reinterpret_cast<long long*>(p);     p += sizeof(long long) * (size_t)N;
+    ws.cu = reinterpret_cast<long long*>(p);  p += sizeof(long long) * sel::WCAP;
+    ws.cj = reinterpret_cast<int*>(p);        p += sizeof(int) * sel::WCAP;
+    ws.win = reinterpret_cast<int*>(p);
+    for (int q = threadIdx.x; q < sel::WBINS + 4; q += blockDim.x) ws.win[q] = 0;
+  }
   for (int j = threadIdx.x; j < N; j += blockDim.x) {
     selz[j] = 0;
     if (tv.base) tv.gains(b, rd, N)[j] = ucur[j];
+    if (win && hint < 0) ug[j] = ucur[j];  // else the window pool's first pass stages them
   }
   for (int h = threadIdx.x; h < sel::HBINS; h += blockDim.x) ps.hist[h] = 0;
   if (threadIdx.x < sel::CBINS) ps.coarse[threadIdx.x] = 0;
   __syncthreads();
   for (int q = threadIdx.x; q < S; q += blockDim.x) selz[order[(size_t)b * K + q]] = 1;
   __syncthreads();
-  const int Pt = sel::select_pool<true>(ucur, selz, N, P, ps, pool, nullptr);
+  int Pt = -1;
+  if (win)
+    Pt = sel::select_pool_window([&](int j) { return ucur[j]; }, ug, selz, N, P, ws, pool, nullptr,
+                                 &hint);
+  if (Pt < 0) Pt = sel::select_pool<true>(win ? ug : ucur, selz, N, P, ps, pool, nullptr, nullptr, &hint);
   for (int k = threadIdx.x; k < P; k += blockDim.x) w.pool[(size_t)b * P + k] = k < Pt ? pool[k] : -1;
   if (threadIdx.x == 0) {
     info[0] = Pt;
     info[3] = S;
     info[4] = rd;
+    info[5] = hint;
   }
   if (tv.base && Pt > 0) {
     int32_t* tp = tv.at<int32_t>(b, tv.off_pool) + (size_t)rd * tv.pool_size;
@@ -633,7 +655,12 @@ cudaError_t launch_wide_select(const WideState& w, const WideGeom& g, const gmc_
                      sizeof(int) * (sel::HBINS + 2 * (size_t)NP + 32 + 8 + sel::CBINS) +
                      sizeof(short) * (size_t)NP + 2 * (size_t)NP + sizeof(int) * (size_t)NP + 80;
   const size_t fsm = sizeof(unsigned long long) * (size_t)N;
-  if ((e = set_smem_limit((const void*)k_w_pool, psm)) != cudaSuccess) return e;
+  // the window pool's extra shared memory: the staged gains and its scratch
+  const size_t wsm = 16 + sizeof(long long) * ((size_t)N + sel::WCAP) + sizeof(int) * sel::WCAP +
+                     sizeof(int) * (sel::WBINS + 4);
+  const int win = P <= sel::WCAP / 2 && psm + wsm <= 227 * 1024 ? 1 : 0;
+  const size_t psm_w = psm + (win ? wsm : 0);
+  if ((e = set_smem_limit((const void*)k_w_pool, psm_w)) != cudaSuccess) return e;
   if ((e = set_smem_limit((const void*)k_w_rho<true>, rsm_dense)) != cudaSuccess) return e;
   if ((e = set_smem_limit((const void*)k_w_rho<false>, rsm_sparse)) != cudaSuccess) return e;
   if ((e = set_smem_limit((const void*)k_w_batch, bsm)) != cudaSuccess) return e;
@@ -648,7 +675,8 @@ cudaError_t launch_wide_select(const WideState& w, const WideGeom& g, const gmc_
   const dim3 fgrid(ceil_div(g.Mstride, FROWS * rpw), g.B);
   const int R = wide_rounds(g.K, p);
   for (int rnd = 0; rnd < R; ++rnd) {
-    launch_k(k_w_pool, g.B, WP_THREADS, psm, st, 1, w, g, P, rnd, u0, (const int32_t*)order, tv);
+    launch_k(k_w_pool, g.B, WP_THREADS, psm_w, st, 1, w, g, P, rnd, u0, (const int32_t*)order, tv,
+             win);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     if (rnd == 0)
       launch_k(k_w_rho<true>, rgrid, 32 * WROWS, rsm_dense, st, 1, w, g, P, (const float*)C,
