@@ -290,6 +290,33 @@ __global__ void __launch_bounds__(WP_THREADS) k_w_batch(WideState w, WideGeom g,
   const int nb = min(bsz, min(Pt, K - S));
   long long* ks = reinterpret_cast<long long*>(sm_wb);   // [NP] scores
   int* kj = reinterpret_cast<int*>(ks + NP);             // [NP] tokens
+  if (Pt <= sel::WCAP) {
+    // a small pool: every slot's exact rank by (score desc, token asc) is its
+    // place in the batch (the order the histogram selection and the sort
+    // below give)
+    for (int k = threadIdx.x; k < Pt; k += blockDim.x) {
+      ks[k] = w.sc[(size_t)b * P + k];
+      kj[k] = w.pool[(size_t)b * P + k];
+    }
+    __syncthreads();
+    for (int k = threadIdx.x; k < Pt; k += blockDim.x) {
+      const long long sk = ks[k];
+      const int jk = kj[k];
+      int r = 0;
+      for (int q = 0; q < Pt; ++q) r += sel::key_before(ks[q], kj[q], sk, jk);
+      if (r < nb) {
+        w.batch[(size_t)b * P + r] = jk;
+        w.stamp[(size_t)b * g.N + jk] = rd + 1;
+        order[(size_t)b * K + S + r] = jk;
+      }
+    }
+    if (threadIdx.x == 0) {
+      info[1] = S + nb;
+      info[2] = rd + 1;
+      if (tv.base) tv.at<int32_t>(b, tv.off_round_end)[rd] = S + nb;
+    }
+    return;
+  }
   // The batch is the top nb of the pool by (score desc, token asc): the
   // histogram selection over the pool slots with the tokens as tie-breakers.
   // Scores of zero are no candidates there; if fewer than nb are positive,
