@@ -79,14 +79,17 @@ __device__ __forceinline__ long long* gains_out(const WideState& w, int rnd) {
 }  // namespace
 
 // ---- pool ------------------------------------------------------------------------
-// win: pools of at most WCAP / 2 tokens take the window pool (the boundary
+// WIN: pools of at most WCAP / 2 tokens take the window pool (the boundary
 // bucket of a round lies at or below the last one), with the gains staged in
 // shared memory; the full histogram pool runs in round 0, when the window
-// misses, and for larger pools.
-__global__ void __launch_bounds__(WP_THREADS) k_w_pool(WideState w, WideGeom g, int P, int rnd,
+// misses, and for larger pools (a separate instance, without the window's
+// registers).
+template <bool WIN>
+__global__ void __launch_bounds__(WP_THREADS, 1) k_w_pool(WideState w, WideGeom g, int P, int rnd,
                                                        const long long* __restrict__ u0,
                                                        const int32_t* __restrict__ order,
-                                                       TraceView tv, int win) {
+                                                       TraceView tv) {
+  constexpr bool win = WIN;
   grid_dep_wait();
   extern __shared__ __align__(16) char sm_wp[];
   const int b = blockIdx.x, N = g.N, K = g.K;
@@ -154,7 +157,7 @@ __global__ void __launch_bounds__(WP_THREADS) k_w_pool(WideState w, WideGeom g, 
   for (int q = threadIdx.x; q < S; q += blockDim.x) selz[order[(size_t)b * K + q]] = 1;
   __syncthreads();
   int Pt = -1;
-  if (win)
+  if constexpr (WIN)
     Pt = sel::select_pool_window([&](int j) { return ucur[j]; }, ug, selz, N, P, ws, pool, nullptr,
                                  &hint);
   if (Pt < 0) Pt = sel::select_pool<true>(win ? ug : ucur, selz, N, P, ps, pool, nullptr, nullptr, &hint);
@@ -687,7 +690,8 @@ cudaError_t launch_wide_select(const WideState& w, const WideGeom& g, const gmc_
                      sizeof(int) * (sel::WBINS + 4);
   const int win = P <= sel::WCAP / 2 && psm + wsm <= 227 * 1024 ? 1 : 0;
   const size_t psm_w = psm + (win ? wsm : 0);
-  if ((e = set_smem_limit((const void*)k_w_pool, psm_w)) != cudaSuccess) return e;
+  const void* kpool = win ? (const void*)k_w_pool<true> : (const void*)k_w_pool<false>;
+  if ((e = set_smem_limit(kpool, psm_w)) != cudaSuccess) return e;
   if ((e = set_smem_limit((const void*)k_w_rho<true>, rsm_dense)) != cudaSuccess) return e;
   if ((e = set_smem_limit((const void*)k_w_rho<false>, rsm_sparse)) != cudaSuccess) return e;
   if ((e = set_smem_limit((const void*)k_w_batch, bsm)) != cudaSuccess) return e;
@@ -702,8 +706,12 @@ cudaError_t launch_wide_select(const WideState& w, const WideGeom& g, const gmc_
   const dim3 fgrid(ceil_div(g.Mstride, FROWS * rpw), g.B);
   const int R = wide_rounds(g.K, p);
   for (int rnd = 0; rnd < R; ++rnd) {
-    launch_k(k_w_pool, g.B, WP_THREADS, psm_w, st, 1, w, g, P, rnd, u0, (const int32_t*)order, tv,
-             win);
+    if (win)
+      launch_k(k_w_pool<true>, g.B, WP_THREADS, psm_w, st, 1, w, g, P, rnd, u0,
+               (const int32_t*)order, tv);
+    else
+      launch_k(k_w_pool<false>, g.B, WP_THREADS, psm_w, st, 1, w, g, P, rnd, u0,
+               (const int32_t*)order, tv);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     if (rnd == 0)
       launch_k(k_w_rho<true>, rgrid, 32 * WROWS, rsm_dense, st, 1, w, g, P, (const float*)C,
